@@ -1,0 +1,513 @@
+#!/usr/bin/env python
+"""Benchmark of the PHSA sparse-attention hot path on GB300.
+
+One step = the whole hot path over one batch of the workload: block
+representation (a), block selection (b), sparse attention forward (c1) and
+its backward (c2-c5, with a synthetic upstream gradient dO). The default
+workload is the 32k prefill: B=1, L=32768, 16 query / 8 KV heads, D=128,
+blocks of 64 tokens, 14 blocks per query block (97.27% sparsity).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0). Multi-GPU runs (torchrun) shard independent
+sequences across ranks (weak scaling, no data-path collective); the only
+collectives are the barrier and the max-over-ranks of the elapsed time.
+``--impl reference`` times the CPU oracle on bounded samples of the same
+workload on this host's cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2601_02819_gb300 import inputs  # noqa: E402
+
+METRIC = ("sparse-attn prefill tokens/s + effective TFLOPS at 32k, 97.3% sparsity; "
+          "% roofline")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ---------------------------------------------------------------- helpers
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def algorithmic(w, cnt: np.ndarray):
+    """FLOPs and bytes the method must do/move, per stage and per kernel.
+
+    pairs = sum over (b, kv head, query block) of the selected block count,
+    times G query heads: every (query head, query block, selected block) pair
+    is one 64x64 tile (the diagonal tile counted whole).
+    """
+    m, D, G = w.block_size, w.D, w.G
+    pairs = float(cnt.astype(np.int64).sum()) * G
+    bf = 2
+    q = w.B * w.Hq * w.L * D * bf
+    kv = w.B * w.Hkv * w.L * D * bf
+    krepr = w.B * w.Hkv * w.T * D * bf
+    idx = cnt.size * (w.topk + 1) * 4
+    lse = w.B * w.Hq * w.L * 4
+    # candidates actually scored: nC = qb - n_local - n_init + 1 when the budget
+    # does not cover them all
+    scored = 0
+    for qb in range(w.NQB):
+        n_c = max(0, qb - w.n_local - w.n_init + 1)
+        n_f = min(w.n_init, qb + 1) + (qb - max(min(w.n_init, qb + 1), qb - w.n_local + 1) + 1)
+        if w.topk - n_f < n_c:
+            scored += n_c
+    f_sel = 2.0 * D * m * scored * G * w.B * w.Hkv
+    t = {
+        "block_repr": {"flops": 0.0, "bytes": kv + w.B * w.L + krepr},
+        "select_blocks": {"flops": f_sel, "bytes": q + krepr + idx},
+        "attn_fwd": {"flops": 4.0 * m * m * D * pairs, "bytes": q + 2 * kv + q + lse + idx},
+        "bwd_delta": {"flops": 0.0, "bytes": 2 * q + lse},
+        "bwd_dkdv": {"flops": 8.0 * m * m * D * pairs,
+                     "bytes": 2 * q + 2 * kv + 2 * lse + idx + 2 * kv},
+        "bwd_dq": {"flops": 6.0 * m * m * D * pairs, "bytes": 2 * q + 2 * kv + 2 * lse + idx + q},
+    }
+    stages = {
+        "fwd": {"flops": f_sel + 4.0 * m * m * D * pairs,
+                "parts": ["block_repr", "select_blocks", "attn_fwd"]},
+        # reads Q, K, V, O, dO, lse, idx; writes dQ, dK, dV; Delta written and read once
+        "bwd": {"flops": 10.0 * m * m * D * pairs, "bytes": 4 * q + 4 * kv + 3 * lse + idx},
+    }
+    return t, stages, pairs
+
+
+def roofline_time(t, P_tf, BW_gbs, parts):
+    return sum(max(t[k]["flops"] / (P_tf * 1e12), t[k]["bytes"] / (BW_gbs * 1e9)) for k in parts)
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks/throttle reasons in the background."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, local_rank: int):
+        self.proc = None
+        self.path = None
+        dev = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")[0].strip()
+        self.dev = dev if dev else str(local_rank)
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="phsa_clocks_", suffix=".csv")
+            os.close(fd)
+            self.t0 = time.time()
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu=timestamp,{self.FIELDS}", "--format=csv,noheader",
+                 "-lms", "50", "-i", self.dev], stdout=open(self.path, "w"),
+                stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self, t_begin: float, t_end: float):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.12)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 10:
+                    continue
+                try:
+                    ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                    ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                except (ValueError, IndexError):
+                    ts = None
+                rows.append((ts, parts))
+        os.unlink(self.path)
+        inside = [p for ts, p in rows if ts is not None and t_begin - 0.05 <= ts <= t_end + 0.05]
+        window = "timed region" if inside else "whole run (no sample fell in the timed region)"
+        rows = inside if inside else [p for _, p in rows]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def mhz(s):
+            try:
+                return float(s.split()[0])
+            except (ValueError, IndexError):
+                return None
+        sm = [mhz(r[2]) for r in rows if mhz(r[2]) is not None]
+        smax = [mhz(r[3]) for r in rows if mhz(r[3]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in rows:
+            for k, name in enumerate(names):
+                if r[6 + k].lower().startswith("active"):
+                    reasons.add(name)
+        power = [mhz(r[4]) for r in rows if mhz(r[4]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(rows), "window": window,
+                "power_w_max": max(power) if power else None}
+
+
+# ---------------------------------------------------------------- oracle sample
+def oracle_sample_step(w, x, n_units: int, seed: int):
+    """Times the CPU oracle on a bounded sample of one step; returns estimated seconds
+    for the whole step, the parts and a description. Sample: stage (a) in full;
+    stages (b), (c) forward and dQ for `n_units` random (b, g, qb) units; dK/dV
+    for `n_units` random KV blocks. Each part is scaled by (total units / sampled)."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    U = w.B * w.Hkv * w.NQB
+    units = rng.choice(U, size=min(n_units, U), replace=False)
+    scale = w.sm_scale
+    t = {}
+    t0 = time.perf_counter()
+    Kr = oracle.block_repr(x["K"], x["mask"], w.block_size, w.lam)
+    t["repr"] = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    si, sc, _ = oracle.select_units(x["Q"], Kr, w.L, w.block_size, w.topk, w.n_init, w.n_local,
+                                    scale, units)
+    t["select"] = (time.perf_counter() - t0) * U / len(units)
+    # full index table for the attention parts: forced + the first candidates
+    idx = np.full((w.B, w.Hkv, w.NQB, w.topk), -1, np.int32)
+    cnt = np.zeros((w.B, w.Hkv, w.NQB), np.int32)
+    for qb in range(w.NQB):
+        s = sorted(set(range(min(w.n_init, qb + 1))) | set(range(max(0, qb - w.n_local + 1), qb + 1)))
+        extra = [c for c in range(qb) if c not in s][::-1][: max(0, w.topk - len(s))]
+        s = sorted(set(s) | set(extra))
+        idx[:, :, qb, :len(s)] = s
+        cnt[:, :, qb] = len(s)
+    rows = []
+    for u in units:
+        qb = u % w.NQB
+        bg = u // w.NQB
+        b, g = bg // w.Hkv, bg % w.Hkv
+        for hh in range(w.G):
+            for i in range(qb * w.block_size, min((qb + 1) * w.block_size, w.L)):
+                rows.append((b, g * w.G + hh, i))
+    rows = np.array(rows, np.int32)
+    frac = U / len(units)
+    t0 = time.perf_counter()
+    oracle.sparse_attn_rows(x["Q"], x["K"], x["V"], idx, cnt, w.block_size, scale, rows)
+    t["fwd"] = (time.perf_counter() - t0) * frac
+    t0 = time.perf_counter()
+    oracle.sparse_attn_bwd_dq_rows(x["Q"], x["K"], x["V"], x["dO"], idx, cnt, w.block_size, scale,
+                                   rows)
+    t["bwd_dq"] = (time.perf_counter() - t0) * frac
+    kvb = np.stack([units // w.NQB // w.Hkv, (units // w.NQB) % w.Hkv,
+                    rng.integers(0, w.NQB, len(units))], axis=1).astype(np.int32)
+    t0 = time.perf_counter()
+    oracle.sparse_attn_bwd_kv_blocks(x["Q"], x["K"], x["V"], x["dO"], idx, cnt, w.block_size,
+                                     scale, kvb)
+    t["bwd_dkdv"] = (time.perf_counter() - t0) * frac
+    desc = (f"stage (a) in full; stages (b), (c) fwd and dQ on {len(units)}"
+            f" of {U} (query block, KV head) units; dK/dV on {len(units)} of {U} KV blocks;"
+            f" each part scaled to the full step")
+    return sum(t.values()), t, desc
+
+
+def oracle_threads():
+    import oracle
+    n = len(os.sched_getaffinity(0))
+    oracle.set_threads(n)
+    return oracle.max_threads()
+
+
+# ---------------------------------------------------------------- GPU arm
+def run_ours(args):
+    from paper_2601_02819_gb300 import phsa
+    rank, world, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    w = inputs.WORKLOADS[args.workload]
+    x = inputs.make_inputs(w, with_grad=True, seed=w.seed + 7919 * rank)
+
+    def dev_bf16(a):
+        return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
+
+    Q, K, V, dO = (dev_bf16(x[k]) for k in ("Q", "K", "V", "dO"))
+    mask = torch.from_numpy(x["mask"]).to(dev)
+    Kr = torch.empty((w.B, w.Hkv, w.T, w.D), dtype=torch.bfloat16, device=dev)
+    idx = torch.empty((w.B, w.Hkv, w.NQB, w.topk), dtype=torch.int32, device=dev)
+    cnt = torch.empty((w.B, w.Hkv, w.NQB), dtype=torch.int32, device=dev)
+    O = torch.empty_like(Q)
+    lse = torch.empty((w.B, w.Hq, w.L), dtype=torch.float32, device=dev)
+    dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
+    ws = torch.empty(phsa.phsa_sparse_attn_bwd_workspace(w.B, w.L, w.Hq, w.Hkv, w.topk),
+                     dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        phsa.phsa_build_block_repr(K, mask, w.lam, Krepr=Kr)
+        phsa.phsa_select_blocks(Q, Kr, w.Hkv, w.topk, w.n_init, w.n_local, w.sm_scale,
+                                block_idx=idx, block_cnt=cnt)
+        phsa.phsa_sparse_attn_fwd(Q, K, V, idx, cnt, w.sm_scale, O=O, lse=lse)
+        phsa.phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, idx, cnt, w.sm_scale, workspace=ws,
+                                  dQ=dQ, dK=dK, dV=dV)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = phsa.phsa_get_device_status()
+    if status != 0:
+        raise SystemExit(f"device status after warm-up: {phsa.phsa_status_string(status)}")
+    cnt_np = cnt.cpu().numpy()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    phsa.phsa_profile_read()
+    phsa.phsa_profile_enable(True)
+    barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    t_wall1 = time.time()
+    phsa.phsa_profile_enable(False)
+    prof = phsa.phsa_profile_read()
+    clk = clocks.stop(t_wall0, t_wall1)
+    ms_total = ev0.elapsed_time(ev1)
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([ms_total], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    ms_step = ms_total / args.steps
+    status = phsa.phsa_get_device_status()
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        pin = lambda a: torch.from_numpy(a).pin_memory()
+        hQ, hK, hV, hdO = (pin(x[k].view(np.int16)) for k in ("Q", "K", "V", "dO"))
+        hmask = pin(x["mask"])
+        hO, hdQ = (torch.empty(Q.shape, dtype=torch.int16).pin_memory() for _ in range(2))
+        hdK, hdV = (torch.empty(K.shape, dtype=torch.int16).pin_memory() for _ in range(2))
+        h2d = sum(t.numel() * t.element_size() for t in (hQ, hK, hV, hdO, hmask))
+        d2h = sum(t.numel() * t.element_size() for t in (hO, hdQ, hdK, hdV))
+
+        def e2e_step():
+            Q.view(torch.int16).copy_(hQ, non_blocking=True)
+            K.view(torch.int16).copy_(hK, non_blocking=True)
+            V.view(torch.int16).copy_(hV, non_blocking=True)
+            dO.view(torch.int16).copy_(hdO, non_blocking=True)
+            mask.copy_(hmask, non_blocking=True)
+            step()
+            hO.copy_(O.view(torch.int16), non_blocking=True)
+            hdQ.copy_(dQ.view(torch.int16), non_blocking=True)
+            hdK.copy_(dK.view(torch.int16), non_blocking=True)
+            hdV.copy_(dV.view(torch.int16), non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        n_e2e = max(3, min(args.steps, 20))
+        barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ms_e2e = e0.elapsed_time(e1) / n_e2e
+        if world > 1:
+            import torch.distributed as dist
+            tt = torch.tensor([ms_e2e], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            ms_e2e = float(tt.item())
+        e2e = {"value": world * w.B * w.L / (ms_e2e / 1e3), "unit": "tokens/s",
+               "ms_per_step": ms_e2e, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "steps": n_e2e}
+
+    if rank != 0:
+        return None
+
+    # ---- roofline and per-kernel accounting
+    peaks, peak_src = load_peaks()
+    P_burst, P_sus, BW = peaks["bf16_tflops"], peaks["bf16_tflops_sustained"], peaks["hbm_gbs"]
+    kt, stages, pairs = algorithmic(w, cnt_np)
+    kernels = {}
+    for name, (ms, n) in prof.items():
+        if n == 0:
+            continue
+        avg_s = ms / n / 1e3
+        e = {"launches": n, "ms_total": round(ms, 4), "us_per_launch": round(avg_s * 1e6, 2),
+             "share": None}
+        if name in kt:
+            a = kt[name]
+            t_f = a["flops"] / (P_burst * 1e12)
+            t_b = a["bytes"] / (BW * 1e9)
+            e["bound"] = "tensor" if t_f >= t_b else "hbm"
+            e["achieved_tflops"] = round(a["flops"] / avg_s / 1e12, 1)
+            e["achieved_gbs"] = round(a["bytes"] / avg_s / 1e9, 1)
+            e["frac"] = round(max(t_f, t_b) / avg_s, 4)
+        kernels[name] = e
+    tot = sum(v["ms_total"] for v in kernels.values()) or 1.0
+    for v in kernels.values():
+        v["share"] = round(v["ms_total"] / tot, 4)
+    dom = max((k for k in kernels if k in kt), key=lambda k: kernels[k]["ms_total"])
+    a = kt[dom]
+    avg_s = kernels[dom]["ms_total"] / kernels[dom]["launches"] / 1e3
+    if kernels[dom]["bound"] == "tensor":
+        roof = {"kernel": dom, "bound": "tensor", "achieved": round(a["flops"] / avg_s / 1e12, 1),
+                "peak": P_burst, "unit": "TFLOP/s",
+                "frac": round(a["flops"] / avg_s / 1e12 / P_burst, 4),
+                "peak_source": f"{peak_src} bf16 burst", "traffic": None,
+                "algorithmic_per_launch": a["flops"]}
+    else:
+        roof = {"kernel": dom, "bound": "hbm", "achieved": round(a["bytes"] / avg_s / 1e9, 1),
+                "peak": BW, "unit": "GB/s", "frac": round(a["bytes"] / avg_s / 1e9 / BW, 4),
+                "peak_source": f"{peak_src} HBM copy", "traffic": None,
+                "algorithmic_per_launch": a["bytes"]}
+    fwd_ms = sum(kernels[k]["ms_total"] for k in ("block_repr", "select_blocks", "attn_fwd")
+                 if k in kernels) / args.steps
+    bwd_ms = sum(v["ms_total"] for k, v in kernels.items() if k.startswith("bwd")) / args.steps
+    fwd_roof = roofline_time(kt, P_burst, BW, ["block_repr", "select_blocks", "attn_fwd"])
+    bwd_roof = max(stages["bwd"]["flops"] / (P_burst * 1e12), stages["bwd"]["bytes"] / (BW * 1e9))
+    tokens = world * w.B * w.L
+
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        cores = oracle_threads()
+        est_s, parts, desc = oracle_sample_step(w, x, args.cpu_units, seed=5)
+        cpu = {"value": w.B * w.L / est_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+               "sample": desc, "est_s_per_step": round(est_s, 2),
+               "parts_s": {k: round(v, 3) for k, v in parts.items()}}
+
+    out = {
+        "metric": METRIC, "value": tokens / (ms_step / 1e3), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "L": w.L, "Hq": w.Hq, "Hkv": w.Hkv, "D": w.D,
+                   "block_size": w.block_size, "topk": w.topk, "n_init": w.n_init,
+                   "n_local": w.n_local, "lambda": w.lam,
+                   "sparsity": round(1 - w.topk * w.block_size / w.L, 5),
+                   "step": "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)",
+                   "l2": "inputs larger than L2 (Q 134 MB, K 67 MB, V 67 MB, dO 134 MB per step)",
+                   "parallelism": f"dp{world} (independent sequences)"},
+        "fwd": {"ms": round(fwd_ms, 4), "tokens_per_s": tokens / (fwd_ms / 1e3) if fwd_ms else None,
+                "eff_tflops": round(stages["fwd"]["flops"] / (fwd_ms / 1e3) / 1e12, 1) if fwd_ms else None,
+                "roofline_us": round(fwd_roof * 1e6, 1),
+                "roofline_frac": round(fwd_roof / (fwd_ms / 1e3), 4) if fwd_ms else None},
+        "bwd": {"ms": round(bwd_ms, 4),
+                "eff_tflops": round(stages["bwd"]["flops"] / (bwd_ms / 1e3) / 1e12, 1) if bwd_ms else None,
+                "roofline_us": round(bwd_roof * 1e6, 1),
+                "roofline_frac": round(bwd_roof / (bwd_ms / 1e3), 4) if bwd_ms else None},
+        "roofline": roof,
+        "kernels": kernels,
+        "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
+        "selected_pairs_per_step": int(pairs),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "clocks": clk,
+        "device_status": status,
+        "peaks": {"source": peak_src, "hbm_gbs": BW, "bf16_tflops": P_burst,
+                  "bf16_tflops_sustained": P_sus},
+    }
+    return out
+
+
+# ---------------------------------------------------------------- reference arm
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return None
+    w = inputs.WORKLOADS[args.workload]
+    x = inputs.make_inputs(w, with_grad=True)
+    cores = oracle_threads()
+    for s in range(args.warmup):
+        oracle_sample_step(w, x, args.ref_units, seed=100 + s)
+    ests, descs = [], None
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        est, _, descs = oracle_sample_step(w, x, args.ref_units, seed=1000 + s)
+        ests.append(est)
+    wall = time.perf_counter() - t0
+    est = statistics.mean(ests)
+    value = w.B * w.L / est
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": est * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "L": w.L, "Hq": w.Hq, "Hkv": w.Hkv, "D": w.D,
+                   "block_size": w.block_size, "topk": w.topk,
+                   "step": "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)"},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": descs},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "wall_s": round(wall, 2),
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="prefill_32k", choices=sorted(inputs.WORKLOADS))
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-units", type=int, default=48,
+                    help="units in the oracle sample of the cpu_baseline")
+    ap.add_argument("--ref-units", type=int, default=8,
+                    help="units in each oracle sample step of --impl reference")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    out = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+    if int(os.environ.get("WORLD_SIZE", "1")) > 1 and args.impl == "ours":
+        import torch.distributed as dist
+        if dist.is_initialized():
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

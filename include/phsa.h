@@ -1,0 +1,180 @@
+/*
+ * phsa.h -- C ABI of the PHSA sparse-attention library for NVIDIA GB300 (sm_103a).
+ *
+ * PHSA (Punctuation-aware Hybrid Sparse Attention) replaces dense causal
+ * attention by attention over a few selected key/value blocks. The library
+ * implements its three stages as CUDA kernels:
+ *   (a) phsa_build_block_repr  -- one representative key per KV block, mixing
+ *       the block's mean key with the mean of its punctuation-token keys
+ *       (Section 3.2, Eq. 3, 6, 7, 8; Algorithm 1 step 2);
+ *   (b) phsa_select_blocks     -- query-to-block relevance and Top-K block
+ *       selection with forced initial and local blocks (Eq. 8; Section 3.2
+ *       "Block Selection"; Algorithm 1 step 3);
+ *   (c) phsa_sparse_attn_fwd / phsa_sparse_attn_bwd -- causal attention over
+ *       the selected blocks only (Eq. 10-11; Algorithm 1 step 4) and its
+ *       gradient, which the paper's native sparse training uses.
+ *
+ * Conventions shared by every call
+ *   - Tensors are dense, row-major, layout [B, H, L, D]; bf16 values are
+ *     IEEE bfloat16 (uint16 storage). Query head h reads KV head h / G with
+ *     G = Hq / Hkv (grouped-query attention).
+ *   - Blocks have block_size = m tokens; block t covers tokens [t*m, (t+1)*m).
+ *     T = floor(L/m) blocks have a representative key (Eq. 3); NQB = ceil(L/m)
+ *     query blocks exist (the last may be partial).
+ *   - Selection is shared by the G*m query rows of one (query block, KV head):
+ *     block_idx[b][g][qb][0..cnt) lists block indices in ascending order,
+ *     padded with -1 up to topk; block_cnt[b][g][qb] = cnt.
+ *   - Every tensor pointer is a DEVICE pointer owned by the caller, 16-byte
+ *     aligned. The library never frees or retains caller memory.
+ *   - All work is enqueued on `stream` (a cudaStream_t passed as void*; NULL
+ *     is the legacy default stream) and is asynchronous. The return value
+ *     reports argument validation and launch errors only. Errors detected by
+ *     a kernel (an out-of-range block index, a bounded wait that expired) are
+ *     recorded in a device status word read by phsa_get_device_status.
+ *   - Supported today: D = 128, block_size = 64, G in {1, 2}. Other shapes
+ *     return PHSA_ERR_UNSUPPORTED, never a wrong answer.
+ *   - Calls are thread-safe with respect to each other; concurrent calls on
+ *     different streams that write the same output race, as any CUDA work.
+ */
+#ifndef PHSA_H
+#define PHSA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PHSA_OK = 0,
+    PHSA_ERR_INVALID_ARG = -1,  /* null/misaligned pointer, bad size or parameter */
+    PHSA_ERR_UNSUPPORTED = -2,  /* valid but unsupported shape (D, block_size, G) */
+    PHSA_ERR_CUDA = -3,         /* a CUDA runtime call or launch failed */
+    PHSA_ERR_TIMEOUT = -4,      /* device: a bounded wait inside a kernel expired */
+    PHSA_ERR_DEVICE_INDEX = -5, /* device: a block index outside [0, qb] was skipped */
+    PHSA_ERR_WORKSPACE = -6     /* workspace pointer null or smaller than required */
+} phsa_status;
+
+/* Problem shape. Layout [B, H, L, D]; block_size = m tokens per block. */
+typedef struct {
+    int B, L, Hq, Hkv, D, block_size;
+} phsa_shape;
+
+/* Selection parameters (Algorithm 1 inputs k, n_init and w).
+ *   topk     total blocks per (query block, KV head), forced blocks included
+ *            (the paper's 32k setting of 128 initial + 512 local tokens plus 16
+ *            chosen 16-token blocks is 896 tokens = 14 blocks of 64);
+ *   n_init   forced initial blocks {0 .. n_init-1};
+ *   n_local  forced local blocks {qb-n_local+1 .. qb}, n_local >= 1 (the query's
+ *            own block is always attended);
+ *   sm_scale score scale, normally 1/sqrt(D) (Eq. 2, 8, 11).
+ * Requires topk >= n_init + n_local, so every query block's forced set fits. */
+typedef struct {
+    int topk, n_init, n_local;
+    float sm_scale;
+} phsa_select_params;
+
+/*
+ * Stage (a): representative keys, Section 3.2 Eq. 6-8 / Algorithm 1 step 2.
+ * For every (b, g, t < T): M_0 = mean of the block's m keys (Eq. 6);
+ * c = number of punctuation tokens in the block; M_p = mean of their keys if
+ * c > 0 (Eq. 7), else M_0; Krepr = lambda*M_0 + (1-lambda)*M_p (Eq. 8).
+ * Sums in fp32, one round-to-nearest-even to bf16 at the end.
+ *   K          bf16 [B, Hkv, L, D]   in
+ *   punct_mask uint8 [B, L]          in, nonzero = token is punctuation (I(x in P))
+ *   lambda     gate in [0, 1]
+ *   Krepr      bf16 [B, Hkv, T, D]   out (nothing is written when T = 0)
+ */
+int phsa_build_block_repr(const void* K, const uint8_t* punct_mask, phsa_shape s, float lambda,
+                          void* Krepr, void* stream);
+
+/*
+ * Stage (b): relevance scoring and block selection, Eq. 8 / Algorithm 1 step 3,
+ * made once per (query block qb, KV head g) for all G*m rows r of that block:
+ *   forced   F = {0..n_init-1} U {qb-n_local+1..qb}, clipped to [0, qb];
+ *   candidates C = {t <= qb-1, t < T, t not in F} (strictly earlier full blocks);
+ *   S[r][t] = sm_scale * q_r . Krepr[t];  p[r][t] = softmax over t in C of S[r][.];
+ *   A[t]    = sum over rows r of p[r][t];
+ *   choose min(topk-|F|, |C|) candidates by A descending, ties to the lower t;
+ *   output F U chosen in ascending order, -1 padded to topk.
+ * Scores stay on chip (they are never written to memory).
+ *   Q         bf16 [B, Hq, L, D]        in
+ *   Krepr     bf16 [B, Hkv, T, D]       in (from phsa_build_block_repr)
+ *   block_idx int32 [B, Hkv, NQB, topk] out
+ *   block_cnt int32 [B, Hkv, NQB]       out
+ */
+int phsa_select_blocks(const void* Q, const void* Krepr, phsa_shape s, phsa_select_params p,
+                       int32_t* block_idx, int32_t* block_cnt, void* stream);
+
+/*
+ * Stage (c) forward: Eq. 10-11 / Algorithm 1 step 4. Row i of query head h
+ * attends the keys j of the listed blocks of (qb = i/m, g = h/G) with j <= i,
+ * o_i = sum_j softmax_j(sm_scale * q_i . k_j) v_j; lse_i = natural-log
+ * log-sum-exp of those scores (kept for the backward pass).
+ * block_idx entries must satisfy -1 or 0 <= t <= qb; entries beyond block_cnt
+ * are ignored. An entry outside that range is skipped and recorded as
+ * PHSA_ERR_DEVICE_INDEX in the device status word.
+ *   Q            bf16 [B, Hq, L, D]   in
+ *   K, V         bf16 [B, Hkv, L, D]  in
+ *   block_idx    int32 [B, Hkv, NQB, topk], block_cnt int32 [B, Hkv, NQB]  in
+ *   O            bf16 [B, Hq, L, D]   out
+ *   lse          fp32 [B, Hq, L]      out
+ */
+int phsa_sparse_attn_fwd(const void* Q, const void* K, const void* V, const int32_t* block_idx,
+                         const int32_t* block_cnt, phsa_shape s, int topk, float sm_scale,
+                         void* O, float* lse, void* stream);
+
+/* Bytes of device workspace phsa_sparse_attn_bwd needs for this shape/topk. */
+size_t phsa_sparse_attn_bwd_workspace(phsa_shape s, int topk);
+
+/*
+ * Stage (c) backward: gradients of the forward above with the selection held
+ * fixed (a hard Top-K passes no gradient to Krepr, lambda or the scores).
+ * With P_ij = exp(sm_scale q_i.k_j - lse_i), Delta_i = dO_i . O_i,
+ * dS_ij = P_ij (dO_i . v_j - Delta_i):
+ *   dV_j = sum_i P_ij dO_i;  dK_j = sm_scale sum_i dS_ij q_i;  dQ_i = sm_scale sum_j dS_ij k_j.
+ * Sums run over every query head of the KV group. Deterministic: the same
+ * inputs give bit-identical gradients.
+ *   O, lse      the forward's outputs; dO bf16 [B, Hq, L, D] in
+ *   workspace   device buffer of at least phsa_sparse_attn_bwd_workspace()
+ *               bytes, owned by the caller, contents need not be initialised
+ *   dQ          bf16 [B, Hq, L, D] out; dK, dV bf16 [B, Hkv, L, D] out
+ */
+int phsa_sparse_attn_bwd(const void* Q, const void* K, const void* V, const void* O,
+                         const void* dO, const float* lse, const int32_t* block_idx,
+                         const int32_t* block_cnt, phsa_shape s, int topk, float sm_scale,
+                         void* workspace, size_t workspace_bytes, void* dQ, void* dK, void* dV,
+                         void* stream);
+
+/*
+ * Synchronises `stream`, returns the device status word of the current
+ * device (PHSA_OK or the first device-side error code recorded since the
+ * last call) and clears it. Returns PHSA_ERR_CUDA if the synchronisation
+ * itself fails.
+ */
+int phsa_get_device_status(void* stream);
+
+/* Static, human-readable name of a phsa_status code. */
+const char* phsa_status_string(int code);
+
+/*
+ * Optional per-kernel timing (no counterpart in the paper; an instrumentation
+ * aid). phsa_profile_enable(1) makes every later kernel launch of the library
+ * record a CUDA event before and after it on the launch stream; (0) stops it.
+ * Returns the previous setting. phsa_profile_read waits for the recorded
+ * events, fills up to max_kinds entries (static kernel names, total
+ * milliseconds, launch counts; any pointer may be NULL) and clears the
+ * records. Returns the number of kernel kinds, or PHSA_ERR_CUDA.
+ */
+int phsa_profile_enable(int on);
+int phsa_profile_read(int max_kinds, const char** names, double* total_ms, int* launches);
+
+/* Library version as "major.minor.patch". */
+const char* phsa_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PHSA_H */

@@ -63,6 +63,13 @@ def _declare(L):
     L.phsa_oracle_select_blocks.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, i32,
                                             i32, f64, P, P, P]
     L.phsa_oracle_select_blocks.restype = i32
+    L.phsa_oracle_select_units.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, i32, i32,
+                                           f64, P, i64, P, P, P]
+    L.phsa_oracle_select_units.restype = i32
+    L.phsa_oracle_sparse_attn_bwd_dq_rows.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32,
+                                                      i32, i32, f64, P, i64, P]
+    L.phsa_oracle_sparse_attn_bwd_kv_blocks.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32,
+                                                        i32, i32, i32, f64, P, i64, P, P]
     L.phsa_oracle_sparse_attn_rows.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32,
                                                i32, f64, P, i64, P, P]
     L.phsa_oracle_sparse_attn_fwd.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, i32,
@@ -152,6 +159,63 @@ def select_blocks(Q, Krepr, L: int, block_size: int, topk: int, n_init: int, n_l
     if rc != 0:
         raise ValueError("topk is smaller than the forced block count")
     return (idx, cnt, agg) if want_agg else (idx, cnt)
+
+
+def select_units(Q, Krepr, L: int, block_size: int, topk: int, n_init: int, n_local: int,
+                 sm_scale: float, units):
+    """Selection for a list of flat units u = (b*Hkv + g)*NQB + qb only.
+
+    Returns (idx [n, topk], cnt [n], agg [n, T]).
+    """
+    Q = _u16(Q)
+    Krepr = _u16(Krepr)
+    B, Hq, Lq, D = Q.shape
+    assert Lq == L
+    Hkv = Krepr.shape[1]
+    T = L // block_size
+    units = np.ascontiguousarray(np.asarray(units, dtype=np.int64).ravel())
+    n = units.size
+    idx = np.empty((n, topk), dtype=np.int32)
+    cnt = np.empty((n,), dtype=np.int32)
+    agg = np.empty((n, max(T, 1)), dtype=np.float64)
+    rc = lib().phsa_oracle_select_units(_p(Q), _p(Krepr), B, Hq, Hkv, L, D, block_size, topk,
+                                        n_init, n_local, float(sm_scale), _p(units), n, _p(idx),
+                                        _p(cnt), _p(agg))
+    if rc != 0:
+        raise ValueError("topk is smaller than the forced block count")
+    return idx, cnt, agg
+
+
+def sparse_attn_bwd_dq_rows(Q, K, V, dO, block_idx, block_cnt, block_size: int,
+                            sm_scale: float, rows):
+    """dQ in fp64 for the listed rows (b, h, i) only: [n, D]."""
+    Q, K, V, dO = _u16(Q), _u16(K), _u16(V), _u16(dO)
+    block_idx, block_cnt = _i32(block_idx), _i32(block_cnt)
+    rows = _i32(rows).reshape(-1, 3)
+    B, Hq, L, D = Q.shape
+    out = np.empty((rows.shape[0], D), dtype=np.float64)
+    lib().phsa_oracle_sparse_attn_bwd_dq_rows(_p(Q), _p(K), _p(V), _p(dO), _p(block_idx),
+                                              _p(block_cnt), B, Hq, K.shape[1], L, D, block_size,
+                                              block_idx.shape[-1], float(sm_scale), _p(rows),
+                                              rows.shape[0], _p(out))
+    return out
+
+
+def sparse_attn_bwd_kv_blocks(Q, K, V, dO, block_idx, block_cnt, block_size: int,
+                              sm_scale: float, blocks):
+    """dK, dV in fp64 for every key of the listed KV blocks (b, g, t): [n, m, D] each."""
+    Q, K, V, dO = _u16(Q), _u16(K), _u16(V), _u16(dO)
+    block_idx, block_cnt = _i32(block_idx), _i32(block_cnt)
+    blocks = _i32(blocks).reshape(-1, 3)
+    B, Hq, L, D = Q.shape
+    n = blocks.shape[0]
+    dK = np.empty((n, block_size, D), dtype=np.float64)
+    dV = np.empty((n, block_size, D), dtype=np.float64)
+    lib().phsa_oracle_sparse_attn_bwd_kv_blocks(_p(Q), _p(K), _p(V), _p(dO), _p(block_idx),
+                                                _p(block_cnt), B, Hq, K.shape[1], L, D,
+                                                block_size, block_idx.shape[-1], float(sm_scale),
+                                                _p(blocks), n, _p(dK), _p(dV))
+    return dK, dV
 
 
 def sparse_attn_fwd(Q, K, V, block_idx, block_cnt, block_size: int, sm_scale: float):

@@ -175,6 +175,72 @@ static int is_forced(int t, int qb, int n_init, int n_local) {
     return t < n_init || t >= qb - n_local + 1;
 }
 
+/* Selection for one (b, g, qb) unit u = (b*Hkv + g)*NQB + qb. Writes topk
+ * entries to out, returns the count, or -1 if topk < |F_b|. If agg is not NULL
+ * it receives A_t for the T blocks (NaN where t was not scored). */
+static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv, int L, int D,
+                       int m, int topk, int n_init, int n_local, double scale, int64_t u,
+                       int32_t* out, double* agg) {
+    const int G = Hq / Hkv, T = L / m, NQB = (L + m - 1) / m;
+    const int qb = (int)(u % NQB);
+    const int g = (int)((u / NQB) % Hkv);
+    const int b = (int)(u / ((int64_t)NQB * Hkv));
+    double* A = (double*)calloc((size_t)(T > 0 ? T : 1), sizeof(double));
+    int* cand = (int*)malloc(sizeof(int) * (size_t)(qb + 1));
+    int* chosen = (int*)calloc((size_t)(qb + 1), sizeof(int));
+    int nC = 0, nF = 0, n = -1;
+    for (int t = 0; t <= qb; ++t) {
+        if (is_forced(t, qb, n_init, n_local)) { chosen[t] = 1; ++nF; }
+        else if (t <= qb - 1 && t < T) cand[nC++] = t; /* causal: strictly past */
+    }
+    if (agg)
+        for (int t = 0; t < T; ++t) agg[t] = NAN;
+    if (topk >= nF) {
+        int ksel = topk - nF;
+        if (ksel >= nC) {
+            for (int c = 0; c < nC; ++c) chosen[cand[c]] = 1;
+        } else if (ksel > 0) {
+            double* s = (double*)malloc(sizeof(double) * (size_t)nC);
+            for (int hh = 0; hh < G; ++hh) {
+                const int h = g * G + hh;
+                for (int i = qb * m; i < (qb + 1) * m && i < L; ++i) {
+                    const uint16_t* q = Q + (((int64_t)b * Hq + h) * L + i) * D;
+                    double mx = -INFINITY;
+                    for (int c = 0; c < nC; ++c) {
+                        const uint16_t* M = Krepr + (((int64_t)b * Hkv + g) * T + cand[c]) * D;
+                        double dot = 0.0;
+                        for (int d = 0; d < D; ++d)
+                            dot += phsa_oracle_bf16_to_f64(q[d]) * phsa_oracle_bf16_to_f64(M[d]);
+                        s[c] = dot * scale; /* S_{i,t} */
+                        if (s[c] > mx) mx = s[c];
+                    }
+                    double z = 0.0;
+                    for (int c = 0; c < nC; ++c) z += exp(s[c] - mx);
+                    for (int c = 0; c < nC; ++c) A[cand[c]] += exp(s[c] - mx) / z; /* R2 */
+                }
+            }
+            free(s);
+            cand_t* order = (cand_t*)malloc(sizeof(cand_t) * (size_t)nC);
+            for (int c = 0; c < nC; ++c) {
+                order[c].a32 = (float)A[cand[c]];
+                order[c].t = cand[c];
+                if (agg) agg[cand[c]] = A[cand[c]];
+            }
+            qsort(order, (size_t)nC, sizeof(cand_t), cand_cmp);
+            for (int c = 0; c < ksel; ++c) chosen[order[c].t] = 1;
+            free(order);
+        }
+        n = 0;
+        for (int t = 0; t <= qb; ++t)
+            if (chosen[t]) out[n++] = t; /* Unique, ascending */
+        for (int j = n; j < topk; ++j) out[j] = -1;
+    }
+    free(A);
+    free(cand);
+    free(chosen);
+    return n;
+}
+
 /* Q [B,Hq,L,D] bf16, Krepr [B,Hkv,T,D] bf16.
  * Outputs block_idx [B,Hkv,NQB,topk] (ascending, -1 padded), block_cnt
  * [B,Hkv,NQB]. If agg is not NULL it receives A_t [B,Hkv,NQB,T] for every
@@ -185,75 +251,38 @@ int phsa_oracle_select_blocks(const uint16_t* Q, const uint16_t* Krepr, int B, i
                               int Hkv, int L, int D, int m, int topk, int n_init, int n_local,
                               double scale, int32_t* block_idx, int32_t* block_cnt,
                               double* agg) {
-    const int G = Hq / Hkv, T = L / m, NQB = (L + m - 1) / m;
+    const int T = L / m, NQB = (L + m - 1) / m;
     int bad = 0;
     const int64_t units = (int64_t)B * Hkv * NQB;
 #ifdef _OPENMP
 #pragma omp parallel for schedule(dynamic, 1) num_threads(NTH) reduction(| : bad)
 #endif
     for (int64_t u = 0; u < units; ++u) {
-        const int qb = (int)(u % NQB);
-        const int g = (int)((u / NQB) % Hkv);
-        const int b = (int)(u / ((int64_t)NQB * Hkv));
-        int32_t* out = block_idx + u * topk;
-        double* A = (double*)calloc((size_t)(T > 0 ? T : 1), sizeof(double));
-        int* cand = (int*)malloc(sizeof(int) * (size_t)(qb + 1));
-        int* chosen = (int*)calloc((size_t)(qb + 1), sizeof(int));
-        int nC = 0, nF = 0;
-        for (int t = 0; t <= qb; ++t) {
-            if (is_forced(t, qb, n_init, n_local)) { chosen[t] = 1; ++nF; }
-            else if (t <= qb - 1 && t < T) cand[nC++] = t; /* causal: strictly past */
-        }
-        if (agg)
-            for (int t = 0; t < T; ++t) agg[u * T + t] = NAN;
-        if (topk < nF) {
-            bad = 1;
-        } else {
-            int ksel = topk - nF;
-            if (ksel >= nC) {
-                for (int c = 0; c < nC; ++c) chosen[cand[c]] = 1;
-            } else if (ksel > 0) {
-                double* s = (double*)malloc(sizeof(double) * (size_t)nC);
-                for (int hh = 0; hh < G; ++hh) {
-                    const int h = g * G + hh;
-                    for (int i = qb * m; i < (qb + 1) * m && i < L; ++i) {
-                        const uint16_t* q = Q + (((int64_t)b * Hq + h) * L + i) * D;
-                        double mx = -INFINITY;
-                        for (int c = 0; c < nC; ++c) {
-                            const uint16_t* M =
-                                Krepr + (((int64_t)b * Hkv + g) * T + cand[c]) * D;
-                            double dot = 0.0;
-                            for (int d = 0; d < D; ++d)
-                                dot += phsa_oracle_bf16_to_f64(q[d]) *
-                                       phsa_oracle_bf16_to_f64(M[d]);
-                            s[c] = dot * scale; /* S_{i,t} */
-                            if (s[c] > mx) mx = s[c];
-                        }
-                        double z = 0.0;
-                        for (int c = 0; c < nC; ++c) z += exp(s[c] - mx);
-                        for (int c = 0; c < nC; ++c) A[cand[c]] += exp(s[c] - mx) / z; /* R2 */
-                    }
-                }
-                free(s);
-                cand_t* order = (cand_t*)malloc(sizeof(cand_t) * (size_t)nC);
-                for (int c = 0; c < nC; ++c) {
-                    order[c].a32 = (float)A[cand[c]];
-                    order[c].t = cand[c];
-                    if (agg) agg[u * T + cand[c]] = A[cand[c]];
-                }
-                qsort(order, (size_t)nC, sizeof(cand_t), cand_cmp);
-                for (int c = 0; c < ksel; ++c) chosen[order[c].t] = 1;
-                free(order);
-            }
-            int n = 0;
-            for (int t = 0; t <= qb; ++t)
-                if (chosen[t]) out[n++] = t; /* Unique, ascending */
-            block_cnt[u] = n;
-            for (int j = n; j < topk; ++j) out[j] = -1;
-        }
-        free(A);
-        free(cand);
-        free(chosen);
+        int n = select_unit(Q, Krepr, Hq, Hkv, L, D, m, topk, n_init, n_local, scale, u,
+                            block_idx + u * topk, agg ? agg + u * T : NULL);
+        block_cnt[u] = n;
+        if (n < 0) bad = 1;
+    }
+    return bad ? -1 : 0;
+}
+
+/* The same selection for a list of units only (sampled checks of large
+ * problems): idx [n_units, topk], cnt [n_units], agg [n_units, T] or NULL. */
+int phsa_oracle_select_units(const uint16_t* Q, const uint16_t* Krepr, int B, int Hq, int Hkv,
+                             int L, int D, int m, int topk, int n_init, int n_local,
+                             double scale, const int64_t* units, int64_t n_units,
+                             int32_t* idx, int32_t* cnt, double* agg) {
+    const int T = L / m;
+    int bad = 0;
+    (void)B;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(NTH) reduction(| : bad)
+#endif
+    for (int64_t k = 0; k < n_units; ++k) {
+        int n = select_unit(Q, Krepr, Hq, Hkv, L, D, m, topk, n_init, n_local, scale, units[k],
+                            idx + k * topk, agg ? agg + k * T : NULL);
+        cnt[k] = n;
+        if (n < 0) bad = 1;
     }
     return bad ? -1 : 0;
 }
@@ -412,6 +441,119 @@ void phsa_oracle_sparse_attn_bwd(const uint16_t* Q, const uint16_t* K, const uin
                         dVg[(int64_t)j * D + d] += p * phsa_oracle_bf16_to_f64(go[d]);
                         dKg[(int64_t)j * D + d] += ds * phsa_oracle_bf16_to_f64(q[d]) * scale;
                         dQ[r * D + d] += ds * phsa_oracle_bf16_to_f64(k[d]) * scale;
+                    }
+                }
+            }
+        }
+        free(keys);
+        free(s);
+        free(o);
+    }
+}
+
+/* Sampled gradients for large problems. Same definitions as above.
+ * dQ for the listed rows (b, h, i): dQ_rows [n_rows, D]. */
+void phsa_oracle_sparse_attn_bwd_dq_rows(const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+                                         const uint16_t* dO, const int32_t* block_idx,
+                                         const int32_t* block_cnt, int B, int Hq, int Hkv, int L,
+                                         int D, int m, int topk, double scale, const int32_t* rows,
+                                         int64_t n_rows, double* dQ_rows) {
+    const int G = Hq / Hkv, NQB = (L + m - 1) / m;
+    (void)B;
+#ifdef _OPENMP
+#pragma omp parallel num_threads(NTH)
+#endif
+    {
+        int* keys = (int*)malloc(sizeof(int) * (size_t)L);
+        double* s = (double*)malloc(sizeof(double) * (size_t)L);
+        double* o = (double*)malloc(sizeof(double) * (size_t)D);
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 4)
+#endif
+        for (int64_t r = 0; r < n_rows; ++r) {
+            const int b = rows[3 * r], h = rows[3 * r + 1], i = rows[3 * r + 2];
+            const int g = h / G;
+            const int64_t su = ((int64_t)b * Hkv + g) * NQB + i / m;
+            const uint16_t* Kg = K + ((int64_t)b * Hkv + g) * L * D;
+            const uint16_t* Vg = V + ((int64_t)b * Hkv + g) * L * D;
+            const uint16_t* q = Q + (((int64_t)b * Hq + h) * L + i) * D;
+            const uint16_t* go = dO + (((int64_t)b * Hq + h) * L + i) * D;
+            int nk = row_keys(block_idx + su * topk, block_cnt[su], i, L, m, keys);
+            double lse;
+            attn_row(q, Kg, Vg, keys, nk, D, scale, s, o, &lse);
+            double delta = 0.0;
+            for (int d = 0; d < D; ++d) delta += phsa_oracle_bf16_to_f64(go[d]) * o[d];
+            double* dq = dQ_rows + r * D;
+            for (int d = 0; d < D; ++d) dq[d] = 0.0;
+            for (int n = 0; n < nk; ++n) {
+                const uint16_t* k = Kg + (int64_t)keys[n] * D;
+                const uint16_t* v = Vg + (int64_t)keys[n] * D;
+                double p = exp(s[n] - lse), dp = 0.0;
+                for (int d = 0; d < D; ++d)
+                    dp += phsa_oracle_bf16_to_f64(go[d]) * phsa_oracle_bf16_to_f64(v[d]);
+                double ds = p * (dp - delta);
+                for (int d = 0; d < D; ++d) dq[d] += ds * phsa_oracle_bf16_to_f64(k[d]) * scale;
+            }
+        }
+        free(keys);
+        free(s);
+        free(o);
+    }
+}
+
+/* dK and dV of every key of the listed KV blocks (b, g, t): dK_out, dV_out
+ * [n_blocks, m, D] (rows past L are zero). Every query row that attends a
+ * key of block t lies in a query block qb >= t whose list contains t. */
+void phsa_oracle_sparse_attn_bwd_kv_blocks(const uint16_t* Q, const uint16_t* K,
+                                           const uint16_t* V, const uint16_t* dO,
+                                           const int32_t* block_idx, const int32_t* block_cnt,
+                                           int B, int Hq, int Hkv, int L, int D, int m, int topk,
+                                           double scale, const int32_t* blocks, int64_t n_blocks,
+                                           double* dK_out, double* dV_out) {
+    const int G = Hq / Hkv, NQB = (L + m - 1) / m;
+    (void)B;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(NTH)
+#endif
+    for (int64_t k = 0; k < n_blocks; ++k) {
+        const int b = blocks[3 * k], g = blocks[3 * k + 1], t = blocks[3 * k + 2];
+        int* keys = (int*)malloc(sizeof(int) * (size_t)L);
+        double* s = (double*)malloc(sizeof(double) * (size_t)L);
+        double* o = (double*)malloc(sizeof(double) * (size_t)D);
+        double* dKb = dK_out + k * (int64_t)m * D;
+        double* dVb = dV_out + k * (int64_t)m * D;
+        memset(dKb, 0, sizeof(double) * (size_t)m * D);
+        memset(dVb, 0, sizeof(double) * (size_t)m * D);
+        const uint16_t* Kg = K + ((int64_t)b * Hkv + g) * L * D;
+        const uint16_t* Vg = V + ((int64_t)b * Hkv + g) * L * D;
+        for (int qb = t; qb < NQB; ++qb) {
+            const int64_t su = ((int64_t)b * Hkv + g) * NQB + qb;
+            int listed = 0;
+            for (int c = 0; c < block_cnt[su]; ++c) listed |= block_idx[su * topk + c] == t;
+            if (!listed) continue;
+            for (int hh = 0; hh < G; ++hh) {
+                const int h = g * G + hh;
+                for (int i = qb * m; i < (qb + 1) * m && i < L; ++i) {
+                    const uint16_t* q = Q + (((int64_t)b * Hq + h) * L + i) * D;
+                    const uint16_t* go = dO + (((int64_t)b * Hq + h) * L + i) * D;
+                    int nk = row_keys(block_idx + su * topk, block_cnt[su], i, L, m, keys);
+                    double lse;
+                    attn_row(q, Kg, Vg, keys, nk, D, scale, s, o, &lse);
+                    double delta = 0.0;
+                    for (int d = 0; d < D; ++d) delta += phsa_oracle_bf16_to_f64(go[d]) * o[d];
+                    for (int n = 0; n < nk; ++n) {
+                        const int j = keys[n];
+                        if (j / m != t) continue;
+                        const uint16_t* v = Vg + (int64_t)j * D;
+                        double p = exp(s[n] - lse), dp = 0.0;
+                        for (int d = 0; d < D; ++d)
+                            dp += phsa_oracle_bf16_to_f64(go[d]) * phsa_oracle_bf16_to_f64(v[d]);
+                        double ds = p * (dp - delta);
+                        for (int d = 0; d < D; ++d) {
+                            dVb[(int64_t)(j - t * m) * D + d] += p * phsa_oracle_bf16_to_f64(go[d]);
+                            dKb[(int64_t)(j - t * m) * D + d] +=
+                                ds * phsa_oracle_bf16_to_f64(q[d]) * scale;
+                        }
                     }
                 }
             }

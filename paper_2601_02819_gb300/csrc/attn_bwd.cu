@@ -1,0 +1,662 @@
+// Stage (c) backward: gradients of the block-sparse causal attention with the
+// block selection held fixed (the selection is a hard Top-K, so no gradient
+// reaches the representative keys, lambda or the scores).
+//
+// Kernels, in launch order, all on the caller's stream:
+//   delta      Delta_i = dO_i . O_i (fp32), half a warp per row.
+//   idx_mark   sets bit qb of bitmap[(b,g,t)] for every selected (qb -> t).
+//   idx_build  one CTA per (b,g): counts each KV block's selecting query
+//              blocks, scans, writes the ascending query-block list of every
+//              KV block (a CSR transpose of block_idx), and cuts lists longer
+//              than kChunk into chunks (one work item each) so that the first
+//              block, which every query block selects, does not serialise.
+//   dkdv       one CTA per work item (KV block t, chunk): for every listed
+//              query block and every query head of the group recomputes
+//              S^T = K Q^T, P^T, dP^T = V dO^T, dS^T and accumulates
+//              dV += P^T dO, dK += dS^T Q in registers. Single-chunk blocks
+//              write bf16 directly; multi-chunk blocks write fp32 partials.
+//   dkdv_sum   sums the partials of multi-chunk blocks in chunk order.
+//   dq         one CTA per (query block, KV head): recomputes S, P, dP, dS
+//              over the selected blocks and accumulates dQ += dS K.
+// Every sum runs in a fixed order, so results are bit-reproducible.
+#include "phsa_common.cuh"
+#include "phsa_internal.h"
+
+namespace phsa {
+
+namespace {
+
+constexpr int kChunk = 32;  // query blocks per dK/dV work item
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// ---------------------------------------------------------------- delta
+__global__ void __launch_bounds__(256)
+delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restrict__ dO,
+             long long rows, float* __restrict__ delta) {
+    const long long row = ((long long)blockIdx.x * 256 + threadIdx.x) >> 4;
+    const int c = threadIdx.x & 15;
+    float acc = 0.f;
+    if (row < rows) {
+        const uint4 a = __ldg(reinterpret_cast<const uint4*>(O + row * kD + c * 8));
+        const uint4 d = __ldg(reinterpret_cast<const uint4*>(dO + row * kD + c * 8));
+        const __nv_bfloat162* ha = reinterpret_cast<const __nv_bfloat162*>(&a);
+        const __nv_bfloat162* hd = reinterpret_cast<const __nv_bfloat162*>(&d);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 fa = __bfloat1622float2(ha[j]);
+            const float2 fd = __bfloat1622float2(hd[j]);
+            acc += fa.x * fd.x + fa.y * fd.y;
+        }
+    }
+#pragma unroll
+    for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    if (row < rows && c == 0) delta[row] = acc;
+}
+
+// ---------------------------------------------------------------- index transpose
+__global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt,
+                                long long units, int NQB, int topk, int words,
+                                uint32_t* __restrict__ bits, int* status) {
+    const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (u >= units) return;
+    const int qb = (int)(u % NQB);
+    const long long bg = u / NQB;
+    int n = cnt[u];
+    if (n < 0 || n > topk) {
+        set_status(status, PHSA_ERR_DEVICE_INDEX);
+        n = n < 0 ? 0 : topk;
+    }
+    int prev = -1;
+    for (int j = 0; j < n; ++j) {
+        const int t = idx[u * topk + j];
+        if (t == -1) continue;
+        if (t < 0 || t > qb || t <= prev) {
+            set_status(status, PHSA_ERR_DEVICE_INDEX);
+            continue;
+        }
+        prev = t;
+        atomicOr(&bits[(bg * NQB + t) * words + (qb >> 5)], 1u << (qb & 31));
+    }
+}
+
+struct TInfo {
+    int off, n, nch, slot;  // list offset, list length, chunks, first partial slot (-1: none)
+};
+
+// Block-wide exclusive scan of one int per thread (blockDim.x = 1024).
+__device__ int block_excl_scan(int v, int* tmp, int& total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, off);
+        if (lane >= off) x += y;
+    }
+    if (lane == 31) tmp[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = tmp[lane];
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, w, off);
+            if (lane >= off) w += y;
+        }
+        tmp[lane] = w;  // inclusive over warps
+    }
+    __syncthreads();
+    const int before = (warp > 0 ? tmp[warp - 1] : 0) + x - v;
+    total = tmp[31];
+    __syncthreads();
+    return before;
+}
+
+__global__ void __launch_bounds__(1024)
+idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words, int work_max,
+                 int slot_max, TInfo* __restrict__ tinfo, int32_t* __restrict__ qlist,
+                 int2* __restrict__ work, int32_t* __restrict__ nwork, int* status) {
+    __shared__ int tmp[32];
+    const int bg = blockIdx.x;
+    const int per = (NQB + 1023) / 1024;  // KV blocks handled by each thread
+    const int t0 = threadIdx.x * per;
+    const uint32_t* bb = bits + (size_t)bg * NQB * words;
+    int sn = 0, sch = 0, ssl = 0;
+    for (int k = 0; k < per; ++k) {
+        const int t = t0 + k;
+        if (t >= NQB) break;
+        int n = 0;
+        for (int w = 0; w < words; ++w) n += __popc(bb[(size_t)t * words + w]);
+        const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
+        sn += n;
+        sch += nch;
+        ssl += nch > 1 ? nch : 0;
+    }
+    int tn, tch, tsl;
+    int on = block_excl_scan(sn, tmp, tn);
+    int och = block_excl_scan(sch, tmp, tch);
+    int osl = block_excl_scan(ssl, tmp, tsl);
+    if (threadIdx.x == 0) {
+        nwork[bg] = min(tch, work_max);
+        if (tch > work_max || tsl > slot_max || tn > NQB * topk) set_status(status, PHSA_ERR_DEVICE_INDEX);
+    }
+    TInfo* ti = tinfo + (size_t)bg * NQB;
+    int32_t* ql = qlist + (size_t)bg * NQB * topk;
+    int2* wk = work + (size_t)bg * work_max;
+    for (int k = 0; k < per; ++k) {
+        const int t = t0 + k;
+        if (t >= NQB) break;
+        int n = 0;
+        for (int w = 0; w < words; ++w) {
+            uint32_t m = bb[(size_t)t * words + w];
+            while (m) {
+                const int q = w * 32 + __ffs(m) - 1;
+                m &= m - 1;
+                if (on + n < NQB * topk) ql[on + n] = q;
+                ++n;
+            }
+        }
+        const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
+        TInfo info;
+        info.off = on;
+        info.n = n;
+        info.nch = nch;
+        info.slot = (nch > 1 && osl + nch <= slot_max) ? osl : -1;
+        ti[t] = info;
+        for (int c = 0; c < nch; ++c)
+            if (och + c < work_max) wk[och + c] = make_int2(t, c);
+        on += n;
+        och += nch;
+        osl += nch > 1 ? nch : 0;
+    }
+}
+
+// ---------------------------------------------------------------- dK / dV
+constexpr int kKvThreads = 128;  // 4 warps, 16 keys each
+constexpr int kTile = kM * kD * 2;
+// smem: K, V (2 tiles) | 2 stages x (Q, dO) | 2 stages x (lse2, delta) [64 floats each]
+constexpr int kKvStageOff = 2 * kTile;
+constexpr int kKvVecOff = kKvStageOff + 4 * kTile;
+constexpr int kKvSmem = kKvVecOff + 2 * 2 * 64 * 4;
+
+__global__ void __launch_bounds__(kKvThreads)
+dkdv_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+            const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ dO,
+            const float* __restrict__ lse, const float* __restrict__ delta,
+            const TInfo* __restrict__ tinfo, const int32_t* __restrict__ qlist,
+            const int2* __restrict__ work, const int32_t* __restrict__ nwork, int Hq, int Hkv,
+            int L, int NQB, int topk, int work_max, int slot_max, float scale_log2,
+            float sm_scale, __nv_bfloat16* __restrict__ dK, __nv_bfloat16* __restrict__ dV,
+            float* __restrict__ partial) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int bg = blockIdx.y;
+    if ((int)blockIdx.x >= nwork[bg]) return;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int G = Hq / Hkv;
+    const int b = bg / Hkv, g = bg % Hkv;
+    const int2 wi = work[(size_t)bg * work_max + blockIdx.x];
+    const int t = wi.x, chunk = wi.y;
+    const TInfo info = tinfo[(size_t)bg * NQB + t];
+    const int q_begin = chunk * kChunk;
+    const int q_end = min(info.n, q_begin + kChunk);
+    const int n_iter = max(0, q_end - q_begin) * G;
+    const int32_t* ql = qlist + (size_t)bg * NQB * topk + info.off;
+
+    const uint32_t sK = smem_u32(smem), sV = sK + kTile;
+    const uint32_t sStage = sK + kKvStageOff;
+    float* vecs = reinterpret_cast<float*>(smem + kKvVecOff);
+
+    const __nv_bfloat16* Kg = K + (size_t)bg * L * kD;
+    const __nv_bfloat16* Vg = V + (size_t)bg * L * kD;
+    load_tile64<kKvThreads>(sK, Kg, t * kM, L, tid);
+    load_tile64<kKvThreads>(sV, Vg, t * kM, L, tid);
+
+    // iteration j -> (query block ql[q_begin + j / G], head g*G + j % G)
+    auto issue = [&](int j, int stage) {
+        const int qb = ql[q_begin + j / G];
+        const int h = g * G + j % G;
+        const size_t hoff = (size_t)(b * Hq + h) * L;
+        const uint32_t st = sStage + stage * 2 * kTile;
+        load_tile64<kKvThreads>(st, Q + hoff * kD, qb * kM, L, tid);
+        load_tile64<kKvThreads>(st + kTile, dO + hoff * kD, qb * kM, L, tid);
+        if (tid < 64) {
+            const int i = qb * kM + tid;
+            float* v = vecs + stage * 128;
+            v[tid] = i < L ? lse[hoff + i] * kLog2e : 0.f;
+            v[64 + tid] = i < L ? delta[hoff + i] : 0.f;
+        }
+    };
+    if (n_iter > 0) issue(0, 0);
+    cp_async_commit();
+
+    float dk[16][4], dv[16][4];
+#pragma unroll
+    for (int n = 0; n < 16; ++n)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) { dk[n][e] = 0.f; dv[n][e] = 0.f; }
+
+    const int key0 = warp * 16 + (lane >> 2);  // this lane's keys: key0, key0 + 8
+    for (int it = 0; it < n_iter; ++it) {
+        if (it + 1 < n_iter) {
+            issue(it + 1, (it + 1) & 1);
+            cp_async_commit();
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncthreads();
+        const int qb = ql[q_begin + it / G];
+        const uint32_t sQ = sStage + (it & 1) * 2 * kTile;
+        const uint32_t sdO = sQ + kTile;
+        const float* lse2 = vecs + (it & 1) * 128;
+        const float* dl = lse2 + 64;
+        const bool diag = (qb == t);
+#pragma unroll
+        for (int hq = 0; hq < 2; ++hq) {  // two halves of 32 queries
+            float sT[4][4], dpT[4][4];
+#pragma unroll
+            for (int n = 0; n < 4; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) { sT[n][e] = 0.f; dpT[n][e] = 0.f; }
+#pragma unroll
+            for (int kc = 0; kc < 8; ++kc) {
+                uint32_t ka[4], va[4];
+                load_a_frag(sK, warp * 16, kc, lane, ka);
+                load_a_frag(sV, warp * 16, kc, lane, va);
+#pragma unroll
+                for (int np = 0; np < 2; ++np) {
+                    uint32_t qb4[4], ob4[4];
+                    load_b_nk(sQ, hq * 32 + np * 16, kc, lane, qb4);
+                    load_b_nk(sdO, hq * 32 + np * 16, kc, lane, ob4);
+                    mma16816(sT[2 * np], ka, qb4[0], qb4[1]);
+                    mma16816(sT[2 * np + 1], ka, qb4[2], qb4[3]);
+                    mma16816(dpT[2 * np], va, ob4[0], ob4[1]);
+                    mma16816(dpT[2 * np + 1], va, ob4[2], ob4[3]);
+                }
+            }
+            // P^T and dS^T (rows: keys, columns: queries)
+#pragma unroll
+            for (int n = 0; n < 4; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int key = key0 + ((e >> 1) << 3);
+                    const int q = hq * 32 + n * 8 + (lane & 3) * 2 + (e & 1);
+                    const bool ok = (qb * kM + q < L) && !(diag && key > q);
+                    const float p = ok ? exp2f(sT[n][e] * scale_log2 - lse2[q]) : 0.f;
+                    sT[n][e] = p;
+                    dpT[n][e] = p * (dpT[n][e] - dl[q]);
+                }
+            // dV += P^T dO, dK += dS^T Q (k = the 32 queries of this half)
+#pragma unroll
+            for (int ks = 0; ks < 2; ++ks) {
+                uint32_t pa[4], sa[4];
+                pa[0] = pack_bf16(sT[2 * ks][0], sT[2 * ks][1]);
+                pa[1] = pack_bf16(sT[2 * ks][2], sT[2 * ks][3]);
+                pa[2] = pack_bf16(sT[2 * ks + 1][0], sT[2 * ks + 1][1]);
+                pa[3] = pack_bf16(sT[2 * ks + 1][2], sT[2 * ks + 1][3]);
+                sa[0] = pack_bf16(dpT[2 * ks][0], dpT[2 * ks][1]);
+                sa[1] = pack_bf16(dpT[2 * ks][2], dpT[2 * ks][3]);
+                sa[2] = pack_bf16(dpT[2 * ks + 1][0], dpT[2 * ks + 1][1]);
+                sa[3] = pack_bf16(dpT[2 * ks + 1][2], dpT[2 * ks + 1][3]);
+#pragma unroll
+                for (int np = 0; np < 8; ++np) {
+                    uint32_t ob[4], qb2[4];
+                    load_b_kn(sdO, hq * 32 + ks * 16, np * 2, lane, ob);
+                    load_b_kn(sQ, hq * 32 + ks * 16, np * 2, lane, qb2);
+                    mma16816(dv[2 * np], pa, ob[0], ob[1]);
+                    mma16816(dv[2 * np + 1], pa, ob[2], ob[3]);
+                    mma16816(dk[2 * np], sa, qb2[0], qb2[1]);
+                    mma16816(dk[2 * np + 1], sa, qb2[2], qb2[3]);
+                }
+            }
+        }
+        __syncthreads();
+    }
+    cp_async_wait<0>();
+    __syncthreads();
+
+    if (info.nch > 1) {
+        if (info.slot < 0) return;  // workspace bound exceeded (status already set)
+        float* pk = partial + ((size_t)bg * slot_max + info.slot + chunk) * 2 * kM * kD;
+        float* pv = pk + kM * kD;
+#pragma unroll
+        for (int n = 0; n < 16; ++n)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+                const int r = key0 + hh * 8;
+                const int c = n * 8 + (lane & 3) * 2;
+                *reinterpret_cast<float2*>(pk + r * kD + c) =
+                    make_float2(dk[n][2 * hh] * sm_scale, dk[n][2 * hh + 1] * sm_scale);
+                *reinterpret_cast<float2*>(pv + r * kD + c) = make_float2(dv[n][2 * hh], dv[n][2 * hh + 1]);
+            }
+        return;
+    }
+    // bf16 output through shared memory (K tile <- dK, V tile <- dV)
+#pragma unroll
+    for (int n = 0; n < 16; ++n)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int r = key0 + hh * 8;
+            const int c = n * 8 + (lane & 3) * 2;
+            const uint32_t off = swz(r, c >> 3) + (c & 7) * 2;
+            *reinterpret_cast<uint32_t*>(smem + off) =
+                pack_bf16(dk[n][2 * hh] * sm_scale, dk[n][2 * hh + 1] * sm_scale);
+            *reinterpret_cast<uint32_t*>(smem + kTile + off) = pack_bf16(dv[n][2 * hh], dv[n][2 * hh + 1]);
+        }
+    __syncthreads();
+    __nv_bfloat16* dKg = dK + (size_t)bg * L * kD;
+    __nv_bfloat16* dVg = dV + (size_t)bg * L * kD;
+    for (int e = tid; e < kM * kRowChunks; e += kKvThreads) {
+        const int r = e >> 4, c = e & 15;
+        const int i = t * kM + r;
+        if (i < L) {
+            *reinterpret_cast<uint4*>(dKg + (size_t)i * kD + c * 8) =
+                *reinterpret_cast<const uint4*>(smem + swz(r, c));
+            *reinterpret_cast<uint4*>(dVg + (size_t)i * kD + c * 8) =
+                *reinterpret_cast<const uint4*>(smem + kTile + swz(r, c));
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256)
+dkdv_sum_kernel(const TInfo* __restrict__ tinfo, const float* __restrict__ partial, int Hkv,
+                int L, int NQB, int slot_max, __nv_bfloat16* __restrict__ dK,
+                __nv_bfloat16* __restrict__ dV) {
+    const int t = blockIdx.x, bg = blockIdx.y;
+    const TInfo info = tinfo[(size_t)bg * NQB + t];
+    if (info.nch <= 1 || info.slot < 0) return;
+    const float* base = partial + ((size_t)bg * slot_max + info.slot) * 2 * kM * kD;
+    for (int e = threadIdx.x * 4; e < 2 * kM * kD; e += 256 * 4) {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int c = 0; c < info.nch; ++c) {
+            const float4 v = *reinterpret_cast<const float4*>(base + (size_t)c * 2 * kM * kD + e);
+            acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+        }
+        const int which = e / (kM * kD);
+        const int r = (e % (kM * kD)) / kD, col = e % kD;
+        const int i = t * kM + r;
+        if (i < L) {
+            __nv_bfloat16* dst = (which == 0 ? dK : dV) + ((size_t)bg * L + i) * kD + col;
+            uint2 pk;
+            pk.x = pack_bf16(acc.x, acc.y);
+            pk.y = pack_bf16(acc.z, acc.w);
+            *reinterpret_cast<uint2*>(dst) = pk;
+        }
+    }
+}
+
+// ---------------------------------------------------------------- dQ
+template <int G>
+struct DqCfg {
+    static constexpr int kWarps = 4 * G;
+    static constexpr int kThreads = 32 * kWarps;
+    static constexpr int kRows = 64 * G;
+    static constexpr int kQOff = 0;
+    static constexpr int kdOOff = G * kTile;
+    static constexpr int kKVOff = 2 * G * kTile;        // 2 stages x (K, V)
+    static constexpr int kVecOff = kKVOff + 4 * kTile;  // lse2[kRows], delta[kRows]
+    static constexpr int kListOff = kVecOff + 2 * kRows * 4;
+    static size_t smem_bytes(int topk) { return (size_t)kListOff + (size_t)(topk + 1) * 4; }
+};
+
+template <int G>
+__global__ void __launch_bounds__(DqCfg<G>::kThreads)
+dq_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+          const __nv_bfloat16* __restrict__ V, const __nv_bfloat16* __restrict__ dO,
+          const float* __restrict__ lse, const float* __restrict__ delta,
+          const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt, int Hq, int Hkv,
+          int L, int NQB, int topk, float scale_log2, float sm_scale,
+          __nv_bfloat16* __restrict__ dQ, int* status) {
+    using C = DqCfg<G>;
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int unit = blockIdx.x;
+    const int qb = NQB - 1 - (unit % NQB);
+    const int bg = unit / NQB;
+    const int b = bg / Hkv, g = bg % Hkv;
+    const long long lu = (long long)bg * NQB + qb;
+
+    const uint32_t sQ = smem_u32(smem) + C::kQOff;
+    const uint32_t sdO = smem_u32(smem) + C::kdOOff;
+    const uint32_t sKV = smem_u32(smem) + C::kKVOff;
+    float* lse2 = reinterpret_cast<float*>(smem + C::kVecOff);
+    float* dl = lse2 + C::kRows;
+    int* blist = reinterpret_cast<int*>(smem + C::kListOff);
+    if (tid == 0) blist[topk] = compact_block_list(idx + lu * topk, cnt[lu], topk, qb, blist, nullptr);
+
+    const __nv_bfloat16* Kg = K + (size_t)bg * L * kD;
+    const __nv_bfloat16* Vg = V + (size_t)bg * L * kD;
+#pragma unroll
+    for (int hl = 0; hl < G; ++hl) {
+        const size_t hoff = (size_t)(b * Hq + g * G + hl) * L;
+        load_tile64<C::kThreads>(sQ + hl * kTile, Q + hoff * kD, qb * kM, L, tid);
+        load_tile64<C::kThreads>(sdO + hl * kTile, dO + hoff * kD, qb * kM, L, tid);
+    }
+    for (int r = tid; r < C::kRows; r += C::kThreads) {
+        const int i = qb * kM + (r & 63);
+        const size_t hoff = (size_t)(b * Hq + g * G + (r >> 6)) * L;
+        lse2[r] = i < L ? lse[hoff + i] * kLog2e : 0.f;
+        dl[r] = i < L ? delta[hoff + i] : 0.f;
+    }
+    cp_async_commit();
+    __syncthreads();
+    const int nblk = blist[topk];
+    if (nblk > 0) {
+        load_tile64<C::kThreads>(sKV, Kg, blist[0] * kM, L, tid);
+        load_tile64<C::kThreads>(sKV + kTile, Vg, blist[0] * kM, L, tid);
+    }
+    cp_async_commit();
+
+    const int rq0 = (warp & 3) * 16 + (lane >> 2);
+    const int rw0 = warp * 16 + (lane >> 2);  // row in the stacked G*64 tile
+    uint32_t qf[8][4];
+    float dq[16][4];
+#pragma unroll
+    for (int n = 0; n < 16; ++n)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) dq[n][e] = 0.f;
+
+    for (int it = 0; it < nblk; ++it) {
+        if (it + 1 < nblk) {
+            const uint32_t st = sKV + ((it + 1) & 1) * 2 * kTile;
+            load_tile64<C::kThreads>(st, Kg, blist[it + 1] * kM, L, tid);
+            load_tile64<C::kThreads>(st + kTile, Vg, blist[it + 1] * kM, L, tid);
+            cp_async_commit();
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncthreads();
+        if (it == 0) {
+#pragma unroll
+            for (int kc = 0; kc < 8; ++kc) load_a_frag(sQ, warp * 16, kc, lane, qf[kc]);
+        }
+        const uint32_t sK = sKV + (it & 1) * 2 * kTile;
+        const uint32_t sV = sK + kTile;
+        const bool diag = (blist[it] == qb);
+        float s[8][4], dp[8][4];
+#pragma unroll
+        for (int n = 0; n < 8; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) { s[n][e] = 0.f; dp[n][e] = 0.f; }
+#pragma unroll
+        for (int kc = 0; kc < 8; ++kc) {
+            uint32_t oa[4];
+            load_a_frag(sdO, warp * 16, kc, lane, oa);
+#pragma unroll
+            for (int np = 0; np < 4; ++np) {
+                uint32_t kb[4], vb[4];
+                load_b_nk(sK, np * 16, kc, lane, kb);
+                load_b_nk(sV, np * 16, kc, lane, vb);
+                mma16816(s[2 * np], qf[kc], kb[0], kb[1]);
+                mma16816(s[2 * np + 1], qf[kc], kb[2], kb[3]);
+                mma16816(dp[2 * np], oa, vb[0], vb[1]);
+                mma16816(dp[2 * np + 1], oa, vb[2], vb[3]);
+            }
+        }
+#pragma unroll
+        for (int n = 0; n < 8; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int key = n * 8 + (lane & 3) * 2 + (e & 1);
+                const int hh = e >> 1;
+                const int row = rq0 + hh * 8;
+                const int rw = rw0 + hh * 8;
+                const bool ok = (qb * kM + row < L) && !(diag && key > row);
+                const float p = ok ? exp2f(s[n][e] * scale_log2 - lse2[rw]) : 0.f;
+                s[n][e] = p * (dp[n][e] - dl[rw]);  // dS
+            }
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+            uint32_t sa[4];
+            sa[0] = pack_bf16(s[2 * ks][0], s[2 * ks][1]);
+            sa[1] = pack_bf16(s[2 * ks][2], s[2 * ks][3]);
+            sa[2] = pack_bf16(s[2 * ks + 1][0], s[2 * ks + 1][1]);
+            sa[3] = pack_bf16(s[2 * ks + 1][2], s[2 * ks + 1][3]);
+#pragma unroll
+            for (int np = 0; np < 8; ++np) {
+                uint32_t kb[4];
+                load_b_kn(sK, ks * 16, np * 2, lane, kb);
+                mma16816(dq[2 * np], sa, kb[0], kb[1]);
+                mma16816(dq[2 * np + 1], sa, kb[2], kb[3]);
+            }
+        }
+        __syncthreads();
+    }
+    cp_async_wait<0>();
+    __syncthreads();
+
+    const int h = g * G + (warp >> 2);
+#pragma unroll
+    for (int n = 0; n < 16; ++n)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int r = rw0 + hh * 8;
+            const int c = n * 8 + (lane & 3) * 2;
+            *reinterpret_cast<uint32_t*>(smem + C::kQOff + swz(r, c >> 3) + (c & 7) * 2) =
+                pack_bf16(dq[n][2 * hh] * sm_scale, dq[n][2 * hh + 1] * sm_scale);
+        }
+    __syncwarp();
+    __nv_bfloat16* dQh = dQ + (size_t)(b * Hq + h) * L * kD;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int e = k * 32 + lane;
+        const int r = e >> 4, c = e & 15;
+        const int i = qb * kM + (warp & 3) * 16 + r;
+        if (i < L)
+            *reinterpret_cast<uint4*>(dQh + (size_t)i * kD + c * 8) =
+                *reinterpret_cast<const uint4*>(smem + C::kQOff + swz(warp * 16 + r, c));
+    }
+}
+
+template <int G>
+cudaError_t launch_dq_g(const void* Q, const void* K, const void* V, const void* dO,
+                        const float* lse, const float* delta, const int32_t* idx,
+                        const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                        void* dQ, int* status, cudaStream_t st) {
+    const int NQB = (s.L + kM - 1) / kM;
+    const size_t smem = DqCfg<G>::smem_bytes(topk);
+    auto kern = dq_kernel<G>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    ProfScope prof(K_BWD_DQ, st);
+    kern<<<(unsigned)((long long)s.B * s.Hkv * NQB), DqCfg<G>::kThreads, smem, st>>>(
+        static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(K),
+        static_cast<const __nv_bfloat16*>(V), static_cast<const __nv_bfloat16*>(dO), lse, delta,
+        idx, cnt, s.Hq, s.Hkv, s.L, NQB, topk, sm_scale * kLog2e, sm_scale,
+        static_cast<__nv_bfloat16*>(dQ), status);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+BwdLayout bwd_layout(const phsa_shape& s, int topk) {
+    BwdLayout l{};
+    l.nqb = (s.L + kM - 1) / kM;
+    l.words = (l.nqb + 31) / 32;
+    l.chunk = kChunk;
+    const long long bgs = (long long)s.B * s.Hkv;
+    const long long nnz_max = (long long)l.nqb * topk;  // per (b, g)
+    l.work_max = (int)(l.nqb + (nnz_max + kChunk - 1) / kChunk);
+    l.slot_max = (int)((2 * nnz_max + kChunk - 1) / kChunk);
+    size_t off = 0;
+    l.bits = off;    off = align256(off + (size_t)bgs * l.nqb * l.words * 4);
+    l.tinfo = off;   off = align256(off + (size_t)bgs * l.nqb * sizeof(TInfo));
+    l.qlist = off;   off = align256(off + (size_t)bgs * nnz_max * 4);
+    l.work = off;    off = align256(off + (size_t)bgs * l.work_max * sizeof(int2));
+    l.nwork = off;   off = align256(off + (size_t)bgs * 4);
+    l.delta = off;   off = align256(off + (size_t)s.B * s.Hq * s.L * 4);
+    l.partial = off; off = align256(off + (size_t)bgs * l.slot_max * 2 * kM * kD * 4);
+    l.total = off;
+    return l;
+}
+
+cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const void* O,
+                            const void* dO, const float* lse, const int32_t* idx,
+                            const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                            void* ws, void* dQ, void* dK, void* dV, int* status,
+                            cudaStream_t st) {
+    if ((long long)s.B * s.Hkv * s.L == 0) return cudaSuccess;
+    const BwdLayout l = bwd_layout(s, topk);
+    uint8_t* w = static_cast<uint8_t*>(ws);
+    uint32_t* bits = reinterpret_cast<uint32_t*>(w + l.bits);
+    TInfo* tinfo = reinterpret_cast<TInfo*>(w + l.tinfo);
+    int32_t* qlist = reinterpret_cast<int32_t*>(w + l.qlist);
+    int2* work = reinterpret_cast<int2*>(w + l.work);
+    int32_t* nwork = reinterpret_cast<int32_t*>(w + l.nwork);
+    float* delta = reinterpret_cast<float*>(w + l.delta);
+    float* partial = reinterpret_cast<float*>(w + l.partial);
+    const int bgs = s.B * s.Hkv;
+    const long long rows = (long long)s.B * s.Hq * s.L;
+    cudaError_t e;
+
+    {
+        ProfScope prof(K_BWD_DELTA, st);
+        delta_kernel<<<(unsigned)((rows * 16 + 255) / 256), 256, 0, st>>>(
+            static_cast<const __nv_bfloat16*>(O), static_cast<const __nv_bfloat16*>(dO), rows,
+            delta);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+
+    if ((e = cudaMemsetAsync(bits, 0, (size_t)bgs * l.nqb * l.words * 4, st)) != cudaSuccess)
+        return e;
+    const long long units = (long long)bgs * l.nqb;
+    {
+        ProfScope prof(K_BWD_MARK, st);
+        idx_mark_kernel<<<(unsigned)((units + 255) / 256), 256, 0, st>>>(
+            idx, cnt, units, l.nqb, topk, l.words, bits, status);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    {
+        ProfScope prof(K_BWD_BUILD, st);
+        idx_build_kernel<<<bgs, 1024, 0, st>>>(bits, l.nqb, topk, l.words, l.work_max,
+                                               l.slot_max, tinfo, qlist, work, nwork, status);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+
+    e = cudaFuncSetAttribute(dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kKvSmem);
+    if (e != cudaSuccess) return e;
+    {
+        ProfScope prof(K_BWD_DKDV, st);
+        dkdv_kernel<<<dim3(l.work_max, bgs), kKvThreads, kKvSmem, st>>>(
+            static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(K),
+            static_cast<const __nv_bfloat16*>(V), static_cast<const __nv_bfloat16*>(dO), lse,
+            delta, tinfo, qlist, work, nwork, s.Hq, s.Hkv, s.L, l.nqb, topk, l.work_max,
+            l.slot_max, sm_scale * kLog2e, sm_scale, static_cast<__nv_bfloat16*>(dK),
+            static_cast<__nv_bfloat16*>(dV), partial);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    {
+        ProfScope prof(K_BWD_DKDV_SUM, st);
+        dkdv_sum_kernel<<<dim3(l.nqb, bgs), 256, 0, st>>>(
+            tinfo, partial, s.Hkv, s.L, l.nqb, l.slot_max, static_cast<__nv_bfloat16*>(dK),
+            static_cast<__nv_bfloat16*>(dV));
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+
+    return (s.Hq / s.Hkv == 2)
+               ? launch_dq_g<2>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st)
+               : launch_dq_g<1>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
+}
+
+}  // namespace phsa

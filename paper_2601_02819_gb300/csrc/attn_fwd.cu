@@ -1,0 +1,239 @@
+// Stage (c) forward: causal attention over the selected KV blocks (Eq. 10-11;
+// Algorithm 1 step 4), one CTA per (query block qb, KV head g).
+//
+// The G query heads of the KV group are packed into one G*64-row tile, so each
+// gathered 64 x 128 K/V block is loaded once and used by every head of the
+// group. Blocks are visited in ascending order with a double-buffered cp.async
+// pipeline; S = Q K^T and O += P V run as bf16 warp MMAs with fp32
+// accumulators, and the softmax is computed online in the log2 domain
+// (FlashAttention-style). Inside the query's own block the token-level causal
+// mask applies. Outputs: O in bf16 and the natural-log LSE per row.
+#include "phsa_common.cuh"
+#include "phsa_internal.h"
+
+namespace phsa {
+
+namespace {
+
+template <int G>
+struct FwdCfg {
+    static constexpr int kWarps = 4 * G;
+    static constexpr int kThreads = 32 * kWarps;
+    static constexpr int kRows = 64 * G;
+    static constexpr int kTile = kM * kD * 2;          // one 64 x 128 bf16 tile
+    static constexpr int kQBytes = G * kTile;
+    static constexpr int kStage = 2 * kTile;           // K and V of one block
+    static constexpr int kListOff = kQBytes + 2 * kStage;
+    static size_t smem_bytes(int topk) { return (size_t)kListOff + (size_t)(topk + 1) * 4; }
+};
+
+}  // namespace
+
+namespace {
+
+template <int G>
+__global__ void __launch_bounds__(FwdCfg<G>::kThreads)
+attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
+                const __nv_bfloat16* __restrict__ V, const int32_t* __restrict__ idx,
+                const int32_t* __restrict__ cnt, int Hq, int Hkv, int L, int NQB, int topk,
+                float scale_log2, __nv_bfloat16* __restrict__ O, float* __restrict__ lse,
+                int* status) {
+    using C = FwdCfg<G>;
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int unit = blockIdx.x;
+    const int qb = NQB - 1 - (unit % NQB);
+    const int bg = unit / NQB;
+    const int b = bg / Hkv, g = bg % Hkv;
+    const long long lu = (long long)bg * NQB + qb;
+
+    const uint32_t sQ = smem_u32(smem);
+    const uint32_t sKV = sQ + C::kQBytes;
+    int* blist = reinterpret_cast<int*>(smem + C::kListOff);
+    if (tid == 0) blist[topk] = compact_block_list(idx + lu * topk, cnt[lu], topk, qb, blist, status);
+
+    const __nv_bfloat16* Kg = K + (size_t)bg * L * kD;
+    const __nv_bfloat16* Vg = V + (size_t)bg * L * kD;
+#pragma unroll
+    for (int hl = 0; hl < G; ++hl)
+        load_tile64<C::kThreads>(sQ + hl * C::kTile, Q + (size_t)(b * Hq + g * G + hl) * L * kD,
+                                 qb * kM, L, tid);
+    cp_async_commit();
+    __syncthreads();
+    const int nblk = blist[topk];
+    if (nblk > 0) {
+        load_tile64<C::kThreads>(sKV, Kg, blist[0] * kM, L, tid);
+        load_tile64<C::kThreads>(sKV + C::kTile, Vg, blist[0] * kM, L, tid);
+    }
+    cp_async_commit();
+
+    const int rq0 = (warp & 3) * 16 + (lane >> 2);  // query row within the block (and +8)
+    uint32_t qf[8][4];
+    float o[16][4];
+#pragma unroll
+    for (int n = 0; n < 16; ++n)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) o[n][e] = 0.f;
+    float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+
+    for (int it = 0; it < nblk; ++it) {
+        if (it + 1 < nblk) {
+            const uint32_t st = sKV + ((it + 1) & 1) * C::kStage;
+            load_tile64<C::kThreads>(st, Kg, blist[it + 1] * kM, L, tid);
+            load_tile64<C::kThreads>(st + C::kTile, Vg, blist[it + 1] * kM, L, tid);
+            cp_async_commit();
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncthreads();
+        if (it == 0) {
+#pragma unroll
+            for (int kc = 0; kc < 8; ++kc) load_a_frag(sQ, warp * 16, kc, lane, qf[kc]);
+        }
+        const uint32_t sK = sKV + (it & 1) * C::kStage;
+        const uint32_t sV = sK + C::kTile;
+        const int t = blist[it];
+
+        float s[8][4];
+#pragma unroll
+        for (int n = 0; n < 8; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) s[n][e] = 0.f;
+#pragma unroll
+        for (int kc = 0; kc < 8; ++kc) {
+#pragma unroll
+            for (int np = 0; np < 4; ++np) {
+                uint32_t bb[4];
+                load_b_nk(sK, np * 16, kc, lane, bb);
+                mma16816(s[2 * np], qf[kc], bb[0], bb[1]);
+                mma16816(s[2 * np + 1], qf[kc], bb[2], bb[3]);
+            }
+        }
+        const bool diag = (t == qb);
+#pragma unroll
+        for (int n = 0; n < 8; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int key = n * 8 + (lane & 3) * 2 + (e & 1);
+                const int row = rq0 + ((e >> 1) << 3);
+                s[n][e] = (diag && key > row) ? -INFINITY : s[n][e] * scale_log2;
+            }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            float mx = -INFINITY;
+#pragma unroll
+            for (int n = 0; n < 8; ++n) mx = fmaxf(mx, fmaxf(s[n][2 * h], s[n][2 * h + 1]));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+            const float mnew = fmaxf(mrow[h], mx);
+            const float base = (mnew == -INFINITY) ? 0.f : mnew;
+            const float alpha = exp2f(mrow[h] - base);
+            mrow[h] = mnew;
+            float rs = 0.f;
+#pragma unroll
+            for (int n = 0; n < 8; ++n) {
+                s[n][2 * h] = exp2f(s[n][2 * h] - base);
+                s[n][2 * h + 1] = exp2f(s[n][2 * h + 1] - base);
+                rs += s[n][2 * h] + s[n][2 * h + 1];
+            }
+            lrow[h] = lrow[h] * alpha + rs;
+#pragma unroll
+            for (int n = 0; n < 16; ++n) {
+                o[n][2 * h] *= alpha;
+                o[n][2 * h + 1] *= alpha;
+            }
+        }
+        // O += P V, P re-used from the S accumulators as bf16 A fragments.
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+            uint32_t pa[4];
+            pa[0] = pack_bf16(s[2 * ks][0], s[2 * ks][1]);
+            pa[1] = pack_bf16(s[2 * ks][2], s[2 * ks][3]);
+            pa[2] = pack_bf16(s[2 * ks + 1][0], s[2 * ks + 1][1]);
+            pa[3] = pack_bf16(s[2 * ks + 1][2], s[2 * ks + 1][3]);
+#pragma unroll
+            for (int np = 0; np < 8; ++np) {
+                uint32_t bb[4];
+                load_b_kn(sV, ks * 16, np * 2, lane, bb);
+                mma16816(o[2 * np], pa, bb[0], bb[1]);
+                mma16816(o[2 * np + 1], pa, bb[2], bb[3]);
+            }
+        }
+        __syncthreads();
+    }
+    cp_async_wait<0>();
+    __syncthreads();
+
+    // Epilogue: normalise, stage the warp's 16 rows in its own Q rows, store.
+    const int h = g * G + (warp >> 2);
+    float inv[2];
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+        float l = lrow[hh];
+        l += __shfl_xor_sync(0xffffffffu, l, 1);
+        l += __shfl_xor_sync(0xffffffffu, l, 2);
+        inv[hh] = l > 0.f ? 1.0f / l : 0.f;
+        const int i = qb * kM + rq0 + hh * 8;
+        if ((lane & 3) == 0 && i < L) {
+            lse[(size_t)(b * Hq + h) * L + i] =
+                l > 0.f ? (mrow[hh] + log2f(l)) * kLn2 : -INFINITY;
+        }
+    }
+    uint8_t* sq = smem;
+#pragma unroll
+    for (int n = 0; n < 16; ++n) {
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int r = warp * 16 + (lane >> 2) + hh * 8;
+            const int c = n * 8 + (lane & 3) * 2;  // column
+            const uint32_t off = swz(r, c >> 3) + (c & 7) * 2;
+            *reinterpret_cast<uint32_t*>(sq + off) =
+                pack_bf16(o[n][2 * hh] * inv[hh], o[n][2 * hh + 1] * inv[hh]);
+        }
+    }
+    __syncwarp();
+    __nv_bfloat16* Oh = O + (size_t)(b * Hq + h) * L * kD;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int e = k * 32 + lane;
+        const int r = e >> 4, c = e & 15;
+        const int i = qb * kM + (warp & 3) * 16 + r;
+        if (i < L) {
+            const uint4 v = *reinterpret_cast<const uint4*>(sq + swz(warp * 16 + r, c));
+            *reinterpret_cast<uint4*>(Oh + (size_t)i * kD + c * 8) = v;
+        }
+    }
+}
+
+template <int G>
+cudaError_t launch_fwd_g(const void* Q, const void* K, const void* V, const int32_t* idx,
+                         const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                         void* O, float* lse, int* status, cudaStream_t st) {
+    const int NQB = (s.L + kM - 1) / kM;
+    const size_t smem = FwdCfg<G>::smem_bytes(topk);
+    auto kern = attn_fwd_kernel<G>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const long long grid = (long long)s.B * s.Hkv * NQB;
+    ProfScope prof(K_FWD, st);
+    kern<<<(unsigned)grid, FwdCfg<G>::kThreads, smem, st>>>(
+        static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(K),
+        static_cast<const __nv_bfloat16*>(V), idx, cnt, s.Hq, s.Hkv, s.L, NQB, topk,
+        sm_scale * kLog2e, static_cast<__nv_bfloat16*>(O), lse, status);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const int32_t* idx,
+                            const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                            void* O, float* lse, int* status, cudaStream_t st) {
+    if ((long long)s.B * s.Hkv * s.L == 0) return cudaSuccess;
+    return (s.Hq / s.Hkv == 2)
+               ? launch_fwd_g<2>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st)
+               : launch_fwd_g<1>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st);
+}
+
+}  // namespace phsa

@@ -1,0 +1,110 @@
+// Stage (a): representative key of every KV block (Section 3.2, Eq. 6-8;
+// Algorithm 1 step 2).
+//
+// One warp reduces one 64 x 128 bf16 block (16 KB). Each half-warp streams one
+// 256-byte row per step with 16-byte read-only loads (lane c of the half owns
+// columns 8c..8c+7), so a warp keeps eight 512-byte row pairs in flight. The
+// punctuation count of the block comes from two warp ballots over the 64 mask
+// bytes. The sum and the punctuation-masked sum are kept in fp32 and combined
+// once across the two half-warps; the result is rounded to bf16 once.
+// The kernel is bound by HBM: it reads K and the mask once and writes T rows.
+#include "phsa_common.cuh"
+#include "phsa_internal.h"
+
+namespace phsa {
+
+namespace {
+
+constexpr int kWarpsPerCta = 8;
+
+__device__ __forceinline__ void add8(float* acc, const uint4& v) {
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        float2 f = __bfloat1622float2(h[j]);
+        acc[2 * j] += f.x;
+        acc[2 * j + 1] += f.y;
+    }
+}
+
+__global__ void __launch_bounds__(kWarpsPerCta * 32)
+block_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict__ mask, int Hkv,
+                  int L, int T, long long n_blocks, float lambda,
+                  __nv_bfloat16* __restrict__ Krepr) {
+    const int lane = threadIdx.x & 31;
+    const long long wid = (long long)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
+    if (wid >= n_blocks) return;
+    const int t = (int)(wid % T);
+    const long long bg = wid / T;  // b * Hkv + g
+    const int b = (int)(bg / Hkv);
+
+    // Punctuation indicator of the block's 64 tokens.
+    const uint8_t* mrow = mask + (size_t)b * L + (size_t)t * kM;
+    const unsigned lo = __ballot_sync(0xffffffffu, mrow[lane] != 0);
+    const unsigned hi = __ballot_sync(0xffffffffu, mrow[32 + lane] != 0);
+    const int c = __popc(lo) + __popc(hi);
+
+    const int half = lane >> 4;
+    const int col = lane & 15;
+    const __nv_bfloat16* kb = K + ((size_t)bg * L + (size_t)t * kM) * kD + col * 8;
+
+    float s0[8], sp[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) { s0[j] = 0.f; sp[j] = 0.f; }
+
+#pragma unroll
+    for (int base = 0; base < kM; base += 16) {
+        uint4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int r = base + 2 * u + half;
+            v[u] = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)r * kD));
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int r = base + 2 * u + half;
+            add8(s0, v[u]);
+            const bool p = ((r < 32 ? lo >> r : hi >> (r - 32)) & 1u) != 0;
+            if (p) add8(sp, v[u]);
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        s0[j] += __shfl_xor_sync(0xffffffffu, s0[j], 16);
+        sp[j] += __shfl_xor_sync(0xffffffffu, sp[j], 16);
+    }
+    if (half == 0) {
+        float out[8];
+        const float inv_m = 1.0f / kM;
+        const float inv_c = c > 0 ? 1.0f / (float)c : 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const float m0 = s0[j] * inv_m;                                // Eq. 6
+            out[j] = c > 0 ? lambda * m0 + (1.0f - lambda) * (sp[j] * inv_c)  // Eq. 7-8
+                           : m0;                                           // no punctuation
+        }
+        uint4 pk;
+        pk.x = pack_bf16(out[0], out[1]);
+        pk.y = pack_bf16(out[2], out[3]);
+        pk.z = pack_bf16(out[4], out[5]);
+        pk.w = pack_bf16(out[6], out[7]);
+        *reinterpret_cast<uint4*>(Krepr + ((size_t)bg * T + t) * kD + col * 8) = pk;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_block_repr(const void* K, const uint8_t* mask, const phsa_shape& s,
+                              float lambda, void* Krepr, cudaStream_t st) {
+    const int T = s.L / kM;
+    const long long n_blocks = (long long)s.B * s.Hkv * T;
+    if (n_blocks == 0) return cudaSuccess;
+    const long long grid = (n_blocks + kWarpsPerCta - 1) / kWarpsPerCta;
+    ProfScope prof(K_REPR, st);
+    block_repr_kernel<<<(unsigned)grid, kWarpsPerCta * 32, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(K), mask, s.Hkv, s.L, T, n_blocks, lambda,
+        static_cast<__nv_bfloat16*>(Krepr));
+    return cudaGetLastError();
+}
+
+}  // namespace phsa

@@ -1,0 +1,170 @@
+// The C ABI (include/phsa.h): argument validation, the per-device status
+// word, and dispatch to the kernel launchers.
+#include <mutex>
+
+#include "phsa_common.cuh"
+#include "phsa_internal.h"
+
+namespace phsa {
+size_t select_smem_bytes(const phsa_shape& s, int topk);
+}
+
+namespace {
+
+// One status word per device, in a file-scope device variable (no allocation).
+__device__ int g_device_status = 0;
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+int* g_status_ptr[kMaxDevices] = {nullptr};
+
+// Device address of the status word on the current device (looked up once).
+int* status_ptr() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_status_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
+        g_status_ptr[dev] = static_cast<int*>(p);
+    }
+    return g_status_ptr[dev];
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Common shape checks; returns PHSA_OK or an error code.
+int check_shape(const phsa_shape& s) {
+    if (s.B < 0 || s.L < 0 || s.Hq <= 0 || s.Hkv <= 0 || s.D <= 0 || s.block_size <= 0)
+        return PHSA_ERR_INVALID_ARG;
+    if (s.Hq % s.Hkv != 0) return PHSA_ERR_INVALID_ARG;
+    if (s.D != phsa::kD || s.block_size != phsa::kM) return PHSA_ERR_UNSUPPORTED;
+    const int G = s.Hq / s.Hkv;
+    if (G != 1 && G != 2) return PHSA_ERR_UNSUPPORTED;
+    const long long nqb = ((long long)s.L + phsa::kM - 1) / phsa::kM;
+    if ((long long)s.B * s.Hkv * nqb > 0x7fffffffLL) return PHSA_ERR_UNSUPPORTED;
+    if ((long long)s.B * s.Hq > 0x7fffffffLL / (s.L > 0 ? s.L : 1)) return PHSA_ERR_UNSUPPORTED;
+    if (s.B > 65535 * 8 || (long long)s.B * s.Hkv > 65535) return PHSA_ERR_UNSUPPORTED;
+    return PHSA_OK;
+}
+
+bool empty(const phsa_shape& s) { return s.B == 0 || s.L == 0; }
+
+int from_cuda(cudaError_t e) { return e == cudaSuccess ? PHSA_OK : PHSA_ERR_CUDA; }
+
+int check_topk(const phsa_shape& s, int topk) {
+    if (topk < 1) return PHSA_ERR_INVALID_ARG;
+    if (topk > 4096) return PHSA_ERR_UNSUPPORTED;
+    (void)s;
+    return PHSA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int phsa_build_block_repr(const void* K, const uint8_t* punct_mask, phsa_shape s, float lambda,
+                          void* Krepr, void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
+    if (empty(s) || s.L < phsa::kM) return PHSA_OK;  // no full block: nothing to write
+    if (!K || !punct_mask || !Krepr || !aligned16(K) || !aligned16(Krepr))
+        return PHSA_ERR_INVALID_ARG;
+    return from_cuda(phsa::launch_block_repr(K, punct_mask, s, lambda, Krepr,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
+int phsa_select_blocks(const void* Q, const void* Krepr, phsa_shape s, phsa_select_params p,
+                       int32_t* block_idx, int32_t* block_cnt, void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
+    if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
+    if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
+    if (empty(s)) return PHSA_OK;
+    const bool need_repr = s.L >= 2 * phsa::kM;  // some query block has a candidate
+    if (!Q || !block_idx || !block_cnt || !aligned16(Q) || (need_repr && (!Krepr || !aligned16(Krepr))))
+        return PHSA_ERR_INVALID_ARG;
+    if (phsa::select_smem_bytes(s, p.topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
+    return from_cuda(phsa::launch_select_blocks(Q, Krepr, s, p, block_idx, block_cnt, status_ptr(),
+                                                static_cast<cudaStream_t>(stream)));
+}
+
+int phsa_sparse_attn_fwd(const void* Q, const void* K, const void* V, const int32_t* block_idx,
+                         const int32_t* block_cnt, phsa_shape s, int topk, float sm_scale,
+                         void* O, float* lse, void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = check_topk(s, topk)) != PHSA_OK) return rc;
+    if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;
+    if (empty(s)) return PHSA_OK;
+    if (!Q || !K || !V || !block_idx || !block_cnt || !O || !lse) return PHSA_ERR_INVALID_ARG;
+    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
+        return PHSA_ERR_INVALID_ARG;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_attn_fwd(Q, K, V, block_idx, block_cnt, s, topk, sm_scale, O,
+                                           lse, st, static_cast<cudaStream_t>(stream)));
+}
+
+size_t phsa_sparse_attn_bwd_workspace(phsa_shape s, int topk) {
+    if (check_shape(s) != PHSA_OK || check_topk(s, topk) != PHSA_OK) return 0;
+    if (empty(s)) return 0;
+    return phsa::bwd_layout(s, topk).total;
+}
+
+int phsa_sparse_attn_bwd(const void* Q, const void* K, const void* V, const void* O,
+                         const void* dO, const float* lse, const int32_t* block_idx,
+                         const int32_t* block_cnt, phsa_shape s, int topk, float sm_scale,
+                         void* workspace, size_t workspace_bytes, void* dQ, void* dK, void* dV,
+                         void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = check_topk(s, topk)) != PHSA_OK) return rc;
+    if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;
+    if (empty(s)) return PHSA_OK;
+    if (!Q || !K || !V || !O || !dO || !lse || !block_idx || !block_cnt || !dQ || !dK || !dV)
+        return PHSA_ERR_INVALID_ARG;
+    const void* ptrs[] = {Q, K, V, O, dO, dQ, dK, dV};
+    for (const void* p : ptrs)
+        if (!aligned16(p)) return PHSA_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) ||
+        workspace_bytes < phsa::bwd_layout(s, topk).total)
+        return PHSA_ERR_WORKSPACE;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, s, topk,
+                                           sm_scale, workspace, dQ, dK, dV, st,
+                                           static_cast<cudaStream_t>(stream)));
+}
+
+int phsa_get_device_status(void* stream) {
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return PHSA_ERR_CUDA;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpy(&v, st, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return PHSA_ERR_CUDA;
+    const int zero = 0;
+    if (cudaMemcpy(st, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess)
+        return PHSA_ERR_CUDA;
+    return v;
+}
+
+const char* phsa_status_string(int code) {
+    switch (code) {
+        case PHSA_OK: return "PHSA_OK";
+        case PHSA_ERR_INVALID_ARG: return "PHSA_ERR_INVALID_ARG: invalid argument";
+        case PHSA_ERR_UNSUPPORTED: return "PHSA_ERR_UNSUPPORTED: unsupported shape or parameter";
+        case PHSA_ERR_CUDA: return "PHSA_ERR_CUDA: CUDA runtime error";
+        case PHSA_ERR_TIMEOUT: return "PHSA_ERR_TIMEOUT: a bounded device wait expired";
+        case PHSA_ERR_DEVICE_INDEX: return "PHSA_ERR_DEVICE_INDEX: invalid block index skipped";
+        case PHSA_ERR_WORKSPACE: return "PHSA_ERR_WORKSPACE: workspace missing or too small";
+        default: return "unknown phsa status";
+    }
+}
+
+const char* phsa_version(void) { return "0.1.0"; }
+
+}  // extern "C"

@@ -1,0 +1,53 @@
+// Kernel launchers behind the C ABI. Arguments are validated by the ABI layer
+// (phsa_api.cu) before any of these run.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "phsa.h"
+
+namespace phsa {
+
+// Kernel identities for the optional per-kernel timing (profile.cu).
+enum KernelId {
+    K_REPR = 0, K_SELECT, K_FWD, K_BWD_DELTA, K_BWD_MARK, K_BWD_BUILD, K_BWD_DKDV,
+    K_BWD_DKDV_SUM, K_BWD_DQ, K_COUNT
+};
+void prof_begin(int kid, cudaStream_t st);
+void prof_end(int kid, cudaStream_t st);
+
+// Brackets one kernel launch with the timing hooks.
+struct ProfScope {
+    int kid;
+    cudaStream_t st;
+    ProfScope(int k, cudaStream_t s) : kid(k), st(s) { prof_begin(kid, st); }
+    ~ProfScope() { prof_end(kid, st); }
+};
+
+cudaError_t launch_block_repr(const void* K, const uint8_t* mask, const phsa_shape& s,
+                              float lambda, void* Krepr, cudaStream_t st);
+
+cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_shape& s,
+                                 const phsa_select_params& p, int32_t* idx, int32_t* cnt,
+                                 int* status, cudaStream_t st);
+
+cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const int32_t* idx,
+                            const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                            void* O, float* lse, int* status, cudaStream_t st);
+
+// Backward workspace layout (all offsets 256-byte aligned).
+struct BwdLayout {
+    size_t bits, tinfo, qlist, work, nwork, delta, partial, total;
+    int nqb, words, chunk, work_max, slot_max;
+};
+BwdLayout bwd_layout(const phsa_shape& s, int topk);
+
+cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const void* O,
+                            const void* dO, const float* lse, const int32_t* idx,
+                            const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                            void* ws, void* dQ, void* dK, void* dV, int* status,
+                            cudaStream_t st);
+
+}  // namespace phsa

@@ -1,0 +1,248 @@
+"""Python binding of the PHSA C ABI (``include/phsa.h``).
+
+Argument marshalling only: each function checks tensor dtypes/devices,
+allocates outputs with PyTorch when the caller passes none, and calls the
+entry point of the same name in ``libphsa.so`` on the current CUDA stream.
+Every step of the computation runs in the library's CUDA kernels; there is no
+fallback of any kind. If the library cannot be loaded, calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+BLOCK_SIZE = 64
+HEAD_DIM = 128
+
+_lock = threading.Lock()
+_lib = None
+
+
+class PhsaError(RuntimeError):
+    """A PHSA entry point returned a non-zero status."""
+
+    def __init__(self, fn: str, code: int):
+        self.code = code
+        super().__init__(f"{fn} failed: {phsa_status_string(code)} ({code})")
+
+
+class phsa_shape(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("L", ctypes.c_int), ("Hq", ctypes.c_int),
+                ("Hkv", ctypes.c_int), ("D", ctypes.c_int), ("block_size", ctypes.c_int)]
+
+
+class phsa_select_params(ctypes.Structure):
+    _fields_ = [("topk", ctypes.c_int), ("n_init", ctypes.c_int), ("n_local", ctypes.c_int),
+                ("sm_scale", ctypes.c_float)]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load():
+    """Load ``libphsa.so`` (building it first if it is missing or stale)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.build()
+            lib = ctypes.CDLL(path)
+            _declare(lib)
+            _lib = lib
+    return _lib
+
+
+def _declare(L):
+    P, I, F, SZ = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+    L.phsa_build_block_repr.argtypes = [P, P, phsa_shape, F, P, P]
+    L.phsa_select_blocks.argtypes = [P, P, phsa_shape, phsa_select_params, P, P, P]
+    L.phsa_sparse_attn_fwd.argtypes = [P, P, P, P, P, phsa_shape, I, F, P, P, P]
+    L.phsa_sparse_attn_bwd_workspace.argtypes = [phsa_shape, I]
+    L.phsa_sparse_attn_bwd_workspace.restype = SZ
+    L.phsa_sparse_attn_bwd.argtypes = [P, P, P, P, P, P, P, P, phsa_shape, I, F, P, SZ, P, P, P, P]
+    L.phsa_get_device_status.argtypes = [P]
+    L.phsa_status_string.argtypes = [I]
+    L.phsa_status_string.restype = ctypes.c_char_p
+    L.phsa_version.restype = ctypes.c_char_p
+    L.phsa_profile_enable.argtypes = [I]
+    L.phsa_profile_enable.restype = I
+    L.phsa_profile_read.argtypes = [I, ctypes.POINTER(ctypes.c_char_p),
+                                    ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)]
+    L.phsa_profile_read.restype = I
+    for fn in ("phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
+               "phsa_sparse_attn_bwd", "phsa_get_device_status"):
+        getattr(L, fn).restype = I
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else None
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(t, name, dtype, ndim=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got {tuple(t.shape)}")
+
+
+def make_shape(B, L, Hq, Hkv, D=HEAD_DIM, block_size=BLOCK_SIZE) -> phsa_shape:
+    return phsa_shape(int(B), int(L), int(Hq), int(Hkv), int(D), int(block_size))
+
+
+def _raise(fn, rc):
+    if rc != 0:
+        raise PhsaError(fn, rc)
+
+
+def phsa_status_string(code: int) -> str:
+    return load().phsa_status_string(int(code)).decode()
+
+
+def phsa_version() -> str:
+    return load().phsa_version().decode()
+
+
+def phsa_build_block_repr(K, punct_mask, lam: float, Krepr=None, stream=None):
+    """Stage (a): representative keys [B, Hkv, L // 64, D] (bf16)."""
+    _check(K, "K", torch.bfloat16, 4)
+    _check(punct_mask, "punct_mask", torch.uint8, 2)
+    B, Hkv, L, D = K.shape
+    if tuple(punct_mask.shape) != (B, L):
+        raise ValueError("punct_mask must be [B, L]")
+    T = L // BLOCK_SIZE
+    if Krepr is None:
+        Krepr = torch.empty((B, Hkv, T, D), dtype=torch.bfloat16, device=K.device)
+    _check(Krepr, "Krepr", torch.bfloat16, 4)
+    rc = load().phsa_build_block_repr(_ptr(K), _ptr(punct_mask), make_shape(B, L, Hkv, Hkv, D),
+                                      float(lam), _ptr(Krepr), _stream(stream))
+    _raise("phsa_build_block_repr", rc)
+    return Krepr
+
+
+def phsa_select_blocks(Q, Krepr, Hkv: int, topk: int, n_init: int = 1, n_local: int = 1,
+                       sm_scale: float | None = None, block_idx=None, block_cnt=None,
+                       stream=None):
+    """Stage (b): (block_idx [B, Hkv, NQB, topk] int32, block_cnt [B, Hkv, NQB] int32)."""
+    _check(Q, "Q", torch.bfloat16, 4)
+    _check(Krepr, "Krepr", torch.bfloat16, 4)
+    B, Hq, L, D = Q.shape
+    NQB = -(-L // BLOCK_SIZE)
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    if block_idx is None:
+        block_idx = torch.empty((B, Hkv, NQB, topk), dtype=torch.int32, device=Q.device)
+    if block_cnt is None:
+        block_cnt = torch.empty((B, Hkv, NQB), dtype=torch.int32, device=Q.device)
+    _check(block_idx, "block_idx", torch.int32, 4)
+    _check(block_cnt, "block_cnt", torch.int32, 3)
+    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    rc = load().phsa_select_blocks(_ptr(Q), _ptr(Krepr), make_shape(B, L, Hq, Hkv, D), p,
+                                   _ptr(block_idx), _ptr(block_cnt), _stream(stream))
+    _raise("phsa_select_blocks", rc)
+    return block_idx, block_cnt
+
+
+def phsa_sparse_attn_fwd(Q, K, V, block_idx, block_cnt, sm_scale: float | None = None, O=None,
+                         lse=None, stream=None):
+    """Stage (c) forward: (O [B, Hq, L, D] bf16, lse [B, Hq, L] fp32)."""
+    _check(Q, "Q", torch.bfloat16, 4)
+    _check(K, "K", torch.bfloat16, 4)
+    _check(V, "V", torch.bfloat16, 4)
+    _check(block_idx, "block_idx", torch.int32, 4)
+    _check(block_cnt, "block_cnt", torch.int32, 3)
+    B, Hq, L, D = Q.shape
+    Hkv = K.shape[1]
+    topk = block_idx.shape[-1]
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    if O is None:
+        O = torch.empty_like(Q)
+    if lse is None:
+        lse = torch.empty((B, Hq, L), dtype=torch.float32, device=Q.device)
+    _check(O, "O", torch.bfloat16, 4)
+    _check(lse, "lse", torch.float32, 3)
+    rc = load().phsa_sparse_attn_fwd(_ptr(Q), _ptr(K), _ptr(V), _ptr(block_idx), _ptr(block_cnt),
+                                     make_shape(B, L, Hq, Hkv, D), int(topk), float(sm_scale),
+                                     _ptr(O), _ptr(lse), _stream(stream))
+    _raise("phsa_sparse_attn_fwd", rc)
+    return O, lse
+
+
+def phsa_sparse_attn_bwd_workspace(B, L, Hq, Hkv, topk, D=HEAD_DIM) -> int:
+    return int(load().phsa_sparse_attn_bwd_workspace(make_shape(B, L, Hq, Hkv, D), int(topk)))
+
+
+def phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_scale=None,
+                         workspace=None, dQ=None, dK=None, dV=None, stream=None):
+    """Stage (c) backward: (dQ, dK, dV) in bf16."""
+    for name, t in (("Q", Q), ("K", K), ("V", V), ("O", O), ("dO", dO)):
+        _check(t, name, torch.bfloat16, 4)
+    _check(lse, "lse", torch.float32, 3)
+    _check(block_idx, "block_idx", torch.int32, 4)
+    _check(block_cnt, "block_cnt", torch.int32, 3)
+    B, Hq, L, D = Q.shape
+    Hkv = K.shape[1]
+    topk = block_idx.shape[-1]
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    ws_bytes = phsa_sparse_attn_bwd_workspace(B, L, Hq, Hkv, topk, D)
+    if workspace is None:
+        workspace = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=Q.device)
+    _check(workspace, "workspace", torch.uint8, 1)
+    dQ = torch.empty_like(Q) if dQ is None else dQ
+    dK = torch.empty_like(K) if dK is None else dK
+    dV = torch.empty_like(V) if dV is None else dV
+    rc = load().phsa_sparse_attn_bwd(
+        _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(dO), _ptr(lse), _ptr(block_idx), _ptr(block_cnt),
+        make_shape(B, L, Hq, Hkv, D), int(topk), float(sm_scale), _ptr(workspace),
+        ctypes.c_size_t(workspace.numel()), _ptr(dQ), _ptr(dK), _ptr(dV), _stream(stream))
+    _raise("phsa_sparse_attn_bwd", rc)
+    return dQ, dK, dV
+
+
+def phsa_get_device_status(stream=None) -> int:
+    """Synchronise the stream; return and clear the device status word."""
+    return int(load().phsa_get_device_status(_stream(stream)))
+
+
+def phsa_profile_enable(on: bool) -> bool:
+    """Turn per-kernel event timing on or off; returns the previous setting."""
+    return bool(load().phsa_profile_enable(1 if on else 0))
+
+
+def phsa_profile_read() -> dict:
+    """{kernel name: (total ms, launches)} since the last read; clears the records."""
+    n = 32
+    names = (ctypes.c_char_p * n)()
+    ms = (ctypes.c_double * n)()
+    cnt = (ctypes.c_int * n)()
+    k = load().phsa_profile_read(n, names, ms, cnt)
+    if k < 0:
+        raise PhsaError("phsa_profile_read", k)
+    return {names[i].decode(): (float(ms[i]), int(cnt[i])) for i in range(k)}
+
+
+def phsa_forward(Q, K, V, punct_mask, lam: float, topk: int, n_init: int = 1, n_local: int = 1,
+                 sm_scale: float | None = None, stream=None):
+    """The whole forward hot path: (a) -> (b) -> (c). Returns (O, lse, block_idx, block_cnt, Krepr)."""
+    Krepr = phsa_build_block_repr(K, punct_mask, lam, stream=stream)
+    idx, cnt = phsa_select_blocks(Q, Krepr, K.shape[1], topk, n_init, n_local, sm_scale,
+                                  stream=stream)
+    O, lse = phsa_sparse_attn_fwd(Q, K, V, idx, cnt, sm_scale, stream=stream)
+    return O, lse, idx, cnt, Krepr

@@ -1,0 +1,75 @@
+"""The C-ABI library builds, loads and exports every entry point its header declares.
+
+CPU only: nothing here launches a kernel.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2601_02819_gb300 import build as libbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(phsa_[a-z0-9_]+)\s*\(", src))
+    return sorted(names)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return ctypes.CDLL(libbuild.build())
+
+
+def test_header_declares_the_hot_path():
+    names = declared_functions()
+    for n in ("phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
+              "phsa_sparse_attn_bwd", "phsa_sparse_attn_bwd_workspace", "phsa_get_device_status"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for n in declared_functions():
+        assert hasattr(lib, n), n
+
+
+def test_status_strings_and_version(lib):
+    lib.phsa_status_string.restype = ctypes.c_char_p
+    lib.phsa_version.restype = ctypes.c_char_p
+    assert lib.phsa_status_string(0) == b"PHSA_OK"
+    assert b"UNSUPPORTED" in lib.phsa_status_string(-2)
+    assert lib.phsa_version().count(b".") == 2
+
+
+def test_host_validation_needs_no_gpu(lib):
+    # Shape and parameter checks run before any CUDA call, so they answer on a CPU machine.
+    from paper_2601_02819_gb300.phsa import phsa_shape, phsa_select_params
+    lib.phsa_build_block_repr.argtypes = [ctypes.c_void_p, ctypes.c_void_p, phsa_shape,
+                                          ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p]
+    lib.phsa_select_blocks.argtypes = [ctypes.c_void_p, ctypes.c_void_p, phsa_shape,
+                                       phsa_select_params, ctypes.c_void_p, ctypes.c_void_p,
+                                       ctypes.c_void_p]
+    lib.phsa_sparse_attn_bwd_workspace.argtypes = [phsa_shape, ctypes.c_int]
+    lib.phsa_sparse_attn_bwd_workspace.restype = ctypes.c_size_t
+    ok = phsa_shape(1, 4096, 16, 8, 128, 64)
+    assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 16, 8, 64, 64), 0.5, None,
+                                     None) == -2  # D = 64 unsupported
+    assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 16, 8, 128, 16), 0.5, None,
+                                     None) == -2  # block size 16 unsupported
+    assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 12, 8, 128, 64), 0.5, None,
+                                     None) == -1  # Hq not a multiple of Hkv
+    assert lib.phsa_build_block_repr(None, None, ok, 1.5, None, None) == -1  # lambda > 1
+    assert lib.phsa_build_block_repr(None, None, ok, 0.5, None, None) == -1  # null pointers
+    p = phsa_select_params(2, 1, 2, 0.088)  # topk < n_init + n_local
+    assert lib.phsa_select_blocks(None, None, ok, p, None, None, None) == -1
+    p = phsa_select_params(8, 1, 0, 0.088)  # n_local must be >= 1
+    assert lib.phsa_select_blocks(None, None, ok, p, None, None, None) == -1
+    assert lib.phsa_sparse_attn_bwd_workspace(ok, 14) > 0
+    assert lib.phsa_sparse_attn_bwd_workspace(phsa_shape(1, 4096, 16, 8, 96, 64), 14) == 0

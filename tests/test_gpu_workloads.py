@@ -1,0 +1,82 @@
+"""End-to-end parity on the named workloads at full size (sampled where the
+oracle would be too slow), run in the launch configuration bench.py times."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2601_02819_gb300 import inputs
+from paper_2601_02819_gb300 import phsa
+from parity import LSE_ABS, assert_close, bf16_to_f64, compare_selection, to_dev_bf16
+
+pytestmark = pytest.mark.gpu
+
+SCALE = 128 ** -0.5
+
+
+def gpu_forward(w, x):
+    Qd, Kd, Vd = (to_dev_bf16(x[k]) for k in ("Q", "K", "V"))
+    md = torch.from_numpy(x["mask"]).cuda()
+    O, lse, idx, cnt, Kr = phsa.phsa_forward(Qd, Kd, Vd, md, w.lam, w.topk, w.n_init, w.n_local)
+    torch.cuda.synchronize()
+    return Qd, Kd, Vd, O, lse, idx, cnt
+
+
+def test_tiny_workload_end_to_end():
+    w = inputs.WORKLOADS["tiny_2k"]
+    x = inputs.make_inputs(w)
+    _, _, _, O, lse, idx, cnt = gpu_forward(w, x)
+    Kr, oi, oc, Or, lser = oracle.forward(x["Q"], x["K"], x["V"], x["mask"], 64, w.lam, w.topk,
+                                          w.n_init, w.n_local, SCALE)
+    _, _, oa = oracle.select_blocks(x["Q"], Kr, w.L, 64, w.topk, w.n_init, w.n_local, SCALE,
+                                    want_agg=True)
+    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
+    bad, excl, _, msgs = compare_selection(gi, gc, oi, oc, oa)
+    assert bad == 0, msgs[:5]
+    same = np.all(gi == oi, axis=-1)[0, 0]  # query blocks whose selection matches exactly
+    rows = np.repeat(same, 64)[:w.L]
+    assert_close("O", bf16_to_f64(O)[:, :, rows], Or[:, :, rows])
+    assert np.abs(lse.cpu().numpy()[:, :, rows] - lser[:, :, rows]).max() <= LSE_ABS
+
+
+@pytest.mark.parametrize("name", ["prefill_32k", "train_8k_x4", "long_131k_p3"])
+def test_full_size_forward_sampled_rows(name):
+    w = inputs.WORKLOADS[name]
+    x = inputs.make_inputs(w)
+    _, _, _, O, lse, idx, cnt = gpu_forward(w, x)
+    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
+    rng = np.random.default_rng(1)
+    n = 256
+    rows = np.stack([rng.integers(0, w.B, n), rng.integers(0, w.Hq, n),
+                     rng.integers(0, w.L, n)], axis=1).astype(np.int32)
+    rows[:4] = [[0, 0, 0], [w.B - 1, w.Hq - 1, w.L - 1], [0, 1, 63], [0, 0, 64]]
+    # Attention parity on the GPU's own selection (valid by the selection test).
+    Or, lser = oracle.sparse_attn_rows(x["Q"], x["K"], x["V"], gi, gc, 64, SCALE, rows)
+    Og = bf16_to_f64(O)[rows[:, 0], rows[:, 1], rows[:, 2]]
+    assert_close("O rows", Og, Or)
+    lg = lse.cpu().numpy()[rows[:, 0], rows[:, 1], rows[:, 2]]
+    assert np.abs(lg - lser).max() <= LSE_ABS
+    assert np.all(gc == np.minimum(w.topk, np.arange(w.NQB) + 1)[None, None, :])
+
+
+def test_train_workload_backward_sampled():
+    w = inputs.WORKLOADS["train_8k_x4"]
+    x = inputs.make_inputs(w, with_grad=True)
+    Qd, Kd, Vd, O, lse, idx, cnt = gpu_forward(w, x)
+    dOd = to_dev_bf16(x["dO"])
+    dQ, dK, dV = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, idx, cnt)
+    torch.cuda.synchronize()
+    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
+    rng = np.random.default_rng(2)
+    rows = np.stack([rng.integers(0, w.B, 64), rng.integers(0, w.Hq, 64),
+                     rng.integers(0, w.L, 64)], axis=1).astype(np.int32)
+    rq = oracle.sparse_attn_bwd_dq_rows(x["Q"], x["K"], x["V"], x["dO"], gi, gc, 64, SCALE, rows)
+    assert_close("dQ rows", bf16_to_f64(dQ)[rows[:, 0], rows[:, 1], rows[:, 2]], rq)
+    blocks = np.array([[0, 0, 0], [1, 3, 1], [2, 5, 7], [3, 7, w.NQB - 1], [0, 2, 64],
+                       [1, 1, 100]], np.int32)
+    rk, rv = oracle.sparse_attn_bwd_kv_blocks(x["Q"], x["K"], x["V"], x["dO"], gi, gc, 64, SCALE,
+                                              blocks)
+    dKh, dVh = bf16_to_f64(dK), bf16_to_f64(dV)
+    for n, (b, g, t) in enumerate(blocks):
+        assert_close(f"dK block {t}", dKh[b, g, t * 64:(t + 1) * 64], rk[n])
+        assert_close(f"dV block {t}", dVh[b, g, t * 64:(t + 1) * 64], rv[n])

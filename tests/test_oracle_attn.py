@@ -170,3 +170,30 @@ def test_backward_invariants():
     go = oracle.bf16_to_f64(dO).reshape(2, 2, 2, L, D).sum(axis=(2, 3))
     np.testing.assert_allclose(dV.sum(axis=2), go, rtol=0, atol=1e-9)
     np.testing.assert_allclose(dK.sum(axis=2), 0.0, rtol=0, atol=1e-9)
+
+
+def test_sampled_oracle_entry_points_agree_with_full_ones():
+    # The sampled forms used at full size must give exactly the full computation's values.
+    rng = np.random.default_rng(17)
+    L, m = 64 * 7 + 11, 64
+    Q, K, V = rand_qkv(rng, 2, 4, 2, L)
+    dO = bf(rng.standard_normal(Q.shape))
+    Kr = oracle.block_repr(K, (rng.random((2, L)) < 0.1).astype(np.uint8), m, 0.5)
+    idx, cnt, agg = oracle.select_blocks(Q, Kr, L, m, 4, 1, 1, D ** -0.5, want_agg=True)
+    units = np.array([0, 5, 7, 8 + 6, 3 * 8 + 7])
+    i2, c2, a2 = oracle.select_units(Q, Kr, L, m, 4, 1, 1, D ** -0.5, units)
+    fi = idx.reshape(-1, 4)[units]
+    assert np.array_equal(i2, fi) and np.array_equal(c2, cnt.reshape(-1)[units])
+    np.testing.assert_array_equal(a2, agg.reshape(-1, agg.shape[-1])[units])
+    dQ, dK, dV = oracle.sparse_attn_bwd(Q, K, V, dO, idx, cnt, m, D ** -0.5)
+    rows = np.array([[0, 0, 3], [1, 3, L - 1], [1, 2, 200]], np.int32)
+    dq = oracle.sparse_attn_bwd_dq_rows(Q, K, V, dO, idx, cnt, m, D ** -0.5, rows)
+    for n, (b, h, i) in enumerate(rows):
+        np.testing.assert_allclose(dq[n], dQ[b, h, i], rtol=0, atol=1e-12)
+    blocks = np.array([[0, 0, 0], [1, 1, 3], [1, 0, 7]], np.int32)
+    dk, dv = oracle.sparse_attn_bwd_kv_blocks(Q, K, V, dO, idx, cnt, m, D ** -0.5, blocks)
+    for n, (b, g, t) in enumerate(blocks):
+        hi = min(L, (t + 1) * m) - t * m
+        np.testing.assert_allclose(dk[n, :hi], dK[b, g, t * m:t * m + hi], rtol=0, atol=1e-12)
+        np.testing.assert_allclose(dv[n, :hi], dV[b, g, t * m:t * m + hi], rtol=0, atol=1e-12)
+        assert np.all(dk[n, hi:] == 0) and np.all(dv[n, hi:] == 0)
