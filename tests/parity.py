@@ -60,14 +60,17 @@ def compare_selection(g_idx, g_cnt, o_idx, o_cnt, o_agg, band=SELECT_BAND):
     """Compare GPU and oracle selections unit by unit.
 
     ``*_idx`` [U, topk], ``*_cnt`` [U], ``o_agg`` [U, T] (NaN where not scored).
-    Returns (n_bad_units, n_excluded_candidates, n_units_with_exclusions, messages).
+    Returns (n_bad_units, n_excluded_candidates, n_units_differing, messages):
+    bad units differ outside the ambiguity band; excluded candidates are those
+    inside the band (reported, never compared); differing units are units whose
+    GPU and oracle sets differ only inside the band.
     """
     g_idx = np.asarray(g_idx).reshape(len(g_cnt.reshape(-1)), -1)
     o_idx = np.asarray(o_idx).reshape(g_idx.shape)
     g_cnt = np.asarray(g_cnt).reshape(-1)
     o_cnt = np.asarray(o_cnt).reshape(-1)
     o_agg = np.asarray(o_agg).reshape(len(o_cnt), -1)
-    bad, excluded, units_ex, msgs = 0, 0, 0, []
+    bad, excluded, differ, msgs = 0, 0, 0, []
     for u in range(len(o_cnt)):
         if g_cnt[u] != o_cnt[u]:
             bad += 1
@@ -89,12 +92,12 @@ def compare_selection(g_idx, g_cnt, o_idx, o_cnt, o_agg, band=SELECT_BAND):
         hi = A[sel].min() if sel else np.inf
         lo = A[uns].max() if uns else -np.inf
         amb = {t for t in sel if A[t] - lo <= band} | {t for t in uns if hi - A[t] <= band}
-        if amb:
-            excluded += len(amb)
-            units_ex += 1
+        excluded += len(amb)
         diff = gs ^ os_
+        if diff:
+            differ += 1
         if not diff <= amb:
             bad += 1
             msgs.append(f"unit {u}: gpu {sorted(gs)} vs oracle {sorted(os_)}; "
                         f"boundary gap {hi - lo:.3e}")
-    return bad, excluded, units_ex, msgs
+    return bad, excluded, differ, msgs

@@ -23,15 +23,16 @@ def gpu_select(Q, Kr, Hkv, topk, n_init, n_local, scale):
     return idx.cpu().numpy(), cnt.cpu().numpy()
 
 
-def check(Q, Kr, L, Hkv, topk, n_init=1, n_local=1, max_excl_frac=0.01):
+def check(Q, Kr, L, Hkv, topk, n_init=1, n_local=1):
     scale = 128 ** -0.5
     gi, gc = gpu_select(Q, Kr, Hkv, topk, n_init, n_local, scale)
     oi, oc, oa = oracle.select_blocks(Q, Kr, L, 64, topk, n_init, n_local, scale, want_agg=True)
-    bad, excl, units_ex, msgs = compare_selection(gi, gc, oi, oc, oa)
+    bad, excl, differ, msgs = compare_selection(gi, gc, oi, oc, oa)
     assert bad == 0, msgs[:5]
-    n_sel = int(oc.sum())
-    assert excl <= max(2, max_excl_frac * n_sel), (excl, n_sel)
-    return excl, n_sel
+    # sets may differ only inside the 1e-3 band, and only rarely
+    assert differ <= max(2, 0.01 * oc.size), (differ, oc.size)
+    print(f"selection: {oc.size} units, {differ} differ inside the band, "
+          f"{excl} candidates in the band (not compared)")
 
 
 def test_tiny_workload():
@@ -90,7 +91,7 @@ def test_full_size_sampled_units(name):
                                       [0, U - 1, w.NQB - 1, w.NQB // 2]]))
     oi, oc, oa = oracle.select_units(x["Q"], Kr, w.L, 64, w.topk, w.n_init, w.n_local, scale,
                                      units)
-    bad, excl, _, msgs = compare_selection(gi.reshape(U, -1)[units], gc.reshape(-1)[units],
-                                           oi, oc, oa)
+    bad, excl, differ, msgs = compare_selection(gi.reshape(U, -1)[units],
+                                                gc.reshape(-1)[units], oi, oc, oa)
     assert bad == 0, msgs[:5]
-    assert excl <= max(2, 0.01 * oc.sum())
+    assert differ <= max(2, 0.02 * len(units)), (differ, len(units))
