@@ -170,6 +170,19 @@ const char* phsa_status_string(int code);
 int phsa_profile_enable(int on);
 int phsa_profile_read(int max_kinds, const char** names, double* total_ms, int* launches);
 
+/*
+ * Diagnostic (no counterpart in the paper): runs the two tensor-core MMA
+ * shapes of the forward kernel once on one CTA, S = A B^T and O = bf16(S) V,
+ * with operands staged by TMA and accumulators in tensor memory, so that a
+ * test can check the hardware path against a plain matrix product.
+ *   A bf16 [128][128], B bf16 [64][128], V bf16 [64][128]  (device, in)
+ *   S fp32 [128][64], O fp32 [128][128]                    (device, out)
+ * Asynchronous on `stream`; a wait that times out is reported through
+ * phsa_get_device_status as PHSA_ERR_TIMEOUT.
+ */
+int phsa_selftest_tcgen05(const void* A, const void* B, const void* V, float* S, float* O,
+                          void* stream);
+
 /* Library version as "major.minor.patch". */
 const char* phsa_version(void);
 

@@ -231,9 +231,11 @@ cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const i
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                             void* O, float* lse, int* status, cudaStream_t st) {
     if ((long long)s.B * s.Hkv * s.L == 0) return cudaSuccess;
-    return (s.Hq / s.Hkv == 2)
-               ? launch_fwd_g<2>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st)
-               : launch_fwd_g<1>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st);
+    // Two query heads per KV head fill a 128-row tcgen05 tile; a single head
+    // (64 rows) runs on the warp-level MMA kernel in this file.
+    if (s.Hq / s.Hkv == 2)
+        return launch_attn_fwd_tc(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st);
+    return launch_fwd_g<1>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st);
 }
 
 }  // namespace phsa

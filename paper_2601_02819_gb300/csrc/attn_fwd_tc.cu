@@ -1,0 +1,453 @@
+// Stage (c) forward on the 5th-generation tensor cores (tcgen05 + TMEM + TMA),
+// for GQA groups of two query heads (G*64 = 128 query rows per tile).
+//
+// One CTA per (query block qb, KV head g), 192 threads in three roles:
+//   warp 4 (one lane)  TMA producer: the 128 x 128 Q tile once, then for every
+//                      selected block its 64 x 128 K and V tiles into a
+//                      two-stage shared-memory ring (gathered by block index).
+//   warp 5 (one lane)  MMA issuer: S_j = Q K_j^T (M=128, N=64, K=128) into one
+//                      of two TMEM score buffers, and O += P_j V_j (M=128,
+//                      N=128, K=64) with P_j read from TMEM. QK of block j+1 is
+//                      issued before PV of block j, so the tensor core works
+//                      while the softmax of block j runs.
+//   warps 0-3          softmax: thread r owns query row r (TMEM lane r). It
+//                      loads its 64 scores, applies the causal mask inside the
+//                      query's own block, keeps a running max and sum in the
+//                      log2 domain, and writes P (bf16) over its scores in
+//                      TMEM. O is rescaled in TMEM only when the block max
+//                      exceeds the running max by more than 2^8 (exact: the
+//                      final normalisation uses the same running max).
+//                      Epilogue: O / l -> bf16 -> shared memory -> TMA store;
+//                      LSE = (max + log2 l) ln 2.
+// TMEM: O in columns [0,128), score buffers in [128,192) and [192,256).
+// Every wait is bounded in time (tc_common.cuh); on expiry the kernel records
+// PHSA_ERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
+#include "phsa_common.cuh"
+#include "phsa_internal.h"
+#include "tc_common.cuh"
+
+namespace phsa {
+
+namespace {
+
+using namespace tc;
+
+constexpr int kStages = 2;
+constexpr int kHalfQ = 128 * 64 * 2;        // one 64-column half of the Q tile (16 KB)
+constexpr int kQBytes = 2 * kHalfQ;         // 32 KB
+constexpr int kKVHalf = 64 * 64 * 2;        // one 64-column half of a K or V block (8 KB)
+constexpr int kKBytes = 2 * kKVHalf;        // 16 KB
+constexpr int kStageBytes = 2 * kKBytes;    // K and V of one block
+constexpr int kOffQ = 0;
+constexpr int kOffKV = kQBytes;
+constexpr int kOffBar = kOffKV + kStages * kStageBytes;
+// barriers
+constexpr int B_Q = 0;
+constexpr int B_KVFULL = 1;                 // + stage
+constexpr int B_KVEMPTY = B_KVFULL + kStages;
+constexpr int B_SFULL = B_KVEMPTY + kStages;  // + buffer
+constexpr int B_PFULL = B_SFULL + 2;
+constexpr int B_PVDONE = B_PFULL + 2;
+constexpr int B_OFINAL = B_PVDONE + 1;
+constexpr int B_DRAIN = B_OFINAL + 1;
+constexpr int kNumBars = B_DRAIN + 1;
+constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag, block count
+constexpr int kOffList = kOffMisc + 16;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kColO = 0;
+constexpr float kRescaleLog2 = 8.0f;
+
+__host__ __device__ constexpr size_t fwd_tc_smem(int topk) {
+    return 1024 + (size_t)kOffList + (size_t)(topk + 1) * 4;
+}
+
+struct FwdTcArgs {
+    const int32_t* idx;
+    const int32_t* cnt;
+    float* lse;
+    int* status;
+    int Hq, Hkv, L, NQB, topk;
+    float scale_log2;
+};
+
+__device__ __forceinline__ uint32_t col_s(int buf) { return 128u + 64u * (uint32_t)buf; }
+
+__global__ void __launch_bounds__(kThreads, 2)
+attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                   const FwdTcArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    const uint32_t sb = smem_u32(smem);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int unit = blockIdx.x;
+    const int qb = a.NQB - 1 - (unit % a.NQB);
+    const int bg = unit / a.NQB;
+    const int b = bg / a.Hkv, g = bg % a.Hkv;
+    const long long lu = (long long)bg * a.NQB + qb;
+    auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
+    int* list = reinterpret_cast<int*>(smem + kOffList);
+
+    if (threadIdx.x == 0) {
+        mbar_init(bar(B_Q), 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(bar(B_KVFULL + s), 1);
+            mbar_init(bar(B_KVEMPTY + s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(B_SFULL + i), 1);
+            mbar_init(bar(B_PFULL + i), 128);
+        }
+        mbar_init(bar(B_PVDONE), 1);
+        mbar_init(bar(B_OFINAL), 1);
+        mbar_init(bar(B_DRAIN), 1);
+        fence_barrier_init();
+        *abort_flag = 0;
+        reinterpret_cast<int*>(smem + kOffMisc)[2] =
+            compact_block_list(a.idx + lu * a.topk, a.cnt[lu], a.topk, qb, list, a.status);
+    }
+    if (warp == 5) {
+        tmem_alloc(sb + kOffMisc, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
+    const int n = reinterpret_cast<volatile int*>(smem + kOffMisc)[2];
+    const int hq0 = b * a.Hq + g * 2;  // first query head (plane) of the group
+
+    if (warp == 4) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0 && n > 0) {
+            prefetch_tmap(&tmQ);
+            prefetch_tmap(&tmK);
+            prefetch_tmap(&tmV);
+            mbar_expect_tx(bar(B_Q), kQBytes);
+            for (int hl = 0; hl < 2; ++hl)
+                for (int dh = 0; dh < 2; ++dh)
+                    tma_load_3d(sb + kOffQ + dh * kHalfQ + hl * (kHalfQ / 2), &tmQ, bar(B_Q),
+                                dh * 64, qb * 64, hq0 + hl);
+            int issued = 0;
+            for (int j = 0; j < n; ++j) {
+                const int s = j % kStages;
+                if (j >= kStages &&
+                    !mbar_wait(bar(B_KVEMPTY + s), ((j / kStages) - 1) & 1, abort_flag, a.status))
+                    break;
+                const uint32_t kb = sb + kOffKV + s * kStageBytes;
+                const int t = list[j];
+                mbar_expect_tx(bar(B_KVFULL + s), kStageBytes);
+                for (int dh = 0; dh < 2; ++dh) {
+                    tma_load_3d(kb + dh * kKVHalf, &tmK, bar(B_KVFULL + s), dh * 64, t * 64, bg);
+                    tma_load_3d(kb + kKBytes + dh * kKVHalf, &tmV, bar(B_KVFULL + s), dh * 64,
+                                t * 64, bg);
+                }
+                issued = j + 1;
+            }
+            // Own copies must have landed before the CTA may exit.
+            mbar_wait_drain(bar(B_Q), 0);
+            for (int j = issued - kStages; j < issued; ++j)
+                if (j >= 0) mbar_wait_drain(bar(B_KVFULL + j % kStages), (j / kStages) & 1);
+        }
+    } else if (warp == 5) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0 && n > 0) {
+            constexpr uint32_t idesc_qk = idesc_bf16(128, 64, false);
+            constexpr uint32_t idesc_pv = idesc_bf16(128, 128, true);
+            bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
+            tc_fence_after();
+            for (int j = 0; ok && j <= n; ++j) {
+                if (j < n) {
+                    const int s = j % kStages;
+                    if (!mbar_wait(bar(B_KVFULL + s), (j / kStages) & 1, abort_flag, a.status)) break;
+                    tc_fence_after();
+                    const uint32_t kb = sb + kOffKV + s * kStageBytes;
+                    const uint32_t d = tmem + col_s(j & 1);
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t off = (uint32_t)((ks & 3) * 32);
+                        const uint64_t ad = sdesc_sw128(sb + kOffQ + (ks >> 2) * kHalfQ + off, 16, 1024);
+                        const uint64_t bd = sdesc_sw128(kb + (ks >> 2) * kKVHalf + off, 16, 1024);
+                        mma_ss(d, ad, bd, idesc_qk, ks > 0 ? 1u : 0u);
+                    }
+                    mma_commit(bar(B_SFULL + (j & 1)));
+                }
+                if (j >= 1) {
+                    const int jj = j - 1, s = jj % kStages;
+                    if (!mbar_wait(bar(B_PFULL + (jj & 1)), (jj >> 1) & 1, abort_flag, a.status)) break;
+                    tc_fence_after();
+                    const uint32_t vb = sb + kOffKV + s * kStageBytes + kKBytes;
+                    const uint32_t pt = tmem + col_s(jj & 1);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks) {
+                        const uint64_t bd = sdesc_sw128(vb + ks * 2048, kKVHalf, 1024);
+                        mma_ts(tmem + kColO, pt + ks * 8, bd, idesc_pv, (jj > 0 || ks > 0) ? 1u : 0u);
+                    }
+                    mma_commit(bar(B_KVEMPTY + s));
+                    mma_commit(bar(B_PVDONE));
+                    if (jj == n - 1) mma_commit(bar(B_OFINAL));
+                }
+            }
+            // Every MMA issued above must be complete before TMEM is freed.
+            mma_commit(bar(B_DRAIN));
+            mbar_wait_drain(bar(B_DRAIN), 0);
+        }
+    } else {
+        // ------------------------------------------------ softmax + epilogue
+        const int row = threadIdx.x;  // TMEM lane
+        const int tok = row & 63, hl = row >> 6;
+        const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+        float m_used = -INFINITY, l = 0.f;
+        bool ok = true;
+        for (int j = 0; j < n; ++j) {
+            const int buf = j & 1;
+            ok = mbar_wait(bar(B_SFULL + buf), (j >> 1) & 1, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            tc_fence_after();
+            uint32_t sr[64];
+            tmem_ld32(lane_base + col_s(buf), sr);
+            tmem_ld32(lane_base + col_s(buf) + 32, sr + 32);
+            const bool diag = list[j] == qb;
+            float mx = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+                float v = __uint_as_float(sr[c]) * a.scale_log2;
+                if (diag && c > tok) v = -INFINITY;
+                sr[c] = __float_as_uint(v);
+                mx = fmaxf(mx, v);
+            }
+            if (j == 0) {
+                m_used = mx;
+            } else {
+                const bool need = mx > m_used + kRescaleLog2;
+                if (__any_sync(0xffffffffu, need)) {
+                    // PV of the previous block must be complete before O is touched.
+                    ok = mbar_wait(bar(B_PVDONE), (j - 1) & 1, abort_flag, a.status);
+                    ok = __all_sync(0xffffffffu, ok);
+                    if (!ok) break;
+                    tc_fence_after();
+                    const float f = need ? exp2f(m_used - mx) : 1.0f;
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        uint32_t o[32];
+                        tmem_ld32(lane_base + kColO + 32 * c4, o);
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
+                        tmem_st32(lane_base + kColO + 32 * c4, o);
+                    }
+                    if (need) {
+                        l *= f;
+                        m_used = mx;
+                    }
+                }
+            }
+            uint32_t pk[32];
+            float rs = 0.f;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                const float p0 = exp2f(__uint_as_float(sr[2 * c]) - m_used);
+                const float p1 = exp2f(__uint_as_float(sr[2 * c + 1]) - m_used);
+                rs += p0 + p1;
+                pk[c] = pack2_bf16(p0, p1);
+            }
+            l += rs;
+            tmem_st32(lane_base + col_s(buf), pk);
+            tc_fence_before();
+            mbar_arrive(bar(B_PFULL + buf));
+        }
+        // Epilogue: the whole O accumulation must be complete.
+        if (ok && n > 0) {
+            ok = mbar_wait(bar(B_OFINAL), 0, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+        }
+        if (ok) {
+            tc_fence_after();
+            const float inv = l > 0.f ? 1.0f / l : 0.f;
+            uint8_t* sq = smem + kOffQ;
+#pragma unroll
+            for (int c4 = 0; c4 < 4; ++c4) {
+                uint32_t o[32];
+                if (n > 0) {
+                    tmem_ld32(lane_base + kColO + 32 * c4, o);
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) o[c] = 0u;
+                }
+                const int dh = c4 >> 1;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int chunk = (c4 & 1) * 4 + q;
+                    uint4 v;
+                    v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
+                    v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
+                    v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
+                    v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
+                    *reinterpret_cast<uint4*>(sq + dh * kHalfQ + row * 128 + ((chunk ^ (row & 7)) << 4)) = v;
+                }
+            }
+            fence_proxy_async_smem();
+            const int i = qb * 64 + tok;
+            if (i < a.L)
+                a.lse[(size_t)(hq0 + hl) * a.L + i] = l > 0.f ? (m_used + log2f(l)) * kLn2 : -INFINITY;
+        }
+        named_barrier(1, 128);
+        if (threadIdx.x == 0 && ok) {
+            for (int h2 = 0; h2 < 2; ++h2)
+                for (int dh = 0; dh < 2; ++dh)
+                    tma_store_3d(&tmO, sb + kOffQ + dh * kHalfQ + h2 * (kHalfQ / 2), dh * 64,
+                                 qb * 64, hq0 + h2);
+            tma_store_commit();
+            tma_store_wait_read();
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 5) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_attn_fwd_tc(const void* Q, const void* K, const void* V, const int32_t* idx,
+                               const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                               void* O, float* lse, int* status, cudaStream_t st) {
+    const int NQB = (s.L + 63) / 64;
+    CUtensorMap tq, tk, tv, to;
+    if (!make_tmap_bf16_rows128(&tq, Q, s.L, (uint64_t)s.B * s.Hq, 64) ||
+        !make_tmap_bf16_rows128(&tk, K, s.L, (uint64_t)s.B * s.Hkv, 64) ||
+        !make_tmap_bf16_rows128(&tv, V, s.L, (uint64_t)s.B * s.Hkv, 64) ||
+        !make_tmap_bf16_rows128(&to, O, s.L, (uint64_t)s.B * s.Hq, 64))
+        return cudaErrorInvalidValue;
+    const size_t smem = fwd_tc_smem(topk);
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    FwdTcArgs args{idx, cnt, lse, status, s.Hq, s.Hkv, s.L, NQB, topk, sm_scale * kLog2e};
+    const long long grid = (long long)s.B * s.Hkv * NQB;
+    ProfScope prof(K_FWD, st);
+    attn_fwd_tc_kernel<<<(unsigned)grid, kThreads, smem, st>>>(tq, tk, tv, to, args);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- self-test
+// One CTA runs the two MMA shapes of the kernel above on fixed operands:
+//   S = A B^T (A: 128 x 128, B: 64 x 128, both K-major from TMA tiles),
+//   O = bf16(S) V (bf16(S) written to TMEM, V: 64 x 128 as an MN-major B).
+namespace {
+
+__global__ void __launch_bounds__(128)
+tc_selftest_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmV, float* S, float* O, int* status) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    const uint32_t sb = smem_u32(smem);
+    const int warp = threadIdx.x >> 5;
+    const uint32_t sA = sb, sB = sb + kQBytes, sV = sB + kKBytes;
+    const uint32_t bars = sV + kKBytes;  // 0: loads, 1: S done, 2: P stored, 3: O done
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (bars - sb) + 64);
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 4; ++i) mbar_init(bars + 8 * i, i == 2 ? 128 : 1);
+        fence_barrier_init();
+        *abort_flag = 0;
+    }
+    if (warp == 0) {
+        tmem_alloc(bars + 48, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + (bars - sb) + 48);
+    bool ok = true;
+    if (threadIdx.x == 0) {
+        mbar_expect_tx(bars, kQBytes + 2 * kKBytes);
+        for (int dh = 0; dh < 2; ++dh) {
+            for (int hl = 0; hl < 2; ++hl)
+                tma_load_3d(sA + dh * kHalfQ + hl * (kHalfQ / 2), &tmA, bars, dh * 64, hl * 64, 0);
+            tma_load_3d(sB + dh * kKVHalf, &tmB, bars, dh * 64, 0, 0);
+            tma_load_3d(sV + dh * kKVHalf, &tmV, bars, dh * 64, 0, 0);
+        }
+        ok = mbar_wait(bars, 0, abort_flag, status);
+        if (!ok) mbar_wait_drain(bars, 0);  // the copies must land before exit
+        tc_fence_after();
+        if (ok) {
+#pragma unroll
+            for (int ks = 0; ks < 8; ++ks) {
+                const uint32_t off = (uint32_t)((ks & 3) * 32);
+                mma_ss(tmem + 128, sdesc_sw128(sA + (ks >> 2) * kHalfQ + off, 16, 1024),
+                       sdesc_sw128(sB + (ks >> 2) * kKVHalf + off, 16, 1024),
+                       idesc_bf16(128, 64, false), ks > 0 ? 1u : 0u);
+            }
+        }
+        mma_commit(bars + 8);
+    }
+    ok = mbar_wait(bars + 8, 0, abort_flag, status);
+    ok = __all_sync(0xffffffffu, ok);
+    const int row = threadIdx.x;
+    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+    if (ok) {
+        tc_fence_after();
+        uint32_t sr[64];
+        tmem_ld32(lane_base + 128, sr);
+        tmem_ld32(lane_base + 160, sr + 32);
+        for (int c = 0; c < 64; ++c) S[row * 64 + c] = __uint_as_float(sr[c]);
+        uint32_t pk[32];
+        for (int c = 0; c < 32; ++c)
+            pk[c] = pack2_bf16(__uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]));
+        tmem_st32(lane_base + 128, pk);
+        tc_fence_before();
+        mbar_arrive(bars + 16);
+    }
+    if (threadIdx.x == 0 && ok) {
+        ok = mbar_wait(bars + 16, 0, abort_flag, status);
+        tc_fence_after();
+        if (ok) {
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+                mma_ts(tmem, tmem + 128 + ks * 8, sdesc_sw128(sV + ks * 2048, kKVHalf, 1024),
+                       idesc_bf16(128, 128, true), ks > 0 ? 1u : 0u);
+        }
+        mma_commit(bars + 24);
+    }
+    ok = mbar_wait(bars + 24, 0, abort_flag, status);
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok) {
+        tc_fence_after();
+        for (int c4 = 0; c4 < 4; ++c4) {
+            uint32_t o[32];
+            tmem_ld32(lane_base + 32 * c4, o);
+            for (int c = 0; c < 32; ++c) O[row * 128 + 32 * c4 + c] = __uint_as_float(o[c]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_tc_selftest(const void* A, const void* B, const void* V, float* S, float* O,
+                               int* status, cudaStream_t st) {
+    CUtensorMap ta, tb, tv;
+    if (!make_tmap_bf16_rows128(&ta, A, 128, 1, 64) || !make_tmap_bf16_rows128(&tb, B, 64, 1, 64) ||
+        !make_tmap_bf16_rows128(&tv, V, 64, 1, 64))
+        return cudaErrorInvalidValue;
+    const size_t smem = 1024 + kQBytes + 2 * kKBytes + 256;
+    cudaError_t e = cudaFuncSetAttribute(tc_selftest_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    tc_selftest_kernel<<<1, 128, smem, st>>>(ta, tb, tv, S, O, status);
+    return cudaGetLastError();
+}
+
+}  // namespace phsa

@@ -152,6 +152,15 @@ int phsa_get_device_status(void* stream) {
     return v;
 }
 
+int phsa_selftest_tcgen05(const void* A, const void* B, const void* V, float* S, float* O,
+                          void* stream) {
+    if (!A || !B || !V || !S || !O) return PHSA_ERR_INVALID_ARG;
+    if (!aligned16(A) || !aligned16(B) || !aligned16(V)) return PHSA_ERR_INVALID_ARG;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_tc_selftest(A, B, V, S, O, st, static_cast<cudaStream_t>(stream)));
+}
+
 const char* phsa_status_string(int code) {
     switch (code) {
         case PHSA_OK: return "PHSA_OK";

@@ -2,6 +2,7 @@
 // (phsa_api.cu) before any of these run.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -32,6 +33,15 @@ cudaError_t launch_block_repr(const void* K, const uint8_t* mask, const phsa_sha
 cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_shape& s,
                                  const phsa_select_params& p, int32_t* idx, int32_t* cnt,
                                  int* status, cudaStream_t st);
+
+// tcgen05 forward for G = 2 (attn_fwd_tc.cu); launch_attn_fwd dispatches to it.
+cudaError_t launch_attn_fwd_tc(const void* Q, const void* K, const void* V, const int32_t* idx,
+                               const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                               void* O, float* lse, int* status, cudaStream_t st);
+cudaError_t launch_tc_selftest(const void* A, const void* B, const void* V, float* S, float* O,
+                               int* status, cudaStream_t st);
+bool make_tmap_bf16_rows128(CUtensorMap* map, const void* base, uint64_t rows, uint64_t planes,
+                            uint32_t box_rows);
 
 cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const int32_t* idx,
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,

@@ -74,8 +74,9 @@ def _declare(L):
     L.phsa_profile_read.argtypes = [I, ctypes.POINTER(ctypes.c_char_p),
                                     ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)]
     L.phsa_profile_read.restype = I
+    L.phsa_selftest_tcgen05.argtypes = [P, P, P, P, P, P]
     for fn in ("phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
-               "phsa_sparse_attn_bwd", "phsa_get_device_status"):
+               "phsa_sparse_attn_bwd", "phsa_get_device_status", "phsa_selftest_tcgen05"):
         getattr(L, fn).restype = I
 
 
@@ -236,6 +237,20 @@ def phsa_profile_read() -> dict:
     if k < 0:
         raise PhsaError("phsa_profile_read", k)
     return {names[i].decode(): (float(ms[i]), int(cnt[i])) for i in range(k)}
+
+
+def phsa_selftest_tcgen05(A, B, V, stream=None):
+    """Diagnostic: (S = A B^T, O = bf16(S) V) computed on the tensor cores, fp32."""
+    _check(A, "A", torch.bfloat16, 2)
+    _check(B, "B", torch.bfloat16, 2)
+    _check(V, "V", torch.bfloat16, 2)
+    if tuple(A.shape) != (128, 128) or tuple(B.shape) != (64, 128) or tuple(V.shape) != (64, 128):
+        raise ValueError("A must be [128,128], B and V [64,128]")
+    S = torch.empty((128, 64), dtype=torch.float32, device=A.device)
+    O = torch.empty((128, 128), dtype=torch.float32, device=A.device)
+    rc = load().phsa_selftest_tcgen05(_ptr(A), _ptr(B), _ptr(V), _ptr(S), _ptr(O), _stream(stream))
+    _raise("phsa_selftest_tcgen05", rc)
+    return S, O
 
 
 def phsa_forward(Q, K, V, punct_mask, lam: float, topk: int, n_init: int = 1, n_local: int = 1,
