@@ -33,6 +33,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 from paper_2601_02819_gb300 import inputs  # noqa: E402
+from paper_2601_02819_gb300.sharding import max_over_ranks, rank_seed, shard_sequences  # noqa: E402
 
 METRIC = ("sparse-attn prefill tokens/s + effective TFLOPS at 32k, 97.3% sparsity; "
           "% roofline")
@@ -250,7 +251,9 @@ def run_ours(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     w = inputs.WORKLOADS[args.workload]
-    x = inputs.make_inputs(w, with_grad=True, seed=w.seed + 7919 * rank)
+    # weak scaling: every rank runs one batch of the workload on its own sequences
+    mine = shard_sequences(world * w.B, world, rank)
+    x = inputs.make_inputs(w, with_grad=True, seed=rank_seed(w.seed, mine[0]))
 
     def dev_bf16(a):
         return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
@@ -307,12 +310,7 @@ def run_ours(args):
     phsa.phsa_profile_enable(False)
     prof = phsa.phsa_profile_read()
     clk = clocks.stop(t_wall0, t_wall1)
-    ms_total = ev0.elapsed_time(ev1)
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([ms_total], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(ev0.elapsed_time(ev1), device=dev)
     ms_step = ms_total / args.steps
     status = phsa.phsa_get_device_status()
 
@@ -351,12 +349,7 @@ def run_ours(args):
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-        ms_e2e = e0.elapsed_time(e1) / n_e2e
-        if world > 1:
-            import torch.distributed as dist
-            tt = torch.tensor([ms_e2e], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            ms_e2e = float(tt.item())
+        ms_e2e = max_over_ranks(e0.elapsed_time(e1) / n_e2e, device=dev)
         e2e = {"value": world * w.B * w.L / (ms_e2e / 1e3), "unit": "tokens/s",
                "ms_per_step": ms_e2e, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "steps": n_e2e}
