@@ -148,6 +148,31 @@ int phsa_sparse_attn_bwd(const void* Q, const void* K, const void* V, const void
                          void* stream);
 
 /*
+ * The backward pass above for callers that cannot allocate device memory (no
+ * counterpart in the paper). Some callers may not call cudaMalloc where they
+ * run the backward pass: engines that reserve all of HBM for their own pools
+ * at start-up, plugin interfaces whose execute step must not allocate, or hot
+ * loops that cannot afford cudaMalloc's implicit device synchronisation. This
+ * entry point allocates nothing: its scratch is a fixed 64 MiB device array
+ * inside the library, held by every GPU that loads the library until the
+ * process exits. The caller still passes inputs and outputs, as for
+ * phsa_sparse_attn_bwd, whose results it reproduces.
+ *   - Shapes whose phsa_sparse_attn_bwd_workspace() exceeds 64 MiB return
+ *     PHSA_ERR_WORKSPACE before any launch (for example B=1, Hq=16, Hkv=8,
+ *     topk=8 fits up to L = 8192).
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current) and caches it; make that first call before any
+ *     stream capture begins.
+ *   - All calls share the array and it keeps the last call's contents (each
+ *     call clears what must start at zero). Calls that overlap on the GPU, for
+ *     example on two streams, race on it: serialise them.
+ */
+int phsa_sparse_attn_bwd_noalloc(const void* Q, const void* K, const void* V, const void* O,
+                                 const void* dO, const float* lse, const int32_t* block_idx,
+                                 const int32_t* block_cnt, phsa_shape s, int topk, float sm_scale,
+                                 void* dQ, void* dK, void* dV, void* stream);
+
+/*
  * Synchronises `stream`, returns the device status word of the current
  * device (PHSA_OK or the first device-side error code recorded since the
  * last call) and clears it. Returns PHSA_ERR_CUDA if the synchronisation

@@ -61,6 +61,11 @@ int check_topk(const phsa_shape& s, int topk) {
 
 }  // namespace
 
+namespace phsa {
+// The status word of the current device, for entry points in other files.
+int* device_status_word() { return status_ptr(); }
+}  // namespace phsa
+
 extern "C" {
 
 int phsa_build_block_repr(const void* K, const uint8_t* punct_mask, phsa_shape s, float lambda,

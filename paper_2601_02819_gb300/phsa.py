@@ -75,6 +75,9 @@ def _declare(L):
                                     ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)]
     L.phsa_profile_read.restype = I
     L.phsa_selftest_tcgen05.argtypes = [P, P, P, P, P, P]
+    L.phsa_sparse_attn_bwd_noalloc.argtypes = [P, P, P, P, P, P, P, P, phsa_shape, I, F, P, P, P,
+                                               P]
+    L.phsa_sparse_attn_bwd_noalloc.restype = I
     for fn in ("phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
                "phsa_sparse_attn_bwd", "phsa_get_device_status", "phsa_selftest_tcgen05"):
         getattr(L, fn).restype = I
@@ -214,6 +217,31 @@ def phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_scale=Non
         make_shape(B, L, Hq, Hkv, D), int(topk), float(sm_scale), _ptr(workspace),
         ctypes.c_size_t(workspace.numel()), _ptr(dQ), _ptr(dK), _ptr(dV), _stream(stream))
     _raise("phsa_sparse_attn_bwd", rc)
+    return dQ, dK, dV
+
+
+def phsa_sparse_attn_bwd_noalloc(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_scale=None,
+                                 dQ=None, dK=None, dV=None, stream=None):
+    """The backward pass without any workspace: for callers that cannot allocate
+    device memory where they run it. The library's fixed 64 MiB scratch array is
+    used instead (shapes needing more are rejected); calls must not overlap on
+    the GPU. Output tensors are allocated here only when not passed in."""
+    for name, t in (("Q", Q), ("K", K), ("V", V), ("O", O), ("dO", dO)):
+        _check(t, name, torch.bfloat16, 4)
+    _check(lse, "lse", torch.float32, 3)
+    _check(block_idx, "block_idx", torch.int32, 4)
+    _check(block_cnt, "block_cnt", torch.int32, 3)
+    B, Hq, L, D = Q.shape
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    dQ = torch.empty_like(Q) if dQ is None else dQ
+    dK = torch.empty_like(K) if dK is None else dK
+    dV = torch.empty_like(V) if dV is None else dV
+    rc = load().phsa_sparse_attn_bwd_noalloc(
+        _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(dO), _ptr(lse), _ptr(block_idx), _ptr(block_cnt),
+        make_shape(B, L, Hq, K.shape[1], D), int(block_idx.shape[-1]), float(sm_scale), _ptr(dQ),
+        _ptr(dK), _ptr(dV), _stream(stream))
+    _raise("phsa_sparse_attn_bwd_noalloc", rc)
     return dQ, dK, dV
 
 
