@@ -26,7 +26,7 @@ namespace phsa {
 
 namespace {
 
-constexpr int kChunk = 32;  // query blocks per dK/dV work item
+constexpr int kChunk = kBwdChunk;  // query blocks per dK/dV work item
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -80,9 +80,7 @@ __global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* 
     }
 }
 
-struct TInfo {
-    int off, n, nch, slot;  // list offset, list length, chunks, first partial slot (-1: none)
-};
+using TInfo = BwdTInfo;
 
 // Block-wide exclusive scan of one int per thread (blockDim.x = 1024).
 __device__ int block_excl_scan(int v, int* tmp, int& total) {

@@ -1,15 +1,19 @@
 // Stage (c) forward on the 5th-generation tensor cores (tcgen05 + TMEM + TMA),
 // for GQA groups of two query heads (G*64 = 128 query rows per tile).
 //
-// One CTA per (query block qb, KV head g), 192 threads in three roles:
-//   warp 4 (one lane)  TMA producer: the 128 x 128 Q tile once, then for every
-//                      selected block its 64 x 128 K and V tiles into a
-//                      two-stage shared-memory ring (gathered by block index).
+// One CTA per (query block qb, KV head g), 224 threads in four roles:
+//   warp 4 (one lane)  TMA producer of Q (the 128 x 128 tile, once) and of the
+//                      selected K tiles (64 x 128, gathered by block index)
+//                      into a two-slot ring; a slot is refilled as soon as the
+//                      QK MMA that read it has finished.
+//   warp 6 (one lane)  TMA producer of the selected V tiles into their own
+//                      two-slot ring, refilled when the PV MMA is done.
 //   warp 5 (one lane)  MMA issuer: S_j = Q K_j^T (M=128, N=64, K=128) into one
 //                      of two TMEM score buffers, and O += P_j V_j (M=128,
-//                      N=128, K=64) with P_j read from TMEM. QK of block j+1 is
-//                      issued before PV of block j, so the tensor core works
-//                      while the softmax of block j runs.
+//                      N=128, K=64) with P_j read from TMEM. It polls and issues
+//                      whichever is ready first, QK of block j+1 (once PV of
+//                      block j-1 is issued) or PV of block j, so the tensor
+//                      core works while the softmax of block j runs.
 //   warps 0-3          softmax: thread r owns query row r (TMEM lane r). It
 //                      loads its 64 scores, applies the causal mask inside the
 //                      query's own block, keeps a running max and sum in the
@@ -32,20 +36,22 @@ namespace {
 
 using namespace tc;
 
-constexpr int kStages = 2;
+constexpr int kSlots = 2;                   // K ring and V ring
 constexpr int kHalfQ = 128 * 64 * 2;        // one 64-column half of the Q tile (16 KB)
 constexpr int kQBytes = 2 * kHalfQ;         // 32 KB
 constexpr int kKVHalf = 64 * 64 * 2;        // one 64-column half of a K or V block (8 KB)
 constexpr int kKBytes = 2 * kKVHalf;        // 16 KB
-constexpr int kStageBytes = 2 * kKBytes;    // K and V of one block
 constexpr int kOffQ = 0;
-constexpr int kOffKV = kQBytes;
-constexpr int kOffBar = kOffKV + kStages * kStageBytes;
+constexpr int kOffK = kQBytes;                        // K slots
+constexpr int kOffV = kOffK + kSlots * kKBytes;       // V slots
+constexpr int kOffBar = kOffV + kSlots * kKBytes;
 // barriers
 constexpr int B_Q = 0;
-constexpr int B_KVFULL = 1;                 // + stage
-constexpr int B_KVEMPTY = B_KVFULL + kStages;
-constexpr int B_SFULL = B_KVEMPTY + kStages;  // + buffer
+constexpr int B_KFULL = 1;                  // + slot
+constexpr int B_KEMPTY = B_KFULL + kSlots;
+constexpr int B_VFULL = B_KEMPTY + kSlots;
+constexpr int B_VEMPTY = B_VFULL + kSlots;
+constexpr int B_SFULL = B_VEMPTY + kSlots;  // + buffer
 constexpr int B_PFULL = B_SFULL + 2;
 constexpr int B_PVDONE = B_PFULL + 2;
 constexpr int B_OFINAL = B_PVDONE + 1;
@@ -53,7 +59,7 @@ constexpr int B_DRAIN = B_OFINAL + 1;
 constexpr int kNumBars = B_DRAIN + 1;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag, block count
 constexpr int kOffList = kOffMisc + 16;
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kColO = 0;
 constexpr float kRescaleLog2 = 8.0f;
@@ -93,9 +99,11 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_Q), 1);
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(bar(B_KVFULL + s), 1);
-            mbar_init(bar(B_KVEMPTY + s), 1);
+        for (int s = 0; s < kSlots; ++s) {
+            mbar_init(bar(B_KFULL + s), 1);
+            mbar_init(bar(B_KEMPTY + s), 1);
+            mbar_init(bar(B_VFULL + s), 1);
+            mbar_init(bar(B_VEMPTY + s), 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(B_SFULL + i), 1);
@@ -120,37 +128,39 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     const int n = reinterpret_cast<volatile int*>(smem + kOffMisc)[2];
     const int hq0 = b * a.Hq + g * 2;  // first query head (plane) of the group
 
-    if (warp == 4) {
-        // ------------------------------------------------ TMA producer
+    if (warp == 4 || warp == 6) {
+        // ------------------------------------------------ TMA producers (K / V)
         if (lane == 0 && n > 0) {
-            prefetch_tmap(&tmQ);
-            prefetch_tmap(&tmK);
-            prefetch_tmap(&tmV);
-            mbar_expect_tx(bar(B_Q), kQBytes);
-            for (int hl = 0; hl < 2; ++hl)
-                for (int dh = 0; dh < 2; ++dh)
-                    tma_load_3d(sb + kOffQ + dh * kHalfQ + hl * (kHalfQ / 2), &tmQ, bar(B_Q),
-                                dh * 64, qb * 64, hq0 + hl);
+            const bool is_k = warp == 4;
+            const CUtensorMap* map = is_k ? &tmK : &tmV;
+            prefetch_tmap(map);
+            if (is_k) {
+                prefetch_tmap(&tmQ);
+                mbar_expect_tx(bar(B_Q), kQBytes);
+                for (int hl = 0; hl < 2; ++hl)
+                    for (int dh = 0; dh < 2; ++dh)
+                        tma_load_3d(sb + kOffQ + dh * kHalfQ + hl * (kHalfQ / 2), &tmQ, bar(B_Q),
+                                    dh * 64, qb * 64, hq0 + hl);
+            }
+            const int full = is_k ? B_KFULL : B_VFULL, empty = is_k ? B_KEMPTY : B_VEMPTY;
+            const uint32_t ring = sb + (is_k ? kOffK : kOffV);
             int issued = 0;
             for (int j = 0; j < n; ++j) {
-                const int s = j % kStages;
-                if (j >= kStages &&
-                    !mbar_wait(bar(B_KVEMPTY + s), ((j / kStages) - 1) & 1, abort_flag, a.status))
+                const int s = j % kSlots;
+                if (j >= kSlots &&
+                    !mbar_wait(bar(empty + s), ((j / kSlots) - 1) & 1, abort_flag, a.status))
                     break;
-                const uint32_t kb = sb + kOffKV + s * kStageBytes;
                 const int t = list[j];
-                mbar_expect_tx(bar(B_KVFULL + s), kStageBytes);
-                for (int dh = 0; dh < 2; ++dh) {
-                    tma_load_3d(kb + dh * kKVHalf, &tmK, bar(B_KVFULL + s), dh * 64, t * 64, bg);
-                    tma_load_3d(kb + kKBytes + dh * kKVHalf, &tmV, bar(B_KVFULL + s), dh * 64,
+                mbar_expect_tx(bar(full + s), kKBytes);
+                for (int dh = 0; dh < 2; ++dh)
+                    tma_load_3d(ring + s * kKBytes + dh * kKVHalf, map, bar(full + s), dh * 64,
                                 t * 64, bg);
-                }
                 issued = j + 1;
             }
             // Own copies must have landed before the CTA may exit.
-            mbar_wait_drain(bar(B_Q), 0);
-            for (int j = issued - kStages; j < issued; ++j)
-                if (j >= 0) mbar_wait_drain(bar(B_KVFULL + j % kStages), (j / kStages) & 1);
+            if (is_k) mbar_wait_drain(bar(B_Q), 0);
+            for (int j = issued - kSlots; j < issued; ++j)
+                if (j >= 0) mbar_wait_drain(bar(full + j % kSlots), (j / kSlots) & 1);
         }
     } else if (warp == 5) {
         // ------------------------------------------------ MMA issuer
@@ -159,13 +169,15 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             constexpr uint32_t idesc_pv = idesc_bf16(128, 128, true);
             bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
             tc_fence_after();
-            for (int j = 0; ok && j <= n; ++j) {
-                if (j < n) {
-                    const int s = j % kStages;
-                    if (!mbar_wait(bar(B_KVFULL + s), (j / kStages) & 1, abort_flag, a.status)) break;
+            int nq = 0, np = 0;  // next QK and next PV to issue
+            uint64_t t0 = global_ns();
+            while (ok && np < n) {
+                bool progressed = false;
+                // QK_nq reuses score buffer nq&1, free once PV_{nq-2} has been issued.
+                if (nq < n && nq <= np + 1 && mbar_try_wait(bar(B_KFULL + nq % kSlots), (nq / kSlots) & 1)) {
                     tc_fence_after();
-                    const uint32_t kb = sb + kOffKV + s * kStageBytes;
-                    const uint32_t d = tmem + col_s(j & 1);
+                    const uint32_t kb = sb + kOffK + (nq % kSlots) * kKBytes;
+                    const uint32_t d = tmem + col_s(nq & 1);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks) {
                         const uint32_t off = (uint32_t)((ks & 3) * 32);
@@ -173,22 +185,38 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                         const uint64_t bd = sdesc_sw128(kb + (ks >> 2) * kKVHalf + off, 16, 1024);
                         mma_ss(d, ad, bd, idesc_qk, ks > 0 ? 1u : 0u);
                     }
-                    mma_commit(bar(B_SFULL + (j & 1)));
+                    mma_commit(bar(B_SFULL + (nq & 1)));
+                    mma_commit(bar(B_KEMPTY + nq % kSlots));
+                    ++nq;
+                    progressed = true;
                 }
-                if (j >= 1) {
-                    const int jj = j - 1, s = jj % kStages;
-                    if (!mbar_wait(bar(B_PFULL + (jj & 1)), (jj >> 1) & 1, abort_flag, a.status)) break;
+                if (np < nq && mbar_try_wait(bar(B_PFULL + (np & 1)), (np >> 1) & 1)) {
+                    if (!mbar_wait(bar(B_VFULL + np % kSlots), (np / kSlots) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
                     tc_fence_after();
-                    const uint32_t vb = sb + kOffKV + s * kStageBytes + kKBytes;
-                    const uint32_t pt = tmem + col_s(jj & 1);
+                    const uint32_t vb = sb + kOffV + (np % kSlots) * kKBytes;
+                    const uint32_t pt = tmem + col_s(np & 1);
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks) {
                         const uint64_t bd = sdesc_sw128(vb + ks * 2048, kKVHalf, 1024);
-                        mma_ts(tmem + kColO, pt + ks * 8, bd, idesc_pv, (jj > 0 || ks > 0) ? 1u : 0u);
+                        mma_ts(tmem + kColO, pt + ks * 8, bd, idesc_pv, (np > 0 || ks > 0) ? 1u : 0u);
                     }
-                    mma_commit(bar(B_KVEMPTY + s));
+                    mma_commit(bar(B_VEMPTY + np % kSlots));
                     mma_commit(bar(B_PVDONE));
-                    if (jj == n - 1) mma_commit(bar(B_OFINAL));
+                    if (np == n - 1) mma_commit(bar(B_OFINAL));
+                    ++np;
+                    progressed = true;
+                }
+                if (progressed) {
+                    t0 = global_ns();
+                } else if (*abort_flag) {
+                    ok = false;
+                } else if (global_ns() - t0 > kWaitLimitNs) {
+                    *abort_flag = 1;
+                    atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
+                    ok = false;
                 }
             }
             // Every MMA issued above must be complete before TMEM is freed.
@@ -209,17 +237,17 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             if (!ok) break;
             tc_fence_after();
             uint32_t sr[64];
-            tmem_ld32(lane_base + col_s(buf), sr);
-            tmem_ld32(lane_base + col_s(buf) + 32, sr + 32);
-            const bool diag = list[j] == qb;
-            float mx = -INFINITY;
+            tmem_ld64(lane_base + col_s(buf), sr);
+            if (list[j] == qb) {  // the query's own block: token-level causal mask
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                float v = __uint_as_float(sr[c]) * a.scale_log2;
-                if (diag && c > tok) v = -INFINITY;
-                sr[c] = __float_as_uint(v);
-                mx = fmaxf(mx, v);
+                for (int c = 0; c < 64; ++c)
+                    if (c > tok) sr[c] = __float_as_uint(-INFINITY);
             }
+            // row max of the raw scores (the scale is positive)
+            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int c = 0; c < 64; ++c) m4[c & 3] = fmaxf(m4[c & 3], __uint_as_float(sr[c]));
+            const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;
             if (j == 0) {
                 m_used = mx;
             } else {
@@ -230,14 +258,14 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     ok = __all_sync(0xffffffffu, ok);
                     if (!ok) break;
                     tc_fence_after();
-                    const float f = need ? exp2f(m_used - mx) : 1.0f;
+                    const float f = need ? ex2_approx(m_used - mx) : 1.0f;
+#pragma unroll 1
+                    for (int c8 = 0; c8 < 8; ++c8) {
+                        uint32_t o[16];
+                        tmem_ld16(lane_base + kColO + 16 * c8, o);
 #pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) {
-                        uint32_t o[32];
-                        tmem_ld32(lane_base + kColO + 32 * c4, o);
-#pragma unroll
-                        for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
-                        tmem_st32(lane_base + kColO + 32 * c4, o);
+                        for (int c = 0; c < 16; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
+                        tmem_st16(lane_base + kColO + 16 * c8, o);
                     }
                     if (need) {
                         l *= f;
@@ -245,17 +273,21 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     }
                 }
             }
-            uint32_t pk[32];
-            float rs = 0.f;
+            // p = 2^(s * scale_log2 - m): one FFMA and one SFU op per score
+            // P is packed in place: entry c (c < 32) takes the pair (2c, 2c+1), both
+            // read before entry c is overwritten.
+            float r4[4] = {0.f, 0.f, 0.f, 0.f};
+            const float neg_m = -m_used;
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                const float p0 = exp2f(__uint_as_float(sr[2 * c]) - m_used);
-                const float p1 = exp2f(__uint_as_float(sr[2 * c + 1]) - m_used);
-                rs += p0 + p1;
-                pk[c] = pack2_bf16(p0, p1);
+                const float p0 = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), a.scale_log2, neg_m));
+                const float p1 = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), a.scale_log2, neg_m));
+                r4[c & 3] += p0 + p1;
+                sr[c] = pack2_bf16(p0, p1);
             }
+            const float rs = (r4[0] + r4[1]) + (r4[2] + r4[3]);
             l += rs;
-            tmem_st32(lane_base + col_s(buf), pk);
+            tmem_st32(lane_base + col_s(buf), sr);
             tc_fence_before();
             mbar_arrive(bar(B_PFULL + buf));
         }

@@ -47,6 +47,26 @@ cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const i
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                             void* O, float* lse, int* status, cudaStream_t st);
 
+// Transposed selection, one entry per (b, kv head, KV block t): the offset and
+// length of t's ascending list of selecting query blocks, its number of work
+// chunks, and its first fp32 partial slot (-1 when it has a single chunk).
+struct BwdTInfo {
+    int off, n, nch, slot;
+};
+constexpr int kBwdChunk = 32;  // query blocks per dK/dV work item
+
+// tcgen05 backward kernels for G = 2 (attn_bwd_tc.cu).
+cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
+                           const float* lse, const float* delta, const BwdTInfo* tinfo,
+                           const int32_t* qlist, const int2* work, const int32_t* nwork,
+                           const phsa_shape& s, int topk, int work_max, int slot_max,
+                           float sm_scale, void* dK, void* dV, float* partial, int* status,
+                           cudaStream_t st);
+cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* dO,
+                         const float* lse, const float* delta, const int32_t* idx,
+                         const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                         void* dQ, int* status, cudaStream_t st);
+
 // Backward workspace layout (all offsets 256-byte aligned).
 struct BwdLayout {
     size_t bits, tinfo, qlist, work, nwork, delta, partial, total;
