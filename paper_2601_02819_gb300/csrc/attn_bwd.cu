@@ -632,6 +632,12 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
+    const bool pair = s.Hq / s.Hkv == 2;  // two query heads per KV head: tcgen05 kernels
+    if (pair) {
+        e = launch_dkdv_tc(Q, K, V, dO, lse, delta, tinfo, qlist, work, nwork, s, topk,
+                           l.work_max, l.slot_max, sm_scale, dK, dV, partial, status, st);
+        if (e != cudaSuccess) return e;
+    } else {
     e = cudaFuncSetAttribute(dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kKvSmem);
     if (e != cudaSuccess) return e;
     {
@@ -644,6 +650,7 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
             static_cast<__nv_bfloat16*>(dV), partial);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     {
         ProfScope prof(K_BWD_DKDV_SUM, st);
         dkdv_sum_kernel<<<dim3(l.nqb, bgs), 256, 0, st>>>(
@@ -652,9 +659,8 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
-    return (s.Hq / s.Hkv == 2)
-               ? launch_dq_g<2>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st)
-               : launch_dq_g<1>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
+    return pair ? launch_dq_tc(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st)
+                : launch_dq_g<1>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
 }
 
 }  // namespace phsa

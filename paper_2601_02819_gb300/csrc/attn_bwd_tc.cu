@@ -1,0 +1,653 @@
+// Stage (c) backward on the tensor cores (tcgen05 + TMEM + TMA), for GQA
+// groups of two query heads, so that every MMA has M = 128.
+//
+// dq_tc_kernel: one CTA per (query block qb, KV head g), 352 threads.
+//   For every selected block j (K_j, V_j gathered by TMA into 4- and 3-slot rings):
+//     S_j  = Q K_j^T      (M128 N64 K128, A = Q, B = K_j, both K-major)
+//     dP_j = dO V_j^T     (M128 N64 K128)
+//     dS_j = P_j (dP_j - Delta), P_j = exp(S_j * scale - lse)   (8 warps, TMEM)
+//     dQ  += dS_j K_j     (M128 N128 K64, A = dS_j in TMEM, B = K_j MN-major)
+//   S/dP are double-buffered in TMEM so the tensor core computes block j+1
+//   while the elementwise warps work on block j. dQ * scale -> TMA store.
+//
+// dkdv_tc_kernel: one CTA per work item (KV block t, chunk of <= 32 query
+//   blocks that selected t), 320 threads. K_t and V_t stay in shared memory;
+//   the Q and dO tiles (both heads stacked: 128 rows) of every listed query
+//   block stream through a two-stage ring:
+//     S  = Q K_t^T, dP = dO V_t^T            (M128 N64 K128)
+//     P, dS (8 warps) -> shared memory (bf16, 128 rows x 64 keys)
+//     dV^T += dO^T P, dK^T += Q^T dS          (M128 N64 K128; A = dO / Q read
+//                                             MN-major, B = P / dS MN-major)
+//   dK^T and dV^T live in TMEM with the head dimension on the lanes. A KV
+//   block with a single chunk writes bf16 dK, dV through TMA stores; a longer
+//   list writes fp32 partials that dkdv_sum (attn_bwd.cu) adds in chunk order.
+//
+// Every wait is bounded in time; on expiry the kernel records
+// PHSA_ERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
+#include "phsa_common.cuh"
+#include "phsa_internal.h"
+#include "tc_common.cuh"
+
+namespace phsa {
+
+namespace {
+
+using namespace tc;
+
+constexpr int kHalf128 = 128 * 64 * 2;  // 128 rows x 64 columns, bf16 (16 KB)
+constexpr int kHalf64 = 64 * 64 * 2;    // 64 rows x 64 columns (8 KB)
+constexpr int kTile128 = 2 * kHalf128;  // 128 x 128 (32 KB)
+constexpr int kTile64 = 2 * kHalf64;    // 64 x 128 (16 KB)
+constexpr uint32_t kTmemCols = 512;
+
+__device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
+    return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+// ============================================================== dQ
+namespace dq {
+constexpr int kKSlots = 4, kVSlots = 3;
+constexpr int kOffQ = 0;
+constexpr int kOffDO = kOffQ + kTile128;
+constexpr int kOffK = kOffDO + kTile128;
+constexpr int kOffV = kOffK + kKSlots * kTile64;
+constexpr int kOffBar = kOffV + kVSlots * kTile64;
+constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = B_KFULL + kKSlots, B_VFULL = B_KEMPTY + kKSlots,
+              B_VEMPTY = B_VFULL + kVSlots, B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2,
+              B_FINAL = B_DSFULL + 2, B_DRAIN = B_FINAL + 1, kNumBars = B_DRAIN + 1;
+constexpr int kOffMisc = kOffBar + kNumBars * 8;
+constexpr int kOffList = kOffMisc + 16;
+constexpr int kThreads = 352;  // 8 elementwise warps, K/Q/dO producer, MMA, V producer
+constexpr uint32_t kColDQ = 0;
+__device__ __forceinline__ uint32_t col_s(int b) { return 128u + 128u * (uint32_t)b; }
+__device__ __forceinline__ uint32_t col_dp(int b) { return 192u + 128u * (uint32_t)b; }
+__device__ __forceinline__ uint32_t col_ds(int b) { return 384u + 32u * (uint32_t)b; }
+constexpr size_t smem_bytes(int topk) { return 1024 + (size_t)kOffList + (size_t)(topk + 1) * 4; }
+}  // namespace dq
+
+struct DqArgs {
+    const int32_t* idx;
+    const int32_t* cnt;
+    const float* lse;
+    const float* delta;
+    int* status;
+    int Hq, Hkv, L, NQB, topk;
+    float scale_log2, sm_scale;
+};
+
+__global__ void __launch_bounds__(dq::kThreads, 1)
+dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+             const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
+             const __grid_constant__ CUtensorMap tmdQ, const DqArgs a) {
+    using namespace dq;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    const uint32_t sb = smem_u32(smem);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int unit = blockIdx.x;
+    const int qb = a.NQB - 1 - (unit % a.NQB);
+    const int bg = unit / a.NQB;
+    const int b = bg / a.Hkv, g = bg % a.Hkv;
+    const long long lu = (long long)bg * a.NQB + qb;
+    auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
+    int* list = reinterpret_cast<int*>(smem + kOffList);
+    const int hq0 = b * a.Hq + g * 2;
+
+    if (threadIdx.x == 0) {
+        mbar_init(bar(B_Q), 1);
+        for (int s = 0; s < kKSlots; ++s) {
+            mbar_init(bar(B_KFULL + s), 1);
+            mbar_init(bar(B_KEMPTY + s), 1);
+        }
+        for (int s = 0; s < kVSlots; ++s) {
+            mbar_init(bar(B_VFULL + s), 1);
+            mbar_init(bar(B_VEMPTY + s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(B_SPFULL + i), 1);
+            mbar_init(bar(B_DSFULL + i), 256);
+        }
+        mbar_init(bar(B_FINAL), 1);
+        mbar_init(bar(B_DRAIN), 1);
+        fence_barrier_init();
+        *abort_flag = 0;
+        reinterpret_cast<int*>(smem + kOffMisc)[2] =
+            compact_block_list(a.idx + lu * a.topk, a.cnt[lu], a.topk, qb, list, nullptr);
+    }
+    if (warp == 9) {
+        tmem_alloc(sb + kOffMisc, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
+    const int n = reinterpret_cast<volatile int*>(smem + kOffMisc)[2];
+
+    if (warp == 8 || warp == 10) {
+        // ------------------------------------------------ TMA producers
+        if (lane == 0 && n > 0) {
+            const bool is_k = warp == 8;
+            const CUtensorMap* map = is_k ? &tmK : &tmV;
+            const int slots = is_k ? kKSlots : kVSlots;
+            const int full = is_k ? B_KFULL : B_VFULL, empty = is_k ? B_KEMPTY : B_VEMPTY;
+            const uint32_t ring = sb + (is_k ? kOffK : kOffV);
+            prefetch_tmap(map);
+            if (is_k) {
+                mbar_expect_tx(bar(B_Q), 2 * kTile128);
+                for (int hl = 0; hl < 2; ++hl)
+                    for (int dh = 0; dh < 2; ++dh) {
+                        tma_load_3d(sb + kOffQ + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_Q),
+                                    dh * 64, qb * 64, hq0 + hl);
+                        tma_load_3d(sb + kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(B_Q),
+                                    dh * 64, qb * 64, hq0 + hl);
+                    }
+            }
+            int issued = 0;
+            for (int j = 0; j < n; ++j) {
+                const int s = j % slots;
+                if (j >= slots &&
+                    !mbar_wait(bar(empty + s), ((j / slots) - 1) & 1, abort_flag, a.status))
+                    break;
+                mbar_expect_tx(bar(full + s), kTile64);
+                for (int dh = 0; dh < 2; ++dh)
+                    tma_load_3d(ring + s * kTile64 + dh * kHalf64, map, bar(full + s), dh * 64,
+                                list[j] * 64, bg);
+                issued = j + 1;
+            }
+            if (is_k) mbar_wait_drain(bar(B_Q), 0);
+            for (int j = issued - slots; j < issued; ++j)
+                if (j >= 0) mbar_wait_drain(bar(full + j % slots), (j / slots) & 1);
+        }
+    } else if (warp == 9) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0 && n > 0) {
+            constexpr uint32_t id_s = idesc_bf16(128, 64, false);
+            constexpr uint32_t id_dq = idesc_bf16(128, 128, true);
+            bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
+            tc_fence_after();
+            int ns = 0, nd = 0;
+            uint64_t t0 = global_ns();
+            while (ok && nd < n) {
+                bool progressed = false;
+                if (ns < n && ns <= nd + 1 &&
+                    mbar_try_wait(bar(B_KFULL + ns % kKSlots), (ns / kKSlots) & 1) &&
+                    mbar_try_wait(bar(B_VFULL + ns % kVSlots), (ns / kVSlots) & 1)) {
+                    tc_fence_after();
+                    const uint32_t kb = sb + kOffK + (ns % kKSlots) * kTile64;
+                    const uint32_t vb = sb + kOffV + (ns % kVSlots) * kTile64;
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t off = (uint32_t)((ks & 3) * 32);
+                        mma_ss(tmem + col_s(ns & 1),
+                               sdesc_sw128(sb + kOffQ + (ks >> 2) * kHalf128 + off, 16, 1024),
+                               sdesc_sw128(kb + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
+                               ks > 0 ? 1u : 0u);
+                    }
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t off = (uint32_t)((ks & 3) * 32);
+                        mma_ss(tmem + col_dp(ns & 1),
+                               sdesc_sw128(sb + kOffDO + (ks >> 2) * kHalf128 + off, 16, 1024),
+                               sdesc_sw128(vb + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
+                               ks > 0 ? 1u : 0u);
+                    }
+                    mma_commit(bar(B_SPFULL + (ns & 1)));
+                    mma_commit(bar(B_VEMPTY + ns % kVSlots));
+                    ++ns;
+                    progressed = true;
+                }
+                if (nd < ns && mbar_try_wait(bar(B_DSFULL + (nd & 1)), (nd >> 1) & 1)) {
+                    tc_fence_after();
+                    const uint32_t kb = sb + kOffK + (nd % kKSlots) * kTile64;
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_ts(tmem + kColDQ, tmem + col_ds(nd & 1) + ks * 8,
+                               sdesc_sw128(kb + ks * 2048, kHalf64, 1024), id_dq,
+                               (nd > 0 || ks > 0) ? 1u : 0u);
+                    mma_commit(bar(B_KEMPTY + nd % kKSlots));
+                    if (nd == n - 1) mma_commit(bar(B_FINAL));
+                    ++nd;
+                    progressed = true;
+                }
+                if (progressed) {
+                    t0 = global_ns();
+                } else if (*abort_flag) {
+                    ok = false;
+                } else if (global_ns() - t0 > kWaitLimitNs) {
+                    *abort_flag = 1;
+                    atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
+                    ok = false;
+                }
+            }
+            mma_commit(bar(B_DRAIN));
+            mbar_wait_drain(bar(B_DRAIN), 0);
+        }
+    } else {
+        // ------------------------------------------------ elementwise (8 warps)
+        const int row = (warp & 3) * 32 + lane;  // TMEM lane
+        const int half = warp >> 2;              // key half for dS, column half for dQ
+        const int tok = row & 63, hl = row >> 6;
+        const int i = qb * 64 + tok;
+        const bool valid = i < a.L;
+        const size_t ridx = (size_t)(hq0 + hl) * a.L + (valid ? i : 0);
+        const float neg_lse2 = valid ? -a.lse[ridx] * kLog2e : -INFINITY;
+        const float dlt = valid ? a.delta[ridx] : 0.f;
+        const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+        bool ok = true;
+        for (int j = 0; j < n; ++j) {
+            const int buf = j & 1;
+            ok = mbar_wait(bar(B_SPFULL + buf), (j >> 1) & 1, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            tc_fence_after();
+            uint32_t sv[32], dp[32];
+            tmem_ld32(lane_base + col_s(buf) + 32 * half, sv);
+            tmem_ld32(lane_base + col_dp(buf) + 32 * half, dp);
+            const bool diag = list[j] == qb;
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                float ds[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int key = 32 * half + 2 * c + e;
+                    float p = ex2_approx(fmaf(__uint_as_float(sv[2 * c + e]), a.scale_log2, neg_lse2));
+                    if (diag && key > tok) p = 0.f;
+                    ds[e] = p * (__uint_as_float(dp[2 * c + e]) - dlt);
+                }
+                sv[c] = pack2_bf16(ds[0], ds[1]);
+            }
+            tmem_st16(lane_base + col_ds(buf) + 16 * half, sv);
+            tc_fence_before();
+            mbar_arrive(bar(B_DSFULL + buf));
+        }
+        if (ok && n > 0) {
+            ok = mbar_wait(bar(B_FINAL), 0, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+        }
+        if (ok) {
+            tc_fence_after();
+            uint8_t* sq = smem + kOffQ + half * kHalf128;  // this warp's 64 columns = one d-half
+#pragma unroll
+            for (int c2 = 0; c2 < 2; ++c2) {
+                uint32_t o[32];
+                if (n > 0) {
+                    tmem_ld32(lane_base + kColDQ + 64 * half + 32 * c2, o);
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) o[c] = 0u;
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    uint4 v;
+                    const float s = a.sm_scale;
+                    v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * s, __uint_as_float(o[8 * q + 1]) * s);
+                    v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * s, __uint_as_float(o[8 * q + 3]) * s);
+                    v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * s, __uint_as_float(o[8 * q + 5]) * s);
+                    v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * s, __uint_as_float(o[8 * q + 7]) * s);
+                    *reinterpret_cast<uint4*>(sq + sw_off(row, c2 * 4 + q)) = v;
+                }
+            }
+            fence_proxy_async_smem();
+        }
+        named_barrier(1, 256);
+        if (threadIdx.x == 0 && ok) {
+            for (int h2 = 0; h2 < 2; ++h2)
+                for (int dh = 0; dh < 2; ++dh)
+                    tma_store_3d(&tmdQ, sb + kOffQ + dh * kHalf128 + h2 * kHalf64, dh * 64, qb * 64,
+                                 hq0 + h2);
+            tma_store_commit();
+            tma_store_wait_read();
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// ============================================================== dK / dV
+namespace kv {
+constexpr int kOffK = 0;
+constexpr int kOffV = kOffK + kTile64;
+constexpr int kOffStage = kOffV + kTile64;      // 2 x (Q 32 KB, dO 32 KB)
+constexpr int kStage = 2 * kTile128;
+constexpr int kOffP = kOffStage + 2 * kStage;   // P  [128 rows][64 keys] bf16
+constexpr int kOffDS = kOffP + kHalf128;        // dS [128 rows][64 keys] bf16
+constexpr int kOffBar = kOffDS + kHalf128;
+constexpr int B_KV = 0, B_QFULL = 1, B_QEMPTY = 3, B_SPFULL = 5, B_PDSFULL = 7, B_PDSFREE = 8,
+              B_FINAL = 9, B_DRAIN = 10, kNumBars = 11;
+constexpr int kOffMisc = kOffBar + kNumBars * 8;
+constexpr int kThreads = 320;  // 8 elementwise warps, producer, MMA
+constexpr uint32_t kColDV = 256, kColDK = 320;
+__device__ __forceinline__ uint32_t col_s(int b) { return 128u * (uint32_t)b; }
+__device__ __forceinline__ uint32_t col_dp(int b) { return 64u + 128u * (uint32_t)b; }
+constexpr size_t kSmem = 1024 + (size_t)kOffMisc + 16;
+}  // namespace kv
+
+struct KvArgs {
+    const float* lse;
+    const float* delta;
+    const BwdTInfo* tinfo;
+    const int32_t* qlist;
+    const int2* work;
+    const int32_t* nwork;
+    float* partial;
+    int* status;
+    int Hq, Hkv, L, NQB, topk, work_max, slot_max;
+    float scale_log2, sm_scale;
+};
+
+__global__ void __launch_bounds__(kv::kThreads, 1)
+dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+               const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
+               const __grid_constant__ CUtensorMap tmdK, const __grid_constant__ CUtensorMap tmdV,
+               const KvArgs a) {
+    using namespace kv;
+    const int bg = blockIdx.y;
+    if ((int)blockIdx.x >= a.nwork[bg]) return;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    const uint32_t sb = smem_u32(smem);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = bg / a.Hkv, g = bg % a.Hkv;
+    const int2 wi = a.work[(size_t)bg * a.work_max + blockIdx.x];
+    const int t = wi.x, chunk = wi.y;
+    const BwdTInfo info = a.tinfo[(size_t)bg * a.NQB + t];
+    const int q_begin = chunk * kBwdChunk;
+    const int n_it = max(0, min(info.n, q_begin + kBwdChunk) - q_begin);
+    const int32_t* ql = a.qlist + (size_t)bg * a.NQB * a.topk + info.off + q_begin;
+    auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
+    const int hq0 = b * a.Hq + g * 2;
+
+    if (threadIdx.x == 0) {
+        mbar_init(bar(B_KV), 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(bar(B_QFULL + s), 1);
+            mbar_init(bar(B_QEMPTY + s), 1);
+            mbar_init(bar(B_SPFULL + s), 1);
+        }
+        mbar_init(bar(B_PDSFULL), 256);
+        mbar_init(bar(B_PDSFREE), 1);
+        mbar_init(bar(B_FINAL), 1);
+        mbar_init(bar(B_DRAIN), 1);
+        fence_barrier_init();
+        *abort_flag = 0;
+    }
+    if (warp == 9) {
+        tmem_alloc(sb + kOffMisc, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
+
+    if (warp == 8) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0 && n_it > 0) {
+            prefetch_tmap(&tmQ);
+            prefetch_tmap(&tmdO);
+            mbar_expect_tx(bar(B_KV), 2 * kTile64);
+            for (int dh = 0; dh < 2; ++dh) {
+                tma_load_3d(sb + kOffK + dh * kHalf64, &tmK, bar(B_KV), dh * 64, t * 64, bg);
+                tma_load_3d(sb + kOffV + dh * kHalf64, &tmV, bar(B_KV), dh * 64, t * 64, bg);
+            }
+            int issued = 0;
+            for (int i = 0; i < n_it; ++i) {
+                const int s = i & 1;
+                if (i >= 2 && !mbar_wait(bar(B_QEMPTY + s), ((i >> 1) - 1) & 1, abort_flag, a.status))
+                    break;
+                const int qb = ql[i];
+                const uint32_t st = sb + kOffStage + s * kStage;
+                mbar_expect_tx(bar(B_QFULL + s), kStage);
+                for (int hl = 0; hl < 2; ++hl)
+                    for (int dh = 0; dh < 2; ++dh) {
+                        tma_load_3d(st + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_QFULL + s),
+                                    dh * 64, qb * 64, hq0 + hl);
+                        tma_load_3d(st + kTile128 + dh * kHalf128 + hl * kHalf64, &tmdO,
+                                    bar(B_QFULL + s), dh * 64, qb * 64, hq0 + hl);
+                    }
+                issued = i + 1;
+            }
+            mbar_wait_drain(bar(B_KV), 0);
+            for (int i = issued - 2; i < issued; ++i)
+                if (i >= 0) mbar_wait_drain(bar(B_QFULL + (i & 1)), (i >> 1) & 1);
+        }
+    } else if (warp == 9) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0 && n_it > 0) {
+            constexpr uint32_t id_s = idesc_bf16(128, 64, false);
+            constexpr uint32_t id_t = idesc_bf16(128, 64, true, true);  // A and B MN-major
+            bool ok = mbar_wait(bar(B_KV), 0, abort_flag, a.status);
+            tc_fence_after();
+            int ns = 0, nv = 0;
+            uint64_t t0 = global_ns();
+            while (ok && nv < n_it) {
+                bool progressed = false;
+                if (ns < n_it && ns <= nv + 1 &&
+                    mbar_try_wait(bar(B_QFULL + (ns & 1)), (ns >> 1) & 1)) {
+                    tc_fence_after();
+                    const uint32_t st = sb + kOffStage + (ns & 1) * kStage;
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t off = (uint32_t)((ks & 3) * 32);
+                        mma_ss(tmem + col_s(ns & 1),
+                               sdesc_sw128(st + (ks >> 2) * kHalf128 + off, 16, 1024),
+                               sdesc_sw128(sb + kOffK + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
+                               ks > 0 ? 1u : 0u);
+                    }
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t off = (uint32_t)((ks & 3) * 32);
+                        mma_ss(tmem + col_dp(ns & 1),
+                               sdesc_sw128(st + kTile128 + (ks >> 2) * kHalf128 + off, 16, 1024),
+                               sdesc_sw128(sb + kOffV + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
+                               ks > 0 ? 1u : 0u);
+                    }
+                    mma_commit(bar(B_SPFULL + (ns & 1)));
+                    ++ns;
+                    progressed = true;
+                }
+                if (nv < ns && mbar_try_wait(bar(B_PDSFULL), nv & 1)) {
+                    tc_fence_after();
+                    const uint32_t st = sb + kOffStage + (nv & 1) * kStage;
+                    // K dimension = the 128 stacked query rows, 16 per MMA
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(tmem + kColDV, sdesc_sw128(st + kTile128 + ks * 2048, kHalf128, 1024),
+                               sdesc_sw128(sb + kOffP + ks * 2048, kHalf128, 1024), id_t,
+                               (nv > 0 || ks > 0) ? 1u : 0u);
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(tmem + kColDK, sdesc_sw128(st + ks * 2048, kHalf128, 1024),
+                               sdesc_sw128(sb + kOffDS + ks * 2048, kHalf128, 1024), id_t,
+                               (nv > 0 || ks > 0) ? 1u : 0u);
+                    mma_commit(bar(B_PDSFREE));
+                    mma_commit(bar(B_QEMPTY + (nv & 1)));
+                    if (nv == n_it - 1) mma_commit(bar(B_FINAL));
+                    ++nv;
+                    progressed = true;
+                }
+                if (progressed) {
+                    t0 = global_ns();
+                } else if (*abort_flag) {
+                    ok = false;
+                } else if (global_ns() - t0 > kWaitLimitNs) {
+                    *abort_flag = 1;
+                    atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
+                    ok = false;
+                }
+            }
+            mma_commit(bar(B_DRAIN));
+            mbar_wait_drain(bar(B_DRAIN), 0);
+        }
+    } else {
+        // ------------------------------------------------ elementwise (8 warps)
+        const int row = (warp & 3) * 32 + lane;  // TMEM lane: query row (head hl, token tok)
+        const int kh = warp >> 2;                // keys [32 kh, 32 kh + 32)
+        const int tok = row & 63, hl = row >> 6;
+        const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+        const size_t hoff = (size_t)(hq0 + hl) * a.L;
+        bool ok = true;
+        for (int it = 0; it < n_it; ++it) {
+            const int qb = ql[it];
+            const int i = qb * 64 + tok;
+            const bool valid = i < a.L;
+            const float neg_lse2 = valid ? -a.lse[hoff + i] * kLog2e : -INFINITY;
+            const float dlt = valid ? a.delta[hoff + i] : 0.f;
+            const int buf = it & 1;
+            ok = mbar_wait(bar(B_SPFULL + buf), (it >> 1) & 1, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            tc_fence_after();
+            uint32_t sv[32], dp[32];
+            tmem_ld32(lane_base + col_s(buf) + 32 * kh, sv);
+            tmem_ld32(lane_base + col_dp(buf) + 32 * kh, dp);
+            const bool diag = qb == t;
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                float p[2], ds[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int key = 32 * kh + 2 * c + e;
+                    float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + e]), a.scale_log2, neg_lse2));
+                    if (diag && key > tok) pv = 0.f;
+                    p[e] = pv;
+                    ds[e] = pv * (__uint_as_float(dp[2 * c + e]) - dlt);
+                }
+                sv[c] = pack2_bf16(p[0], p[1]);
+                dp[c] = pack2_bf16(ds[0], ds[1]);
+            }
+            tc_fence_before();
+            if (it > 0) {  // the previous dV/dK MMAs must have read P and dS
+                ok = mbar_wait(bar(B_PDSFREE), (it - 1) & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t off = sw_off(row, 4 * kh + q);
+                *reinterpret_cast<uint4*>(smem + kOffP + off) =
+                    make_uint4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
+                *reinterpret_cast<uint4*>(smem + kOffDS + off) =
+                    make_uint4(dp[4 * q], dp[4 * q + 1], dp[4 * q + 2], dp[4 * q + 3]);
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(bar(B_PDSFULL));
+        }
+        if (ok && n_it > 0) {
+            ok = mbar_wait(bar(B_FINAL), 0, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+        }
+        // dV^T / dK^T: lane = head-dimension index d, columns = keys [32 kh, 32 kh + 32)
+        const int d = row;
+        uint32_t v[32], k[32];
+        if (ok && n_it > 0) {
+            tc_fence_after();
+            tmem_ld32(lane_base + kColDV + 32 * kh, v);
+            tmem_ld32(lane_base + kColDK + 32 * kh, k);
+        } else {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) { v[c] = 0u; k[c] = 0u; }
+        }
+        if (info.nch > 1) {
+            if (ok && info.slot >= 0) {
+                float* pk = a.partial + ((size_t)bg * a.slot_max + info.slot + chunk) * 2 * 64 * 128;
+                float* pv = pk + 64 * 128;
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    const int key = 32 * kh + c;
+                    pk[key * 128 + d] = __uint_as_float(k[c]) * a.sm_scale;
+                    pv[key * 128 + d] = __uint_as_float(v[c]);
+                }
+            }
+        } else if (ok) {
+            // bf16 tiles [64 keys][128 d] in the swizzled layout (stage-0 Q and dO regions)
+            uint8_t* tv = smem + kOffStage;
+            uint8_t* tk = smem + kOffStage + kTile128;
+            const int dh = d >> 6, dc = (d & 63) >> 3, de = d & 7;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                const int key = 32 * kh + c;
+                const uint32_t off = dh * kHalf64 + sw_off(key, dc) + de * 2;
+                *reinterpret_cast<__nv_bfloat16*>(tv + off) = __float2bfloat16_rn(__uint_as_float(v[c]));
+                *reinterpret_cast<__nv_bfloat16*>(tk + off) =
+                    __float2bfloat16_rn(__uint_as_float(k[c]) * a.sm_scale);
+            }
+            fence_proxy_async_smem();
+        }
+        named_barrier(1, 256);
+        if (threadIdx.x == 0 && ok && info.nch <= 1) {
+            for (int dh = 0; dh < 2; ++dh) {
+                tma_store_3d(&tmdV, sb + kOffStage + dh * kHalf64, dh * 64, t * 64, bg);
+                tma_store_3d(&tmdK, sb + kOffStage + kTile128 + dh * kHalf64, dh * 64, t * 64, bg);
+            }
+            tma_store_commit();
+            tma_store_wait_read();
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* dO,
+                         const float* lse, const float* delta, const int32_t* idx,
+                         const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                         void* dQ, int* status, cudaStream_t st) {
+    const int NQB = (s.L + 63) / 64;
+    CUtensorMap tq, tk, tv, tdo, tdq;
+    const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
+    if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) || !make_tmap_bf16_rows128(&tk, K, s.L, pk, 64) ||
+        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64) ||
+        !make_tmap_bf16_rows128(&tdq, dQ, s.L, pq, 64))
+        return cudaErrorInvalidValue;
+    const size_t smem = dq::smem_bytes(topk);
+    cudaError_t e =
+        cudaFuncSetAttribute(dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    DqArgs args{idx, cnt, lse, delta, status, s.Hq, s.Hkv, s.L, NQB, topk, sm_scale * kLog2e,
+                sm_scale};
+    ProfScope prof(K_BWD_DQ, st);
+    dq_tc_kernel<<<(unsigned)((long long)s.B * s.Hkv * NQB), dq::kThreads, smem, st>>>(
+        tq, tk, tv, tdo, tdq, args);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
+                           const float* lse, const float* delta, const BwdTInfo* tinfo,
+                           const int32_t* qlist, const int2* work, const int32_t* nwork,
+                           const phsa_shape& s, int topk, int work_max, int slot_max,
+                           float sm_scale, void* dK, void* dV, float* partial, int* status,
+                           cudaStream_t st) {
+    const int NQB = (s.L + 63) / 64;
+    CUtensorMap tq, tk, tv, tdo, tdk, tdv;
+    const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
+    if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) || !make_tmap_bf16_rows128(&tk, K, s.L, pk, 64) ||
+        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64) ||
+        !make_tmap_bf16_rows128(&tdk, dK, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdv, dV, s.L, pk, 64))
+        return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(dkdv_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kv::kSmem);
+    if (e != cudaSuccess) return e;
+    KvArgs args{lse, delta, tinfo, qlist, work, nwork, partial, status, s.Hq, s.Hkv, s.L, NQB,
+                topk, work_max, slot_max, sm_scale * kLog2e, sm_scale};
+    ProfScope prof(K_BWD_DKDV, st);
+    dkdv_tc_kernel<<<dim3(work_max, s.B * s.Hkv), kv::kThreads, kv::kSmem, st>>>(tq, tk, tv, tdo,
+                                                                                 tdk, tdv, args);
+    return cudaGetLastError();
+}
+
+}  // namespace phsa
