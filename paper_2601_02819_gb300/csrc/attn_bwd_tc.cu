@@ -1,14 +1,16 @@
 // Stage (c) backward on the tensor cores (tcgen05 + TMEM + TMA), for GQA
 // groups of two query heads, so that every MMA has M = 128.
 //
-// dq_tc_kernel: one CTA per (query block qb, KV head g), 352 threads.
-//   For every selected block j (K_j, V_j gathered by TMA into 4- and 3-slot rings):
-//     S_j  = Q K_j^T      (M128 N64 K128, A = Q, B = K_j, both K-major)
-//     dP_j = dO V_j^T     (M128 N64 K128)
-//     dS_j = P_j (dP_j - Delta), P_j = exp(S_j * scale - lse)   (8 warps, TMEM)
-//     dQ  += dS_j K_j     (M128 N128 K64, A = dS_j in TMEM, B = K_j MN-major)
-//   S/dP are double-buffered in TMEM so the tensor core computes block j+1
-//   while the elementwise warps work on block j. dQ * scale -> TMA store.
+// dq_tc_kernel: one CTA per (query block qb, KV head g), 352 threads. The
+//   selected blocks are taken in pairs (an odd count pairs the last block with
+//   a masked copy of itself); each pair's K and V tiles (128 keys) are gathered
+//   by TMA into 3- and 2-slot rings. Per pair p:
+//     S_p  = Q Kp^T       (M128 N128 K128)
+//     dP_p = dO Vp^T      (M128 N128 K128)
+//     dS_p = P_p (dP_p - Delta), P_p = exp(S_p * scale - lse)   (8 warps, TMEM)
+//     dQ  += dS_p Kp      (M128 N128 K128, A = dS_p in TMEM, B = Kp MN-major)
+//   S is double-buffered in TMEM, so S_{p+1} runs while the elementwise warps
+//   work on pair p. dQ * scale -> TMA store.
 //
 // dkdv_tc_kernel: one CTA per work item (KV block t, chunk of <= 32 query
 //   blocks that selected t), 320 threads. K_t and V_t stay in shared memory;
@@ -45,24 +47,26 @@ __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
 }
 
 // ============================================================== dQ
+// Blocks are processed in pairs, so the S and dP MMAs have N = 128 keys.
 namespace dq {
-constexpr int kKSlots = 4, kVSlots = 3;
+constexpr int kKSlots = 3, kVSlots = 2;        // ring slots, one block pair each
+constexpr int kPair = 2 * kTile64;              // two 64 x 128 blocks (32 KB)
 constexpr int kOffQ = 0;
 constexpr int kOffDO = kOffQ + kTile128;
 constexpr int kOffK = kOffDO + kTile128;
-constexpr int kOffV = kOffK + kKSlots * kTile64;
-constexpr int kOffBar = kOffV + kVSlots * kTile64;
+constexpr int kOffV = kOffK + kKSlots * kPair;
+constexpr int kOffBar = kOffV + kVSlots * kPair;
 constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = B_KFULL + kKSlots, B_VFULL = B_KEMPTY + kKSlots,
               B_VEMPTY = B_VFULL + kVSlots, B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2,
-              B_FINAL = B_DSFULL + 2, B_DRAIN = B_FINAL + 1, kNumBars = B_DRAIN + 1;
+              B_FINAL = B_DSFULL + 1, B_DRAIN = B_FINAL + 1, kNumBars = B_DRAIN + 1;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kOffList = kOffMisc + 16;
 constexpr int kThreads = 352;  // 8 elementwise warps, K/Q/dO producer, MMA, V producer
-constexpr uint32_t kColDQ = 0;
+// TMEM: dQ [0,128), S of pair buffer b at [128 + 128b, +128), dP [384, 512).
+// dS of key half h overwrites S columns [64h, 64h + 32) (read by the same thread).
+constexpr uint32_t kColDQ = 0, kColDP = 384;
 __device__ __forceinline__ uint32_t col_s(int b) { return 128u + 128u * (uint32_t)b; }
-__device__ __forceinline__ uint32_t col_dp(int b) { return 192u + 128u * (uint32_t)b; }
-__device__ __forceinline__ uint32_t col_ds(int b) { return 384u + 32u * (uint32_t)b; }
-constexpr size_t smem_bytes(int topk) { return 1024 + (size_t)kOffList + (size_t)(topk + 1) * 4; }
+constexpr size_t smem_bytes(int topk) { return 1024 + (size_t)kOffList + (size_t)(topk + 2) * 4; }
 }  // namespace dq
 
 struct DqArgs {
@@ -105,16 +109,16 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             mbar_init(bar(B_VFULL + s), 1);
             mbar_init(bar(B_VEMPTY + s), 1);
         }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(bar(B_SPFULL + i), 1);
-            mbar_init(bar(B_DSFULL + i), 256);
-        }
+        mbar_init(bar(B_SPFULL), 1);
+        mbar_init(bar(B_SPFULL + 1), 1);
+        mbar_init(bar(B_DSFULL), 256);
         mbar_init(bar(B_FINAL), 1);
         mbar_init(bar(B_DRAIN), 1);
         fence_barrier_init();
         *abort_flag = 0;
-        reinterpret_cast<int*>(smem + kOffMisc)[2] =
-            compact_block_list(a.idx + lu * a.topk, a.cnt[lu], a.topk, qb, list, nullptr);
+        const int n = compact_block_list(a.idx + lu * a.topk, a.cnt[lu], a.topk, qb, list, nullptr);
+        list[n] = n > 0 ? list[n - 1] : 0;  // an odd count pairs the last block with itself
+        reinterpret_cast<int*>(smem + kOffMisc)[2] = n;
     }
     if (warp == 9) {
         tmem_alloc(sb + kOffMisc, kTmemCols);
@@ -125,9 +129,10 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
     const int n = reinterpret_cast<volatile int*>(smem + kOffMisc)[2];
+    const int np = (n + 1) >> 1;  // block pairs
 
     if (warp == 8 || warp == 10) {
-        // ------------------------------------------------ TMA producers
+        // ------------------------------------------------ TMA producers (pairs of blocks)
         if (lane == 0 && n > 0) {
             const bool is_k = warp == 8;
             const CUtensorMap* map = is_k ? &tmK : &tmV;
@@ -146,80 +151,86 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                     }
             }
             int issued = 0;
-            for (int j = 0; j < n; ++j) {
-                const int s = j % slots;
-                if (j >= slots &&
-                    !mbar_wait(bar(empty + s), ((j / slots) - 1) & 1, abort_flag, a.status))
+            for (int p = 0; p < np; ++p) {
+                const int s = p % slots;
+                if (p >= slots &&
+                    !mbar_wait(bar(empty + s), ((p / slots) - 1) & 1, abort_flag, a.status))
                     break;
-                mbar_expect_tx(bar(full + s), kTile64);
-                for (int dh = 0; dh < 2; ++dh)
-                    tma_load_3d(ring + s * kTile64 + dh * kHalf64, map, bar(full + s), dh * 64,
-                                list[j] * 64, bg);
-                issued = j + 1;
+                mbar_expect_tx(bar(full + s), kPair);
+                // slot layout: [d half][block of the pair][64 rows][64 columns]
+                for (int e = 0; e < 2; ++e)
+                    for (int dh = 0; dh < 2; ++dh)
+                        tma_load_3d(ring + s * kPair + dh * kHalf128 + e * kHalf64, map,
+                                    bar(full + s), dh * 64, list[2 * p + e] * 64, bg);
+                issued = p + 1;
             }
             if (is_k) mbar_wait_drain(bar(B_Q), 0);
-            for (int j = issued - slots; j < issued; ++j)
-                if (j >= 0) mbar_wait_drain(bar(full + j % slots), (j / slots) & 1);
+            for (int p = issued - slots; p < issued; ++p)
+                if (p >= 0) mbar_wait_drain(bar(full + p % slots), (p / slots) & 1);
         }
     } else if (warp == 9) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0 && n > 0) {
-            constexpr uint32_t id_s = idesc_bf16(128, 64, false);
+            constexpr uint32_t id_s = idesc_bf16(128, 128, false);
             constexpr uint32_t id_dq = idesc_bf16(128, 128, true);
             bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
             tc_fence_after();
-            int ns = 0, nd = 0;
-            uint64_t t0 = global_ns();
-            while (ok && nd < n) {
-                bool progressed = false;
-                if (ns < n && ns <= nd + 1 &&
-                    mbar_try_wait(bar(B_KFULL + ns % kKSlots), (ns / kKSlots) & 1) &&
-                    mbar_try_wait(bar(B_VFULL + ns % kVSlots), (ns / kVSlots) & 1)) {
-                    tc_fence_after();
-                    const uint32_t kb = sb + kOffK + (ns % kKSlots) * kTile64;
-                    const uint32_t vb = sb + kOffV + (ns % kVSlots) * kTile64;
+            auto issue_s = [&](int p) {  // S_p = Q Kpair_p^T into buffer p & 1
+                const uint32_t kb = sb + kOffK + (p % kKSlots) * kPair;
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (uint32_t)((ks & 3) * 32);
-                        mma_ss(tmem + col_s(ns & 1),
-                               sdesc_sw128(sb + kOffQ + (ks >> 2) * kHalf128 + off, 16, 1024),
-                               sdesc_sw128(kb + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
-                               ks > 0 ? 1u : 0u);
-                    }
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (uint32_t)((ks & 3) * 32);
-                        mma_ss(tmem + col_dp(ns & 1),
-                               sdesc_sw128(sb + kOffDO + (ks >> 2) * kHalf128 + off, 16, 1024),
-                               sdesc_sw128(vb + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
-                               ks > 0 ? 1u : 0u);
-                    }
-                    mma_commit(bar(B_SPFULL + (ns & 1)));
-                    mma_commit(bar(B_VEMPTY + ns % kVSlots));
-                    ++ns;
-                    progressed = true;
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
+                    mma_ss(tmem + col_s(p & 1), sdesc_sw128(sb + kOffQ + off, 16, 1024),
+                           sdesc_sw128(kb + off, 16, 1024), id_s, ks > 0 ? 1u : 0u);
                 }
-                if (nd < ns && mbar_try_wait(bar(B_DSFULL + (nd & 1)), (nd >> 1) & 1)) {
-                    tc_fence_after();
-                    const uint32_t kb = sb + kOffK + (nd % kKSlots) * kTile64;
+            };
+            auto issue_dp = [&](int p) {  // dP_p = dO Vpair_p^T; releases the V slot
+                const uint32_t vb = sb + kOffV + (p % kVSlots) * kPair;
 #pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_ts(tmem + kColDQ, tmem + col_ds(nd & 1) + ks * 8,
-                               sdesc_sw128(kb + ks * 2048, kHalf64, 1024), id_dq,
-                               (nd > 0 || ks > 0) ? 1u : 0u);
-                    mma_commit(bar(B_KEMPTY + nd % kKSlots));
-                    if (nd == n - 1) mma_commit(bar(B_FINAL));
-                    ++nd;
-                    progressed = true;
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
+                    mma_ss(tmem + kColDP, sdesc_sw128(sb + kOffDO + off, 16, 1024),
+                           sdesc_sw128(vb + off, 16, 1024), id_s, ks > 0 ? 1u : 0u);
                 }
-                if (progressed) {
-                    t0 = global_ns();
-                } else if (*abort_flag) {
-                    ok = false;
-                } else if (global_ns() - t0 > kWaitLimitNs) {
-                    *abort_flag = 1;
-                    atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
-                    ok = false;
+                mma_commit(bar(B_SPFULL + (p & 1)));  // S_p and dP_p are both complete
+                mma_commit(bar(B_VEMPTY + p % kVSlots));
+            };
+            // Order: S_0 dP_0 S_1 | dS_0 -> dQ_0 dP_1 S_2 | dS_1 -> dQ_1 dP_2 S_3 | ...
+            // (dP has one buffer: dP_{p+1} follows the elementwise pass over dP_p.)
+            ok = ok && mbar_wait(bar(B_KFULL), 0, abort_flag, a.status) &&
+                 mbar_wait(bar(B_VFULL), 0, abort_flag, a.status);
+            if (ok) {
+                tc_fence_after();
+                issue_s(0);
+                issue_dp(0);
+            }
+            for (int p = 0; ok && p < np; ++p) {
+                if (p + 1 < np) {  // S_{p+1} overlaps the elementwise pass over pair p
+                    ok = mbar_wait(bar(B_KFULL + (p + 1) % kKSlots), ((p + 1) / kKSlots) & 1,
+                                   abort_flag, a.status);
+                    if (!ok) break;
+                    tc_fence_after();
+                    issue_s(p + 1);
+                }
+                ok = mbar_wait(bar(B_DSFULL), p & 1, abort_flag, a.status);
+                if (!ok) break;
+                tc_fence_after();
+                // dQ += dS_p Kpair_p: A = dS (TMEM), B = the K pair read MN-major
+                const uint32_t kb = sb + kOffK + (p % kKSlots) * kPair;
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ts(tmem + kColDQ, tmem + col_s(p & 1) + (ks >> 2) * 64 + (ks & 3) * 8,
+                           sdesc_sw128(kb + ks * 2048, kHalf128, 1024), id_dq,
+                           (p > 0 || ks > 0) ? 1u : 0u);
+                mma_commit(bar(B_KEMPTY + p % kKSlots));
+                if (p == np - 1) {
+                    mma_commit(bar(B_FINAL));
+                } else {
+                    ok = mbar_wait(bar(B_VFULL + (p + 1) % kVSlots), ((p + 1) / kVSlots) & 1,
+                                   abort_flag, a.status);
+                    if (!ok) break;
+                    tc_fence_after();
+                    issue_dp(p + 1);
                 }
             }
             mma_commit(bar(B_DRAIN));
@@ -228,7 +239,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
     } else {
         // ------------------------------------------------ elementwise (8 warps)
         const int row = (warp & 3) * 32 + lane;  // TMEM lane
-        const int half = warp >> 2;              // key half for dS, column half for dQ
+        const int half = warp >> 2;              // block of the pair (64 keys); d half for dQ
         const int tok = row & 63, hl = row >> 6;
         const int i = qb * 64 + tok;
         const bool valid = i < a.L;
@@ -237,31 +248,37 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         const float dlt = valid ? a.delta[ridx] : 0.f;
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         bool ok = true;
-        for (int j = 0; j < n; ++j) {
-            const int buf = j & 1;
-            ok = mbar_wait(bar(B_SPFULL + buf), (j >> 1) & 1, abort_flag, a.status);
+        for (int p = 0; p < np; ++p) {
+            const int buf = p & 1;
+            ok = mbar_wait(bar(B_SPFULL + buf), (p >> 1) & 1, abort_flag, a.status);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             tc_fence_after();
-            uint32_t sv[32], dp[32];
-            tmem_ld32(lane_base + col_s(buf) + 32 * half, sv);
-            tmem_ld32(lane_base + col_dp(buf) + 32 * half, dp);
-            const bool diag = list[j] == qb;
+            const int e = 2 * p + half;       // this half's block in the list
+            const bool live = e < n;          // false: the duplicate of an odd count
+            const bool diag = list[e] == qb;
+#pragma unroll 1
+            for (int q = 0; q < 2; ++q) {     // two 32-key chunks of this half
+                uint32_t sv[32], dp[32];
+                tmem_ld32(lane_base + col_s(buf) + 64 * half + 32 * q, sv);
+                tmem_ld32(lane_base + kColDP + 64 * half + 32 * q, dp);
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
-                float ds[2];
+                for (int c = 0; c < 16; ++c) {
+                    float ds[2];
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int key = 32 * half + 2 * c + e;
-                    float p = ex2_approx(fmaf(__uint_as_float(sv[2 * c + e]), a.scale_log2, neg_lse2));
-                    if (diag && key > tok) p = 0.f;
-                    ds[e] = p * (__uint_as_float(dp[2 * c + e]) - dlt);
+                    for (int x = 0; x < 2; ++x) {
+                        const int key = 32 * q + 2 * c + x;
+                        float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + x]), a.scale_log2, neg_lse2));
+                        if (!live || (diag && key > tok)) pv = 0.f;
+                        ds[x] = pv * (__uint_as_float(dp[2 * c + x]) - dlt);
+                    }
+                    sv[c] = pack2_bf16(ds[0], ds[1]);
                 }
-                sv[c] = pack2_bf16(ds[0], ds[1]);
+                // dS columns [64 half + 16 q, +16): inside this thread's own S range
+                tmem_st16(lane_base + col_s(buf) + 64 * half + 16 * q, sv);
             }
-            tmem_st16(lane_base + col_ds(buf) + 16 * half, sv);
             tc_fence_before();
-            mbar_arrive(bar(B_DSFULL + buf));
+            mbar_arrive(bar(B_DSFULL));
         }
         if (ok && n > 0) {
             ok = mbar_wait(bar(B_FINAL), 0, abort_flag, a.status);
@@ -428,11 +445,11 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             bool ok = mbar_wait(bar(B_KV), 0, abort_flag, a.status);
             tc_fence_after();
             int ns = 0, nv = 0;
-            uint64_t t0 = global_ns();
+            Deadline dl;
             while (ok && nv < n_it) {
                 bool progressed = false;
                 if (ns < n_it && ns <= nv + 1 &&
-                    mbar_try_wait(bar(B_QFULL + (ns & 1)), (ns >> 1) & 1)) {
+                    mbar_test_wait(bar(B_QFULL + (ns & 1)), (ns >> 1) & 1)) {
                     tc_fence_after();
                     const uint32_t st = sb + kOffStage + (ns & 1) * kStage;
 #pragma unroll
@@ -455,7 +472,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     ++ns;
                     progressed = true;
                 }
-                if (nv < ns && mbar_try_wait(bar(B_PDSFULL), nv & 1)) {
+                if (nv < ns && mbar_test_wait(bar(B_PDSFULL), nv & 1)) {
                     tc_fence_after();
                     const uint32_t st = sb + kOffStage + (nv & 1) * kStage;
                     // K dimension = the 128 stacked query rows, 16 per MMA
@@ -476,10 +493,10 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     progressed = true;
                 }
                 if (progressed) {
-                    t0 = global_ns();
+                    dl.reset();
                 } else if (*abort_flag) {
                     ok = false;
-                } else if (global_ns() - t0 > kWaitLimitNs) {
+                } else if (dl.expired()) {
                     *abort_flag = 1;
                     atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
                     ok = false;
@@ -495,13 +512,24 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const int tok = row & 63, hl = row >> 6;
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         const size_t hoff = (size_t)(hq0 + hl) * a.L;
+        // Row data (query block, lse, Delta) is fetched one iteration ahead so its
+        // global-memory latency overlaps the previous iteration.
+        auto fetch = [&](int it2, int& qb2, float& nl2, float& dl2) {
+            qb2 = ql[it2];
+            const int i2 = qb2 * 64 + tok;
+            const bool v2 = i2 < a.L;
+            nl2 = v2 ? -a.lse[hoff + i2] * kLog2e : -INFINITY;
+            dl2 = v2 ? a.delta[hoff + i2] : 0.f;
+        };
+        int qb_n = 0;
+        float nl_n = 0.f, dl_n = 0.f;
+        if (n_it > 0) fetch(0, qb_n, nl_n, dl_n);
         bool ok = true;
         for (int it = 0; it < n_it; ++it) {
-            const int qb = ql[it];
-            const int i = qb * 64 + tok;
-            const bool valid = i < a.L;
-            const float neg_lse2 = valid ? -a.lse[hoff + i] * kLog2e : -INFINITY;
-            const float dlt = valid ? a.delta[hoff + i] : 0.f;
+            const int qb = qb_n;
+            const float neg_lse2 = nl_n;
+            const float dlt = dl_n;
+            if (it + 1 < n_it) fetch(it + 1, qb_n, nl_n, dl_n);
             const int buf = it & 1;
             ok = mbar_wait(bar(B_SPFULL + buf), (it >> 1) & 1, abort_flag, a.status);
             ok = __all_sync(0xffffffffu, ok);

@@ -170,11 +170,11 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
             tc_fence_after();
             int nq = 0, np = 0;  // next QK and next PV to issue
-            uint64_t t0 = global_ns();
+            Deadline dl;
             while (ok && np < n) {
                 bool progressed = false;
                 // QK_nq reuses score buffer nq&1, free once PV_{nq-2} has been issued.
-                if (nq < n && nq <= np + 1 && mbar_try_wait(bar(B_KFULL + nq % kSlots), (nq / kSlots) & 1)) {
+                if (nq < n && nq <= np + 1 && mbar_test_wait(bar(B_KFULL + nq % kSlots), (nq / kSlots) & 1)) {
                     tc_fence_after();
                     const uint32_t kb = sb + kOffK + (nq % kSlots) * kKBytes;
                     const uint32_t d = tmem + col_s(nq & 1);
@@ -190,7 +190,7 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     ++nq;
                     progressed = true;
                 }
-                if (np < nq && mbar_try_wait(bar(B_PFULL + (np & 1)), (np >> 1) & 1)) {
+                if (np < nq && mbar_test_wait(bar(B_PFULL + (np & 1)), (np >> 1) & 1)) {
                     if (!mbar_wait(bar(B_VFULL + np % kSlots), (np / kSlots) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
@@ -210,10 +210,10 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     progressed = true;
                 }
                 if (progressed) {
-                    t0 = global_ns();
+                    dl.reset();
                 } else if (*abort_flag) {
                     ok = false;
-                } else if (global_ns() - t0 > kWaitLimitNs) {
+                } else if (dl.expired()) {
                     *abort_flag = 1;
                     atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
                     ok = false;

@@ -30,6 +30,11 @@ struct ProfScope {
 cudaError_t launch_block_repr(const void* K, const uint8_t* mask, const phsa_shape& s,
                               float lambda, void* Krepr, cudaStream_t st);
 
+cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape& s,
+                             const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,
+                             cudaStream_t st);
+size_t select_tc_smem_bytes(const phsa_shape& s, int topk);
+
 cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_shape& s,
                                  const phsa_select_params& p, int32_t* idx, int32_t* cnt,
                                  int* status, cudaStream_t st);

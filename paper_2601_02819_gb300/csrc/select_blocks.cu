@@ -272,16 +272,17 @@ cudaError_t launch_select_g(const phsa_shape& s, const phsa_select_params& p, co
 
 size_t select_smem_bytes(const phsa_shape& s, int topk) {
     const int NQB = (s.L + kM - 1) / kM;
-    return (s.Hq / s.Hkv == 2) ? SelCfg<2>::smem_bytes(NQB, topk) : SelCfg<1>::smem_bytes(NQB, topk);
+    return (s.Hq / s.Hkv == 2) ? select_tc_smem_bytes(s, topk) : SelCfg<1>::smem_bytes(NQB, topk);
 }
 
 cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_shape& s,
                                  const phsa_select_params& p, int32_t* idx, int32_t* cnt,
                                  int* status, cudaStream_t st) {
-    (void)status;
     if ((long long)s.B * s.Hkv * ((s.L + kM - 1) / kM) == 0) return cudaSuccess;
-    return (s.Hq / s.Hkv == 2) ? launch_select_g<2>(s, p, Q, Krepr, idx, cnt, st)
-                               : launch_select_g<1>(s, p, Q, Krepr, idx, cnt, st);
+    // Two query heads per KV head fill a 128-row tcgen05 tile (select_tc.cu); a
+    // single head runs on the warp-level MMA kernel in this file.
+    if (s.Hq / s.Hkv == 2) return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
+    return launch_select_g<1>(s, p, Q, Krepr, idx, cnt, st);
 }
 
 }  // namespace phsa

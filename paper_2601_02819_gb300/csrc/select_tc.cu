@@ -1,0 +1,354 @@
+// Stage (b) on the tensor cores for GQA pairs (G*64 = 128 query rows):
+// query-to-block relevance and Top-K selection (Eq. 8; Algorithm 1 step 3),
+// one CTA per (query block qb, KV head g), 320 threads.
+//
+// The candidate representative keys C = [n_init, qb - n_local] stream through
+// a two-slot shared-memory ring in chunks of 128 rows (TMA). Each chunk is
+// used twice, and the scores never leave the SM:
+//   pass 1  S = Q Kr^T   (M = 128 query rows, N = 128 candidates) in TMEM;
+//           two threads per row (TMEM lane r, one per half of the columns)
+//           keep a running max and sum of 2^(S*scale - max) (online
+//           softmax); the halves are merged once, after the last chunk;
+//   pass 2  S^T = Kr Q^T (M = 128 candidates, N = 128 rows) in TMEM;
+//           two threads per candidate j (lane j, one per half of the rows)
+//           sum p = 2^(S*scale - m_r)/Z_r over their 64 rows in row order;
+//           A[t] = half 0 + half 1. Every candidate follows the same order,
+//           so equal candidates get bit-identical sums.
+//   top-k   one warp: rounds of a warp-wide argmax over the 64-bit key
+//           (bits(A) << 32 | ~t): larger A first, lower t on exact ties.
+// Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs.
+// Every wait is bounded in time (tc_common.cuh).
+#include "phsa_common.cuh"
+#include "phsa_internal.h"
+#include "tc_common.cuh"
+
+namespace phsa {
+
+namespace {
+
+using namespace tc;
+
+constexpr int kCand = 128;                 // candidates per chunk
+constexpr int kHalf = 128 * 64 * 2;        // 128 rows x 64 columns bf16 (16 KB)
+constexpr int kTile = 2 * kHalf;           // 128 x 128 (32 KB)
+constexpr int kOffQ = 0;
+constexpr int kOffKr = kOffQ + kTile;      // 2 slots
+constexpr int kOffStats = kOffKr + 2 * kTile;  // m2[128], iz[128], half partials m[2][128], z[2][128]
+constexpr int kOffBar = kOffStats + 6 * 128 * 4;
+constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = 3, B_SFULL = 5, B_SFREE = 7, B_DRAIN = 9,
+              kNumBars = 10;
+constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
+constexpr int kOffA = kOffMisc + 16;              // A0[NQB], A1[NQB], then sel[topk]
+constexpr int kThreads = 320;
+constexpr uint32_t kTmemCols = 256;
+
+size_t select_tc_smem(int nqb, int topk) {
+    return 1024 + (size_t)kOffA + (size_t)nqb * 8 + (size_t)topk * 4 + 16;
+}
+
+struct SelArgs {
+    int32_t* idx_out;
+    int32_t* cnt_out;
+    int* status;
+    int Hq, Hkv, L, T, NQB, topk, n_init, n_local;
+    float scale_log2;
+};
+
+__device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {
+    return a > b ? a : b;
+}
+
+__global__ void __launch_bounds__(kThreads, 2)
+select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKr,
+                 const SelArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    const uint32_t sb = smem_u32(smem);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int unit = blockIdx.x;
+    const int qb = a.NQB - 1 - (unit % a.NQB);  // heaviest query blocks first
+    const int bg = unit / a.NQB;
+    const int b = bg / a.Hkv, g = bg % a.Hkv;
+    const long long lu = (long long)bg * a.NQB + qb;
+    int32_t* out = a.idx_out + lu * a.topk;
+
+    const int n_init_q = min(a.n_init, qb + 1);            // forced initial [0, n_init_q)
+    const int loc_lo = max(n_init_q, qb - a.n_local + 1);  // forced local [loc_lo, qb]
+    const int c_lo = a.n_init, c_hi = qb - a.n_local;      // candidates [c_lo, c_hi]
+    const int nC = max(0, c_hi - c_lo + 1);
+    const int nF = n_init_q + (qb - loc_lo + 1);
+    const int ksel = a.topk - nF;
+
+    if (ksel >= nC) {  // the budget covers every candidate: nothing to score
+        const int n = nF + nC;
+        for (int j = tid; j < a.topk; j += kThreads) {
+            int v = -1;
+            if (j < n_init_q) v = j;
+            else if (j < n_init_q + nC) v = c_lo + (j - n_init_q);
+            else if (j < n) v = loc_lo + (j - n_init_q - nC);
+            out[j] = v;
+        }
+        if (tid == 0) a.cnt_out[lu] = n;
+        return;
+    }
+
+    auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
+    float* m2s = reinterpret_cast<float*>(smem + kOffStats);
+    float* izs = m2s + 128;
+    float* pm = izs + 128;  // [2][128] per-half running max (pass 1)
+    float* pz = pm + 256;   // [2][128] per-half running sum
+    float* A0 = reinterpret_cast<float*>(smem + kOffA);  // per-half aggregates (pass 2)
+    float* A1 = A0 + a.NQB;
+    int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 8);
+    const int nch = (nC + kCand - 1) / kCand;  // chunks per pass
+    const int steps = 2 * nch;
+
+    if (tid == 0) {
+        mbar_init(bar(B_Q), 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(bar(B_KFULL + s), 1);
+            mbar_init(bar(B_KEMPTY + s), 1);
+            mbar_init(bar(B_SFULL + s), 1);
+            mbar_init(bar(B_SFREE + s), 256);
+        }
+        mbar_init(bar(B_DRAIN), 1);
+        fence_barrier_init();
+        *abort_flag = 0;
+    }
+    if (warp == 9) {
+        tmem_alloc(sb + kOffMisc, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
+    const int hq0 = b * a.Hq + g * 2;
+
+    if (warp == 8) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            prefetch_tmap(&tmKr);
+            mbar_expect_tx(bar(B_Q), kTile);
+            for (int hl = 0; hl < 2; ++hl)
+                for (int dh = 0; dh < 2; ++dh)
+                    tma_load_3d(sb + kOffQ + dh * kHalf + hl * (kHalf / 2), &tmQ, bar(B_Q), dh * 64,
+                                qb * 64, hq0 + hl);
+            int issued = 0;
+            for (int s = 0; s < steps; ++s) {
+                const int slot = s & 1, c = s % nch;
+                if (s >= 2 && !mbar_wait(bar(B_KEMPTY + slot), ((s >> 1) - 1) & 1, abort_flag, a.status))
+                    break;
+                mbar_expect_tx(bar(B_KFULL + slot), kTile);
+                for (int dh = 0; dh < 2; ++dh)
+                    tma_load_3d(sb + kOffKr + slot * kTile + dh * kHalf, &tmKr, bar(B_KFULL + slot),
+                                dh * 64, c_lo + c * kCand, bg);
+                issued = s + 1;
+            }
+            mbar_wait_drain(bar(B_Q), 0);
+            for (int s = issued - 2; s < issued; ++s)
+                if (s >= 0) mbar_wait_drain(bar(B_KFULL + (s & 1)), (s >> 1) & 1);
+        }
+    } else if (warp == 9) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(128, 128, false);
+            bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
+            tc_fence_after();
+            for (int s = 0; ok && s < steps; ++s) {
+                const int slot = s & 1;
+                if (!mbar_wait(bar(B_KFULL + slot), (s >> 1) & 1, abort_flag, a.status)) break;
+                if (s >= 2 && !mbar_wait(bar(B_SFREE + slot), ((s >> 1) - 1) & 1, abort_flag, a.status))
+                    break;
+                tc_fence_after();
+                const uint32_t kr = sb + kOffKr + slot * kTile;
+                const uint32_t qa = sb + kOffQ;
+                const bool pass1 = s < nch;
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
+                    const uint64_t dq = sdesc_sw128(qa + off, 16, 1024);
+                    const uint64_t dk = sdesc_sw128(kr + off, 16, 1024);
+                    // pass 1: rows x candidates; pass 2: candidates x rows
+                    mma_ss(tmem + 128u * slot, pass1 ? dq : dk, pass1 ? dk : dq, idesc,
+                           ks > 0 ? 1u : 0u);
+                }
+                mma_commit(bar(B_SFULL + slot));
+                mma_commit(bar(B_KEMPTY + slot));
+            }
+            mma_commit(bar(B_DRAIN));
+            mbar_wait_drain(bar(B_DRAIN), 0);
+        }
+    } else {
+        // ------------------------------------------------ elementwise (8 warps)
+        const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+        const int r = (warp & 3) * 32 + lane;  // pass 1: query row; pass 2: candidate
+        const int hh = warp >> 2;              // half of the TMEM columns this thread reads
+        const bool row_ok = qb * 64 + (r & 63) < a.L;
+        float m = -INFINITY, z = 0.f;
+        bool ok = true;
+        // After a failed wait the loop keeps running without work, so that all eight
+        // warps reach the named barriers after pass 1 the same number of times.
+        for (int s = 0; s < steps; ++s) {
+            const int slot = s & 1, c = s % nch;
+            if (ok) {
+                ok = mbar_wait(bar(B_SFULL + slot), (s >> 1) & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+            }
+            if (ok) tc_fence_after();
+            if (ok && s < nch) {
+                // pass 1: row r against 64 candidates of the chunk, two loads of 32
+                const int t0 = c_lo + c * kCand + 64 * hh;
+                const bool full = t0 + 63 <= c_hi;
+#pragma unroll 1
+                for (int q = 0; q < 2; ++q) {
+                    uint32_t v[32];
+                    tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+                    float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        float x = __uint_as_float(v[j]) * a.scale_log2;
+                        if (!full && t0 + 32 * q + j > c_hi) x = -INFINITY;
+                        v[j] = __float_as_uint(x);
+                        m4[j & 3] = fmaxf(m4[j & 3], x);
+                    }
+                    const float mn = fmaxf(m, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])));
+                    if (mn != -INFINITY) {
+                        float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) s4[j & 3] += ex2_approx(__uint_as_float(v[j]) - mn);
+                        z = z * ex2_approx(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+                        m = mn;
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(bar(B_SFREE + slot));
+            } else if (ok) {
+                // pass 2: candidate r against the 64 rows of half hh, in row order
+                const float* mrow = m2s + 64 * hh;
+                const float* irow = izs + 64 * hh;
+                float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+                for (int q = 0; q < 2; ++q) {
+                    uint32_t v[32];
+                    tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+#pragma unroll
+                    for (int j = 0; j < 32; j += 4) {
+                        const float4 mm = *reinterpret_cast<const float4*>(mrow + 32 * q + j);
+                        const float4 iz = *reinterpret_cast<const float4*>(irow + 32 * q + j);
+                        acc[0] += ex2_approx(fmaf(__uint_as_float(v[j + 0]), a.scale_log2, -mm.x)) * iz.x;
+                        acc[1] += ex2_approx(fmaf(__uint_as_float(v[j + 1]), a.scale_log2, -mm.y)) * iz.y;
+                        acc[2] += ex2_approx(fmaf(__uint_as_float(v[j + 2]), a.scale_log2, -mm.z)) * iz.z;
+                        acc[3] += ex2_approx(fmaf(__uint_as_float(v[j + 3]), a.scale_log2, -mm.w)) * iz.w;
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(bar(B_SFREE + slot));
+                const int cj = c * kCand + r;
+                if (cj < nC) (hh ? A1 : A0)[cj] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+            }
+            if (s == nch - 1) {
+                // merge the two column halves of every row: (m, z) -> max and 1/sum
+                pm[hh * 128 + r] = m;
+                pz[hh * 128 + r] = z;
+                named_barrier(1, 256);
+                if (hh == 0) {
+                    const float ma = pm[r], mb = pm[128 + r];
+                    const float mx = fmaxf(ma, mb);
+                    const float za = ma == -INFINITY ? 0.f : pz[r] * ex2_approx(ma - mx);
+                    const float zb = mb == -INFINITY ? 0.f : pz[128 + r] * ex2_approx(mb - mx);
+                    const float zz = za + zb;
+                    m2s[r] = row_ok ? mx : 0.f;
+                    izs[r] = (row_ok && zz > 0.f) ? 1.0f / zz : 0.f;
+                }
+                named_barrier(1, 256);
+            }
+        }
+        named_barrier(1, 256);  // every A0/A1 entry written
+        if (ok && warp == 0) {
+            // top-k: lane l owns candidates l, l+32, ...; its best untaken key is cached.
+            // A = half 0 + half 1 (the same order for every candidate); taken: A0 = -1.
+            auto lane_best = [&]() {
+                unsigned long long best = 0ull;
+                for (int cj = lane; cj < nC; cj += 32) {
+                    const float a0 = A0[cj];
+                    if (a0 >= 0.f) {
+                        float v = a0 + A1[cj];
+                        if (!(v >= 0.f)) v = 0.f;  // NaN inputs rank as zero
+                        best = umax64(best, ((unsigned long long)__float_as_uint(v) << 32) |
+                                                (unsigned long long)(0xffffffffu - (unsigned)(c_lo + cj)));
+                    }
+                }
+                return best;
+            };
+            unsigned long long mine = lane_best();
+            for (int k = 0; k < ksel; ++k) {
+                unsigned long long best = mine;
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, off));
+                // every untaken candidate has a nonzero key, so best != 0 while k < ksel < nC
+                const int t = best ? (int)(0xffffffffu - (unsigned)(best & 0xffffffffull)) : c_lo;
+                if (lane == 0) sel[k] = t;
+                const int cj = t - c_lo;
+                if (best && (cj & 31) == lane) {
+                    A0[cj] = -1.0f;
+                    mine = lane_best();
+                }
+                __syncwarp();
+            }
+        }
+        named_barrier(1, 256);
+        if (ok) {
+            for (int j = threadIdx.x; j < a.topk; j += 256) {
+                if (j < n_init_q) out[j] = j;
+                else if (j >= n_init_q + ksel && j < nF + ksel) out[j] = loc_lo + (j - n_init_q - ksel);
+                else if (j >= nF + ksel) out[j] = -1;
+            }
+            if (threadIdx.x < ksel) {
+                const int v = sel[threadIdx.x];
+                int rank = 0;
+                for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
+                out[n_init_q + rank] = v;
+            }
+            if (threadIdx.x == 0) a.cnt_out[lu] = nF + ksel;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace
+
+size_t select_tc_smem_bytes(const phsa_shape& s, int topk) {
+    return select_tc_smem((s.L + 63) / 64, topk);
+}
+
+cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape& s,
+                             const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,
+                             cudaStream_t st) {
+    const int T = s.L / 64, NQB = (s.L + 63) / 64;
+    CUtensorMap tq, tkr;
+    if (!make_tmap_bf16_rows128(&tq, Q, s.L, (uint64_t)s.B * s.Hq, 64)) return cudaErrorInvalidValue;
+    // Krepr may be absent when no query block has a candidate (T < 2): the map is
+    // then built over Q, which is never read through it.
+    if (!make_tmap_bf16_rows128(&tkr, T > 0 ? Krepr : Q, T > 0 ? T : 1,
+                                (uint64_t)s.B * s.Hkv, 128))
+        return cudaErrorInvalidValue;
+    const size_t smem = select_tc_smem(NQB, p.topk);
+    cudaError_t e = cudaFuncSetAttribute(select_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local,
+                 p.sm_scale * kLog2e};
+    ProfScope prof(K_SELECT, st);
+    select_tc_kernel<<<(unsigned)((long long)s.B * s.Hkv * NQB), kThreads, smem, st>>>(tq, tkr, args);
+    return cudaGetLastError();
+}
+
+}  // namespace phsa

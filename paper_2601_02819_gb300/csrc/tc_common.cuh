@@ -27,15 +27,31 @@ namespace phsa {
 namespace tc {
 
 // ---------------------------------------------------------------- time limit
-// Every wait in these kernels gives up after this many nanoseconds of the
-// global timer, records PHSA_ERR_TIMEOUT and lets the CTA unwind.
-constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
+// Every wait in these kernels gives up after this many SM cycles (about one
+// second at the GB300's 2 GHz clock), records PHSA_ERR_TIMEOUT and lets the
+// CTA unwind. The cycle counter is cheap to read, and it is read only every
+// 64 polls, so a spinning thread reacts quickly to the condition it tests.
+constexpr uint64_t kWaitLimitCycles = 2000000000ull;
 
-__device__ __forceinline__ uint64_t global_ns() {
+__device__ __forceinline__ uint64_t sm_cycles() {
     uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    asm volatile("mov.u64 %0, %%clock64;" : "=l"(t));
     return t;
 }
+
+struct Deadline {
+    uint64_t t0;
+    uint32_t polls;
+    __device__ __forceinline__ Deadline() : t0(sm_cycles()), polls(0) {}
+    __device__ __forceinline__ void reset() {
+        t0 = sm_cycles();
+        polls = 0;
+    }
+    __device__ __forceinline__ bool expired() {
+        if ((++polls & 63u) != 0) return false;
+        return sm_cycles() - t0 > kWaitLimitCycles;
+    }
+};
 
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
@@ -65,16 +81,30 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Non-blocking test of the same condition (for issuers that poll several
+// barriers: try_wait may suspend the thread on one barrier while another is
+// already complete).
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n.reg .pred p;\nmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Waits for the phase of the given parity to complete. Returns false (and
 // raises *abort) if the time limit passes or another thread already aborted.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort,
                                           int* status) {
     if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = global_ns();
+    Deadline dl;
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort) return false;
-        if (global_ns() - t0 > kWaitLimitNs) {
+        if (dl.expired()) {
             *abort = 1;
             if (status) atomicCAS(status, 0, PHSA_ERR_TIMEOUT);
             return false;
@@ -85,9 +115,9 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
 // Drain wait used on the way out: waits for this CTA's own copies or MMAs to
 // finish even after an abort, bounded by the same time limit.
 __device__ __forceinline__ void mbar_wait_drain(uint32_t bar, uint32_t parity) {
-    const uint64_t t0 = global_ns();
+    Deadline dl;
     while (!mbar_try_wait(bar, parity))
-        if (global_ns() - t0 > kWaitLimitNs) return;
+        if (dl.expired()) return;
 }
 
 // ---------------------------------------------------------------- TMA
