@@ -58,7 +58,8 @@ constexpr int kOffV = kOffK + kKSlots * kPair;
 constexpr int kOffBar = kOffV + kVSlots * kPair;
 constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = B_KFULL + kKSlots, B_VFULL = B_KEMPTY + kKSlots,
               B_VEMPTY = B_VFULL + kVSlots, B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2,
-              B_FINAL = B_DSFULL + 1, B_DRAIN = B_FINAL + 1, kNumBars = B_DRAIN + 1;
+              B_DPFREE = B_DSFULL + 2, B_FINAL = B_DPFREE + 1, B_DRAIN = B_FINAL + 1,
+              kNumBars = B_DRAIN + 1;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kOffList = kOffMisc + 16;
 constexpr int kThreads = 352;  // 8 elementwise warps, K/Q/dO producer, MMA, V producer
@@ -111,7 +112,13 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         }
         mbar_init(bar(B_SPFULL), 1);
         mbar_init(bar(B_SPFULL + 1), 1);
+        // dS barriers alternate by pair: once dP is released early, a thread may
+        // finish pair p+1 before another has finished pair p, so their arrivals
+        // must go to different barriers. dP_{p+1} needs every thread's release of
+        // dP_p, so no thread gets two pairs ahead and two barriers suffice.
         mbar_init(bar(B_DSFULL), 256);
+        mbar_init(bar(B_DSFULL + 1), 256);
+        mbar_init(bar(B_DPFREE), 256);
         mbar_init(bar(B_FINAL), 1);
         mbar_init(bar(B_DRAIN), 1);
         fence_barrier_init();
@@ -173,30 +180,36 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         if (lane == 0 && n > 0) {
             constexpr uint32_t id_s = idesc_bf16(128, 128, false);
             constexpr uint32_t id_dq = idesc_bf16(128, 128, true);
+            const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
+            const uint64_t dDO0 = sdesc_sw128(sb + kOffDO, 16, 1024);
+            const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
+            const uint64_t dKmn0 = sdesc_sw128(sb + kOffK, kHalf128, 1024);  // K read MN-major
+            const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
             bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
             tc_fence_after();
             auto issue_s = [&](int p) {  // S_p = Q Kpair_p^T into buffer p & 1
-                const uint32_t kb = sb + kOffK + (p % kKSlots) * kPair;
+                const uint64_t kd = sdesc_at(dK0, (p % kKSlots) * kPair);
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
                     const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
-                    mma_ss(tmem + col_s(p & 1), sdesc_sw128(sb + kOffQ + off, 16, 1024),
-                           sdesc_sw128(kb + off, 16, 1024), id_s, ks > 0 ? 1u : 0u);
+                    mma_ss(tmem + col_s(p & 1), sdesc_at(dQ0, off), sdesc_at(kd, off), id_s,
+                           ks > 0 ? 1u : 0u);
                 }
             };
             auto issue_dp = [&](int p) {  // dP_p = dO Vpair_p^T; releases the V slot
-                const uint32_t vb = sb + kOffV + (p % kVSlots) * kPair;
+                const uint64_t vd = sdesc_at(dV0, (p % kVSlots) * kPair);
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
                     const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
-                    mma_ss(tmem + kColDP, sdesc_sw128(sb + kOffDO + off, 16, 1024),
-                           sdesc_sw128(vb + off, 16, 1024), id_s, ks > 0 ? 1u : 0u);
+                    mma_ss(tmem + kColDP, sdesc_at(dDO0, off), sdesc_at(vd, off), id_s,
+                           ks > 0 ? 1u : 0u);
                 }
                 mma_commit(bar(B_SPFULL + (p & 1)));  // S_p and dP_p are both complete
                 mma_commit(bar(B_VEMPTY + p % kVSlots));
             };
-            // Order: S_0 dP_0 S_1 | dS_0 -> dQ_0 dP_1 S_2 | dS_1 -> dQ_1 dP_2 S_3 | ...
-            // (dP has one buffer: dP_{p+1} follows the elementwise pass over dP_p.)
+            // Order: S_0 dP_0 S_1 | dP consumed_0 -> dP_1 | dS_0 -> dQ_0 S_2 | ...
+            // dP has one TMEM buffer: dP_{p+1} is issued as soon as the elementwise
+            // warps have loaded dP_p, while they still compute dS_p.
             ok = ok && mbar_wait(bar(B_KFULL), 0, abort_flag, a.status) &&
                  mbar_wait(bar(B_VFULL), 0, abort_flag, a.status);
             if (ok) {
@@ -204,33 +217,40 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 issue_s(0);
                 issue_dp(0);
             }
-            for (int p = 0; ok && p < np; ++p) {
-                if (p + 1 < np) {  // S_{p+1} overlaps the elementwise pass over pair p
-                    ok = mbar_wait(bar(B_KFULL + (p + 1) % kKSlots), ((p + 1) / kKSlots) & 1,
-                                   abort_flag, a.status);
-                    if (!ok) break;
+            if (ok && np > 1) {
+                ok = mbar_wait(bar(B_KFULL + 1), 0, abort_flag, a.status);
+                if (ok) {
                     tc_fence_after();
-                    issue_s(p + 1);
+                    issue_s(1);
                 }
-                ok = mbar_wait(bar(B_DSFULL), p & 1, abort_flag, a.status);
-                if (!ok) break;
-                tc_fence_after();
-                // dQ += dS_p Kpair_p: A = dS (TMEM), B = the K pair read MN-major
-                const uint32_t kb = sb + kOffK + (p % kKSlots) * kPair;
-#pragma unroll
-                for (int ks = 0; ks < 8; ++ks)
-                    mma_ts(tmem + kColDQ, tmem + col_s(p & 1) + (ks >> 2) * 64 + (ks & 3) * 8,
-                           sdesc_sw128(kb + ks * 2048, kHalf128, 1024), id_dq,
-                           (p > 0 || ks > 0) ? 1u : 0u);
-                mma_commit(bar(B_KEMPTY + p % kKSlots));
-                if (p == np - 1) {
-                    mma_commit(bar(B_FINAL));
-                } else {
-                    ok = mbar_wait(bar(B_VFULL + (p + 1) % kVSlots), ((p + 1) / kVSlots) & 1,
+            }
+            for (int p = 0; ok && p < np; ++p) {
+                if (p + 1 < np) {  // dP_{p+1} once the elementwise warps hold dP_p
+                    ok = mbar_wait(bar(B_DPFREE), p & 1, abort_flag, a.status) &&
+                         mbar_wait(bar(B_VFULL + (p + 1) % kVSlots), ((p + 1) / kVSlots) & 1,
                                    abort_flag, a.status);
                     if (!ok) break;
                     tc_fence_after();
                     issue_dp(p + 1);
+                }
+                ok = mbar_wait(bar(B_DSFULL + (p & 1)), (p >> 1) & 1, abort_flag, a.status);
+                if (!ok) break;
+                tc_fence_after();
+                // dQ += dS_p Kpair_p: A = dS (TMEM), B = the K pair read MN-major
+                const uint64_t kmn = sdesc_at(dKmn0, (p % kKSlots) * kPair);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ts(tmem + kColDQ, tmem + col_s(p & 1) + (ks >> 2) * 64 + (ks & 3) * 8,
+                           sdesc_at(kmn, ks * 2048), id_dq, (p > 0 || ks > 0) ? 1u : 0u);
+                mma_commit(bar(B_KEMPTY + p % kKSlots));
+                if (p == np - 1) {
+                    mma_commit(bar(B_FINAL));
+                } else if (p + 2 < np) {  // S_{p+2} reuses the S buffer dQ_p has just read
+                    ok = mbar_wait(bar(B_KFULL + (p + 2) % kKSlots), ((p + 2) / kKSlots) & 1,
+                                   abort_flag, a.status);
+                    if (!ok) break;
+                    tc_fence_after();
+                    issue_s(p + 2);
                 }
             }
             mma_commit(bar(B_DRAIN));
@@ -257,28 +277,27 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const int e = 2 * p + half;       // this half's block in the list
             const bool live = e < n;          // false: the duplicate of an odd count
             const bool diag = list[e] == qb;
-#pragma unroll 1
-            for (int q = 0; q < 2; ++q) {     // two 32-key chunks of this half
-                uint32_t sv[32], dp[32];
-                tmem_ld32(lane_base + col_s(buf) + 64 * half + 32 * q, sv);
-                tmem_ld32(lane_base + kColDP + 64 * half + 32 * q, dp);
-#pragma unroll
-                for (int c = 0; c < 16; ++c) {
-                    float ds[2];
-#pragma unroll
-                    for (int x = 0; x < 2; ++x) {
-                        const int key = 32 * q + 2 * c + x;
-                        float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + x]), a.scale_log2, neg_lse2));
-                        if (!live || (diag && key > tok)) pv = 0.f;
-                        ds[x] = pv * (__uint_as_float(dp[2 * c + x]) - dlt);
-                    }
-                    sv[c] = pack2_bf16(ds[0], ds[1]);
-                }
-                // dS columns [64 half + 16 q, +16): inside this thread's own S range
-                tmem_st16(lane_base + col_s(buf) + 64 * half + 16 * q, sv);
-            }
+            uint32_t sv[64], dp[64];
+            tmem_ld64(lane_base + col_s(buf) + 64 * half, sv);
+            tmem_ld64(lane_base + kColDP + 64 * half, dp);
             tc_fence_before();
-            mbar_arrive(bar(B_DSFULL));
+            mbar_arrive(bar(B_DPFREE));  // dP_p is in registers: the buffer may be refilled
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                float ds[2];
+#pragma unroll
+                for (int x = 0; x < 2; ++x) {
+                    const int key = 2 * c + x;
+                    float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + x]), a.scale_log2, neg_lse2));
+                    if (!live || (diag && key > tok)) pv = 0.f;
+                    ds[x] = pv * (__uint_as_float(dp[2 * c + x]) - dlt);
+                }
+                sv[c] = pack2_bf16(ds[0], ds[1]);
+            }
+            // dS columns [64 half, 64 half + 32): inside this thread's own S range
+            tmem_st32(lane_base + col_s(buf) + 64 * half, sv);
+            tc_fence_before();
+            mbar_arrive(bar(B_DSFULL + buf));
         }
         if (ok && n > 0) {
             ok = mbar_wait(bar(B_FINAL), 0, abort_flag, a.status);
@@ -442,6 +461,12 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         if (lane == 0 && n_it > 0) {
             constexpr uint32_t id_s = idesc_bf16(128, 64, false);
             constexpr uint32_t id_t = idesc_bf16(128, 64, true, true);  // A and B MN-major
+            const uint64_t dSt0 = sdesc_sw128(sb + kOffStage, 16, 1024);          // Q/dO K-major
+            const uint64_t dStT0 = sdesc_sw128(sb + kOffStage, kHalf128, 1024);   // Q/dO MN-major
+            const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
+            const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
+            const uint64_t dP0 = sdesc_sw128(sb + kOffP, kHalf128, 1024);
+            const uint64_t dS0 = sdesc_sw128(sb + kOffDS, kHalf128, 1024);
             bool ok = mbar_wait(bar(B_KV), 0, abort_flag, a.status);
             tc_fence_after();
             int ns = 0, nv = 0;
@@ -451,41 +476,35 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 if (ns < n_it && ns <= nv + 1 &&
                     mbar_test_wait(bar(B_QFULL + (ns & 1)), (ns >> 1) & 1)) {
                     tc_fence_after();
-                    const uint32_t st = sb + kOffStage + (ns & 1) * kStage;
+                    const uint64_t qd = sdesc_at(dSt0, (ns & 1) * kStage);
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (uint32_t)((ks & 3) * 32);
+                    for (int ks = 0; ks < 8; ++ks)
                         mma_ss(tmem + col_s(ns & 1),
-                               sdesc_sw128(st + (ks >> 2) * kHalf128 + off, 16, 1024),
-                               sdesc_sw128(sb + kOffK + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
+                               sdesc_at(qd, (ks >> 2) * kHalf128 + (ks & 3) * 32),
+                               sdesc_at(dK0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s,
                                ks > 0 ? 1u : 0u);
-                    }
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (uint32_t)((ks & 3) * 32);
+                    for (int ks = 0; ks < 8; ++ks)
                         mma_ss(tmem + col_dp(ns & 1),
-                               sdesc_sw128(st + kTile128 + (ks >> 2) * kHalf128 + off, 16, 1024),
-                               sdesc_sw128(sb + kOffV + (ks >> 2) * kHalf64 + off, 16, 1024), id_s,
+                               sdesc_at(qd, kTile128 + (ks >> 2) * kHalf128 + (ks & 3) * 32),
+                               sdesc_at(dV0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s,
                                ks > 0 ? 1u : 0u);
-                    }
                     mma_commit(bar(B_SPFULL + (ns & 1)));
                     ++ns;
                     progressed = true;
                 }
                 if (nv < ns && mbar_test_wait(bar(B_PDSFULL), nv & 1)) {
                     tc_fence_after();
-                    const uint32_t st = sb + kOffStage + (nv & 1) * kStage;
+                    const uint64_t qt = sdesc_at(dStT0, (nv & 1) * kStage);
                     // K dimension = the 128 stacked query rows, 16 per MMA
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + kColDV, sdesc_sw128(st + kTile128 + ks * 2048, kHalf128, 1024),
-                               sdesc_sw128(sb + kOffP + ks * 2048, kHalf128, 1024), id_t,
-                               (nv > 0 || ks > 0) ? 1u : 0u);
+                        mma_ss(tmem + kColDV, sdesc_at(qt, kTile128 + ks * 2048),
+                               sdesc_at(dP0, ks * 2048), id_t, (nv > 0 || ks > 0) ? 1u : 0u);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + kColDK, sdesc_sw128(st + ks * 2048, kHalf128, 1024),
-                               sdesc_sw128(sb + kOffDS + ks * 2048, kHalf128, 1024), id_t,
-                               (nv > 0 || ks > 0) ? 1u : 0u);
+                        mma_ss(tmem + kColDK, sdesc_at(qt, ks * 2048), sdesc_at(dS0, ks * 2048),
+                               id_t, (nv > 0 || ks > 0) ? 1u : 0u);
                     mma_commit(bar(B_PDSFREE));
                     mma_commit(bar(B_QEMPTY + (nv & 1)));
                     if (nv == n_it - 1) mma_commit(bar(B_FINAL));

@@ -167,6 +167,9 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         if (lane == 0 && n > 0) {
             constexpr uint32_t idesc_qk = idesc_bf16(128, 64, false);
             constexpr uint32_t idesc_pv = idesc_bf16(128, 128, true);
+            const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
+            const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
+            const uint64_t dV0 = sdesc_sw128(sb + kOffV, kKVHalf, 1024);
             bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
             tc_fence_after();
             int nq = 0, np = 0;  // next QK and next PV to issue
@@ -176,15 +179,13 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 // QK_nq reuses score buffer nq&1, free once PV_{nq-2} has been issued.
                 if (nq < n && nq <= np + 1 && mbar_test_wait(bar(B_KFULL + nq % kSlots), (nq / kSlots) & 1)) {
                     tc_fence_after();
-                    const uint32_t kb = sb + kOffK + (nq % kSlots) * kKBytes;
+                    const uint64_t kd = sdesc_at(dK0, (nq % kSlots) * kKBytes);
                     const uint32_t d = tmem + col_s(nq & 1);
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (uint32_t)((ks & 3) * 32);
-                        const uint64_t ad = sdesc_sw128(sb + kOffQ + (ks >> 2) * kHalfQ + off, 16, 1024);
-                        const uint64_t bd = sdesc_sw128(kb + (ks >> 2) * kKVHalf + off, 16, 1024);
-                        mma_ss(d, ad, bd, idesc_qk, ks > 0 ? 1u : 0u);
-                    }
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(d, sdesc_at(dQ0, (ks >> 2) * kHalfQ + (ks & 3) * 32),
+                               sdesc_at(kd, (ks >> 2) * kKVHalf + (ks & 3) * 32), idesc_qk,
+                               ks > 0 ? 1u : 0u);
                     mma_commit(bar(B_SFULL + (nq & 1)));
                     mma_commit(bar(B_KEMPTY + nq % kSlots));
                     ++nq;
@@ -196,13 +197,12 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t vb = sb + kOffV + (np % kSlots) * kKBytes;
+                    const uint64_t vd = sdesc_at(dV0, (np % kSlots) * kKBytes);
                     const uint32_t pt = tmem + col_s(np & 1);
 #pragma unroll
-                    for (int ks = 0; ks < 4; ++ks) {
-                        const uint64_t bd = sdesc_sw128(vb + ks * 2048, kKVHalf, 1024);
-                        mma_ts(tmem + kColO, pt + ks * 8, bd, idesc_pv, (np > 0 || ks > 0) ? 1u : 0u);
-                    }
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_ts(tmem + kColO, pt + ks * 8, sdesc_at(vd, ks * 2048), idesc_pv,
+                               (np > 0 || ks > 0) ? 1u : 0u);
                     mma_commit(bar(B_VEMPTY + np % kSlots));
                     mma_commit(bar(B_PVDONE));
                     if (np == n - 1) mma_commit(bar(B_OFINAL));

@@ -155,6 +155,8 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(128, 128, false);
+            const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
+            const uint64_t dKr0 = sdesc_sw128(sb + kOffKr, 16, 1024);
             bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
             tc_fence_after();
             for (int s = 0; ok && s < steps; ++s) {
@@ -163,14 +165,13 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 if (s >= 2 && !mbar_wait(bar(B_SFREE + slot), ((s >> 1) - 1) & 1, abort_flag, a.status))
                     break;
                 tc_fence_after();
-                const uint32_t kr = sb + kOffKr + slot * kTile;
-                const uint32_t qa = sb + kOffQ;
+                const uint64_t kr = sdesc_at(dKr0, slot * kTile);
                 const bool pass1 = s < nch;
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
                     const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
-                    const uint64_t dq = sdesc_sw128(qa + off, 16, 1024);
-                    const uint64_t dk = sdesc_sw128(kr + off, 16, 1024);
+                    const uint64_t dq = sdesc_at(dQ0, off);
+                    const uint64_t dk = sdesc_at(kr, off);
                     // pass 1: rows x candidates; pass 2: candidates x rows
                     mma_ss(tmem + 128u * slot, pass1 ? dq : dk, pass1 ? dk : dq, idesc,
                            ks > 0 ? 1u : 0u);

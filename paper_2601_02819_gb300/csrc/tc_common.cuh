@@ -183,6 +183,16 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, ui
     return d;
 }
 
+// The descriptor of the same layout `bytes` further on (a multiple of 16). The
+// start address field holds address / 16 in its low 14 bits and shared-memory
+// addresses stay below 256 KB, so the addition cannot carry out of the field.
+// Issue loops build descriptors this way from bases computed once: a
+// tcgen05.mma issue loop that recomputes full descriptors runs at about half
+// the rate of the tensor core for N = 128 tiles.
+__device__ __forceinline__ uint64_t sdesc_at(uint64_t base, uint32_t bytes) {
+    return base + (uint64_t)(bytes >> 4);
+}
+
 // Instruction descriptor, kind::f16: bf16 A and B, fp32 D, dense.
 // b_mn_major / a_mn_major select MN-major B / A operands in shared memory.
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major,
