@@ -46,7 +46,7 @@ cudaError_t launch_attn_fwd_tc(const void* Q, const void* K, const void* V, cons
 cudaError_t launch_tc_selftest(const void* A, const void* B, const void* V, float* S, float* O,
                                int* status, cudaStream_t st);
 bool make_tmap_bf16_rows128(CUtensorMap* map, const void* base, uint64_t rows, uint64_t planes,
-                            uint32_t box_rows);
+                            uint32_t box_rows, uint32_t box_planes = 1);
 
 cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const int32_t* idx,
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
