@@ -77,6 +77,11 @@ def _declare(L):
     L.phsa_oracle_sparse_attn_bwd.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32,
                                               i32, i32, f64, P, P, P]
     L.phsa_oracle_dense_causal.argtypes = [P, P, P, i32, i32, i32, i32, i32, f64, P, P]
+    L.phsa_oracle_decode_select.argtypes = [P, P, P, i32, i32, i32, i32, i32, i32, i32, i32,
+                                            i32, f64, P, P, P]
+    L.phsa_oracle_decode_select.restype = i32
+    L.phsa_oracle_decode_attn.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, i32,
+                                          f64, P, P]
 
 
 def _p(a: np.ndarray):
@@ -274,6 +279,47 @@ def dense_causal(Q, K, V, sm_scale: float):
     lse = np.empty((B, Hq, L), dtype=np.float64)
     lib().phsa_oracle_dense_causal(_p(Q), _p(K), _p(V), B, Hq, Hkv, L, D, float(sm_scale),
                                    _p(O), _p(lse))
+    return O, lse
+
+
+def decode_select(q, Krepr, lens, Lc: int, block_size: int, topk: int, n_init: int,
+                  n_local: int, sm_scale: float, want_agg: bool = False):
+    """Selection for one new token per sequence (the token at lens[b] - 1).
+
+    q [B,Hq,D], Krepr [B,Hkv,Lc/m,D] (full blocks valid). Returns (block_idx
+    [B,Hkv,topk], block_cnt [B,Hkv]) and, if ``want_agg``, A [B,Hkv,Lc/m].
+    """
+    q, Krepr, lens = _u16(q), _u16(Krepr), _i32(lens)
+    B, Hq, D = q.shape
+    Hkv = Krepr.shape[1]
+    Tc = Lc // block_size
+    assert Krepr.shape[2] == Tc and lens.shape == (B,)
+    idx = np.empty((B, Hkv, topk), dtype=np.int32)
+    cnt = np.empty((B, Hkv), dtype=np.int32)
+    agg = np.empty((B, Hkv, max(Tc, 1)), dtype=np.float64) if want_agg else None
+    rc = lib().phsa_oracle_decode_select(_p(q), _p(Krepr), _p(lens), B, Hq, Hkv, Lc, D,
+                                         block_size, topk, n_init, n_local, float(sm_scale),
+                                         _p(idx), _p(cnt), _p(agg) if want_agg else None)
+    if rc != 0:
+        raise ValueError("topk is smaller than the forced block count, or a length exceeds Lc")
+    return (idx, cnt, agg) if want_agg else (idx, cnt)
+
+
+def decode_attn(q, K, V, block_idx, block_cnt, lens, block_size: int, sm_scale: float):
+    """Attention of each sequence's new token over its selected blocks.
+
+    q [B,Hq,D], K/V [B,Hkv,Lc,D]; returns O [B,Hq,D] and lse [B,Hq] in fp64.
+    """
+    q, K, V = _u16(q), _u16(K), _u16(V)
+    block_idx, block_cnt, lens = _i32(block_idx), _i32(block_cnt), _i32(lens)
+    B, Hq, D = q.shape
+    Hkv, Lc = K.shape[1], K.shape[2]
+    topk = block_idx.shape[-1]
+    O = np.empty((B, Hq, D), dtype=np.float64)
+    lse = np.empty((B, Hq), dtype=np.float64)
+    lib().phsa_oracle_decode_attn(_p(q), _p(K), _p(V), _p(block_idx), _p(block_cnt), _p(lens),
+                                  B, Hq, Hkv, Lc, D, block_size, topk, float(sm_scale), _p(O),
+                                  _p(lse))
     return O, lse
 
 

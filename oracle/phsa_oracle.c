@@ -175,16 +175,15 @@ static int is_forced(int t, int qb, int n_init, int n_local) {
     return t < n_init || t >= qb - n_local + 1;
 }
 
-/* Selection for one (b, g, qb) unit u = (b*Hkv + g)*NQB + qb. Writes topk
- * entries to out, returns the count, or -1 if topk < |F_b|. If agg is not NULL
- * it receives A_t for the T blocks (NaN where t was not scored). */
-static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv, int L, int D,
-                       int m, int topk, int n_init, int n_local, double scale, int64_t u,
-                       int32_t* out, double* agg) {
-    const int G = Hq / Hkv, T = L / m, NQB = (L + m - 1) / m;
-    const int qb = (int)(u % NQB);
-    const int g = (int)((u / NQB) % Hkv);
-    const int b = (int)(u / ((int64_t)NQB * Hkv));
+/* The selection rule (R2-R4) for one query block qb of one KV head, whose
+ * query rows are rows[0..nrows) (D bf16 values each, in the order their
+ * probabilities are summed). Kr holds the KV head's representative keys, one
+ * per block; only the first T of them exist. Writes topk entries to out and
+ * returns the count, or -1 if topk < |F_b|. If agg is not NULL it receives A_t
+ * for t < T (NaN where t was not scored). */
+static int select_core(const uint16_t* const* rows, int nrows, const uint16_t* Kr, int T, int qb,
+                       int D, int topk, int n_init, int n_local, double scale, int32_t* out,
+                       double* agg) {
     double* A = (double*)calloc((size_t)(T > 0 ? T : 1), sizeof(double));
     int* cand = (int*)malloc(sizeof(int) * (size_t)(qb + 1));
     int* chosen = (int*)calloc((size_t)(qb + 1), sizeof(int));
@@ -201,23 +200,20 @@ static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv
             for (int c = 0; c < nC; ++c) chosen[cand[c]] = 1;
         } else if (ksel > 0) {
             double* s = (double*)malloc(sizeof(double) * (size_t)nC);
-            for (int hh = 0; hh < G; ++hh) {
-                const int h = g * G + hh;
-                for (int i = qb * m; i < (qb + 1) * m && i < L; ++i) {
-                    const uint16_t* q = Q + (((int64_t)b * Hq + h) * L + i) * D;
-                    double mx = -INFINITY;
-                    for (int c = 0; c < nC; ++c) {
-                        const uint16_t* M = Krepr + (((int64_t)b * Hkv + g) * T + cand[c]) * D;
-                        double dot = 0.0;
-                        for (int d = 0; d < D; ++d)
-                            dot += phsa_oracle_bf16_to_f64(q[d]) * phsa_oracle_bf16_to_f64(M[d]);
-                        s[c] = dot * scale; /* S_{i,t} */
-                        if (s[c] > mx) mx = s[c];
-                    }
-                    double z = 0.0;
-                    for (int c = 0; c < nC; ++c) z += exp(s[c] - mx);
-                    for (int c = 0; c < nC; ++c) A[cand[c]] += exp(s[c] - mx) / z; /* R2 */
+            for (int r = 0; r < nrows; ++r) {
+                const uint16_t* q = rows[r];
+                double mx = -INFINITY;
+                for (int c = 0; c < nC; ++c) {
+                    const uint16_t* M = Kr + (int64_t)cand[c] * D;
+                    double dot = 0.0;
+                    for (int d = 0; d < D; ++d)
+                        dot += phsa_oracle_bf16_to_f64(q[d]) * phsa_oracle_bf16_to_f64(M[d]);
+                    s[c] = dot * scale; /* S_{r,t} */
+                    if (s[c] > mx) mx = s[c];
                 }
+                double z = 0.0;
+                for (int c = 0; c < nC; ++c) z += exp(s[c] - mx);
+                for (int c = 0; c < nC; ++c) A[cand[c]] += exp(s[c] - mx) / z; /* R2 */
             }
             free(s);
             cand_t* order = (cand_t*)malloc(sizeof(cand_t) * (size_t)nC);
@@ -238,6 +234,28 @@ static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv
     free(A);
     free(cand);
     free(chosen);
+    return n;
+}
+
+/* Selection for one (b, g, qb) unit u = (b*Hkv + g)*NQB + qb: the rows are the
+ * block's tokens of each query head of the group, head by head. */
+static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv, int L, int D,
+                       int m, int topk, int n_init, int n_local, double scale, int64_t u,
+                       int32_t* out, double* agg) {
+    const int G = Hq / Hkv, T = L / m, NQB = (L + m - 1) / m;
+    const int qb = (int)(u % NQB);
+    const int g = (int)((u / NQB) % Hkv);
+    const int b = (int)(u / ((int64_t)NQB * Hkv));
+    const uint16_t** rows = (const uint16_t**)malloc(sizeof(uint16_t*) * (size_t)(G * m));
+    int nrows = 0;
+    for (int hh = 0; hh < G; ++hh) {
+        const int h = g * G + hh;
+        for (int i = qb * m; i < (qb + 1) * m && i < L; ++i)
+            rows[nrows++] = Q + (((int64_t)b * Hq + h) * L + i) * D;
+    }
+    int n = select_core(rows, nrows, Krepr + ((int64_t)b * Hkv + g) * T * D, T, qb, D, topk,
+                        n_init, n_local, scale, out, agg);
+    free(rows);
     return n;
 }
 
@@ -561,6 +579,83 @@ void phsa_oracle_sparse_attn_bwd_kv_blocks(const uint16_t* Q, const uint16_t* K,
         free(keys);
         free(s);
         free(o);
+    }
+}
+
+/* ---- Decode: one new token per sequence ----------------------------------
+ * Sequence b holds lens[b] tokens of a cache with capacity Lc: K, V
+ * [B,Hkv,Lc,D], Krepr [B,Hkv,Lc/m,D] (the representative keys of its full
+ * blocks), q [B,Hq,D] the token at position p = lens[b] - 1. This is the same
+ * rule as for a query block that holds the single row p (Section 3.3,
+ * Algorithm 1 for one token, with the group's G heads as its rows): forced
+ * F = {0..n_init-1} U {qb-n_local+1..qb} with qb = floor(p/m); candidates are
+ * the strictly earlier full blocks. A sequence with lens[b] <= 0 has no query:
+ * count 0, indices -1, output 0 and lse -inf. */
+int phsa_oracle_decode_select(const uint16_t* q, const uint16_t* Krepr, const int32_t* lens,
+                              int B, int Hq, int Hkv, int Lc, int D, int m, int topk, int n_init,
+                              int n_local, double scale, int32_t* block_idx, int32_t* block_cnt,
+                              double* agg) {
+    const int G = Hq / Hkv, Tc = Lc / m;
+    int bad = 0;
+    const int64_t units = (int64_t)B * Hkv;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(NTH) reduction(| : bad)
+#endif
+    for (int64_t u = 0; u < units; ++u) {
+        const int b = (int)(u / Hkv), g = (int)(u % Hkv);
+        const int len = lens[b];
+        int32_t* out = block_idx + u * topk;
+        double* ag = agg ? agg + u * Tc : NULL;
+        if (ag)
+            for (int t = 0; t < Tc; ++t) ag[t] = NAN;
+        if (len <= 0 || len > Lc) {
+            for (int j = 0; j < topk; ++j) out[j] = -1;
+            block_cnt[u] = 0;
+            if (len > Lc) bad = 1;
+            continue;
+        }
+        const int p = len - 1;
+        const uint16_t* rows[64];
+        for (int hh = 0; hh < G && hh < 64; ++hh) rows[hh] = q + ((int64_t)b * Hq + g * G + hh) * D;
+        int n = select_core(rows, G, Krepr + ((int64_t)b * Hkv + g) * Tc * D, len / m, p / m, D,
+                            topk, n_init, n_local, scale, out, ag);
+        block_cnt[u] = n;
+        if (n < 0) bad = 1;
+    }
+    return bad ? -1 : 0;
+}
+
+/* Decode attention (Eq. 10-11 for row p): O [B,Hq,D] fp64, lse [B,Hq]. */
+void phsa_oracle_decode_attn(const uint16_t* q, const uint16_t* K, const uint16_t* V,
+                             const int32_t* block_idx, const int32_t* block_cnt,
+                             const int32_t* lens, int B, int Hq, int Hkv, int Lc, int D, int m,
+                             int topk, double scale, double* O, double* lse) {
+    const int G = Hq / Hkv;
+    const int64_t n_rows = (int64_t)B * Hq;
+#ifdef _OPENMP
+#pragma omp parallel num_threads(NTH)
+#endif
+    {
+        int* keys = (int*)malloc(sizeof(int) * (size_t)(Lc > 0 ? Lc : 1));
+        double* s = (double*)malloc(sizeof(double) * (size_t)(Lc > 0 ? Lc : 1));
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 4)
+#endif
+        for (int64_t r = 0; r < n_rows; ++r) {
+            const int b = (int)(r / Hq), h = (int)(r % Hq), g = h / G;
+            const int len = lens[b];
+            if (len <= 0 || len > Lc) {
+                for (int d = 0; d < D; ++d) O[r * D + d] = 0.0;
+                lse[r] = -INFINITY;
+                continue;
+            }
+            const int64_t u = (int64_t)b * Hkv + g;
+            int nk = row_keys(block_idx + u * topk, block_cnt[u], len - 1, len, m, keys);
+            attn_row(q + r * D, K + u * Lc * D, V + u * Lc * D, keys, nk, D, scale, s, O + r * D,
+                     lse + r);
+        }
+        free(keys);
+        free(s);
     }
 }
 
