@@ -37,6 +37,8 @@ from paper_2601_02819_gb300.sharding import max_over_ranks, rank_seed, shard_seq
 
 METRIC = ("sparse-attn prefill tokens/s + effective TFLOPS at 32k, 97.3% sparsity; "
           "% roofline")
+DECODE_METRIC = ("sparse-attn decode tokens/s, 64 sequences x 32k cached tokens, top-k 14; "
+                 "% HBM roofline")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -443,6 +445,233 @@ def run_ours(args):
     return out
 
 
+# ---------------------------------------------------------------- decode
+def decode_algorithmic(w, lens: np.ndarray, cnt: np.ndarray):
+    """Bytes each decode kernel must move per step (all three are HBM-bound).
+
+    repr: the block a sequence has just filled (its keys and punctuation
+    bytes, one representative key written) per KV head; select: the candidates'
+    representative keys, q, the block lists; attn: q, the selected keys and
+    values up to the new token, O and lse, the block lists.
+    """
+    m, D, bf = w.block_size, w.D, 2
+    filled = int(((lens > 0) & (lens % m == 0)).sum())
+    rep = filled * w.Hkv * (m * D * bf + D * bf) + filled * m
+    n_c = np.maximum(0, (lens - 1) // m - w.n_local - w.n_init + 1)
+    sel = int(n_c.sum()) * w.Hkv * D * bf + w.B * w.Hq * D * bf + cnt.size * (w.topk + 1) * 4
+    keys = 0
+    for b in range(w.B):
+        qb = (lens[b] - 1) // m
+        for g in range(w.Hkv):
+            n = int(cnt[b, g])
+            keys += n * m - ((qb + 1) * m - lens[b])  # the local block is filled up to p
+    att = keys * 2 * D * bf + 2 * w.B * w.Hq * D * bf + w.B * w.Hq * 4 + cnt.size * (w.topk + 1) * 4
+    return {"decode_repr": {"flops": 0.0, "bytes": float(rep)},
+            "decode_select": {"flops": 2.0 * D * float(n_c.sum()) * w.Hq, "bytes": float(sel)},
+            "decode_attn": {"flops": 4.0 * D * keys * w.G, "bytes": float(att)}}
+
+
+def oracle_decode_sample(w, x, n_units: int, seed: int):
+    """Times the oracle on `n_units` random (sequence, KV head) units of one
+    decode step (the just-filled block's repr, the selection, the attention)
+    and scales to the whole batch. Representative keys of the cached blocks are
+    computed beforehand (they belong to the cache, not to the step)."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    U = w.B * w.Hkv
+    units = rng.choice(U, size=min(n_units, U), replace=False)
+    bits = lambda t: t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    m, secs = w.block_size, 0.0
+    for u in units:
+        b, g = int(u // w.Hkv), int(u % w.Hkv)
+        Kbg, Vbg = bits(x["K"][b:b + 1, g:g + 1]), bits(x["V"][b:b + 1, g:g + 1])
+        qbg = bits(x["q"][b:b + 1, w.G * g:w.G * (g + 1)])
+        mb, lb = x["mask"][b:b + 1], x["lens"][b:b + 1]
+        Kr = oracle.block_repr(Kbg, mb, m, w.lam)
+        t0 = time.perf_counter()
+        L = int(lb[0])
+        if L % m == 0:
+            oracle.block_repr(Kbg[:, :, L - m:L], mb[:, L - m:L], m, w.lam)
+        idx, cnt = oracle.decode_select(qbg, Kr, lb, w.L, m, w.topk, w.n_init, w.n_local,
+                                        w.sm_scale)
+        oracle.decode_attn(qbg, Kbg, Vbg, idx, cnt, lb, m, w.sm_scale)
+        secs += time.perf_counter() - t0
+    est = secs * U / len(units)
+    desc = (f"{len(units)} of {U} (sequence, KV head) units of one decode step (repr of the"
+            f" filled block, selection, attention), scaled to the batch")
+    return est, desc
+
+
+def run_decode(args):
+    from paper_2601_02819_gb300 import phsa
+    rank, world, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    w = inputs.DECODE_WORKLOADS[args.workload]
+    x = inputs.make_decode_inputs(w, dev, seed=rank_seed(w.seed, rank * w.B))
+    q, K, V, mask, lens = x["q"], x["K"], x["V"], x["mask_dev"], x["lens_dev"]
+    Kr = phsa.phsa_build_block_repr(K, mask, w.lam)  # the cache's prefill: not part of a step
+    idx = torch.empty((w.B, w.Hkv, w.topk), dtype=torch.int32, device=dev)
+    cnt = torch.empty((w.B, w.Hkv), dtype=torch.int32, device=dev)
+    O = torch.empty_like(q)
+    lse = torch.empty((w.B, w.Hq), dtype=torch.float32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        phsa.phsa_decode_update_repr(K, mask, lens, w.lam, Kr)
+        phsa.phsa_decode_select(q, Kr, lens, w.L, w.topk, w.n_init, w.n_local, w.sm_scale,
+                                block_idx=idx, block_cnt=cnt)
+        phsa.phsa_decode_attn(q, K, V, idx, cnt, lens, w.sm_scale, O=O, lse=lse)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    status = phsa.phsa_get_device_status()
+    if status != 0:
+        raise SystemExit(f"device status after warm-up: {phsa.phsa_status_string(status)}")
+    cnt_np = cnt.cpu().numpy()
+
+    # L2 is flushed (256 MB written) before every step, outside the timed events.
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    phsa.phsa_profile_read()
+    phsa.phsa_profile_enable(True)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    for e0, e1 in evs:
+        flush.zero_()
+        e0.record(stream)
+        step()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    t_wall1 = time.time()
+    phsa.phsa_profile_enable(False)
+    prof = phsa.phsa_profile_read()
+    clk = clocks.stop(t_wall0, t_wall1)
+    ms_step = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / args.steps, device=dev)
+    status = phsa.phsa_get_device_status()
+
+    e2e = None
+    if not args.no_e2e:
+        # The caches stay on the device; each step uploads the new token's q, k, v
+        # and punctuation flag, appends them at position L - 1, and reads O back.
+        hq = torch.empty(q.shape, dtype=torch.int16).pin_memory()
+        hk = torch.empty((w.B, w.Hkv, w.D), dtype=torch.int16).pin_memory()
+        hv = torch.empty((w.B, w.Hkv, w.D), dtype=torch.int16).pin_memory()
+        hm = torch.empty((w.B,), dtype=torch.uint8).pin_memory()
+        hq.copy_(q.view(torch.int16).cpu())
+        hk.copy_(K[:, :, w.L - 1].contiguous().view(torch.int16).cpu())
+        hv.copy_(V[:, :, w.L - 1].contiguous().view(torch.int16).cpu())
+        hm.copy_(mask[:, w.L - 1].cpu())
+        hO = torch.empty(O.shape, dtype=torch.int16).pin_memory()
+        kn = torch.empty((w.B, w.Hkv, w.D), dtype=torch.bfloat16, device=dev)
+        vn = torch.empty_like(kn)
+        mn = torch.empty((w.B,), dtype=torch.uint8, device=dev)
+        h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hm))
+        d2h = hO.numel() * hO.element_size()
+
+        def e2e_step():
+            q.view(torch.int16).copy_(hq, non_blocking=True)
+            kn.view(torch.int16).copy_(hk, non_blocking=True)
+            vn.view(torch.int16).copy_(hv, non_blocking=True)
+            mn.copy_(hm, non_blocking=True)
+            K[:, :, w.L - 1].copy_(kn)
+            V[:, :, w.L - 1].copy_(vn)
+            mask[:, w.L - 1].copy_(mn)
+            step()
+            hO.copy_(O.view(torch.int16), non_blocking=True)
+
+        for _ in range(3):
+            e2e_step()
+        n_e2e = max(3, min(args.steps, 50))
+        barrier()
+        torch.cuda.synchronize()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        a1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ms_e2e = max_over_ranks(a0.elapsed_time(a1) / n_e2e, device=dev)
+        e2e = {"value": world * w.B / (ms_e2e / 1e3), "unit": "tokens/s", "ms_per_step": ms_e2e,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": n_e2e,
+               "note": "caches resident on the device; the new token's q, k, v and flag "
+                       "are uploaded and appended, O read back (the K/V appends are torch copies)"}
+
+    if rank != 0:
+        return None
+    peaks, peak_src = load_peaks()
+    BW = peaks["hbm_gbs"]
+    kt = decode_algorithmic(w, x["lens"], cnt_np)
+    kernels = {}
+    for name, (ms, n) in prof.items():
+        if n == 0:
+            continue
+        avg_s = ms / n / 1e3
+        e = {"launches": n, "ms_total": round(ms, 4), "us_per_launch": round(avg_s * 1e6, 2)}
+        if name in kt:
+            e["bound"] = "hbm"
+            e["achieved_gbs"] = round(kt[name]["bytes"] / avg_s / 1e9, 1)
+            e["frac"] = round(kt[name]["bytes"] / avg_s / 1e9 / BW, 4)
+        kernels[name] = e
+    tot = sum(v["ms_total"] for v in kernels.values()) or 1.0
+    for v in kernels.values():
+        v["share"] = round(v["ms_total"] / tot, 4)
+    dom = max((k for k in kernels if k in kt), key=lambda k: kernels[k]["ms_total"])
+    avg_s = kernels[dom]["ms_total"] / kernels[dom]["launches"] / 1e3
+    roof = {"kernel": dom, "bound": "hbm", "achieved": round(kt[dom]["bytes"] / avg_s / 1e9, 1),
+            "peak": BW, "unit": "GB/s", "frac": round(kt[dom]["bytes"] / avg_s / 1e9 / BW, 4),
+            "peak_source": f"{peak_src} HBM copy", "traffic": None,
+            "algorithmic_per_launch": kt[dom]["bytes"]}
+    step_bytes = sum(v["bytes"] for v in kt.values())
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        cores = oracle_threads()
+        est, desc = oracle_decode_sample(w, x, args.cpu_units, seed=5)
+        cpu = {"value": w.B / est, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+               "sample": desc, "est_s_per_step": round(est, 3)}
+    return {
+        "metric": DECODE_METRIC, "value": world * w.B / (ms_step / 1e3), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "cache_len": w.L, "Hq": w.Hq, "Hkv": w.Hkv,
+                   "D": w.D, "block_size": w.block_size, "topk": w.topk, "n_init": w.n_init,
+                   "n_local": w.n_local, "lambda": w.lam,
+                   "step": "decode: repr of the just-filled block + selection + attention",
+                   "l2": "flushed (256 MB written) before every step, outside the timed events",
+                   "parallelism": f"dp{world} (independent sequences)"},
+        "step_roofline": {"bytes": step_bytes, "us": round(step_bytes / (BW * 1e9) * 1e6, 2),
+                          "frac": round(step_bytes / (BW * 1e9) / (ms_step / 1e3), 4)},
+        "roofline": roof,
+        "kernels": kernels,
+        "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "clocks": clk,
+        "device_status": status,
+        "peaks": {"source": peak_src, "hbm_gbs": BW},
+    }
+
+
 # ---------------------------------------------------------------- reference arm
 def run_reference(args):
     rank, world, _ = dist_env()
@@ -483,7 +712,8 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="prefill_32k", choices=sorted(inputs.WORKLOADS))
+    ap.add_argument("--workload", default="prefill_32k",
+                    choices=sorted(inputs.WORKLOADS) + sorted(inputs.DECODE_WORKLOADS))
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-units", type=int, default=48,
@@ -493,7 +723,12 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
-    out = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if args.workload in inputs.DECODE_WORKLOADS:
+        if args.impl == "reference":
+            raise SystemExit("--impl reference times the prefill workloads only")
+        out = run_decode(args)
+    else:
+        out = run_reference(args) if args.impl == "reference" else run_ours(args)
     if out is not None:
         print(json.dumps(out), flush=True)
     if int(os.environ.get("WORLD_SIZE", "1")) > 1 and args.impl == "ours":

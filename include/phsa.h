@@ -173,6 +173,54 @@ int phsa_sparse_attn_bwd_noalloc(const void* Q, const void* K, const void* V, co
                                  void* dQ, void* dK, void* dV, void* stream);
 
 /*
+ * Decode: one new token per sequence, against per-sequence caches.
+ * Layout: s.L is the cache capacity; K, V bf16 [B, Hkv, L, D]; punct_mask
+ * uint8 [B, L]; Krepr bf16 [B, Hkv, floor(L/m), D]; seq_lens int32 [B] (device)
+ * holds each sequence's token count, the new token included, so its query is
+ * the token at p = seq_lens[b] - 1, with query block qb = floor(p/m). A length
+ * of 0 means no query; a length < 0 or > L is a device-side error
+ * (PHSA_ERR_DEVICE_INDEX) and that sequence is treated as empty.
+ */
+
+/*
+ * Block-level caching of the representative keys (Section 3.2): for every
+ * sequence whose length is a positive multiple of m, the block that the new
+ * token has just filled, t = seq_lens[b]/m - 1, gets its representative key
+ * (Eq. 6-8, the same arithmetic as phsa_build_block_repr); every other block
+ * of Krepr is left as it is. Call after appending each token's K and mask;
+ * build the initial Krepr of a prefilled cache with phsa_build_block_repr.
+ */
+int phsa_decode_update_repr(const void* K, const uint8_t* punct_mask, const int32_t* seq_lens,
+                            phsa_shape s, float lambda, void* Krepr, void* stream);
+
+/*
+ * Selection for the new token (Eq. 8 / Algorithm 1 step 3 for one token):
+ * the rule of phsa_select_blocks for a unit whose rows are the token p in
+ * each of the G query heads of KV head g: forced F = {0..n_init-1} U
+ * {qb-n_local+1..qb} clipped to [0, qb]; candidates are the full blocks
+ * t <= qb-1 not in F; A[t] = sum over the G heads of softmax_t(sm_scale
+ * q_h . Krepr[t]); min(topk-|F|, |C|) candidates by A descending, ties to
+ * the lower t; ascending output, -1 padded.
+ *   q         bf16 [B, Hq, D]       in (the new token of every sequence)
+ *   block_idx int32 [B, Hkv, topk]  out; block_cnt int32 [B, Hkv] out
+ */
+int phsa_decode_select(const void* q, const void* Krepr, const int32_t* seq_lens, phsa_shape s,
+                       phsa_select_params p, int32_t* block_idx, int32_t* block_cnt,
+                       void* stream);
+
+/*
+ * Attention of the new token (Eq. 10-11 for row p): o = sum over keys j <= p
+ * of the listed blocks of softmax_j(sm_scale q . k_j) v_j; lse its natural-log
+ * log-sum-exp. Entries of block_idx must be -1 or 0 <= t <= qb, ascending;
+ * others are skipped and recorded as PHSA_ERR_DEVICE_INDEX. A sequence with
+ * no query gets o = 0 and lse = -inf.
+ *   q    bf16 [B, Hq, D] in;  O bf16 [B, Hq, D] out;  lse fp32 [B, Hq] out
+ */
+int phsa_decode_attn(const void* q, const void* K, const void* V, const int32_t* block_idx,
+                     const int32_t* block_cnt, const int32_t* seq_lens, phsa_shape s, int topk,
+                     float sm_scale, void* O, float* lse, void* stream);
+
+/*
  * Synchronises `stream`, returns the device status word of the current
  * device (PHSA_OK or the first device-side error code recorded since the
  * last call) and clears it. Returns PHSA_ERR_CUDA if the synchronisation

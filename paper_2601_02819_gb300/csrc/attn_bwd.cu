@@ -112,10 +112,11 @@ __device__ int block_excl_scan(int v, int* tmp, int& total) {
 __global__ void __launch_bounds__(1024)
 idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words, int work_max,
                  int slot_max, TInfo* __restrict__ tinfo, int32_t* __restrict__ qlist,
-                 int2* __restrict__ work, int32_t* __restrict__ nwork, int* status) {
+                 int2* __restrict__ work, int32_t* __restrict__ nwork, int* __restrict__ arrive,
+                 int* status) {
     __shared__ int tmp[32];
     const int bg = blockIdx.x;
-    const int per = (NQB + 1023) / 1024;  // KV blocks handled by each thread
+    const int per = (NQB + 1023) / 1024;  // KV blocks counted by each thread
     const int t0 = threadIdx.x * per;
     const uint32_t* bb = bits + (size_t)bg * NQB * words;
     int sn = 0, sch = 0, ssl = 0;
@@ -138,21 +139,12 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
         if (tch > work_max || tsl > slot_max || tn > NQB * topk) set_status(status, PHSA_ERR_DEVICE_INDEX);
     }
     TInfo* ti = tinfo + (size_t)bg * NQB;
-    int32_t* ql = qlist + (size_t)bg * NQB * topk;
     int2* wk = work + (size_t)bg * work_max;
     for (int k = 0; k < per; ++k) {
         const int t = t0 + k;
         if (t >= NQB) break;
         int n = 0;
-        for (int w = 0; w < words; ++w) {
-            uint32_t m = bb[(size_t)t * words + w];
-            while (m) {
-                const int q = w * 32 + __ffs(m) - 1;
-                m &= m - 1;
-                if (on + n < NQB * topk) ql[on + n] = q;
-                ++n;
-            }
-        }
+        for (int w = 0; w < words; ++w) n += __popc(bb[(size_t)t * words + w]);
         const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
         TInfo info;
         info.off = on;
@@ -160,11 +152,56 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
         info.nch = nch;
         info.slot = (nch > 1 && osl + nch <= slot_max) ? osl : -1;
         ti[t] = info;
+        arrive[(size_t)bg * NQB + t] = 0;
         for (int c = 0; c < nch; ++c)
             if (och + c < work_max) wk[och + c] = make_int2(t, c);
         on += n;
         och += nch;
         osl += nch > 1 ? nch : 0;
+    }
+    __syncthreads();  // tinfo of every block is written and visible to the whole CTA
+    // List of each KV block: one warp per block, 32 bitmap words per round; a
+    // warp scan of the words' popcounts gives every lane its output position.
+    // Each warp takes 8 blocks at a time and issues all their loads first.
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int32_t* ql = qlist + (size_t)bg * NQB * topk;
+    const int cap = NQB * topk;
+    constexpr int kBatch = 8;
+    for (int tb = warp; tb < NQB; tb += 32 * kBatch) {
+        int pos[kBatch];
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            const int t = tb + 32 * j;
+            pos[j] = t < NQB ? ti[t].off : 0;
+        }
+        for (int w0 = 0; w0 < words; w0 += 32) {
+            const int w = w0 + lane;
+            uint32_t m[kBatch];
+#pragma unroll
+            for (int j = 0; j < kBatch; ++j) {
+                const int t = tb + 32 * j;
+                m[j] = (t < NQB && w < words) ? bb[(size_t)t * words + w] : 0u;
+            }
+#pragma unroll
+            for (int j = 0; j < kBatch; ++j) {
+                const int c = __popc(m[j]);
+                int x = c;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, x, off);
+                    if (lane >= off) x += y;
+                }
+                int o = pos[j] + x - c;
+                uint32_t mm = m[j];
+                while (mm) {
+                    const int q = w * 32 + __ffs(mm) - 1;
+                    mm &= mm - 1;
+                    if (o < cap) ql[o] = q;
+                    ++o;
+                }
+                pos[j] += __shfl_sync(0xffffffffu, x, 31);
+            }
+        }
     }
 }
 
@@ -585,6 +622,7 @@ BwdLayout bwd_layout(const phsa_shape& s, int topk) {
     l.nwork = off;   off = align256(off + (size_t)bgs * 4);
     l.delta = off;   off = align256(off + (size_t)s.B * s.Hq * s.L * 4);
     l.partial = off; off = align256(off + (size_t)bgs * l.slot_max * 2 * kM * kD * 4);
+    l.arrive = off;  off = align256(off + (size_t)bgs * l.nqb * 4);
     l.total = off;
     return l;
 }
@@ -604,11 +642,19 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     int32_t* nwork = reinterpret_cast<int32_t*>(w + l.nwork);
     float* delta = reinterpret_cast<float*>(w + l.delta);
     float* partial = reinterpret_cast<float*>(w + l.partial);
+    int* arrive = reinterpret_cast<int*>(w + l.arrive);
     const int bgs = s.B * s.Hkv;
     const long long rows = (long long)s.B * s.Hq * s.L;
     cudaError_t e;
 
-    {
+    // Two query heads per KV head: tcgen05 kernels (M = 128 rows per MMA), as
+    // long as the block list fits beside dq_tc_kernel's tiles.
+    const bool pair = s.Hq / s.Hkv == 2 && dq_tc_fits(topk);
+    if (pair) {
+        // dQ first: it also computes Delta from O and dO, which dK/dV then read.
+        e = launch_dq_tc(Q, K, V, O, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
+        if (e != cudaSuccess) return e;
+    } else {
         ProfScope prof(K_BWD_DELTA, st);
         delta_kernel<<<(unsigned)((rows * 16 + 255) / 256), 256, 0, st>>>(
             static_cast<const __nv_bfloat16*>(O), static_cast<const __nv_bfloat16*>(dO), rows,
@@ -628,16 +674,16 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     {
         ProfScope prof(K_BWD_BUILD, st);
         idx_build_kernel<<<bgs, 1024, 0, st>>>(bits, l.nqb, topk, l.words, l.work_max,
-                                               l.slot_max, tinfo, qlist, work, nwork, status);
+                                               l.slot_max, tinfo, qlist, work, nwork, arrive,
+                                               status);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
-    const bool pair = s.Hq / s.Hkv == 2;  // two query heads per KV head: tcgen05 kernels
-    if (pair) {
-        e = launch_dkdv_tc(Q, K, V, dO, lse, delta, tinfo, qlist, work, nwork, s, topk,
-                           l.work_max, l.slot_max, sm_scale, dK, dV, partial, status, st);
-        if (e != cudaSuccess) return e;
-    } else {
+    if (pair)  // sums multi-chunk partials itself
+        return launch_dkdv_tc(Q, K, V, dO, lse, delta, tinfo, qlist, work, nwork, s, topk,
+                              l.work_max, l.slot_max, sm_scale, dK, dV, partial, arrive, status,
+                              st);
+
     e = cudaFuncSetAttribute(dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kKvSmem);
     if (e != cudaSuccess) return e;
     {
@@ -650,7 +696,6 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
             static_cast<__nv_bfloat16*>(dV), partial);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
     {
         ProfScope prof(K_BWD_DKDV_SUM, st);
         dkdv_sum_kernel<<<dim3(l.nqb, bgs), 256, 0, st>>>(
@@ -658,9 +703,9 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
             static_cast<__nv_bfloat16*>(dV));
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-
-    return pair ? launch_dq_tc(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st)
-                : launch_dq_g<1>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
+    return s.Hq == s.Hkv
+               ? launch_dq_g<1>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st)
+               : launch_dq_g<2>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
 }
 
 }  // namespace phsa

@@ -10,7 +10,10 @@
 //     dS_p = P_p (dP_p - Delta), P_p = exp(S_p * scale - lse)   (8 warps, TMEM)
 //     dQ  += dS_p Kp      (M128 N128 K128, A = dS_p in TMEM, B = Kp MN-major)
 //   S is double-buffered in TMEM, so S_{p+1} runs while the elementwise warps
-//   work on pair p. dQ * scale -> TMA store.
+//   work on pair p. dQ * scale -> TMA store. Before the first pair the
+//   elementwise warps compute Delta_i = dO_i . O_i (O read from global memory,
+//   dO from the loaded tile) and write it for the dK/dV kernel, which runs
+//   after this one.
 //
 // dkdv_tc_kernel: one CTA per work item (KV block t, chunk of <= 32 query
 //   blocks that selected t), 320 threads. K_t and V_t stay in shared memory;
@@ -22,7 +25,9 @@
 //                                             MN-major, B = P / dS MN-major)
 //   dK^T and dV^T live in TMEM with the head dimension on the lanes. A KV
 //   block with a single chunk writes bf16 dK, dV through TMA stores; a longer
-//   list writes fp32 partials that dkdv_sum (attn_bwd.cu) adds in chunk order.
+//   list writes fp32 partials, and the chunk that finishes last (an atomic
+//   counter per KV block) adds them in chunk order and stores the bf16 tile, so
+//   the sum does not depend on which CTA finishes last.
 //
 // Every wait is bounded in time; on expiry the kernel records
 // PHSA_ERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
@@ -61,7 +66,8 @@ constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = B_KFULL + kKSlots, B_VFULL = B_KE
               B_DPFREE = B_DSFULL + 2, B_FINAL = B_DPFREE + 1, B_DRAIN = B_FINAL + 1,
               kNumBars = B_DRAIN + 1;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
-constexpr int kOffList = kOffMisc + 16;
+constexpr int kOffDPart = kOffMisc + 16;  // Delta of the 128 rows, fp32
+constexpr int kOffList = kOffDPart + 128 * 4;
 constexpr int kThreads = 352;  // 8 elementwise warps, K/Q/dO producer, MMA, V producer
 // TMEM: dQ [0,128), S of pair buffer b at [128 + 128b, +128), dP [384, 512).
 // dS of key half h overwrites S columns [64h, 64h + 32) (read by the same thread).
@@ -74,7 +80,8 @@ struct DqArgs {
     const int32_t* idx;
     const int32_t* cnt;
     const float* lse;
-    const float* delta;
+    const __nv_bfloat16* O;
+    float* delta;  // written: Delta_i = dO_i . O_i for every valid row
     int* status;
     int Hq, Hkv, L, NQB, topk;
     float scale_log2, sm_scale;
@@ -265,9 +272,49 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         const bool valid = i < a.L;
         const size_t ridx = (size_t)(hq0 + hl) * a.L + (valid ? i : 0);
         const float neg_lse2 = valid ? -a.lse[ridx] * kLog2e : -INFINITY;
-        const float dlt = valid ? a.delta[ridx] : 0.f;
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-        bool ok = true;
+        // Delta_i = dO_i . O_i, computed before the first pair: O is read from
+        // global memory in coalesced 16-byte pieces (16 threads per 256-byte
+        // row, 8 rows per pass), dO from the tile loaded for the dP MMAs; the 16
+        // partial dot products of a row are added by a fixed shuffle tree.
+        const int et = threadIdx.x;  // 0..255 over the elementwise warps
+        const int pc = et & 15;      // 16-byte piece of the row
+        uint4 ov[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int rr = k * 16 + (et >> 4);
+            const int ii = qb * 64 + (rr & 63);
+            ov[k] = ii < a.L ? __ldg(reinterpret_cast<const uint4*>(
+                                   a.O + ((size_t)(hq0 + (rr >> 6)) * a.L + ii) * 128) + pc)
+                             : make_uint4(0u, 0u, 0u, 0u);
+        }
+        bool ok = n == 0 || mbar_wait(bar(B_Q), 0, abort_flag, a.status);
+        ok = __all_sync(0xffffffffu, ok);
+        float* dpart = reinterpret_cast<float*>(smem + kOffDPart);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int rr = k * 16 + (et >> 4);
+            float acc = 0.f;
+            if (ok && n > 0) {
+                const uint4 dv = *reinterpret_cast<const uint4*>(
+                    smem + kOffDO + (pc >> 3) * kHalf128 + (rr >> 6) * kHalf64 + sw_off(rr & 63, pc & 7));
+                const uint32_t ow[4] = {ov[k].x, ov[k].y, ov[k].z, ov[k].w};
+                const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float2 fo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ow[j]));
+                    const float2 fd = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&dw[j]));
+                    acc = fmaf(fo.x, fd.x, acc);
+                    acc = fmaf(fo.y, fd.y, acc);
+                }
+            }
+#pragma unroll
+            for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+            if (pc == 0) dpart[rr] = acc;
+        }
+        named_barrier(1, 256);
+        const float dlt = dpart[row];
+        if (half == 0 && valid) a.delta[ridx] = dlt;
         for (int p = 0; p < np; ++p) {
             const int buf = p & 1;
             ok = mbar_wait(bar(B_SPFULL + buf), (p >> 1) & 1, abort_flag, a.status);
@@ -373,6 +420,7 @@ struct KvArgs {
     const int2* work;
     const int32_t* nwork;
     float* partial;
+    int* arrive;  // per (b, g, t): chunks of t finished so far
     int* status;
     int Hq, Hkv, L, NQB, topk, work_max, slot_max;
     float scale_log2, sm_scale;
@@ -604,9 +652,14 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
             for (int c = 0; c < 32; ++c) { v[c] = 0u; k[c] = 0u; }
         }
+        bool store = ok;
         if (info.nch > 1) {
+            // Multi-chunk list: write this chunk's fp32 partial; the chunk that
+            // arrives last adds all partials in chunk order and stores the tile.
+            float* base = a.partial + ((size_t)bg * a.slot_max + (info.slot < 0 ? 0 : info.slot)) *
+                                          2 * 64 * 128;
             if (ok && info.slot >= 0) {
-                float* pk = a.partial + ((size_t)bg * a.slot_max + info.slot + chunk) * 2 * 64 * 128;
+                float* pk = base + (size_t)chunk * 2 * 64 * 128;
                 float* pv = pk + 64 * 128;
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
@@ -615,8 +668,39 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     pv[key * 128 + d] = __uint_as_float(v[c]);
                 }
             }
-        } else if (ok) {
-            // bf16 tiles [64 keys][128 d] in the swizzled layout (stage-0 Q and dO regions)
+            __threadfence();
+            named_barrier(1, 256);
+            volatile int* last_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 8);
+            if (threadIdx.x == 0)
+                *last_flag = (info.slot >= 0 &&
+                              atomicAdd(a.arrive + (size_t)bg * a.NQB + t, 1) == info.nch - 1);
+            named_barrier(1, 256);
+            store = ok && *last_flag;
+            if (store) {
+                __threadfence();
+                float sk[32], sv2[32];
+#pragma unroll
+                for (int c = 0; c < 32; ++c) { sk[c] = 0.f; sv2[c] = 0.f; }
+                for (int ch = 0; ch < info.nch; ++ch) {
+                    const float* pk = base + (size_t)ch * 2 * 64 * 128;
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) {
+                        const int key = 32 * kh + c;
+                        sk[c] += __ldcg(pk + key * 128 + d);
+                        sv2[c] += __ldcg(pk + 64 * 128 + key * 128 + d);
+                    }
+                }
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    k[c] = __float_as_uint(sk[c]);
+                    v[c] = __float_as_uint(sv2[c]);
+                }
+            }
+        }
+        if (store) {
+            // bf16 tiles [64 keys][128 d] in the swizzled layout (stage-0 Q and dO
+            // regions); partial sums already carry the softmax scale.
+            const float kscale = info.nch > 1 ? 1.f : a.sm_scale;
             uint8_t* tv = smem + kOffStage;
             uint8_t* tk = smem + kOffStage + kTile128;
             const int dh = d >> 6, dc = (d & 63) >> 3, de = d & 7;
@@ -626,12 +710,12 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const uint32_t off = dh * kHalf64 + sw_off(key, dc) + de * 2;
                 *reinterpret_cast<__nv_bfloat16*>(tv + off) = __float2bfloat16_rn(__uint_as_float(v[c]));
                 *reinterpret_cast<__nv_bfloat16*>(tk + off) =
-                    __float2bfloat16_rn(__uint_as_float(k[c]) * a.sm_scale);
+                    __float2bfloat16_rn(__uint_as_float(k[c]) * kscale);
             }
             fence_proxy_async_smem();
         }
         named_barrier(1, 256);
-        if (threadIdx.x == 0 && ok && info.nch <= 1) {
+        if (threadIdx.x == 0 && store) {
             for (int dh = 0; dh < 2; ++dh) {
                 tma_store_3d(&tmdV, sb + kOffStage + dh * kHalf64, dh * 64, t * 64, bg);
                 tma_store_3d(&tmdK, sb + kOffStage + kTile128 + dh * kHalf64, dh * 64, t * 64, bg);
@@ -650,8 +734,10 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 
 }  // namespace
 
-cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* dO,
-                         const float* lse, const float* delta, const int32_t* idx,
+bool dq_tc_fits(int topk) { return dq::smem_bytes(topk) <= 227u * 1024u; }
+
+cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* O,
+                         const void* dO, const float* lse, float* delta, const int32_t* idx,
                          const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                          void* dQ, int* status, cudaStream_t st) {
     const int NQB = (s.L + 63) / 64;
@@ -665,7 +751,7 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
     cudaError_t e =
         cudaFuncSetAttribute(dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    DqArgs args{idx, cnt, lse, delta, status, s.Hq, s.Hkv, s.L, NQB, topk, sm_scale * kLog2e,
+    DqArgs args{idx, cnt, lse, static_cast<const __nv_bfloat16*>(O), delta, status, s.Hq, s.Hkv, s.L, NQB, topk, sm_scale * kLog2e,
                 sm_scale};
     ProfScope prof(K_BWD_DQ, st);
     dq_tc_kernel<<<(unsigned)((long long)s.B * s.Hkv * NQB), dq::kThreads, smem, st>>>(
@@ -677,8 +763,8 @@ cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const vo
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
                            const int32_t* qlist, const int2* work, const int32_t* nwork,
                            const phsa_shape& s, int topk, int work_max, int slot_max,
-                           float sm_scale, void* dK, void* dV, float* partial, int* status,
-                           cudaStream_t st) {
+                           float sm_scale, void* dK, void* dV, float* partial, int* arrive,
+                           int* status, cudaStream_t st) {
     const int NQB = (s.L + 63) / 64;
     CUtensorMap tq, tk, tv, tdo, tdk, tdv;
     const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
@@ -689,7 +775,7 @@ cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const vo
     cudaError_t e = cudaFuncSetAttribute(dkdv_tc_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kv::kSmem);
     if (e != cudaSuccess) return e;
-    KvArgs args{lse, delta, tinfo, qlist, work, nwork, partial, status, s.Hq, s.Hkv, s.L, NQB,
+    KvArgs args{lse, delta, tinfo, qlist, work, nwork, partial, arrive, status, s.Hq, s.Hkv, s.L, NQB,
                 topk, work_max, slot_max, sm_scale * kLog2e, sm_scale};
     ProfScope prof(K_BWD_DKDV, st);
     dkdv_tc_kernel<<<dim3(work_max, s.B * s.Hkv), kv::kThreads, kv::kSmem, st>>>(tq, tk, tv, tdo,

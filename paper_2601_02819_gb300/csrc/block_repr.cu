@@ -8,6 +8,8 @@
 // bytes. The sum and the punctuation-masked sum are kept in fp32 and combined
 // once across the two half-warps; the result is rounded to bf16 once.
 // The kernel is bound by HBM: it reads K and the mask once and writes T rows.
+// decode_repr_kernel reuses the per-block routine for the block a decode step
+// has just filled (block-level caching of the representative keys).
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 
@@ -27,26 +29,19 @@ __device__ __forceinline__ void add8(float* acc, const uint4& v) {
     }
 }
 
-__global__ void __launch_bounds__(kWarpsPerCta * 32)
-block_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict__ mask, int Hkv,
-                  int L, int T, long long n_blocks, float lambda,
-                  __nv_bfloat16* __restrict__ Krepr) {
-    const int lane = threadIdx.x & 31;
-    const long long wid = (long long)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
-    if (wid >= n_blocks) return;
-    const int t = (int)(wid % T);
-    const long long bg = wid / T;  // b * Hkv + g
-    const int b = (int)(bg / Hkv);
-
+// One warp: the representative key of the 64 x 128 block at Kb (row stride 128)
+// with punctuation bytes mb[0..64), written as 128 bf16 values to out.
+__device__ __forceinline__ void repr_one_block(const __nv_bfloat16* __restrict__ Kb,
+                                               const uint8_t* __restrict__ mb, float lambda,
+                                               __nv_bfloat16* __restrict__ out, int lane) {
     // Punctuation indicator of the block's 64 tokens.
-    const uint8_t* mrow = mask + (size_t)b * L + (size_t)t * kM;
-    const unsigned lo = __ballot_sync(0xffffffffu, mrow[lane] != 0);
-    const unsigned hi = __ballot_sync(0xffffffffu, mrow[32 + lane] != 0);
+    const unsigned lo = __ballot_sync(0xffffffffu, mb[lane] != 0);
+    const unsigned hi = __ballot_sync(0xffffffffu, mb[32 + lane] != 0);
     const int c = __popc(lo) + __popc(hi);
 
     const int half = lane >> 4;
     const int col = lane & 15;
-    const __nv_bfloat16* kb = K + ((size_t)bg * L + (size_t)t * kM) * kD + col * 8;
+    const __nv_bfloat16* kb = Kb + col * 8;
 
     float s0[8], sp[8];
 #pragma unroll
@@ -74,22 +69,58 @@ block_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict
         sp[j] += __shfl_xor_sync(0xffffffffu, sp[j], 16);
     }
     if (half == 0) {
-        float out[8];
+        float o[8];
         const float inv_m = 1.0f / kM;
         const float inv_c = c > 0 ? 1.0f / (float)c : 0.f;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
             const float m0 = s0[j] * inv_m;                                // Eq. 6
-            out[j] = c > 0 ? lambda * m0 + (1.0f - lambda) * (sp[j] * inv_c)  // Eq. 7-8
-                           : m0;                                           // no punctuation
+            o[j] = c > 0 ? lambda * m0 + (1.0f - lambda) * (sp[j] * inv_c)  // Eq. 7-8
+                         : m0;                                           // no punctuation
         }
         uint4 pk;
-        pk.x = pack_bf16(out[0], out[1]);
-        pk.y = pack_bf16(out[2], out[3]);
-        pk.z = pack_bf16(out[4], out[5]);
-        pk.w = pack_bf16(out[6], out[7]);
-        *reinterpret_cast<uint4*>(Krepr + ((size_t)bg * T + t) * kD + col * 8) = pk;
+        pk.x = pack_bf16(o[0], o[1]);
+        pk.y = pack_bf16(o[2], o[3]);
+        pk.z = pack_bf16(o[4], o[5]);
+        pk.w = pack_bf16(o[6], o[7]);
+        *reinterpret_cast<uint4*>(out + col * 8) = pk;
     }
+}
+
+__global__ void __launch_bounds__(kWarpsPerCta * 32)
+block_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict__ mask, int Hkv,
+                  int L, int T, long long n_blocks, float lambda,
+                  __nv_bfloat16* __restrict__ Krepr) {
+    const int lane = threadIdx.x & 31;
+    const long long wid = (long long)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
+    if (wid >= n_blocks) return;
+    const int t = (int)(wid % T);
+    const long long bg = wid / T;  // b * Hkv + g
+    const int b = (int)(bg / Hkv);
+    repr_one_block(K + ((size_t)bg * L + (size_t)t * kM) * kD, mask + (size_t)b * L + (size_t)t * kM,
+                   lambda, Krepr + ((size_t)bg * T + t) * kD, lane);
+}
+
+// Decode: one warp per (sequence, KV head). A sequence whose length is a
+// positive multiple of m has just filled its last block: that block's
+// representative key is computed; nothing else is touched.
+__global__ void __launch_bounds__(kWarpsPerCta * 32)
+decode_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict__ mask,
+                   const int32_t* __restrict__ lens, int Hkv, int L, int T, long long n_units,
+                   float lambda, __nv_bfloat16* __restrict__ Krepr, int* status) {
+    const int lane = threadIdx.x & 31;
+    const long long bg = (long long)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
+    if (bg >= n_units) return;
+    const int b = (int)(bg / Hkv);
+    const int len = lens[b];
+    if (len < 0 || len > L) {
+        if (lane == 0) set_status(status, PHSA_ERR_DEVICE_INDEX);
+        return;
+    }
+    if (len == 0 || len % kM != 0) return;
+    const int t = len / kM - 1;
+    repr_one_block(K + ((size_t)bg * L + (size_t)t * kM) * kD, mask + (size_t)b * L + (size_t)t * kM,
+                   lambda, Krepr + ((size_t)bg * T + t) * kD, lane);
 }
 
 }  // namespace
@@ -104,6 +135,24 @@ cudaError_t launch_block_repr(const void* K, const uint8_t* mask, const phsa_sha
     block_repr_kernel<<<(unsigned)grid, kWarpsPerCta * 32, 0, st>>>(
         static_cast<const __nv_bfloat16*>(K), mask, s.Hkv, s.L, T, n_blocks, lambda,
         static_cast<__nv_bfloat16*>(Krepr));
+    return cudaGetLastError();
+}
+
+}  // namespace phsa
+
+namespace phsa {
+
+cudaError_t launch_decode_repr(const void* K, const uint8_t* mask, const int32_t* lens,
+                               const phsa_shape& s, float lambda, void* Krepr, int* status,
+                               cudaStream_t st) {
+    const int T = s.L / kM;
+    const long long n_units = (long long)s.B * s.Hkv;
+    if (n_units == 0 || T == 0) return cudaSuccess;
+    const long long grid = (n_units + kWarpsPerCta - 1) / kWarpsPerCta;
+    ProfScope prof(K_DEC_REPR, st);
+    decode_repr_kernel<<<(unsigned)grid, kWarpsPerCta * 32, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(K), mask, lens, s.Hkv, s.L, T, n_units, lambda,
+        static_cast<__nv_bfloat16*>(Krepr), status);
     return cudaGetLastError();
 }
 

@@ -144,6 +144,59 @@ int phsa_sparse_attn_bwd(const void* Q, const void* K, const void* V, const void
                                            static_cast<cudaStream_t>(stream)));
 }
 
+int phsa_decode_update_repr(const void* K, const uint8_t* punct_mask, const int32_t* seq_lens,
+                            phsa_shape s, float lambda, void* Krepr, void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
+    if (empty(s) || s.L < phsa::kM) return PHSA_OK;  // no block can fill
+    if (!K || !punct_mask || !seq_lens || !Krepr || !aligned16(K) || !aligned16(Krepr))
+        return PHSA_ERR_INVALID_ARG;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_decode_repr(K, punct_mask, seq_lens, s, lambda, Krepr, st,
+                                              static_cast<cudaStream_t>(stream)));
+}
+
+int phsa_decode_select(const void* q, const void* Krepr, const int32_t* seq_lens, phsa_shape s,
+                       phsa_select_params p, int32_t* block_idx, int32_t* block_cnt,
+                       void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
+    if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
+    if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
+    if (empty(s)) return PHSA_OK;
+    const bool need_repr = s.L >= 2 * phsa::kM;  // some length can have a candidate
+    if (!q || !seq_lens || !block_idx || !block_cnt || !aligned16(q) ||
+        (need_repr && (!Krepr || !aligned16(Krepr))))
+        return PHSA_ERR_INVALID_ARG;
+    if (phsa::decode_select_smem_bytes(s, p.topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_decode_select(q, Krepr, seq_lens, s, p, block_idx, block_cnt, st,
+                                                static_cast<cudaStream_t>(stream)));
+}
+
+int phsa_decode_attn(const void* q, const void* K, const void* V, const int32_t* block_idx,
+                     const int32_t* block_cnt, const int32_t* seq_lens, phsa_shape s, int topk,
+                     float sm_scale, void* O, float* lse, void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = check_topk(s, topk)) != PHSA_OK) return rc;
+    if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;
+    if (s.B == 0) return PHSA_OK;
+    if (!q || !K || !V || !block_idx || !block_cnt || !seq_lens || !O || !lse)
+        return PHSA_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
+        return PHSA_ERR_INVALID_ARG;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, s, topk,
+                                              sm_scale, O, lse, st,
+                                              static_cast<cudaStream_t>(stream)));
+}
+
 int phsa_get_device_status(void* stream) {
     if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
         return PHSA_ERR_CUDA;

@@ -14,7 +14,7 @@ namespace phsa {
 // Kernel identities for the optional per-kernel timing (profile.cu).
 enum KernelId {
     K_REPR = 0, K_SELECT, K_FWD, K_BWD_DELTA, K_BWD_MARK, K_BWD_BUILD, K_BWD_DKDV,
-    K_BWD_DKDV_SUM, K_BWD_DQ, K_COUNT
+    K_BWD_DKDV_SUM, K_BWD_DQ, K_DEC_REPR, K_DEC_SELECT, K_DEC_ATTN, K_COUNT
 };
 void prof_begin(int kid, cudaStream_t st);
 void prof_end(int kid, cudaStream_t st);
@@ -29,6 +29,20 @@ struct ProfScope {
 
 cudaError_t launch_block_repr(const void* K, const uint8_t* mask, const phsa_shape& s,
                               float lambda, void* Krepr, cudaStream_t st);
+
+// Decode (one new token per sequence): repr of the block just filled, the
+// selection and the attention of the newest token (decode.cu, block_repr.cu).
+cudaError_t launch_decode_repr(const void* K, const uint8_t* mask, const int32_t* lens,
+                               const phsa_shape& s, float lambda, void* Krepr, int* status,
+                               cudaStream_t st);
+size_t decode_select_smem_bytes(const phsa_shape& s, int topk);
+cudaError_t launch_decode_select(const void* q, const void* Krepr, const int32_t* lens,
+                                 const phsa_shape& s, const phsa_select_params& p, int32_t* idx,
+                                 int32_t* cnt, int* status, cudaStream_t st);
+cudaError_t launch_decode_attn(const void* q, const void* K, const void* V, const int32_t* idx,
+                               const int32_t* cnt, const int32_t* lens, const phsa_shape& s,
+                               int topk, float sm_scale, void* O, float* lse, int* status,
+                               cudaStream_t st);
 
 cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape& s,
                              const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,
@@ -65,16 +79,18 @@ cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const vo
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
                            const int32_t* qlist, const int2* work, const int32_t* nwork,
                            const phsa_shape& s, int topk, int work_max, int slot_max,
-                           float sm_scale, void* dK, void* dV, float* partial, int* status,
-                           cudaStream_t st);
-cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* dO,
-                         const float* lse, const float* delta, const int32_t* idx,
+                           float sm_scale, void* dK, void* dV, float* partial, int* arrive,
+                           int* status, cudaStream_t st);
+// Whether dq_tc_kernel's shared memory (tiles + the block list) fits for topk.
+bool dq_tc_fits(int topk);
+cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* O,
+                         const void* dO, const float* lse, float* delta, const int32_t* idx,
                          const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                          void* dQ, int* status, cudaStream_t st);
 
 // Backward workspace layout (all offsets 256-byte aligned).
 struct BwdLayout {
-    size_t bits, tinfo, qlist, work, nwork, delta, partial, total;
+    size_t bits, tinfo, qlist, work, nwork, delta, partial, arrive, total;
     int nqb, words, chunk, work_max, slot_max;
 };
 BwdLayout bwd_layout(const phsa_shape& s, int topk);

@@ -14,7 +14,8 @@ namespace {
 
 const char* const kNames[K_COUNT] = {
     "block_repr", "select_blocks", "attn_fwd", "bwd_delta", "bwd_idx_mark",
-    "bwd_idx_build", "bwd_dkdv", "bwd_dkdv_sum", "bwd_dq",
+    "bwd_idx_build", "bwd_dkdv", "bwd_dkdv_sum", "bwd_dq", "decode_repr", "decode_select",
+    "decode_attn",
 };
 
 struct Record {

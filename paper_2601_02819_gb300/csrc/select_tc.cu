@@ -14,13 +14,14 @@
 //           sum p = 2^(S*scale - m_r)/Z_r over their 64 rows in row order;
 //           A[t] = half 0 + half 1. Every candidate follows the same order,
 //           so equal candidates get bit-identical sums.
-//   top-k   one warp: rounds of a warp-wide argmax over the 64-bit key
-//           (bits(A) << 32 | ~t): larger A first, lower t on exact ties.
+//   top-k   over the 64-bit key (bits(A) << 32 | ~t): larger A first, lower
+//           t on exact ties; two levels over the 8 warps (topk.cuh).
 // Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs.
 // Every wait is bounded in time (tc_common.cuh).
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "tc_common.cuh"
+#include "topk.cuh"
 
 namespace phsa {
 
@@ -38,7 +39,8 @@ constexpr int kOffBar = kOffStats + 6 * 128 * 4;
 constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = 3, B_SFULL = 5, B_SFREE = 7, B_DRAIN = 9,
               kNumBars = 10;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
-constexpr int kOffA = kOffMisc + 16;              // A0[NQB], A1[NQB], then sel[topk]
+constexpr int kOffFin = kOffMisc + 48;            // top-k finalist keys [8 warps][kFinalMax], u64
+constexpr int kOffA = kOffFin + 8 * topk::kFinalMax * 8;  // A0[NQB], A1[NQB], then sel[topk]
 constexpr int kThreads = 320;
 constexpr uint32_t kTmemCols = 256;
 
@@ -53,10 +55,6 @@ struct SelArgs {
     int Hq, Hkv, L, T, NQB, topk, n_init, n_local;
     float scale_log2;
 };
-
-__device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {
-    return a > b ? a : b;
-}
 
 __global__ void __launch_bounds__(kThreads, 2)
 select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKr,
@@ -205,6 +203,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 const bool full = t0 + 63 <= c_hi;
 #pragma unroll 1
                 for (int q = 0; q < 2; ++q) {
+                    if (t0 + 32 * q > c_hi) break;  // no candidate left in this group (warp-uniform)
                     uint32_t v[32];
                     tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
                     float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
@@ -227,12 +226,14 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 tc_fence_before();
                 mbar_arrive(bar(B_SFREE + slot));
             } else if (ok) {
-                // pass 2: candidate r against the 64 rows of half hh, in row order
+                // pass 2: candidate r against the 64 rows of half hh, in row order;
+                // a warp whose 32 candidates all lie past the last one skips the work
                 const float* mrow = m2s + 64 * hh;
                 const float* irow = izs + 64 * hh;
                 float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                const bool live = c * kCand + (warp & 3) * 32 < nC;
 #pragma unroll 1
-                for (int q = 0; q < 2; ++q) {
+                for (int q = 0; q < (live ? 2 : 0); ++q) {
                     uint32_t v[32];
                     tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
 #pragma unroll
@@ -268,38 +269,21 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             }
         }
         named_barrier(1, 256);  // every A0/A1 entry written
-        if (ok && warp == 0) {
-            // top-k: lane l owns candidates l, l+32, ...; its best untaken key is cached.
-            // A = half 0 + half 1 (the same order for every candidate); taken: A0 = -1.
-            auto lane_best = [&]() {
-                unsigned long long best = 0ull;
-                for (int cj = lane; cj < nC; cj += 32) {
-                    const float a0 = A0[cj];
-                    if (a0 >= 0.f) {
-                        float v = a0 + A1[cj];
-                        if (!(v >= 0.f)) v = 0.f;  // NaN inputs rank as zero
-                        best = umax64(best, ((unsigned long long)__float_as_uint(v) << 32) |
-                                                (unsigned long long)(0xffffffffu - (unsigned)(c_lo + cj)));
-                    }
-                }
-                return best;
-            };
-            unsigned long long mine = lane_best();
-            for (int k = 0; k < ksel; ++k) {
-                unsigned long long best = mine;
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, off));
-                // every untaken candidate has a nonzero key, so best != 0 while k < ksel < nC
-                const int t = best ? (int)(0xffffffffu - (unsigned)(best & 0xffffffffull)) : c_lo;
-                if (lane == 0) sel[k] = t;
-                const int cj = t - c_lo;
-                if (best && (cj & 31) == lane) {
-                    A0[cj] = -1.0f;
-                    mine = lane_best();
-                }
-                __syncwarp();
-            }
+        // top-k (topk.cuh): key = bits(A) << 32 | ~t with A = half 0 + half 1 (the
+        // same order for every candidate); a taken candidate is marked A0 = -1
+        // on the one-warp path.
+        auto key_of = [&](int cj) { return topk::make_key(A0[cj] + A1[cj], c_lo + cj); };
+        unsigned long long* fin = reinterpret_cast<unsigned long long*>(smem + kOffFin);
+        const bool fast = topk::two_level(nC, ksel);
+        if (ok && fast) {
+            topk::level1(nC, ksel, key_of, fin, warp, lane);
+        } else if (ok && warp == 0) {
+            topk::rounds_one_warp(
+                nC, ksel, key_of, [&](int cj) { return A0[cj] == -1.0f; },
+                [&](int t) { A0[t - c_lo] = -1.0f; }, sel, lane);
         }
+        named_barrier(1, 256);
+        if (ok && fast) topk::level2(fin, ksel, sel, threadIdx.x);
         named_barrier(1, 256);
         if (ok) {
             for (int j = threadIdx.x; j < a.topk; j += 256) {
@@ -307,8 +291,8 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 else if (j >= n_init_q + ksel && j < nF + ksel) out[j] = loc_lo + (j - n_init_q - ksel);
                 else if (j >= nF + ksel) out[j] = -1;
             }
-            if (threadIdx.x < ksel) {
-                const int v = sel[threadIdx.x];
+            for (int j = threadIdx.x; j < ksel; j += 256) {
+                const int v = sel[j];
                 int rank = 0;
                 for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
                 out[n_init_q + rank] = v;

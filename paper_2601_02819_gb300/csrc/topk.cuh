@@ -1,0 +1,123 @@
+// Top-k block choice shared by the selection kernels (Algorithm 1 step 3):
+// the k candidates with the largest aggregate A, ties to the lower block index.
+//
+// Every candidate gets the 64-bit key bits(A) << 32 | ~t (A >= 0, so the bit
+// pattern orders like the value; NaN ranks as zero), and keys are distinct.
+//
+// Two levels over 8 warps (256 threads):
+//   level1  each warp takes an eighth of the candidates, keeps its lanes' keys
+//           in registers (at most kLaneKeys per lane) and picks its best
+//           min(k, slice) by rounds of a warp-wide maximum; the winners go to
+//           fin[warp][0..), the remaining slots stay 0.
+//   level2  each finalist counts the finalists with a larger key; rank < k is
+//           a pick. The global top k are all finalists, since each of them is
+//           within the top k of its own slice.
+// Budgets above kFinalMax picks, or more than 8 * 32 * kLaneKeys candidates,
+// take one warp's rounds over all candidates instead (rounds_one_warp).
+#pragma once
+
+#include <cstdint>
+
+namespace phsa {
+namespace topk {
+
+constexpr int kFinalMax = 32;  // picks handled by the two-level path
+constexpr int kLaneKeys = 8;   // candidate keys per lane in level 1
+constexpr int kMaxCand = 8 * 32 * kLaneKeys;
+
+__device__ __forceinline__ unsigned long long make_key(float a, int t) {
+    if (!(a >= 0.f)) a = 0.f;
+    return ((unsigned long long)__float_as_uint(a) << 32) |
+           (unsigned long long)(0xffffffffu - (unsigned)t);
+}
+
+__device__ __forceinline__ int key_block(unsigned long long key) {
+    return (int)(0xffffffffu - (unsigned)(key & 0xffffffffull));
+}
+
+__device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {
+    return a > b ? a : b;
+}
+
+__device__ __forceinline__ bool two_level(int nC, int ksel) {
+    return ksel <= kFinalMax && nC <= kMaxCand;
+}
+
+// Level 1, called by each of the 8 warps with its warp index; key_of(cj) gives
+// the key of candidate cj in [0, nC). fin holds 8 * kFinalMax keys.
+template <class KeyOf>
+__device__ __forceinline__ void level1(int nC, int ksel, KeyOf key_of, unsigned long long* fin,
+                                       int warp, int lane) {
+    const int per = (nC + 7) >> 3;
+    const int lo = min(nC, warp * per), hi = min(nC, lo + per);
+    const int nf = min(ksel, hi - lo);
+    unsigned long long key[kLaneKeys];
+#pragma unroll
+    for (int r = 0; r < kLaneKeys; ++r) {
+        const int cj = lo + lane + 32 * r;
+        key[r] = cj < hi ? key_of(cj) : 0ull;
+    }
+    for (int k = lane; k < kFinalMax; k += 32) fin[warp * kFinalMax + k] = 0ull;
+    __syncwarp();
+    for (int k = 0; k < nf; ++k) {
+        unsigned long long best = key[0];
+#pragma unroll
+        for (int r = 1; r < kLaneKeys; ++r) best = umax64(best, key[r]);
+        const unsigned mh = (unsigned)(best >> 32), ml = (unsigned)best;
+        const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
+        const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
+        const unsigned long long win = ((unsigned long long)bh << 32) | bl;
+        if (lane == 0) fin[warp * kFinalMax + k] = win;
+#pragma unroll
+        for (int r = 0; r < kLaneKeys; ++r)
+            if (key[r] == win) key[r] = 0ull;
+    }
+}
+
+// Level 2, called by all 256 threads after level 1 is visible to them: writes
+// the block index of the pick of rank r to sel[r], r < ksel.
+__device__ __forceinline__ void level2(const unsigned long long* fin, int ksel, int* sel,
+                                       int tid) {
+    const unsigned long long mykey = tid < 8 * kFinalMax ? fin[tid] : 0ull;
+    if (mykey == 0ull) return;
+    int rank = 0;
+    const int pairs = (ksel + 1) >> 1;  // finalists sit at the front of each warp's slots
+    for (int w = 0; w < 8; ++w) {
+        const ulonglong2* f2 = reinterpret_cast<const ulonglong2*>(fin + w * kFinalMax);
+#pragma unroll 4
+        for (int j = 0; j < pairs; ++j) {
+            const ulonglong2 v = f2[j];
+            rank += (v.x > mykey) + (v.y > mykey);
+        }
+    }
+    if (rank < ksel) sel[rank] = key_block(mykey);
+}
+
+// One warp, any budget: rounds over all candidates; taken(cj) / take(cj) mark a
+// candidate as chosen (the caller's storage). sel[k] = k-th pick.
+template <class KeyOf, class Taken, class Take>
+__device__ __forceinline__ void rounds_one_warp(int nC, int ksel, KeyOf key_of, Taken taken,
+                                                Take take, int* sel, int lane) {
+    auto lane_best = [&]() {
+        unsigned long long best = 0ull;
+        for (int cj = lane; cj < nC; cj += 32)
+            if (!taken(cj)) best = umax64(best, key_of(cj));
+        return best;
+    };
+    unsigned long long mine = lane_best();
+    for (int k = 0; k < ksel; ++k) {
+        const unsigned mh = (unsigned)(mine >> 32), ml = (unsigned)mine;
+        const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
+        const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
+        const unsigned long long win = ((unsigned long long)bh << 32) | bl;
+        if (lane == 0) sel[k] = key_block(win);
+        if (bl != 0u && mine == win) {
+            take(key_block(win));
+            mine = lane_best();
+        }
+        __syncwarp();
+    }
+}
+
+}  // namespace topk
+}  // namespace phsa

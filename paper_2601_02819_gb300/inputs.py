@@ -84,6 +84,14 @@ WORKLOADS = {
 }
 
 
+# Decode: B sequences, each with a cache of L tokens whose last token (position
+# L - 1) is the new one, the query of that step.
+DECODE_WORKLOADS = {
+    "decode_32k_b64": Workload("decode_32k_b64", B=64, L=32768, Hq=16, Hkv=8, topk=14,
+                               punct="sentence", punct_gap=(9, 25), seed=1234 + 4),
+}
+
+
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
     """Round float32 values to bf16 (nearest, ties to even); return uint16 bits."""
     u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
@@ -162,6 +170,41 @@ def make_inputs(w: Workload, with_grad: bool = False, seed: int | None = None) -
         out["dO"] = f32_to_bf16_bits(rng.standard_normal(size=(w.B, w.Hq, w.L, w.D),
                                                           dtype=np.float32))
     return out
+
+
+def make_decode_inputs(w: Workload, device, seed: int | None = None) -> dict:
+    """Draw one decode batch for workload ``w`` directly on a torch ``device``.
+
+    The caches are too large to draw on the host (4.3 GB each at 64 x 32k), so
+    the N(0,1) values come from torch's seeded generator on that device, in
+    float32, rounded to bf16 (nearest, ties to even). Returns q [B,Hq,D], K, V
+    [B,Hkv,L,D] bf16 tensors on the device; mask [B,L] as numpy uint8 and as a
+    device tensor (mask_dev); lens [B] int32 (numpy and lens_dev), all equal to L.
+    """
+    import torch
+
+    s = w.seed if seed is None else seed
+    rng = np.random.default_rng(s)
+    pset = punct_id_set(rng)
+    ids = draw_token_ids(rng, w.B, w.L, w.punct, w.punct_gap, pset)
+    mask = np.isin(ids, pset).astype(np.uint8)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(s)
+
+    def normal(shape):
+        out = torch.empty(shape, dtype=torch.bfloat16, device=device)
+        for b in range(shape[0]):  # one sequence at a time keeps the fp32 draw small
+            out[b] = torch.randn(shape[1:], generator=gen, device=device,
+                                 dtype=torch.float32).to(torch.bfloat16)
+        return out
+
+    K = normal((w.B, w.Hkv, w.L, w.D))
+    V = normal((w.B, w.Hkv, w.L, w.D))
+    q = normal((w.B, w.Hq, w.D))
+    lens = np.full((w.B,), w.L, dtype=np.int32)
+    return {"q": q, "K": K, "V": V, "mask": mask, "ids": ids, "punct_ids": pset,
+            "mask_dev": torch.from_numpy(mask).to(device), "lens": lens,
+            "lens_dev": torch.from_numpy(lens).to(device)}
 
 
 def custom(name: str = "custom", **kw) -> Workload:

@@ -78,7 +78,11 @@ def _declare(L):
     L.phsa_sparse_attn_bwd_noalloc.argtypes = [P, P, P, P, P, P, P, P, phsa_shape, I, F, P, P, P,
                                                P]
     L.phsa_sparse_attn_bwd_noalloc.restype = I
-    for fn in ("phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
+    L.phsa_decode_update_repr.argtypes = [P, P, P, phsa_shape, F, P, P]
+    L.phsa_decode_select.argtypes = [P, P, P, phsa_shape, phsa_select_params, P, P, P]
+    L.phsa_decode_attn.argtypes = [P, P, P, P, P, P, phsa_shape, I, F, P, P, P]
+    for fn in ("phsa_decode_update_repr", "phsa_decode_select", "phsa_decode_attn",
+               "phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
                "phsa_sparse_attn_bwd", "phsa_get_device_status", "phsa_selftest_tcgen05"):
         getattr(L, fn).restype = I
 
@@ -243,6 +247,76 @@ def phsa_sparse_attn_bwd_noalloc(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_s
         _ptr(dK), _ptr(dV), _stream(stream))
     _raise("phsa_sparse_attn_bwd_noalloc", rc)
     return dQ, dK, dV
+
+
+def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=None):
+    """Decode: refresh the representative key of every block the new token has
+    just filled (a sequence whose length is a positive multiple of 64).
+    K [B, Hkv, Lc, D] bf16 cache, punct_mask [B, Lc] uint8, seq_lens [B] int32,
+    Krepr [B, Hkv, Lc // 64, D] bf16 (updated in place; returned)."""
+    _check(K, "K", torch.bfloat16, 4)
+    _check(punct_mask, "punct_mask", torch.uint8, 2)
+    _check(seq_lens, "seq_lens", torch.int32, 1)
+    _check(Krepr, "Krepr", torch.bfloat16, 4)
+    B, Hkv, Lc, D = K.shape
+    if tuple(punct_mask.shape) != (B, Lc) or tuple(seq_lens.shape) != (B,):
+        raise ValueError("punct_mask must be [B, Lc] and seq_lens [B]")
+    rc = load().phsa_decode_update_repr(_ptr(K), _ptr(punct_mask), _ptr(seq_lens),
+                                        make_shape(B, Lc, Hkv, Hkv, D), float(lam), _ptr(Krepr),
+                                        _stream(stream))
+    _raise("phsa_decode_update_repr", rc)
+    return Krepr
+
+
+def phsa_decode_select(q, Krepr, seq_lens, Lc: int, topk: int, n_init: int = 1,
+                       n_local: int = 1, sm_scale: float | None = None, block_idx=None,
+                       block_cnt=None, stream=None):
+    """Decode selection for the new token of every sequence: q [B, Hq, D] bf16,
+    Krepr [B, Hkv, Lc // 64, D]; returns (block_idx [B, Hkv, topk], block_cnt [B, Hkv])."""
+    _check(q, "q", torch.bfloat16, 3)
+    _check(Krepr, "Krepr", torch.bfloat16, 4)
+    _check(seq_lens, "seq_lens", torch.int32, 1)
+    B, Hq, D = q.shape
+    Hkv = Krepr.shape[1]
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    if block_idx is None:
+        block_idx = torch.empty((B, Hkv, topk), dtype=torch.int32, device=q.device)
+    if block_cnt is None:
+        block_cnt = torch.empty((B, Hkv), dtype=torch.int32, device=q.device)
+    _check(block_idx, "block_idx", torch.int32, 3)
+    _check(block_cnt, "block_cnt", torch.int32, 2)
+    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    rc = load().phsa_decode_select(_ptr(q), _ptr(Krepr), _ptr(seq_lens),
+                                   make_shape(B, Lc, Hq, Hkv, D), p, _ptr(block_idx),
+                                   _ptr(block_cnt), _stream(stream))
+    _raise("phsa_decode_select", rc)
+    return block_idx, block_cnt
+
+
+def phsa_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, sm_scale: float | None = None,
+                     O=None, lse=None, stream=None):
+    """Decode attention of the new token: (O [B, Hq, D] bf16, lse [B, Hq] fp32)."""
+    _check(q, "q", torch.bfloat16, 3)
+    _check(K, "K", torch.bfloat16, 4)
+    _check(V, "V", torch.bfloat16, 4)
+    _check(block_idx, "block_idx", torch.int32, 3)
+    _check(block_cnt, "block_cnt", torch.int32, 2)
+    _check(seq_lens, "seq_lens", torch.int32, 1)
+    B, Hq, D = q.shape
+    Hkv, Lc = K.shape[1], K.shape[2]
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    O = torch.empty_like(q) if O is None else O
+    lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device) if lse is None else lse
+    _check(O, "O", torch.bfloat16, 3)
+    _check(lse, "lse", torch.float32, 2)
+    rc = load().phsa_decode_attn(_ptr(q), _ptr(K), _ptr(V), _ptr(block_idx), _ptr(block_cnt),
+                                 _ptr(seq_lens), make_shape(B, Lc, Hq, Hkv, D),
+                                 int(block_idx.shape[-1]), float(sm_scale), _ptr(O), _ptr(lse),
+                                 _stream(stream))
+    _raise("phsa_decode_attn", rc)
+    return O, lse
 
 
 def phsa_get_device_status(stream=None) -> int:

@@ -31,7 +31,8 @@ def lib():
 def test_header_declares_the_hot_path():
     names = declared_functions()
     for n in ("phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
-              "phsa_sparse_attn_bwd", "phsa_sparse_attn_bwd_workspace", "phsa_get_device_status"):
+              "phsa_sparse_attn_bwd", "phsa_sparse_attn_bwd_workspace", "phsa_get_device_status",
+              "phsa_decode_update_repr", "phsa_decode_select", "phsa_decode_attn"):
         assert n in names
 
 

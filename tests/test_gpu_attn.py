@@ -113,6 +113,27 @@ def test_backward_long_lists_use_chunked_partials_and_are_deterministic():
     assert_close("dV", bf16_to_f64(g1[2]), rV)
 
 
+def test_backward_large_budget_for_pairs():
+    # A list capacity of 220 blocks (the selection padded with -1) no longer fits
+    # beside the tcgen05 dQ kernel's tiles, so pairs of heads take the
+    # register-MMA backward kernels; the forward keeps its tcgen05 kernel.
+    Q, K, V, dO, idx, cnt = rand_case(21, 1, 4, 2, 64 * 30 + 17, 8, grad=True)
+    wide = np.full(idx.shape[:-1] + (220,), -1, np.int32)
+    wide[..., :idx.shape[-1]] = idx
+    Qd, Kd, Vd, dOd = (to_dev_bf16(a) for a in (Q, K, V, dO))
+    it, ct = torch.from_numpy(wide).cuda(), torch.from_numpy(cnt).cuda()
+    O, lse = phsa.phsa_sparse_attn_fwd(Qd, Kd, Vd, it, ct)
+    dQ, dK, dV = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct)
+    torch.cuda.synchronize()
+    assert phsa.phsa_get_device_status() == 0
+    Or, _ = oracle.sparse_attn_fwd(Q, K, V, idx, cnt, 64, SCALE)
+    assert_close("O", bf16_to_f64(O), Or)
+    rQ, rK, rV = oracle.sparse_attn_bwd(Q, K, V, dO, idx, cnt, 64, SCALE)
+    assert_close("dQ", bf16_to_f64(dQ), rQ)
+    assert_close("dK", bf16_to_f64(dK), rK)
+    assert_close("dV", bf16_to_f64(dV), rV)
+
+
 def test_invalid_block_indices_are_skipped_and_reported():
     Q, K, V, _, idx, cnt = rand_case(12, 1, 2, 1, 64 * 6, 3)
     bad = idx.copy()

@@ -47,6 +47,8 @@ def test_tiny_workload():
     (1, 3, 3, 64 * 40, 9, 2, 3),        # G = 1, wider forced set
     (1, 2, 1, 64 * 300, 12, 1, 2),      # many candidate tiles
     (1, 2, 1, 64 * 20, 25, 1, 1),       # budget covers everything: dense rows
+    (1, 4, 2, 64 * 40 + 5, 20, 1, 1),   # G = 2: warp slices smaller than the budget
+    (1, 2, 1, 64 * 160, 80, 1, 1),      # G = 2: budget above the two-level top-k limit
 ])
 def test_shapes_and_forced_sets(B, Hq, Hkv, L, topk, n_init, n_local):
     rng = np.random.default_rng(B * 1000 + L)
