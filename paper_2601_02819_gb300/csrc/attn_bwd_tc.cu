@@ -1,7 +1,8 @@
 // Stage (c) backward on the tensor cores (tcgen05 + TMEM + TMA), for GQA
 // groups of two query heads, so that every MMA has M = 128.
 //
-// dq_tc_kernel: one CTA per (query block qb, KV head g), 352 threads. The
+// dq_tc_kernel: persistent, one CTA per SM over the units (query block qb,
+//   KV head g), 384 threads; rings and barriers continue across units. The
 //   selected blocks are taken in pairs (an odd count pairs the last block with
 //   a masked copy of itself); each pair's K and V tiles (128 keys) are gathered
 //   by TMA into 3- and 2-slot rings. Per pair p:
@@ -10,10 +11,11 @@
 //     dS_p = P_p (dP_p - Delta), P_p = exp(S_p * scale - lse)   (8 warps, TMEM)
 //     dQ  += dS_p Kp      (M128 N128 K128, A = dS_p in TMEM, B = Kp MN-major)
 //   S is double-buffered in TMEM, so S_{p+1} runs while the elementwise warps
-//   work on pair p. dQ * scale -> TMA store. Before the first pair the
-//   elementwise warps compute Delta_i = dO_i . O_i (O read from global memory,
-//   dO from the loaded tile) and write it for the dK/dV kernel, which runs
-//   after this one.
+//   work on pair p; dQ * scale is stored from registers. Before the first pair
+//   the elementwise warps compute Delta_i = dO_i . O_i (O read from global
+//   memory, dO from the loaded tile) and write it for the dK/dV kernel, which
+//   runs after this one. A fourth producer warp loads each unit's Q and dO as
+//   soon as the previous unit's last dP has been issued and its Delta read.
 //
 // dkdv_tc_kernel: one CTA per work item (KV block t, chunk of <= 32 query
 //   blocks that selected t), 320 threads. K_t and V_t stay in shared memory;
@@ -52,6 +54,10 @@ __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
 }
 
 // ============================================================== dQ
+// Persistent: one CTA per SM walks the units (query block, KV head) u =
+// blockIdx.x, blockIdx.x + gridDim.x, ...; the K/V rings, the S/dP buffers and
+// every barrier run on counters that continue across units, so the next
+// unit's Q/dO and first K/V pairs load while the current one finishes.
 // Blocks are processed in pairs, so the S and dP MMAs have N = 128 keys.
 namespace dq {
 constexpr int kKSlots = 3, kVSlots = 2;        // ring slots, one block pair each
@@ -61,19 +67,23 @@ constexpr int kOffDO = kOffQ + kTile128;
 constexpr int kOffK = kOffDO + kTile128;
 constexpr int kOffV = kOffK + kKSlots * kPair;
 constexpr int kOffBar = kOffV + kVSlots * kPair;
-constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = B_KFULL + kKSlots, B_VFULL = B_KEMPTY + kKSlots,
-              B_VEMPTY = B_VFULL + kVSlots, B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2,
-              B_DPFREE = B_DSFULL + 2, B_FINAL = B_DPFREE + 1, B_DRAIN = B_FINAL + 1,
+constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = B_KFULL + kKSlots,
+              B_VFULL = B_KEMPTY + kKSlots, B_VEMPTY = B_VFULL + kVSlots,
+              B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2, B_DPFREE = B_DSFULL + 2,
+              B_FINAL = B_DPFREE + 1, B_DQFREE = B_FINAL + 1, B_DRAIN = B_DQFREE + 1,
               kNumBars = B_DRAIN + 1;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kOffDPart = kOffMisc + 16;  // Delta of the 128 rows, fp32
-constexpr int kOffList = kOffDPart + 128 * 4;
-constexpr int kThreads = 352;  // 8 elementwise warps, K/Q/dO producer, MMA, V producer
+constexpr int kOffList = kOffDPart + 128 * 4;  // block lists: 7 slots of list_stride(topk) ints
+constexpr int kListK = 0, kListV = 2, kListM = 4, kListE = 5, kListSlots = 7;
+constexpr int kThreads = 384;  // 8 elementwise warps, K producer, MMA, V producer, Q/dO producer
 // TMEM: dQ [0,128), S of pair buffer b at [128 + 128b, +128), dP [384, 512).
 // dS of key half h overwrites S columns [64h, 64h + 32) (read by the same thread).
 constexpr uint32_t kColDQ = 0, kColDP = 384;
 __device__ __forceinline__ uint32_t col_s(int b) { return 128u + 128u * (uint32_t)b; }
-constexpr size_t smem_bytes(int topk) { return 1024 + (size_t)kOffList + (size_t)(topk + 2) * 4; }
+constexpr size_t smem_bytes(int topk) {
+    return 1024 + (size_t)kOffList + (size_t)kListSlots * ((topk + 2 + 15) & ~15) * 4;
+}
 }  // namespace dq
 
 struct DqArgs {
@@ -82,33 +92,73 @@ struct DqArgs {
     const float* lse;
     const __nv_bfloat16* O;
     float* delta;  // written: Delta_i = dO_i . O_i for every valid row
+    __nv_bfloat16* dQ;
     int* status;
-    int Hq, Hkv, L, NQB, topk;
+    int Hq, Hkv, L, NQB, topk, units;
     float scale_log2, sm_scale;
 };
+
+// Copies one unit's block list row to shared memory with independent loads
+// (one memory latency per 16 entries, the count fetched alongside) and
+// compacts it there: -1 entries are skipped, and so is an entry outside
+// [0, qb] or not above its predecessor (the rule of compact_block_list).
+// Returns the number of valid blocks; out holds list_stride() ints.
+__device__ __forceinline__ int stage_list(const int32_t* __restrict__ row,
+                                          const int32_t* __restrict__ cntp, int topk, int qb,
+                                          int* out) {
+    const int cnt = __ldg(cntp);
+    for (int j0 = 0; j0 < topk; j0 += 16) {
+        int v[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) v[k] = j0 + k < topk ? __ldg(row + j0 + k) : -1;
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+            if (j0 + k < topk) out[j0 + k] = v[k];
+    }
+    const int n_raw = cnt < 0 ? 0 : min(cnt, topk);
+    int k = 0, prev = -1;
+    for (int j = 0; j < n_raw; ++j) {
+        const int t = out[j];
+        if (t == -1 || t < 0 || t > qb || t <= prev) continue;
+        out[k++] = t;
+        prev = t;
+    }
+    out[k] = k > 0 ? out[k - 1] : 0;  // an odd count pairs the last block with itself
+    return k;
+}
+
+__host__ __device__ constexpr int list_stride(int topk) { return (topk + 2 + 15) & ~15; }
+
+struct DqUnit {
+    int qb, bg, hq0;
+    long long lu;
+};
+
+__device__ __forceinline__ DqUnit dq_unit(const DqArgs& a, int u) {
+    DqUnit d;
+    d.qb = a.NQB - 1 - (u % a.NQB);  // heaviest query blocks first
+    d.bg = u / a.NQB;
+    d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
+    d.lu = (long long)d.bg * a.NQB + d.qb;
+    return d;
+}
 
 __global__ void __launch_bounds__(dq::kThreads, 1)
 dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
              const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
-             const __grid_constant__ CUtensorMap tmdQ, const DqArgs a) {
+             const DqArgs a) {
     using namespace dq;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     const uint32_t sb = smem_u32(smem);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int unit = blockIdx.x;
-    const int qb = a.NQB - 1 - (unit % a.NQB);
-    const int bg = unit / a.NQB;
-    const int b = bg / a.Hkv, g = bg % a.Hkv;
-    const long long lu = (long long)bg * a.NQB + qb;
     auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
-    int* list = reinterpret_cast<int*>(smem + kOffList);
-    const int hq0 = b * a.Hq + g * 2;
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_Q), 1);
+        mbar_init(bar(B_QFREE), 257);  // the MMA commit after the unit's last dP + 256 Delta readers
         for (int s = 0; s < kKSlots; ++s) {
             mbar_init(bar(B_KFULL + s), 1);
             mbar_init(bar(B_KEMPTY + s), 1);
@@ -127,12 +177,10 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         mbar_init(bar(B_DSFULL + 1), 256);
         mbar_init(bar(B_DPFREE), 256);
         mbar_init(bar(B_FINAL), 1);
+        mbar_init(bar(B_DQFREE), 256);
         mbar_init(bar(B_DRAIN), 1);
         fence_barrier_init();
         *abort_flag = 0;
-        const int n = compact_block_list(a.idx + lu * a.topk, a.cnt[lu], a.topk, qb, list, nullptr);
-        list[n] = n > 0 ? list[n - 1] : 0;  // an odd count pairs the last block with itself
-        reinterpret_cast<int*>(smem + kOffMisc)[2] = n;
     }
     if (warp == 9) {
         tmem_alloc(sb + kOffMisc, kTmemCols);
@@ -142,49 +190,94 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
-    const int n = reinterpret_cast<volatile int*>(smem + kOffMisc)[2];
-    const int np = (n + 1) >> 1;  // block pairs
 
     if (warp == 8 || warp == 10) {
-        // ------------------------------------------------ TMA producers (pairs of blocks)
-        if (lane == 0 && n > 0) {
+        // ------------------------------------------------ K and V producers (block pairs)
+        if (lane == 0) {
             const bool is_k = warp == 8;
             const CUtensorMap* map = is_k ? &tmK : &tmV;
             const int slots = is_k ? kKSlots : kVSlots;
             const int full = is_k ? B_KFULL : B_VFULL, empty = is_k ? B_KEMPTY : B_VEMPTY;
             const uint32_t ring = sb + (is_k ? kOffK : kOffV);
             prefetch_tmap(map);
-            if (is_k) {
+            const int ls = list_stride(a.topk);
+            int* lists = reinterpret_cast<int*>(smem + kOffList) + (is_k ? kListK : kListV) * ls;
+            // Two list slots by unit parity. The next unit's list is staged once the
+            // current unit's pairs are all issued, while the ring is still full, so
+            // its memory latency stays off the load path.
+            auto stage = [&](int u, int slot) {
+                const DqUnit d = dq_unit(a, u);
+                return stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb,
+                                  lists + slot * ls);
+            };
+            int n_cur = blockIdx.x < a.units ? stage(blockIdx.x, 0) : 0;
+            int gp = 0;  // pairs issued so far, over all units
+            bool ok = true;
+            int ul = 0;
+            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++ul) {
+                const DqUnit d = dq_unit(a, u);
+                const int* list = lists + (ul & 1) * ls;
+                const int n = n_cur;
+                const int np = (n + 1) >> 1;
+                for (int p = 0; p < np; ++p, ++gp) {
+                    const int s = gp % slots;
+                    if (gp >= slots &&
+                        !mbar_wait(bar(empty + s), ((gp / slots) - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(bar(full + s), kPair);
+                    // slot layout: [d half][block of the pair][64 rows][64 columns]; an
+                    // odd count pairs the last block with itself (masked by the consumer)
+                    for (int dh = 0; dh < 2; ++dh) {
+                        tma_load_3d(ring + s * kPair + dh * kHalf128, map, bar(full + s), dh * 64,
+                                    list[2 * p] * 64, d.bg);
+                        tma_load_3d(ring + s * kPair + dh * kHalf128 + kHalf64, map, bar(full + s),
+                                    dh * 64, list[2 * p + 1] * 64, d.bg);
+                    }
+                }
+                const int u2 = u + (int)gridDim.x;
+                n_cur = ok && u2 < a.units ? stage(u2, (ul + 1) & 1) : 0;
+            }
+            for (int q = gp - slots; q < gp; ++q)
+                if (q >= 0) mbar_wait_drain(bar(full + q % slots), (q / slots) & 1);
+        }
+    } else if (warp == 11) {
+        // ------------------------------------------------ Q / dO producer, one load per unit
+        if (lane == 0) {
+            prefetch_tmap(&tmQ);
+            prefetch_tmap(&tmdO);
+            int ul = 0, last = -1;
+            for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
+                if (ul > 0 && !mbar_wait(bar(B_QFREE), (ul - 1) & 1, abort_flag, a.status)) break;
+                last = ul;
+                const DqUnit d = dq_unit(a, u);
                 mbar_expect_tx(bar(B_Q), 2 * kTile128);
                 for (int hl = 0; hl < 2; ++hl)
                     for (int dh = 0; dh < 2; ++dh) {
                         tma_load_3d(sb + kOffQ + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_Q),
-                                    dh * 64, qb * 64, hq0 + hl);
+                                    dh * 64, d.qb * 64, d.hq0 + hl);
                         tma_load_3d(sb + kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(B_Q),
-                                    dh * 64, qb * 64, hq0 + hl);
+                                    dh * 64, d.qb * 64, d.hq0 + hl);
                     }
+                // The next unit's Q and dO come from HBM: start bringing them into L2
+                // now, a whole unit before they are loaded.
+                const int u2 = u + (int)gridDim.x;
+                if (u2 < a.units) {
+                    const int qb2 = a.NQB - 1 - (u2 % a.NQB), bg2 = u2 / a.NQB;
+                    const int hq2 = (bg2 / a.Hkv) * a.Hq + (bg2 % a.Hkv) * 2;
+                    for (int hl = 0; hl < 2; ++hl)
+                        for (int dh = 0; dh < 2; ++dh) {
+                            tma_prefetch_3d(&tmQ, dh * 64, qb2 * 64, hq2 + hl);
+                            tma_prefetch_3d(&tmdO, dh * 64, qb2 * 64, hq2 + hl);
+                        }
+                }
             }
-            int issued = 0;
-            for (int p = 0; p < np; ++p) {
-                const int s = p % slots;
-                if (p >= slots &&
-                    !mbar_wait(bar(empty + s), ((p / slots) - 1) & 1, abort_flag, a.status))
-                    break;
-                mbar_expect_tx(bar(full + s), kPair);
-                // slot layout: [d half][block of the pair][64 rows][64 columns]
-                for (int e = 0; e < 2; ++e)
-                    for (int dh = 0; dh < 2; ++dh)
-                        tma_load_3d(ring + s * kPair + dh * kHalf128 + e * kHalf64, map,
-                                    bar(full + s), dh * 64, list[2 * p + e] * 64, bg);
-                issued = p + 1;
-            }
-            if (is_k) mbar_wait_drain(bar(B_Q), 0);
-            for (int p = issued - slots; p < issued; ++p)
-                if (p >= 0) mbar_wait_drain(bar(full + p % slots), (p / slots) & 1);
+            if (last >= 0) mbar_wait_drain(bar(B_Q), last & 1);
         }
     } else if (warp == 9) {
         // ------------------------------------------------ MMA issuer
-        if (lane == 0 && n > 0) {
+        if (lane == 0) {
             constexpr uint32_t id_s = idesc_bf16(128, 128, false);
             constexpr uint32_t id_dq = idesc_bf16(128, 128, true);
             const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
@@ -192,73 +285,99 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
             const uint64_t dKmn0 = sdesc_sw128(sb + kOffK, kHalf128, 1024);  // K read MN-major
             const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
-            bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
-            tc_fence_after();
-            auto issue_s = [&](int p) {  // S_p = Q Kpair_p^T into buffer p & 1
-                const uint64_t kd = sdesc_at(dK0, (p % kKSlots) * kPair);
+            auto issue_s = [&](int gp) {  // S = Q Kpair^T into buffer gp & 1
+                const uint64_t kd = sdesc_at(dK0, (gp % kKSlots) * kPair);
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
                     const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
-                    mma_ss(tmem + col_s(p & 1), sdesc_at(dQ0, off), sdesc_at(kd, off), id_s,
+                    mma_ss(tmem + col_s(gp & 1), sdesc_at(dQ0, off), sdesc_at(kd, off), id_s,
                            ks > 0 ? 1u : 0u);
                 }
             };
-            auto issue_dp = [&](int p) {  // dP_p = dO Vpair_p^T; releases the V slot
-                const uint64_t vd = sdesc_at(dV0, (p % kVSlots) * kPair);
+            auto issue_dp = [&](int gp) {  // dP = dO Vpair^T; releases the V slot
+                const uint64_t vd = sdesc_at(dV0, (gp % kVSlots) * kPair);
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
                     const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
                     mma_ss(tmem + kColDP, sdesc_at(dDO0, off), sdesc_at(vd, off), id_s,
                            ks > 0 ? 1u : 0u);
                 }
-                mma_commit(bar(B_SPFULL + (p & 1)));  // S_p and dP_p are both complete
-                mma_commit(bar(B_VEMPTY + p % kVSlots));
+                mma_commit(bar(B_SPFULL + (gp & 1)));  // S and dP of this pair are both complete
+                mma_commit(bar(B_VEMPTY + gp % kVSlots));
             };
-            // Order: S_0 dP_0 S_1 | dP consumed_0 -> dP_1 | dS_0 -> dQ_0 S_2 | ...
-            // dP has one TMEM buffer: dP_{p+1} is issued as soon as the elementwise
-            // warps have loaded dP_p, while they still compute dS_p.
-            ok = ok && mbar_wait(bar(B_KFULL), 0, abort_flag, a.status) &&
-                 mbar_wait(bar(B_VFULL), 0, abort_flag, a.status);
-            if (ok) {
-                tc_fence_after();
-                issue_s(0);
-                issue_dp(0);
-            }
-            if (ok && np > 1) {
-                ok = mbar_wait(bar(B_KFULL + 1), 0, abort_flag, a.status);
-                if (ok) {
-                    tc_fence_after();
-                    issue_s(1);
-                }
-            }
-            for (int p = 0; ok && p < np; ++p) {
-                if (p + 1 < np) {  // dP_{p+1} once the elementwise warps hold dP_p
-                    ok = mbar_wait(bar(B_DPFREE), p & 1, abort_flag, a.status) &&
-                         mbar_wait(bar(B_VFULL + (p + 1) % kVSlots), ((p + 1) / kVSlots) & 1,
-                                   abort_flag, a.status);
-                    if (!ok) break;
-                    tc_fence_after();
-                    issue_dp(p + 1);
-                }
-                ok = mbar_wait(bar(B_DSFULL + (p & 1)), (p >> 1) & 1, abort_flag, a.status);
+            auto wait_k = [&](int gp) {
+                return mbar_wait(bar(B_KFULL + gp % kKSlots), (gp / kKSlots) & 1, abort_flag, a.status);
+            };
+            auto wait_v = [&](int gp) {
+                return mbar_wait(bar(B_VFULL + gp % kVSlots), (gp / kVSlots) & 1, abort_flag, a.status);
+            };
+            // dP has one TMEM buffer: dP(gp) waits until the elementwise warps hold
+            // dP(gp - 1) in registers (they release it before computing dS).
+            auto wait_dpfree = [&](int gp) {
+                return gp == 0 || mbar_wait(bar(B_DPFREE), (gp - 1) & 1, abort_flag, a.status);
+            };
+            bool ok = true;
+            int gp0 = 0, ul = 0;
+            // Order per unit: S_0 dP_0 S_1 | dP_1 | dS_0 -> dQ_0 S_2 | dP_2 | dS_1 -> dQ_1 S_3 ...
+            int* mlist = reinterpret_cast<int*>(smem + kOffList) + kListM * list_stride(a.topk);
+            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++ul) {
+                const DqUnit d = dq_unit(a, u);
+                const int np = (stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, mlist) + 1) >> 1;
+                ok = mbar_wait(bar(B_Q), ul & 1, abort_flag, a.status);
                 if (!ok) break;
                 tc_fence_after();
-                // dQ += dS_p Kpair_p: A = dS (TMEM), B = the K pair read MN-major
-                const uint64_t kmn = sdesc_at(dKmn0, (p % kKSlots) * kPair);
-#pragma unroll
-                for (int ks = 0; ks < 8; ++ks)
-                    mma_ts(tmem + kColDQ, tmem + col_s(p & 1) + (ks >> 2) * 64 + (ks & 3) * 8,
-                           sdesc_at(kmn, ks * 2048), id_dq, (p > 0 || ks > 0) ? 1u : 0u);
-                mma_commit(bar(B_KEMPTY + p % kKSlots));
-                if (p == np - 1) {
-                    mma_commit(bar(B_FINAL));
-                } else if (p + 2 < np) {  // S_{p+2} reuses the S buffer dQ_p has just read
-                    ok = mbar_wait(bar(B_KFULL + (p + 2) % kKSlots), ((p + 2) / kKSlots) & 1,
-                                   abort_flag, a.status);
+                if (np >= 1) {
+                    ok = wait_k(gp0) && wait_v(gp0) && wait_dpfree(gp0);
                     if (!ok) break;
                     tc_fence_after();
-                    issue_s(p + 2);
+                    issue_s(gp0);
+                    issue_dp(gp0);
+                    if (np == 1) mma_commit(bar(B_QFREE));
                 }
+                if (np >= 2) {
+                    ok = wait_k(gp0 + 1);
+                    if (!ok) break;
+                    tc_fence_after();
+                    issue_s(gp0 + 1);
+                }
+                if (np == 0) {
+                    mma_commit(bar(B_QFREE));
+                    // the previous unit's dQ must be read out before FINAL completes again
+                    ok = ul == 0 || mbar_wait(bar(B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
+                    if (!ok) break;
+                    mma_commit(bar(B_FINAL));
+                }
+                for (int p = 0; ok && p < np; ++p) {
+                    const int gp = gp0 + p;
+                    if (p + 1 < np) {
+                        ok = wait_dpfree(gp + 1) && wait_v(gp + 1);
+                        if (!ok) break;
+                        tc_fence_after();
+                        issue_dp(gp + 1);
+                        if (p + 2 == np) mma_commit(bar(B_QFREE));  // last MMA reading Q/dO
+                    }
+                    ok = mbar_wait(bar(B_DSFULL + (gp & 1)), (gp >> 1) & 1, abort_flag, a.status);
+                    if (ok && p == 0 && ul > 0)  // dQ's accumulator: the previous unit is read out
+                        ok = mbar_wait(bar(B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
+                    if (!ok) break;
+                    tc_fence_after();
+                    // dQ += dS Kpair: A = dS (TMEM), B = the K pair read MN-major
+                    const uint64_t kmn = sdesc_at(dKmn0, (gp % kKSlots) * kPair);
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ts(tmem + kColDQ, tmem + col_s(gp & 1) + (ks >> 2) * 64 + (ks & 3) * 8,
+                               sdesc_at(kmn, ks * 2048), id_dq, (p > 0 || ks > 0) ? 1u : 0u);
+                    mma_commit(bar(B_KEMPTY + gp % kKSlots));
+                    if (p == np - 1) {
+                        mma_commit(bar(B_FINAL));
+                    } else if (p + 2 < np) {  // S_{p+2} reuses the S buffer dQ_p has just read
+                        ok = wait_k(gp + 2);
+                        if (!ok) break;
+                        tc_fence_after();
+                        issue_s(gp + 2);
+                    }
+                }
+                gp0 += np;
             }
             mma_commit(bar(B_DRAIN));
             mbar_wait_drain(bar(B_DRAIN), 0);
@@ -268,121 +387,170 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         const int row = (warp & 3) * 32 + lane;  // TMEM lane
         const int half = warp >> 2;              // block of the pair (64 keys); d half for dQ
         const int tok = row & 63, hl = row >> 6;
-        const int i = qb * 64 + tok;
-        const bool valid = i < a.L;
-        const size_t ridx = (size_t)(hq0 + hl) * a.L + (valid ? i : 0);
-        const float neg_lse2 = valid ? -a.lse[ridx] * kLog2e : -INFINITY;
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-        // Delta_i = dO_i . O_i, computed before the first pair: O is read from
-        // global memory in coalesced 16-byte pieces (16 threads per 256-byte
-        // row, 8 rows per pass), dO from the tile loaded for the dP MMAs; the 16
-        // partial dot products of a row are added by a fixed shuffle tree.
         const int et = threadIdx.x;  // 0..255 over the elementwise warps
-        const int pc = et & 15;      // 16-byte piece of the row
-        uint4 ov[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int rr = k * 16 + (et >> 4);
-            const int ii = qb * 64 + (rr & 63);
-            ov[k] = ii < a.L ? __ldg(reinterpret_cast<const uint4*>(
-                                   a.O + ((size_t)(hq0 + (rr >> 6)) * a.L + ii) * 128) + pc)
-                             : make_uint4(0u, 0u, 0u, 0u);
-        }
-        bool ok = n == 0 || mbar_wait(bar(B_Q), 0, abort_flag, a.status);
-        ok = __all_sync(0xffffffffu, ok);
+        const int pc = et & 15;      // 16-byte piece of a row in the Delta pass
         float* dpart = reinterpret_cast<float*>(smem + kOffDPart);
+        bool ok = true;
+        int gp0 = 0, ul = 0;
+        const int ls = list_stride(a.topk);
+        int* lists = reinterpret_cast<int*>(smem + kOffList) + kListE * ls;
+        // A unit's inputs that come from global memory (its block list, staged by
+        // thread 0; O rows and lse for Delta and P) are fetched during the
+        // previous unit, so that they are in hand when its Q and dO arrive.
+        uint4 ov[8];
+        float neg_lse2 = 0.f;
+        auto fetch_unit = [&](int u, int slot) {
+            const DqUnit d = dq_unit(a, u);
+            if (et == 0) lists[slot * ls + ls - 1] = stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu,
+                                                                a.topk, d.qb, lists + slot * ls);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int rr = k * 16 + (et >> 4);
-            float acc = 0.f;
-            if (ok && n > 0) {
-                const uint4 dv = *reinterpret_cast<const uint4*>(
-                    smem + kOffDO + (pc >> 3) * kHalf128 + (rr >> 6) * kHalf64 + sw_off(rr & 63, pc & 7));
-                const uint32_t ow[4] = {ov[k].x, ov[k].y, ov[k].z, ov[k].w};
-                const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w};
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float2 fo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ow[j]));
-                    const float2 fd = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&dw[j]));
-                    acc = fmaf(fo.x, fd.x, acc);
-                    acc = fmaf(fo.y, fd.y, acc);
+            for (int k = 0; k < 8; ++k) {
+                const int rr = k * 16 + (et >> 4);
+                const int ii = d.qb * 64 + (rr & 63);
+                ov[k] = ii < a.L ? __ldg(reinterpret_cast<const uint4*>(
+                                       a.O + ((size_t)(d.hq0 + (rr >> 6)) * a.L + ii) * 128) + pc)
+                                 : make_uint4(0u, 0u, 0u, 0u);
+            }
+            const int i = d.qb * 64 + tok;
+            neg_lse2 = i < a.L ? -__ldg(a.lse + (size_t)(d.hq0 + hl) * a.L + i) * kLog2e : -INFINITY;
+        };
+        if (blockIdx.x < a.units) fetch_unit(blockIdx.x, 0);
+        // Every warp runs every unit (doing no work after an abort), so the one
+        // named barrier per unit is reached the same number of times by all.
+        for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
+            const int* list = lists + (ul & 1) * ls;
+            const DqUnit d = dq_unit(a, u);
+            const int qb = d.qb;
+            const int i = qb * 64 + tok;
+            const bool valid = i < a.L;
+            const size_t ridx = (size_t)(d.hq0 + hl) * a.L + (valid ? i : 0);
+            const float nl2 = neg_lse2;
+            {  // two units ahead: block list, count, O rows and lse into L2 (all roles
+               // read a unit's list; O and lse are fetched into registers a unit ahead)
+                const int u3 = u + 2 * (int)gridDim.x;
+                if (u3 < a.units) {
+                    const DqUnit d3 = dq_unit(a, u3);
+                    const int r3 = et >> 1, i3 = d3.qb * 64 + (r3 & 63);
+                    if (i3 < a.L) {
+                        const size_t row3 = (size_t)(d3.hq0 + (r3 >> 6)) * a.L + i3;
+                        prefetch_l2(a.O + row3 * 128 + 64 * (et & 1));
+                        if ((r3 & 31) == 0 && (et & 1) == 0) prefetch_l2(a.lse + row3);
+                    }
+                    if (et == 0) prefetch_l2(a.cnt + d3.lu);
+                    if (et < 4 && et * 32 < a.topk) prefetch_l2(a.idx + d3.lu * a.topk + et * 32);
+                    if (et == 4) prefetch_l2(a.idx + d3.lu * a.topk + a.topk - 1);
                 }
             }
-#pragma unroll
-            for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-            if (pc == 0) dpart[rr] = acc;
-        }
-        named_barrier(1, 256);
-        const float dlt = dpart[row];
-        if (half == 0 && valid) a.delta[ridx] = dlt;
-        for (int p = 0; p < np; ++p) {
-            const int buf = p & 1;
-            ok = mbar_wait(bar(B_SPFULL + buf), (p >> 1) & 1, abort_flag, a.status);
-            ok = __all_sync(0xffffffffu, ok);
-            if (!ok) break;
-            tc_fence_after();
-            const int e = 2 * p + half;       // this half's block in the list
-            const bool live = e < n;          // false: the duplicate of an odd count
-            const bool diag = list[e] == qb;
-            uint32_t sv[64], dp[64];
-            tmem_ld64(lane_base + col_s(buf) + 64 * half, sv);
-            tmem_ld64(lane_base + kColDP + 64 * half, dp);
-            tc_fence_before();
-            mbar_arrive(bar(B_DPFREE));  // dP_p is in registers: the buffer may be refilled
-#pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                float ds[2];
-#pragma unroll
-                for (int x = 0; x < 2; ++x) {
-                    const int key = 2 * c + x;
-                    float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + x]), a.scale_log2, neg_lse2));
-                    if (!live || (diag && key > tok)) pv = 0.f;
-                    ds[x] = pv * (__uint_as_float(dp[2 * c + x]) - dlt);
-                }
-                sv[c] = pack2_bf16(ds[0], ds[1]);
+            if (ok) {
+                ok = mbar_wait(bar(B_Q), ul & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
             }
-            // dS columns [64 half, 64 half + 32): inside this thread's own S range
-            tmem_st32(lane_base + col_s(buf) + 64 * half, sv);
-            tc_fence_before();
-            mbar_arrive(bar(B_DSFULL + buf));
-        }
-        if (ok && n > 0) {
-            ok = mbar_wait(bar(B_FINAL), 0, abort_flag, a.status);
-            ok = __all_sync(0xffffffffu, ok);
-        }
-        if (ok) {
-            tc_fence_after();
-            uint8_t* sq = smem + kOffQ + half * kHalf128;  // this warp's 64 columns = one d-half
+            // Delta_i = dO_i . O_i: O in coalesced 16-byte pieces (16 threads per
+            // 256-byte row, 16 rows per pass), dO from the tile loaded for the dP
+            // MMAs; a fixed shuffle tree adds the pieces.
 #pragma unroll
-            for (int c2 = 0; c2 < 2; ++c2) {
-                uint32_t o[32];
-                if (n > 0) {
-                    tmem_ld32(lane_base + kColDQ + 64 * half + 32 * c2, o);
-                } else {
+            for (int k = 0; k < 8; ++k) {
+                const int rr = k * 16 + (et >> 4);
+                float acc = 0.f;
+                if (ok) {
+                    const uint4 dv = *reinterpret_cast<const uint4*>(
+                        smem + kOffDO + (pc >> 3) * kHalf128 + (rr >> 6) * kHalf64 + sw_off(rr & 63, pc & 7));
+                    const uint32_t ow[4] = {ov[k].x, ov[k].y, ov[k].z, ov[k].w};
+                    const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w};
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) o[c] = 0u;
+                    for (int j = 0; j < 4; ++j) {
+                        const float2 fo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ow[j]));
+                        const float2 fd = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&dw[j]));
+                        acc = fmaf(fo.x, fd.x, acc);
+                        acc = fmaf(fo.y, fd.y, acc);
+                    }
                 }
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint4 v;
-                    const float s = a.sm_scale;
-                    v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * s, __uint_as_float(o[8 * q + 1]) * s);
-                    v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * s, __uint_as_float(o[8 * q + 3]) * s);
-                    v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * s, __uint_as_float(o[8 * q + 5]) * s);
-                    v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * s, __uint_as_float(o[8 * q + 7]) * s);
-                    *reinterpret_cast<uint4*>(sq + sw_off(row, c2 * 4 + q)) = v;
+                for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+                if (pc == 0) dpart[rr] = acc;
+            }
+            named_barrier(1, 256);  // Delta's pieces and this unit's list are visible
+            const float dlt = dpart[row];
+            // This thread is done with dO and with Delta's exchange slots: the next
+            // unit's dO may be loaded (and dpart rewritten) once all have arrived.
+            if (ok) mbar_arrive(bar(B_QFREE));
+            const int n = list[ls - 1];
+            const int np = (n + 1) >> 1;
+            if (ok && half == 0 && valid) a.delta[ridx] = dlt;
+            const int u2 = u + (int)gridDim.x;
+            for (int p = 0; ok && p < np; ++p) {
+                const int gp = gp0 + p;
+                const int buf = gp & 1;
+                ok = mbar_wait(bar(B_SPFULL + buf), (gp >> 1) & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+                tc_fence_after();
+                const int e = 2 * p + half;       // this half's block in the list
+                const bool live = e < n;          // false: the duplicate of an odd count
+                const bool diag = list[e] == qb;
+                uint32_t sv[64], dp[64];
+                tmem_ld64(lane_base + col_s(buf) + 64 * half, sv);
+                tmem_ld64(lane_base + kColDP + 64 * half, dp);
+                tc_fence_before();
+                mbar_arrive(bar(B_DPFREE));  // dP is in registers: the buffer may be refilled
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    float ds[2];
+#pragma unroll
+                    for (int x = 0; x < 2; ++x) {
+                        const int key = 2 * c + x;
+                        float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + x]), a.scale_log2, nl2));
+                        if (!live || (diag && key > tok)) pv = 0.f;
+                        ds[x] = pv * (__uint_as_float(dp[2 * c + x]) - dlt);
+                    }
+                    sv[c] = pack2_bf16(ds[0], ds[1]);
+                }
+                // dS columns [64 half, 64 half + 32): inside this thread's own S range
+                tmem_st32(lane_base + col_s(buf) + 64 * half, sv);
+                tc_fence_before();
+                mbar_arrive(bar(B_DSFULL + buf));
+            }
+            gp0 += np;
+            // the next unit's inputs: their latency overlaps this unit's last dQ
+            // MMAs and its epilogue
+            if (u2 < a.units) fetch_unit(u2, (ul + 1) & 1);
+            if (ok) {
+                ok = mbar_wait(bar(B_FINAL), ul & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+            }
+            if (ok) {
+                // dQ row `row`, columns [64 half, 64 half + 64), straight to global
+                // memory, 32 columns at a time
+                tc_fence_after();
+#pragma unroll 1
+                for (int c2 = 0; c2 < 2; ++c2) {
+                    uint32_t o[32];
+                    if (n > 0) {
+                        tmem_ld32(lane_base + kColDQ + 64 * half + 32 * c2, o);
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) o[c] = 0u;
+                    }
+                    if (c2 == 1) {
+                        tc_fence_before();
+                        mbar_arrive(bar(B_DQFREE));
+                    }
+                    if (valid) {
+                        uint4* dst = reinterpret_cast<uint4*>(a.dQ + ridx * 128 + 64 * half + 32 * c2);
+                        const float s = a.sm_scale;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            uint4 v;
+                            v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * s, __uint_as_float(o[8 * q + 1]) * s);
+                            v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * s, __uint_as_float(o[8 * q + 3]) * s);
+                            v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * s, __uint_as_float(o[8 * q + 5]) * s);
+                            v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * s, __uint_as_float(o[8 * q + 7]) * s);
+                            dst[q] = v;
+                        }
+                    }
                 }
             }
-            fence_proxy_async_smem();
-        }
-        named_barrier(1, 256);
-        if (threadIdx.x == 0 && ok) {
-            for (int h2 = 0; h2 < 2; ++h2)
-                for (int dh = 0; dh < 2; ++dh)
-                    tma_store_3d(&tmdQ, sb + kOffQ + dh * kHalf128 + h2 * kHalf64, dh * 64, qb * 64,
-                                 hq0 + h2);
-            tma_store_commit();
-            tma_store_wait_read();
         }
     }
     tc_fence_before();
@@ -741,21 +909,25 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
                          const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                          void* dQ, int* status, cudaStream_t st) {
     const int NQB = (s.L + 63) / 64;
-    CUtensorMap tq, tk, tv, tdo, tdq;
+    CUtensorMap tq, tk, tv, tdo;
     const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
     if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) || !make_tmap_bf16_rows128(&tk, K, s.L, pk, 64) ||
-        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64) ||
-        !make_tmap_bf16_rows128(&tdq, dQ, s.L, pq, 64))
+        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64))
         return cudaErrorInvalidValue;
     const size_t smem = dq::smem_bytes(topk);
     cudaError_t e =
         cudaFuncSetAttribute(dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    DqArgs args{idx, cnt, lse, static_cast<const __nv_bfloat16*>(O), delta, status, s.Hq, s.Hkv, s.L, NQB, topk, sm_scale * kLog2e,
-                sm_scale};
+    int dev = 0, nsm = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    const int units = s.B * s.Hkv * NQB;
+    DqArgs args{idx, cnt, lse, static_cast<const __nv_bfloat16*>(O), delta,
+                static_cast<__nv_bfloat16*>(dQ), status, s.Hq, s.Hkv, s.L, NQB, topk, units,
+                sm_scale * kLog2e, sm_scale};
     ProfScope prof(K_BWD_DQ, st);
-    dq_tc_kernel<<<(unsigned)((long long)s.B * s.Hkv * NQB), dq::kThreads, smem, st>>>(
-        tq, tk, tv, tdo, tdq, args);
+    dq_tc_kernel<<<(unsigned)min(units, nsm), dq::kThreads, smem, st>>>(tq, tk, tv, tdo, args);
     return cudaGetLastError();
 }
 
