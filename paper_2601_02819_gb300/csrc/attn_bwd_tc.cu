@@ -22,7 +22,7 @@
 //   the Q and dO tiles (both heads stacked: 128 rows) of every listed query
 //   block stream through a two-stage ring:
 //     S  = Q K_t^T, dP = dO V_t^T            (M128 N64 K128)
-//     P, dS (8 warps) -> shared memory (bf16, 128 rows x 64 keys)
+//     P, dS (8 warps) -> shared memory (bf16, 128 rows x 64 keys, two buffers)
 //     dV^T += dO^T P, dK^T += Q^T dS          (M128 N64 K128; A = dO / Q read
 //                                             MN-major, B = P / dS MN-major)
 //   dK^T and dV^T live in TMEM with the head dimension on the lanes. A KV
@@ -567,17 +567,20 @@ constexpr int kOffK = 0;
 constexpr int kOffV = kOffK + kTile64;
 constexpr int kOffStage = kOffV + kTile64;      // 2 x (Q 32 KB, dO 32 KB)
 constexpr int kStage = 2 * kTile128;
-constexpr int kOffP = kOffStage + 2 * kStage;   // P  [128 rows][64 keys] bf16
-constexpr int kOffDS = kOffP + kHalf128;        // dS [128 rows][64 keys] bf16
-constexpr int kOffBar = kOffDS + kHalf128;
-constexpr int B_KV = 0, B_QFULL = 1, B_QEMPTY = 3, B_SPFULL = 5, B_PDSFULL = 7, B_PDSFREE = 8,
-              B_FINAL = 9, B_DRAIN = 10, kNumBars = 11;
+// P and dS [128 rows][64 keys] bf16, double-buffered: buffer b holds P at
+// kOffPDS + b * kPDS and dS kHalf128 after it
+constexpr int kOffPDS = kOffStage + 2 * kStage;
+constexpr int kPDS = 2 * kHalf128;
+constexpr int kOffBar = kOffPDS + 2 * kPDS;
+constexpr int B_KV = 0, B_QFULL = 1, B_QEMPTY = 3, B_SPFULL = 5, B_PDSFULL = 7, B_PDSFREE = 9,
+              B_FINAL = 11, B_DRAIN = 12, kNumBars = 13;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
+constexpr int kOffQL = kOffMisc + 16;  // the work item's query blocks (at most kBwdChunk)
 constexpr int kThreads = 320;  // 8 elementwise warps, producer, MMA
 constexpr uint32_t kColDV = 256, kColDK = 320;
 __device__ __forceinline__ uint32_t col_s(int b) { return 128u * (uint32_t)b; }
 __device__ __forceinline__ uint32_t col_dp(int b) { return 64u + 128u * (uint32_t)b; }
-constexpr size_t kSmem = 1024 + (size_t)kOffMisc + 16;
+constexpr size_t kSmem = 1024 + (size_t)kOffQL + kBwdChunk * 4;
 }  // namespace kv
 
 struct KvArgs {
@@ -625,13 +628,19 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             mbar_init(bar(B_QEMPTY + s), 1);
             mbar_init(bar(B_SPFULL + s), 1);
         }
-        mbar_init(bar(B_PDSFULL), 256);
-        mbar_init(bar(B_PDSFREE), 1);
+        for (int b2 = 0; b2 < 2; ++b2) {
+            mbar_init(bar(B_PDSFULL + b2), 256);
+            mbar_init(bar(B_PDSFREE + b2), 1);
+        }
         mbar_init(bar(B_FINAL), 1);
         mbar_init(bar(B_DRAIN), 1);
         fence_barrier_init();
         *abort_flag = 0;
     }
+    // The query-block list of this work item, staged once (one load per thread)
+    // so that no load or row fetch waits on it later.
+    int* qls = reinterpret_cast<int*>(smem + kOffQL);
+    if ((int)threadIdx.x < n_it) qls[threadIdx.x] = __ldg(ql + threadIdx.x);
     if (warp == 9) {
         tmem_alloc(sb + kOffMisc, kTmemCols);
         tmem_relinquish();
@@ -656,7 +665,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const int s = i & 1;
                 if (i >= 2 && !mbar_wait(bar(B_QEMPTY + s), ((i >> 1) - 1) & 1, abort_flag, a.status))
                     break;
-                const int qb = ql[i];
+                const int qb = qls[i];
                 const uint32_t st = sb + kOffStage + s * kStage;
                 mbar_expect_tx(bar(B_QFULL + s), kStage);
                 for (int hl = 0; hl < 2; ++hl)
@@ -681,8 +690,8 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const uint64_t dStT0 = sdesc_sw128(sb + kOffStage, kHalf128, 1024);   // Q/dO MN-major
             const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
             const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
-            const uint64_t dP0 = sdesc_sw128(sb + kOffP, kHalf128, 1024);
-            const uint64_t dS0 = sdesc_sw128(sb + kOffDS, kHalf128, 1024);
+            const uint64_t dP0 = sdesc_sw128(sb + kOffPDS, kHalf128, 1024);
+            const uint64_t dS0 = sdesc_sw128(sb + kOffPDS + kHalf128, kHalf128, 1024);
             bool ok = mbar_wait(bar(B_KV), 0, abort_flag, a.status);
             tc_fence_after();
             int ns = 0, nv = 0;
@@ -709,19 +718,20 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     ++ns;
                     progressed = true;
                 }
-                if (nv < ns && mbar_test_wait(bar(B_PDSFULL), nv & 1)) {
+                if (nv < ns && mbar_test_wait(bar(B_PDSFULL + (nv & 1)), (nv >> 1) & 1)) {
                     tc_fence_after();
                     const uint64_t qt = sdesc_at(dStT0, (nv & 1) * kStage);
+                    const uint32_t pb = (nv & 1) * kPDS;
                     // K dimension = the 128 stacked query rows, 16 per MMA
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
                         mma_ss(tmem + kColDV, sdesc_at(qt, kTile128 + ks * 2048),
-                               sdesc_at(dP0, ks * 2048), id_t, (nv > 0 || ks > 0) ? 1u : 0u);
+                               sdesc_at(dP0, pb + ks * 2048), id_t, (nv > 0 || ks > 0) ? 1u : 0u);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + kColDK, sdesc_at(qt, ks * 2048), sdesc_at(dS0, ks * 2048),
+                        mma_ss(tmem + kColDK, sdesc_at(qt, ks * 2048), sdesc_at(dS0, pb + ks * 2048),
                                id_t, (nv > 0 || ks > 0) ? 1u : 0u);
-                    mma_commit(bar(B_PDSFREE));
+                    mma_commit(bar(B_PDSFREE + (nv & 1)));
                     mma_commit(bar(B_QEMPTY + (nv & 1)));
                     if (nv == n_it - 1) mma_commit(bar(B_FINAL));
                     ++nv;
@@ -750,7 +760,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // Row data (query block, lse, Delta) is fetched one iteration ahead so its
         // global-memory latency overlaps the previous iteration.
         auto fetch = [&](int it2, int& qb2, float& nl2, float& dl2) {
-            qb2 = ql[it2];
+            qb2 = qls[it2];
             const int i2 = qb2 * 64 + tok;
             const bool v2 = i2 < a.L;
             nl2 = v2 ? -a.lse[hoff + i2] * kLog2e : -INFINITY;
@@ -789,21 +799,22 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 dp[c] = pack2_bf16(ds[0], ds[1]);
             }
             tc_fence_before();
-            if (it > 0) {  // the previous dV/dK MMAs must have read P and dS
-                ok = mbar_wait(bar(B_PDSFREE), (it - 1) & 1, abort_flag, a.status);
+            if (it >= 2) {  // the dV/dK MMAs of it - 2 must have read this P/dS buffer
+                ok = mbar_wait(bar(B_PDSFREE + buf), ((it >> 1) - 1) & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
             }
+            uint8_t* pds = smem + kOffPDS + buf * kPDS;
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const uint32_t off = sw_off(row, 4 * kh + q);
-                *reinterpret_cast<uint4*>(smem + kOffP + off) =
+                *reinterpret_cast<uint4*>(pds + off) =
                     make_uint4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
-                *reinterpret_cast<uint4*>(smem + kOffDS + off) =
+                *reinterpret_cast<uint4*>(pds + kHalf128 + off) =
                     make_uint4(dp[4 * q], dp[4 * q + 1], dp[4 * q + 2], dp[4 * q + 3]);
             }
             fence_proxy_async_smem();
-            mbar_arrive(bar(B_PDSFULL));
+            mbar_arrive(bar(B_PDSFULL + buf));
         }
         if (ok && n_it > 0) {
             ok = mbar_wait(bar(B_FINAL), 0, abort_flag, a.status);
