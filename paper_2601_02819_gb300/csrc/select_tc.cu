@@ -1,6 +1,7 @@
 // Stage (b) on the tensor cores for GQA pairs (G*64 = 128 query rows):
-// query-to-block relevance and Top-K selection (Eq. 8; Algorithm 1 step 3),
-// one CTA per (query block qb, KV head g), 320 threads.
+// query-to-block relevance and Top-K selection (Eq. 8; Algorithm 1 step 3).
+// Persistent: a CTA (352 threads, 2 per SM) walks the units (query block qb,
+// KV head g) u = blockIdx.x, blockIdx.x + gridDim.x, ...
 //
 // The candidate representative keys C = [n_init, qb - n_local] stream through
 // a two-slot shared-memory ring in chunks of 128 rows (TMA). Each chunk is
@@ -14,10 +15,12 @@
 //           sum p = 2^(S*scale - m_r)/Z_r over their 64 rows in row order;
 //           A[t] = half 0 + half 1. Every candidate follows the same order,
 //           so equal candidates get bit-identical sums.
-//   top-k   over the 64-bit key (bits(A) << 32 | ~t): larger A first, lower
-//           t on exact ties; two levels over the 8 warps (topk.cuh).
-// Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs.
-// Every wait is bounded in time (tc_common.cuh).
+//   top-k   a dedicated warp, on a double-buffered copy of A, while the
+//           elementwise warps already score the next unit: larger A first,
+//           lower t on exact ties (topk.cuh).
+// Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs,
+// warp 10 the top-k. The ring, the TMEM buffers and every barrier run on
+// counters that continue across units. Every wait is bounded in time.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "tc_common.cuh"
@@ -36,25 +39,50 @@ constexpr int kOffQ = 0;
 constexpr int kOffKr = kOffQ + kTile;      // 2 slots
 constexpr int kOffStats = kOffKr + 2 * kTile;  // m2[128], iz[128], half partials m[2][128], z[2][128]
 constexpr int kOffBar = kOffStats + 6 * 128 * 4;
-constexpr int B_Q = 0, B_KFULL = 1, B_KEMPTY = 3, B_SFULL = 5, B_SFREE = 7, B_DRAIN = 9,
-              kNumBars = 10;
+constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = 4, B_SFULL = 6, B_SFREE = 8,
+              B_AFULL = 10, B_AFREE = 12, B_DRAIN = 14, kNumBars = 15;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
-constexpr int kOffFin = kOffMisc + 48;            // top-k finalist keys [8 warps][kFinalMax], u64
-constexpr int kOffA = kOffFin + 8 * topk::kFinalMax * 8;  // A0[NQB], A1[NQB], then sel[topk]
-constexpr int kThreads = 320;
+constexpr int kOffA = kOffMisc + 16;  // 2 buffers x (A0[NQB], A1[NQB]), then sel[topk]
+constexpr int kThreads = 352;
 constexpr uint32_t kTmemCols = 256;
+constexpr int kRegKeys = 16;  // candidate keys per lane kept in registers by the top-k warp
 
 size_t select_tc_smem(int nqb, int topk) {
-    return 1024 + (size_t)kOffA + (size_t)nqb * 8 + (size_t)topk * 4 + 16;
+    return 1024 + (size_t)kOffA + (size_t)nqb * 16 + (size_t)topk * 4 + 16;
 }
 
 struct SelArgs {
     int32_t* idx_out;
     int32_t* cnt_out;
     int* status;
-    int Hq, Hkv, L, T, NQB, topk, n_init, n_local;
+    int Hq, Hkv, L, T, NQB, topk, n_init, n_local, units;
     float scale_log2;
 };
+
+// Everything about a unit that every role derives the same way.
+struct SelUnit {
+    int qb, bg, hq0, n_init_q, loc_lo, c_lo, c_hi, nC, nF, ksel, nch;
+    long long lu;
+    bool scored;  // false: the budget covers every candidate, nothing to score
+};
+
+__device__ __forceinline__ SelUnit sel_unit(const SelArgs& a, int u) {
+    SelUnit d;
+    d.qb = a.NQB - 1 - (u % a.NQB);  // heaviest query blocks first
+    d.bg = u / a.NQB;
+    d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
+    d.lu = (long long)d.bg * a.NQB + d.qb;
+    d.n_init_q = min(a.n_init, d.qb + 1);                // forced initial [0, n_init_q)
+    d.loc_lo = max(d.n_init_q, d.qb - a.n_local + 1);    // forced local [loc_lo, qb]
+    d.c_lo = a.n_init;                                   // candidates [c_lo, c_hi]
+    d.c_hi = d.qb - a.n_local;
+    d.nC = max(0, d.c_hi - d.c_lo + 1);
+    d.nF = d.n_init_q + (d.qb - d.loc_lo + 1);
+    d.ksel = a.topk - d.nF;
+    d.scored = d.ksel < d.nC;
+    d.nch = d.scored ? (d.nC + kCand - 1) / kCand : 0;  // chunks per pass
+    return d;
+}
 
 __global__ void __launch_bounds__(kThreads, 2)
 select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKr,
@@ -64,52 +92,25 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                                                ~uintptr_t(1023));
     const uint32_t sb = smem_u32(smem);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int unit = blockIdx.x;
-    const int qb = a.NQB - 1 - (unit % a.NQB);  // heaviest query blocks first
-    const int bg = unit / a.NQB;
-    const int b = bg / a.Hkv, g = bg % a.Hkv;
-    const long long lu = (long long)bg * a.NQB + qb;
-    int32_t* out = a.idx_out + lu * a.topk;
-
-    const int n_init_q = min(a.n_init, qb + 1);            // forced initial [0, n_init_q)
-    const int loc_lo = max(n_init_q, qb - a.n_local + 1);  // forced local [loc_lo, qb]
-    const int c_lo = a.n_init, c_hi = qb - a.n_local;      // candidates [c_lo, c_hi]
-    const int nC = max(0, c_hi - c_lo + 1);
-    const int nF = n_init_q + (qb - loc_lo + 1);
-    const int ksel = a.topk - nF;
-
-    if (ksel >= nC) {  // the budget covers every candidate: nothing to score
-        const int n = nF + nC;
-        for (int j = tid; j < a.topk; j += kThreads) {
-            int v = -1;
-            if (j < n_init_q) v = j;
-            else if (j < n_init_q + nC) v = c_lo + (j - n_init_q);
-            else if (j < n) v = loc_lo + (j - n_init_q - nC);
-            out[j] = v;
-        }
-        if (tid == 0) a.cnt_out[lu] = n;
-        return;
-    }
-
     auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
     float* m2s = reinterpret_cast<float*>(smem + kOffStats);
     float* izs = m2s + 128;
     float* pm = izs + 128;  // [2][128] per-half running max (pass 1)
     float* pz = pm + 256;   // [2][128] per-half running sum
-    float* A0 = reinterpret_cast<float*>(smem + kOffA);  // per-half aggregates (pass 2)
-    float* A1 = A0 + a.NQB;
-    int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 8);
-    const int nch = (nC + kCand - 1) / kCand;  // chunks per pass
-    const int steps = 2 * nch;
+    float* Abuf = reinterpret_cast<float*>(smem + kOffA);  // [2][A0 | A1], NQB each
+    int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 16);
 
     if (tid == 0) {
         mbar_init(bar(B_Q), 1);
+        mbar_init(bar(B_QFREE), 1);
         for (int s = 0; s < 2; ++s) {
             mbar_init(bar(B_KFULL + s), 1);
             mbar_init(bar(B_KEMPTY + s), 1);
             mbar_init(bar(B_SFULL + s), 1);
             mbar_init(bar(B_SFREE + s), 256);
+            mbar_init(bar(B_AFULL + s), 256);
+            mbar_init(bar(B_AFREE + s), 1);
         }
         mbar_init(bar(B_DRAIN), 1);
         fence_barrier_init();
@@ -123,30 +124,46 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
-    const int hq0 = b * a.Hq + g * 2;
 
     if (warp == 8) {
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
             prefetch_tmap(&tmKr);
-            mbar_expect_tx(bar(B_Q), kTile);
-            for (int hl = 0; hl < 2; ++hl)
-                for (int dh = 0; dh < 2; ++dh)
-                    tma_load_3d(sb + kOffQ + dh * kHalf + hl * (kHalf / 2), &tmQ, bar(B_Q), dh * 64,
-                                qb * 64, hq0 + hl);
-            int issued = 0;
-            for (int s = 0; s < steps; ++s) {
-                const int slot = s & 1, c = s % nch;
-                if (s >= 2 && !mbar_wait(bar(B_KEMPTY + slot), ((s >> 1) - 1) & 1, abort_flag, a.status))
-                    break;
-                mbar_expect_tx(bar(B_KFULL + slot), kTile);
-                for (int dh = 0; dh < 2; ++dh)
-                    tma_load_3d(sb + kOffKr + slot * kTile + dh * kHalf, &tmKr, bar(B_KFULL + slot),
-                                dh * 64, c_lo + c * kCand, bg);
-                issued = s + 1;
+            prefetch_tmap(&tmQ);
+            int gs = 0, su = 0, q_last = -1;  // chunk loads issued; scored units begun
+            bool ok = true;
+            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+                const SelUnit d = sel_unit(a, u);
+                if (!d.scored) continue;
+                const int steps = 2 * d.nch;
+                for (int s = 0; ok && s < steps; ++s, ++gs) {
+                    const int slot = gs & 1, c = s % d.nch;
+                    if (gs >= 2 && !mbar_wait(bar(B_KEMPTY + slot), ((gs >> 1) - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(bar(B_KFULL + slot), kTile);
+                    for (int dh = 0; dh < 2; ++dh)
+                        tma_load_3d(sb + kOffKr + slot * kTile + dh * kHalf, &tmKr, bar(B_KFULL + slot),
+                                    dh * 64, d.c_lo + c * kCand, d.bg);
+                    if (s == 0) {  // Q once the previous unit's last MMA has read the old one
+                        if (su > 0 && !mbar_wait(bar(B_QFREE), (su - 1) & 1, abort_flag, a.status)) {
+                            ok = false;
+                            ++gs;
+                            break;
+                        }
+                        mbar_expect_tx(bar(B_Q), kTile);
+                        for (int hl = 0; hl < 2; ++hl)
+                            for (int dh = 0; dh < 2; ++dh)
+                                tma_load_3d(sb + kOffQ + dh * kHalf + hl * (kHalf / 2), &tmQ, bar(B_Q),
+                                            dh * 64, d.qb * 64, d.hq0 + hl);
+                        q_last = su;
+                    }
+                }
+                ++su;
             }
-            mbar_wait_drain(bar(B_Q), 0);
-            for (int s = issued - 2; s < issued; ++s)
+            if (q_last >= 0) mbar_wait_drain(bar(B_Q), q_last & 1);
+            for (int s = gs - 2; s < gs; ++s)
                 if (s >= 0) mbar_wait_drain(bar(B_KFULL + (s & 1)), (s >> 1) & 1);
         }
     } else if (warp == 9) {
@@ -155,149 +172,214 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             constexpr uint32_t idesc = idesc_bf16(128, 128, false);
             const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
             const uint64_t dKr0 = sdesc_sw128(sb + kOffKr, 16, 1024);
-            bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
-            tc_fence_after();
-            for (int s = 0; ok && s < steps; ++s) {
-                const int slot = s & 1;
-                if (!mbar_wait(bar(B_KFULL + slot), (s >> 1) & 1, abort_flag, a.status)) break;
-                if (s >= 2 && !mbar_wait(bar(B_SFREE + slot), ((s >> 1) - 1) & 1, abort_flag, a.status))
-                    break;
+            int gs = 0, su = 0;
+            bool ok = true;
+            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+                const SelUnit d = sel_unit(a, u);
+                if (!d.scored) continue;
+                ok = mbar_wait(bar(B_Q), su & 1, abort_flag, a.status);
                 tc_fence_after();
-                const uint64_t kr = sdesc_at(dKr0, slot * kTile);
-                const bool pass1 = s < nch;
+                const int steps = 2 * d.nch;
+                for (int s = 0; ok && s < steps; ++s, ++gs) {
+                    const int slot = gs & 1;
+                    ok = mbar_wait(bar(B_KFULL + slot), (gs >> 1) & 1, abort_flag, a.status) &&
+                         (gs < 2 || mbar_wait(bar(B_SFREE + slot), ((gs >> 1) - 1) & 1, abort_flag, a.status));
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint64_t kr = sdesc_at(dKr0, slot * kTile);
+                    const bool pass1 = s < d.nch;
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {
-                    const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
-                    const uint64_t dq = sdesc_at(dQ0, off);
-                    const uint64_t dk = sdesc_at(kr, off);
-                    // pass 1: rows x candidates; pass 2: candidates x rows
-                    mma_ss(tmem + 128u * slot, pass1 ? dq : dk, pass1 ? dk : dq, idesc,
-                           ks > 0 ? 1u : 0u);
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
+                        const uint64_t dq = sdesc_at(dQ0, off);
+                        const uint64_t dk = sdesc_at(kr, off);
+                        // pass 1: rows x candidates; pass 2: candidates x rows
+                        mma_ss(tmem + 128u * slot, pass1 ? dq : dk, pass1 ? dk : dq, idesc,
+                               ks > 0 ? 1u : 0u);
+                    }
+                    mma_commit(bar(B_SFULL + slot));
+                    mma_commit(bar(B_KEMPTY + slot));
                 }
-                mma_commit(bar(B_SFULL + slot));
-                mma_commit(bar(B_KEMPTY + slot));
+                if (ok) mma_commit(bar(B_QFREE));  // this unit's MMAs are all issued
+                ++su;
             }
             mma_commit(bar(B_DRAIN));
             mbar_wait_drain(bar(B_DRAIN), 0);
+        }
+    } else if (warp == 10) {
+        // ------------------------------------------------ top-k (one warp)
+        int su = 0;
+        bool ok = true;
+        for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+            const SelUnit d = sel_unit(a, u);
+            int32_t* out = a.idx_out + d.lu * a.topk;
+            if (!d.scored) {  // the budget covers every candidate
+                const int n = d.nF + d.nC;
+                for (int j = lane; j < a.topk; j += 32) {
+                    int v = -1;
+                    if (j < d.n_init_q) v = j;
+                    else if (j < d.n_init_q + d.nC) v = d.c_lo + (j - d.n_init_q);
+                    else if (j < n) v = d.loc_lo + (j - d.n_init_q - d.nC);
+                    out[j] = v;
+                }
+                if (lane == 0) a.cnt_out[d.lu] = n;
+                continue;
+            }
+            const int buf = su & 1;
+            ok = mbar_wait(bar(B_AFULL + buf), (su >> 1) & 1, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
+            float* A1 = A0 + a.NQB;
+            // key = bits(A) << 32 | ~t, A = half 0 + half 1 (the same order for every
+            // candidate); each lane holds its candidates' keys in registers
+            const int nC = d.nC, ksel = d.ksel, c_lo = d.c_lo;
+            if (nC <= 32 * kRegKeys) {
+                unsigned long long key[kRegKeys];
+#pragma unroll
+                for (int r = 0; r < kRegKeys; ++r) {
+                    const int cj = lane + 32 * r;
+                    key[r] = cj < nC ? topk::make_key(A0[cj] + A1[cj], c_lo + cj) : 0ull;
+                }
+                for (int k = 0; k < ksel; ++k) {
+                    unsigned long long best = key[0];
+#pragma unroll
+                    for (int r = 1; r < kRegKeys; ++r) best = topk::umax64(best, key[r]);
+                    const unsigned mh = (unsigned)(best >> 32), ml = (unsigned)best;
+                    const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
+                    const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
+                    const unsigned long long win = ((unsigned long long)bh << 32) | bl;
+                    if (lane == 0) sel[k] = topk::key_block(win);
+#pragma unroll
+                    for (int r = 0; r < kRegKeys; ++r)
+                        if (key[r] == win) key[r] = 0ull;
+                }
+            } else {
+                topk::rounds_one_warp(
+                    nC, ksel, [&](int cj) { return topk::make_key(A0[cj] + A1[cj], c_lo + cj); },
+                    [&](int cj) { return A0[cj] == -1.0f; }, [&](int t) { A0[t - c_lo] = -1.0f; }, sel,
+                    lane);
+            }
+            __syncwarp();
+            // A is no longer needed: the elementwise warps may refill this buffer
+            if (lane == 0) mbar_arrive(bar(B_AFREE + buf));
+            for (int j = lane; j < a.topk; j += 32) {
+                if (j < d.n_init_q) out[j] = j;
+                else if (j >= d.n_init_q + ksel && j < d.nF + ksel) out[j] = d.loc_lo + (j - d.n_init_q - ksel);
+                else if (j >= d.nF + ksel) out[j] = -1;
+            }
+            for (int j = lane; j < ksel; j += 32) {
+                const int v = sel[j];
+                int rank = 0;
+                for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
+                out[d.n_init_q + rank] = v;
+            }
+            if (lane == 0) a.cnt_out[d.lu] = d.nF + ksel;
+            __syncwarp();  // sel is reused by the next unit
+            ++su;
         }
     } else {
         // ------------------------------------------------ elementwise (8 warps)
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         const int r = (warp & 3) * 32 + lane;  // pass 1: query row; pass 2: candidate
         const int hh = warp >> 2;              // half of the TMEM columns this thread reads
-        const bool row_ok = qb * 64 + (r & 63) < a.L;
-        float m = -INFINITY, z = 0.f;
         bool ok = true;
-        // After a failed wait the loop keeps running without work, so that all eight
+        int gs = 0, su = 0;
+        // After a failed wait the loops keep running without work, so that all eight
         // warps reach the named barriers after pass 1 the same number of times.
-        for (int s = 0; s < steps; ++s) {
-            const int slot = s & 1, c = s % nch;
-            if (ok) {
-                ok = mbar_wait(bar(B_SFULL + slot), (s >> 1) & 1, abort_flag, a.status);
+        for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
+            const SelUnit d = sel_unit(a, u);
+            if (!d.scored) continue;
+            const int nch = d.nch, steps = 2 * nch, c_lo = d.c_lo, c_hi = d.c_hi, nC = d.nC;
+            const bool row_ok = d.qb * 64 + (r & 63) < a.L;
+            const int buf = su & 1;
+            float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
+            float* A1 = A0 + a.NQB;
+            if (ok && su >= 2) {  // the top-k warp is done with this buffer's previous unit
+                ok = mbar_wait(bar(B_AFREE + buf), ((su >> 1) - 1) & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
-            if (ok) tc_fence_after();
-            if (ok && s < nch) {
-                // pass 1: row r against 64 candidates of the chunk, two loads of 32
-                const int t0 = c_lo + c * kCand + 64 * hh;
-                const bool full = t0 + 63 <= c_hi;
+            float m = -INFINITY, z = 0.f;
+            for (int s = 0; s < steps; ++s, ++gs) {
+                const int slot = gs & 1, c = s % nch;
+                if (ok) {
+                    ok = mbar_wait(bar(B_SFULL + slot), (gs >> 1) & 1, abort_flag, a.status);
+                    ok = __all_sync(0xffffffffu, ok);
+                }
+                if (ok) tc_fence_after();
+                if (ok && s < nch) {
+                    // pass 1: row r against 64 candidates of the chunk, two loads of 32
+                    const int t0 = c_lo + c * kCand + 64 * hh;
+                    const bool full = t0 + 63 <= c_hi;
 #pragma unroll 1
-                for (int q = 0; q < 2; ++q) {
-                    if (t0 + 32 * q > c_hi) break;  // no candidate left in this group (warp-uniform)
-                    uint32_t v[32];
-                    tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
-                    float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    for (int q = 0; q < 2; ++q) {
+                        if (t0 + 32 * q > c_hi) break;  // no candidate left in this group (warp-uniform)
+                        uint32_t v[32];
+                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+                        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        float x = __uint_as_float(v[j]) * a.scale_log2;
-                        if (!full && t0 + 32 * q + j > c_hi) x = -INFINITY;
-                        v[j] = __float_as_uint(x);
-                        m4[j & 3] = fmaxf(m4[j & 3], x);
-                    }
-                    const float mn = fmaxf(m, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])));
-                    if (mn != -INFINITY) {
-                        float s4[4] = {0.f, 0.f, 0.f, 0.f};
+                        for (int j = 0; j < 32; ++j) {
+                            float x = __uint_as_float(v[j]) * a.scale_log2;
+                            if (!full && t0 + 32 * q + j > c_hi) x = -INFINITY;
+                            v[j] = __float_as_uint(x);
+                            m4[j & 3] = fmaxf(m4[j & 3], x);
+                        }
+                        const float mn = fmaxf(m, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])));
+                        if (mn != -INFINITY) {
+                            float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) s4[j & 3] += ex2_approx(__uint_as_float(v[j]) - mn);
-                        z = z * ex2_approx(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
-                        m = mn;
+                            for (int j = 0; j < 32; ++j) s4[j & 3] += ex2_approx(__uint_as_float(v[j]) - mn);
+                            z = z * ex2_approx(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+                            m = mn;
+                        }
                     }
-                }
-                tc_fence_before();
-                mbar_arrive(bar(B_SFREE + slot));
-            } else if (ok) {
-                // pass 2: candidate r against the 64 rows of half hh, in row order;
-                // a warp whose 32 candidates all lie past the last one skips the work
-                const float* mrow = m2s + 64 * hh;
-                const float* irow = izs + 64 * hh;
-                float acc[4] = {0.f, 0.f, 0.f, 0.f};
-                const bool live = c * kCand + (warp & 3) * 32 < nC;
+                    tc_fence_before();
+                    mbar_arrive(bar(B_SFREE + slot));
+                } else if (ok) {
+                    // pass 2: candidate r against the 64 rows of half hh, in row order;
+                    // a warp whose 32 candidates all lie past the last one skips the work
+                    const float* mrow = m2s + 64 * hh;
+                    const float* irow = izs + 64 * hh;
+                    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                    const bool live = c * kCand + (warp & 3) * 32 < nC;
 #pragma unroll 1
-                for (int q = 0; q < (live ? 2 : 0); ++q) {
-                    uint32_t v[32];
-                    tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+                    for (int q = 0; q < (live ? 2 : 0); ++q) {
+                        uint32_t v[32];
+                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
 #pragma unroll
-                    for (int j = 0; j < 32; j += 4) {
-                        const float4 mm = *reinterpret_cast<const float4*>(mrow + 32 * q + j);
-                        const float4 iz = *reinterpret_cast<const float4*>(irow + 32 * q + j);
-                        acc[0] += ex2_approx(fmaf(__uint_as_float(v[j + 0]), a.scale_log2, -mm.x)) * iz.x;
-                        acc[1] += ex2_approx(fmaf(__uint_as_float(v[j + 1]), a.scale_log2, -mm.y)) * iz.y;
-                        acc[2] += ex2_approx(fmaf(__uint_as_float(v[j + 2]), a.scale_log2, -mm.z)) * iz.z;
-                        acc[3] += ex2_approx(fmaf(__uint_as_float(v[j + 3]), a.scale_log2, -mm.w)) * iz.w;
+                        for (int j = 0; j < 32; j += 4) {
+                            const float4 mm = *reinterpret_cast<const float4*>(mrow + 32 * q + j);
+                            const float4 iz = *reinterpret_cast<const float4*>(irow + 32 * q + j);
+                            acc[0] += ex2_approx(fmaf(__uint_as_float(v[j + 0]), a.scale_log2, -mm.x)) * iz.x;
+                            acc[1] += ex2_approx(fmaf(__uint_as_float(v[j + 1]), a.scale_log2, -mm.y)) * iz.y;
+                            acc[2] += ex2_approx(fmaf(__uint_as_float(v[j + 2]), a.scale_log2, -mm.z)) * iz.z;
+                            acc[3] += ex2_approx(fmaf(__uint_as_float(v[j + 3]), a.scale_log2, -mm.w)) * iz.w;
+                        }
                     }
+                    tc_fence_before();
+                    mbar_arrive(bar(B_SFREE + slot));
+                    const int cj = c * kCand + r;
+                    if (cj < nC) (hh ? A1 : A0)[cj] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
                 }
-                tc_fence_before();
-                mbar_arrive(bar(B_SFREE + slot));
-                const int cj = c * kCand + r;
-                if (cj < nC) (hh ? A1 : A0)[cj] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-            }
-            if (s == nch - 1) {
-                // merge the two column halves of every row: (m, z) -> max and 1/sum
-                pm[hh * 128 + r] = m;
-                pz[hh * 128 + r] = z;
-                named_barrier(1, 256);
-                if (hh == 0) {
-                    const float ma = pm[r], mb = pm[128 + r];
-                    const float mx = fmaxf(ma, mb);
-                    const float za = ma == -INFINITY ? 0.f : pz[r] * ex2_approx(ma - mx);
-                    const float zb = mb == -INFINITY ? 0.f : pz[128 + r] * ex2_approx(mb - mx);
-                    const float zz = za + zb;
-                    m2s[r] = row_ok ? mx : 0.f;
-                    izs[r] = (row_ok && zz > 0.f) ? 1.0f / zz : 0.f;
+                if (s == nch - 1) {
+                    // merge the two column halves of every row: (m, z) -> max and 1/sum
+                    pm[hh * 128 + r] = m;
+                    pz[hh * 128 + r] = z;
+                    named_barrier(1, 256);
+                    if (hh == 0) {
+                        const float ma = pm[r], mb = pm[128 + r];
+                        const float mx = fmaxf(ma, mb);
+                        const float za = ma == -INFINITY ? 0.f : pz[r] * ex2_approx(ma - mx);
+                        const float zb = mb == -INFINITY ? 0.f : pz[128 + r] * ex2_approx(mb - mx);
+                        const float zz = za + zb;
+                        m2s[r] = row_ok ? mx : 0.f;
+                        izs[r] = (row_ok && zz > 0.f) ? 1.0f / zz : 0.f;
+                    }
+                    named_barrier(1, 256);
                 }
-                named_barrier(1, 256);
             }
-        }
-        named_barrier(1, 256);  // every A0/A1 entry written
-        // top-k (topk.cuh): key = bits(A) << 32 | ~t with A = half 0 + half 1 (the
-        // same order for every candidate); a taken candidate is marked A0 = -1
-        // on the one-warp path.
-        auto key_of = [&](int cj) { return topk::make_key(A0[cj] + A1[cj], c_lo + cj); };
-        unsigned long long* fin = reinterpret_cast<unsigned long long*>(smem + kOffFin);
-        const bool fast = topk::two_level(nC, ksel);
-        if (ok && fast) {
-            topk::level1(nC, ksel, key_of, fin, warp, lane);
-        } else if (ok && warp == 0) {
-            topk::rounds_one_warp(
-                nC, ksel, key_of, [&](int cj) { return A0[cj] == -1.0f; },
-                [&](int t) { A0[t - c_lo] = -1.0f; }, sel, lane);
-        }
-        named_barrier(1, 256);
-        if (ok && fast) topk::level2(fin, ksel, sel, threadIdx.x);
-        named_barrier(1, 256);
-        if (ok) {
-            for (int j = threadIdx.x; j < a.topk; j += 256) {
-                if (j < n_init_q) out[j] = j;
-                else if (j >= n_init_q + ksel && j < nF + ksel) out[j] = loc_lo + (j - n_init_q - ksel);
-                else if (j >= nF + ksel) out[j] = -1;
-            }
-            for (int j = threadIdx.x; j < ksel; j += 256) {
-                const int v = sel[j];
-                int rank = 0;
-                for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
-                out[n_init_q + rank] = v;
-            }
-            if (threadIdx.x == 0) a.cnt_out[lu] = nF + ksel;
+            if (ok) mbar_arrive(bar(B_AFULL + buf));  // this thread's A entries are written
+            ++su;
         }
     }
     tc_fence_before();
@@ -329,10 +411,16 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
     cudaError_t e = cudaFuncSetAttribute(select_tc_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local,
+    int dev = 0, nsm = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    const int units = s.B * s.Hkv * NQB;
+    const int per_sm = smem * 2 + 2048 <= 228 * 1024 ? 2 : 1;  // two CTAs when shared memory allows
+    SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, units,
                  p.sm_scale * kLog2e};
     ProfScope prof(K_SELECT, st);
-    select_tc_kernel<<<(unsigned)((long long)s.B * s.Hkv * NQB), kThreads, smem, st>>>(tq, tkr, args);
+    select_tc_kernel<<<(unsigned)min(units, per_sm * nsm), kThreads, smem, st>>>(tq, tkr, args);
     return cudaGetLastError();
 }
 
