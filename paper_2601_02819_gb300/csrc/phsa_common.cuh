@@ -120,13 +120,23 @@ __device__ __forceinline__ void load_tile64(uint32_t dst, const __nv_bfloat16* s
 // anything else is skipped and recorded in the status word. Returns the count.
 __device__ __forceinline__ int compact_block_list(const int32_t* list, int n, int topk, int qb, int* out,
                                   int* status) {
+    // The whole row is read first, with independent loads (one memory latency
+    // per 16 entries), and compacted afterwards.
+    for (int j0 = 0; j0 < topk; j0 += 16) {
+        int v[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) v[k] = j0 + k < topk ? __ldg(list + j0 + k) : -1;
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+            if (j0 + k < topk) out[j0 + k] = v[k];
+    }
     if (n < 0 || n > topk) {
         set_status(status, PHSA_ERR_DEVICE_INDEX);
         n = n < 0 ? 0 : topk;
     }
     int k = 0, prev = -1;
     for (int j = 0; j < n; ++j) {
-        const int t = list[j];
+        const int t = out[j];
         if (t == -1) continue;
         if (t < 0 || t > qb || t <= prev) {
             set_status(status, PHSA_ERR_DEVICE_INDEX);
