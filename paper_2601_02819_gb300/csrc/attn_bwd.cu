@@ -113,8 +113,9 @@ __global__ void __launch_bounds__(1024)
 idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words, int work_max,
                  int slot_max, TInfo* __restrict__ tinfo, int32_t* __restrict__ qlist,
                  int2* __restrict__ work, int32_t* __restrict__ nwork, int* __restrict__ arrive,
-                 int* status) {
+                 int2* __restrict__ queue, int* __restrict__ qcount, int* status) {
     __shared__ int tmp[32];
+    __shared__ int cls_n[kQueueClasses];
     const int bg = blockIdx.x;
     const int per = (NQB + 1023) / 1024;  // KV blocks counted by each thread
     const int t0 = threadIdx.x * per;
@@ -137,7 +138,26 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     if (threadIdx.x == 0) {
         nwork[bg] = min(tch, work_max);
         if (tch > work_max || tsl > slot_max || tn > NQB * topk) set_status(status, PHSA_ERR_DEVICE_INDEX);
+        for (int c = 0; c < kQueueClasses; ++c) cls_n[c] = 0;
     }
+    __syncthreads();
+    // Items per size class (those that fit work_max), then one range of each
+    // class's queue for this (b, g)
+    for (int k = 0, ch = och; k < per; ++k) {
+        const int t = t0 + k;
+        if (t >= NQB) break;
+        int n = 0;
+        for (int w = 0; w < words; ++w) n += __popc(bb[(size_t)t * words + w]);
+        const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
+        for (int c = 0; c < nch && ch + c < work_max; ++c)
+            atomicAdd(&cls_n[queue_class(min(n, kChunk * c + kChunk) - kChunk * c)], 1);
+        ch += nch;
+    }
+    __syncthreads();
+    if (threadIdx.x < kQueueClasses)
+        cls_n[threadIdx.x] = atomicAdd(qcount + threadIdx.x, cls_n[threadIdx.x]);
+    __syncthreads();
+    const size_t qcap = (size_t)gridDim.x * work_max;
     TInfo* ti = tinfo + (size_t)bg * NQB;
     int2* wk = work + (size_t)bg * work_max;
     for (int k = 0; k < per; ++k) {
@@ -153,8 +173,11 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
         info.slot = (nch > 1 && osl + nch <= slot_max) ? osl : -1;
         ti[t] = info;
         arrive[(size_t)bg * NQB + t] = 0;
-        for (int c = 0; c < nch; ++c)
-            if (och + c < work_max) wk[och + c] = make_int2(t, c);
+        for (int c = 0; c < nch && och + c < work_max; ++c) {
+            wk[och + c] = make_int2(t, c);
+            const int cls = queue_class(min(n, kChunk * c + kChunk) - kChunk * c);
+            queue[cls * qcap + atomicAdd(&cls_n[cls], 1)] = make_int2(bg * NQB + t, c);
+        }
         on += n;
         och += nch;
         osl += nch > 1 ? nch : 0;
@@ -615,11 +638,13 @@ BwdLayout bwd_layout(const phsa_shape& s, int topk) {
     l.work_max = (int)(l.nqb + (nnz_max + kChunk - 1) / kChunk);
     l.slot_max = (int)((2 * nnz_max + kChunk - 1) / kChunk);
     size_t off = 0;
+    l.qctl = off;    off = align256(off + 8 * 4);
     l.bits = off;    off = align256(off + (size_t)bgs * l.nqb * l.words * 4);
     l.tinfo = off;   off = align256(off + (size_t)bgs * l.nqb * sizeof(TInfo));
     l.qlist = off;   off = align256(off + (size_t)bgs * nnz_max * 4);
     l.work = off;    off = align256(off + (size_t)bgs * l.work_max * sizeof(int2));
     l.nwork = off;   off = align256(off + (size_t)bgs * 4);
+    l.queue = off;   off = align256(off + (size_t)kQueueClasses * bgs * l.work_max * sizeof(int2));
     l.delta = off;   off = align256(off + (size_t)s.B * s.Hq * s.L * 4);
     l.partial = off; off = align256(off + (size_t)bgs * l.slot_max * 2 * kM * kD * 4);
     l.arrive = off;  off = align256(off + (size_t)bgs * l.nqb * 4);
@@ -643,6 +668,8 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     float* delta = reinterpret_cast<float*>(w + l.delta);
     float* partial = reinterpret_cast<float*>(w + l.partial);
     int* arrive = reinterpret_cast<int*>(w + l.arrive);
+    int2* queue = reinterpret_cast<int2*>(w + l.queue);
+    int* qctl = reinterpret_cast<int*>(w + l.qctl);
     const int bgs = s.B * s.Hkv;
     const long long rows = (long long)s.B * s.Hq * s.L;
     cudaError_t e;
@@ -662,7 +689,9 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
-    if ((e = cudaMemsetAsync(bits, 0, (size_t)bgs * l.nqb * l.words * 4, st)) != cudaSuccess)
+    // the queue counters and the bitmap, in one memset
+    if ((e = cudaMemsetAsync(w + l.qctl, 0, l.bits - l.qctl + (size_t)bgs * l.nqb * l.words * 4,
+                             st)) != cudaSuccess)
         return e;
     const long long units = (long long)bgs * l.nqb;
     {
@@ -675,12 +704,12 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
         ProfScope prof(K_BWD_BUILD, st);
         idx_build_kernel<<<bgs, 1024, 0, st>>>(bits, l.nqb, topk, l.words, l.work_max,
                                                l.slot_max, tinfo, qlist, work, nwork, arrive,
-                                               status);
+                                               queue, qctl, status);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
     if (pair)  // sums multi-chunk partials itself
-        return launch_dkdv_tc(Q, K, V, dO, lse, delta, tinfo, qlist, work, nwork, s, topk,
+        return launch_dkdv_tc(Q, K, V, dO, lse, delta, tinfo, qlist, queue, qctl, s, topk,
                               l.work_max, l.slot_max, sm_scale, dK, dV, partial, arrive, status,
                               st);
 

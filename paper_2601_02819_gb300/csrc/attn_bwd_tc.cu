@@ -17,8 +17,10 @@
 //   runs after this one. A fourth producer warp loads each unit's Q and dO as
 //   soon as the previous unit's last dP has been issued and its Delta read.
 //
-// dkdv_tc_kernel: one CTA per work item (KV block t, chunk of <= 32 query
-//   blocks that selected t), 320 threads. K_t and V_t stay in shared memory;
+// dkdv_tc_kernel: persistent, one CTA per SM over the work items (KV block t,
+//   chunk of <= 32 query blocks that selected t), 320 threads; K_t and V_t are
+//   reloaded per item as soon as its predecessor's S/dP MMAs are done, and the
+//   dV^T/dK^T accumulators are double-buffered in TMEM. K_t and V_t stay in shared memory;
 //   the Q and dO tiles (both heads stacked: 128 rows) of every listed query
 //   block stream through a two-stage ring:
 //     S  = Q K_t^T, dP = dO V_t^T            (M128 N64 K128)
@@ -26,7 +28,7 @@
 //     dV^T += dO^T P, dK^T += Q^T dS          (M128 N64 K128; A = dO / Q read
 //                                             MN-major, B = P / dS MN-major)
 //   dK^T and dV^T live in TMEM with the head dimension on the lanes. A KV
-//   block with a single chunk writes bf16 dK, dV through TMA stores; a longer
+//   block with a single chunk writes bf16 dK, dV straight from registers; a longer
 //   list writes fp32 partials, and the chunk that finishes last (an atomic
 //   counter per KV block) adds them in chunk order and stores the bf16 tile, so
 //   the sum does not depend on which CTA finishes last.
@@ -562,6 +564,15 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
 }
 
 // ============================================================== dK / dV
+// Persistent: one CTA per SM takes work items (KV block t of one (b, g), chunk
+// of <= 32 query blocks that selected t) from a global queue ordered by size
+// class, longest first, by tickets from one counter, so the SMs end together.
+// The producer thread takes the tickets and hands each item to the MMA and
+// elementwise roles through a ring in shared memory. K_t/V_t are reloaded as
+// soon as the previous item's last S/dP MMAs are done, the Q/dO ring, the S/dP
+// and P/dS buffers run on counters that continue across items, and the
+// dV^T/dK^T accumulators are double-buffered in TMEM, so an item's epilogue
+// overlaps the next item's work.
 namespace kv {
 constexpr int kOffK = 0;
 constexpr int kOffV = kOffK + kTile64;
@@ -572,15 +583,24 @@ constexpr int kStage = 2 * kTile128;
 constexpr int kOffPDS = kOffStage + 2 * kStage;
 constexpr int kPDS = 2 * kHalf128;
 constexpr int kOffBar = kOffPDS + 2 * kPDS;
-constexpr int B_KV = 0, B_QFULL = 1, B_QEMPTY = 3, B_SPFULL = 5, B_PDSFULL = 7, B_PDSFREE = 9,
-              B_FINAL = 11, B_DRAIN = 12, kNumBars = 13;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;
-constexpr int kOffQL = kOffMisc + 16;  // the work item's query blocks (at most kBwdChunk)
+constexpr int kRing = 8;  // item descriptors in flight
+constexpr int B_KV = 0, B_KVFREE = 1, B_QFULL = 2, B_QEMPTY = 4, B_SPFULL = 6, B_PDSFULL = 8,
+              B_PDSFREE = 10, B_FINAL = 12, B_DKVFREE = 14, B_DRAIN = 16, B_IFULL = 17,
+              B_IFREE = B_IFULL + kRing, kNumBars = B_IFREE + kRing;
+constexpr int kIFreeCount = 9;  // the MMA thread and the 8 elementwise warps
+constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag, last-arriver flag
+constexpr int kOffQL = kOffMisc + 16;  // the producer's copy of an item's query blocks
+constexpr int kOffN = kOffQL + kBwdChunk * 4;  // iteration counts of recent items [4]
+constexpr int kOffRing = (kOffN + 16 + 15) / 16 * 16;  // item descriptors [kRing][8 ints]
 constexpr int kThreads = 320;  // 8 elementwise warps, producer, MMA
-constexpr uint32_t kColDV = 256, kColDK = 320;
+// TMEM: S of iteration buffer b at 128b, dP at 64 + 128b; dV^T and dK^T of
+// accumulator buffer c at 256 + 128c and 320 + 128c.
 __device__ __forceinline__ uint32_t col_s(int b) { return 128u * (uint32_t)b; }
 __device__ __forceinline__ uint32_t col_dp(int b) { return 64u + 128u * (uint32_t)b; }
-constexpr size_t kSmem = 1024 + (size_t)kOffQL + kBwdChunk * 4;
+__device__ __forceinline__ uint32_t col_dv(int c) { return 256u + 128u * (uint32_t)c; }
+__device__ __forceinline__ uint32_t col_dk(int c) { return 320u + 128u * (uint32_t)c; }
+constexpr size_t kSmem = 1024 + (size_t)kOffRing + kRing * 32;
+static_assert(kSmem <= 227 * 1024, "dK/dV shared memory");
 }  // namespace kv
 
 struct KvArgs {
@@ -588,59 +608,106 @@ struct KvArgs {
     const float* delta;
     const BwdTInfo* tinfo;
     const int32_t* qlist;
-    const int2* work;
-    const int32_t* nwork;
+    const int2* queue;    // [kQueueClasses][qcap] {bg * NQB + t, chunk}
+    const int* qcount;    // items per class
+    int* ticket;          // next queue position to take
     float* partial;
     int* arrive;  // per (b, g, t): chunks of t finished so far
+    __nv_bfloat16* dK;
+    __nv_bfloat16* dV;
     int* status;
-    int Hq, Hkv, L, NQB, topk, work_max, slot_max;
+    long long qcap;
+    int Hq, Hkv, L, NQB, topk, slot_max;
     float scale_log2, sm_scale;
 };
+
+// One work item as the ring carries it (8 ints); n_it < 0 ends the stream.
+struct KvItem {
+    int bg, t, chunk, n_it;
+    BwdTInfo info;
+};
+
+// Queue position j -> its entry {bg * NQB + t, chunk}; valid = false past the end.
+__device__ __forceinline__ int2 queue_entry(const KvArgs& a, const int* qn, int j, bool& valid) {
+    int c = 0;
+#pragma unroll
+    for (int k = 0; k < kQueueClasses; ++k)
+        if (c == k && j >= qn[k]) {
+            j -= qn[k];
+            ++c;
+        }
+    valid = c < kQueueClasses;
+    return valid ? a.queue[(size_t)c * a.qcap + j] : make_int2(0, 0);
+}
+
+__device__ __forceinline__ KvItem item_of(const KvArgs& a, int2 e, const BwdTInfo& info) {
+    KvItem it;
+    it.bg = e.x / a.NQB;
+    it.t = e.x - it.bg * a.NQB;
+    it.chunk = e.y;
+    it.info = info;
+    const int q_begin = e.y * kBwdChunk;
+    it.n_it = max(0, min(info.n, q_begin + kBwdChunk) - q_begin);
+    return it;
+}
+
+__device__ __forceinline__ const int32_t* item_qlist(const KvArgs& a, const KvItem& it) {
+    return a.qlist + (size_t)it.bg * a.NQB * a.topk + it.info.off + it.chunk * kBwdChunk;
+}
+
+__device__ __forceinline__ void ring_put(int* e, const KvItem& it) {
+    *reinterpret_cast<int4*>(e) = make_int4(it.bg, it.t, it.chunk, it.n_it);
+    *reinterpret_cast<int4*>(e + 4) = make_int4(it.info.off, it.info.n, it.info.nch, it.info.slot);
+}
+
+__device__ __forceinline__ KvItem ring_get(const int* e) {
+    const int4 x = *reinterpret_cast<const int4*>(e);
+    const int4 y = *reinterpret_cast<const int4*>(e + 4);
+    KvItem it;
+    it.bg = x.x;
+    it.t = x.y;
+    it.chunk = x.z;
+    it.n_it = x.w;
+    it.info.off = y.x;
+    it.info.n = y.y;
+    it.info.nch = y.z;
+    it.info.slot = y.w;
+    return it;
+}
 
 __global__ void __launch_bounds__(kv::kThreads, 1)
 dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
-               const __grid_constant__ CUtensorMap tmdK, const __grid_constant__ CUtensorMap tmdV,
                const KvArgs a) {
     using namespace kv;
-    const int bg = blockIdx.y;
-    if ((int)blockIdx.x >= a.nwork[bg]) return;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     const uint32_t sb = smem_u32(smem);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = bg / a.Hkv, g = bg % a.Hkv;
-    const int2 wi = a.work[(size_t)bg * a.work_max + blockIdx.x];
-    const int t = wi.x, chunk = wi.y;
-    const BwdTInfo info = a.tinfo[(size_t)bg * a.NQB + t];
-    const int q_begin = chunk * kBwdChunk;
-    const int n_it = max(0, min(info.n, q_begin + kBwdChunk) - q_begin);
-    const int32_t* ql = a.qlist + (size_t)bg * a.NQB * a.topk + info.off + q_begin;
     auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
-    const int hq0 = b * a.Hq + g * 2;
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_KV), 1);
+        mbar_init(bar(B_KVFREE), 1);
         for (int s = 0; s < 2; ++s) {
             mbar_init(bar(B_QFULL + s), 1);
             mbar_init(bar(B_QEMPTY + s), 1);
             mbar_init(bar(B_SPFULL + s), 1);
+            mbar_init(bar(B_PDSFULL + s), 256);
+            mbar_init(bar(B_PDSFREE + s), 1);
+            mbar_init(bar(B_FINAL + s), 1);
+            mbar_init(bar(B_DKVFREE + s), 256);
         }
-        for (int b2 = 0; b2 < 2; ++b2) {
-            mbar_init(bar(B_PDSFULL + b2), 256);
-            mbar_init(bar(B_PDSFREE + b2), 1);
-        }
-        mbar_init(bar(B_FINAL), 1);
         mbar_init(bar(B_DRAIN), 1);
+        for (int r = 0; r < kRing; ++r) {
+            mbar_init(bar(B_IFULL + r), 1);
+            mbar_init(bar(B_IFREE + r), kIFreeCount);
+        }
         fence_barrier_init();
         *abort_flag = 0;
     }
-    // The query-block list of this work item, staged once (one load per thread)
-    // so that no load or row fetch waits on it later.
-    int* qls = reinterpret_cast<int*>(smem + kOffQL);
-    if ((int)threadIdx.x < n_it) qls[threadIdx.x] = __ldg(ql + threadIdx.x);
     if (warp == 9) {
         tmem_alloc(sb + kOffMisc, kTmemCols);
         tmem_relinquish();
@@ -652,38 +719,97 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 
     if (warp == 8) {
         // ------------------------------------------------ TMA producer
-        if (lane == 0 && n_it > 0) {
+        if (lane == 0) {
             prefetch_tmap(&tmQ);
             prefetch_tmap(&tmdO);
-            mbar_expect_tx(bar(B_KV), 2 * kTile64);
-            for (int dh = 0; dh < 2; ++dh) {
-                tma_load_3d(sb + kOffK + dh * kHalf64, &tmK, bar(B_KV), dh * 64, t * 64, bg);
-                tma_load_3d(sb + kOffV + dh * kHalf64, &tmV, bar(B_KV), dh * 64, t * 64, bg);
-            }
-            int issued = 0;
-            for (int i = 0; i < n_it; ++i) {
-                const int s = i & 1;
-                if (i >= 2 && !mbar_wait(bar(B_QEMPTY + s), ((i >> 1) - 1) & 1, abort_flag, a.status))
-                    break;
-                const int qb = qls[i];
-                const uint32_t st = sb + kOffStage + s * kStage;
-                mbar_expect_tx(bar(B_QFULL + s), kStage);
-                for (int hl = 0; hl < 2; ++hl)
-                    for (int dh = 0; dh < 2; ++dh) {
-                        tma_load_3d(st + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_QFULL + s),
-                                    dh * 64, qb * 64, hq0 + hl);
-                        tma_load_3d(st + kTile128 + dh * kHalf128 + hl * kHalf64, &tmdO,
-                                    bar(B_QFULL + s), dh * 64, qb * 64, hq0 + hl);
+            prefetch_tmap(&tmK);
+            prefetch_tmap(&tmV);
+            int* qls = reinterpret_cast<int*>(smem + kOffQL);
+            int* ring = reinterpret_cast<int*>(smem + kOffRing);
+            int qn[kQueueClasses];
+#pragma unroll
+            for (int c = 0; c < kQueueClasses; ++c)
+                qn[c] = (int)min((long long)max(a.qcount[c], 0), a.qcap);
+            int gi = 0, kvc = 0, r = 0;  // Q/dO stages issued; items with K/V loaded; ring items
+            bool ok = true;
+            // hands item x to the other roles once its ring slot's last reader is done
+            auto publish = [&](const KvItem& x) {
+                const int slot = r % kRing;
+                if (r >= kRing &&
+                    !mbar_wait(bar(B_IFREE + slot), ((r / kRing) - 1) & 1, abort_flag, a.status))
+                    return false;
+                ring_put(ring + slot * 8, x);
+                mbar_arrive(bar(B_IFULL + slot));
+                ++r;
+                return true;
+            };
+            auto entry_of = [&](int j, bool& valid) { return queue_entry(a, qn, j, valid); };
+            bool valid;
+            int2 e = entry_of(atomicAdd(a.ticket, 1), valid);
+            KvItem it;
+            it.n_it = -1;
+            if (valid) it = item_of(a, e, a.tinfo[e.x]);
+            ok = publish(it);
+            while (ok && it.n_it >= 0) {
+                // the next item's ticket now, its queue entry after this item's
+                // K/V loads and its block info after the Q/dO loads, so no load
+                // latency lies on the producer's path
+                const int j_nx = atomicAdd(a.ticket, 1);
+                bool nx_valid = false;
+                if (it.n_it > 0) {
+                    const int32_t* ql = item_qlist(a, it);
+                    // this item's query blocks, one batch of independent loads
+                    int v[kBwdChunk];
+#pragma unroll
+                    for (int j = 0; j < kBwdChunk; ++j) v[j] = j < it.n_it ? __ldg(ql + j) : 0;
+#pragma unroll
+                    for (int j = 0; j < kBwdChunk; ++j) qls[j] = v[j];
+                    // K_t and V_t, once the previous item's S/dP MMAs have read theirs
+                    if (kvc > 0 && !mbar_wait(bar(B_KVFREE), (kvc - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
                     }
-                issued = i + 1;
+                    mbar_expect_tx(bar(B_KV), 2 * kTile64);
+                    for (int dh = 0; dh < 2; ++dh) {
+                        tma_load_3d(sb + kOffK + dh * kHalf64, &tmK, bar(B_KV), dh * 64, it.t * 64, it.bg);
+                        tma_load_3d(sb + kOffV + dh * kHalf64, &tmV, bar(B_KV), dh * 64, it.t * 64, it.bg);
+                    }
+                    ++kvc;
+                    e = entry_of(j_nx, nx_valid);
+                    const int hq0 = (it.bg / a.Hkv) * a.Hq + (it.bg % a.Hkv) * 2;
+                    for (int i = 0; i < it.n_it; ++i, ++gi) {
+                        const int s = gi & 1;
+                        if (gi >= 2 &&
+                            !mbar_wait(bar(B_QEMPTY + s), ((gi >> 1) - 1) & 1, abort_flag, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        const int qb = qls[i];
+                        const uint32_t st = sb + kOffStage + s * kStage;
+                        mbar_expect_tx(bar(B_QFULL + s), kStage);
+                        for (int hl = 0; hl < 2; ++hl)
+                            for (int dh = 0; dh < 2; ++dh) {
+                                tma_load_3d(st + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_QFULL + s),
+                                            dh * 64, qb * 64, hq0 + hl);
+                                tma_load_3d(st + kTile128 + dh * kHalf128 + hl * kHalf64, &tmdO,
+                                            bar(B_QFULL + s), dh * 64, qb * 64, hq0 + hl);
+                            }
+                    }
+                    if (!ok) break;
+                } else {
+                    e = entry_of(j_nx, nx_valid);
+                }
+                it.n_it = -1;
+                if (nx_valid) it = item_of(a, e, a.tinfo[e.x]);
+                ok = publish(it);
             }
-            mbar_wait_drain(bar(B_KV), 0);
-            for (int i = issued - 2; i < issued; ++i)
+            if (kvc > 0) mbar_wait_drain(bar(B_KV), (kvc - 1) & 1);
+            for (int i = gi - 2; i < gi; ++i)
                 if (i >= 0) mbar_wait_drain(bar(B_QFULL + (i & 1)), (i >> 1) & 1);
         }
     } else if (warp == 9) {
         // ------------------------------------------------ MMA issuer
-        if (lane == 0 && n_it > 0) {
+        if (lane == 0) {
             constexpr uint32_t id_s = idesc_bf16(128, 64, false);
             constexpr uint32_t id_t = idesc_bf16(128, 64, true, true);  // A and B MN-major
             const uint64_t dSt0 = sdesc_sw128(sb + kOffStage, 16, 1024);          // Q/dO K-major
@@ -692,13 +818,30 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
             const uint64_t dP0 = sdesc_sw128(sb + kOffPDS, kHalf128, 1024);
             const uint64_t dS0 = sdesc_sw128(sb + kOffPDS + kHalf128, kHalf128, 1024);
-            bool ok = mbar_wait(bar(B_KV), 0, abort_flag, a.status);
-            tc_fence_after();
-            int ns = 0, nv = 0;
+            int* nring = reinterpret_cast<int*>(smem + kOffN);  // iteration counts, by item & 3
+            // Two streams over the items with at least one iteration:
+            //   S/dP stream  (ns: global iteration, s_item/s_pos/s_n: its item)
+            //   dV/dK stream (nv, v_item/v_pos), at most two iterations behind.
+            const int* ring = reinterpret_cast<const int*>(smem + kOffRing);
+            int ns = 0, nv = 0, s_item = 0, s_pos = 0, v_item = 0, v_pos = 0;
+            int r = 0, s_n = 0;       // ring items read; iterations of the S/dP stream's item
+            bool s_more = true;       // the ring has not ended
+            bool ok = true;
             Deadline dl;
-            while (ok && nv < n_it) {
+            while (ok && (s_more || nv < ns)) {
                 bool progressed = false;
-                if (ns < n_it && ns <= nv + 1 &&
+                if (s_more && s_n == 0 && mbar_test_wait(bar(B_IFULL + r % kRing), (r / kRing) & 1)) {
+                    // the next item; one without iterations has nothing to multiply
+                    const int n = ring_get(ring + (r % kRing) * 8).n_it;
+                    mbar_arrive(bar(B_IFREE + r % kRing));
+                    ++r;
+                    if (n < 0) s_more = false;
+                    s_n = max(n, 0);
+                    if (s_n > 0) nring[s_item & 3] = s_n;
+                    progressed = true;
+                }
+                if (s_n > 0 && ns <= nv + 1 &&
+                    (s_pos > 0 || mbar_test_wait(bar(B_KV), s_item & 1)) &&
                     mbar_test_wait(bar(B_QFULL + (ns & 1)), (ns >> 1) & 1)) {
                     tc_fence_after();
                     const uint64_t qd = sdesc_at(dSt0, (ns & 1) * kStage);
@@ -716,25 +859,37 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                                ks > 0 ? 1u : 0u);
                     mma_commit(bar(B_SPFULL + (ns & 1)));
                     ++ns;
+                    if (++s_pos == s_n) {  // the item's last S/dP: K_t/V_t may be replaced
+                        mma_commit(bar(B_KVFREE));
+                        ++s_item;
+                        s_pos = 0;
+                        s_n = 0;
+                    }
                     progressed = true;
                 }
-                if (nv < ns && mbar_test_wait(bar(B_PDSFULL + (nv & 1)), (nv >> 1) & 1)) {
+                const int c = v_item & 1;  // accumulator buffer
+                if (nv < ns && mbar_test_wait(bar(B_PDSFULL + (nv & 1)), (nv >> 1) & 1) &&
+                    (v_pos > 0 || v_item < 2 || mbar_test_wait(bar(B_DKVFREE + c), ((v_item >> 1) - 1) & 1))) {
                     tc_fence_after();
                     const uint64_t qt = sdesc_at(dStT0, (nv & 1) * kStage);
                     const uint32_t pb = (nv & 1) * kPDS;
                     // K dimension = the 128 stacked query rows, 16 per MMA
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + kColDV, sdesc_at(qt, kTile128 + ks * 2048),
-                               sdesc_at(dP0, pb + ks * 2048), id_t, (nv > 0 || ks > 0) ? 1u : 0u);
+                        mma_ss(tmem + col_dv(c), sdesc_at(qt, kTile128 + ks * 2048),
+                               sdesc_at(dP0, pb + ks * 2048), id_t, (v_pos > 0 || ks > 0) ? 1u : 0u);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + kColDK, sdesc_at(qt, ks * 2048), sdesc_at(dS0, pb + ks * 2048),
-                               id_t, (nv > 0 || ks > 0) ? 1u : 0u);
+                        mma_ss(tmem + col_dk(c), sdesc_at(qt, ks * 2048), sdesc_at(dS0, pb + ks * 2048),
+                               id_t, (v_pos > 0 || ks > 0) ? 1u : 0u);
                     mma_commit(bar(B_PDSFREE + (nv & 1)));
                     mma_commit(bar(B_QEMPTY + (nv & 1)));
-                    if (nv == n_it - 1) mma_commit(bar(B_FINAL));
                     ++nv;
+                    if (++v_pos == nring[v_item & 3]) {
+                        mma_commit(bar(B_FINAL + c));
+                        ++v_item;
+                        v_pos = 0;
+                    }
                     progressed = true;
                 }
                 if (progressed) {
@@ -756,151 +911,163 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const int kh = warp >> 2;                // keys [32 kh, 32 kh + 32)
         const int tok = row & 63, hl = row >> 6;
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-        const size_t hoff = (size_t)(hq0 + hl) * a.L;
-        // Row data (query block, lse, Delta) is fetched one iteration ahead so its
-        // global-memory latency overlaps the previous iteration.
-        auto fetch = [&](int it2, int& qb2, float& nl2, float& dl2) {
-            qb2 = qls[it2];
-            const int i2 = qb2 * 64 + tok;
-            const bool v2 = i2 < a.L;
-            nl2 = v2 ? -a.lse[hoff + i2] * kLog2e : -INFINITY;
-            dl2 = v2 ? a.delta[hoff + i2] : 0.f;
-        };
-        int qb_n = 0;
-        float nl_n = 0.f, dl_n = 0.f;
-        if (n_it > 0) fetch(0, qb_n, nl_n, dl_n);
         bool ok = true;
-        for (int it = 0; it < n_it; ++it) {
-            const int qb = qb_n;
-            const float neg_lse2 = nl_n;
-            const float dlt = dl_n;
-            if (it + 1 < n_it) fetch(it + 1, qb_n, nl_n, dl_n);
-            const int buf = it & 1;
-            ok = mbar_wait(bar(B_SPFULL + buf), (it >> 1) & 1, abort_flag, a.status);
-            ok = __all_sync(0xffffffffu, ok);
-            if (!ok) break;
-            tc_fence_after();
-            uint32_t sv[32], dp[32];
-            tmem_ld32(lane_base + col_s(buf) + 32 * kh, sv);
-            tmem_ld32(lane_base + col_dp(buf) + 32 * kh, dp);
-            const bool diag = qb == t;
-#pragma unroll
-            for (int c = 0; c < 16; ++c) {
-                float p[2], ds[2];
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int key = 32 * kh + 2 * c + e;
-                    float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + e]), a.scale_log2, neg_lse2));
-                    if (diag && key > tok) pv = 0.f;
-                    p[e] = pv;
-                    ds[e] = pv * (__uint_as_float(dp[2 * c + e]) - dlt);
-                }
-                sv[c] = pack2_bf16(p[0], p[1]);
-                dp[c] = pack2_bf16(ds[0], ds[1]);
-            }
-            tc_fence_before();
-            if (it >= 2) {  // the dV/dK MMAs of it - 2 must have read this P/dS buffer
-                ok = mbar_wait(bar(B_PDSFREE + buf), ((it >> 1) - 1) & 1, abort_flag, a.status);
+        int gi = 0, cu = 0;  // global iteration; items with iterations (accumulator uses)
+        const int* ring = reinterpret_cast<const int*>(smem + kOffRing);
+        for (int r = 0;; ++r) {
+            const int slot = r % kRing;
+            bool got = ok && mbar_wait(bar(B_IFULL + slot), (r / kRing) & 1, abort_flag, a.status);
+            got = __all_sync(0xffffffffu, got);
+            // the eight warps leave at the same item (the epilogue has barriers among them)
+            if (!named_barrier_and(2, 256, got)) break;
+            const KvItem it = ring_get(ring + slot * 8);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(B_IFREE + slot));
+            if (it.n_it < 0) break;
+            const int32_t* ql = item_qlist(a, it);
+            const int n_it = it.n_it, t = it.t, bg = it.bg;
+            const size_t hoff = (size_t)((bg / a.Hkv) * a.Hq + (bg % a.Hkv) * 2 + hl) * a.L;
+            // Row data (query block, lse, Delta) is fetched one iteration ahead so its
+            // global-memory latency overlaps the previous iteration.
+            auto fetch = [&](int it2, int& qb2, float& nl2, float& dl2) {
+                qb2 = __ldg(ql + it2);
+                const int i2 = qb2 * 64 + tok;
+                const bool v2 = i2 < a.L;
+                nl2 = v2 ? -__ldg(a.lse + hoff + i2) * kLog2e : -INFINITY;
+                dl2 = v2 ? __ldg(a.delta + hoff + i2) : 0.f;
+            };
+            int qb_n = 0;
+            float nl_n = 0.f, dl_n = 0.f;
+            if (n_it > 0) fetch(0, qb_n, nl_n, dl_n);
+            for (int i = 0; ok && i < n_it; ++i, ++gi) {
+                const int qb = qb_n;
+                const float neg_lse2 = nl_n;
+                const float dlt = dl_n;
+                if (i + 1 < n_it) fetch(i + 1, qb_n, nl_n, dl_n);
+                const int buf = gi & 1;
+                ok = mbar_wait(bar(B_SPFULL + buf), (gi >> 1) & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
+                tc_fence_after();
+                uint32_t sv[32], dp[32];
+                tmem_ld32(lane_base + col_s(buf) + 32 * kh, sv);
+                tmem_ld32(lane_base + col_dp(buf) + 32 * kh, dp);
+                const bool diag = qb == t;
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    float p[2], ds[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int key = 32 * kh + 2 * c + e;
+                        float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + e]), a.scale_log2, neg_lse2));
+                        if (diag && key > tok) pv = 0.f;
+                        p[e] = pv;
+                        ds[e] = pv * (__uint_as_float(dp[2 * c + e]) - dlt);
+                    }
+                    sv[c] = pack2_bf16(p[0], p[1]);
+                    dp[c] = pack2_bf16(ds[0], ds[1]);
+                }
+                tc_fence_before();
+                if (gi >= 2) {  // the dV/dK MMAs two iterations back must have read this buffer
+                    ok = mbar_wait(bar(B_PDSFREE + buf), ((gi >> 1) - 1) & 1, abort_flag, a.status);
+                    ok = __all_sync(0xffffffffu, ok);
+                    if (!ok) break;
+                }
+                uint8_t* pds = smem + kOffPDS + buf * kPDS;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint32_t off = sw_off(row, 4 * kh + q);
+                    *reinterpret_cast<uint4*>(pds + off) =
+                        make_uint4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
+                    *reinterpret_cast<uint4*>(pds + kHalf128 + off) =
+                        make_uint4(dp[4 * q], dp[4 * q + 1], dp[4 * q + 2], dp[4 * q + 3]);
+                }
+                fence_proxy_async_smem();
+                mbar_arrive(bar(B_PDSFULL + buf));
             }
-            uint8_t* pds = smem + kOffPDS + buf * kPDS;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint32_t off = sw_off(row, 4 * kh + q);
-                *reinterpret_cast<uint4*>(pds + off) =
-                    make_uint4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
-                *reinterpret_cast<uint4*>(pds + kHalf128 + off) =
-                    make_uint4(dp[4 * q], dp[4 * q + 1], dp[4 * q + 2], dp[4 * q + 3]);
-            }
-            fence_proxy_async_smem();
-            mbar_arrive(bar(B_PDSFULL + buf));
-        }
-        if (ok && n_it > 0) {
-            ok = mbar_wait(bar(B_FINAL), 0, abort_flag, a.status);
-            ok = __all_sync(0xffffffffu, ok);
-        }
-        // dV^T / dK^T: lane = head-dimension index d, columns = keys [32 kh, 32 kh + 32)
-        const int d = row;
-        uint32_t v[32], k[32];
-        if (ok && n_it > 0) {
-            tc_fence_after();
-            tmem_ld32(lane_base + kColDV + 32 * kh, v);
-            tmem_ld32(lane_base + kColDK + 32 * kh, k);
-        } else {
-#pragma unroll
-            for (int c = 0; c < 32; ++c) { v[c] = 0u; k[c] = 0u; }
-        }
-        bool store = ok;
-        if (info.nch > 1) {
-            // Multi-chunk list: write this chunk's fp32 partial; the chunk that
-            // arrives last adds all partials in chunk order and stores the tile.
-            float* base = a.partial + ((size_t)bg * a.slot_max + (info.slot < 0 ? 0 : info.slot)) *
-                                          2 * 64 * 128;
-            if (ok && info.slot >= 0) {
-                float* pk = base + (size_t)chunk * 2 * 64 * 128;
-                float* pv = pk + 64 * 128;
-#pragma unroll
-                for (int c = 0; c < 32; ++c) {
-                    const int key = 32 * kh + c;
-                    pk[key * 128 + d] = __uint_as_float(k[c]) * a.sm_scale;
-                    pv[key * 128 + d] = __uint_as_float(v[c]);
+            // ---- epilogue: dV^T / dK^T, lane = head-dimension index d, keys [32 kh, +32)
+            const int d = row;
+            uint32_t v[32], k[32];
+            if (ok && n_it > 0) {
+                const int c = cu & 1;
+                ok = mbar_wait(bar(B_FINAL + c), (cu >> 1) & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (ok) {
+                    tc_fence_after();
+                    tmem_ld32(lane_base + col_dv(c) + 32 * kh, v);
+                    tmem_ld32(lane_base + col_dk(c) + 32 * kh, k);
+                    tc_fence_before();
+                    mbar_arrive(bar(B_DKVFREE + c));  // the accumulators may be reused
                 }
             }
-            __threadfence();
-            named_barrier(1, 256);
-            volatile int* last_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 8);
-            if (threadIdx.x == 0)
-                *last_flag = (info.slot >= 0 &&
-                              atomicAdd(a.arrive + (size_t)bg * a.NQB + t, 1) == info.nch - 1);
-            named_barrier(1, 256);
-            store = ok && *last_flag;
-            if (store) {
-                __threadfence();
-                float sk[32], sv2[32];
+            if (!(ok && n_it > 0)) {
 #pragma unroll
-                for (int c = 0; c < 32; ++c) { sk[c] = 0.f; sv2[c] = 0.f; }
-                for (int ch = 0; ch < info.nch; ++ch) {
-                    const float* pk = base + (size_t)ch * 2 * 64 * 128;
+                for (int c = 0; c < 32; ++c) { v[c] = 0u; k[c] = 0u; }
+            }
+            if (n_it > 0) ++cu;
+            const BwdTInfo info = it.info;
+            bool store = ok;
+            float kscale = a.sm_scale;
+            if (info.nch > 1) {
+                // Multi-chunk list: write this chunk's fp32 partial; the chunk that
+                // arrives last adds all partials in chunk order and stores the tile.
+                float* base = a.partial + ((size_t)bg * a.slot_max + (info.slot < 0 ? 0 : info.slot)) *
+                                              2 * 64 * 128;
+                if (ok && info.slot >= 0) {
+                    float* pk = base + (size_t)it.chunk * 2 * 64 * 128;
+                    float* pv = pk + 64 * 128;
 #pragma unroll
                     for (int c = 0; c < 32; ++c) {
                         const int key = 32 * kh + c;
-                        sk[c] += __ldcg(pk + key * 128 + d);
-                        sv2[c] += __ldcg(pk + 64 * 128 + key * 128 + d);
+                        pk[key * 128 + d] = __uint_as_float(k[c]) * a.sm_scale;
+                        pv[key * 128 + d] = __uint_as_float(v[c]);
                     }
                 }
+                __threadfence();
+                named_barrier(1, 256);
+                volatile int* last_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 8);
+                if (threadIdx.x == 0)
+                    *last_flag = (ok && info.slot >= 0 &&
+                                  atomicAdd(a.arrive + (size_t)bg * a.NQB + t, 1) == info.nch - 1);
+                named_barrier(1, 256);
+                store = ok && *last_flag;
+                named_barrier(1, 256);  // every thread has read the flag before it is reused
+                kscale = 1.f;  // partial sums already carry the softmax scale
+                if (store) {
+                    __threadfence();
+                    float sk[32], sv2[32];
 #pragma unroll
-                for (int c = 0; c < 32; ++c) {
-                    k[c] = __float_as_uint(sk[c]);
-                    v[c] = __float_as_uint(sv2[c]);
+                    for (int c = 0; c < 32; ++c) { sk[c] = 0.f; sv2[c] = 0.f; }
+                    for (int ch = 0; ch < info.nch; ++ch) {
+                        const float* pk = base + (size_t)ch * 2 * 64 * 128;
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) {
+                            const int key = 32 * kh + c;
+                            sk[c] += __ldcg(pk + key * 128 + d);
+                            sv2[c] += __ldcg(pk + 64 * 128 + key * 128 + d);
+                        }
+                    }
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) {
+                        k[c] = __float_as_uint(sk[c]);
+                        v[c] = __float_as_uint(sv2[c]);
+                    }
                 }
             }
-        }
-        if (store) {
-            // bf16 tiles [64 keys][128 d] in the swizzled layout (stage-0 Q and dO
-            // regions); partial sums already carry the softmax scale.
-            const float kscale = info.nch > 1 ? 1.f : a.sm_scale;
-            uint8_t* tv = smem + kOffStage;
-            uint8_t* tk = smem + kOffStage + kTile128;
-            const int dh = d >> 6, dc = (d & 63) >> 3, de = d & 7;
+            if (store) {
+                // bf16 rows of dK and dV: for each key the 128 lanes of a warp group
+                // write one contiguous 256-byte row
+                __nv_bfloat16* dKr = a.dK + ((size_t)bg * a.L + (size_t)t * 64) * 128 + d;
+                __nv_bfloat16* dVr = a.dV + ((size_t)bg * a.L + (size_t)t * 64) * 128 + d;
 #pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                const int key = 32 * kh + c;
-                const uint32_t off = dh * kHalf64 + sw_off(key, dc) + de * 2;
-                *reinterpret_cast<__nv_bfloat16*>(tv + off) = __float2bfloat16_rn(__uint_as_float(v[c]));
-                *reinterpret_cast<__nv_bfloat16*>(tk + off) =
-                    __float2bfloat16_rn(__uint_as_float(k[c]) * kscale);
+                for (int c = 0; c < 32; ++c) {
+                    const int key = 32 * kh + c;
+                    if (t * 64 + key < a.L) {
+                        dVr[(size_t)key * 128] = __float2bfloat16_rn(__uint_as_float(v[c]));
+                        dKr[(size_t)key * 128] = __float2bfloat16_rn(__uint_as_float(k[c]) * kscale);
+                    }
+                }
             }
-            fence_proxy_async_smem();
-        }
-        named_barrier(1, 256);
-        if (threadIdx.x == 0 && store) {
-            for (int dh = 0; dh < 2; ++dh) {
-                tma_store_3d(&tmdV, sb + kOffStage + dh * kHalf64, dh * 64, t * 64, bg);
-                tma_store_3d(&tmdK, sb + kOffStage + kTile128 + dh * kHalf64, dh * 64, t * 64, bg);
-            }
-            tma_store_commit();
-            tma_store_wait_read();
         }
     }
     tc_fence_before();
@@ -944,25 +1111,30 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
 
 cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
-                           const int32_t* qlist, const int2* work, const int32_t* nwork,
+                           const int32_t* qlist, const int2* queue, int* qctl,
                            const phsa_shape& s, int topk, int work_max, int slot_max,
                            float sm_scale, void* dK, void* dV, float* partial, int* arrive,
                            int* status, cudaStream_t st) {
     const int NQB = (s.L + 63) / 64;
-    CUtensorMap tq, tk, tv, tdo, tdk, tdv;
+    CUtensorMap tq, tk, tv, tdo;
     const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
     if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) || !make_tmap_bf16_rows128(&tk, K, s.L, pk, 64) ||
-        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64) ||
-        !make_tmap_bf16_rows128(&tdk, dK, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdv, dV, s.L, pk, 64))
+        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64))
         return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(dkdv_tc_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kv::kSmem);
     if (e != cudaSuccess) return e;
-    KvArgs args{lse, delta, tinfo, qlist, work, nwork, partial, arrive, status, s.Hq, s.Hkv, s.L, NQB,
-                topk, work_max, slot_max, sm_scale * kLog2e, sm_scale};
+    int dev = 0, nsm = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    const long long qcap = (long long)s.B * s.Hkv * work_max;  // entries per queue class
+    KvArgs args{lse, delta, tinfo, qlist, queue, qctl, qctl + kQueueClasses, partial, arrive,
+                static_cast<__nv_bfloat16*>(dK), static_cast<__nv_bfloat16*>(dV), status, qcap,
+                s.Hq, s.Hkv, s.L, NQB, topk, slot_max, sm_scale * kLog2e, sm_scale};
     ProfScope prof(K_BWD_DKDV, st);
-    dkdv_tc_kernel<<<dim3(work_max, s.B * s.Hkv), kv::kThreads, kv::kSmem, st>>>(tq, tk, tv, tdo,
-                                                                                 tdk, tdv, args);
+    dkdv_tc_kernel<<<(unsigned)(qcap < nsm ? qcap : nsm), kv::kThreads, kv::kSmem, st>>>(
+        tq, tk, tv, tdo, args);
     return cudaGetLastError();
 }
 

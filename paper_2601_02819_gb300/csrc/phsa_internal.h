@@ -73,11 +73,18 @@ struct BwdTInfo {
     int off, n, nch, slot;
 };
 constexpr int kBwdChunk = 32;  // query blocks per dK/dV work item
+// dK/dV work items are queued by size class (iterations 32 | 16-31 | 8-15 |
+// 0-7), so a persistent kernel that takes them in queue order starts the long
+// ones first and ends on short ones.
+constexpr int kQueueClasses = 4;
+__host__ __device__ __forceinline__ int queue_class(int n_it) {
+    return n_it >= kBwdChunk ? 0 : n_it >= 16 ? 1 : n_it >= 8 ? 2 : 3;
+}
 
 // tcgen05 backward kernels for G = 2 (attn_bwd_tc.cu).
 cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
-                           const int32_t* qlist, const int2* work, const int32_t* nwork,
+                           const int32_t* qlist, const int2* queue, int* qctl,
                            const phsa_shape& s, int topk, int work_max, int slot_max,
                            float sm_scale, void* dK, void* dV, float* partial, int* arrive,
                            int* status, cudaStream_t st);
@@ -90,7 +97,9 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
 
 // Backward workspace layout (all offsets 256-byte aligned).
 struct BwdLayout {
-    size_t bits, tinfo, qlist, work, nwork, delta, partial, arrive, total;
+    // qctl: item counts of the kQueueClasses queue classes, then the ticket
+    // counter of the persistent dK/dV kernel (zeroed with bits by one memset)
+    size_t qctl, bits, tinfo, qlist, work, nwork, queue, delta, partial, arrive, total;
     int nqb, words, chunk, work_max, slot_max;
 };
 BwdLayout bwd_layout(const phsa_shape& s, int topk);
