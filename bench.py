@@ -180,31 +180,41 @@ class ClockSampler:
 # ---------------------------------------------------------------- oracle sample
 def oracle_sample_step(w, x, n_units: int, seed: int):
     """Times the CPU oracle on a bounded sample of one step; returns estimated seconds
-    for the whole step, the parts and a description. Sample: stage (a) in full;
-    stages (b), (c) forward and dQ for `n_units` random (b, g, qb) units; dK/dV
-    for `n_units` random KV blocks. Each part is scaled by (total units / sampled)."""
+    for the whole step, the parts and a description.
+
+    Sample: stage (a) in full; stages (b), (c) forward and dQ for `n_units` random
+    (b, g, qb) units; dK/dV for `n_units` random KV blocks other than block 0. The
+    attention parts use a fixed selection table (the forced blocks plus the most
+    recent candidates). The oracle's cost per unit is linear in its work (scored
+    candidates for (b), selected blocks for (c) and dQ, listed (query block,
+    selected block) pairs for dK/dV), so each part is scaled by total work /
+    sampled work. Block 0, listed by every query block, carries ~40 typical
+    blocks' work; it is left out of the timed sample (one such unit would dominate
+    a parallel sample's elapsed time) and counted in the total work."""
     import oracle
     rng = np.random.default_rng(seed)
     U = w.B * w.Hkv * w.NQB
     units = rng.choice(U, size=min(n_units, U), replace=False)
     scale = w.sm_scale
-    t = {}
-    t0 = time.perf_counter()
-    Kr = oracle.block_repr(x["K"], x["mask"], w.block_size, w.lam)
-    t["repr"] = time.perf_counter() - t0
-    t0 = time.perf_counter()
-    si, sc, _ = oracle.select_units(x["Q"], Kr, w.L, w.block_size, w.topk, w.n_init, w.n_local,
-                                    scale, units)
-    t["select"] = (time.perf_counter() - t0) * U / len(units)
-    # full index table for the attention parts: forced + the first candidates
     idx = np.full((w.B, w.Hkv, w.NQB, w.topk), -1, np.int32)
     cnt = np.zeros((w.B, w.Hkv, w.NQB), np.int32)
+    lists = np.zeros(w.NQB, np.int64)  # per KV block t: sum of cnt over the query blocks listing t
     for qb in range(w.NQB):
         s = sorted(set(range(min(w.n_init, qb + 1))) | set(range(max(0, qb - w.n_local + 1), qb + 1)))
         extra = [c for c in range(qb) if c not in s][::-1][: max(0, w.topk - len(s))]
         s = sorted(set(s) | set(extra))
         idx[:, :, qb, :len(s)] = s
         cnt[:, :, qb] = len(s)
+        lists[s] += len(s)
+    qbs = units % w.NQB
+    t = {}
+    t0 = time.perf_counter()
+    Kr = oracle.block_repr(x["K"], x["mask"], w.block_size, w.lam)
+    t["repr"] = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    oracle.select_units(x["Q"], Kr, w.L, w.block_size, w.topk, w.n_init, w.n_local, scale, units)
+    cand_all = w.B * w.Hkv * float(np.sum(np.arange(1, w.NQB + 1)))
+    t["select"] = (time.perf_counter() - t0) * cand_all / float(np.sum(qbs + 1))
     rows = []
     for u in units:
         qb = u % w.NQB
@@ -214,7 +224,7 @@ def oracle_sample_step(w, x, n_units: int, seed: int):
             for i in range(qb * w.block_size, min((qb + 1) * w.block_size, w.L)):
                 rows.append((b, g * w.G + hh, i))
     rows = np.array(rows, np.int32)
-    frac = U / len(units)
+    frac = float(cnt.sum()) / float(cnt.reshape(-1)[units].sum())
     t0 = time.perf_counter()
     oracle.sparse_attn_rows(x["Q"], x["K"], x["V"], idx, cnt, w.block_size, scale, rows)
     t["fwd"] = (time.perf_counter() - t0) * frac
@@ -222,15 +232,17 @@ def oracle_sample_step(w, x, n_units: int, seed: int):
     oracle.sparse_attn_bwd_dq_rows(x["Q"], x["K"], x["V"], x["dO"], idx, cnt, w.block_size, scale,
                                    rows)
     t["bwd_dq"] = (time.perf_counter() - t0) * frac
-    kvb = np.stack([units // w.NQB // w.Hkv, (units // w.NQB) % w.Hkv,
-                    rng.integers(0, w.NQB, len(units))], axis=1).astype(np.int32)
+    kt = rng.integers(1, w.NQB, len(units)) if w.NQB > 1 else np.zeros(len(units), np.int64)
+    kvb = np.stack([units // w.NQB // w.Hkv, (units // w.NQB) % w.Hkv, kt],
+                   axis=1).astype(np.int32)
     t0 = time.perf_counter()
     oracle.sparse_attn_bwd_kv_blocks(x["Q"], x["K"], x["V"], x["dO"], idx, cnt, w.block_size,
                                      scale, kvb)
-    t["bwd_dkdv"] = (time.perf_counter() - t0) * frac
+    t["bwd_dkdv"] = ((time.perf_counter() - t0) * w.B * w.Hkv * float(lists.sum())
+                     / float(lists[kt].sum()))
     desc = (f"stage (a) in full; stages (b), (c) fwd and dQ on {len(units)}"
-            f" of {U} (query block, KV head) units; dK/dV on {len(units)} of {U} KV blocks;"
-            f" each part scaled to the full step")
+            f" of {U} (query block, KV head) units; dK/dV on {len(units)} of {U} KV blocks"
+            f" (block 0 excluded); each part scaled by total / sampled work")
     return sum(t.values()), t, desc
 
 
@@ -680,12 +692,13 @@ def run_reference(args):
     w = inputs.WORKLOADS[args.workload]
     x = inputs.make_inputs(w, with_grad=True)
     cores = oracle_threads()
+    n_units = max(args.ref_units, cores)  # at least one unit per thread
     for s in range(args.warmup):
-        oracle_sample_step(w, x, args.ref_units, seed=100 + s)
+        oracle_sample_step(w, x, n_units, seed=100 + s)
     ests, descs = [], None
     t0 = time.perf_counter()
     for s in range(args.steps):
-        est, _, descs = oracle_sample_step(w, x, args.ref_units, seed=1000 + s)
+        est, _, descs = oracle_sample_step(w, x, n_units, seed=1000 + s)
         ests.append(est)
     wall = time.perf_counter() - t0
     est = statistics.mean(ests)
@@ -718,7 +731,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-units", type=int, default=48,
                     help="units in the oracle sample of the cpu_baseline")
-    ap.add_argument("--ref-units", type=int, default=8,
+    ap.add_argument("--ref-units", type=int, default=16,
                     help="units in each oracle sample step of --impl reference")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
