@@ -328,45 +328,53 @@ def run_ours(args):
     ms_step = ms_total / args.steps
     status = phsa.phsa_get_device_status()
 
-    # ---- end to end through the public API with host buffers
+    # ---- end to end through the C ABI's host-buffer call: every step copies its
+    # inputs from pinned host memory and its results back, inside the timed region
     e2e = None
     if not args.no_e2e:
         pin = lambda a: torch.from_numpy(a).pin_memory()
         hQ, hK, hV, hdO = (pin(x[k].view(np.int16)) for k in ("Q", "K", "V", "dO"))
         hmask = pin(x["mask"])
-        hO, hdQ = (torch.empty(Q.shape, dtype=torch.int16).pin_memory() for _ in range(2))
-        hdK, hdV = (torch.empty(K.shape, dtype=torch.int16).pin_memory() for _ in range(2))
+        pinned = lambda shape, dt: torch.empty(shape, dtype=dt).pin_memory()
+        outs = [{"O": pinned(Q.shape, torch.int16), "lse": pinned(lse.shape, torch.float32),
+                 "dQ": pinned(Q.shape, torch.int16), "dK": pinned(K.shape, torch.int16),
+                 "dV": pinned(K.shape, torch.int16)} for _ in range(2)]
         h2d = sum(t.numel() * t.element_size() for t in (hQ, hK, hV, hdO, hmask))
-        d2h = sum(t.numel() * t.element_size() for t in (hO, hdQ, hdK, hdV))
+        d2h = sum(t.numel() * t.element_size() for t in outs[0].values())
+        nbytes = phsa.phsa_step_host_workspace(w.B, w.L, w.Hq, w.Hkv, w.topk)
+        wss = [torch.empty(nbytes, dtype=torch.uint8, device=dev) for _ in range(2)]
+        evs = [torch.cuda.Event() for _ in range(2)]
 
-        def e2e_step():
-            Q.view(torch.int16).copy_(hQ, non_blocking=True)
-            K.view(torch.int16).copy_(hK, non_blocking=True)
-            V.view(torch.int16).copy_(hV, non_blocking=True)
-            dO.view(torch.int16).copy_(hdO, non_blocking=True)
-            mask.copy_(hmask, non_blocking=True)
-            step()
-            hO.copy_(O.view(torch.int16), non_blocking=True)
-            hdQ.copy_(dQ.view(torch.int16), non_blocking=True)
-            hdK.copy_(dK.view(torch.int16), non_blocking=True)
-            hdV.copy_(dV.view(torch.int16), non_blocking=True)
+        def e2e_step(i):
+            # two workspaces alternate, so one step's copies overlap the other's kernels
+            phsa.phsa_step_host(hQ, hK, hV, hdO, hmask, w.lam, w.topk, w.n_init, w.n_local,
+                                w.sm_scale, workspace=wss[i % 2], done_event=evs[i % 2],
+                                stream=stream, **outs[i % 2])
 
-        for _ in range(2):
-            e2e_step()
+        for i in range(2):
+            e2e_step(i)
+        torch.cuda.synchronize()
         n_e2e = max(3, min(args.steps, 20))
         barrier()
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for _ in range(n_e2e):
-            e2e_step()
+        for i in range(n_e2e):
+            e2e_step(i)
+        for ev in evs:
+            stream.wait_event(ev)
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
         ms_e2e = max_over_ranks(e0.elapsed_time(e1) / n_e2e, device=dev)
+        for ws in wss:
+            phsa.phsa_step_host_release(ws)
         e2e = {"value": world * w.B * w.L / (ms_e2e / 1e3), "unit": "tokens/s",
                "ms_per_step": ms_e2e, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-               "steps": n_e2e}
+               "steps": n_e2e,
+               "note": "phsa_step_host (C ABI) on pinned host buffers: Q, K, V, dO and the mask "
+                       "copied in, O, lse, dQ, dK, dV copied back every step; the library "
+                       "overlaps the copies with the kernels, two workspaces alternate"}
 
     if rank != 0:
         return None

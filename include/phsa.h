@@ -173,6 +173,51 @@ int phsa_sparse_attn_bwd_noalloc(const void* Q, const void* K, const void* V, co
                                  void* dQ, void* dK, void* dV, void* stream);
 
 /*
+ * The whole path for tensors in HOST memory (no counterpart in the paper): one
+ * training step of the attention -- stage (a), (b), the forward of (c) and its
+ * backward pass for a given dO -- with the host<->device copies overlapped
+ * with the kernels. Inputs Q, K, V, dO, punct_mask and outputs O, lse, dQ, dK,
+ * dV, block_idx, block_cnt have the layouts of the calls above but are HOST
+ * pointers; they should be page-locked (cudaHostAlloc / cudaHostRegister),
+ * else the CUDA runtime stages the copies and they do not overlap. Any output
+ * pointer may be NULL: that result is not copied back.
+ *
+ * Copies run on two streams the library owns (one per direction per device):
+ * K and the mask are copied first, then Q, V and dO; stage (a) starts when K
+ * has arrived, (b) when Q has, the forward when V has and the backward when
+ * dO has. O, lse and the selection are copied back while the backward runs, dQ
+ * while dK/dV are computed, dK and dV at the end. The kernels run on `stream`.
+ *
+ *   workspace   device buffer of at least phsa_step_host_workspace() bytes,
+ *               256-byte aligned, owned by the caller: it holds the device
+ *               copies of every input and output, the representative keys,
+ *               the selection and the backward pass's scratch.
+ *   done_event  NULL: `stream` is made to wait for the copies back, so that
+ *               synchronising `stream` means the outputs are in host memory.
+ *               Otherwise a cudaEvent_t (as void*) that the call records when
+ *               the outputs are in host memory; `stream` then waits only for
+ *               the kernels, and the next call's kernels can overlap this
+ *               call's copies back.
+ *
+ * The copies in do not wait for earlier work on `stream`; they wait for the
+ * previous call that used the same workspace to be done with it (copies back
+ * included). A caller that alternates two workspaces therefore overlaps one
+ * step's copies in with the previous step's kernels. The host buffers must
+ * not be written (inputs) or read (outputs) until the call's work is done.
+ * Validation as for the calls above; PHSA_ERR_WORKSPACE if the workspace is
+ * NULL, misaligned or too small. Returns after enqueueing.
+ */
+size_t phsa_step_host_workspace(phsa_shape s, int topk);
+int phsa_step_host(const void* Q, const void* K, const void* V, const void* dO,
+                   const uint8_t* punct_mask, phsa_shape s, float lambda, phsa_select_params p,
+                   void* O, float* lse, void* dQ, void* dK, void* dV, int32_t* block_idx,
+                   int32_t* block_cnt, void* workspace, size_t workspace_bytes, void* done_event,
+                   void* stream);
+/* Waits for the last call on `workspace` and frees the library's events for
+ * it; call before freeing a workspace that phsa_step_host used. */
+int phsa_step_host_release(void* workspace);
+
+/*
  * Decode: one new token per sequence, against per-sequence caches.
  * Layout: s.L is the cache capacity; K, V bf16 [B, Hkv, L, D]; punct_mask
  * uint8 [B, L]; Krepr bf16 [B, Hkv, floor(L/m), D]; seq_lens int32 [B] (device)

@@ -656,8 +656,9 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
                             const void* dO, const float* lse, const int32_t* idx,
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                             void* ws, void* dQ, void* dK, void* dV, int* status,
-                            cudaStream_t st) {
-    if ((long long)s.B * s.Hkv * s.L == 0) return cudaSuccess;
+                            cudaStream_t st, cudaEvent_t after_dq) {
+    if ((long long)s.B * s.Hkv * s.L == 0)
+        return after_dq ? cudaEventRecord(after_dq, st) : cudaSuccess;
     const BwdLayout l = bwd_layout(s, topk);
     uint8_t* w = static_cast<uint8_t*>(ws);
     uint32_t* bits = reinterpret_cast<uint32_t*>(w + l.bits);
@@ -681,6 +682,7 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
         // dQ first: it also computes Delta from O and dO, which dK/dV then read.
         e = launch_dq_tc(Q, K, V, O, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
         if (e != cudaSuccess) return e;
+        if (after_dq && (e = cudaEventRecord(after_dq, st)) != cudaSuccess) return e;
     } else {
         ProfScope prof(K_BWD_DELTA, st);
         delta_kernel<<<(unsigned)((rows * 16 + 255) / 256), 256, 0, st>>>(
@@ -732,9 +734,11 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
             static_cast<__nv_bfloat16*>(dV));
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    return s.Hq == s.Hkv
-               ? launch_dq_g<1>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st)
-               : launch_dq_g<2>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
+    e = s.Hq == s.Hkv
+            ? launch_dq_g<1>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st)
+            : launch_dq_g<2>(Q, K, V, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
+    if (e != cudaSuccess) return e;
+    return after_dq ? cudaEventRecord(after_dq, st) : cudaSuccess;
 }
 
 }  // namespace phsa

@@ -22,10 +22,6 @@
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 
-namespace phsa {
-int* device_status_word();
-}
-
 namespace {
 
 constexpr size_t kScratchBytes = size_t(64) << 20;

@@ -5,10 +5,6 @@
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 
-namespace phsa {
-size_t select_smem_bytes(const phsa_shape& s, int topk);
-}
-
 namespace {
 
 // One status word per device, in a file-scope device variable (no allocation).
@@ -64,6 +60,8 @@ int check_topk(const phsa_shape& s, int topk) {
 namespace phsa {
 // The status word of the current device, for entry points in other files.
 int* device_status_word() { return status_ptr(); }
+int validate_shape(const phsa_shape& s) { return check_shape(s); }
+int validate_topk(const phsa_shape& s, int topk) { return check_topk(s, topk); }
 }  // namespace phsa
 
 extern "C" {

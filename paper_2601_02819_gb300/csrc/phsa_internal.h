@@ -104,10 +104,20 @@ struct BwdLayout {
 };
 BwdLayout bwd_layout(const phsa_shape& s, int topk);
 
+// after_dq (optional) is recorded on st once dQ is complete, before dK/dV
+// finish, so that a caller can start copying dQ out early.
 cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const void* O,
                             const void* dO, const float* lse, const int32_t* idx,
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                             void* ws, void* dQ, void* dK, void* dV, int* status,
-                            cudaStream_t st);
+                            cudaStream_t st, cudaEvent_t after_dq = nullptr);
+
+// The status word of the current device (phsa_api.cu); null if it cannot be found.
+int* device_status_word();
+// Shape and budget checks of the C ABI (phsa_api.cu): PHSA_OK or an error code.
+int validate_shape(const phsa_shape& s);
+int validate_topk(const phsa_shape& s, int topk);
+// Shared-memory bytes of the selection kernel for this shape and budget.
+size_t select_smem_bytes(const phsa_shape& s, int topk);
 
 }  // namespace phsa

@@ -78,6 +78,13 @@ def _declare(L):
     L.phsa_sparse_attn_bwd_noalloc.argtypes = [P, P, P, P, P, P, P, P, phsa_shape, I, F, P, P, P,
                                                P]
     L.phsa_sparse_attn_bwd_noalloc.restype = I
+    L.phsa_step_host_workspace.argtypes = [phsa_shape, I]
+    L.phsa_step_host_workspace.restype = SZ
+    L.phsa_step_host.argtypes = [P, P, P, P, P, phsa_shape, F, phsa_select_params, P, P, P, P, P,
+                                 P, P, P, SZ, P, P]
+    L.phsa_step_host.restype = I
+    L.phsa_step_host_release.argtypes = [P]
+    L.phsa_step_host_release.restype = I
     L.phsa_decode_update_repr.argtypes = [P, P, P, phsa_shape, F, P, P]
     L.phsa_decode_select.argtypes = [P, P, P, phsa_shape, phsa_select_params, P, P, P]
     L.phsa_decode_attn.argtypes = [P, P, P, P, P, P, phsa_shape, I, F, P, P, P]
@@ -103,6 +110,19 @@ def _check(t, name, dtype, ndim=None):
         raise ValueError(f"{name} must be a CUDA tensor")
     if t.dtype != dtype:
         raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got {tuple(t.shape)}")
+
+
+def _check_host(t, name, dtypes, ndim=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.is_cuda:
+        raise ValueError(f"{name} must be a host (CPU) tensor")
+    if t.dtype not in dtypes:
+        raise TypeError(f"{name} must be one of {dtypes}, got {t.dtype}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     if ndim is not None and t.dim() != ndim:
@@ -247,6 +267,67 @@ def phsa_sparse_attn_bwd_noalloc(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_s
         _ptr(dK), _ptr(dV), _stream(stream))
     _raise("phsa_sparse_attn_bwd_noalloc", rc)
     return dQ, dK, dV
+
+
+def phsa_step_host_workspace(B, L, Hq, Hkv, topk, D=HEAD_DIM) -> int:
+    return int(load().phsa_step_host_workspace(make_shape(B, L, Hq, Hkv, D), int(topk)))
+
+
+def phsa_step_host(Q, K, V, dO, punct_mask, lam: float, topk: int, n_init: int = 1,
+                   n_local: int = 1, sm_scale: float | None = None, O=None, lse=None, dQ=None,
+                   dK=None, dV=None, block_idx=None, block_cnt=None, workspace=None,
+                   done_event=None, stream=None):
+    """One step of the whole path for HOST tensors (preferably pinned): stage (a),
+    (b), the forward and the backward for dO, with the copies overlapped with the
+    kernels inside the library. Q, K, V, dO: bf16 (or int16 holding bf16 bits) CPU
+    tensors [B, H, L, D]; punct_mask uint8 [B, L]. Outputs O, lse, dQ, dK, dV are
+    allocated pinned when not passed; block_idx / block_cnt are copied back only
+    when passed. workspace: CUDA uint8 tensor of phsa_step_host_workspace() bytes.
+    done_event: a torch.cuda.Event the library records when the outputs are in
+    host memory (the stream then waits only for the kernels); None makes the
+    stream wait for the copies back. Returns (O, lse, dQ, dK, dV)."""
+    bf = (torch.bfloat16, torch.int16)
+    for name, t in (("Q", Q), ("K", K), ("V", V), ("dO", dO)):
+        _check_host(t, name, bf, 4)
+    _check_host(punct_mask, "punct_mask", (torch.uint8,), 2)
+    B, Hq, L, D = Q.shape
+    Hkv = K.shape[1]
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    pinned = lambda shape, dt: torch.empty(shape, dtype=dt).pin_memory()
+    O = pinned(Q.shape, Q.dtype) if O is None else O
+    dQ = pinned(Q.shape, Q.dtype) if dQ is None else dQ
+    dK = pinned(K.shape, K.dtype) if dK is None else dK
+    dV = pinned(K.shape, K.dtype) if dV is None else dV
+    lse = pinned((B, Hq, L), torch.float32) if lse is None else lse
+    for name, t in (("O", O), ("dQ", dQ), ("dK", dK), ("dV", dV)):
+        _check_host(t, name, bf, 4)
+    _check_host(lse, "lse", (torch.float32,), 3)
+    if block_idx is not None:
+        _check_host(block_idx, "block_idx", (torch.int32,), 4)
+    if block_cnt is not None:
+        _check_host(block_cnt, "block_cnt", (torch.int32,), 3)
+    ws_bytes = phsa_step_host_workspace(B, L, Hq, Hkv, topk, D)
+    if workspace is None:
+        workspace = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device="cuda")
+    _check(workspace, "workspace", torch.uint8, 1)
+    ev = None
+    if done_event is not None:
+        done_event.record(stream)  # creates the CUDA event; the library records it again
+        ev = ctypes.c_void_p(done_event.cuda_event)
+    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    rc = load().phsa_step_host(_ptr(Q), _ptr(K), _ptr(V), _ptr(dO), _ptr(punct_mask),
+                               make_shape(B, L, Hq, Hkv, D), float(lam), p, _ptr(O), _ptr(lse),
+                               _ptr(dQ), _ptr(dK), _ptr(dV), _ptr(block_idx), _ptr(block_cnt),
+                               _ptr(workspace), ctypes.c_size_t(workspace.numel()), ev,
+                               _stream(stream))
+    _raise("phsa_step_host", rc)
+    return O, lse, dQ, dK, dV
+
+
+def phsa_step_host_release(workspace):
+    """Waits for the last phsa_step_host call on `workspace` and drops its events."""
+    _raise("phsa_step_host_release", load().phsa_step_host_release(_ptr(workspace)))
 
 
 def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=None):

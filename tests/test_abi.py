@@ -74,3 +74,29 @@ def test_host_validation_needs_no_gpu(lib):
     assert lib.phsa_select_blocks(None, None, ok, p, None, None, None) == -1
     assert lib.phsa_sparse_attn_bwd_workspace(ok, 14) > 0
     assert lib.phsa_sparse_attn_bwd_workspace(phsa_shape(1, 4096, 16, 8, 96, 64), 14) == 0
+
+
+def test_host_step_validation_needs_no_gpu(lib):
+    # The host-buffer step checks its arguments and workspace before any CUDA call.
+    from paper_2601_02819_gb300.phsa import phsa_shape, phsa_select_params
+    P = ctypes.c_void_p
+    lib.phsa_step_host_workspace.argtypes = [phsa_shape, ctypes.c_int]
+    lib.phsa_step_host_workspace.restype = ctypes.c_size_t
+    lib.phsa_step_host.argtypes = [P, P, P, P, P, phsa_shape, ctypes.c_float, phsa_select_params,
+                                   P, P, P, P, P, P, P, P, ctypes.c_size_t, P, P]
+    ok = phsa_shape(1, 4096, 16, 8, 128, 64)
+    ws = lib.phsa_step_host_workspace(ok, 14)
+    # device copies of Q, dO, O, dQ (16 MB each) and K, V, dK, dV (8 MB each) alone
+    assert ws > 4 * 16 * 2**20 + 4 * 8 * 2**20
+    assert ws >= lib.phsa_sparse_attn_bwd_workspace(ok, 14)
+    assert lib.phsa_step_host_workspace(phsa_shape(1, 4096, 16, 8, 96, 64), 14) == 0
+    p = phsa_select_params(14, 1, 1, 0.088)
+    dummy = ctypes.c_void_p(256)  # never dereferenced: every case fails validation first
+    args = [dummy] * 5
+    assert lib.phsa_step_host(*args, ok, 1.5, p, *([None] * 7), dummy, ws, None, None) == -1
+    assert lib.phsa_step_host(*args, ok, 0.5, phsa_select_params(2, 1, 2, 0.088),
+                              *([None] * 7), dummy, ws, None, None) == -1
+    assert lib.phsa_step_host(*args, ok, 0.5, p, *([None] * 7), None, ws, None, None) == -6
+    assert lib.phsa_step_host(*args, ok, 0.5, p, *([None] * 7), dummy, ws - 1, None, None) == -6
+    assert lib.phsa_step_host(*args, phsa_shape(1, 4096, 16, 8, 64, 64), 0.5, p, *([None] * 7),
+                              dummy, ws, None, None) == -2
