@@ -115,7 +115,7 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
                  int2* __restrict__ work, int32_t* __restrict__ nwork, int* __restrict__ arrive,
                  int2* __restrict__ queue, int* __restrict__ qcount, int* status) {
     __shared__ int tmp[32];
-    __shared__ int cls_n[kQueueClasses];
+    __shared__ int bin[kChunk + 1];  // items per iteration count, then queue cursors
     const int bg = blockIdx.x;
     const int per = (NQB + 1023) / 1024;  // KV blocks counted by each thread
     const int t0 = threadIdx.x * per;
@@ -138,11 +138,11 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     if (threadIdx.x == 0) {
         nwork[bg] = min(tch, work_max);
         if (tch > work_max || tsl > slot_max || tn > NQB * topk) set_status(status, PHSA_ERR_DEVICE_INDEX);
-        for (int c = 0; c < kQueueClasses; ++c) cls_n[c] = 0;
     }
+    for (int n = threadIdx.x; n <= kChunk; n += blockDim.x) bin[n] = 0;
     __syncthreads();
-    // Items per size class (those that fit work_max), then one range of each
-    // class's queue for this (b, g)
+    // Items per iteration count (those that fit work_max), then one range of
+    // each class's queue for this (b, g), sorted by iteration count, descending
     for (int k = 0, ch = och; k < per; ++k) {
         const int t = t0 + k;
         if (t >= NQB) break;
@@ -150,12 +150,21 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
         for (int w = 0; w < words; ++w) n += __popc(bb[(size_t)t * words + w]);
         const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
         for (int c = 0; c < nch && ch + c < work_max; ++c)
-            atomicAdd(&cls_n[queue_class(min(n, kChunk * c + kChunk) - kChunk * c)], 1);
+            atomicAdd(&bin[min(n, kChunk * c + kChunk) - kChunk * c], 1);
         ch += nch;
     }
     __syncthreads();
-    if (threadIdx.x < kQueueClasses)
-        cls_n[threadIdx.x] = atomicAdd(qcount + threadIdx.x, cls_n[threadIdx.x]);
+    if (threadIdx.x == 0) {
+        int nc[kQueueClasses] = {};
+        for (int n = 0; n <= kChunk; ++n) nc[queue_class(n)] += bin[n];
+        int pos[kQueueClasses];
+        for (int c = 0; c < kQueueClasses; ++c) pos[c] = atomicAdd(qcount + c, nc[c]);
+        for (int n = kChunk; n >= 0; --n) {  // bin[n] becomes the cursor of its items
+            const int c = queue_class(n), cnt_n = bin[n];
+            bin[n] = pos[c];
+            pos[c] += cnt_n;
+        }
+    }
     __syncthreads();
     const size_t qcap = (size_t)gridDim.x * work_max;
     TInfo* ti = tinfo + (size_t)bg * NQB;
@@ -175,8 +184,8 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
         arrive[(size_t)bg * NQB + t] = 0;
         for (int c = 0; c < nch && och + c < work_max; ++c) {
             wk[och + c] = make_int2(t, c);
-            const int cls = queue_class(min(n, kChunk * c + kChunk) - kChunk * c);
-            queue[cls * qcap + atomicAdd(&cls_n[cls], 1)] = make_int2(bg * NQB + t, c);
+            const int n_it = min(n, kChunk * c + kChunk) - kChunk * c;
+            queue[queue_class(n_it) * qcap + atomicAdd(&bin[n_it], 1)] = make_int2(bg * NQB + t, c);
         }
         on += n;
         och += nch;

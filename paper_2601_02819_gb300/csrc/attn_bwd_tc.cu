@@ -565,8 +565,11 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
 
 // ============================================================== dK / dV
 // Persistent: one CTA per SM takes work items (KV block t of one (b, g), chunk
-// of <= 32 query blocks that selected t) from a global queue ordered by size
-// class, longest first, by tickets from one counter, so the SMs end together.
+// of <= 32 query blocks that selected t) from a global queue by tickets from
+// one counter. The queue (built by idx_build) holds the items of >= 4
+// iterations, (b, g) after (b, g) and longest first within each, then the
+// short ones: the Q/dO tiles of the (b, g) in progress stay in L2 and the SMs
+// end together on short items.
 // The producer thread takes the tickets and hands each item to the MMA and
 // elementwise roles through a ring in shared memory. K_t/V_t are reloaded as
 // soon as the previous item's last S/dP MMAs are done, the Q/dO ring, the S/dP

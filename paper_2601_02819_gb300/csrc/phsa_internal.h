@@ -73,12 +73,15 @@ struct BwdTInfo {
     int off, n, nch, slot;
 };
 constexpr int kBwdChunk = 32;  // query blocks per dK/dV work item
-// dK/dV work items are queued by size class (iterations 32 | 16-31 | 8-15 |
-// 0-7), so a persistent kernel that takes them in queue order starts the long
-// ones first and ends on short ones.
-constexpr int kQueueClasses = 4;
+// dK/dV work items are queued in two classes, items of at least 4 iterations
+// first, then the shorter ones; inside a class each (b, g) holds one contiguous
+// range, longest items first. A persistent kernel that takes the items in
+// queue order keeps the Q/dO tiles of one or two (b, g) in L2 at a time and
+// ends on short items, so the SMs finish together.
+constexpr int kQueueClasses = 2;
+constexpr int kShortItem = 4;
 __host__ __device__ __forceinline__ int queue_class(int n_it) {
-    return n_it >= kBwdChunk ? 0 : n_it >= 16 ? 1 : n_it >= 8 ? 2 : 3;
+    return n_it >= kShortItem ? 0 : 1;
 }
 
 // tcgen05 backward kernels for G = 2 (attn_bwd_tc.cu).
