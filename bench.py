@@ -18,6 +18,7 @@ workload on this host's cores.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -246,6 +247,29 @@ def oracle_sample_step(w, x, n_units: int, seed: int):
     return sum(t.values()), t, desc
 
 
+def profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu summary
+    profiles/dram_<kernel>_<workload>.txt, or None when there is none or the kernel's
+    sources (listed in it) no longer hash to the value it records."""
+    path = os.path.join(ROOT, "profiles", f"dram_{kernel}_{workload}.txt")
+    if not os.path.exists(path):
+        return None
+    fields = {}
+    for line in open(path):
+        key, sep, val = line.partition(":")
+        if sep and key.strip() in ("dram_bytes_per_launch", "sources", "source_sha256"):
+            fields[key.strip()] = val.strip()
+    if len(fields) != 3:
+        return None
+    h = hashlib.sha256()
+    for rel in fields["sources"].split():
+        try:
+            h.update(open(os.path.join(ROOT, rel), "rb").read())
+        except OSError:
+            return None
+    return int(fields["dram_bytes_per_launch"]) if h.hexdigest() == fields["source_sha256"] else None
+
+
 def oracle_threads():
     import oracle
     n = len(os.sched_getaffinity(0))
@@ -416,6 +440,7 @@ def run_ours(args):
                 "peak": BW, "unit": "GB/s", "frac": round(a["bytes"] / avg_s / 1e9 / BW, 4),
                 "peak_source": f"{peak_src} HBM copy", "traffic": None,
                 "algorithmic_per_launch": a["bytes"]}
+    roof["traffic"] = profiled_traffic(dom, w.name)
     fwd_ms = sum(kernels[k]["ms_total"] for k in ("block_repr", "select_blocks", "attn_fwd")
                  if k in kernels) / args.steps
     bwd_ms = sum(v["ms_total"] for k, v in kernels.items() if k.startswith("bwd")) / args.steps
