@@ -266,6 +266,21 @@ int phsa_decode_attn(const void* q, const void* K, const void* V, const int32_t*
                      float sm_scale, void* O, float* lse, void* stream);
 
 /*
+ * One whole decode step in two launches: the selection of phsa_decode_select,
+ * then the attention of phsa_decode_attn fused with phsa_decode_update_repr.
+ * The block a sequence's new token has just filled is the query's own (local)
+ * block: the attention reads it anyway and refreshes its representative key
+ * from the copy in shared memory, and it is never a candidate of the same step,
+ * so the selection does not depend on the refresh. Results are bit-identical
+ * to the three calls update_repr, select, attn. Arguments as for those calls;
+ * Krepr is read (candidates) and written (the filled blocks).
+ */
+int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t* punct_mask,
+                     const int32_t* seq_lens, phsa_shape s, float lambda, phsa_select_params p,
+                     void* Krepr, int32_t* block_idx, int32_t* block_cnt, void* O, float* lse,
+                     void* stream);
+
+/*
  * Synchronises `stream`, returns the device status word of the current
  * device (PHSA_OK or the first device-side error code recorded since the
  * last call) and clears it. Returns PHSA_ERR_CUDA if the synchronisation

@@ -2,29 +2,50 @@
 // p = len_b - 1) is the query; the selection rule of Section 3.3 (Algorithm 1
 // step 3) is applied to the unit whose rows are that token in each of the
 // GQA group's G query heads, and Eq. 10-11 to the token's row. The block
-// representations are cached and updated as blocks fill (block_repr.cu).
+// representations are cached and updated as blocks fill (Section 3.2).
 //
 // Both kernels read little per unit and are bound by HBM bandwidth, so they
-// run on the CUDA cores: one CTA (8 warps) per (sequence, KV head), with a
-// half-warp per 256-byte key row (lane c holds columns 8c..8c+7, 16-byte
-// read-only loads, four rows in flight per half-warp).
+// run on the CUDA cores. What a unit (sequence, KV head) reads is contiguous
+// in memory -- its candidates' representative keys are consecutive rows of
+// Krepr, every selected K or V block is 64 consecutive rows -- so one thread
+// streams it into a shared-memory ring with 1-D bulk copies (cp.async.bulk,
+// completion counted on an mbarrier per slot) and the warps compute from
+// shared memory: a half-warp per 256-byte key row (lane c holds columns
+// 8c..8c+7). Both kernels are persistent: a CTA walks the units u =
+// blockIdx.x, blockIdx.x + gridDim.x, ..., and its ring runs across unit
+// boundaries, so the next unit's rows are in flight while a unit finishes.
+// After each slot is consumed the CTA synchronises (agreeing on any abort)
+// and the slot is refilled.
 //
 // decode_select_kernel  S[h][t] = q_h . Krepr_t for the candidates, per head
 //   the softmax over candidates (max, sum), A_t = sum over heads of the
 //   probabilities (head order), then the top-k of topk.cuh.
-// decode_attn_kernel  each half-warp runs an online softmax over a share of
-//   the selected keys (4 keys per step); the 16 partial states are merged in
-//   shared memory. Keys after p (the unfilled part of the local block) are
-//   masked.
+// decode_attn_kernel  each half-warp runs an online softmax over 4 keys of
+//   every selected block; the 16 partial states are merged (two per warp with
+//   shuffles, then the 8 warps in shared memory). Keys after p (the unfilled
+//   part of the local block) are neither copied nor attended. Optionally it
+//   also refreshes the representative key of the block the new token has just
+//   filled: that block is the query's own (local) block, which the kernel
+//   copies anyway, and it is never a candidate of the same step.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
+#include "tc_common.cuh"
 #include "topk.cuh"
 
 namespace phsa {
 
 namespace {
 
+using namespace tc;
+
 constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kRowBytes = kD * 2;                  // one bf16 key row
+constexpr int kSlotRows = 64;                      // rows per ring slot (one block)
+constexpr int kSlotBytes = kSlotRows * kRowBytes;  // 16 KB
+constexpr int kSelSlotsMax = 12;  // selection ring: up to 192 KB (one CTA per SM), fewer when
+                                  // the scores of a long context need the room
+constexpr int kAttnSlots = 3;                      // attention ring: 3 x (K, V) = 96 KB
 
 // Dot product of a 16-byte piece of a bf16 row with 8 fp32 values, added over
 // the 16 lanes of a half-warp (a fixed xor tree: all 16 lanes get the sum).
@@ -43,34 +64,7 @@ __device__ __forceinline__ float dot8_half(const float* q, const uint4& k) {
     return acc;
 }
 
-__device__ __forceinline__ void load_q8(const __nv_bfloat16* q, float scale, float* out) {
-    const uint4 v = __ldg(reinterpret_cast<const uint4*>(q));
-    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const float2 f = __bfloat1622float2(h[j]);
-        out[2 * j] = f.x * scale;
-        out[2 * j + 1] = f.y * scale;
-    }
-}
-
-// Block-wide reduction of one float per thread (max or sum) over 256 threads.
-template <bool kMax>
-__device__ __forceinline__ float block_reduce(float v, float* red) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-        const float o = __shfl_xor_sync(0xffffffffu, v, off);
-        v = kMax ? fmaxf(v, o) : v + o;
-    }
-    __syncthreads();  // red may still be read from a previous reduction
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
-    __syncthreads();
-    float r = red[0];
-#pragma unroll
-    for (int w = 1; w < kThreads / 32; ++w) r = kMax ? fmaxf(r, red[w]) : r + red[w];
-    return r;
-}
-
+// ============================================================== selection
 struct DecSelArgs {
     const __nv_bfloat16* q;
     const __nv_bfloat16* Kr;
@@ -78,133 +72,433 @@ struct DecSelArgs {
     int32_t* idx;
     int32_t* cnt;
     int* status;
-    int Hq, Hkv, L, Tc, topk, n_init, n_local;
+    int Hq, Hkv, L, Tc, topk, n_init, n_local, units, slots;
     float scale_log2;
 };
 
-// Shared memory: S [G][Tc] (scores, log2 units), A [Tc], finalists, picks.
-size_t dec_select_smem(int G, int Tc, int topk) {
-    return (size_t)(G + 1) * Tc * 4 + 8 * topk::kFinalMax * 8 + (size_t)topk * 4 + 64;
+// What one (sequence, KV head) unit asks of the selection. mode 0: no query
+// (length 0, or a bad length); 1: the budget covers every candidate; 2: scored.
+struct SelUnit {
+    int qb, n_init_q, loc_lo, c_lo, nC, nF, ksel, mode;
+};
+
+__device__ __forceinline__ SelUnit sel_unit(const DecSelArgs& a, int len) {
+    SelUnit s{};
+    if (len <= 0 || len > a.L) return s;
+    s.qb = (len - 1) / kM;
+    s.n_init_q = min(a.n_init, s.qb + 1);              // forced initial [0, n_init_q)
+    s.loc_lo = max(s.n_init_q, s.qb - a.n_local + 1);  // forced local [loc_lo, qb]
+    s.c_lo = a.n_init;                                 // candidates [c_lo, qb - n_local]
+    s.nC = max(0, s.qb - a.n_local - s.c_lo + 1);
+    s.nF = s.n_init_q + (s.qb - s.loc_lo + 1);
+    s.ksel = a.topk - s.nF;
+    s.mode = s.ksel >= s.nC ? 1 : 2;
+    return s;
+}
+
+__device__ __forceinline__ int sel_chunks(const SelUnit& s) {
+    return s.mode == 2 ? (s.nC + kSlotRows - 1) / kSlotRows : 0;
+}
+
+// Reduction of one float per thread (max or sum) over the 8 compute warps,
+// synchronised by named barrier 1 (the producer warp does not take part).
+template <bool kMax>
+__device__ __forceinline__ float warps_reduce(float v, float* red) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float o = __shfl_xor_sync(0xffffffffu, v, off);
+        v = kMax ? fmaxf(v, o) : v + o;
+    }
+    named_barrier(1, kThreads);  // red may still be read from a previous reduction
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    named_barrier(1, kThreads);
+    float r = red[0];
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) r = kMax ? fmaxf(r, red[w]) : r + red[w];
+    return r;
+}
+
+// Roles: warps 0-7 score the candidates, warp 8 stages each unit (its length
+// and the G query rows) into a unit slot and streams the candidates'
+// representative keys through the ring, 64 rows per slot, and warp 9 takes the
+// top-k of a unit while warps 0-7 score the next one. The scores and each
+// head's softmax statistics (running max and sum, kept online while scoring)
+// are double-buffered between the scoring warps and the top-k warp.
+constexpr int kSelThreads = 320;
+constexpr int kSelRegKeys = 16;  // candidate keys per lane kept in registers by the top-k warp
+constexpr int kSelUnitSlots = 3;
+constexpr int kSB_FULL = 0, kSB_EMPTY = kSelSlotsMax, kSB_UFULL = 2 * kSelSlotsMax,
+              kSB_UFREE = kSB_UFULL + kSelUnitSlots, kSB_AFULL = kSB_UFREE + kSelUnitSlots,
+              kSB_AFREE = kSB_AFULL + 2, kSelBars = kSB_AFREE + 2;
+constexpr int kSelBarBytes = (8 * kSelBars + 4 + 127) / 128 * 128;  // + abort flag
+static_assert(kSelBarBytes >= 8 * kSelBars + 4, "barriers and abort flag fit");
+// unit slot: {len, -, -, -} | q bf16 [G][128]
+__host__ __device__ constexpr int sel_unit_bytes(int G) { return 16 + G * kD * 2; }
+// Shared memory: ring [slots][16 KB] | barriers | unit slots | per-warp
+// statistics [8][G][2] | score buffers [2]{header {unit, len, -, -}, max [G],
+// 1/sum [G], S [G][Tc] (scores, log2 units)} | picks [topk].
+__host__ __device__ constexpr int sel_sbuf_floats(int G, int Tc) { return 4 + 2 * G + G * Tc; }
+size_t dec_select_fixed_smem(int G, int Tc, int topk) {
+    return (size_t)kSelBarBytes + (size_t)kSelUnitSlots * sel_unit_bytes(G) +
+           (size_t)kWarps * G * 2 * 4 + 2 * (size_t)sel_sbuf_floats(G, Tc) * 4 +
+           (size_t)topk * 4 + 16;
+}
+// ring slots that fit beside the rest when per_sm CTAs share an SM's 228 KB
+// (0 if not even two)
+int dec_select_slots(int G, int Tc, int topk, int per_sm) {
+    const size_t fixed = dec_select_fixed_smem(G, Tc, topk);
+    const size_t cap = per_sm <= 1 ? 227 * 1024 : 228 * 1024 / per_sm - 2 * 1024;
+    size_t fit = fixed >= cap ? 0 : (cap - fixed) / kSlotBytes;
+    if (fit > (size_t)kSelSlotsMax) fit = kSelSlotsMax;
+    const int n = (int)fit;
+    return n >= 2 ? n : 0;
+}
+size_t dec_select_smem(int G, int Tc, int topk, int slots) {
+    return (size_t)(slots > 0 ? slots : 2) * kSlotBytes + dec_select_fixed_smem(G, Tc, topk);
 }
 
 template <int G>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kSelThreads, 2)
 decode_select_kernel(const DecSelArgs a) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    unsigned long long* fin = reinterpret_cast<unsigned long long*>(smem);
-    float* red = reinterpret_cast<float*>(smem + 8 * topk::kFinalMax * 8);   // 8 floats
-    float* S = red + 16;                                                        // [G][Tc]
-    float* A = S + (size_t)G * a.Tc;                                            // [Tc]
-    int* sel = reinterpret_cast<int*>(A + a.Tc);                                // [topk]
+    extern __shared__ __align__(128) uint8_t smem[];
+    const uint32_t sb = smem_u32(smem);
+    const int nslots = a.slots, off_bar = nslots * kSlotBytes;
+    auto bar = [&](int i) { return sb + off_bar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + off_bar + 8 * kSelBars);
+    uint8_t* units0 = smem + off_bar + kSelBarBytes;
+    float* wstat = reinterpret_cast<float*>(units0 + kSelUnitSlots * sel_unit_bytes(G));  // [8][G][2]
+    float* sbuf0 = wstat + kWarps * G * 2;                       // [2][sel_sbuf_floats]
+    const int sbuf_floats = sel_sbuf_floats(G, a.Tc);
+    int* sel = reinterpret_cast<int*>(sbuf0 + 2 * sbuf_floats);  // [topk]
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int u = blockIdx.x;
-    const int b = u / a.Hkv, g = u % a.Hkv;
-    const int len = a.lens[b];
-    int32_t* out = a.idx + (size_t)u * a.topk;
-    if (len <= 0 || len > a.L) {  // no query (or a bad length): empty selection
-        if (tid == 0 && (len < 0 || len > a.L)) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
-        for (int j = tid; j < a.topk; j += kThreads) out[j] = -1;
-        if (tid == 0) a.cnt[u] = 0;
-        return;
-    }
-    const int qb = (len - 1) / kM;
-    const int n_init_q = min(a.n_init, qb + 1);            // forced initial [0, n_init_q)
-    const int loc_lo = max(n_init_q, qb - a.n_local + 1);  // forced local [loc_lo, qb]
-    const int c_lo = a.n_init, c_hi = qb - a.n_local;      // candidates, all full blocks
-    const int nC = max(0, c_hi - c_lo + 1);
-    const int nF = n_init_q + (qb - loc_lo + 1);
-    const int ksel = a.topk - nF;
-    if (ksel >= nC) {  // the budget covers every candidate
-        const int n = nF + nC;
-        for (int j = tid; j < a.topk; j += kThreads) {
-            int v = -1;
-            if (j < n_init_q) v = j;
-            else if (j < n_init_q + nC) v = c_lo + (j - n_init_q);
-            else if (j < n) v = loc_lo + (j - n_init_q - nC);
-            out[j] = v;
+    auto unit_of = [&](int k) { return (int)blockIdx.x + k * (int)gridDim.x; };
+
+    if (tid == 0) {
+        for (int i = 0; i < nslots; ++i) {
+            mbar_init(bar(kSB_FULL + i), 1);
+            mbar_init(bar(kSB_EMPTY + i), kWarps);
         }
-        if (tid == 0) a.cnt[u] = n;
+        for (int i = 0; i < kSelUnitSlots; ++i) {
+            mbar_init(bar(kSB_UFULL + i), 1);
+            mbar_init(bar(kSB_UFREE + i), kWarps);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(kSB_AFULL + i), 1);
+            mbar_init(bar(kSB_AFREE + i), 1);
+        }
+        fence_barrier_init();
+        *abort_flag = 0;
+    }
+    __syncthreads();
+
+    if (warp == kWarps) {
+        // ------------------------------------------------ producer
+        bool ok = true;
+        int issued = 0, staged = -1, ik = 0, ic = 0;  // copies; last unit staged; cursor
+        Deadline dl;
+        while (ok) {
+            bool progressed = false;
+            const bool more = unit_of(ik) < a.units;
+            if (more && ik <= staged) {
+                const int len = *reinterpret_cast<const int*>(units0 + (ik % kSelUnitSlots) *
+                                                                           sel_unit_bytes(G));
+                const SelUnit su = sel_unit(a, len);
+                if (ic >= sel_chunks(su)) {
+                    ++ik;
+                    ic = 0;
+                    continue;
+                }
+                const int sl = issued % nslots;
+                bool free_slot = issued < nslots;
+                if (!free_slot && lane == 0)
+                    free_slot = mbar_test_wait(bar(kSB_EMPTY + sl), ((issued / nslots) - 1) & 1);
+                if (__shfl_sync(0xffffffffu, free_slot, 0)) {
+                    if (lane == 0) {
+                        const uint32_t bytes =
+                            (uint32_t)min(kSlotRows, su.nC - ic * kSlotRows) * kRowBytes;
+                        const __nv_bfloat16* src =
+                            a.Kr + ((size_t)unit_of(ik) * a.Tc + su.c_lo + (size_t)ic * kSlotRows) * kD;
+                        mbar_expect_tx(bar(kSB_FULL + sl), bytes);
+                        bulk_load(sb + sl * kSlotBytes, src, bytes, bar(kSB_FULL + sl));
+                    }
+                    ++issued;
+                    ++ic;
+                    progressed = true;
+                }
+            }
+            const int ks = staged + 1;
+            if (!progressed && unit_of(ks) < a.units && ks <= ik + 2) {
+                bool free_unit = ks < kSelUnitSlots;
+                if (!free_unit && lane == 0)
+                    free_unit = mbar_test_wait(bar(kSB_UFREE + ks % kSelUnitSlots),
+                                               ((ks / kSelUnitSlots) - 1) & 1);
+                if (__shfl_sync(0xffffffffu, free_unit, 0)) {
+                    // stage unit ks: its length and the group's query rows
+                    const int u = unit_of(ks), b = u / a.Hkv, g = u % a.Hkv;
+                    uint8_t* slot = units0 + (ks % kSelUnitSlots) * sel_unit_bytes(G);
+                    if (lane < G * 16)
+                        reinterpret_cast<uint4*>(slot + 16)[lane] = __ldg(
+                            reinterpret_cast<const uint4*>(a.q + ((size_t)b * a.Hq + g * G) * kD) + lane);
+                    if (lane == 0) *reinterpret_cast<int*>(slot) = __ldg(a.lens + b);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar(kSB_UFULL + ks % kSelUnitSlots));
+                    staged = ks;
+                    progressed = true;
+                }
+            }
+            if (!more && unit_of(staged + 1) >= a.units) break;  // every copy issued
+            if (progressed) {
+                dl.reset();
+            } else {
+                __nanosleep(64);  // nothing to do yet: leave the issue slots to the other warps
+                if (*abort_flag) {
+                    ok = false;
+                } else if (dl.expired()) {
+                    *abort_flag = 1;
+                    if (lane == 0) atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
+                    ok = false;
+                }
+            }
+            ok = __all_sync(0xffffffffu, ok) != 0;
+        }
+        if (lane == 0)  // own copies land before the CTA may exit
+            for (int j = max(0, issued - nslots); j < issued; ++j)
+                mbar_wait_drain(bar(kSB_FULL + j % nslots), (j / nslots) & 1);
         return;
     }
 
-    // ---- scores: half-warp hw takes candidates hw, hw + 16, ... four at a time
-    const int hw = tid >> 4, c16 = tid & 15;
-    float qv[G][8];
+    if (warp == kWarps + 1) {
+        // ------------------------------------------------ top-k (one warp)
+        bool ok = true;
+        for (int su = 0; ok; ++su) {
+            const int buf = su & 1;
+            ok = mbar_wait(bar(kSB_AFULL + buf), (su >> 1) & 1, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok) != 0;
+            if (!ok) break;
+            float* sbuf = sbuf0 + buf * sbuf_floats;
+            const int u = reinterpret_cast<const int*>(sbuf)[0];
+            if (u < 0) break;  // the end of the CTA's units
+            const SelUnit d = sel_unit(a, reinterpret_cast<const int*>(sbuf)[1]);
+            const float* mx = sbuf + 4;
+            const float* iz = mx + G;
+            float* Sb = sbuf + 4 + 2 * G;
+            const int nC = d.nC, ksel = d.ksel, c_lo = d.c_lo;
+            // A_t = sum over the heads of the head's softmax probability, head order
+            auto key_of = [&](int cj) {
+                float acc = 0.f;
 #pragma unroll
-    for (int h = 0; h < G; ++h)
-        load_q8(a.q + ((size_t)b * a.Hq + g * G + h) * kD + c16 * 8, a.scale_log2, qv[h]);
-    const __nv_bfloat16* Krg = a.Kr + ((size_t)u * a.Tc + c_lo) * kD + c16 * 8;
-    // The trip count is the same for every thread, so both half-warps of a warp
-    // always reach the shuffles of dot8_half together.
-    for (int base = hw; base - hw < nC; base += 64) {
-        uint4 kv[4];
+                for (int h = 0; h < G; ++h) acc += ex2_approx(Sb[h * a.Tc + cj] - mx[h]) * iz[h];
+                return topk::make_key(acc, c_lo + cj);
+            };
+            if (nC <= 32 * kSelRegKeys) {
+                unsigned long long key[kSelRegKeys];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            const int cj = base + 16 * r;
-            kv[r] = cj < nC ? __ldg(reinterpret_cast<const uint4*>(Krg + (size_t)cj * kD))
-                            : make_uint4(0u, 0u, 0u, 0u);
+                for (int rr = 0; rr < kSelRegKeys; ++rr) {
+                    const int cj = lane + 32 * rr;
+                    key[rr] = cj < nC ? key_of(cj) : 0ull;
+                }
+                for (int kk = 0; kk < ksel; ++kk) {
+                    unsigned long long best = key[0];
+#pragma unroll
+                    for (int rr = 1; rr < kSelRegKeys; ++rr) best = topk::umax64(best, key[rr]);
+                    const unsigned mh = (unsigned)(best >> 32), ml = (unsigned)best;
+                    const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
+                    const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
+                    const unsigned long long win = ((unsigned long long)bh << 32) | bl;
+                    if (lane == 0) sel[kk] = topk::key_block(win);
+#pragma unroll
+                    for (int rr = 0; rr < kSelRegKeys; ++rr)
+                        if (key[rr] == win) key[rr] = 0ull;
+                }
+            } else {  // long contexts: rounds over shared memory; a pick is marked by a NaN score
+                topk::rounds_one_warp(
+                    nC, ksel, key_of, [&](int cj) { return Sb[cj] != Sb[cj]; },
+                    [&](int t) { Sb[t - c_lo] = __int_as_float(0x7fc00000); }, sel, lane);
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kSB_AFREE + buf));  // the scoring warps may refill it
+            int32_t* out = a.idx + (size_t)u * a.topk;
+            for (int j = lane; j < a.topk; j += 32) {
+                if (j < d.n_init_q) out[j] = j;
+                else if (j >= d.n_init_q + ksel && j < d.nF + ksel)
+                    out[j] = d.loc_lo + (j - d.n_init_q - ksel);
+                else if (j >= d.nF + ksel) out[j] = -1;
+            }
+            for (int j = lane; j < ksel; j += 32) {
+                const int v = sel[j];
+                int rank = 0;
+                for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
+                out[d.n_init_q + rank] = v;
+            }
+            if (lane == 0) a.cnt[u] = d.nF + ksel;
+            __syncwarp();  // sel is reused by the next unit
         }
+        return;
+    }
+
+    // ---------------------------------------------------- compute (warps 0-7)
+    int gc = 0, su = 0;  // chunks consumed; units scored
+    bool ok = true;
+    for (int k = 0;; ++k) {
+        const int u = unit_of(k);
+        if (u >= a.units) break;
+        const int us = k % kSelUnitSlots;
+        ok = ok && mbar_wait(bar(kSB_UFULL + us), (k / kSelUnitSlots) & 1, abort_flag, a.status);
+        ok = __all_sync(0xffffffffu, ok) != 0;
+        // the eight warps leave at the same unit (they meet at a barrier below)
+        if (!named_barrier_and(1, kThreads, ok)) break;
+        const uint8_t* slot = units0 + us * sel_unit_bytes(G);
+        const int len = *reinterpret_cast<const int*>(slot);
+        const SelUnit su_ = sel_unit(a, len);
+        if (su_.mode != 2) {
+            int32_t* out = a.idx + (size_t)u * a.topk;
+            if (su_.mode == 0) {  // no query (or a bad length): empty selection
+                if (tid == 0 && (len < 0 || len > a.L)) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
+                for (int j = tid; j < a.topk; j += kThreads) out[j] = -1;
+                if (tid == 0) a.cnt[u] = 0;
+            } else {  // the budget covers every candidate
+                const int n = su_.nF + su_.nC;
+                for (int j = tid; j < a.topk; j += kThreads) {
+                    int v = -1;
+                    if (j < su_.n_init_q) v = j;
+                    else if (j < su_.n_init_q + su_.nC) v = su_.c_lo + (j - su_.n_init_q);
+                    else if (j < n) v = su_.loc_lo + (j - su_.n_init_q - su_.nC);
+                    out[j] = v;
+                }
+                if (tid == 0) a.cnt[u] = n;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kSB_UFREE + us));
+            continue;
+        }
+        const int nC = su_.nC;
+        const int buf = su & 1;
+        if (su >= 2)  // the top-k warp is done with this buffer's unit before last
+            ok = ok && mbar_wait(bar(kSB_AFREE + buf), ((su >> 1) - 1) & 1, abort_flag, a.status);
+        float* sbuf = sbuf0 + buf * sbuf_floats;
+        float* Sb = sbuf + 4 + 2 * G;
+
+        // ---- scores: four threads per candidate row, each 32 of the 128 columns
+        // (thread 4r + qd: row r of each 64-row chunk, columns [32 qd, 32 qd + 32)).
+        // Its four 16-byte pieces are taken in the order rotated by r, so that a
+        // warp's eight rows fall on distinct banks; q is kept in the same order.
+        const int r = tid >> 2, qd = tid & 3, rot = r & 3;
+        float qv[G][4][8];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            const int cj = base + 16 * r;
+        for (int h = 0; h < G; ++h)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int piece = 4 * qd + ((c + rot) & 3);
+                const uint4 v = *reinterpret_cast<const uint4*>(slot + 16 + h * kRowBytes + piece * 16);
+                const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float2 f = __bfloat1622float2(h2[j]);
+                    qv[h][c][2 * j] = f.x * a.scale_log2;
+                    qv[h][c][2 * j + 1] = f.y * a.scale_log2;
+                }
+            }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(kSB_UFREE + us));  // the slot's q and length are read
+        // each head's softmax statistics over the candidates, online: running
+        // max and sum of 2^(S - max) over the rows this thread writes
+        float m_run[G], z_run[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            m_run[h] = -INFINITY;
+            z_run[h] = 0.f;
+        }
+        const int nch = sel_chunks(su_);
+        for (int i = 0; i < nch; ++i, ++gc) {
+            const int sl = gc % nslots;
+            ok = ok && mbar_wait(bar(kSB_FULL + sl), (gc / nslots) & 1, abort_flag, a.status);
+            const int rows = min(kSlotRows, nC - i * kSlotRows);
+            const bool v = ok && r < rows;
+            const uint8_t* row = smem + sl * kSlotBytes + r * kRowBytes;
+            float acc[G][4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const uint4 kv = v ? *reinterpret_cast<const uint4*>(row + (4 * qd + ((c + rot) & 3)) * 16)
+                                   : make_uint4(0u, 0u, 0u, 0u);
+                const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    float t = 0.f;
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float2 f = __bfloat1622float2(k2[j]);
+                        t = fmaf(qv[h][c][2 * j], f.x, t);
+                        t = fmaf(qv[h][c][2 * j + 1], f.y, t);
+                    }
+                    acc[h][c] = t;
+                }
+            }
+            // every lane takes part in the shuffles (a row past the chunk holds zeros)
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                const float s = dot8_half(qv[h], kv[r]);
-                if (c16 == 0 && cj < nC) S[h * a.Tc + cj] = s;
+                float sc = (acc[h][0] + acc[h][1]) + (acc[h][2] + acc[h][3]);
+                sc += __shfl_xor_sync(0xffffffffu, sc, 1);
+                sc += __shfl_xor_sync(0xffffffffu, sc, 2);
+                if (qd == 0 && v) {
+                    Sb[h * a.Tc + i * kSlotRows + r] = sc;
+                    const float mn = fmaxf(m_run[h], sc);
+                    z_run[h] = z_run[h] * ex2_approx(m_run[h] - mn) + ex2_approx(sc - mn);
+                    m_run[h] = mn;
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kSB_EMPTY + sl));  // this warp is done with the slot
+        }
+        // statistics of the warp's rows, then of the eight warps (thread 0)
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            float m = m_run[h], z = z_run[h];
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                const float mo = __shfl_xor_sync(0xffffffffu, m, off);
+                const float zo = __shfl_xor_sync(0xffffffffu, z, off);
+                const float mn = fmaxf(m, mo);
+                z = mn == -INFINITY ? 0.f : z * ex2_approx(m - mn) + zo * ex2_approx(mo - mn);
+                m = mn;
+            }
+            if (lane == 0) {
+                wstat[(warp * G + h) * 2] = m;
+                wstat[(warp * G + h) * 2 + 1] = z;
             }
         }
-    }
-    __syncthreads();
-
-    // ---- per head: softmax over the candidates; A_t = sum over heads
-    float mx[G], iz[G];
+        if (!named_barrier_and(1, kThreads, ok)) break;  // scores and statistics complete
+        if (tid == 0) {
 #pragma unroll
-    for (int h = 0; h < G; ++h) {
-        float m = -INFINITY;
-        for (int cj = tid; cj < nC; cj += kThreads) m = fmaxf(m, S[h * a.Tc + cj]);
-        mx[h] = block_reduce<true>(m, red);
-        float z = 0.f;
-        for (int cj = tid; cj < nC; cj += kThreads) z += exp2f(S[h * a.Tc + cj] - mx[h]);
-        z = block_reduce<false>(z, red);
-        iz[h] = z > 0.f ? 1.0f / z : 0.f;
+            for (int h = 0; h < G; ++h) {
+                float m = -INFINITY, z = 0.f;
+                for (int w = 0; w < kWarps; ++w) {
+                    const float mo = wstat[(w * G + h) * 2], zo = wstat[(w * G + h) * 2 + 1];
+                    const float mn = fmaxf(m, mo);
+                    z = mn == -INFINITY ? 0.f : z * ex2_approx(m - mn) + zo * ex2_approx(mo - mn);
+                    m = mn;
+                }
+                sbuf[4 + h] = m;
+                sbuf[4 + G + h] = z > 0.f ? 1.0f / z : 0.f;
+            }
+            reinterpret_cast<int*>(sbuf)[0] = u;
+            reinterpret_cast<int*>(sbuf)[1] = len;
+            mbar_arrive(bar(kSB_AFULL + buf));  // hand the unit to the top-k warp
+        }
+        ++su;
     }
-    for (int cj = tid; cj < nC; cj += kThreads) {
-        float acc = 0.f;
-#pragma unroll
-        for (int h = 0; h < G; ++h) acc += exp2f(S[h * a.Tc + cj] - mx[h]) * iz[h];
-        A[cj] = acc;
+    if (tid == 0 && ok) {  // the end of the CTA's units for the top-k warp
+        const int buf = su & 1;
+        bool free_buf = true;
+        if (su >= 2)
+            free_buf = mbar_wait(bar(kSB_AFREE + buf), ((su >> 1) - 1) & 1, abort_flag, a.status);
+        if (free_buf) {
+            reinterpret_cast<int*>(sbuf0 + buf * sbuf_floats)[0] = -1;
+            mbar_arrive(bar(kSB_AFULL + buf));
+        }
     }
-    __syncthreads();
-
-    // ---- top-k
-    auto key_of = [&](int cj) { return topk::make_key(A[cj], c_lo + cj); };
-    const bool fast = topk::two_level(nC, ksel);
-    if (fast) {
-        topk::level1(nC, ksel, key_of, fin, warp, lane);
-    } else if (warp == 0) {
-        topk::rounds_one_warp(
-            nC, ksel, key_of, [&](int cj) { return A[cj] == -1.0f; },
-            [&](int t) { A[t - c_lo] = -1.0f; }, sel, lane);
-    }
-    __syncthreads();
-    if (fast) topk::level2(fin, ksel, sel, tid);
-    __syncthreads();
-
-    // ---- forced + picked, ascending, -1 padded
-    for (int j = tid; j < a.topk; j += kThreads) {
-        if (j < n_init_q) out[j] = j;
-        else if (j >= n_init_q + ksel && j < nF + ksel) out[j] = loc_lo + (j - n_init_q - ksel);
-        else if (j >= nF + ksel) out[j] = -1;
-    }
-    for (int j = tid; j < ksel; j += kThreads) {
-        const int v = sel[j];
-        int rank = 0;
-        for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
-        out[n_init_q + rank] = v;
-    }
-    if (tid == 0) a.cnt[u] = nF + ksel;
 }
 
+// ============================================================== attention
 struct DecAttnArgs {
     const __nv_bfloat16* q;
     const __nv_bfloat16* K;
@@ -215,150 +509,490 @@ struct DecAttnArgs {
     __nv_bfloat16* O;
     float* lse;
     int* status;
-    int Hq, Hkv, L, topk;
+    const uint8_t* mask;   // with Krepr: refresh the block the new token has just filled
+    __nv_bfloat16* Krepr;  // null: no refresh
+    float lambda;
+    int Hq, Hkv, L, T, topk, units;
     float scale_log2;
 };
 
-// Shared memory: block list [topk] | per half-warp state [16][G][2 + 128].
+// Warp-wide copy of one unit's block list to shared memory (out holds topk
+// ints), with the rule of compact_block_list: -1 entries are skipped, and so
+// is an entry outside [0, qb] or not above the last kept one (reported). A
+// list whose first cnt entries are all valid and ascending -- every list the
+// selection writes -- takes one load per lane; anything else goes through
+// compact_block_list on lane 0. Returns the count on every lane.
+__device__ __forceinline__ int stage_list_warp(const int32_t* row, const int32_t* cntp, int topk,
+                                               int qb, int* out, int* status, int lane) {
+    const int cnt = __ldg(cntp);
+    bool good = cnt >= 0 && cnt <= topk;
+    for (int j0 = 0; j0 < topk; j0 += 32) {
+        const int j = j0 + lane;
+        const int t = j < topk ? __ldg(row + j) : 0;
+        int prev = __shfl_up_sync(0xffffffffu, t, 1);
+        if (lane == 0) prev = j0 > 0 ? out[j0 - 1] : -1;
+        good &= __all_sync(0xffffffffu, j >= cnt || (t >= 0 && t <= qb && t > prev)) != 0;
+        if (j < topk) out[j] = t;
+        __syncwarp();
+    }
+    if (good) return cnt;
+    int n = 0;
+    if (lane == 0) n = compact_block_list(row, cnt, topk, qb, out, status);
+    return __shfl_sync(0xffffffffu, n, 0);
+}
+
+// Roles: warps 0-7 compute; warp 8 is the producer. The producer stages each
+// unit (length, block list, the G query rows, the punctuation bits of a
+// just-filled block) into one of kUnitSlots unit slots, up to two units ahead,
+// and streams the selected K/V blocks through the ring. Barriers: full / empty per
+// ring slot (empty counts the 8 compute warps), ufull / ufree per unit slot.
+// The compute warps meet only once per unit (the merge).
+constexpr int kAttnThreads = 288;
+constexpr int kUnitSlots = 3;
+constexpr int kAB_FULL = 0, kAB_EMPTY = kAttnSlots, kAB_UFULL = 2 * kAttnSlots,
+              kAB_UFREE = kAB_UFULL + kUnitSlots, kAttnBars = kAB_UFREE + kUnitSlots;
+constexpr int kAttnOffBar = kAttnSlots * 2 * kSlotBytes;
+constexpr int kAttnOffUnit = kAttnOffBar + (8 * kAttnBars + 4 + 127) / 128 * 128;  // + abort flag
+static_assert(kAttnOffUnit - kAttnOffBar >= 8 * kAttnBars + 4, "barriers and abort flag fit");
+// unit slot: {len, n, plo, phi} | q bf16 [G][128] | block list [topk rounded up to 4]
+__host__ __device__ constexpr int unit_slot_bytes(int G, int topk) {
+    return 16 + G * kD * 2 + ((topk + 3) & ~3) * 4;
+}
 size_t dec_attn_smem(int G, int topk) {
-    return (size_t)((topk + 4) & ~3) * 4 + (size_t)16 * G * 130 * 4;
+    return (size_t)kAttnOffUnit + (size_t)kUnitSlots * unit_slot_bytes(G, topk) +
+           (size_t)kWarps * G * 130 * 4 + 4 * 2 * kD * 4;
 }
 
 template <int G>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kAttnThreads, 2)
 decode_attn_kernel(const DecAttnArgs a) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    int* list = reinterpret_cast<int*>(smem);
-    float* part = reinterpret_cast<float*>(smem + (size_t)((a.topk + 4) & ~3) * 4);
-    __shared__ int s_n;
-    const int tid = threadIdx.x;
-    const int u = blockIdx.x;
-    const int b = u / a.Hkv, g = u % a.Hkv;
-    const int len = a.lens[b];
-    const size_t orow = (size_t)b * a.Hq + g * G;  // first query head of the group
-    if (len <= 0 || len > a.L) {  // no query: zero output, lse = -inf
-        if (tid == 0 && (len < 0 || len > a.L)) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
-        for (int e = tid; e < G * kD; e += kThreads)
-            a.O[orow * kD + e] = __float2bfloat16_rn(0.f);
-        if (tid < G) a.lse[orow + tid] = -INFINITY;
-        return;
-    }
-    const int p = len - 1, qb = p / kM;
-    if (tid == 0) s_n = compact_block_list(a.idx + (size_t)u * a.topk, a.cnt[u], a.topk, qb, list, a.status);
-    __syncthreads();
-    const int nk = s_n * kM;
+    extern __shared__ __align__(128) uint8_t smem[];
+    const uint32_t sb = smem_u32(smem);
+    auto bar = [&](int i) { return sb + kAttnOffBar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kAttnOffBar + 8 * kAttnBars);
+    const int ubytes = unit_slot_bytes(G, a.topk);
+    uint8_t* units0 = smem + kAttnOffUnit;
+    float* part = reinterpret_cast<float*>(units0 + kUnitSlots * ubytes);  // [8][G][130]
+    float* rpart = part + kWarps * G * 130;                               // [4][2][128]
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    auto unit_of = [&](int k) { return (int)blockIdx.x + k * (int)gridDim.x; };
+    const bool refresh = a.Krepr != nullptr;
 
-    const int hw = tid >> 4, c16 = tid & 15;
-    float qv[G][8];
-#pragma unroll
-    for (int h = 0; h < G; ++h) load_q8(a.q + (orow + h) * kD + c16 * 8, a.scale_log2, qv[h]);
-    const __nv_bfloat16* Kg = a.K + (size_t)u * a.L * kD + c16 * 8;
-    const __nv_bfloat16* Vg = a.V + (size_t)u * a.L * kD + c16 * 8;
-
-    float m[G], l[G], o[G][8];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-        m[h] = -INFINITY;
-        l[h] = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) o[h][e] = 0.f;
-    }
-    // Half-warp hw takes keys [4 hw, 4 hw + 4) of every 64: four consecutive rows.
-    for (int kb = 4 * hw; kb < nk; kb += 64) {
-        uint4 kr[4], vr[4];
-        int pos[4];
-#pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            const int key = kb + r;
-            pos[r] = list[key >> 6] * kM + (key & 63);
-            const bool ok = pos[r] <= p;
-            kr[r] = ok ? __ldg(reinterpret_cast<const uint4*>(Kg + (size_t)pos[r] * kD))
-                       : make_uint4(0u, 0u, 0u, 0u);
-            vr[r] = ok ? __ldg(reinterpret_cast<const uint4*>(Vg + (size_t)pos[r] * kD))
-                       : make_uint4(0u, 0u, 0u, 0u);
+    if (tid == 0) {
+        for (int i = 0; i < kAttnSlots; ++i) {
+            mbar_init(bar(kAB_FULL + i), 1);
+            mbar_init(bar(kAB_EMPTY + i), kWarps);
         }
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            float s[4];
-            float mn = m[h];
-#pragma unroll
-            for (int r = 0; r < 4; ++r) {
-                // dot8_half shuffles across the whole warp: call it on every lane
-                // (a masked key holds zeros), then mask the score
-                const float d = dot8_half(qv[h], kr[r]);
-                s[r] = pos[r] <= p ? d : -INFINITY;
-                mn = fmaxf(mn, s[r]);
+        for (int i = 0; i < kUnitSlots; ++i) {
+            mbar_init(bar(kAB_UFULL + i), 1);
+            mbar_init(bar(kAB_UFREE + i), kWarps);
+        }
+        fence_barrier_init();
+        *abort_flag = 0;
+    }
+    __syncthreads();
+
+    if (warp == kWarps) {
+        // ------------------------------------------------ producer
+        bool ok = true;
+        int issued = 0;  // blocks copied
+        // stage the CTA's k-th unit into unit slot k % kUnitSlots
+        auto stage = [&](int k) {
+            const int us = k % kUnitSlots;  // free: the loop has seen its ufree phase
+            const int u = unit_of(k), b = u / a.Hkv, g = u % a.Hkv;
+            uint8_t* slot = units0 + us * ubytes;
+            int* hdr = reinterpret_cast<int*>(slot);
+            int* list = hdr + 4 + G * kD / 2;
+            const int len = __ldg(a.lens + b);
+            const bool valid = len > 0 && len <= a.L;
+            if (lane < G * 16)  // the group's query rows, 16 bytes per lane
+                reinterpret_cast<uint4*>(slot + 16)[lane] = __ldg(
+                    reinterpret_cast<const uint4*>(a.q + ((size_t)b * a.Hq + g * G) * kD) + lane);
+            int n = 0;
+            if (valid)
+                n = stage_list_warp(a.idx + (size_t)u * a.topk, a.cnt + u, a.topk, (len - 1) / kM,
+                                    list, a.status, lane);
+            unsigned plo = 0, phi = 0;
+            if (refresh && valid && len % kM == 0) {
+                const uint8_t* mb = a.mask + (size_t)b * a.L + (size_t)(len / kM - 1) * kM;
+                plo = __ballot_sync(0xffffffffu, mb[lane] != 0);
+                phi = __ballot_sync(0xffffffffu, mb[32 + lane] != 0);
             }
-            if (mn == -INFINITY) continue;  // no key of this step is visible
-            const float sc = exp2f(m[h] - mn);
-            l[h] *= sc;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) o[h][e] *= sc;
-#pragma unroll
-            for (int r = 0; r < 4; ++r) {
-                const float pr = exp2f(s[r] - mn);
-                l[h] += pr;
-                const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&vr[r]);
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float2 f = __bfloat1622float2(v2[j]);
-                    o[h][2 * j] = fmaf(pr, f.x, o[h][2 * j]);
-                    o[h][2 * j + 1] = fmaf(pr, f.y, o[h][2 * j + 1]);
+            if (lane == 0) {
+                hdr[0] = len;
+                hdr[1] = n;
+                hdr[2] = (int)plo;
+                hdr[3] = (int)phi;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kAB_UFULL + us));
+        };
+        // Event loop: a copy whenever a ring slot is free and the next block is
+        // known; otherwise stage the next unit (up to two ahead of the copies),
+        // so that the loads of staging never hold back a copy.
+        int staged = -1, ik = 0, ii = 0;  // last unit staged; copy cursor (unit, block)
+        Deadline dl;
+        while (ok) {
+            bool progressed = false;
+            const bool more = unit_of(ik) < a.units;
+            if (more && ik <= staged) {
+                const int* hdr = reinterpret_cast<const int*>(units0 + (ik % kUnitSlots) * ubytes);
+                const int n = hdr[1];
+                if (ii >= n) {
+                    ++ik;
+                    ii = 0;
+                    continue;
+                }
+                const int sl = issued % kAttnSlots;
+                bool free_slot = issued < kAttnSlots;
+                if (!free_slot && lane == 0)
+                    free_slot = mbar_test_wait(bar(kAB_EMPTY + sl), ((issued / kAttnSlots) - 1) & 1);
+                free_slot = __shfl_sync(0xffffffffu, free_slot, 0) != 0;
+                if (free_slot) {
+                    if (lane == 0) {
+                        const int t = hdr[4 + G * kD / 2 + ii];
+                        const int len = hdr[0], p = len - 1;
+                        const int rows = t == p / kM ? p - t * kM + 1 : kM;  // keys up to p
+                        const size_t off = ((size_t)unit_of(ik) * a.L + (size_t)t * kM) * kD;
+                        const uint32_t bytes = (uint32_t)rows * kRowBytes;
+                        mbar_expect_tx(bar(kAB_FULL + sl), 2 * bytes);
+                        bulk_load(sb + sl * 2 * kSlotBytes, a.K + off, bytes, bar(kAB_FULL + sl));
+                        bulk_load(sb + sl * 2 * kSlotBytes + kSlotBytes, a.V + off, bytes,
+                                  bar(kAB_FULL + sl));
+                    }
+                    ++issued;
+                    ++ii;
+                    progressed = true;
                 }
             }
-            m[h] = mn;
+            const int ks = staged + 1;
+            if (!progressed && unit_of(ks) < a.units && ks <= ik + 2) {
+                bool free_unit = ks < kUnitSlots;
+                if (!free_unit && lane == 0)
+                    free_unit = mbar_test_wait(bar(kAB_UFREE + ks % kUnitSlots),
+                                               ((ks / kUnitSlots) - 1) & 1);
+                if (__shfl_sync(0xffffffffu, free_unit, 0)) {
+                    stage(ks);
+                    staged = ks;
+                    progressed = true;
+                }
+            }
+            if (!more && unit_of(staged + 1) >= a.units) break;  // every copy issued
+            if (progressed) {
+                dl.reset();
+            } else {
+                __nanosleep(64);  // nothing to do yet: leave the issue slots to the other warps
+                if (*abort_flag) {
+                    ok = false;
+                } else if (dl.expired()) {
+                    *abort_flag = 1;
+                    if (lane == 0) atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
+                    ok = false;
+                }
+            }
+            ok = __all_sync(0xffffffffu, ok) != 0;
         }
+        if (lane == 0)  // own copies land before the CTA may exit
+            for (int j = max(0, issued - kAttnSlots); j < issued; ++j)
+                mbar_wait_drain(bar(kAB_FULL + j % kAttnSlots), (j / kAttnSlots) & 1);
+        return;
     }
-    // ---- merge the 16 half-warp states
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-        float* st = part + ((size_t)hw * G + h) * 130;
-        if (c16 == 0) {
-            st[0] = m[h];
-            st[1] = l[h];
+
+    // ---------------------------------------------------- compute (warps 0-7)
+    const int hw = tid >> 4, c16 = tid & 15;
+    int gc = 0;  // blocks consumed
+    bool ok = true;
+    for (int k = 0;; ++k) {
+        const int u = unit_of(k);
+        if (u >= a.units) break;
+        const int us = k % kUnitSlots;
+        ok = ok && mbar_wait(bar(kAB_UFULL + us), (k / kUnitSlots) & 1, abort_flag, a.status);
+        ok = __all_sync(0xffffffffu, ok) != 0;
+        // the eight warps leave at the same unit (the merge has a barrier among them)
+        if (!named_barrier_and(1, kThreads, ok)) break;
+        const uint8_t* slot = units0 + us * ubytes;
+        const int* hdr = reinterpret_cast<const int*>(slot);
+        const int* list = hdr + 4 + G * kD / 2;
+        const int len = hdr[0], nb = hdr[1];
+        const unsigned plo = (unsigned)hdr[2], phi = (unsigned)hdr[3];
+        const int b = u / a.Hkv, g = u % a.Hkv;
+        const size_t orow = (size_t)b * a.Hq + g * G;  // first query head of the group
+        if (len <= 0 || len > a.L) {  // no query: zero output, lse = -inf
+            if (tid == 0 && (len < 0 || len > a.L)) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
+            for (int e = tid; e < G * kD; e += kThreads) a.O[orow * kD + e] = __float2bfloat16_rn(0.f);
+            if (tid < G) a.lse[orow + tid] = -INFINITY;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kAB_UFREE + us));
+            continue;
         }
+        const int p = len - 1, qb = p / kM;
+        const bool fill = refresh && len % kM == 0;  // refresh block qb's representative key
+        float qv[G][8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) st[2 + c16 * 8 + e] = o[h][e];
-    }
-    __syncthreads();
-    if (tid < G * kD) {
-        const int h = tid / kD, d = tid % kD;
-        float M = -INFINITY;
-        for (int w = 0; w < 16; ++w) M = fmaxf(M, part[((size_t)w * G + h) * 130]);
-        float Ls = 0.f, acc = 0.f;
-        if (M != -INFINITY) {
-            for (int w = 0; w < 16; ++w) {
-                const float* st = part + ((size_t)w * G + h) * 130;
-                const float f = exp2f(st[0] - M);  // 0 for a half-warp that saw no key
-                Ls += st[1] * f;
-                acc += st[2 + d] * f;
+        for (int h = 0; h < G; ++h) {
+            const uint4 v = *reinterpret_cast<const uint4*>(slot + 16 + h * kRowBytes + c16 * 16);
+            const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float2 f = __bfloat1622float2(h2[j]);
+                qv[h][2 * j] = f.x * a.scale_log2;
+                qv[h][2 * j + 1] = f.y * a.scale_log2;
             }
         }
-        a.O[(orow + h) * kD + d] = __float2bfloat16_rn(Ls > 0.f ? acc / Ls : 0.f);
-        if (d == 0) a.lse[orow + h] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
+        float m[G], l[G], o[G][8];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            m[h] = -INFINITY;
+            l[h] = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[h][e] = 0.f;
+        }
+        bool filled = false;
+        // Half-warp hw takes keys [4 hw, 4 hw + 4) of each block: four consecutive rows.
+        for (int i = 0; i < nb; ++i, ++gc) {
+            const int sl = gc % kAttnSlots;
+            ok = ok && mbar_wait(bar(kAB_FULL + sl), (gc / kAttnSlots) & 1, abort_flag, a.status);
+            const int t = list[i];
+            const int rows = t == qb ? p - t * kM + 1 : kM;
+            const uint8_t* ks = smem + sl * 2 * kSlotBytes;
+            const uint8_t* vs = ks + kSlotBytes;
+            // scores first, then the values: K and V fragments are not live together
+            bool vis[4];
+            float sc4[G][4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int key = 4 * hw + r;
+                vis[r] = ok && key < rows;
+                const uint4 kr = vis[r] ? *reinterpret_cast<const uint4*>(ks + key * kRowBytes + c16 * 16)
+                                        : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    // dot8_half shuffles across the whole warp: call it on every lane
+                    // (a masked key holds zeros), then mask the score
+                    const float d = dot8_half(qv[h], kr);
+                    sc4[h][r] = vis[r] ? d : -INFINITY;
+                }
+            }
+            uint4 vr[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+                vr[r] = vis[r] ? *reinterpret_cast<const uint4*>(vs + (4 * hw + r) * kRowBytes + c16 * 16)
+                               : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                const float* s = sc4[h];
+                float mn = m[h];
+#pragma unroll
+                for (int r = 0; r < 4; ++r) mn = fmaxf(mn, s[r]);
+                if (mn == -INFINITY) continue;  // no key of this step is visible
+                const float sc = ex2_approx(m[h] - mn);
+                l[h] *= sc;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) o[h][e] *= sc;
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    const float pr = ex2_approx(s[r] - mn);
+                    l[h] += pr;
+                    const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&vr[r]);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float2 f = __bfloat1622float2(v2[j]);
+                        o[h][2 * j] = fmaf(pr, f.x, o[h][2 * j]);
+                        o[h][2 * j + 1] = fmaf(pr, f.y, o[h][2 * j + 1]);
+                    }
+                }
+                m[h] = mn;
+            }
+            if (fill && t == qb && ok && warp < 4) {
+                // Eq. 6-8 over the 64 rows in the slot, in the summation order of
+                // decode_repr_kernel: warp w rows [16w, 16w + 16), even and odd rows
+                // per lane half, halves added, then the warps in order
+                const int half = lane >> 4, col = lane & 15;
+                float s0[8], sp[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    s0[j] = 0.f;
+                    sp[j] = 0.f;
+                }
+#pragma unroll
+                for (int uu = 0; uu < 8; ++uu) {
+                    const int r = 16 * warp + 2 * uu + half;
+                    const uint4 kv = *reinterpret_cast<const uint4*>(ks + r * kRowBytes + col * 16);
+                    const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
+                    const bool pu = ((r < 32 ? plo >> r : phi >> (r - 32)) & 1u) != 0;
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float2 f = __bfloat1622float2(h2[j]);
+                        s0[2 * j] += f.x;
+                        s0[2 * j + 1] += f.y;
+                        if (pu) {
+                            sp[2 * j] += f.x;
+                            sp[2 * j + 1] += f.y;
+                        }
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    s0[j] += __shfl_xor_sync(0xffffffffu, s0[j], 16);
+                    sp[j] += __shfl_xor_sync(0xffffffffu, sp[j], 16);
+                }
+                if (half == 0) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        rpart[(warp * 2 + 0) * kD + col * 8 + j] = s0[j];
+                        rpart[(warp * 2 + 1) * kD + col * 8 + j] = sp[j];
+                    }
+                }
+                filled = true;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kAB_EMPTY + sl));  // this warp is done with the slot
+        }
+
+        // ---- merge: the two half-warps of a warp with shuffles, then the 8 warps
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            const float mo = __shfl_xor_sync(0xffffffffu, m[h], 16);
+            const float lo2 = __shfl_xor_sync(0xffffffffu, l[h], 16);
+            const float M2 = fmaxf(m[h], mo);
+            const float fa = M2 == -INFINITY ? 0.f : ex2_approx(m[h] - M2);
+            const float fb = M2 == -INFINITY ? 0.f : ex2_approx(mo - M2);
+            l[h] = l[h] * fa + lo2 * fb;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const float oo = __shfl_xor_sync(0xffffffffu, o[h][e], 16);
+                o[h][e] = o[h][e] * fa + oo * fb;
+            }
+            float* st = part + ((size_t)warp * G + h) * 130;
+            if (lane == 0) {
+                st[0] = M2;
+                st[1] = l[h];
+            }
+            if (lane < 16) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) st[2 + c16 * 8 + e] = o[h][e];
+            }
+        }
+        filled = named_barrier_and(1, kThreads, !filled) == false;  // part and rpart complete
+        if (ok && tid < G * kD) {
+            const int h = tid / kD, d = tid % kD;
+            float M = -INFINITY;
+            for (int w = 0; w < kWarps; ++w) M = fmaxf(M, part[((size_t)w * G + h) * 130]);
+            float Ls = 0.f, acc = 0.f;
+            if (M != -INFINITY) {
+                for (int w = 0; w < kWarps; ++w) {
+                    const float* st = part + ((size_t)w * G + h) * 130;
+                    const float f = ex2_approx(st[0] - M);  // 0 for a warp that saw no key
+                    Ls += st[1] * f;
+                    acc += st[2 + d] * f;
+                }
+            }
+            a.O[(orow + h) * kD + d] = __float2bfloat16_rn(Ls > 0.f ? acc / Ls : 0.f);
+            if (d == 0) a.lse[orow + h] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
+        }
+        if (ok && filled && tid < kD) {
+            float a0 = 0.f, ap = 0.f;
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                a0 += rpart[(w * 2 + 0) * kD + tid];
+                ap += rpart[(w * 2 + 1) * kD + tid];
+            }
+            const int c = __popc(plo) + __popc(phi);
+            const float m0 = a0 * (1.0f / kM);  // Eq. 6
+            const float ov = c > 0 ? a.lambda * m0 + (1.0f - a.lambda) * (ap * (1.0f / (float)c))
+                                   : m0;  // Eq. 7-8; no punctuation: the mean
+            a.Krepr[((size_t)u * a.T + qb) * kD + tid] = __float2bfloat16_rn(ov);
+        }
+        // the unit slot is no longer read; part and rpart are written again only
+        // after the next unit's barrier
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(kAB_UFREE + us));
     }
+}
+
+// Persistent grid: one CTA per unit if they all fit at once, else as many
+// CTAs as the device holds.
+template <class Kern>
+cudaError_t persistent_grid(Kern kern, int threads, size_t smem, long long units, unsigned& grid) {
+    int dev = 0, nsm = 0, per_sm = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    // as much shared memory as the SM has, so that several CTAs fit
+    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100)) !=
+        cudaSuccess)
+        return e;
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem)) !=
+        cudaSuccess)
+        return e;
+    const long long cap = (long long)nsm * (per_sm > 0 ? per_sm : 1);
+    grid = (unsigned)(units < cap ? units : cap);
+    return cudaSuccess;
+}
+
+cudaError_t launch_decode_attn_any(const void* q, const void* K, const void* V, const int32_t* idx,
+                                   const int32_t* cnt, const int32_t* lens, const phsa_shape& s,
+                                   int topk, float sm_scale, void* O, float* lse,
+                                   const uint8_t* mask, float lambda, void* Krepr, int* status,
+                                   cudaStream_t st) {
+    const int G = s.Hq / s.Hkv;
+    const size_t smem = dec_attn_smem(G, topk);
+    const long long units = (long long)s.B * s.Hkv;
+    DecAttnArgs args{static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(K),
+                     static_cast<const __nv_bfloat16*>(V), idx, cnt, lens,
+                     static_cast<__nv_bfloat16*>(O), lse, status, mask,
+                     static_cast<__nv_bfloat16*>(Krepr), lambda, s.Hq, s.Hkv, s.L, s.L / kM, topk,
+                     (int)units, sm_scale * kLog2e};
+    auto kern = G == 2 ? decode_attn_kernel<2> : decode_attn_kernel<1>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    unsigned grid = 0;
+    if ((e = persistent_grid(kern, kAttnThreads, smem, units, grid)) != cudaSuccess) return e;
+    ProfScope prof(K_DEC_ATTN, st);
+    kern<<<grid, kAttnThreads, smem, st>>>(args);
+    return cudaGetLastError();
 }
 
 }  // namespace
 
 size_t decode_select_smem_bytes(const phsa_shape& s, int topk) {
-    return dec_select_smem(s.Hq / s.Hkv, s.L / kM, topk);
+    const int G = s.Hq / s.Hkv, Tc = s.L / kM;
+    const int n = dec_select_slots(G, Tc, topk, 1);
+    return n > 0 ? dec_select_smem(G, Tc, topk, n) : (size_t)-1;
+}
+
+size_t decode_attn_smem_bytes(const phsa_shape& s, int topk) {
+    return dec_attn_smem(s.Hq / s.Hkv, topk);
 }
 
 cudaError_t launch_decode_select(const void* q, const void* Krepr, const int32_t* lens,
                                  const phsa_shape& s, const phsa_select_params& p, int32_t* idx,
                                  int32_t* cnt, int* status, cudaStream_t st) {
     const int G = s.Hq / s.Hkv, Tc = s.L / kM;
-    const size_t smem = dec_select_smem(G, Tc, p.topk);
+    const long long units = (long long)s.B * s.Hkv;
+    int dev = 0, nsm = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    // two CTAs per SM once there are units for them (their unit phases overlap),
+    // the ring as deep as that leaves room for
+    const int per_sm = units > nsm ? 2 : 1;
+    int slots = dec_select_slots(G, Tc, p.topk, per_sm);
+    if (slots == 0) slots = dec_select_slots(G, Tc, p.topk, 1);
+    const size_t smem = dec_select_smem(G, Tc, p.topk, slots);
     DecSelArgs args{static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(Krepr),
                     lens, idx, cnt, status, s.Hq, s.Hkv, s.L, Tc, p.topk, p.n_init, p.n_local,
-                    p.sm_scale * kLog2e};
-    const unsigned grid = (unsigned)((long long)s.B * s.Hkv);
+                    (int)units, slots, p.sm_scale * kLog2e};
     auto kern = G == 2 ? decode_select_kernel<2> : decode_select_kernel<1>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
+    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
+        cudaSuccess)
+        return e;
+    unsigned grid = 0;
+    if ((e = persistent_grid(kern, kSelThreads, smem, units, grid)) != cudaSuccess) return e;
     ProfScope prof(K_DEC_SELECT, st);
-    kern<<<grid, kThreads, smem, st>>>(args);
+    kern<<<grid, kSelThreads, smem, st>>>(args);
     return cudaGetLastError();
 }
 
@@ -366,19 +1000,17 @@ cudaError_t launch_decode_attn(const void* q, const void* K, const void* V, cons
                                const int32_t* cnt, const int32_t* lens, const phsa_shape& s,
                                int topk, float sm_scale, void* O, float* lse, int* status,
                                cudaStream_t st) {
-    const int G = s.Hq / s.Hkv;
-    const size_t smem = dec_attn_smem(G, topk);
-    DecAttnArgs args{static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(K),
-                     static_cast<const __nv_bfloat16*>(V), idx, cnt, lens,
-                     static_cast<__nv_bfloat16*>(O), lse, status, s.Hq, s.Hkv, s.L, topk,
-                     sm_scale * kLog2e};
-    const unsigned grid = (unsigned)((long long)s.B * s.Hkv);
-    auto kern = G == 2 ? decode_attn_kernel<2> : decode_attn_kernel<1>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    ProfScope prof(K_DEC_ATTN, st);
-    kern<<<grid, kThreads, smem, st>>>(args);
-    return cudaGetLastError();
+    return launch_decode_attn_any(q, K, V, idx, cnt, lens, s, topk, sm_scale, O, lse, nullptr, 0.f,
+                                  nullptr, status, st);
+}
+
+cudaError_t launch_decode_attn_repr(const void* q, const void* K, const void* V,
+                                    const int32_t* idx, const int32_t* cnt, const int32_t* lens,
+                                    const phsa_shape& s, int topk, float sm_scale, void* O,
+                                    float* lse, const uint8_t* mask, float lambda, void* Krepr,
+                                    int* status, cudaStream_t st) {
+    return launch_decode_attn_any(q, K, V, idx, cnt, lens, s, topk, sm_scale, O, lse, mask, lambda,
+                                  Krepr, status, st);
 }
 
 }  // namespace phsa

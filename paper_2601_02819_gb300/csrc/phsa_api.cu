@@ -188,11 +188,42 @@ int phsa_decode_attn(const void* q, const void* K, const void* V, const int32_t*
         return PHSA_ERR_INVALID_ARG;
     if (!aligned16(q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
         return PHSA_ERR_INVALID_ARG;
+    if (phsa::decode_attn_smem_bytes(s, topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
     int* st = status_ptr();
     if (!st) return PHSA_ERR_CUDA;
     return from_cuda(phsa::launch_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, s, topk,
                                               sm_scale, O, lse, st,
                                               static_cast<cudaStream_t>(stream)));
+}
+
+int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t* punct_mask,
+                     const int32_t* seq_lens, phsa_shape s, float lambda, phsa_select_params p,
+                     void* Krepr, int32_t* block_idx, int32_t* block_cnt, void* O, float* lse,
+                     void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
+    if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
+    if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
+    if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
+    if (s.B == 0) return PHSA_OK;
+    if (!q || !K || !V || !punct_mask || !seq_lens || !block_idx || !block_cnt || !O || !lse ||
+        (s.L >= phsa::kM && !Krepr))
+        return PHSA_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(K) || !aligned16(V) || !aligned16(O) ||
+        (Krepr && !aligned16(Krepr)))
+        return PHSA_ERR_INVALID_ARG;
+    if (phsa::decode_select_smem_bytes(s, p.topk) > 227 * 1024 ||
+        phsa::decode_attn_smem_bytes(s, p.topk) > 227 * 1024)
+        return PHSA_ERR_UNSUPPORTED;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    cudaError_t e = phsa::launch_decode_select(q, Krepr, seq_lens, s, p, block_idx, block_cnt, st, cs);
+    if (e != cudaSuccess) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_decode_attn_repr(q, K, V, block_idx, block_cnt, seq_lens, s,
+                                                   p.topk, p.sm_scale, O, lse, punct_mask, lambda,
+                                                   s.L >= phsa::kM ? Krepr : nullptr, st, cs));
 }
 
 int phsa_get_device_status(void* stream) {

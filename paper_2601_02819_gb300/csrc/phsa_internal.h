@@ -43,6 +43,14 @@ cudaError_t launch_decode_attn(const void* q, const void* K, const void* V, cons
                                const int32_t* cnt, const int32_t* lens, const phsa_shape& s,
                                int topk, float sm_scale, void* O, float* lse, int* status,
                                cudaStream_t st);
+// The attention above, also refreshing the representative key of every block
+// the new token has just filled (the work of launch_decode_repr).
+cudaError_t launch_decode_attn_repr(const void* q, const void* K, const void* V,
+                                    const int32_t* idx, const int32_t* cnt, const int32_t* lens,
+                                    const phsa_shape& s, int topk, float sm_scale, void* O,
+                                    float* lse, const uint8_t* mask, float lambda, void* Krepr,
+                                    int* status, cudaStream_t st);
+size_t decode_attn_smem_bytes(const phsa_shape& s, int topk);
 
 cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape& s,
                              const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,

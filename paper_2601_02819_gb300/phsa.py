@@ -85,6 +85,9 @@ def _declare(L):
     L.phsa_step_host.restype = I
     L.phsa_step_host_release.argtypes = [P]
     L.phsa_step_host_release.restype = I
+    L.phsa_decode_step.argtypes = [P, P, P, P, P, phsa_shape, F, phsa_select_params, P, P, P, P,
+                                   P, P]
+    L.phsa_decode_step.restype = I
     L.phsa_decode_update_repr.argtypes = [P, P, P, phsa_shape, F, P, P]
     L.phsa_decode_select.argtypes = [P, P, P, phsa_shape, phsa_select_params, P, P, P]
     L.phsa_decode_attn.argtypes = [P, P, P, P, P, P, phsa_shape, I, F, P, P, P]
@@ -398,6 +401,41 @@ def phsa_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, sm_scale: float | 
                                  _stream(stream))
     _raise("phsa_decode_attn", rc)
     return O, lse
+
+
+def phsa_decode_step(q, K, V, punct_mask, seq_lens, lam: float, Krepr, topk: int,
+                     n_init: int = 1, n_local: int = 1, sm_scale: float | None = None,
+                     block_idx=None, block_cnt=None, O=None, lse=None, stream=None):
+    """One decode step in two launches (selection; attention fused with the
+    refresh of the blocks the new tokens have just filled). q [B, Hq, D], K/V
+    [B, Hkv, Lc, D] bf16 caches, punct_mask [B, Lc] uint8, seq_lens [B] int32,
+    Krepr [B, Hkv, Lc // 64, D] (read, and updated in place).
+    Returns (block_idx, block_cnt, O, lse)."""
+    _check(q, "q", torch.bfloat16, 3)
+    _check(K, "K", torch.bfloat16, 4)
+    _check(V, "V", torch.bfloat16, 4)
+    _check(punct_mask, "punct_mask", torch.uint8, 2)
+    _check(seq_lens, "seq_lens", torch.int32, 1)
+    _check(Krepr, "Krepr", torch.bfloat16, 4)
+    B, Hq, D = q.shape
+    Hkv, Lc = K.shape[1], K.shape[2]
+    if sm_scale is None:
+        sm_scale = D ** -0.5
+    if block_idx is None:
+        block_idx = torch.empty((B, Hkv, topk), dtype=torch.int32, device=q.device)
+    if block_cnt is None:
+        block_cnt = torch.empty((B, Hkv), dtype=torch.int32, device=q.device)
+    if O is None:
+        O = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device)
+    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    rc = load().phsa_decode_step(_ptr(q), _ptr(K), _ptr(V), _ptr(punct_mask), _ptr(seq_lens),
+                                 make_shape(B, Lc, Hq, Hkv, D), float(lam), p, _ptr(Krepr),
+                                 _ptr(block_idx), _ptr(block_cnt), _ptr(O), _ptr(lse),
+                                 _stream(stream))
+    _raise("phsa_decode_step", rc)
+    return block_idx, block_cnt, O, lse
 
 
 def phsa_get_device_status(stream=None) -> int:

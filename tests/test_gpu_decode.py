@@ -151,3 +151,35 @@ def test_decode_workload_full_size_sampled():
         assert_close(f"O ({b},{g})", bf16_to_f64(O[b:b + 1, 2 * g:2 * g + 2]), Or)
         assert np.abs(lse[b, 2 * g:2 * g + 2].cpu().numpy() - lr[0]).max() <= LSE_ABS
     assert agree >= len(units) - 2
+
+
+@pytest.mark.parametrize("Hq,Hkv,n_init,n_local,topk", [(4, 2, 1, 1, 6), (2, 2, 2, 3, 9)])
+def test_decode_step_equals_the_three_calls(Hq, Hkv, n_init, n_local, topk):
+    # The fused step (selection; attention with the refresh of just-filled blocks)
+    # must reproduce update_repr -> select -> attn bit for bit, over appends that
+    # fill blocks at different steps for different sequences.
+    B, Lc = 5, 64 * 12
+    rng = np.random.default_rng(11 + Hq)
+    f = lambda *s: inputs.f32_to_bf16_bits(rng.standard_normal(s).astype(np.float32))
+    K, V = f(B, Hkv, Lc, D), f(B, Hkv, Lc, D)
+    mask = (rng.random((B, Lc)) < 0.1).astype(np.uint8)
+    lens = np.array([64 * 3 - 2, 64 * 5 - 1, 64 * 2, 1, 64 * 7 - 3], np.int32)
+    Kd, Vd, md = to_dev_bf16(K), to_dev_bf16(V), torch.from_numpy(mask).cuda()
+    Kr_a = phsa.phsa_build_block_repr(Kd, md, 0.5)
+    for b in range(B):  # blocks not yet filled hold nothing
+        Kr_a[b, :, lens[b] // M:] = 0
+    Kr_b = Kr_a.clone()
+    for step in range(6):
+        lens += 1
+        q = to_dev_bf16(f(B, Hq, D))
+        ld = torch.from_numpy(lens).cuda()
+        phsa.phsa_decode_update_repr(Kd, md, ld, 0.5, Kr_a)
+        ia, ca = phsa.phsa_decode_select(q, Kr_a, ld, Lc, topk, n_init, n_local)
+        Oa, la = phsa.phsa_decode_attn(q, Kd, Vd, ia, ca, ld)
+        ib, cb, Ob, lb = phsa.phsa_decode_step(q, Kd, Vd, md, ld, 0.5, Kr_b, topk, n_init, n_local)
+        torch.cuda.synchronize()
+        assert torch.equal(ia, ib) and torch.equal(ca, cb), step
+        assert torch.equal(Oa.view(torch.int16), Ob.view(torch.int16)), step
+        assert torch.equal(la, lb), step
+        assert torch.equal(Kr_a.view(torch.int16), Kr_b.view(torch.int16)), step
+    assert phsa.phsa_get_device_status() == 0
