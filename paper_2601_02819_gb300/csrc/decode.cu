@@ -1,36 +1,28 @@
-// Decode: one new token per sequence. The newest token of sequence b (position
-// p = len_b - 1) is the query; the selection rule of Section 3.3 (Algorithm 1
-// step 3) is applied to the unit whose rows are that token in each of the
-// GQA group's G query heads, and Eq. 10-11 to the token's row. The block
-// representations are cached and updated as blocks fill (Section 3.2).
+// Decode attention: one new token per sequence. The newest token of sequence b
+// (position p = len_b - 1) attends, in each of the GQA group's G query heads,
+// the blocks the selection chose for it (Eq. 10-11 for one row); the
+// selection itself is in decode_select_tc.cu.
 //
-// Both kernels read little per unit and are bound by HBM bandwidth, so they
-// run on the CUDA cores. What a unit (sequence, KV head) reads is contiguous
-// in memory -- its candidates' representative keys are consecutive rows of
-// Krepr, every selected K or V block is 64 consecutive rows -- so one thread
-// streams it into a shared-memory ring with 1-D bulk copies (cp.async.bulk,
-// completion counted on an mbarrier per slot) and the warps compute from
-// shared memory: a half-warp per 256-byte key row (lane c holds columns
-// 8c..8c+7). Both kernels are persistent: a CTA walks the units u =
-// blockIdx.x, blockIdx.x + gridDim.x, ..., and its ring runs across unit
-// boundaries, so the next unit's rows are in flight while a unit finishes.
-// After each slot is consumed the CTA synchronises (agreeing on any abort)
-// and the slot is refilled.
+// The kernel reads little per unit (sequence, KV head) and is bound by HBM
+// bandwidth, so it runs on the CUDA cores. Every selected K or V block is 64
+// consecutive rows, so a producer warp streams them into a shared-memory ring
+// with 1-D bulk copies (cp.async.bulk, completion counted on an mbarrier per
+// slot) and the compute warps work from shared memory: a half-warp per
+// 256-byte key row (lane c holds columns 8c..8c+7). The kernel is persistent:
+// a CTA walks the units u = blockIdx.x, blockIdx.x + gridDim.x, ..., and its
+// ring runs across unit boundaries, so the next unit's blocks are in flight
+// while a unit finishes.
 //
-// decode_select_kernel  S[h][t] = q_h . Krepr_t for the candidates, per head
-//   the softmax over candidates (max, sum), A_t = sum over heads of the
-//   probabilities (head order), then the top-k of topk.cuh.
-// decode_attn_kernel  each half-warp runs an online softmax over 4 keys of
-//   every selected block; the 16 partial states are merged (two per warp with
-//   shuffles, then the 8 warps in shared memory). Keys after p (the unfilled
-//   part of the local block) are neither copied nor attended. Optionally it
-//   also refreshes the representative key of the block the new token has just
-//   filled: that block is the query's own (local) block, which the kernel
-//   copies anyway, and it is never a candidate of the same step.
+// Each half-warp runs an online softmax over 4 keys of every selected block;
+// the 16 partial states are merged (two per warp with shuffles, then the 8
+// warps in shared memory). Keys after p (the unfilled part of the local block)
+// are neither copied nor attended. Optionally the kernel also refreshes the
+// representative key of the block the new token has just filled: that block
+// is the query's own (local) block, which the kernel copies anyway, and it is
+// never a candidate of the same step.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "tc_common.cuh"
-#include "topk.cuh"
 
 namespace phsa {
 
@@ -43,8 +35,6 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kRowBytes = kD * 2;                  // one bf16 key row
 constexpr int kSlotRows = 64;                      // rows per ring slot (one block)
 constexpr int kSlotBytes = kSlotRows * kRowBytes;  // 16 KB
-constexpr int kSelSlotsMax = 12;  // selection ring: up to 192 KB (one CTA per SM), fewer when
-                                  // the scores of a long context need the room
 constexpr int kAttnSlots = 3;                      // attention ring: 3 x (K, V) = 96 KB
 
 // Dot product of a 16-byte piece of a bf16 row with 8 fp32 values, added over
@@ -62,440 +52,6 @@ __device__ __forceinline__ float dot8_half(const float* q, const uint4& k) {
 #pragma unroll
     for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
     return acc;
-}
-
-// ============================================================== selection
-struct DecSelArgs {
-    const __nv_bfloat16* q;
-    const __nv_bfloat16* Kr;
-    const int32_t* lens;
-    int32_t* idx;
-    int32_t* cnt;
-    int* status;
-    int Hq, Hkv, L, Tc, topk, n_init, n_local, units, slots;
-    float scale_log2;
-};
-
-// What one (sequence, KV head) unit asks of the selection. mode 0: no query
-// (length 0, or a bad length); 1: the budget covers every candidate; 2: scored.
-struct SelUnit {
-    int qb, n_init_q, loc_lo, c_lo, nC, nF, ksel, mode;
-};
-
-__device__ __forceinline__ SelUnit sel_unit(const DecSelArgs& a, int len) {
-    SelUnit s{};
-    if (len <= 0 || len > a.L) return s;
-    s.qb = (len - 1) / kM;
-    s.n_init_q = min(a.n_init, s.qb + 1);              // forced initial [0, n_init_q)
-    s.loc_lo = max(s.n_init_q, s.qb - a.n_local + 1);  // forced local [loc_lo, qb]
-    s.c_lo = a.n_init;                                 // candidates [c_lo, qb - n_local]
-    s.nC = max(0, s.qb - a.n_local - s.c_lo + 1);
-    s.nF = s.n_init_q + (s.qb - s.loc_lo + 1);
-    s.ksel = a.topk - s.nF;
-    s.mode = s.ksel >= s.nC ? 1 : 2;
-    return s;
-}
-
-__device__ __forceinline__ int sel_chunks(const SelUnit& s) {
-    return s.mode == 2 ? (s.nC + kSlotRows - 1) / kSlotRows : 0;
-}
-
-// Reduction of one float per thread (max or sum) over the 8 compute warps,
-// synchronised by named barrier 1 (the producer warp does not take part).
-template <bool kMax>
-__device__ __forceinline__ float warps_reduce(float v, float* red) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-        const float o = __shfl_xor_sync(0xffffffffu, v, off);
-        v = kMax ? fmaxf(v, o) : v + o;
-    }
-    named_barrier(1, kThreads);  // red may still be read from a previous reduction
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
-    named_barrier(1, kThreads);
-    float r = red[0];
-#pragma unroll
-    for (int w = 1; w < kWarps; ++w) r = kMax ? fmaxf(r, red[w]) : r + red[w];
-    return r;
-}
-
-// Roles: warps 0-7 score the candidates, warp 8 stages each unit (its length
-// and the G query rows) into a unit slot and streams the candidates'
-// representative keys through the ring, 64 rows per slot, and warp 9 takes the
-// top-k of a unit while warps 0-7 score the next one. The scores and each
-// head's softmax statistics (running max and sum, kept online while scoring)
-// are double-buffered between the scoring warps and the top-k warp.
-constexpr int kSelThreads = 320;
-constexpr int kSelRegKeys = 16;  // candidate keys per lane kept in registers by the top-k warp
-constexpr int kSelUnitSlots = 3;
-constexpr int kSB_FULL = 0, kSB_EMPTY = kSelSlotsMax, kSB_UFULL = 2 * kSelSlotsMax,
-              kSB_UFREE = kSB_UFULL + kSelUnitSlots, kSB_AFULL = kSB_UFREE + kSelUnitSlots,
-              kSB_AFREE = kSB_AFULL + 2, kSelBars = kSB_AFREE + 2;
-constexpr int kSelBarBytes = (8 * kSelBars + 4 + 127) / 128 * 128;  // + abort flag
-static_assert(kSelBarBytes >= 8 * kSelBars + 4, "barriers and abort flag fit");
-// unit slot: {len, -, -, -} | q bf16 [G][128]
-__host__ __device__ constexpr int sel_unit_bytes(int G) { return 16 + G * kD * 2; }
-// Shared memory: ring [slots][16 KB] | barriers | unit slots | per-warp
-// statistics [8][G][2] | score buffers [2]{header {unit, len, -, -}, max [G],
-// 1/sum [G], S [G][Tc] (scores, log2 units)} | picks [topk].
-__host__ __device__ constexpr int sel_sbuf_floats(int G, int Tc) { return 4 + 2 * G + G * Tc; }
-size_t dec_select_fixed_smem(int G, int Tc, int topk) {
-    return (size_t)kSelBarBytes + (size_t)kSelUnitSlots * sel_unit_bytes(G) +
-           (size_t)kWarps * G * 2 * 4 + 2 * (size_t)sel_sbuf_floats(G, Tc) * 4 +
-           (size_t)topk * 4 + 16;
-}
-// ring slots that fit beside the rest when per_sm CTAs share an SM's 228 KB
-// (0 if not even two)
-int dec_select_slots(int G, int Tc, int topk, int per_sm) {
-    const size_t fixed = dec_select_fixed_smem(G, Tc, topk);
-    const size_t cap = per_sm <= 1 ? 227 * 1024 : 228 * 1024 / per_sm - 2 * 1024;
-    size_t fit = fixed >= cap ? 0 : (cap - fixed) / kSlotBytes;
-    if (fit > (size_t)kSelSlotsMax) fit = kSelSlotsMax;
-    const int n = (int)fit;
-    return n >= 2 ? n : 0;
-}
-size_t dec_select_smem(int G, int Tc, int topk, int slots) {
-    return (size_t)(slots > 0 ? slots : 2) * kSlotBytes + dec_select_fixed_smem(G, Tc, topk);
-}
-
-template <int G>
-__global__ void __launch_bounds__(kSelThreads, 2)
-decode_select_kernel(const DecSelArgs a) {
-    extern __shared__ __align__(128) uint8_t smem[];
-    const uint32_t sb = smem_u32(smem);
-    const int nslots = a.slots, off_bar = nslots * kSlotBytes;
-    auto bar = [&](int i) { return sb + off_bar + 8u * (uint32_t)i; };
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + off_bar + 8 * kSelBars);
-    uint8_t* units0 = smem + off_bar + kSelBarBytes;
-    float* wstat = reinterpret_cast<float*>(units0 + kSelUnitSlots * sel_unit_bytes(G));  // [8][G][2]
-    float* sbuf0 = wstat + kWarps * G * 2;                       // [2][sel_sbuf_floats]
-    const int sbuf_floats = sel_sbuf_floats(G, a.Tc);
-    int* sel = reinterpret_cast<int*>(sbuf0 + 2 * sbuf_floats);  // [topk]
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    auto unit_of = [&](int k) { return (int)blockIdx.x + k * (int)gridDim.x; };
-
-    if (tid == 0) {
-        for (int i = 0; i < nslots; ++i) {
-            mbar_init(bar(kSB_FULL + i), 1);
-            mbar_init(bar(kSB_EMPTY + i), kWarps);
-        }
-        for (int i = 0; i < kSelUnitSlots; ++i) {
-            mbar_init(bar(kSB_UFULL + i), 1);
-            mbar_init(bar(kSB_UFREE + i), kWarps);
-        }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(bar(kSB_AFULL + i), 1);
-            mbar_init(bar(kSB_AFREE + i), 1);
-        }
-        fence_barrier_init();
-        *abort_flag = 0;
-    }
-    __syncthreads();
-
-    if (warp == kWarps) {
-        // ------------------------------------------------ producer
-        bool ok = true;
-        int issued = 0, staged = -1, ik = 0, ic = 0;  // copies; last unit staged; cursor
-        Deadline dl;
-        while (ok) {
-            bool progressed = false;
-            const bool more = unit_of(ik) < a.units;
-            if (more && ik <= staged) {
-                const int len = *reinterpret_cast<const int*>(units0 + (ik % kSelUnitSlots) *
-                                                                           sel_unit_bytes(G));
-                const SelUnit su = sel_unit(a, len);
-                if (ic >= sel_chunks(su)) {
-                    ++ik;
-                    ic = 0;
-                    continue;
-                }
-                const int sl = issued % nslots;
-                bool free_slot = issued < nslots;
-                if (!free_slot && lane == 0)
-                    free_slot = mbar_test_wait(bar(kSB_EMPTY + sl), ((issued / nslots) - 1) & 1);
-                if (__shfl_sync(0xffffffffu, free_slot, 0)) {
-                    if (lane == 0) {
-                        const uint32_t bytes =
-                            (uint32_t)min(kSlotRows, su.nC - ic * kSlotRows) * kRowBytes;
-                        const __nv_bfloat16* src =
-                            a.Kr + ((size_t)unit_of(ik) * a.Tc + su.c_lo + (size_t)ic * kSlotRows) * kD;
-                        mbar_expect_tx(bar(kSB_FULL + sl), bytes);
-                        bulk_load(sb + sl * kSlotBytes, src, bytes, bar(kSB_FULL + sl));
-                    }
-                    ++issued;
-                    ++ic;
-                    progressed = true;
-                }
-            }
-            const int ks = staged + 1;
-            if (!progressed && unit_of(ks) < a.units && ks <= ik + 2) {
-                bool free_unit = ks < kSelUnitSlots;
-                if (!free_unit && lane == 0)
-                    free_unit = mbar_test_wait(bar(kSB_UFREE + ks % kSelUnitSlots),
-                                               ((ks / kSelUnitSlots) - 1) & 1);
-                if (__shfl_sync(0xffffffffu, free_unit, 0)) {
-                    // stage unit ks: its length and the group's query rows
-                    const int u = unit_of(ks), b = u / a.Hkv, g = u % a.Hkv;
-                    uint8_t* slot = units0 + (ks % kSelUnitSlots) * sel_unit_bytes(G);
-                    if (lane < G * 16)
-                        reinterpret_cast<uint4*>(slot + 16)[lane] = __ldg(
-                            reinterpret_cast<const uint4*>(a.q + ((size_t)b * a.Hq + g * G) * kD) + lane);
-                    if (lane == 0) *reinterpret_cast<int*>(slot) = __ldg(a.lens + b);
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(bar(kSB_UFULL + ks % kSelUnitSlots));
-                    staged = ks;
-                    progressed = true;
-                }
-            }
-            if (!more && unit_of(staged + 1) >= a.units) break;  // every copy issued
-            if (progressed) {
-                dl.reset();
-            } else {
-                __nanosleep(64);  // nothing to do yet: leave the issue slots to the other warps
-                if (*abort_flag) {
-                    ok = false;
-                } else if (dl.expired()) {
-                    *abort_flag = 1;
-                    if (lane == 0) atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
-                    ok = false;
-                }
-            }
-            ok = __all_sync(0xffffffffu, ok) != 0;
-        }
-        if (lane == 0)  // own copies land before the CTA may exit
-            for (int j = max(0, issued - nslots); j < issued; ++j)
-                mbar_wait_drain(bar(kSB_FULL + j % nslots), (j / nslots) & 1);
-        return;
-    }
-
-    if (warp == kWarps + 1) {
-        // ------------------------------------------------ top-k (one warp)
-        bool ok = true;
-        for (int su = 0; ok; ++su) {
-            const int buf = su & 1;
-            ok = mbar_wait(bar(kSB_AFULL + buf), (su >> 1) & 1, abort_flag, a.status);
-            ok = __all_sync(0xffffffffu, ok) != 0;
-            if (!ok) break;
-            float* sbuf = sbuf0 + buf * sbuf_floats;
-            const int u = reinterpret_cast<const int*>(sbuf)[0];
-            if (u < 0) break;  // the end of the CTA's units
-            const SelUnit d = sel_unit(a, reinterpret_cast<const int*>(sbuf)[1]);
-            const float* mx = sbuf + 4;
-            const float* iz = mx + G;
-            float* Sb = sbuf + 4 + 2 * G;
-            const int nC = d.nC, ksel = d.ksel, c_lo = d.c_lo;
-            // A_t = sum over the heads of the head's softmax probability, head order
-            auto key_of = [&](int cj) {
-                float acc = 0.f;
-#pragma unroll
-                for (int h = 0; h < G; ++h) acc += ex2_approx(Sb[h * a.Tc + cj] - mx[h]) * iz[h];
-                return topk::make_key(acc, c_lo + cj);
-            };
-            if (nC <= 32 * kSelRegKeys) {
-                unsigned long long key[kSelRegKeys];
-#pragma unroll
-                for (int rr = 0; rr < kSelRegKeys; ++rr) {
-                    const int cj = lane + 32 * rr;
-                    key[rr] = cj < nC ? key_of(cj) : 0ull;
-                }
-                for (int kk = 0; kk < ksel; ++kk) {
-                    unsigned long long best = key[0];
-#pragma unroll
-                    for (int rr = 1; rr < kSelRegKeys; ++rr) best = topk::umax64(best, key[rr]);
-                    const unsigned mh = (unsigned)(best >> 32), ml = (unsigned)best;
-                    const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
-                    const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
-                    const unsigned long long win = ((unsigned long long)bh << 32) | bl;
-                    if (lane == 0) sel[kk] = topk::key_block(win);
-#pragma unroll
-                    for (int rr = 0; rr < kSelRegKeys; ++rr)
-                        if (key[rr] == win) key[rr] = 0ull;
-                }
-            } else {  // long contexts: rounds over shared memory; a pick is marked by a NaN score
-                topk::rounds_one_warp(
-                    nC, ksel, key_of, [&](int cj) { return Sb[cj] != Sb[cj]; },
-                    [&](int t) { Sb[t - c_lo] = __int_as_float(0x7fc00000); }, sel, lane);
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kSB_AFREE + buf));  // the scoring warps may refill it
-            int32_t* out = a.idx + (size_t)u * a.topk;
-            for (int j = lane; j < a.topk; j += 32) {
-                if (j < d.n_init_q) out[j] = j;
-                else if (j >= d.n_init_q + ksel && j < d.nF + ksel)
-                    out[j] = d.loc_lo + (j - d.n_init_q - ksel);
-                else if (j >= d.nF + ksel) out[j] = -1;
-            }
-            for (int j = lane; j < ksel; j += 32) {
-                const int v = sel[j];
-                int rank = 0;
-                for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
-                out[d.n_init_q + rank] = v;
-            }
-            if (lane == 0) a.cnt[u] = d.nF + ksel;
-            __syncwarp();  // sel is reused by the next unit
-        }
-        return;
-    }
-
-    // ---------------------------------------------------- compute (warps 0-7)
-    int gc = 0, su = 0;  // chunks consumed; units scored
-    bool ok = true;
-    for (int k = 0;; ++k) {
-        const int u = unit_of(k);
-        if (u >= a.units) break;
-        const int us = k % kSelUnitSlots;
-        ok = ok && mbar_wait(bar(kSB_UFULL + us), (k / kSelUnitSlots) & 1, abort_flag, a.status);
-        ok = __all_sync(0xffffffffu, ok) != 0;
-        // the eight warps leave at the same unit (they meet at a barrier below)
-        if (!named_barrier_and(1, kThreads, ok)) break;
-        const uint8_t* slot = units0 + us * sel_unit_bytes(G);
-        const int len = *reinterpret_cast<const int*>(slot);
-        const SelUnit su_ = sel_unit(a, len);
-        if (su_.mode != 2) {
-            int32_t* out = a.idx + (size_t)u * a.topk;
-            if (su_.mode == 0) {  // no query (or a bad length): empty selection
-                if (tid == 0 && (len < 0 || len > a.L)) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
-                for (int j = tid; j < a.topk; j += kThreads) out[j] = -1;
-                if (tid == 0) a.cnt[u] = 0;
-            } else {  // the budget covers every candidate
-                const int n = su_.nF + su_.nC;
-                for (int j = tid; j < a.topk; j += kThreads) {
-                    int v = -1;
-                    if (j < su_.n_init_q) v = j;
-                    else if (j < su_.n_init_q + su_.nC) v = su_.c_lo + (j - su_.n_init_q);
-                    else if (j < n) v = su_.loc_lo + (j - su_.n_init_q - su_.nC);
-                    out[j] = v;
-                }
-                if (tid == 0) a.cnt[u] = n;
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kSB_UFREE + us));
-            continue;
-        }
-        const int nC = su_.nC;
-        const int buf = su & 1;
-        if (su >= 2)  // the top-k warp is done with this buffer's unit before last
-            ok = ok && mbar_wait(bar(kSB_AFREE + buf), ((su >> 1) - 1) & 1, abort_flag, a.status);
-        float* sbuf = sbuf0 + buf * sbuf_floats;
-        float* Sb = sbuf + 4 + 2 * G;
-
-        // ---- scores: four threads per candidate row, each 32 of the 128 columns
-        // (thread 4r + qd: row r of each 64-row chunk, columns [32 qd, 32 qd + 32)).
-        // Its four 16-byte pieces are taken in the order rotated by r, so that a
-        // warp's eight rows fall on distinct banks; q is kept in the same order.
-        const int r = tid >> 2, qd = tid & 3, rot = r & 3;
-        float qv[G][4][8];
-#pragma unroll
-        for (int h = 0; h < G; ++h)
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                const int piece = 4 * qd + ((c + rot) & 3);
-                const uint4 v = *reinterpret_cast<const uint4*>(slot + 16 + h * kRowBytes + piece * 16);
-                const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float2 f = __bfloat1622float2(h2[j]);
-                    qv[h][c][2 * j] = f.x * a.scale_log2;
-                    qv[h][c][2 * j + 1] = f.y * a.scale_log2;
-                }
-            }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(kSB_UFREE + us));  // the slot's q and length are read
-        // each head's softmax statistics over the candidates, online: running
-        // max and sum of 2^(S - max) over the rows this thread writes
-        float m_run[G], z_run[G];
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            m_run[h] = -INFINITY;
-            z_run[h] = 0.f;
-        }
-        const int nch = sel_chunks(su_);
-        for (int i = 0; i < nch; ++i, ++gc) {
-            const int sl = gc % nslots;
-            ok = ok && mbar_wait(bar(kSB_FULL + sl), (gc / nslots) & 1, abort_flag, a.status);
-            const int rows = min(kSlotRows, nC - i * kSlotRows);
-            const bool v = ok && r < rows;
-            const uint8_t* row = smem + sl * kSlotBytes + r * kRowBytes;
-            float acc[G][4];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                const uint4 kv = v ? *reinterpret_cast<const uint4*>(row + (4 * qd + ((c + rot) & 3)) * 16)
-                                   : make_uint4(0u, 0u, 0u, 0u);
-                const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
-#pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    float t = 0.f;
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const float2 f = __bfloat1622float2(k2[j]);
-                        t = fmaf(qv[h][c][2 * j], f.x, t);
-                        t = fmaf(qv[h][c][2 * j + 1], f.y, t);
-                    }
-                    acc[h][c] = t;
-                }
-            }
-            // every lane takes part in the shuffles (a row past the chunk holds zeros)
-#pragma unroll
-            for (int h = 0; h < G; ++h) {
-                float sc = (acc[h][0] + acc[h][1]) + (acc[h][2] + acc[h][3]);
-                sc += __shfl_xor_sync(0xffffffffu, sc, 1);
-                sc += __shfl_xor_sync(0xffffffffu, sc, 2);
-                if (qd == 0 && v) {
-                    Sb[h * a.Tc + i * kSlotRows + r] = sc;
-                    const float mn = fmaxf(m_run[h], sc);
-                    z_run[h] = z_run[h] * ex2_approx(m_run[h] - mn) + ex2_approx(sc - mn);
-                    m_run[h] = mn;
-                }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kSB_EMPTY + sl));  // this warp is done with the slot
-        }
-        // statistics of the warp's rows, then of the eight warps (thread 0)
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            float m = m_run[h], z = z_run[h];
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) {
-                const float mo = __shfl_xor_sync(0xffffffffu, m, off);
-                const float zo = __shfl_xor_sync(0xffffffffu, z, off);
-                const float mn = fmaxf(m, mo);
-                z = mn == -INFINITY ? 0.f : z * ex2_approx(m - mn) + zo * ex2_approx(mo - mn);
-                m = mn;
-            }
-            if (lane == 0) {
-                wstat[(warp * G + h) * 2] = m;
-                wstat[(warp * G + h) * 2 + 1] = z;
-            }
-        }
-        if (!named_barrier_and(1, kThreads, ok)) break;  // scores and statistics complete
-        if (tid == 0) {
-#pragma unroll
-            for (int h = 0; h < G; ++h) {
-                float m = -INFINITY, z = 0.f;
-                for (int w = 0; w < kWarps; ++w) {
-                    const float mo = wstat[(w * G + h) * 2], zo = wstat[(w * G + h) * 2 + 1];
-                    const float mn = fmaxf(m, mo);
-                    z = mn == -INFINITY ? 0.f : z * ex2_approx(m - mn) + zo * ex2_approx(mo - mn);
-                    m = mn;
-                }
-                sbuf[4 + h] = m;
-                sbuf[4 + G + h] = z > 0.f ? 1.0f / z : 0.f;
-            }
-            reinterpret_cast<int*>(sbuf)[0] = u;
-            reinterpret_cast<int*>(sbuf)[1] = len;
-            mbar_arrive(bar(kSB_AFULL + buf));  // hand the unit to the top-k warp
-        }
-        ++su;
-    }
-    if (tid == 0 && ok) {  // the end of the CTA's units for the top-k warp
-        const int buf = su & 1;
-        bool free_buf = true;
-        if (su >= 2)
-            free_buf = mbar_wait(bar(kSB_AFREE + buf), ((su >> 1) - 1) & 1, abort_flag, a.status);
-        if (free_buf) {
-            reinterpret_cast<int*>(sbuf0 + buf * sbuf_floats)[0] = -1;
-            mbar_arrive(bar(kSB_AFULL + buf));
-        }
-    }
 }
 
 // ============================================================== attention
@@ -956,44 +512,8 @@ cudaError_t launch_decode_attn_any(const void* q, const void* K, const void* V, 
 
 }  // namespace
 
-size_t decode_select_smem_bytes(const phsa_shape& s, int topk) {
-    const int G = s.Hq / s.Hkv, Tc = s.L / kM;
-    const int n = dec_select_slots(G, Tc, topk, 1);
-    return n > 0 ? dec_select_smem(G, Tc, topk, n) : (size_t)-1;
-}
-
 size_t decode_attn_smem_bytes(const phsa_shape& s, int topk) {
     return dec_attn_smem(s.Hq / s.Hkv, topk);
-}
-
-cudaError_t launch_decode_select(const void* q, const void* Krepr, const int32_t* lens,
-                                 const phsa_shape& s, const phsa_select_params& p, int32_t* idx,
-                                 int32_t* cnt, int* status, cudaStream_t st) {
-    const int G = s.Hq / s.Hkv, Tc = s.L / kM;
-    const long long units = (long long)s.B * s.Hkv;
-    int dev = 0, nsm = 0;
-    cudaError_t e;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
-        return e;
-    // two CTAs per SM once there are units for them (their unit phases overlap),
-    // the ring as deep as that leaves room for
-    const int per_sm = units > nsm ? 2 : 1;
-    int slots = dec_select_slots(G, Tc, p.topk, per_sm);
-    if (slots == 0) slots = dec_select_slots(G, Tc, p.topk, 1);
-    const size_t smem = dec_select_smem(G, Tc, p.topk, slots);
-    DecSelArgs args{static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(Krepr),
-                    lens, idx, cnt, status, s.Hq, s.Hkv, s.L, Tc, p.topk, p.n_init, p.n_local,
-                    (int)units, slots, p.sm_scale * kLog2e};
-    auto kern = G == 2 ? decode_select_kernel<2> : decode_select_kernel<1>;
-    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
-        cudaSuccess)
-        return e;
-    unsigned grid = 0;
-    if ((e = persistent_grid(kern, kSelThreads, smem, units, grid)) != cudaSuccess) return e;
-    ProfScope prof(K_DEC_SELECT, st);
-    kern<<<grid, kSelThreads, smem, st>>>(args);
-    return cudaGetLastError();
 }
 
 cudaError_t launch_decode_attn(const void* q, const void* K, const void* V, const int32_t* idx,
