@@ -621,30 +621,32 @@ def run_decode(args):
     e2e = None
     if not args.no_e2e:
         # The caches stay on the device; each step uploads the new token's q, k, v
-        # and punctuation flag, appends them at position L - 1, and reads O back.
+        # and id, marks the id against the resident punctuation set, appends k, v
+        # and the flag at position L - 1, runs the step and reads O back.
         hq = torch.empty(q.shape, dtype=torch.int16).pin_memory()
         hk = torch.empty((w.B, w.Hkv, w.D), dtype=torch.int16).pin_memory()
         hv = torch.empty((w.B, w.Hkv, w.D), dtype=torch.int16).pin_memory()
-        hm = torch.empty((w.B,), dtype=torch.uint8).pin_memory()
+        hid = torch.empty((w.B,), dtype=torch.int32).pin_memory()
         hq.copy_(q.view(torch.int16).cpu())
         hk.copy_(K[:, :, w.L - 1].contiguous().view(torch.int16).cpu())
         hv.copy_(V[:, :, w.L - 1].contiguous().view(torch.int16).cpu())
-        hm.copy_(mask[:, w.L - 1].cpu())
+        hid.copy_(torch.from_numpy(np.ascontiguousarray(x["ids"][:, w.L - 1])))
         hO = torch.empty(O.shape, dtype=torch.int16).pin_memory()
         kn = torch.empty((w.B, w.Hkv, w.D), dtype=torch.bfloat16, device=dev)
         vn = torch.empty_like(kn)
+        idn = torch.empty((w.B,), dtype=torch.int32, device=dev)
         mn = torch.empty((w.B,), dtype=torch.uint8, device=dev)
-        h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hm))
+        pset = torch.from_numpy(x["punct_ids"]).to(dev)
+        h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hid))
         d2h = hO.numel() * hO.element_size()
 
         def e2e_step():
             q.view(torch.int16).copy_(hq, non_blocking=True)
             kn.view(torch.int16).copy_(hk, non_blocking=True)
             vn.view(torch.int16).copy_(hv, non_blocking=True)
-            mn.copy_(hm, non_blocking=True)
-            K[:, :, w.L - 1].copy_(kn)
-            V[:, :, w.L - 1].copy_(vn)
-            mask[:, w.L - 1].copy_(mn)
+            idn.copy_(hid, non_blocking=True)
+            phsa.phsa_punct_mask(idn, pset, mask=mn)
+            phsa.phsa_decode_append(kn, vn, lens, K, V, flag_new=mn, punct_mask=mask)
             step()
             hO.copy_(O.view(torch.int16), non_blocking=True)
 
@@ -663,8 +665,9 @@ def run_decode(args):
         ms_e2e = max_over_ranks(a0.elapsed_time(a1) / n_e2e, device=dev)
         e2e = {"value": world * w.B / (ms_e2e / 1e3), "unit": "tokens/s", "ms_per_step": ms_e2e,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": n_e2e,
-               "note": "caches resident on the device; the new token's q, k, v and flag "
-                       "are uploaded and appended, O read back (the K/V appends are torch copies)"}
+               "note": "caches resident on the device; per step the new token's q, k, v and "
+                       "id are uploaded, the id marked (phsa_punct_mask), k, v and the flag "
+                       "appended (phsa_decode_append), the step run and O read back"}
 
     if rank != 0:
         return None

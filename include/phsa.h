@@ -76,6 +76,19 @@ typedef struct {
 } phsa_select_params;
 
 /*
+ * Punctuation indicator, Section 3.2 Eq. 4-5: mask[i] = 1 if ids[i] is one of
+ * the n_punct ids of the punctuation set P, else 0 (the set is given as ids,
+ * in any order, duplicates allowed; building it from a vocabulary is the
+ * caller's job).
+ *   ids        int32 [n]        in (device)
+ *   punct_ids  int32 [n_punct]  in (device), 0 <= n_punct <= 4096
+ *   mask       uint8 [n]        out (device)
+ * PHSA_ERR_UNSUPPORTED for n_punct > 4096; n = 0 does nothing.
+ */
+int phsa_punct_mask(const int32_t* ids, int64_t n, const int32_t* punct_ids, int n_punct,
+                    uint8_t* mask, void* stream);
+
+/*
  * Stage (a): representative keys, Section 3.2 Eq. 6-8 / Algorithm 1 step 2.
  * For every (b, g, t < T): M_0 = mean of the block's m keys (Eq. 6);
  * c = number of punctuation tokens in the block; M_p = mean of their keys if
@@ -226,6 +239,20 @@ int phsa_step_host_release(void* workspace);
  * of 0 means no query; a length < 0 or > L is a device-side error
  * (PHSA_ERR_DEVICE_INDEX) and that sequence is treated as empty.
  */
+
+/*
+ * Appends each sequence's new token to the caches: with p = seq_lens[b] - 1
+ * (seq_lens counts the new token), K[b][g][p] = k_new[b][g] and
+ * V[b][g][p] = v_new[b][g] for every KV head g, and punct_mask[b][p] =
+ * flag_new[b] (nonzero = punctuation). A length <= 0 appends nothing; a length
+ * > L is a device-side error (PHSA_ERR_DEVICE_INDEX) and appends nothing.
+ *   k_new, v_new  bf16 [B, Hkv, D] in;  flag_new uint8 [B] in (may be NULL:
+ *                 the mask is then left as it is)
+ *   K, V          bf16 [B, Hkv, L, D] in/out;  punct_mask uint8 [B, L] in/out
+ */
+int phsa_decode_append(const void* k_new, const void* v_new, const uint8_t* flag_new,
+                       const int32_t* seq_lens, phsa_shape s, void* K, void* V,
+                       uint8_t* punct_mask, void* stream);
 
 /*
  * Block-level caching of the representative keys (Section 3.2): for every

@@ -533,4 +533,45 @@ cudaError_t launch_decode_attn_repr(const void* q, const void* K, const void* V,
                                   Krepr, status, st);
 }
 
+
+// Appends the new token's key and value (and punctuation flag) at row
+// len - 1 of each sequence: one warp per (b, g), lanes 0-15 copy the 256-byte
+// key row and lanes 16-31 the value row, 16 bytes each.
+constexpr int kAppendWarps = 8;
+
+__global__ void __launch_bounds__(kAppendWarps * 32)
+decode_append_kernel(const int4* __restrict__ knew, const int4* __restrict__ vnew,
+                     const uint8_t* __restrict__ flag, const int32_t* __restrict__ lens, int B,
+                     int Hkv, int L, int4* __restrict__ K, int4* __restrict__ V,
+                     uint8_t* __restrict__ mask, int* status) {
+    const int lane = threadIdx.x & 31;
+    const long long u = (long long)blockIdx.x * kAppendWarps + (threadIdx.x >> 5);
+    if (u >= (long long)B * Hkv) return;
+    const int b = (int)(u / Hkv), g = (int)(u % Hkv);
+    const int len = lens[b];
+    if (len > L) {
+        if (g == 0 && lane == 0) set_status(status, PHSA_ERR_DEVICE_INDEX);
+        return;
+    }
+    if (len <= 0) return;
+    constexpr int kRow = kD * 2 / 16;  // int4 per row
+    const long long dst = (u * L + (len - 1)) * kRow;
+    const int c = lane & 15;
+    if (lane < 16) K[dst + c] = knew[u * kRow + c];
+    else V[dst + c] = vnew[u * kRow + c];
+    if (flag && g == 0 && lane == 0) mask[(long long)b * L + (len - 1)] = flag[b] ? 1 : 0;
+}
+
+cudaError_t launch_decode_append(const void* k_new, const void* v_new, const uint8_t* flag,
+                                 const int32_t* lens, const phsa_shape& s, void* K, void* V,
+                                 uint8_t* mask, int* status, cudaStream_t st) {
+    const long long units = (long long)s.B * s.Hkv;
+    if (units == 0) return cudaSuccess;
+    const unsigned grid = (unsigned)((units + kAppendWarps - 1) / kAppendWarps);
+    decode_append_kernel<<<grid, kAppendWarps * 32, 0, st>>>(
+        static_cast<const int4*>(k_new), static_cast<const int4*>(v_new), flag, lens, s.B, s.Hkv,
+        s.L, static_cast<int4*>(K), static_cast<int4*>(V), mask, status);
+    return cudaGetLastError();
+}
+
 }  // namespace phsa

@@ -226,6 +226,33 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
                                                    s.L >= phsa::kM ? Krepr : nullptr, st, cs));
 }
 
+int phsa_punct_mask(const int32_t* ids, int64_t n, const int32_t* punct_ids, int n_punct,
+                    uint8_t* mask, void* stream) {
+    if (n < 0 || n_punct < 0) return PHSA_ERR_INVALID_ARG;
+    if (n_punct > 4096) return PHSA_ERR_UNSUPPORTED;
+    if (n == 0) return PHSA_OK;
+    if (!ids || !mask || (n_punct > 0 && !punct_ids)) return PHSA_ERR_INVALID_ARG;
+    return from_cuda(phsa::launch_punct_mask(ids, n, punct_ids, n_punct, mask,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
+int phsa_decode_append(const void* k_new, const void* v_new, const uint8_t* flag_new,
+                       const int32_t* seq_lens, phsa_shape s, void* K, void* V,
+                       uint8_t* punct_mask, void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if (s.B == 0) return PHSA_OK;
+    if (!k_new || !v_new || !seq_lens || !K || !V || (flag_new && !punct_mask))
+        return PHSA_ERR_INVALID_ARG;
+    if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(K) || !aligned16(V))
+        return PHSA_ERR_INVALID_ARG;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_decode_append(k_new, v_new, flag_new, seq_lens, s, K, V,
+                                                punct_mask, st,
+                                                static_cast<cudaStream_t>(stream)));
+}
+
 int phsa_get_device_status(void* stream) {
     if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
         return PHSA_ERR_CUDA;

@@ -51,6 +51,13 @@ cudaError_t launch_decode_attn_repr(const void* q, const void* K, const void* V,
                                     float* lse, const uint8_t* mask, float lambda, void* Krepr,
                                     int* status, cudaStream_t st);
 size_t decode_attn_smem_bytes(const phsa_shape& s, int topk);
+// Writes the new token's k, v and punctuation flag at row len - 1 (decode.cu).
+cudaError_t launch_decode_append(const void* k_new, const void* v_new, const uint8_t* flag,
+                                 const int32_t* lens, const phsa_shape& s, void* K, void* V,
+                                 uint8_t* mask, int* status, cudaStream_t st);
+// Punctuation indicator of token ids against a set of <= 4096 ids (punct.cu).
+cudaError_t launch_punct_mask(const int32_t* ids, long long n, const int32_t* punct_ids,
+                              int n_punct, uint8_t* mask, cudaStream_t st);
 
 cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape& s,
                              const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,

@@ -89,9 +89,12 @@ def _declare(L):
                                    P, P]
     L.phsa_decode_step.restype = I
     L.phsa_decode_update_repr.argtypes = [P, P, P, phsa_shape, F, P, P]
+    L.phsa_decode_append.argtypes = [P, P, P, P, phsa_shape, P, P, P, P]
+    L.phsa_punct_mask.argtypes = [P, ctypes.c_int64, P, I, P, P]
     L.phsa_decode_select.argtypes = [P, P, P, phsa_shape, phsa_select_params, P, P, P]
     L.phsa_decode_attn.argtypes = [P, P, P, P, P, P, phsa_shape, I, F, P, P, P]
     for fn in ("phsa_decode_update_repr", "phsa_decode_select", "phsa_decode_attn",
+               "phsa_decode_append", "phsa_punct_mask",
                "phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
                "phsa_sparse_attn_bwd", "phsa_get_device_status", "phsa_selftest_tcgen05"):
         getattr(L, fn).restype = I
@@ -331,6 +334,49 @@ def phsa_step_host(Q, K, V, dO, punct_mask, lam: float, topk: int, n_init: int =
 def phsa_step_host_release(workspace):
     """Waits for the last phsa_step_host call on `workspace` and drops its events."""
     _raise("phsa_step_host_release", load().phsa_step_host_release(_ptr(workspace)))
+
+
+def phsa_punct_mask(ids, punct_ids, mask=None, stream=None):
+    """Punctuation indicator: mask[i] = 1 if ids[i] is in punct_ids, else 0.
+    ids int32 (any shape, contiguous), punct_ids int32 [n_punct <= 4096];
+    returns a uint8 mask of ids' shape."""
+    _check(ids, "ids", torch.int32)
+    _check(punct_ids, "punct_ids", torch.int32, 1)
+    if mask is None:
+        mask = torch.empty(ids.shape, dtype=torch.uint8, device=ids.device)
+    _check(mask, "mask", torch.uint8)
+    if mask.numel() != ids.numel():
+        raise ValueError("mask must have as many elements as ids")
+    rc = load().phsa_punct_mask(_ptr(ids), ids.numel(), _ptr(punct_ids), punct_ids.numel(),
+                                _ptr(mask), _stream(stream))
+    _raise("phsa_punct_mask", rc)
+    return mask
+
+
+def phsa_decode_append(k_new, v_new, seq_lens, K, V, flag_new=None, punct_mask=None,
+                       stream=None):
+    """Write the new token of every sequence at row seq_lens[b] - 1 of the
+    caches: k_new/v_new [B, Hkv, D] bf16 into K/V [B, Hkv, Lc, D], and, when
+    flag_new [B] uint8 is given, its flag into punct_mask [B, Lc]."""
+    _check(k_new, "k_new", torch.bfloat16, 3)
+    _check(v_new, "v_new", torch.bfloat16, 3)
+    _check(seq_lens, "seq_lens", torch.int32, 1)
+    _check(K, "K", torch.bfloat16, 4)
+    _check(V, "V", torch.bfloat16, 4)
+    B, Hkv, Lc, D = K.shape
+    if tuple(V.shape) != tuple(K.shape) or tuple(k_new.shape) != (B, Hkv, D) or \
+            tuple(v_new.shape) != (B, Hkv, D) or tuple(seq_lens.shape) != (B,):
+        raise ValueError("k_new/v_new must be [B, Hkv, D], K/V [B, Hkv, Lc, D], seq_lens [B]")
+    if flag_new is not None:
+        _check(flag_new, "flag_new", torch.uint8, 1)
+        _check(punct_mask, "punct_mask", torch.uint8, 2)
+        if tuple(flag_new.shape) != (B,) or tuple(punct_mask.shape) != (B, Lc):
+            raise ValueError("flag_new must be [B] and punct_mask [B, Lc]")
+    rc = load().phsa_decode_append(_ptr(k_new), _ptr(v_new), _ptr(flag_new), _ptr(seq_lens),
+                                   make_shape(B, Lc, Hkv, Hkv, D), _ptr(K), _ptr(V),
+                                   _ptr(punct_mask), _stream(stream))
+    _raise("phsa_decode_append", rc)
+    return K, V
 
 
 def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=None):

@@ -100,3 +100,28 @@ def test_host_step_validation_needs_no_gpu(lib):
     assert lib.phsa_step_host(*args, ok, 0.5, p, *([None] * 7), dummy, ws - 1, None, None) == -6
     assert lib.phsa_step_host(*args, phsa_shape(1, 4096, 16, 8, 64, 64), 0.5, p, *([None] * 7),
                               dummy, ws, None, None) == -2
+
+
+def test_punct_mask_and_append_validation_needs_no_gpu(lib):
+    # Both entry points reject bad arguments before any CUDA call.
+    from paper_2601_02819_gb300.phsa import phsa_shape
+    P = ctypes.c_void_p
+    lib.phsa_punct_mask.argtypes = [P, ctypes.c_int64, P, ctypes.c_int, P, P]
+    lib.phsa_decode_append.argtypes = [P, P, P, P, phsa_shape, P, P, P, P]
+    dummy = ctypes.c_void_p(256)  # never dereferenced
+    assert lib.phsa_punct_mask(dummy, 10, dummy, 4097, dummy, None) == -2  # set too large
+    assert lib.phsa_punct_mask(dummy, -1, dummy, 4, dummy, None) == -1
+    assert lib.phsa_punct_mask(dummy, 10, dummy, -1, dummy, None) == -1
+    assert lib.phsa_punct_mask(None, 10, dummy, 4, dummy, None) == -1
+    assert lib.phsa_punct_mask(dummy, 10, None, 4, dummy, None) == -1  # set without ids
+    assert lib.phsa_punct_mask(None, 0, None, 4, None, None) == 0  # nothing to do
+    ok = phsa_shape(2, 256, 8, 8, 128, 64)
+    assert lib.phsa_decode_append(dummy, dummy, None, dummy, phsa_shape(2, 256, 8, 8, 64, 64),
+                                  dummy, dummy, None, None) == -2  # D = 64
+    assert lib.phsa_decode_append(None, dummy, None, dummy, ok, dummy, dummy, None, None) == -1
+    assert lib.phsa_decode_append(dummy, dummy, dummy, dummy, ok, dummy, dummy, None,
+                                  None) == -1  # flags without a mask
+    odd = ctypes.c_void_p(264)  # not 16-byte aligned
+    assert lib.phsa_decode_append(odd, dummy, None, dummy, ok, dummy, dummy, None, None) == -1
+    assert lib.phsa_decode_append(None, None, None, None, phsa_shape(0, 256, 8, 8, 128, 64),
+                                  None, None, None, None) == 0  # empty batch
