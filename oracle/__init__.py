@@ -61,10 +61,10 @@ def _declare(L):
     L.phsa_oracle_punct_mask.argtypes = [P, i64, P, i32, P]
     L.phsa_oracle_block_repr.argtypes = [P, P, i32, i32, i32, i32, i32, f64, P, P]
     L.phsa_oracle_select_blocks.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, i32,
-                                            i32, f64, P, P, P]
+                                            i32, f64, i32, P, P, P]
     L.phsa_oracle_select_blocks.restype = i32
     L.phsa_oracle_select_units.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, i32, i32,
-                                           f64, P, i64, P, P, P]
+                                           f64, i32, P, i64, P, P, P]
     L.phsa_oracle_select_units.restype = i32
     L.phsa_oracle_sparse_attn_bwd_dq_rows.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32,
                                                       i32, i32, f64, P, i64, P]
@@ -78,7 +78,7 @@ def _declare(L):
                                               i32, i32, f64, P, P, P]
     L.phsa_oracle_dense_causal.argtypes = [P, P, P, i32, i32, i32, i32, i32, f64, P, P]
     L.phsa_oracle_decode_select.argtypes = [P, P, P, i32, i32, i32, i32, i32, i32, i32, i32,
-                                            i32, f64, P, P, P]
+                                            i32, f64, i32, P, P, P]
     L.phsa_oracle_decode_select.restype = i32
     L.phsa_oracle_decode_attn.argtypes = [P, P, P, P, P, P, i32, i32, i32, i32, i32, i32, i32,
                                           f64, P, P]
@@ -141,10 +141,21 @@ def block_repr(K, mask, block_size: int, lam: float, want_f64: bool = False):
     return (out, out64) if want_f64 else out
 
 
+AGGREGATIONS = {"softmax_sum": 0, "max_logit": 1}
+
+
+def _agg_mode(aggregation: str) -> int:
+    if aggregation not in AGGREGATIONS:
+        raise ValueError(f"aggregation must be one of {sorted(AGGREGATIONS)}")
+    return AGGREGATIONS[aggregation]
+
+
 def select_blocks(Q, Krepr, L: int, block_size: int, topk: int, n_init: int, n_local: int,
-                  sm_scale: float, want_agg: bool = False):
+                  sm_scale: float, want_agg: bool = False, aggregation: str = "softmax_sum"):
     """Algorithm 1 step 3 per (query block, KV head).
 
+    ``aggregation``: "softmax_sum" (the group's rows' softmax probabilities
+    summed, Eq. 8) or "max_logit" (the largest raw score over the rows).
     Returns (block_idx [B,Hkv,NQB,topk], block_cnt [B,Hkv,NQB]) and, if
     ``want_agg``, the aggregates A [B,Hkv,NQB,T] (NaN where not scored).
     """
@@ -159,7 +170,8 @@ def select_blocks(Q, Krepr, L: int, block_size: int, topk: int, n_init: int, n_l
     cnt = np.empty((B, Hkv, NQB), dtype=np.int32)
     agg = np.empty((B, Hkv, NQB, max(T, 1)), dtype=np.float64) if want_agg else None
     rc = lib().phsa_oracle_select_blocks(_p(Q), _p(Krepr), B, Hq, Hkv, L, D, block_size,
-                                         topk, n_init, n_local, float(sm_scale), _p(idx),
+                                         topk, n_init, n_local, float(sm_scale),
+                                         _agg_mode(aggregation), _p(idx),
                                          _p(cnt), _p(agg) if want_agg else None)
     if rc != 0:
         raise ValueError("topk is smaller than the forced block count")
@@ -167,7 +179,7 @@ def select_blocks(Q, Krepr, L: int, block_size: int, topk: int, n_init: int, n_l
 
 
 def select_units(Q, Krepr, L: int, block_size: int, topk: int, n_init: int, n_local: int,
-                 sm_scale: float, units):
+                 sm_scale: float, units, aggregation: str = "softmax_sum"):
     """Selection for a list of flat units u = (b*Hkv + g)*NQB + qb only.
 
     Returns (idx [n, topk], cnt [n], agg [n, T]).
@@ -184,7 +196,8 @@ def select_units(Q, Krepr, L: int, block_size: int, topk: int, n_init: int, n_lo
     cnt = np.empty((n,), dtype=np.int32)
     agg = np.empty((n, max(T, 1)), dtype=np.float64)
     rc = lib().phsa_oracle_select_units(_p(Q), _p(Krepr), B, Hq, Hkv, L, D, block_size, topk,
-                                        n_init, n_local, float(sm_scale), _p(units), n, _p(idx),
+                                        n_init, n_local, float(sm_scale), _agg_mode(aggregation),
+                                        _p(units), n, _p(idx),
                                         _p(cnt), _p(agg))
     if rc != 0:
         raise ValueError("topk is smaller than the forced block count")
@@ -283,7 +296,8 @@ def dense_causal(Q, K, V, sm_scale: float):
 
 
 def decode_select(q, Krepr, lens, Lc: int, block_size: int, topk: int, n_init: int,
-                  n_local: int, sm_scale: float, want_agg: bool = False):
+                  n_local: int, sm_scale: float, want_agg: bool = False,
+                  aggregation: str = "softmax_sum"):
     """Selection for one new token per sequence (the token at lens[b] - 1).
 
     q [B,Hq,D], Krepr [B,Hkv,Lc/m,D] (full blocks valid). Returns (block_idx
@@ -299,7 +313,8 @@ def decode_select(q, Krepr, lens, Lc: int, block_size: int, topk: int, n_init: i
     agg = np.empty((B, Hkv, max(Tc, 1)), dtype=np.float64) if want_agg else None
     rc = lib().phsa_oracle_decode_select(_p(q), _p(Krepr), _p(lens), B, Hq, Hkv, Lc, D,
                                          block_size, topk, n_init, n_local, float(sm_scale),
-                                         _p(idx), _p(cnt), _p(agg) if want_agg else None)
+                                         _agg_mode(aggregation), _p(idx), _p(cnt),
+                                         _p(agg) if want_agg else None)
     if rc != 0:
         raise ValueError("topk is smaller than the forced block count, or a length exceeds Lc")
     return (idx, cnt, agg) if want_agg else (idx, cnt)

@@ -35,6 +35,9 @@
  *   R6 (backward): selection is a hard choice; gradients flow to Q, K, V only.
  *   R7 (Krepr precision): the representative keys are stored as bf16 (round
  *      to nearest even) and scoring reads the stored values.
+ *   R8 (max-logit variant, agg_mode 1): the group's relevance A_t is the
+ *      largest raw score S_{r,t} = q_r . M_t * scale over its rows; for a
+ *      single row this ranks exactly as Eq. 8's softmax does.
  */
 #include <math.h>
 #include <stdint.h>
@@ -182,8 +185,8 @@ static int is_forced(int t, int qb, int n_init, int n_local) {
  * returns the count, or -1 if topk < |F_b|. If agg is not NULL it receives A_t
  * for t < T (NaN where t was not scored). */
 static int select_core(const uint16_t* const* rows, int nrows, const uint16_t* Kr, int T, int qb,
-                       int D, int topk, int n_init, int n_local, double scale, int32_t* out,
-                       double* agg) {
+                       int D, int topk, int n_init, int n_local, double scale, int agg_mode,
+                       int32_t* out, double* agg) {
     double* A = (double*)calloc((size_t)(T > 0 ? T : 1), sizeof(double));
     int* cand = (int*)malloc(sizeof(int) * (size_t)(qb + 1));
     int* chosen = (int*)calloc((size_t)(qb + 1), sizeof(int));
@@ -200,6 +203,8 @@ static int select_core(const uint16_t* const* rows, int nrows, const uint16_t* K
             for (int c = 0; c < nC; ++c) chosen[cand[c]] = 1;
         } else if (ksel > 0) {
             double* s = (double*)malloc(sizeof(double) * (size_t)nC);
+            if (agg_mode == 1)
+                for (int c = 0; c < nC; ++c) A[cand[c]] = -INFINITY;
             for (int r = 0; r < nrows; ++r) {
                 const uint16_t* q = rows[r];
                 double mx = -INFINITY;
@@ -210,6 +215,11 @@ static int select_core(const uint16_t* const* rows, int nrows, const uint16_t* K
                         dot += phsa_oracle_bf16_to_f64(q[d]) * phsa_oracle_bf16_to_f64(M[d]);
                     s[c] = dot * scale; /* S_{r,t} */
                     if (s[c] > mx) mx = s[c];
+                }
+                if (agg_mode == 1) { /* R8 */
+                    for (int c = 0; c < nC; ++c)
+                        if (s[c] > A[cand[c]]) A[cand[c]] = s[c];
+                    continue;
                 }
                 double z = 0.0;
                 for (int c = 0; c < nC; ++c) z += exp(s[c] - mx);
@@ -240,8 +250,8 @@ static int select_core(const uint16_t* const* rows, int nrows, const uint16_t* K
 /* Selection for one (b, g, qb) unit u = (b*Hkv + g)*NQB + qb: the rows are the
  * block's tokens of each query head of the group, head by head. */
 static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv, int L, int D,
-                       int m, int topk, int n_init, int n_local, double scale, int64_t u,
-                       int32_t* out, double* agg) {
+                       int m, int topk, int n_init, int n_local, double scale, int agg_mode,
+                       int64_t u, int32_t* out, double* agg) {
     const int G = Hq / Hkv, T = L / m, NQB = (L + m - 1) / m;
     const int qb = (int)(u % NQB);
     const int g = (int)((u / NQB) % Hkv);
@@ -254,7 +264,7 @@ static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv
             rows[nrows++] = Q + (((int64_t)b * Hq + h) * L + i) * D;
     }
     int n = select_core(rows, nrows, Krepr + ((int64_t)b * Hkv + g) * T * D, T, qb, D, topk,
-                        n_init, n_local, scale, out, agg);
+                        n_init, n_local, scale, agg_mode, out, agg);
     free(rows);
     return n;
 }
@@ -267,7 +277,7 @@ static int select_unit(const uint16_t* Q, const uint16_t* Krepr, int Hq, int Hkv
  * Returns 0, or -1 if topk < |F_b| for some query block. */
 int phsa_oracle_select_blocks(const uint16_t* Q, const uint16_t* Krepr, int B, int Hq,
                               int Hkv, int L, int D, int m, int topk, int n_init, int n_local,
-                              double scale, int32_t* block_idx, int32_t* block_cnt,
+                              double scale, int agg_mode, int32_t* block_idx, int32_t* block_cnt,
                               double* agg) {
     const int T = L / m, NQB = (L + m - 1) / m;
     int bad = 0;
@@ -276,8 +286,8 @@ int phsa_oracle_select_blocks(const uint16_t* Q, const uint16_t* Krepr, int B, i
 #pragma omp parallel for schedule(dynamic, 1) num_threads(NTH) reduction(| : bad)
 #endif
     for (int64_t u = 0; u < units; ++u) {
-        int n = select_unit(Q, Krepr, Hq, Hkv, L, D, m, topk, n_init, n_local, scale, u,
-                            block_idx + u * topk, agg ? agg + u * T : NULL);
+        int n = select_unit(Q, Krepr, Hq, Hkv, L, D, m, topk, n_init, n_local, scale, agg_mode,
+                            u, block_idx + u * topk, agg ? agg + u * T : NULL);
         block_cnt[u] = n;
         if (n < 0) bad = 1;
     }
@@ -288,7 +298,7 @@ int phsa_oracle_select_blocks(const uint16_t* Q, const uint16_t* Krepr, int B, i
  * problems): idx [n_units, topk], cnt [n_units], agg [n_units, T] or NULL. */
 int phsa_oracle_select_units(const uint16_t* Q, const uint16_t* Krepr, int B, int Hq, int Hkv,
                              int L, int D, int m, int topk, int n_init, int n_local,
-                             double scale, const int64_t* units, int64_t n_units,
+                             double scale, int agg_mode, const int64_t* units, int64_t n_units,
                              int32_t* idx, int32_t* cnt, double* agg) {
     const int T = L / m;
     int bad = 0;
@@ -297,8 +307,8 @@ int phsa_oracle_select_units(const uint16_t* Q, const uint16_t* Krepr, int B, in
 #pragma omp parallel for schedule(dynamic, 1) num_threads(NTH) reduction(| : bad)
 #endif
     for (int64_t k = 0; k < n_units; ++k) {
-        int n = select_unit(Q, Krepr, Hq, Hkv, L, D, m, topk, n_init, n_local, scale, units[k],
-                            idx + k * topk, agg ? agg + k * T : NULL);
+        int n = select_unit(Q, Krepr, Hq, Hkv, L, D, m, topk, n_init, n_local, scale, agg_mode,
+                            units[k], idx + k * topk, agg ? agg + k * T : NULL);
         cnt[k] = n;
         if (n < 0) bad = 1;
     }
@@ -593,8 +603,8 @@ void phsa_oracle_sparse_attn_bwd_kv_blocks(const uint16_t* Q, const uint16_t* K,
  * count 0, indices -1, output 0 and lse -inf. */
 int phsa_oracle_decode_select(const uint16_t* q, const uint16_t* Krepr, const int32_t* lens,
                               int B, int Hq, int Hkv, int Lc, int D, int m, int topk, int n_init,
-                              int n_local, double scale, int32_t* block_idx, int32_t* block_cnt,
-                              double* agg) {
+                              int n_local, double scale, int agg_mode, int32_t* block_idx,
+                              int32_t* block_cnt, double* agg) {
     const int G = Hq / Hkv, Tc = Lc / m;
     int bad = 0;
     const int64_t units = (int64_t)B * Hkv;
@@ -618,7 +628,7 @@ int phsa_oracle_decode_select(const uint16_t* q, const uint16_t* Krepr, const in
         const uint16_t* rows[64];
         for (int hh = 0; hh < G && hh < 64; ++hh) rows[hh] = q + ((int64_t)b * Hq + g * G + hh) * D;
         int n = select_core(rows, G, Krepr + ((int64_t)b * Hkv + g) * Tc * D, len / m, p / m, D,
-                            topk, n_init, n_local, scale, out, ag);
+                            topk, n_init, n_local, scale, agg_mode, out, ag);
         block_cnt[u] = n;
         if (n < 0) bad = 1;
     }

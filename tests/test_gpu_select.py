@@ -49,6 +49,8 @@ def test_tiny_workload():
     (1, 2, 1, 64 * 20, 25, 1, 1),       # budget covers everything: dense rows
     (1, 4, 2, 64 * 40 + 5, 20, 1, 1),   # G = 2: warp slices smaller than the budget
     (1, 2, 1, 64 * 160, 80, 1, 1),      # G = 2: budget above the two-level top-k limit
+    (1, 2, 1, 64 * 601, 14, 2, 8),      # G = 2: paper forced sets, odd NQB, chunks reloaded
+    (2, 4, 2, 64 * 3 + 1, 3, 1, 1),     # G = 2: first blocks (no candidates, all forced)
 ])
 def test_shapes_and_forced_sets(B, Hq, Hkv, L, topk, n_init, n_local):
     rng = np.random.default_rng(B * 1000 + L)
@@ -80,9 +82,13 @@ def test_exact_ties_go_to_the_lower_block():
         assert list(gi[0, 0, qb]) == [0, 3, qb], qb
 
 
-@pytest.mark.parametrize("name", ["train_8k_x4", "prefill_32k"])
+@pytest.mark.parametrize("name", ["train_8k_x4", "prefill_32k", "prefill_32k_paper_forced"])
 def test_full_size_sampled_units(name):
-    w = inputs.WORKLOADS[name]
+    if name == "prefill_32k_paper_forced":  # 128 initial + 512 local tokens, as the paper's 32k setting
+        w = inputs.custom(name, B=1, L=32768, Hq=16, Hkv=8, topk=14, n_init=2, n_local=8,
+                          punct="sentence", seed=77)
+    else:
+        w = inputs.WORKLOADS[name]
     x = inputs.make_inputs(w)
     Kr = oracle.block_repr(x["K"], x["mask"], 64, w.lam)
     scale = 128 ** -0.5

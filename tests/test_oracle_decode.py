@@ -35,18 +35,19 @@ def _last_rows(Q, lens):
     return np.stack([Q[b, :, lens[b] - 1] for b in range(len(lens))])
 
 
-def test_decode_select_equals_prefill_block_with_one_row():
+@pytest.mark.parametrize("aggregation", ["softmax_sum", "max_logit"])
+def test_decode_select_equals_prefill_block_with_one_row(aggregation):
     B, Hq, Hkv, Lc = 3, 4, 2, 64 * 20
     lens = np.array([64 * 7 + 1, 64 * 12 + 1, 64 * 19 + 1], np.int32)
     Q, K, _, mask = _case(1, B, Hq, Hkv, Lc)
     Kr = oracle.block_repr(K, mask, M, 0.5)
     topk = 5
     di, dc, da = oracle.decode_select(_last_rows(Q, lens), Kr, lens, Lc, M, topk, 1, 1, SCALE,
-                                      want_agg=True)
+                                      want_agg=True, aggregation=aggregation)
     for b, L in enumerate(lens):
         Krb = oracle.block_repr(K[b:b + 1, :, :L], mask[b:b + 1, :L], M, 0.5)
         pi, pc, pa = oracle.select_blocks(Q[b:b + 1, :, :L], Krb, int(L), M, topk, 1, 1, SCALE,
-                                          want_agg=True)
+                                          want_agg=True, aggregation=aggregation)
         qb = (L - 1) // M
         assert np.array_equal(di[b], pi[0, :, qb]), b
         assert np.array_equal(dc[b], pc[0, :, qb]), b

@@ -211,3 +211,83 @@ def test_output_is_ascending_unique_and_budgeted():
                 assert np.all(np.diff(row[:n]) > 0) and np.all(row[n:] == -1)
                 assert row[0] == 0 and row[n - 1] == qb
                 assert {0, 1} & set(range(qb + 1)) <= set(row[:n])
+
+
+# ---- the max-logit aggregation (A_t = max over the group's rows of S_{r,t}) ----
+
+def sel_max(Q, Kr, L, m, topk, n_init=1, n_local=1, scale=1.0, agg=False):
+    return oracle.select_blocks(Q, Kr, L, m, topk, n_init, n_local, scale, want_agg=agg,
+                                aggregation="max_logit")
+
+
+def test_max_logit_takes_the_largest_raw_score_over_rows():
+    # The case above: one row scores (100, 0, 0), 63 rows (0, 0.5, 0), forced blocks 10.
+    # A = (100, 0.5, 0) exactly; the forced blocks' scores play no part.
+    rows = [(100.0, 0.0, 0.0)] + [(0.0, 0.5, 0.0)] * 63
+    Q, Kr, L, m = _onehot_case(rows, forced_bias=10.0)
+    idx, cnt, A = sel_max(Q, Kr, L, m, topk=3, agg=True)
+    assert list(idx[0, 0, 4]) == [0, 1, 4]
+    assert list(A[0, 0, 4, 1:4]) == [100.0, 0.5, 0.0]
+    assert np.isnan(A[0, 0, 4, 0]) and np.isnan(A[0, 0, 4, 4])
+    idx2, _ = sel_max(Q, Kr, L, m, topk=4)  # second pick: 0.5 beats 0
+    assert list(idx2[0, 0, 4]) == [0, 1, 2, 4]
+
+
+@pytest.mark.parametrize("s,expect", [(0.5, 1), (2.0, 2), (-3.0, 1)])
+def test_max_logit_over_both_heads(s, expect):
+    # head 0 rows score (1, 0, 0), head 1 rows (0, s, 0): A = (1, max(0, s), 0)
+    Q, Kr, L, m = _onehot_case([(1.0, 0.0, 0.0)] * 64, [(0.0, s, 0.0)] * 64)
+    idx, cnt, A = sel_max(Q, Kr, L, m, topk=3, agg=True)
+    assert list(idx[0, 0, 4]) == [0, expect, 4]
+    assert list(A[0, 0, 4, 1:4]) == [1.0, max(0.0, s), 0.0]
+
+
+def test_max_logit_ranks_negative_scores():
+    # every candidate's best score is negative: the least negative wins
+    Q, Kr, L, m = _onehot_case([(-4.0, -1.5, -2.0)] * 64)
+    idx, cnt, A = sel_max(Q, Kr, L, m, topk=4, agg=True)
+    assert list(idx[0, 0, 4]) == [0, 2, 3, 4]
+    assert list(A[0, 0, 4, 1:4]) == [-4.0, -1.5, -2.0]
+
+
+def test_max_logit_per_token_case_is_argsort_of_raw_scores():
+    # With a single row per unit both aggregations rank by q_i . k_t (Algorithm 1).
+    rng = np.random.default_rng(2)
+    L, n_init, n_local, extra = 40, 2, 3, 4
+    topk = n_init + n_local + extra
+    Q = bf(rng.standard_normal((1, 1, L, D)))
+    K = bf(rng.standard_normal((1, 1, L, D)))
+    idx, cnt = sel_max(Q, K, L, 1, topk, n_init, n_local, scale=D ** -0.5)
+    q = oracle.bf16_to_f64(Q)[0, 0]
+    k = oracle.bf16_to_f64(K)[0, 0]
+    S = q @ k.T
+    for i in range(L):
+        forced = set(range(min(n_init, i + 1))) | set(range(max(0, i - n_local + 1), i + 1))
+        order = sorted((t for t in range(i) if t not in forced), key=lambda t: (-S[i, t], t))
+        expect = sorted(forced | set(order[:extra]))
+        assert list(idx[0, 0, i, :len(expect)]) == expect, i
+    idx_sm, cnt_sm = sel(Q, K, L, 1, topk, n_init, n_local, scale=D ** -0.5)
+    assert np.array_equal(idx, idx_sm) and np.array_equal(cnt, cnt_sm)
+
+
+def test_max_logit_is_scale_free_and_linear_in_the_scale():
+    # A positive scale multiplies every score: the choice is unchanged and A scales
+    # exactly by powers of two.
+    rng = np.random.default_rng(12)
+    L, m = 64 * 12 + 7, 64
+    Q = bf(rng.standard_normal((1, 4, L, D)))
+    Kr = bf(rng.standard_normal((1, 2, 12, D)))
+    i1, c1, a1 = sel_max(Q, Kr, L, m, topk=5, scale=1.0, agg=True)
+    i2, c2, a2 = sel_max(Q, Kr, L, m, topk=5, scale=4.0, agg=True)
+    i3, c3 = sel_max(Q, Kr, L, m, topk=5, scale=1e-3)
+    assert np.array_equal(i1, i2) and np.array_equal(i1, i3) and np.array_equal(c1, c3)
+    ok = ~np.isnan(a1)
+    assert np.array_equal(a2[ok], 4.0 * a1[ok])
+    # A is the column maximum of the unit's score matrix: 128 rows for a full query
+    # block, the 2 x 7 rows that exist for the ragged last one (L = 64 * 12 + 7)
+    Qf, Kf = oracle.bf16_to_f64(Q), oracle.bf16_to_f64(Kr)
+    for qb, g in ((9, 1), (12, 0)):
+        rows = np.concatenate([Qf[0, 2 * g + h, qb * m:min(L, (qb + 1) * m)] for h in range(2)])
+        S = rows @ Kf[0, g].T
+        cands = list(range(1, qb))  # n_init = 1, n_local = 1
+        assert np.array_equal(a1[0, g, qb, cands], S[:, cands].max(axis=0)), qb
