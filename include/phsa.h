@@ -61,18 +61,32 @@ typedef struct {
     int B, L, Hq, Hkv, D, block_size;
 } phsa_shape;
 
+/* How the G*m query rows of a (query block, KV head) unit are combined into
+ * one relevance A_t per candidate block t (the paper scores single tokens,
+ * Eq. 8; the group rule is this library's reading):
+ *   PHSA_AGG_SOFTMAX_SUM  A_t = sum over the rows of the row's softmax
+ *                         probability of block t over the candidates (Eq. 8);
+ *   PHSA_AGG_MAX_LOGIT    A_t = max over the rows of the raw score
+ *                         q_r . Krepr_t * sm_scale (one pass, no softmax).
+ * Both reduce to Algorithm 1's per-token ranking for a single row. */
+#define PHSA_AGG_SOFTMAX_SUM 0
+#define PHSA_AGG_MAX_LOGIT 1
+
 /* Selection parameters (Algorithm 1 inputs k, n_init and w).
- *   topk     total blocks per (query block, KV head), forced blocks included
- *            (the paper's 32k setting of 128 initial + 512 local tokens plus 16
- *            chosen 16-token blocks is 896 tokens = 14 blocks of 64);
- *   n_init   forced initial blocks {0 .. n_init-1};
- *   n_local  forced local blocks {qb-n_local+1 .. qb}, n_local >= 1 (the query's
- *            own block is always attended);
- *   sm_scale score scale, normally 1/sqrt(D) (Eq. 2, 8, 11).
+ *   topk        total blocks per (query block, KV head), forced blocks included
+ *               (the paper's 32k setting of 128 initial + 512 local tokens plus
+ *               16 chosen 16-token blocks is 896 tokens = 14 blocks of 64);
+ *   n_init      forced initial blocks {0 .. n_init-1};
+ *   n_local     forced local blocks {qb-n_local+1 .. qb}, n_local >= 1 (the
+ *               query's own block is always attended);
+ *   sm_scale    score scale, normally 1/sqrt(D) (Eq. 2, 8, 11);
+ *   aggregation PHSA_AGG_SOFTMAX_SUM (0, the default of a zeroed struct) or
+ *               PHSA_AGG_MAX_LOGIT; other values are PHSA_ERR_INVALID_ARG.
  * Requires topk >= n_init + n_local, so every query block's forced set fits. */
 typedef struct {
     int topk, n_init, n_local;
     float sm_scale;
+    int aggregation;
 } phsa_select_params;
 
 /*

@@ -24,6 +24,8 @@
 //           the next units (warp 6 takes the units of buffer 0, warp 7 those of
 //           buffer 1): A_t = sum over heads of the head's softmax probability,
 //           the k largest by (A desc, t asc), then the forced blocks merged.
+// Under the max-logit rule (PHSA_AGG_MAX_LOGIT) the scoring warps keep no
+// statistics and A_t is the largest of the G heads' scores.
 // Every wait is bounded in time; on expiry the kernel records PHSA_ERR_TIMEOUT,
 // lets its own copies and MMAs finish, frees TMEM and returns.
 #include "phsa_common.cuh"
@@ -64,8 +66,8 @@ struct Args {
     int32_t* idx;
     int32_t* cnt;
     int* status;
-    int Hq, Hkv, L, Tc, topk, n_init, n_local, units, slots;
-    float scale_log2;
+    int Hq, Hkv, L, Tc, topk, n_init, n_local, units, slots, agg;
+    float scale_log2, scale;
 };
 
 // What one (sequence, KV head) unit asks of the selection. mode 0: no query
@@ -369,7 +371,10 @@ decode_select_tc_kernel(const __grid_constant__ CUtensorMap tmKr,
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(B_TFREE + tb));  // the MMA may overwrite it
                 const int cj = i * kCand + lrow;
-                if (ok && cj < sd.nC) {
+                if (ok && cj < sd.nC && a.agg) {
+#pragma unroll
+                    for (int h = 0; h < G; ++h) Sb[h * a.Tc + cj] = __uint_as_float(v[h]) * a.scale;
+                } else if (ok && cj < sd.nC) {
 #pragma unroll
                     for (int h = 0; h < G; ++h) {
                         const float sc = __uint_as_float(v[h]) * a.scale_log2;
@@ -444,8 +449,15 @@ decode_select_tc_kernel(const __grid_constant__ CUtensorMap tmKr,
             const float* iz = mx + G;
             float* Sb = sbuf + 4 + 2 * G;
             const int nC = d.nC, ksel = d.ksel, c_lo = d.c_lo;
-            // A_t = sum over the heads of the head's softmax probability, head order
+            // A_t = sum over the heads of the head's softmax probability, head order;
+            // or the largest of the heads' scores
             auto key_of = [&](int cj) {
+                if (a.agg) {
+                    float best = Sb[cj];
+#pragma unroll
+                    for (int h = 1; h < G; ++h) best = fmaxf(best, Sb[h * a.Tc + cj]);
+                    return topk::make_key_signed(best, c_lo + cj);
+                }
                 float acc = 0.f;
 #pragma unroll
                 for (int h = 0; h < G; ++h) acc += ex2_approx(Sb[h * a.Tc + cj] - mx[h]) * iz[h];
@@ -537,7 +549,8 @@ cudaError_t launch_decode_select(const void* q, const void* Krepr, const int32_t
         return cudaErrorInvalidValue;
     const size_t smem = smem_bytes(G, Tc, p.topk, slots);
     Args args{static_cast<const __nv_bfloat16*>(q), lens, idx, cnt, status, s.Hq, s.Hkv, s.L, Tc,
-              p.topk, p.n_init, p.n_local, (int)units, slots, p.sm_scale * kLog2e};
+              p.topk, p.n_init, p.n_local, (int)units, slots, p.aggregation, p.sm_scale * kLog2e,
+              p.sm_scale};
     auto kern = G == 2 ? decode_select_tc_kernel<2> : decode_select_tc_kernel<1>;
     cudaError_t e;
     if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=

@@ -131,6 +131,8 @@ int phsa_step_host(const void* Q, const void* K, const void* V, const void* dO,
     if ((rc = phsa::validate_topk(s, p.topk)) != PHSA_OK) return rc;
     if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
     if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
+    if (p.aggregation != PHSA_AGG_SOFTMAX_SUM && p.aggregation != PHSA_AGG_MAX_LOGIT)
+        return PHSA_ERR_INVALID_ARG;
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (phsa::select_smem_bytes(s, p.topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
     cudaStream_t cs = static_cast<cudaStream_t>(stream);

@@ -84,6 +84,8 @@ int phsa_select_blocks(const void* Q, const void* Krepr, phsa_shape s, phsa_sele
     if (rc != PHSA_OK) return rc;
     if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
     if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
+    if (p.aggregation != PHSA_AGG_SOFTMAX_SUM && p.aggregation != PHSA_AGG_MAX_LOGIT)
+        return PHSA_ERR_INVALID_ARG;
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (empty(s)) return PHSA_OK;
     const bool need_repr = s.L >= 2 * phsa::kM;  // some query block has a candidate
@@ -163,6 +165,8 @@ int phsa_decode_select(const void* q, const void* Krepr, const int32_t* seq_lens
     if (rc != PHSA_OK) return rc;
     if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
     if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
+    if (p.aggregation != PHSA_AGG_SOFTMAX_SUM && p.aggregation != PHSA_AGG_MAX_LOGIT)
+        return PHSA_ERR_INVALID_ARG;
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (empty(s)) return PHSA_OK;
     const bool need_repr = s.L >= 2 * phsa::kM;  // some length can have a candidate
@@ -205,6 +209,8 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
     if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
     if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
     if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
+    if (p.aggregation != PHSA_AGG_SOFTMAX_SUM && p.aggregation != PHSA_AGG_MAX_LOGIT)
+        return PHSA_ERR_INVALID_ARG;
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (s.B == 0) return PHSA_OK;
     if (!q || !K || !V || !punct_mask || !seq_lens || !block_idx || !block_cnt || !O || !lse ||

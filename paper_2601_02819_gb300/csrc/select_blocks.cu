@@ -12,9 +12,12 @@
 //           then over warps in warp order, so equal columns get equal sums);
 //   top-k   min(topk - |F|, |C|) rounds of a block-wide argmax over the 64-bit
 //           key (bits(A) << 32 | ~t): larger A first, lower t on exact ties.
+// The max-logit rule (agg = 1) makes one pass: A[t] is the column maximum of
+// S = q . Krepr^T * scale over the group's rows (rows past L excluded).
 // Forced blocks are never scored; the output is ascending and -1 padded.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
+#include "topk.cuh"
 
 namespace phsa {
 
@@ -43,7 +46,7 @@ template <int G>
 __global__ void __launch_bounds__(SelCfg<G>::kThreads)
 select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ Krepr,
                      int Hq, int Hkv, int L, int T, int NQB, int topk, int n_init, int n_local,
-                     float scale_log2, int32_t* __restrict__ idx_out,
+                     int agg, float scale_log2, float scale, int32_t* __restrict__ idx_out,
                      int32_t* __restrict__ cnt_out) {
     using C = SelCfg<G>;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -101,10 +104,11 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
     uint32_t qf[8][4];
     float mrow[2] = {-INFINITY, -INFINITY}, zrow[2] = {0.f, 0.f}, inv_z[2] = {0.f, 0.f};
 
-    for (int pass = 0; pass < 2; ++pass) {
+    const int n_pass = agg ? 1 : 2;
+    for (int pass = 0; pass < n_pass; ++pass) {
         for (int j = 0; j < n_tiles; ++j) {
             const int it = pass * n_tiles + j;
-            if (it + 1 < 2 * n_tiles) {
+            if (it + 1 < n_pass * n_tiles) {
                 const int jn = (j + 1 < n_tiles) ? j + 1 : 0;
                 load_tile64<C::kThreads>(sK + ((it + 1) & 1) * C::kTileBytes, Kr, c_lo + jn * kM,
                                          c_hi + 1, tid);
@@ -134,16 +138,40 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
                     mma16816(acc[2 * np + 1], qf[kc], bb[2], bb[3]);
                 }
             }
-            // scale to the log2 domain and mask columns past the candidate range
+            // scale (to the log2 domain for the softmax) and mask columns past the
+            // candidate range; for max logits also the rows past L
             const int col0 = c_lo + j * kM + (lane & 3) * 2;
+            const float sc = agg ? scale : scale_log2;
 #pragma unroll
             for (int n = 0; n < 8; ++n)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const int t = col0 + n * 8 + (e & 1);
-                    acc[n][e] = (t <= c_hi) ? acc[n][e] * scale_log2 : -INFINITY;
+                    const bool row_ok = e < 2 ? row_ok0 : row_ok1;
+                    acc[n][e] = (t <= c_hi && (row_ok || !agg)) ? acc[n][e] * sc : -INFINITY;
                 }
-            if (pass == 0) {
+            if (agg) {
+                // column maxima over this warp's rows, then over the warps in warp order
+#pragma unroll
+                for (int n = 0; n < 8; ++n) {
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        float v = fmaxf(acc[n][e], acc[n][e + 2]);
+                        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+                        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+                        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
+                        if (lane < 4) part[warp * 64 + n * 8 + lane * 2 + e] = v;
+                    }
+                }
+                __syncthreads();
+                if (tid < kM) {
+                    float a = -INFINITY;
+#pragma unroll
+                    for (int w = 0; w < C::kWarps; ++w) a = fmaxf(a, part[w * 64 + tid]);
+                    const int c = j * kM + tid;
+                    if (c < nC) A[c] = a;
+                }
+            } else if (pass == 0) {
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
                     float mx = -INFINITY;
@@ -205,18 +233,15 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
         }
     }
 
-    // Top-k over A by (A desc, t asc). A >= 0, so its bit pattern orders like
-    // its value; a taken candidate is marked with -1.
+    // Top-k over A by (A desc, t asc) on keys whose unsigned order is that of
+    // A (topk.cuh); a taken candidate is marked by a NaN bit pattern that
+    // arithmetic never produces.
+    constexpr unsigned kTaken = 0xffffffffu;
     for (int r = 0; r < ksel; ++r) {
         unsigned long long best = 0ull;
         for (int c = tid; c < nC; c += C::kThreads) {
             const float a = A[c];
-            if (a >= 0.f) {
-                const unsigned long long key =
-                    ((unsigned long long)__float_as_uint(a) << 32) |
-                    (unsigned long long)(0xffffffffu - (unsigned)(c_lo + c));
-                best = u64_max(best, key);
-            }
+            if (__float_as_uint(a) != kTaken) best = u64_max(best, topk::make_key_agg(a, c_lo + c, agg != 0));
         }
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) {
@@ -231,7 +256,7 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
             // every untaken candidate has a nonzero key, so bb != 0 while r < ksel < nC
             const int t = bb ? (int)(0xffffffffu - (unsigned)(bb & 0xffffffffull)) : c_lo;
             sel[r] = t;
-            if (t >= c_lo && t <= c_hi) A[t - c_lo] = -1.0f;
+            if (t >= c_lo && t <= c_hi) A[t - c_lo] = __uint_as_float(kTaken);
         }
         __syncthreads();
     }
@@ -264,7 +289,8 @@ cudaError_t launch_select_g(const phsa_shape& s, const phsa_select_params& p, co
     ProfScope prof(K_SELECT, st);
     kern<<<(unsigned)grid, SelCfg<G>::kThreads, smem, st>>>(
         static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(Krepr), s.Hq,
-        s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, p.sm_scale * kLog2e, idx, cnt);
+        s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, p.aggregation, p.sm_scale * kLog2e,
+        p.sm_scale, idx, cnt);
     return cudaGetLastError();
 }
 

@@ -18,6 +18,9 @@
 //   top-k   a dedicated warp, on a double-buffered copy of A, while the
 //           elementwise warps already score the next unit: larger A first,
 //           lower t on exact ties (topk.cuh).
+// The max-logit rule (PHSA_AGG_MAX_LOGIT) needs no softmax statistics: it runs
+// pass 2 alone, each thread taking the largest score of its candidate over its
+// 64 rows (rows past L excluded), A[t] = max(half 0, half 1) * scale.
 // Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs,
 // warp 10 the top-k. The ring, the TMEM buffers and every barrier run on
 // counters that continue across units. Every wait is bounded in time.
@@ -55,8 +58,8 @@ struct SelArgs {
     int32_t* idx_out;
     int32_t* cnt_out;
     int* status;
-    int Hq, Hkv, L, T, NQB, topk, n_init, n_local, units;
-    float scale_log2;
+    int Hq, Hkv, L, T, NQB, topk, n_init, n_local, units, agg;
+    float scale_log2, scale;
 };
 
 // Everything about a unit that every role derives the same way.
@@ -135,7 +138,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
                 const SelUnit d = sel_unit(a, u);
                 if (!d.scored) continue;
-                const int steps = 2 * d.nch;
+                const int steps = (a.agg ? 1 : 2) * d.nch;
                 for (int s = 0; ok && s < steps; ++s, ++gs) {
                     const int slot = gs & 1, c = s % d.nch;
                     if (gs >= 2 && !mbar_wait(bar(B_KEMPTY + slot), ((gs >> 1) - 1) & 1, abort_flag, a.status)) {
@@ -179,7 +182,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 if (!d.scored) continue;
                 ok = mbar_wait(bar(B_Q), su & 1, abort_flag, a.status);
                 tc_fence_after();
-                const int steps = 2 * d.nch;
+                const int steps = (a.agg ? 1 : 2) * d.nch;
                 for (int s = 0; ok && s < steps; ++s, ++gs) {
                     const int slot = gs & 1;
                     ok = mbar_wait(bar(B_KFULL + slot), (gs >> 1) & 1, abort_flag, a.status) &&
@@ -187,7 +190,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     if (!ok) break;
                     tc_fence_after();
                     const uint64_t kr = sdesc_at(dKr0, slot * kTile);
-                    const bool pass1 = s < d.nch;
+                    const bool pass1 = !a.agg && s < d.nch;
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks) {
                         const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
@@ -232,14 +235,19 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
             float* A1 = A0 + a.NQB;
             // key = bits(A) << 32 | ~t, A = half 0 + half 1 (the same order for every
-            // candidate); each lane holds its candidates' keys in registers
+            // candidate) or, for max logits, the larger half; each lane holds its
+            // candidates' keys in registers
             const int nC = d.nC, ksel = d.ksel, c_lo = d.c_lo;
+            const bool mx = a.agg != 0;
+            auto key_of = [&](int cj) {
+                return topk::make_key_agg(mx ? fmaxf(A0[cj], A1[cj]) : A0[cj] + A1[cj], c_lo + cj, mx);
+            };
             if (nC <= 32 * kRegKeys) {
                 unsigned long long key[kRegKeys];
 #pragma unroll
                 for (int r = 0; r < kRegKeys; ++r) {
                     const int cj = lane + 32 * r;
-                    key[r] = cj < nC ? topk::make_key(A0[cj] + A1[cj], c_lo + cj) : 0ull;
+                    key[r] = cj < nC ? key_of(cj) : 0ull;
                 }
                 for (int k = 0; k < ksel; ++k) {
                     unsigned long long best = key[0];
@@ -255,10 +263,10 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                         if (key[r] == win) key[r] = 0ull;
                 }
             } else {
+                // a pick is marked by a NaN bit pattern that arithmetic never produces
                 topk::rounds_one_warp(
-                    nC, ksel, [&](int cj) { return topk::make_key(A0[cj] + A1[cj], c_lo + cj); },
-                    [&](int cj) { return A0[cj] == -1.0f; }, [&](int t) { A0[t - c_lo] = -1.0f; }, sel,
-                    lane);
+                    nC, ksel, key_of, [&](int cj) { return __float_as_uint(A1[cj]) == 0xffffffffu; },
+                    [&](int t) { A1[t - c_lo] = __uint_as_float(0xffffffffu); }, sel, lane);
             }
             __syncwarp();
             // A is no longer needed: the elementwise warps may refill this buffer
@@ -290,7 +298,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
         for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
             const SelUnit d = sel_unit(a, u);
             if (!d.scored) continue;
-            const int nch = d.nch, steps = 2 * nch, c_lo = d.c_lo, c_hi = d.c_hi, nC = d.nC;
+            const int nch = d.nch, steps = (a.agg ? 1 : 2) * nch, c_lo = d.c_lo, c_hi = d.c_hi, nC = d.nC;
             const bool row_ok = d.qb * 64 + (r & 63) < a.L;
             const int buf = su & 1;
             float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
@@ -307,7 +315,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     ok = __all_sync(0xffffffffu, ok);
                 }
                 if (ok) tc_fence_after();
-                if (ok && s < nch) {
+                if (ok && !a.agg && s < nch) {
                     // pass 1: row r against 64 candidates of the chunk, two loads of 32
                     const int t0 = c_lo + c * kCand + 64 * hh;
                     const bool full = t0 + 63 <= c_hi;
@@ -335,6 +343,27 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     }
                     tc_fence_before();
                     mbar_arrive(bar(B_SFREE + slot));
+                } else if (ok && a.agg) {
+                    // max logit: candidate r against the 64 rows of half hh (head hh)
+                    float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    const bool live = c * kCand + (warp & 3) * 32 < nC;
+#pragma unroll 1
+                    for (int q = 0; q < (live ? 2 : 0); ++q) {
+                        uint32_t v[32];
+                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+                        const int tok0 = d.qb * 64 + 32 * q;  // rows of head hh: tokens tok0 + j
+                        const bool all_rows = tok0 + 31 < a.L;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            const float x = (all_rows || tok0 + j < a.L) ? __uint_as_float(v[j]) : -INFINITY;
+                            mx4[j & 3] = fmaxf(mx4[j & 3], x);
+                        }
+                    }
+                    tc_fence_before();
+                    mbar_arrive(bar(B_SFREE + slot));
+                    const int cj = c * kCand + r;
+                    if (cj < nC)
+                        (hh ? A1 : A0)[cj] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * a.scale;
                 } else if (ok) {
                     // pass 2: candidate r against the 64 rows of half hh, in row order;
                     // a warp whose 32 candidates all lie past the last one skips the work
@@ -361,7 +390,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     const int cj = c * kCand + r;
                     if (cj < nC) (hh ? A1 : A0)[cj] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
                 }
-                if (s == nch - 1) {
+                if (!a.agg && s == nch - 1) {
                     // merge the two column halves of every row: (m, z) -> max and 1/sum
                     pm[hh * 128 + r] = m;
                     pz[hh * 128 + r] = z;
@@ -418,7 +447,7 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
     const int units = s.B * s.Hkv * NQB;
     const int per_sm = smem * 2 + 2048 <= 228 * 1024 ? 2 : 1;  // two CTAs when shared memory allows
     SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, units,
-                 p.sm_scale * kLog2e};
+                 p.aggregation, p.sm_scale * kLog2e, p.sm_scale};
     ProfScope prof(K_SELECT, st);
     select_tc_kernel<<<(unsigned)min(units, per_sm * nsm), kThreads, smem, st>>>(tq, tkr, args);
     return cudaGetLastError();

@@ -31,6 +31,23 @@ __device__ __forceinline__ unsigned long long make_key(float a, int t) {
            (unsigned long long)(0xffffffffu - (unsigned)t);
 }
 
+// The key of an aggregate of any sign (the max-logit rule): the float's bits
+// mapped so that unsigned order is numeric order (negatives flipped, the sign
+// bit set on the rest); -0 counts as +0 and NaN below every number. Every such
+// key is nonzero, so 0 still marks an empty slot.
+__device__ __forceinline__ unsigned long long make_key_signed(float a, int t) {
+    if (a != a) a = -INFINITY;
+    if (a == 0.f) a = 0.f;
+    unsigned u = __float_as_uint(a);
+    u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    return ((unsigned long long)u << 32) | (unsigned long long)(0xffffffffu - (unsigned)t);
+}
+
+// The key under either rule: summed probabilities (>= 0) or max logits.
+__device__ __forceinline__ unsigned long long make_key_agg(float a, int t, bool max_logit) {
+    return max_logit ? make_key_signed(a, t) : make_key(a, t);
+}
+
 __device__ __forceinline__ int key_block(unsigned long long key) {
     return (int)(0xffffffffu - (unsigned)(key & 0xffffffffull));
 }

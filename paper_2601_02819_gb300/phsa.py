@@ -38,7 +38,18 @@ class phsa_shape(ctypes.Structure):
 
 class phsa_select_params(ctypes.Structure):
     _fields_ = [("topk", ctypes.c_int), ("n_init", ctypes.c_int), ("n_local", ctypes.c_int),
-                ("sm_scale", ctypes.c_float)]
+                ("sm_scale", ctypes.c_float), ("aggregation", ctypes.c_int)]
+
+
+# PHSA_AGG_* of include/phsa.h: how a unit's query rows are combined per candidate
+AGGREGATIONS = {"softmax_sum": 0, "max_logit": 1}
+
+
+def _params(topk, n_init, n_local, sm_scale, aggregation) -> phsa_select_params:
+    if aggregation not in AGGREGATIONS:
+        raise ValueError(f"aggregation must be one of {sorted(AGGREGATIONS)}")
+    return phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale),
+                              AGGREGATIONS[aggregation])
 
 
 def library_path() -> str:
@@ -171,8 +182,10 @@ def phsa_build_block_repr(K, punct_mask, lam: float, Krepr=None, stream=None):
 
 def phsa_select_blocks(Q, Krepr, Hkv: int, topk: int, n_init: int = 1, n_local: int = 1,
                        sm_scale: float | None = None, block_idx=None, block_cnt=None,
-                       stream=None):
-    """Stage (b): (block_idx [B, Hkv, NQB, topk] int32, block_cnt [B, Hkv, NQB] int32)."""
+                       stream=None, aggregation: str = "softmax_sum"):
+    """Stage (b): (block_idx [B, Hkv, NQB, topk] int32, block_cnt [B, Hkv, NQB] int32).
+    ``aggregation``: "softmax_sum" (Eq. 8 probabilities summed over the unit's
+    rows) or "max_logit" (the largest raw score over the rows)."""
     _check(Q, "Q", torch.bfloat16, 4)
     _check(Krepr, "Krepr", torch.bfloat16, 4)
     B, Hq, L, D = Q.shape
@@ -185,7 +198,7 @@ def phsa_select_blocks(Q, Krepr, Hkv: int, topk: int, n_init: int = 1, n_local: 
         block_cnt = torch.empty((B, Hkv, NQB), dtype=torch.int32, device=Q.device)
     _check(block_idx, "block_idx", torch.int32, 4)
     _check(block_cnt, "block_cnt", torch.int32, 3)
-    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    p = _params(topk, n_init, n_local, sm_scale, aggregation)
     rc = load().phsa_select_blocks(_ptr(Q), _ptr(Krepr), make_shape(B, L, Hq, Hkv, D), p,
                                    _ptr(block_idx), _ptr(block_cnt), _stream(stream))
     _raise("phsa_select_blocks", rc)
@@ -282,7 +295,7 @@ def phsa_step_host_workspace(B, L, Hq, Hkv, topk, D=HEAD_DIM) -> int:
 def phsa_step_host(Q, K, V, dO, punct_mask, lam: float, topk: int, n_init: int = 1,
                    n_local: int = 1, sm_scale: float | None = None, O=None, lse=None, dQ=None,
                    dK=None, dV=None, block_idx=None, block_cnt=None, workspace=None,
-                   done_event=None, stream=None):
+                   done_event=None, stream=None, aggregation: str = "softmax_sum"):
     """One step of the whole path for HOST tensors (preferably pinned): stage (a),
     (b), the forward and the backward for dO, with the copies overlapped with the
     kernels inside the library. Q, K, V, dO: bf16 (or int16 holding bf16 bits) CPU
@@ -321,7 +334,7 @@ def phsa_step_host(Q, K, V, dO, punct_mask, lam: float, topk: int, n_init: int =
     if done_event is not None:
         done_event.record(stream)  # creates the CUDA event; the library records it again
         ev = ctypes.c_void_p(done_event.cuda_event)
-    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    p = _params(topk, n_init, n_local, sm_scale, aggregation)
     rc = load().phsa_step_host(_ptr(Q), _ptr(K), _ptr(V), _ptr(dO), _ptr(punct_mask),
                                make_shape(B, L, Hq, Hkv, D), float(lam), p, _ptr(O), _ptr(lse),
                                _ptr(dQ), _ptr(dK), _ptr(dV), _ptr(block_idx), _ptr(block_cnt),
@@ -400,7 +413,7 @@ def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=N
 
 def phsa_decode_select(q, Krepr, seq_lens, Lc: int, topk: int, n_init: int = 1,
                        n_local: int = 1, sm_scale: float | None = None, block_idx=None,
-                       block_cnt=None, stream=None):
+                       block_cnt=None, stream=None, aggregation: str = "softmax_sum"):
     """Decode selection for the new token of every sequence: q [B, Hq, D] bf16,
     Krepr [B, Hkv, Lc // 64, D]; returns (block_idx [B, Hkv, topk], block_cnt [B, Hkv])."""
     _check(q, "q", torch.bfloat16, 3)
@@ -416,7 +429,7 @@ def phsa_decode_select(q, Krepr, seq_lens, Lc: int, topk: int, n_init: int = 1,
         block_cnt = torch.empty((B, Hkv), dtype=torch.int32, device=q.device)
     _check(block_idx, "block_idx", torch.int32, 3)
     _check(block_cnt, "block_cnt", torch.int32, 2)
-    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    p = _params(topk, n_init, n_local, sm_scale, aggregation)
     rc = load().phsa_decode_select(_ptr(q), _ptr(Krepr), _ptr(seq_lens),
                                    make_shape(B, Lc, Hq, Hkv, D), p, _ptr(block_idx),
                                    _ptr(block_cnt), _stream(stream))
@@ -451,7 +464,8 @@ def phsa_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, sm_scale: float | 
 
 def phsa_decode_step(q, K, V, punct_mask, seq_lens, lam: float, Krepr, topk: int,
                      n_init: int = 1, n_local: int = 1, sm_scale: float | None = None,
-                     block_idx=None, block_cnt=None, O=None, lse=None, stream=None):
+                     block_idx=None, block_cnt=None, O=None, lse=None, stream=None,
+                     aggregation: str = "softmax_sum"):
     """One decode step in two launches (selection; attention fused with the
     refresh of the blocks the new tokens have just filled). q [B, Hq, D], K/V
     [B, Hkv, Lc, D] bf16 caches, punct_mask [B, Lc] uint8, seq_lens [B] int32,
@@ -475,7 +489,7 @@ def phsa_decode_step(q, K, V, punct_mask, seq_lens, lam: float, Krepr, topk: int
         O = torch.empty_like(q)
     if lse is None:
         lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device)
-    p = phsa_select_params(int(topk), int(n_init), int(n_local), float(sm_scale))
+    p = _params(topk, n_init, n_local, sm_scale, aggregation)
     rc = load().phsa_decode_step(_ptr(q), _ptr(K), _ptr(V), _ptr(punct_mask), _ptr(seq_lens),
                                  make_shape(B, Lc, Hq, Hkv, D), float(lam), p, _ptr(Krepr),
                                  _ptr(block_idx), _ptr(block_cnt), _ptr(O), _ptr(lse),
@@ -521,10 +535,10 @@ def phsa_selftest_tcgen05(A, B, V, stream=None):
 
 
 def phsa_forward(Q, K, V, punct_mask, lam: float, topk: int, n_init: int = 1, n_local: int = 1,
-                 sm_scale: float | None = None, stream=None):
+                 sm_scale: float | None = None, stream=None, aggregation: str = "softmax_sum"):
     """The whole forward hot path: (a) -> (b) -> (c). Returns (O, lse, block_idx, block_cnt, Krepr)."""
     Krepr = phsa_build_block_repr(K, punct_mask, lam, stream=stream)
     idx, cnt = phsa_select_blocks(Q, Krepr, K.shape[1], topk, n_init, n_local, sm_scale,
-                                  stream=stream)
+                                  stream=stream, aggregation=aggregation)
     O, lse = phsa_sparse_attn_fwd(Q, K, V, idx, cnt, sm_scale, stream=stream)
     return O, lse, idx, cnt, Krepr

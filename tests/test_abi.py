@@ -72,6 +72,8 @@ def test_host_validation_needs_no_gpu(lib):
     assert lib.phsa_select_blocks(None, None, ok, p, None, None, None) == -1
     p = phsa_select_params(8, 1, 0, 0.088)  # n_local must be >= 1
     assert lib.phsa_select_blocks(None, None, ok, p, None, None, None) == -1
+    p = phsa_select_params(8, 1, 1, 0.088, 2)  # no such aggregation rule
+    assert lib.phsa_select_blocks(None, None, ok, p, None, None, None) == -1
     assert lib.phsa_sparse_attn_bwd_workspace(ok, 14) > 0
     assert lib.phsa_sparse_attn_bwd_workspace(phsa_shape(1, 4096, 16, 8, 96, 64), 14) == 0
 

@@ -183,3 +183,31 @@ def test_decode_step_equals_the_three_calls(Hq, Hkv, n_init, n_local, topk):
         assert torch.equal(la, lb), step
         assert torch.equal(Kr_a.view(torch.int16), Kr_b.view(torch.int16)), step
     assert phsa.phsa_get_device_status() == 0
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(4, 2), (2, 2)])
+def test_decode_max_logit_rule_matches_oracle(Hq, Hkv):
+    Lc = 64 * 50 + 8
+    lens = [Lc, 64 * 41 + 1, 64 * 23, 64 * 9 + 17, 65, 1]
+    q, K, V, mask, lens = _case(77 + Hq, len(lens), Hq, Hkv, Lc, lens)
+    Kr = oracle.block_repr(K, mask, M, 0.5)
+    ld = torch.from_numpy(lens).cuda()
+    gi, gc = phsa.phsa_decode_select(to_dev_bf16(q), to_dev_bf16(Kr), ld, Lc, 6, 2, 2,
+                                     aggregation="max_logit")
+    oi, oc, oa = oracle.decode_select(q, Kr, lens, Lc, M, 6, 2, 2, SCALE, want_agg=True,
+                                      aggregation="max_logit")
+    torch.cuda.synchronize()
+    bad, excl, differ, msgs = compare_selection(gi.cpu().numpy().reshape(-1, 6),
+                                                gc.cpu().numpy().reshape(-1),
+                                                oi.reshape(-1, 6), oc.reshape(-1),
+                                                oa.reshape(len(oc.reshape(-1)), -1))
+    assert bad == 0, msgs[:5]
+    assert differ <= 1
+    # the fused step takes the same rule
+    Kd, Vd, md = to_dev_bf16(K), to_dev_bf16(V), torch.from_numpy(mask).cuda()
+    Krd = to_dev_bf16(Kr)
+    si, sc, O, lse = phsa.phsa_decode_step(to_dev_bf16(q), Kd, Vd, md, ld, 0.5, Krd, 6, 2, 2,
+                                           aggregation="max_logit")
+    torch.cuda.synchronize()
+    assert torch.equal(si, gi) and torch.equal(sc, gc)
+    assert phsa.phsa_get_device_status() == 0

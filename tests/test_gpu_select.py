@@ -103,3 +103,37 @@ def test_full_size_sampled_units(name):
                                                 gc.reshape(-1)[units], oi, oc, oa)
     assert bad == 0, msgs[:5]
     assert differ <= max(2, 0.02 * len(units)), (differ, len(units))
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,L,topk,n_init,n_local", [
+    (2, 4, 2, 64 * 37 + 13, 6, 1, 1),   # G = 2, ragged tail (rows past L excluded)
+    (1, 3, 3, 64 * 40 + 9, 9, 2, 3),    # G = 1
+    (1, 2, 1, 64 * 300, 14, 2, 8),      # G = 2, paper forced sets, several candidate tiles
+    (1, 2, 1, 64 * 160, 80, 1, 1),      # G = 2, budget above the two-level top-k limit
+])
+def test_max_logit_rule_matches_oracle(B, Hq, Hkv, L, topk, n_init, n_local):
+    rng = np.random.default_rng(B * 7 + L)
+    Q = inputs.f32_to_bf16_bits(rng.standard_normal((B, Hq, L, 128)).astype(np.float32))
+    K = inputs.f32_to_bf16_bits(rng.standard_normal((B, Hkv, L, 128)).astype(np.float32))
+    mask = (rng.random((B, L)) < 0.06).astype(np.uint8)
+    Kr = oracle.block_repr(K, mask, 64, 0.5)
+    scale = 128 ** -0.5
+    idx, cnt = phsa.phsa_select_blocks(to_dev_bf16(Q), to_dev_bf16(Kr), Hkv, topk, n_init,
+                                       n_local, scale, aggregation="max_logit")
+    torch.cuda.synchronize()
+    oi, oc, oa = oracle.select_blocks(Q, Kr, L, 64, topk, n_init, n_local, scale, want_agg=True,
+                                      aggregation="max_logit")
+    bad, excl, differ, msgs = compare_selection(idx.cpu().numpy(), cnt.cpu().numpy(), oi, oc, oa)
+    assert bad == 0, msgs[:5]
+    assert differ <= max(2, 0.01 * oc.size), (differ, oc.size)
+    # the rule changes the choice: the softmax-sum selection differs somewhere
+    si, _ = phsa.phsa_select_blocks(to_dev_bf16(Q), to_dev_bf16(Kr), Hkv, topk, n_init, n_local,
+                                    scale)
+    assert not torch.equal(si, idx)
+
+
+def test_unknown_aggregation_is_rejected():
+    Q = torch.zeros((1, 2, 128, 128), dtype=torch.bfloat16, device="cuda")
+    Kr = torch.zeros((1, 1, 2, 128), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(ValueError):
+        phsa.phsa_select_blocks(Q, Kr, 1, 2, aggregation="mean")
