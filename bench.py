@@ -18,6 +18,7 @@ workload on this host's cores.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import os
@@ -179,7 +180,7 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- oracle sample
-def oracle_sample_step(w, x, n_units: int, seed: int):
+def oracle_sample_step(w, x, n_units: int, seed: int, aggregation: str = "softmax_sum"):
     """Times the CPU oracle on a bounded sample of one step; returns estimated seconds
     for the whole step, the parts and a description.
 
@@ -213,7 +214,8 @@ def oracle_sample_step(w, x, n_units: int, seed: int):
     Kr = oracle.block_repr(x["K"], x["mask"], w.block_size, w.lam)
     t["repr"] = time.perf_counter() - t0
     t0 = time.perf_counter()
-    oracle.select_units(x["Q"], Kr, w.L, w.block_size, w.topk, w.n_init, w.n_local, scale, units)
+    oracle.select_units(x["Q"], Kr, w.L, w.block_size, w.topk, w.n_init, w.n_local, scale, units,
+                        aggregation=aggregation)
     cand_all = w.B * w.Hkv * float(np.sum(np.arange(1, w.NQB + 1)))
     t["select"] = (time.perf_counter() - t0) * cand_all / float(np.sum(qbs + 1))
     rows = []
@@ -278,6 +280,14 @@ def oracle_threads():
 
 
 # ---------------------------------------------------------------- GPU arm
+def workload_of(args, table):
+    """The named workload, with the paper's forced-set sizes when asked for."""
+    w = table[args.workload]
+    if args.forced == "paper":  # 128 initial + 512 local tokens at m = 64
+        w = dataclasses.replace(w, name=w.name + "_paper_forced", n_init=2, n_local=8)
+    return w
+
+
 def run_ours(args):
     from paper_2601_02819_gb300 import phsa
     rank, world, local = dist_env()
@@ -288,7 +298,7 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    w = inputs.WORKLOADS[args.workload]
+    w = workload_of(args, inputs.WORKLOADS)
     # weak scaling: every rank runs one batch of the workload on its own sequences
     mine = shard_sequences(world * w.B, world, rank)
     x = inputs.make_inputs(w, with_grad=True, seed=rank_seed(w.seed, mine[0]))
@@ -311,7 +321,7 @@ def run_ours(args):
     def step():
         phsa.phsa_build_block_repr(K, mask, w.lam, Krepr=Kr)
         phsa.phsa_select_blocks(Q, Kr, w.Hkv, w.topk, w.n_init, w.n_local, w.sm_scale,
-                                block_idx=idx, block_cnt=cnt)
+                                block_idx=idx, block_cnt=cnt, aggregation=args.aggregation)
         phsa.phsa_sparse_attn_fwd(Q, K, V, idx, cnt, w.sm_scale, O=O, lse=lse)
         phsa.phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, idx, cnt, w.sm_scale, workspace=ws,
                                   dQ=dQ, dK=dK, dV=dV)
@@ -373,7 +383,7 @@ def run_ours(args):
             # two workspaces alternate, so one step's copies overlap the other's kernels
             phsa.phsa_step_host(hQ, hK, hV, hdO, hmask, w.lam, w.topk, w.n_init, w.n_local,
                                 w.sm_scale, workspace=wss[i % 2], done_event=evs[i % 2],
-                                stream=stream, **outs[i % 2])
+                                stream=stream, aggregation=args.aggregation, **outs[i % 2])
 
         for i in range(2):
             e2e_step(i)
@@ -451,7 +461,8 @@ def run_ours(args):
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         cores = oracle_threads()
-        est_s, parts, desc = oracle_sample_step(w, x, args.cpu_units, seed=5)
+        est_s, parts, desc = oracle_sample_step(w, x, args.cpu_units, seed=5,
+                                                aggregation=args.aggregation)
         cpu = {"value": w.B * w.L / est_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                "sample": desc, "est_s_per_step": round(est_s, 2),
                "parts_s": {k: round(v, 3) for k, v in parts.items()}}
@@ -463,7 +474,7 @@ def run_ours(args):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "B": w.B, "L": w.L, "Hq": w.Hq, "Hkv": w.Hkv, "D": w.D,
                    "block_size": w.block_size, "topk": w.topk, "n_init": w.n_init,
-                   "n_local": w.n_local, "lambda": w.lam,
+                   "n_local": w.n_local, "lambda": w.lam, "aggregation": args.aggregation,
                    "sparsity": round(1 - w.topk * w.block_size / w.L, 5),
                    "step": "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)",
                    "l2": "inputs larger than L2 (Q 134 MB, K 67 MB, V 67 MB, dO 134 MB per step)",
@@ -516,7 +527,7 @@ def decode_algorithmic(w, lens: np.ndarray, cnt: np.ndarray):
             "decode_attn": {"flops": 4.0 * D * keys * w.G, "bytes": float(att + rep)}}
 
 
-def oracle_decode_sample(w, x, n_units: int, seed: int):
+def oracle_decode_sample(w, x, n_units: int, seed: int, aggregation: str = "softmax_sum"):
     """Times the oracle on `n_units` random (sequence, KV head) units of one
     decode step (the just-filled block's repr, the selection, the attention)
     and scales to the whole batch. Representative keys of the cached blocks are
@@ -538,7 +549,7 @@ def oracle_decode_sample(w, x, n_units: int, seed: int):
         if L % m == 0:
             oracle.block_repr(Kbg[:, :, L - m:L], mb[:, L - m:L], m, w.lam)
         idx, cnt = oracle.decode_select(qbg, Kr, lb, w.L, m, w.topk, w.n_init, w.n_local,
-                                        w.sm_scale)
+                                        w.sm_scale, aggregation=aggregation)
         oracle.decode_attn(qbg, Kbg, Vbg, idx, cnt, lb, m, w.sm_scale)
         secs += time.perf_counter() - t0
     est = secs * U / len(units)
@@ -557,7 +568,7 @@ def run_decode(args):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    w = inputs.DECODE_WORKLOADS[args.workload]
+    w = workload_of(args, inputs.DECODE_WORKLOADS)
     x = inputs.make_decode_inputs(w, dev, seed=rank_seed(w.seed, rank * w.B))
     q, K, V, mask, lens = x["q"], x["K"], x["V"], x["mask_dev"], x["lens_dev"]
     Kr = phsa.phsa_build_block_repr(K, mask, w.lam)  # the cache's prefill: not part of a step
@@ -577,7 +588,8 @@ def run_decode(args):
 
     def step():  # selection; attention fused with the refresh of just-filled blocks
         phsa.phsa_decode_step(q, K, V, mask, lens, w.lam, Kr, w.topk, w.n_init, w.n_local,
-                              w.sm_scale, block_idx=idx, block_cnt=cnt, O=O, lse=lse)
+                              w.sm_scale, block_idx=idx, block_cnt=cnt, O=O, lse=lse,
+                              aggregation=args.aggregation)
 
     def barrier():
         if world > 1:
@@ -698,7 +710,8 @@ def run_decode(args):
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         cores = oracle_threads()
-        est, desc = oracle_decode_sample(w, x, args.cpu_units, seed=5)
+        est, desc = oracle_decode_sample(w, x, args.cpu_units, seed=5,
+                                         aggregation=args.aggregation)
         cpu = {"value": w.B / est, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                "sample": desc, "est_s_per_step": round(est, 3)}
     return {
@@ -708,7 +721,7 @@ def run_decode(args):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "B": w.B, "cache_len": w.L, "Hq": w.Hq, "Hkv": w.Hkv,
                    "D": w.D, "block_size": w.block_size, "topk": w.topk, "n_init": w.n_init,
-                   "n_local": w.n_local, "lambda": w.lam,
+                   "n_local": w.n_local, "lambda": w.lam, "aggregation": args.aggregation,
                    "step": "decode (phsa_decode_step): selection, then attention fused with the refresh of the just-filled block's representative key",
                    "l2": "flushed before every step, outside the timed events: 256 MB written, then 256 MB of another buffer read (no dirty flush line is written back inside the step)",
                    "parallelism": f"dp{world} (independent sequences)"},
@@ -730,16 +743,17 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return None
-    w = inputs.WORKLOADS[args.workload]
+    w = workload_of(args, inputs.WORKLOADS)
     x = inputs.make_inputs(w, with_grad=True)
     cores = oracle_threads()
     n_units = max(args.ref_units, cores)  # at least one unit per thread
     for s in range(args.warmup):
-        oracle_sample_step(w, x, n_units, seed=100 + s)
+        oracle_sample_step(w, x, n_units, seed=100 + s, aggregation=args.aggregation)
     ests, descs = [], None
     t0 = time.perf_counter()
     for s in range(args.steps):
-        est, _, descs = oracle_sample_step(w, x, n_units, seed=1000 + s)
+        est, _, descs = oracle_sample_step(w, x, n_units, seed=1000 + s,
+                                           aggregation=args.aggregation)
         ests.append(est)
     wall = time.perf_counter() - t0
     est = statistics.mean(ests)
@@ -750,7 +764,8 @@ def run_reference(args):
         "ms_per_step": est * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "B": w.B, "L": w.L, "Hq": w.Hq, "Hkv": w.Hkv, "D": w.D,
-                   "block_size": w.block_size, "topk": w.topk,
+                   "block_size": w.block_size, "topk": w.topk, "n_init": w.n_init,
+                   "n_local": w.n_local, "lambda": w.lam, "aggregation": args.aggregation,
                    "step": "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)"},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                          "sample": descs},
@@ -768,6 +783,10 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="prefill_32k",
                     choices=sorted(inputs.WORKLOADS) + sorted(inputs.DECODE_WORKLOADS))
+    ap.add_argument("--aggregation", choices=["softmax_sum", "max_logit"], default="softmax_sum",
+                    help="how a unit's query rows are combined per candidate block")
+    ap.add_argument("--forced", choices=["workload", "paper"], default="workload",
+                    help="forced blocks: the workload's, or the paper's 2 initial + 8 local")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-units", type=int, default=48,

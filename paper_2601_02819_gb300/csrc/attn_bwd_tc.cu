@@ -249,12 +249,17 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         if (lane == 0) {
             prefetch_tmap(&tmQ);
             prefetch_tmap(&tmdO);
+            const int ls = list_stride(a.topk);
+            int* elists = reinterpret_cast<int*>(smem + kOffList) + kListE * ls;
             int ul = 0, last = -1;
             for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
                 if (ul > 0 && !mbar_wait(bar(B_QFREE), (ul - 1) & 1, abort_flag, a.status)) break;
                 last = ul;
                 const DqUnit d = dq_unit(a, u);
-                mbar_expect_tx(bar(B_Q), 2 * kTile128);
+                // The tiles first; then the elementwise warps' copy of the block list
+                // (its slot's previous unit is done: they have passed that unit's
+                // Delta), published by this thread's arrival on B_Q.
+                mbar_expect_tx_only(bar(B_Q), 2 * kTile128);
                 for (int hl = 0; hl < 2; ++hl)
                     for (int dh = 0; dh < 2; ++dh) {
                         tma_load_3d(sb + kOffQ + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_Q),
@@ -262,6 +267,9 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                         tma_load_3d(sb + kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(B_Q),
                                     dh * 64, d.qb * 64, d.hq0 + hl);
                     }
+                int* el = elists + (ul & 1) * ls;
+                el[ls - 1] = stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, el);
+                mbar_arrive(bar(B_Q));
                 // The next unit's Q and dO come from HBM: start bringing them into L2
                 // now, a whole unit before they are loaded.
                 const int u2 = u + (int)gridDim.x;
@@ -397,15 +405,13 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         int gp0 = 0, ul = 0;
         const int ls = list_stride(a.topk);
         int* lists = reinterpret_cast<int*>(smem + kOffList) + kListE * ls;
-        // A unit's inputs that come from global memory (its block list, staged by
-        // thread 0; O rows and lse for Delta and P) are fetched during the
-        // previous unit, so that they are in hand when its Q and dO arrive.
+        // A unit's O rows and lse (for Delta and P) are fetched at the end of the
+        // previous unit, so that they are in hand when its Q and dO arrive; its
+        // block list is staged by the Q/dO producer before it arrives on B_Q.
         uint4 ov[8];
         float neg_lse2 = 0.f;
-        auto fetch_unit = [&](int u, int slot) {
+        auto fetch_unit = [&](int u) {
             const DqUnit d = dq_unit(a, u);
-            if (et == 0) lists[slot * ls + ls - 1] = stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu,
-                                                                a.topk, d.qb, lists + slot * ls);
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
                 const int rr = k * 16 + (et >> 4);
@@ -417,7 +423,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const int i = d.qb * 64 + tok;
             neg_lse2 = i < a.L ? -__ldg(a.lse + (size_t)(d.hq0 + hl) * a.L + i) * kLog2e : -INFINITY;
         };
-        if (blockIdx.x < a.units) fetch_unit(blockIdx.x, 0);
+        if (blockIdx.x < a.units) fetch_unit(blockIdx.x);
         // Every warp runs every unit (doing no work after an abort), so the one
         // named barrier per unit is reached the same number of times by all.
         for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
@@ -472,7 +478,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
                 if (pc == 0) dpart[rr] = acc;
             }
-            named_barrier(1, 256);  // Delta's pieces and this unit's list are visible
+            named_barrier(1, 256);  // Delta's pieces are visible
             const float dlt = dpart[row];
             // This thread is done with dO and with Delta's exchange slots: the next
             // unit's dO may be loaded (and dpart rewritten) once all have arrived.
@@ -516,7 +522,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             gp0 += np;
             // the next unit's inputs: their latency overlaps this unit's last dQ
             // MMAs and its epilogue
-            if (u2 < a.units) fetch_unit(u2, (ul + 1) & 1);
+            if (u2 < a.units) fetch_unit(u2);
             if (ok) {
                 ok = mbar_wait(bar(B_FINAL), ul & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
