@@ -1,13 +1,19 @@
 // Stage (c) forward on the 5th-generation tensor cores (tcgen05 + TMEM + TMA),
 // for GQA groups of two query heads (G*64 = 128 query rows per tile).
 //
-// One CTA per (query block qb, KV head g), 224 threads in four roles:
-//   warp 4 (one lane)  TMA producer of Q (the 128 x 128 tile, once) and of the
-//                      selected K tiles (64 x 128, gathered by block index)
-//                      into a two-slot ring; a slot is refilled as soon as the
-//                      QK MMA that read it has finished.
-//   warp 6 (one lane)  TMA producer of the selected V tiles into their own
-//                      two-slot ring, refilled when the PV MMA is done.
+// Persistent: two CTAs per SM, each walking the units (query block qb, KV
+// head g) u = blockIdx.x, blockIdx.x + gridDim.x, ... with 256 threads in
+// five roles; rings, TMEM buffers and barriers run on counters that continue
+// across units, so one unit's loads and first MMAs overlap the previous
+// unit's last blocks and epilogue:
+//   warp 4 (one lane)  stages each unit's block list into one of four list
+//                      slots, a unit ahead, and gathers the selected K tiles
+//                      (64 x 128, by block index) into a two-slot ring; a slot
+//                      is refilled as soon as the QK MMA that read it is done.
+//   warp 6 (one lane)  loads each unit's Q tile (128 x 128) once the previous
+//                      unit's last QK MMA is done, and the selected V tiles
+//                      into their own two-slot ring, refilled when the PV MMA
+//                      is done.
 //   warp 5 (one lane)  MMA issuer: S_j = Q K_j^T (M=128, N=64, K=128) into one
 //                      of two TMEM score buffers, and O += P_j V_j (M=128,
 //                      N=128, K=64) with P_j read from TMEM. It polls and issues
@@ -21,8 +27,10 @@
 //                      TMEM. O is rescaled in TMEM only when the block max
 //                      exceeds the running max by more than 2^8 (exact: the
 //                      final normalisation uses the same running max).
-//                      Epilogue: O / l -> bf16 -> shared memory -> TMA store;
-//                      LSE = (max + log2 l) ln 2.
+//                      Epilogue: O / l -> bf16 rows stored from registers;
+//                      LSE = (max + log2 l) ln 2. O's TMEM columns are handed
+//                      back to the next unit's first PV once read.
+//   warp 7             idle (keeps the softmax warps on TMEM lane groups 0-3).
 // TMEM: O in columns [0,128), score buffers in [128,192) and [192,256).
 // Every wait is bounded in time (tc_common.cuh); on expiry the kernel records
 // PHSA_ERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and returns.
@@ -46,59 +54,81 @@ constexpr int kOffK = kQBytes;                        // K slots
 constexpr int kOffV = kOffK + kSlots * kKBytes;       // V slots
 constexpr int kOffBar = kOffV + kSlots * kKBytes;
 // barriers
-constexpr int B_Q = 0;
-constexpr int B_KFULL = 1;                  // + slot
+constexpr int B_Q = 0;                      // this unit's Q tile landed
+constexpr int B_QFREE = 1;                  // the unit's last QK MMA is done
+constexpr int B_KFULL = 2;                  // + slot
 constexpr int B_KEMPTY = B_KFULL + kSlots;
 constexpr int B_VFULL = B_KEMPTY + kSlots;
 constexpr int B_VEMPTY = B_VFULL + kSlots;
 constexpr int B_SFULL = B_VEMPTY + kSlots;  // + buffer
 constexpr int B_PFULL = B_SFULL + 2;
 constexpr int B_PVDONE = B_PFULL + 2;
-constexpr int B_OFINAL = B_PVDONE + 1;
-constexpr int B_DRAIN = B_OFINAL + 1;
+constexpr int B_OFINAL = B_PVDONE + 1;      // the unit's last PV MMA is done
+constexpr int B_OFREE = B_OFINAL + 1;       // the softmax warps have read O out
+constexpr int kListSlots = 4;
+constexpr int B_UFULL = B_OFREE + 1;        // + list slot
+constexpr int B_UFREE = B_UFULL + kListSlots;
+constexpr int B_DRAIN = B_UFREE + kListSlots;
 constexpr int kNumBars = B_DRAIN + 1;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag, block count
-constexpr int kOffList = kOffMisc + 16;
-constexpr int kThreads = 224;
+constexpr int kOffMisc = kOffBar + ((kNumBars * 8 + 15) & ~15);  // tmem base, abort flag
+constexpr int kOffList = kOffMisc + 16;     // list slots: count, then the compacted list
+constexpr int kThreads = 256;
+constexpr int kUFreeCount = 3 + 128;        // K producer, V producer, MMA thread, softmax threads
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kColO = 0;
 constexpr float kRescaleLog2 = 8.0f;
+static_assert(kOffBar + kNumBars * 8 <= kOffMisc, "barrier region");
 
+__host__ __device__ constexpr int list_slot_ints(int topk) { return (topk + 4) & ~3; }
 __host__ __device__ constexpr size_t fwd_tc_smem(int topk) {
-    return 1024 + (size_t)kOffList + (size_t)(topk + 1) * 4;
+    return 1024 + (size_t)kOffList + kListSlots * (size_t)list_slot_ints(topk) * 4;
 }
 
 struct FwdTcArgs {
     const int32_t* idx;
     const int32_t* cnt;
+    __nv_bfloat16* O;
     float* lse;
     int* status;
-    int Hq, Hkv, L, NQB, topk;
+    int Hq, Hkv, L, NQB, topk, units;
     float scale_log2;
 };
+
+struct FwdUnit {
+    int qb, bg, hq0;
+    long long lu;
+};
+
+__device__ __forceinline__ FwdUnit fwd_unit(const FwdTcArgs& a, int u) {
+    FwdUnit d;
+    d.qb = a.NQB - 1 - (u % a.NQB);  // heaviest query blocks first
+    d.bg = u / a.NQB;
+    d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
+    d.lu = (long long)d.bg * a.NQB + d.qb;
+    return d;
+}
 
 __device__ __forceinline__ uint32_t col_s(int buf) { return 128u + 64u * (uint32_t)buf; }
 
 __global__ void __launch_bounds__(kThreads, 2)
 attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
-                   const FwdTcArgs a) {
+                   const __grid_constant__ CUtensorMap tmV, const FwdTcArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     const uint32_t sb = smem_u32(smem);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int unit = blockIdx.x;
-    const int qb = a.NQB - 1 - (unit % a.NQB);
-    const int bg = unit / a.NQB;
-    const int b = bg / a.Hkv, g = bg % a.Hkv;
-    const long long lu = (long long)bg * a.NQB + qb;
     auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
-    int* list = reinterpret_cast<int*>(smem + kOffList);
+    const int lsi = list_slot_ints(a.topk);
+    auto slot_ptr = [&](int k) {
+        return reinterpret_cast<int*>(smem + kOffList) + (k % kListSlots) * lsi;
+    };
+    auto unit_of = [&](int k) { return (int)blockIdx.x + k * (int)gridDim.x; };
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_Q), 1);
+        mbar_init(bar(B_QFREE), 1);
         for (int s = 0; s < kSlots; ++s) {
             mbar_init(bar(B_KFULL + s), 1);
             mbar_init(bar(B_KEMPTY + s), 1);
@@ -109,13 +139,16 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             mbar_init(bar(B_SFULL + i), 1);
             mbar_init(bar(B_PFULL + i), 128);
         }
+        for (int i = 0; i < kListSlots; ++i) {
+            mbar_init(bar(B_UFULL + i), 1);
+            mbar_init(bar(B_UFREE + i), kUFreeCount);
+        }
         mbar_init(bar(B_PVDONE), 1);
         mbar_init(bar(B_OFINAL), 1);
+        mbar_init(bar(B_OFREE), 128);
         mbar_init(bar(B_DRAIN), 1);
         fence_barrier_init();
         *abort_flag = 0;
-        reinterpret_cast<int*>(smem + kOffMisc)[2] =
-            compact_block_list(a.idx + lu * a.topk, a.cnt[lu], a.topk, qb, list, a.status);
     }
     if (warp == 5) {
         tmem_alloc(sb + kOffMisc, kTmemCols);
@@ -125,182 +158,269 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
-    const int n = reinterpret_cast<volatile int*>(smem + kOffMisc)[2];
-    const int hq0 = b * a.Hq + g * 2;  // first query head (plane) of the group
 
-    if (warp == 4 || warp == 6) {
-        // ------------------------------------------------ TMA producers (K / V)
-        if (lane == 0 && n > 0) {
-            const bool is_k = warp == 4;
-            const CUtensorMap* map = is_k ? &tmK : &tmV;
-            prefetch_tmap(map);
-            if (is_k) {
-                prefetch_tmap(&tmQ);
+    if (warp == 4) {
+        // ------------------------------------------------ lists and K tiles
+        if (lane == 0) {
+            prefetch_tmap(&tmK);
+            // unit k's compacted list into its slot, once every role is done with
+            // the slot's previous unit (k - kListSlots)
+            auto stage = [&](int k) {
+                const int ls = k % kListSlots;
+                if (k >= kListSlots &&
+                    !mbar_wait(bar(B_UFREE + ls), ((k / kListSlots) - 1) & 1, abort_flag, a.status))
+                    return false;
+                const FwdUnit d = fwd_unit(a, unit_of(k));
+                int* sl = slot_ptr(k);
+                sl[0] = compact_block_list(a.idx + d.lu * a.topk, a.cnt[d.lu], a.topk, d.qb, sl + 1,
+                                           a.status);
+                mbar_arrive(bar(B_UFULL + ls));
+                return true;
+            };
+            bool ok = unit_of(0) >= a.units || stage(0);
+            int gk = 0;  // K loads issued, over all units
+            for (int k = 0; ok && unit_of(k) < a.units; ++k) {
+                const FwdUnit d = fwd_unit(a, unit_of(k));
+                const int* sl = slot_ptr(k);
+                const int n = sl[0];
+                bool staged = false;  // the next unit's list, once this unit's ring is full
+                for (int j = 0; j < n; ++j, ++gk) {
+                    if (j == kSlots && unit_of(k + 1) < a.units) {
+                        if (!(ok = stage(k + 1))) break;
+                        staged = true;
+                    }
+                    const int s = gk % kSlots;
+                    if (gk >= kSlots &&
+                        !mbar_wait(bar(B_KEMPTY + s), ((gk / kSlots) - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(bar(B_KFULL + s), kKBytes);
+                    for (int dh = 0; dh < 2; ++dh)
+                        tma_load_3d(sb + kOffK + s * kKBytes + dh * kKVHalf, &tmK, bar(B_KFULL + s),
+                                    dh * 64, sl[1 + j] * 64, d.bg);
+                }
+                if (!ok) break;
+                if (!staged && unit_of(k + 1) < a.units) ok = stage(k + 1);
+                mbar_arrive(bar(B_UFREE + k % kListSlots));
+            }
+            // Own copies must have landed before the CTA may exit.
+            for (int g = gk - kSlots; g < gk; ++g)
+                if (g >= 0) mbar_wait_drain(bar(B_KFULL + g % kSlots), (g / kSlots) & 1);
+        }
+    } else if (warp == 6) {
+        // ------------------------------------------------ Q and V tiles
+        if (lane == 0) {
+            prefetch_tmap(&tmQ);
+            prefetch_tmap(&tmV);
+            int gv = 0, q_last = -1;  // V loads issued; last unit whose Q was loaded
+            bool ok = true;
+            for (int k = 0; ok && unit_of(k) < a.units; ++k) {
+                const FwdUnit d = fwd_unit(a, unit_of(k));
+                ok = mbar_wait(bar(B_UFULL + k % kListSlots), (k / kListSlots) & 1, abort_flag, a.status);
+                if (!ok) break;
+                const int* sl = slot_ptr(k);
+                const int n = sl[0];
+                // Q once the previous unit's last QK MMA has read the old tile
+                if (k >= 1 && !mbar_wait(bar(B_QFREE), (k - 1) & 1, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
                 mbar_expect_tx(bar(B_Q), kQBytes);
                 for (int hl = 0; hl < 2; ++hl)
                     for (int dh = 0; dh < 2; ++dh)
                         tma_load_3d(sb + kOffQ + dh * kHalfQ + hl * (kHalfQ / 2), &tmQ, bar(B_Q),
-                                    dh * 64, qb * 64, hq0 + hl);
+                                    dh * 64, d.qb * 64, d.hq0 + hl);
+                q_last = k;
+                for (int j = 0; j < n; ++j, ++gv) {
+                    const int s = gv % kSlots;
+                    if (gv >= kSlots &&
+                        !mbar_wait(bar(B_VEMPTY + s), ((gv / kSlots) - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(bar(B_VFULL + s), kKBytes);
+                    for (int dh = 0; dh < 2; ++dh)
+                        tma_load_3d(sb + kOffV + s * kKBytes + dh * kKVHalf, &tmV, bar(B_VFULL + s),
+                                    dh * 64, sl[1 + j] * 64, d.bg);
+                }
+                if (!ok) break;
+                mbar_arrive(bar(B_UFREE + k % kListSlots));
             }
-            const int full = is_k ? B_KFULL : B_VFULL, empty = is_k ? B_KEMPTY : B_VEMPTY;
-            const uint32_t ring = sb + (is_k ? kOffK : kOffV);
-            int issued = 0;
-            for (int j = 0; j < n; ++j) {
-                const int s = j % kSlots;
-                if (j >= kSlots &&
-                    !mbar_wait(bar(empty + s), ((j / kSlots) - 1) & 1, abort_flag, a.status))
-                    break;
-                const int t = list[j];
-                mbar_expect_tx(bar(full + s), kKBytes);
-                for (int dh = 0; dh < 2; ++dh)
-                    tma_load_3d(ring + s * kKBytes + dh * kKVHalf, map, bar(full + s), dh * 64,
-                                t * 64, bg);
-                issued = j + 1;
-            }
-            // Own copies must have landed before the CTA may exit.
-            if (is_k) mbar_wait_drain(bar(B_Q), 0);
-            for (int j = issued - kSlots; j < issued; ++j)
-                if (j >= 0) mbar_wait_drain(bar(full + j % kSlots), (j / kSlots) & 1);
+            if (q_last >= 0) mbar_wait_drain(bar(B_Q), q_last & 1);
+            for (int g = gv - kSlots; g < gv; ++g)
+                if (g >= 0) mbar_wait_drain(bar(B_VFULL + g % kSlots), (g / kSlots) & 1);
         }
     } else if (warp == 5) {
         // ------------------------------------------------ MMA issuer
-        if (lane == 0 && n > 0) {
+        if (lane == 0) {
             constexpr uint32_t idesc_qk = idesc_bf16(128, 64, false);
             constexpr uint32_t idesc_pv = idesc_bf16(128, 128, true);
             const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
             const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
             const uint64_t dV0 = sdesc_sw128(sb + kOffV, kKVHalf, 1024);
-            bool ok = mbar_wait(bar(B_Q), 0, abort_flag, a.status);
-            tc_fence_after();
-            int nq = 0, np = 0;  // next QK and next PV to issue
-            Deadline dl;
-            while (ok && np < n) {
-                bool progressed = false;
-                // QK_nq reuses score buffer nq&1, free once PV_{nq-2} has been issued.
-                if (nq < n && nq <= np + 1 && mbar_test_wait(bar(B_KFULL + nq % kSlots), (nq / kSlots) & 1)) {
-                    tc_fence_after();
-                    const uint64_t kd = sdesc_at(dK0, (nq % kSlots) * kKBytes);
-                    const uint32_t d = tmem + col_s(nq & 1);
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(d, sdesc_at(dQ0, (ks >> 2) * kHalfQ + (ks & 3) * 32),
-                               sdesc_at(kd, (ks >> 2) * kKVHalf + (ks & 3) * 32), idesc_qk,
-                               ks > 0 ? 1u : 0u);
-                    mma_commit(bar(B_SFULL + (nq & 1)));
-                    mma_commit(bar(B_KEMPTY + nq % kSlots));
-                    ++nq;
-                    progressed = true;
+            int g0 = 0;  // blocks of the previous units (QK and PV MMAs issued so far)
+            bool ok = true;
+            for (int k = 0; ok && unit_of(k) < a.units; ++k) {
+                ok = mbar_wait(bar(B_UFULL + k % kListSlots), (k / kListSlots) & 1, abort_flag, a.status);
+                if (!ok) break;
+                const int n = slot_ptr(k)[0];
+                mbar_arrive(bar(B_UFREE + k % kListSlots));  // only the count is needed here
+                ok = mbar_wait(bar(B_Q), k & 1, abort_flag, a.status);
+                if (!ok) break;
+                tc_fence_after();
+                if (n == 0) {  // nothing to attend: keep the per-unit phases
+                    mma_commit(bar(B_QFREE));
+                    mma_commit(bar(B_OFINAL));
+                    continue;
                 }
-                if (np < nq && mbar_test_wait(bar(B_PFULL + (np & 1)), (np >> 1) & 1)) {
-                    if (!mbar_wait(bar(B_VFULL + np % kSlots), (np / kSlots) & 1, abort_flag, a.status)) {
-                        ok = false;
-                        break;
+                int nq = 0, np = 0;  // next QK and next PV of this unit
+                Deadline dl;
+                while (ok && np < n) {
+                    bool progressed = false;
+                    const int gq = g0 + nq, gv = g0 + np;
+                    // QK_nq reuses score buffer gq&1, free once the PV two blocks back is issued.
+                    if (nq < n && nq <= np + 1 &&
+                        mbar_test_wait(bar(B_KFULL + gq % kSlots), (gq / kSlots) & 1)) {
+                        tc_fence_after();
+                        const uint64_t kd = sdesc_at(dK0, (gq % kSlots) * kKBytes);
+                        const uint32_t d = tmem + col_s(gq & 1);
+#pragma unroll
+                        for (int ks = 0; ks < 8; ++ks)
+                            mma_ss(d, sdesc_at(dQ0, (ks >> 2) * kHalfQ + (ks & 3) * 32),
+                                   sdesc_at(kd, (ks >> 2) * kKVHalf + (ks & 3) * 32), idesc_qk,
+                                   ks > 0 ? 1u : 0u);
+                        mma_commit(bar(B_SFULL + (gq & 1)));
+                        mma_commit(bar(B_KEMPTY + gq % kSlots));
+                        ++nq;
+                        if (nq == n) mma_commit(bar(B_QFREE));  // the Q tile may be replaced
+                        progressed = true;
                     }
-                    tc_fence_after();
-                    const uint64_t vd = sdesc_at(dV0, (np % kSlots) * kKBytes);
-                    const uint32_t pt = tmem + col_s(np & 1);
+                    if (np < nq && mbar_test_wait(bar(B_PFULL + (gv & 1)), (gv >> 1) & 1)) {
+                        // the first PV overwrites O: the previous unit's O must be read out
+                        if ((np == 0 && k >= 1 &&
+                             !mbar_wait(bar(B_OFREE), (k - 1) & 1, abort_flag, a.status)) ||
+                            !mbar_wait(bar(B_VFULL + gv % kSlots), (gv / kSlots) & 1, abort_flag, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint64_t vd = sdesc_at(dV0, (gv % kSlots) * kKBytes);
+                        const uint32_t pt = tmem + col_s(gv & 1);
 #pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_ts(tmem + kColO, pt + ks * 8, sdesc_at(vd, ks * 2048), idesc_pv,
-                               (np > 0 || ks > 0) ? 1u : 0u);
-                    mma_commit(bar(B_VEMPTY + np % kSlots));
-                    mma_commit(bar(B_PVDONE));
-                    if (np == n - 1) mma_commit(bar(B_OFINAL));
-                    ++np;
-                    progressed = true;
+                        for (int ks = 0; ks < 4; ++ks)
+                            mma_ts(tmem + kColO, pt + ks * 8, sdesc_at(vd, ks * 2048), idesc_pv,
+                                   (np > 0 || ks > 0) ? 1u : 0u);
+                        mma_commit(bar(B_VEMPTY + gv % kSlots));
+                        mma_commit(bar(B_PVDONE));
+                        if (np == n - 1) mma_commit(bar(B_OFINAL));
+                        ++np;
+                        progressed = true;
+                    }
+                    if (progressed) {
+                        dl.reset();
+                    } else if (*abort_flag) {
+                        ok = false;
+                    } else if (dl.expired()) {
+                        *abort_flag = 1;
+                        atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
+                        ok = false;
+                    }
                 }
-                if (progressed) {
-                    dl.reset();
-                } else if (*abort_flag) {
-                    ok = false;
-                } else if (dl.expired()) {
-                    *abort_flag = 1;
-                    atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
-                    ok = false;
-                }
+                g0 += n;
             }
             // Every MMA issued above must be complete before TMEM is freed.
             mma_commit(bar(B_DRAIN));
             mbar_wait_drain(bar(B_DRAIN), 0);
         }
-    } else {
+    } else if (warp < 4) {
         // ------------------------------------------------ softmax + epilogue
         const int row = threadIdx.x;  // TMEM lane
         const int tok = row & 63, hl = row >> 6;
         const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-        float m_used = -INFINITY, l = 0.f;
+        int g0 = 0;
         bool ok = true;
-        for (int j = 0; j < n; ++j) {
-            const int buf = j & 1;
-            ok = mbar_wait(bar(B_SFULL + buf), (j >> 1) & 1, abort_flag, a.status);
+        for (int k = 0; unit_of(k) < a.units; ++k) {
+            const FwdUnit d = fwd_unit(a, unit_of(k));
+            ok = ok && mbar_wait(bar(B_UFULL + k % kListSlots), (k / kListSlots) & 1, abort_flag, a.status);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            const int* sl = slot_ptr(k);
+            const int n = sl[0];
+            const int* list = sl + 1;
+            float m_used = -INFINITY, l = 0.f;
+            for (int j = 0; j < n; ++j) {
+                const int g = g0 + j, buf = g & 1;
+                ok = mbar_wait(bar(B_SFULL + buf), (g >> 1) & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+                tc_fence_after();
+                uint32_t sr[64];
+                tmem_ld64(lane_base + col_s(buf), sr);
+                if (list[j] == d.qb) {  // the query's own block: token-level causal mask
+#pragma unroll
+                    for (int c = 0; c < 64; ++c)
+                        if (c > tok) sr[c] = __float_as_uint(-INFINITY);
+                }
+                // row max of the raw scores (the scale is positive)
+                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                for (int c = 0; c < 64; ++c) m4[c & 3] = fmaxf(m4[c & 3], __uint_as_float(sr[c]));
+                const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;
+                if (j == 0) {
+                    m_used = mx;
+                } else {
+                    const bool need = mx > m_used + kRescaleLog2;
+                    if (__any_sync(0xffffffffu, need)) {
+                        // PV of the previous block must be complete before O is touched.
+                        ok = mbar_wait(bar(B_PVDONE), (g - 1) & 1, abort_flag, a.status);
+                        ok = __all_sync(0xffffffffu, ok);
+                        if (!ok) break;
+                        tc_fence_after();
+                        const float f = need ? ex2_approx(m_used - mx) : 1.0f;
+#pragma unroll 1
+                        for (int c8 = 0; c8 < 8; ++c8) {
+                            uint32_t o[16];
+                            tmem_ld16(lane_base + kColO + 16 * c8, o);
+#pragma unroll
+                            for (int c = 0; c < 16; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
+                            tmem_st16(lane_base + kColO + 16 * c8, o);
+                        }
+                        if (need) {
+                            l *= f;
+                            m_used = mx;
+                        }
+                    }
+                }
+                // p = 2^(s * scale_log2 - m): one FFMA and one SFU op per score
+                // P is packed in place: entry c (c < 32) takes the pair (2c, 2c+1), both
+                // read before entry c is overwritten.
+                float r4[4] = {0.f, 0.f, 0.f, 0.f};
+                const float neg_m = -m_used;
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    const float p0 = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), a.scale_log2, neg_m));
+                    const float p1 = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), a.scale_log2, neg_m));
+                    r4[c & 3] += p0 + p1;
+                    sr[c] = pack2_bf16(p0, p1);
+                }
+                const float rs = (r4[0] + r4[1]) + (r4[2] + r4[3]);
+                l += rs;
+                tmem_st32(lane_base + col_s(buf), sr);
+                tc_fence_before();
+                mbar_arrive(bar(B_PFULL + buf));
+            }
+            if (!ok) break;
+            mbar_arrive(bar(B_UFREE + k % kListSlots));  // the list is no longer read
+            // Epilogue: the unit's O accumulation must be complete.
+            ok = mbar_wait(bar(B_OFINAL), k & 1, abort_flag, a.status);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             tc_fence_after();
-            uint32_t sr[64];
-            tmem_ld64(lane_base + col_s(buf), sr);
-            if (list[j] == qb) {  // the query's own block: token-level causal mask
-#pragma unroll
-                for (int c = 0; c < 64; ++c)
-                    if (c > tok) sr[c] = __float_as_uint(-INFINITY);
-            }
-            // row max of the raw scores (the scale is positive)
-            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-            for (int c = 0; c < 64; ++c) m4[c & 3] = fmaxf(m4[c & 3], __uint_as_float(sr[c]));
-            const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;
-            if (j == 0) {
-                m_used = mx;
-            } else {
-                const bool need = mx > m_used + kRescaleLog2;
-                if (__any_sync(0xffffffffu, need)) {
-                    // PV of the previous block must be complete before O is touched.
-                    ok = mbar_wait(bar(B_PVDONE), (j - 1) & 1, abort_flag, a.status);
-                    ok = __all_sync(0xffffffffu, ok);
-                    if (!ok) break;
-                    tc_fence_after();
-                    const float f = need ? ex2_approx(m_used - mx) : 1.0f;
-#pragma unroll 1
-                    for (int c8 = 0; c8 < 8; ++c8) {
-                        uint32_t o[16];
-                        tmem_ld16(lane_base + kColO + 16 * c8, o);
-#pragma unroll
-                        for (int c = 0; c < 16; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
-                        tmem_st16(lane_base + kColO + 16 * c8, o);
-                    }
-                    if (need) {
-                        l *= f;
-                        m_used = mx;
-                    }
-                }
-            }
-            // p = 2^(s * scale_log2 - m): one FFMA and one SFU op per score
-            // P is packed in place: entry c (c < 32) takes the pair (2c, 2c+1), both
-            // read before entry c is overwritten.
-            float r4[4] = {0.f, 0.f, 0.f, 0.f};
-            const float neg_m = -m_used;
-#pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                const float p0 = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), a.scale_log2, neg_m));
-                const float p1 = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), a.scale_log2, neg_m));
-                r4[c & 3] += p0 + p1;
-                sr[c] = pack2_bf16(p0, p1);
-            }
-            const float rs = (r4[0] + r4[1]) + (r4[2] + r4[3]);
-            l += rs;
-            tmem_st32(lane_base + col_s(buf), sr);
-            tc_fence_before();
-            mbar_arrive(bar(B_PFULL + buf));
-        }
-        // Epilogue: the whole O accumulation must be complete.
-        if (ok && n > 0) {
-            ok = mbar_wait(bar(B_OFINAL), 0, abort_flag, a.status);
-            ok = __all_sync(0xffffffffu, ok);
-        }
-        if (ok) {
-            tc_fence_after();
             const float inv = l > 0.f ? 1.0f / l : 0.f;
-            uint8_t* sq = smem + kOffQ;
-#pragma unroll
+            const int i = d.qb * 64 + tok;
+            uint4* dst = reinterpret_cast<uint4*>(a.O + ((size_t)(d.hq0 + hl) * a.L + (i < a.L ? i : 0)) * 128);
+#pragma unroll 1
             for (int c4 = 0; c4 < 4; ++c4) {
                 uint32_t o[32];
                 if (n > 0) {
@@ -309,31 +429,25 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
 #pragma unroll
                     for (int c = 0; c < 32; ++c) o[c] = 0u;
                 }
-                const int dh = c4 >> 1;
+                if (c4 == 3) {  // O is in registers: the next unit's first PV may overwrite it
+                    tc_fence_before();
+                    mbar_arrive(bar(B_OFREE));
+                }
+                if (i < a.L) {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int chunk = (c4 & 1) * 4 + q;
-                    uint4 v;
-                    v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
-                    v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
-                    v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
-                    v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
-                    *reinterpret_cast<uint4*>(sq + dh * kHalfQ + row * 128 + ((chunk ^ (row & 7)) << 4)) = v;
+                    for (int q = 0; q < 4; ++q) {
+                        uint4 v;
+                        v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
+                        v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
+                        v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
+                        v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
+                        dst[4 * c4 + q] = v;
+                    }
                 }
             }
-            fence_proxy_async_smem();
-            const int i = qb * 64 + tok;
             if (i < a.L)
-                a.lse[(size_t)(hq0 + hl) * a.L + i] = l > 0.f ? (m_used + log2f(l)) * kLn2 : -INFINITY;
-        }
-        named_barrier(1, 128);
-        if (threadIdx.x == 0 && ok) {
-            for (int h2 = 0; h2 < 2; ++h2)
-                for (int dh = 0; dh < 2; ++dh)
-                    tma_store_3d(&tmO, sb + kOffQ + dh * kHalfQ + h2 * (kHalfQ / 2), dh * 64,
-                                 qb * 64, hq0 + h2);
-            tma_store_commit();
-            tma_store_wait_read();
+                a.lse[(size_t)(d.hq0 + hl) * a.L + i] = l > 0.f ? (m_used + log2f(l)) * kLn2 : -INFINITY;
+            g0 += n;
         }
     }
     tc_fence_before();
@@ -350,20 +464,31 @@ cudaError_t launch_attn_fwd_tc(const void* Q, const void* K, const void* V, cons
                                const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                                void* O, float* lse, int* status, cudaStream_t st) {
     const int NQB = (s.L + 63) / 64;
-    CUtensorMap tq, tk, tv, to;
+    CUtensorMap tq, tk, tv;
     if (!make_tmap_bf16_rows128(&tq, Q, s.L, (uint64_t)s.B * s.Hq, 64) ||
         !make_tmap_bf16_rows128(&tk, K, s.L, (uint64_t)s.B * s.Hkv, 64) ||
-        !make_tmap_bf16_rows128(&tv, V, s.L, (uint64_t)s.B * s.Hkv, 64) ||
-        !make_tmap_bf16_rows128(&to, O, s.L, (uint64_t)s.B * s.Hq, 64))
+        !make_tmap_bf16_rows128(&tv, V, s.L, (uint64_t)s.B * s.Hkv, 64))
         return cudaErrorInvalidValue;
     const size_t smem = fwd_tc_smem(topk);
     cudaError_t e = cudaFuncSetAttribute(attn_fwd_tc_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    FwdTcArgs args{idx, cnt, lse, status, s.Hq, s.Hkv, s.L, NQB, topk, sm_scale * kLog2e};
-    const long long grid = (long long)s.B * s.Hkv * NQB;
+    if ((e = cudaFuncSetAttribute(attn_fwd_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                  100)) != cudaSuccess)
+        return e;
+    int dev = 0, nsm = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    // Two CTAs per SM (shared memory and registers are sized for it); CTAs never
+    // wait on one another, so the grid is correct whatever number is resident.
+    const long long units = (long long)s.B * s.Hkv * NQB;
+    const long long cap = 2LL * nsm;
+    const unsigned grid = (unsigned)(units < cap ? units : cap);
+    FwdTcArgs args{idx, cnt, static_cast<__nv_bfloat16*>(O), lse, status, s.Hq, s.Hkv, s.L, NQB,
+                   topk, (int)units, sm_scale * kLog2e};
     ProfScope prof(K_FWD, st);
-    attn_fwd_tc_kernel<<<(unsigned)grid, kThreads, smem, st>>>(tq, tk, tv, to, args);
+    attn_fwd_tc_kernel<<<grid, kThreads, smem, st>>>(tq, tk, tv, args);
     return cudaGetLastError();
 }
 
