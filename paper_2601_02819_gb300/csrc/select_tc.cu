@@ -87,6 +87,7 @@ __device__ __forceinline__ SelUnit sel_unit(const SelArgs& a, int u) {
     return d;
 }
 
+template <bool kMaxLogit>
 __global__ void __launch_bounds__(kThreads, 2)
 select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKr,
                  const SelArgs a) {
@@ -138,7 +139,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
                 const SelUnit d = sel_unit(a, u);
                 if (!d.scored) continue;
-                const int steps = (a.agg ? 1 : 2) * d.nch;
+                const int steps = (kMaxLogit ? 1 : 2) * d.nch;
                 for (int s = 0; ok && s < steps; ++s, ++gs) {
                     const int slot = gs & 1, c = s % d.nch;
                     if (gs >= 2 && !mbar_wait(bar(B_KEMPTY + slot), ((gs >> 1) - 1) & 1, abort_flag, a.status)) {
@@ -182,7 +183,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 if (!d.scored) continue;
                 ok = mbar_wait(bar(B_Q), su & 1, abort_flag, a.status);
                 tc_fence_after();
-                const int steps = (a.agg ? 1 : 2) * d.nch;
+                const int steps = (kMaxLogit ? 1 : 2) * d.nch;
                 for (int s = 0; ok && s < steps; ++s, ++gs) {
                     const int slot = gs & 1;
                     ok = mbar_wait(bar(B_KFULL + slot), (gs >> 1) & 1, abort_flag, a.status) &&
@@ -190,7 +191,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     if (!ok) break;
                     tc_fence_after();
                     const uint64_t kr = sdesc_at(dKr0, slot * kTile);
-                    const bool pass1 = !a.agg && s < d.nch;
+                    const bool pass1 = !kMaxLogit && s < d.nch;
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks) {
                         const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
@@ -238,7 +239,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             // candidate) or, for max logits, the larger half; each lane holds its
             // candidates' keys in registers
             const int nC = d.nC, ksel = d.ksel, c_lo = d.c_lo;
-            const bool mx = a.agg != 0;
+            constexpr bool mx = kMaxLogit;
             auto key_of = [&](int cj) {
                 return topk::make_key_agg(mx ? fmaxf(A0[cj], A1[cj]) : A0[cj] + A1[cj], c_lo + cj, mx);
             };
@@ -298,7 +299,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
         for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
             const SelUnit d = sel_unit(a, u);
             if (!d.scored) continue;
-            const int nch = d.nch, steps = (a.agg ? 1 : 2) * nch, c_lo = d.c_lo, c_hi = d.c_hi, nC = d.nC;
+            const int nch = d.nch, steps = (kMaxLogit ? 1 : 2) * nch, c_lo = d.c_lo, c_hi = d.c_hi, nC = d.nC;
             const bool row_ok = d.qb * 64 + (r & 63) < a.L;
             const int buf = su & 1;
             float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
@@ -315,7 +316,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     ok = __all_sync(0xffffffffu, ok);
                 }
                 if (ok) tc_fence_after();
-                if (ok && !a.agg && s < nch) {
+                if (ok && !kMaxLogit && s < nch) {
                     // pass 1: row r against 64 candidates of the chunk, two loads of 32
                     const int t0 = c_lo + c * kCand + 64 * hh;
                     const bool full = t0 + 63 <= c_hi;
@@ -343,7 +344,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     }
                     tc_fence_before();
                     mbar_arrive(bar(B_SFREE + slot));
-                } else if (ok && a.agg) {
+                } else if (ok && kMaxLogit) {
                     // max logit: candidate r against the 64 rows of half hh (head hh)
                     float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
                     const bool live = c * kCand + (warp & 3) * 32 < nC;
@@ -390,7 +391,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     const int cj = c * kCand + r;
                     if (cj < nC) (hh ? A1 : A0)[cj] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
                 }
-                if (!a.agg && s == nch - 1) {
+                if (!kMaxLogit && s == nch - 1) {
                     // merge the two column halves of every row: (m, z) -> max and 1/sum
                     pm[hh * 128 + r] = m;
                     pz[hh * 128 + r] = z;
@@ -437,8 +438,8 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
                                 (uint64_t)s.B * s.Hkv, 128))
         return cudaErrorInvalidValue;
     const size_t smem = select_tc_smem(NQB, p.topk);
-    cudaError_t e = cudaFuncSetAttribute(select_tc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    auto kern = p.aggregation == PHSA_AGG_MAX_LOGIT ? select_tc_kernel<true> : select_tc_kernel<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -449,7 +450,7 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
     SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, units,
                  p.aggregation, p.sm_scale * kLog2e, p.sm_scale};
     ProfScope prof(K_SELECT, st);
-    select_tc_kernel<<<(unsigned)min(units, per_sm * nsm), kThreads, smem, st>>>(tq, tkr, args);
+    kern<<<(unsigned)min(units, per_sm * nsm), kThreads, smem, st>>>(tq, tkr, args);
     return cudaGetLastError();
 }
 
