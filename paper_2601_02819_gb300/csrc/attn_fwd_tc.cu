@@ -110,6 +110,27 @@ __device__ __forceinline__ FwdUnit fwd_unit(const FwdTcArgs& a, int u) {
 
 __device__ __forceinline__ uint32_t col_s(int buf) { return 128u + 64u * (uint32_t)buf; }
 
+__device__ __forceinline__ uint4 shfl_xor4(const uint4& v, int m) {
+    return make_uint4(__shfl_xor_sync(0xffffffffu, v.x, m), __shfl_xor_sync(0xffffffffu, v.y, m),
+                      __shfl_xor_sync(0xffffffffu, v.z, m), __shfl_xor_sync(0xffffffffu, v.w, m));
+}
+
+// One round of a 4 x 4 transpose among lanes r and r ^ m: a lane with sel = 0
+// keeps (a0, a1) and replaces (b0, b1) with its partner's (a0, a1); a lane
+// with sel = 1 keeps (b0, b1) and replaces (a0, a1) with its partner's (b0, b1).
+__device__ __forceinline__ void xchg_pieces(uint4& a0, uint4& a1, uint4& b0, uint4& b1, int sel,
+                                            int m) {
+    const uint4 r0 = shfl_xor4(sel ? a0 : b0, m);
+    const uint4 r1 = shfl_xor4(sel ? a1 : b1, m);
+    if (sel) {
+        a0 = r0;
+        a1 = r1;
+    } else {
+        b0 = r0;
+        b1 = r1;
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 2)
 attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const FwdTcArgs a) {
@@ -419,7 +440,11 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             tc_fence_after();
             const float inv = l > 0.f ? 1.0f / l : 0.f;
             const int i = d.qb * 64 + tok;
-            uint4* dst = reinterpret_cast<uint4*>(a.O + ((size_t)(d.hq0 + hl) * a.L + (i < a.L ? i : 0)) * 128);
+            // Rows go out through a 4 x 4 transpose of 16-byte pieces among each four
+            // lanes (two rounds of xor shuffles): afterwards lane 4j + c holds piece c
+            // of rows 4j .. 4j + 3, so a store instruction writes eight 64-byte row
+            // segments instead of thirty-two 16-byte pieces.
+            const int sel1 = (lane >> 1) & 1, sel0 = lane & 1;
 #pragma unroll 1
             for (int c4 = 0; c4 < 4; ++c4) {
                 uint32_t o[32];
@@ -433,16 +458,23 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     tc_fence_before();
                     mbar_arrive(bar(B_OFREE));
                 }
-                if (i < a.L) {
+                uint4 x[4];
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        uint4 v;
-                        v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
-                        v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
-                        v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
-                        v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
-                        dst[4 * c4 + q] = v;
-                    }
+                for (int q = 0; q < 4; ++q) {
+                    x[q].x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
+                    x[q].y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
+                    x[q].z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
+                    x[q].w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
+                }
+                xchg_pieces(x[0], x[1], x[2], x[3], sel1, 2);  // rows r, r^2: halves of the pieces
+                xchg_pieces(x[0], x[2], x[1], x[3], sel0, 1);  // rows r, r^1: single pieces
+#pragma unroll
+                for (int s4 = 0; s4 < 4; ++s4) {
+                    const int r = warp * 32 + (lane & ~3) + s4;  // the row this piece belongs to
+                    const int ri = d.qb * 64 + (r & 63);
+                    if (ri < a.L)
+                        reinterpret_cast<uint4*>(a.O + ((size_t)(d.hq0 + (r >> 6)) * a.L + ri) * 128)
+                            [4 * c4 + (lane & 3)] = x[s4];
                 }
             }
             if (i < a.L)
