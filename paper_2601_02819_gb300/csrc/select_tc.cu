@@ -325,19 +325,22 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                         if (t0 + 32 * q > c_hi) break;  // no candidate left in this group (warp-uniform)
                         uint32_t v[32];
                         tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+                        // max of the raw scores, then the scale (positive) once
                         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                        if (!full) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            float x = __uint_as_float(v[j]) * a.scale_log2;
-                            if (!full && t0 + 32 * q + j > c_hi) x = -INFINITY;
-                            v[j] = __float_as_uint(x);
-                            m4[j & 3] = fmaxf(m4[j & 3], x);
+                            for (int j = 0; j < 32; ++j)
+                                if (t0 + 32 * q + j > c_hi) v[j] = __float_as_uint(-INFINITY);
                         }
-                        const float mn = fmaxf(m, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])));
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) m4[j & 3] = fmaxf(m4[j & 3], __uint_as_float(v[j]));
+                        const float mn = fmaxf(m, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2);
                         if (mn != -INFINITY) {
                             float s4[4] = {0.f, 0.f, 0.f, 0.f};
+                            const float neg = -mn;
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) s4[j & 3] += ex2_approx(__uint_as_float(v[j]) - mn);
+                            for (int j = 0; j < 32; ++j)
+                                s4[j & 3] += ex2_approx(fmaf(__uint_as_float(v[j]), a.scale_log2, neg));
                             z = z * ex2_approx(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
                             m = mn;
                         }
@@ -368,8 +371,8 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 } else if (ok) {
                     // pass 2: candidate r against the 64 rows of half hh, in row order;
                     // a warp whose 32 candidates all lie past the last one skips the work
+                    // p = 2^(S*scale - m_r - log2 Z_r): the row's max and sum in one offset
                     const float* mrow = m2s + 64 * hh;
-                    const float* irow = izs + 64 * hh;
                     float acc[4] = {0.f, 0.f, 0.f, 0.f};
                     const bool live = c * kCand + (warp & 3) * 32 < nC;
 #pragma unroll 1
@@ -379,11 +382,10 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 #pragma unroll
                         for (int j = 0; j < 32; j += 4) {
                             const float4 mm = *reinterpret_cast<const float4*>(mrow + 32 * q + j);
-                            const float4 iz = *reinterpret_cast<const float4*>(irow + 32 * q + j);
-                            acc[0] += ex2_approx(fmaf(__uint_as_float(v[j + 0]), a.scale_log2, -mm.x)) * iz.x;
-                            acc[1] += ex2_approx(fmaf(__uint_as_float(v[j + 1]), a.scale_log2, -mm.y)) * iz.y;
-                            acc[2] += ex2_approx(fmaf(__uint_as_float(v[j + 2]), a.scale_log2, -mm.z)) * iz.z;
-                            acc[3] += ex2_approx(fmaf(__uint_as_float(v[j + 3]), a.scale_log2, -mm.w)) * iz.w;
+                            acc[0] += ex2_approx(fmaf(__uint_as_float(v[j + 0]), a.scale_log2, -mm.x));
+                            acc[1] += ex2_approx(fmaf(__uint_as_float(v[j + 1]), a.scale_log2, -mm.y));
+                            acc[2] += ex2_approx(fmaf(__uint_as_float(v[j + 2]), a.scale_log2, -mm.z));
+                            acc[3] += ex2_approx(fmaf(__uint_as_float(v[j + 3]), a.scale_log2, -mm.w));
                         }
                     }
                     tc_fence_before();
@@ -402,8 +404,8 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                         const float za = ma == -INFINITY ? 0.f : pz[r] * ex2_approx(ma - mx);
                         const float zb = mb == -INFINITY ? 0.f : pz[128 + r] * ex2_approx(mb - mx);
                         const float zz = za + zb;
-                        m2s[r] = row_ok ? mx : 0.f;
-                        izs[r] = (row_ok && zz > 0.f) ? 1.0f / zz : 0.f;
+                        // a row past L (or without candidates) contributes 2^-inf = 0
+                        m2s[r] = (row_ok && zz > 0.f) ? mx + log2f(zz) : INFINITY;
                     }
                     named_barrier(1, 256);
                 }
