@@ -341,7 +341,8 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 #pragma unroll
                             for (int j = 0; j < 32; ++j)
                                 s4[j & 3] += ex2_approx(fmaf(__uint_as_float(v[j]), a.scale_log2, neg));
-                            z = z * ex2_approx(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+                            if (mn > m) z *= ex2_approx(m - mn);  // the running max moved
+                            z += (s4[0] + s4[1]) + (s4[2] + s4[3]);
                             m = mn;
                         }
                     }
