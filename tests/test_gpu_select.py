@@ -82,7 +82,8 @@ def test_exact_ties_go_to_the_lower_block():
         assert list(gi[0, 0, qb]) == [0, 3, qb], qb
 
 
-@pytest.mark.parametrize("name", ["train_8k_x4", "prefill_32k", "prefill_32k_paper_forced"])
+@pytest.mark.parametrize("name", ["train_8k_x4", "prefill_32k", "prefill_32k_paper_forced",
+                                  "long_131k_p0"])
 def test_full_size_sampled_units(name):
     if name == "prefill_32k_paper_forced":  # 128 initial + 512 local tokens, as the paper's 32k setting
         w = inputs.custom(name, B=1, L=32768, Hq=16, Hkv=8, topk=14, n_init=2, n_local=8,

@@ -39,7 +39,8 @@ def test_tiny_workload_end_to_end():
     assert np.abs(lse.cpu().numpy()[:, :, rows] - lser[:, :, rows]).max() <= LSE_ABS
 
 
-@pytest.mark.parametrize("name", ["prefill_32k", "train_8k_x4", "long_131k_p3"])
+@pytest.mark.parametrize("name", ["prefill_32k", "train_8k_x4", "long_131k_p0", "long_131k_p3",
+                                  "long_131k_p15"])
 def test_full_size_forward_sampled_rows(name):
     w = inputs.WORKLOADS[name]
     x = inputs.make_inputs(w)
@@ -74,6 +75,32 @@ def test_train_workload_backward_sampled():
     assert_close("dQ rows", bf16_to_f64(dQ)[rows[:, 0], rows[:, 1], rows[:, 2]], rq)
     blocks = np.array([[0, 0, 0], [1, 3, 1], [2, 5, 7], [3, 7, w.NQB - 1], [0, 2, 64],
                        [1, 1, 100]], np.int32)
+    rk, rv = oracle.sparse_attn_bwd_kv_blocks(x["Q"], x["K"], x["V"], x["dO"], gi, gc, 64, SCALE,
+                                              blocks)
+    dKh, dVh = bf16_to_f64(dK), bf16_to_f64(dV)
+    for n, (b, g, t) in enumerate(blocks):
+        assert_close(f"dK block {t}", dKh[b, g, t * 64:(t + 1) * 64], rk[n])
+        assert_close(f"dV block {t}", dVh[b, g, t * 64:(t + 1) * 64], rv[n])
+
+
+def test_prefill_32k_backward_sampled():
+    # The bench configuration: dQ on sampled rows, dK/dV on sampled KV blocks (block 0,
+    # selected by every query block, is left to the smaller workloads).
+    w = inputs.WORKLOADS["prefill_32k"]
+    x = inputs.make_inputs(w, with_grad=True)
+    Qd, Kd, Vd, O, lse, idx, cnt = gpu_forward(w, x)
+    dQ, dK, dV = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, to_dev_bf16(x["dO"]), lse, idx, cnt)
+    torch.cuda.synchronize()
+    assert phsa.phsa_get_device_status() == 0
+    gi, gc = idx.cpu().numpy(), cnt.cpu().numpy()
+    rng = np.random.default_rng(3)
+    rows = np.stack([np.zeros(48, np.int64), rng.integers(0, w.Hq, 48),
+                     rng.integers(0, w.L, 48)], axis=1).astype(np.int32)
+    rows[:2] = [[0, 0, w.L - 1], [0, w.Hq - 1, 64 * 300 + 7]]
+    rq = oracle.sparse_attn_bwd_dq_rows(x["Q"], x["K"], x["V"], x["dO"], gi, gc, 64, SCALE, rows)
+    assert_close("dQ rows", bf16_to_f64(dQ)[rows[:, 0], rows[:, 1], rows[:, 2]], rq)
+    blocks = np.array([[0, 0, 1], [0, 3, 17], [0, 5, 200], [0, 7, w.NQB - 1], [0, 2, 450],
+                       [0, 6, 64]], np.int32)
     rk, rv = oracle.sparse_attn_bwd_kv_blocks(x["Q"], x["K"], x["V"], x["dO"], gi, gc, 64, SCALE,
                                               blocks)
     dKh, dVh = bf16_to_f64(dK), bf16_to_f64(dV)
