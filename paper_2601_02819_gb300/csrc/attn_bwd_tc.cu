@@ -15,7 +15,9 @@
 //   the elementwise warps compute Delta_i = dO_i . O_i (O read from global
 //   memory, dO from the loaded tile) and write it for the dK/dV kernel, which
 //   runs after this one. A fourth producer warp loads each unit's Q and dO as
-//   soon as the previous unit's last dP has been issued and its Delta read.
+//   soon as the previous unit's last dP has been issued and its Delta read,
+//   and stages the elementwise warps' copy of the unit's block list before it
+//   arrives on the barrier that the tiles complete.
 //
 // dkdv_tc_kernel: persistent, one CTA per SM over the work items (KV block t,
 //   chunk of <= 32 query blocks that selected t), 320 threads; K_t and V_t are

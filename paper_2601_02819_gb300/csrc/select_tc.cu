@@ -12,7 +12,7 @@
 //           softmax); the halves are merged once, after the last chunk;
 //   pass 2  S^T = Kr Q^T (M = 128 candidates, N = 128 rows) in TMEM;
 //           two threads per candidate j (lane j, one per half of the rows)
-//           sum p = 2^(S*scale - m_r)/Z_r over their 64 rows in row order;
+//           sum p = 2^(S*scale - m_r - log2 Z_r) over their 64 rows in row order;
 //           A[t] = half 0 + half 1. Every candidate follows the same order,
 //           so equal candidates get bit-identical sums.
 //   top-k   a dedicated warp, on a double-buffered copy of A, while the
@@ -40,8 +40,8 @@ constexpr int kHalf = 128 * 64 * 2;        // 128 rows x 64 columns bf16 (16 KB)
 constexpr int kTile = 2 * kHalf;           // 128 x 128 (32 KB)
 constexpr int kOffQ = 0;
 constexpr int kOffKr = kOffQ + kTile;      // 2 slots
-constexpr int kOffStats = kOffKr + 2 * kTile;  // m2[128], iz[128], half partials m[2][128], z[2][128]
-constexpr int kOffBar = kOffStats + 6 * 128 * 4;
+constexpr int kOffStats = kOffKr + 2 * kTile;  // m + log2 Z [128], half partials m[2][128], z[2][128]
+constexpr int kOffBar = kOffStats + 5 * 128 * 4;
 constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = 4, B_SFULL = 6, B_SFREE = 8,
               B_AFULL = 10, B_AFREE = 12, B_DRAIN = 14, kNumBars = 15;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
@@ -98,9 +98,8 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
-    float* m2s = reinterpret_cast<float*>(smem + kOffStats);
-    float* izs = m2s + 128;
-    float* pm = izs + 128;  // [2][128] per-half running max (pass 1)
+    float* m2s = reinterpret_cast<float*>(smem + kOffStats);  // per row: max + log2 of the sum
+    float* pm = m2s + 128;  // [2][128] per-half running max (pass 1)
     float* pz = pm + 256;   // [2][128] per-half running sum
     float* Abuf = reinterpret_cast<float*>(smem + kOffA);  // [2][A0 | A1], NQB each
     int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 16);
