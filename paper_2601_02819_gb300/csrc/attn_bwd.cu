@@ -27,6 +27,7 @@ namespace phsa {
 namespace {
 
 constexpr int kChunk = kBwdChunk;  // query blocks per dK/dV work item
+constexpr int kBuildCache = 8192;   // KV blocks whose counts the index build keeps on chip
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -116,16 +117,33 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
                  int2* __restrict__ queue, int* __restrict__ qcount, int* status) {
     __shared__ int tmp[32];
     __shared__ int bin[kChunk + 1];  // items per iteration count, then queue cursors
+    __shared__ int ncache[kBuildCache];  // selecting-query count of each KV block
     const int bg = blockIdx.x;
     const int per = (NQB + 1023) / 1024;  // KV blocks counted by each thread
     const int t0 = threadIdx.x * per;
     const uint32_t* bb = bits + (size_t)bg * NQB * words;
+    // The count of a block: its bitmap row's popcount, read with independent
+    // loads. The first kBuildCache blocks keep theirs in shared memory for the
+    // later passes (each thread reads back only its own entries); any block
+    // beyond is counted again where it is needed.
+    auto count_row = [&](int t) {
+        const uint32_t* row = bb + (size_t)t * words;
+        int n = 0;
+#pragma unroll 8
+        for (int w = 0; w < words; ++w) n += __popc(__ldg(row + w));
+        return n;
+    };
+    auto count_of = [&](int t) { return t < kBuildCache ? ncache[t] : count_row(t); };
+    for (int k = 0; k < per; ++k) {
+        const int t = t0 + k;
+        if (t >= NQB) break;
+        if (t < kBuildCache) ncache[t] = count_row(t);
+    }
     int sn = 0, sch = 0, ssl = 0;
     for (int k = 0; k < per; ++k) {
         const int t = t0 + k;
         if (t >= NQB) break;
-        int n = 0;
-        for (int w = 0; w < words; ++w) n += __popc(bb[(size_t)t * words + w]);
+        const int n = count_of(t);
         const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
         sn += n;
         sch += nch;
@@ -146,8 +164,7 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     for (int k = 0, ch = och; k < per; ++k) {
         const int t = t0 + k;
         if (t >= NQB) break;
-        int n = 0;
-        for (int w = 0; w < words; ++w) n += __popc(bb[(size_t)t * words + w]);
+        const int n = count_of(t);
         const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
         for (int c = 0; c < nch && ch + c < work_max; ++c)
             atomicAdd(&bin[min(n, kChunk * c + kChunk) - kChunk * c], 1);
@@ -172,8 +189,7 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     for (int k = 0; k < per; ++k) {
         const int t = t0 + k;
         if (t >= NQB) break;
-        int n = 0;
-        for (int w = 0; w < words; ++w) n += __popc(bb[(size_t)t * words + w]);
+        const int n = count_of(t);
         const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
         TInfo info;
         info.off = on;
