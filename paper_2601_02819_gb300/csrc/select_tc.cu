@@ -87,6 +87,22 @@ __device__ __forceinline__ SelUnit sel_unit(const SelArgs& a, int u) {
     return d;
 }
 
+// The chunk that step s of a unit with nch chunks per pass works on. Pass 2
+// takes the last two chunks of pass 1 first: they are still in the ring's two
+// slots (same slot parity, the ring alternates), so they are not loaded again;
+// then chunks 0 .. nch - 3. Each chunk holds its own candidates, so the order
+// of the chunks changes no sum.
+__device__ __forceinline__ int step_chunk(int s, int nch, bool pass2_only) {
+    if (pass2_only || s < nch) return s;
+    const int j = s - nch;
+    if (nch < 2) return 0;
+    return j < 2 ? nch - 2 + j : j - 2;
+}
+// Step s reuses the chunk already in its slot (pass 2's first two steps).
+__device__ __forceinline__ bool step_resident(int s, int nch, bool pass2_only) {
+    return !pass2_only && nch >= 2 && s >= nch && s < nch + 2;
+}
+
 template <bool kMaxLogit>
 __global__ void __launch_bounds__(kThreads, 2)
 select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKr,
@@ -140,10 +156,16 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 if (!d.scored) continue;
                 const int steps = (kMaxLogit ? 1 : 2) * d.nch;
                 for (int s = 0; ok && s < steps; ++s, ++gs) {
-                    const int slot = gs & 1, c = s % d.nch;
+                    const int slot = gs & 1, c = step_chunk(s, d.nch, kMaxLogit);
                     if (gs >= 2 && !mbar_wait(bar(B_KEMPTY + slot), ((gs >> 1) - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
+                    }
+                    if (step_resident(s, d.nch, kMaxLogit)) {
+                        // the slot holds this chunk: its last reader is done (KEMPTY
+                        // above), so the full phase completes without a copy
+                        mbar_arrive(bar(B_KFULL + slot));
+                        continue;
                     }
                     mbar_expect_tx(bar(B_KFULL + slot), kTile);
                     for (int dh = 0; dh < 2; ++dh)
@@ -309,7 +331,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             }
             float m = -INFINITY, z = 0.f;
             for (int s = 0; s < steps; ++s, ++gs) {
-                const int slot = gs & 1, c = s % nch;
+                const int slot = gs & 1, c = step_chunk(s, nch, kMaxLogit);
                 if (ok) {
                     ok = mbar_wait(bar(B_SFULL + slot), (gs >> 1) & 1, abort_flag, a.status);
                     ok = __all_sync(0xffffffffu, ok);
