@@ -31,8 +31,11 @@
  *     reports argument validation and launch errors only. Errors detected by
  *     a kernel (an out-of-range block index, a bounded wait that expired) are
  *     recorded in a device status word read by phsa_get_device_status.
- *   - Supported today: D = 128, block_size = 64, G in {1, 2}. Other shapes
- *     return PHSA_ERR_UNSUPPORTED, never a wrong answer.
+ *   - Supported today: D = 128, G in {1, 2}, block_size = 64 in every call;
+ *     phsa_build_block_repr, phsa_select_blocks and phsa_sparse_attn_fwd also
+ *     take block_size 16 and 32 (16 is the block size of the paper's experiment
+ *     settings).
+ *     Other shapes return PHSA_ERR_UNSUPPORTED, never a wrong answer.
  *   - Calls are thread-safe with respect to each other; concurrent calls on
  *     different streams that write the same output race, as any CUDA work.
  */

@@ -1,11 +1,14 @@
 // Stage (c) forward: causal attention over the selected KV blocks (Eq. 10-11;
-// Algorithm 1 step 4), one CTA per (query block qb, KV head g).
+// Algorithm 1 step 4), one CTA per (query block qb, KV head g), for block
+// sizes m = 16, 32, 64.
 //
-// The G query heads of the KV group are packed into one G*64-row tile, so each
-// gathered 64 x 128 K/V block is loaded once and used by every head of the
-// group. Blocks are visited in ascending order with a double-buffered cp.async
-// pipeline; S = Q K^T and O += P V run as bf16 warp MMAs with fp32
-// accumulators, and the softmax is computed online in the log2 domain
+// The G query heads of the KV group are packed into one G*m-row tile, so each
+// gathered m x 128 K/V block is loaded once and used by every head of the
+// group. Keys are taken 64 at a time: a key tile holds 64/m consecutive
+// entries of the block list (ascending), slots past its end are masked. Tiles
+// are visited in order with a double-buffered cp.async pipeline; S = Q K^T
+// and O += P V run as bf16 warp MMAs with fp32 accumulators, and the softmax
+// is computed online in the log2 domain
 // (FlashAttention-style). Inside the query's own block the token-level causal
 // mask applies. Outputs: O in bf16 and the natural-log LSE per row.
 #include "phsa_common.cuh"
@@ -15,30 +18,45 @@ namespace phsa {
 
 namespace {
 
-template <int G>
+// G query heads x m tokens per unit; keys are taken in tiles of 64, assembled
+// from kNb = 64 / m selected blocks (m rows of K and V each).
+template <int G, int BM>
 struct FwdCfg {
-    static constexpr int kWarps = 4 * G;
+    static constexpr int kNb = 64 / BM;                // selected blocks per key tile
+    static constexpr int kWarps = G * BM / 16;
     static constexpr int kThreads = 32 * kWarps;
-    static constexpr int kRows = 64 * G;
-    static constexpr int kTile = kM * kD * 2;          // one 64 x 128 bf16 tile
-    static constexpr int kQBytes = G * kTile;
-    static constexpr int kStage = 2 * kTile;           // K and V of one block
+    static constexpr int kRows = BM * G;
+    static constexpr int kTile = 64 * kD * 2;          // one 64 x 128 bf16 key tile
+    static constexpr int kQBytes = kRows * kD * 2;   // Q, then the O rows
+    static constexpr int kStage = 2 * kTile;           // K and V of one key tile
     static constexpr int kListOff = kQBytes + 2 * kStage;
     static size_t smem_bytes(int topk) { return (size_t)kListOff + (size_t)(topk + 1) * 4; }
 };
 
-}  // namespace
+template <int G, int BM>
+__device__ __forceinline__ void load_key_tile(uint32_t st, const __nv_bfloat16* Kg,
+                                              const __nv_bfloat16* Vg, const int* blist, int nblk,
+                                              int tile, int L, int tid) {
+    using C = FwdCfg<G, BM>;
+#pragma unroll
+    for (int j = 0; j < C::kNb; ++j) {
+        const int e = tile * C::kNb + j;
+        // a slot past the list is zero-filled (and masked by the caller)
+        const int row0 = e < nblk ? blist[e] * BM : 0;
+        const int lim = e < nblk ? L : 0;
+        load_rows<C::kThreads, BM>(st + j * BM * kD * 2, Kg, row0, lim, tid);
+        load_rows<C::kThreads, BM>(st + C::kTile + j * BM * kD * 2, Vg, row0, lim, tid);
+    }
+}
 
-namespace {
-
-template <int G>
-__global__ void __launch_bounds__(FwdCfg<G>::kThreads)
+template <int G, int BM>
+__global__ void __launch_bounds__(FwdCfg<G, BM>::kThreads)
 attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ K,
                 const __nv_bfloat16* __restrict__ V, const int32_t* __restrict__ idx,
                 const int32_t* __restrict__ cnt, int Hq, int Hkv, int L, int NQB, int topk,
                 float scale_log2, __nv_bfloat16* __restrict__ O, float* __restrict__ lse,
                 int* status) {
-    using C = FwdCfg<G>;
+    using C = FwdCfg<G, BM>;
     extern __shared__ __align__(128) uint8_t smem[];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int unit = blockIdx.x;
@@ -54,20 +72,20 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
 
     const __nv_bfloat16* Kg = K + (size_t)bg * L * kD;
     const __nv_bfloat16* Vg = V + (size_t)bg * L * kD;
+    // rows [hl*BM, hl*BM + BM) hold the query block's tokens of head g*G + hl
 #pragma unroll
     for (int hl = 0; hl < G; ++hl)
-        load_tile64<C::kThreads>(sQ + hl * C::kTile, Q + (size_t)(b * Hq + g * G + hl) * L * kD,
-                                 qb * kM, L, tid);
+        load_rows<C::kThreads, BM>(sQ + hl * BM * kD * 2,
+                                   Q + (size_t)(b * Hq + g * G + hl) * L * kD, qb * BM, L, tid);
     cp_async_commit();
     __syncthreads();
     const int nblk = blist[topk];
-    if (nblk > 0) {
-        load_tile64<C::kThreads>(sKV, Kg, blist[0] * kM, L, tid);
-        load_tile64<C::kThreads>(sKV + C::kTile, Vg, blist[0] * kM, L, tid);
-    }
+    const int ntile = (nblk + C::kNb - 1) / C::kNb;
+    if (ntile > 0) load_key_tile<G, BM>(sKV, Kg, Vg, blist, nblk, 0, L, tid);
     cp_async_commit();
 
-    const int rq0 = (warp & 3) * 16 + (lane >> 2);  // query row within the block (and +8)
+    const int tok0 = (warp * 16) % BM + (lane >> 2);  // token of this lane's rows (and +8)
+    const int hl = (warp * 16) / BM;                   // head of the warp's 16 rows
     uint32_t qf[8][4];
     float o[16][4];
 #pragma unroll
@@ -76,11 +94,10 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
         for (int e = 0; e < 4; ++e) o[n][e] = 0.f;
     float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
 
-    for (int it = 0; it < nblk; ++it) {
-        if (it + 1 < nblk) {
-            const uint32_t st = sKV + ((it + 1) & 1) * C::kStage;
-            load_tile64<C::kThreads>(st, Kg, blist[it + 1] * kM, L, tid);
-            load_tile64<C::kThreads>(st + C::kTile, Vg, blist[it + 1] * kM, L, tid);
+    for (int it = 0; it < ntile; ++it) {
+        if (it + 1 < ntile) {
+            load_key_tile<G, BM>(sKV + ((it + 1) & 1) * C::kStage, Kg, Vg, blist, nblk, it + 1, L,
+                                 tid);
             cp_async_commit();
             cp_async_wait<1>();
         } else {
@@ -93,7 +110,6 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
         }
         const uint32_t sK = sKV + (it & 1) * C::kStage;
         const uint32_t sV = sK + C::kTile;
-        const int t = blist[it];
 
         float s[8][4];
 #pragma unroll
@@ -110,14 +126,21 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
                 mma16816(s[2 * np + 1], qf[kc], bb[2], bb[3]);
             }
         }
-        const bool diag = (t == qb);
+        // key column -> (slot key / BM of the tile, key % BM inside its block);
+        // slots past the list are masked, and so are future tokens of the query's
+        // own block, which (the list being ascending, every entry <= qb) can only
+        // be the list's last entry
+        const int nvalid = nblk - it * C::kNb;
+        const int dslot = blist[nblk - 1] == qb ? nblk - 1 - it * C::kNb : -1;
 #pragma unroll
         for (int n = 0; n < 8; ++n)
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int key = n * 8 + (lane & 3) * 2 + (e & 1);
-                const int row = rq0 + ((e >> 1) << 3);
-                s[n][e] = (diag && key > row) ? -INFINITY : s[n][e] * scale_log2;
+                const int j = key / BM, kk = key % BM;
+                const int row = tok0 + ((e >> 1) << 3);
+                const bool dead = j >= nvalid || (j == dslot && kk > row);
+                s[n][e] = dead ? -INFINITY : s[n][e] * scale_log2;
             }
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -166,7 +189,7 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
     __syncthreads();
 
     // Epilogue: normalise, stage the warp's 16 rows in its own Q rows, store.
-    const int h = g * G + (warp >> 2);
+    const int h = g * G + hl;
     float inv[2];
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
@@ -174,7 +197,7 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
         l += __shfl_xor_sync(0xffffffffu, l, 1);
         l += __shfl_xor_sync(0xffffffffu, l, 2);
         inv[hh] = l > 0.f ? 1.0f / l : 0.f;
-        const int i = qb * kM + rq0 + hh * 8;
+        const int i = qb * BM + tok0 + hh * 8;
         if ((lane & 3) == 0 && i < L) {
             lse[(size_t)(b * Hq + h) * L + i] =
                 l > 0.f ? (mrow[hh] + log2f(l)) * kLn2 : -INFINITY;
@@ -198,7 +221,7 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
     for (int k = 0; k < 8; ++k) {
         const int e = k * 32 + lane;
         const int r = e >> 4, c = e & 15;
-        const int i = qb * kM + (warp & 3) * 16 + r;
+        const int i = qb * BM + (warp * 16) % BM + r;
         if (i < L) {
             const uint4 v = *reinterpret_cast<const uint4*>(sq + swz(warp * 16 + r, c));
             *reinterpret_cast<uint4*>(Oh + (size_t)i * kD + c * 8) = v;
@@ -206,19 +229,19 @@ attn_fwd_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __rest
     }
 }
 
-template <int G>
+template <int G, int BM>
 cudaError_t launch_fwd_g(const void* Q, const void* K, const void* V, const int32_t* idx,
                          const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                          void* O, float* lse, int* status, cudaStream_t st) {
-    const int NQB = (s.L + kM - 1) / kM;
-    const size_t smem = FwdCfg<G>::smem_bytes(topk);
-    auto kern = attn_fwd_kernel<G>;
+    const int NQB = (s.L + BM - 1) / BM;
+    const size_t smem = FwdCfg<G, BM>::smem_bytes(topk);
+    auto kern = attn_fwd_kernel<G, BM>;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const long long grid = (long long)s.B * s.Hkv * NQB;
     ProfScope prof(K_FWD, st);
-    kern<<<(unsigned)grid, FwdCfg<G>::kThreads, smem, st>>>(
+    kern<<<(unsigned)grid, FwdCfg<G, BM>::kThreads, smem, st>>>(
         static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(K),
         static_cast<const __nv_bfloat16*>(V), idx, cnt, s.Hq, s.Hkv, s.L, NQB, topk,
         sm_scale * kLog2e, static_cast<__nv_bfloat16*>(O), lse, status);
@@ -231,11 +254,15 @@ cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const i
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                             void* O, float* lse, int* status, cudaStream_t st) {
     if ((long long)s.B * s.Hkv * s.L == 0) return cudaSuccess;
-    // Two query heads per KV head fill a 128-row tcgen05 tile; a single head
-    // (64 rows) runs on the warp-level MMA kernel in this file.
-    if (s.Hq / s.Hkv == 2)
+    // Two query heads per KV head at m = 64 fill a 128-row tcgen05 tile; every
+    // other group and block size runs on the warp-level MMA kernel in this file.
+    const int G = s.Hq / s.Hkv, bm = s.block_size;
+    if (G == 2 && bm == 64)
         return launch_attn_fwd_tc(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st);
-    return launch_fwd_g<1>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st);
+#define PHSA_FWD(g_, bm_) launch_fwd_g<g_, bm_>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st)
+    if (G == 2) return bm == 16 ? PHSA_FWD(2, 16) : PHSA_FWD(2, 32);
+    return bm == 16 ? PHSA_FWD(1, 16) : bm == 32 ? PHSA_FWD(1, 32) : PHSA_FWD(1, 64);
+#undef PHSA_FWD
 }
 
 }  // namespace phsa

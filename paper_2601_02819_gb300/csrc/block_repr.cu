@@ -1,10 +1,11 @@
 // Stage (a): representative key of every KV block (Section 3.2, Eq. 6-8;
 // Algorithm 1 step 2).
 //
-// One warp reduces one 64 x 128 bf16 block (16 KB). Each half-warp streams one
+// One warp reduces one m x 128 bf16 block (m = 64: 16 KB; the kernel is
+// instantiated for m = 16, 32, 64). Each half-warp streams one
 // 256-byte row per step with 16-byte read-only loads (lane c of the half owns
 // columns 8c..8c+7), so a warp keeps eight 512-byte row pairs in flight. The
-// punctuation count of the block comes from two warp ballots over the 64 mask
+// punctuation count of the block comes from warp ballots over its m mask
 // bytes. The sum and the punctuation-masked sum are kept in fp32 and combined
 // once across the two half-warps; the result is rounded to bf16 once.
 // The kernel is bound by HBM: it reads K and the mask once and writes T rows.
@@ -29,14 +30,16 @@ __device__ __forceinline__ void add8(float* acc, const uint4& v) {
     }
 }
 
-// One warp: the representative key of the 64 x 128 block at Kb (row stride 128)
-// with punctuation bytes mb[0..64), written as 128 bf16 values to out.
+// One warp: the representative key of the BM x 128 block at Kb (row stride
+// 128) with punctuation bytes mb[0..BM), written as 128 bf16 values to out.
+template <int BM>
 __device__ __forceinline__ void repr_one_block(const __nv_bfloat16* __restrict__ Kb,
                                                const uint8_t* __restrict__ mb, float lambda,
                                                __nv_bfloat16* __restrict__ out, int lane) {
-    // Punctuation indicator of the block's 64 tokens.
-    const unsigned lo = __ballot_sync(0xffffffffu, mb[lane] != 0);
-    const unsigned hi = __ballot_sync(0xffffffffu, mb[32 + lane] != 0);
+    static_assert(BM == 16 || BM == 32 || BM == 64, "block size");
+    // Punctuation indicator of the block's BM tokens (bit r: token r).
+    const unsigned lo = __ballot_sync(0xffffffffu, lane < BM && mb[lane < BM ? lane : 0] != 0);
+    const unsigned hi = BM > 32 ? __ballot_sync(0xffffffffu, mb[(BM > 32 ? 32 : 0) + lane] != 0) : 0u;
     const int c = __popc(lo) + __popc(hi);
 
     const int half = lane >> 4;
@@ -48,7 +51,7 @@ __device__ __forceinline__ void repr_one_block(const __nv_bfloat16* __restrict__
     for (int j = 0; j < 8; ++j) { s0[j] = 0.f; sp[j] = 0.f; }
 
 #pragma unroll
-    for (int base = 0; base < kM; base += 16) {
+    for (int base = 0; base < BM; base += 16) {
         uint4 v[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
@@ -70,7 +73,7 @@ __device__ __forceinline__ void repr_one_block(const __nv_bfloat16* __restrict__
     }
     if (half == 0) {
         float o[8];
-        const float inv_m = 1.0f / kM;
+        const float inv_m = 1.0f / BM;
         const float inv_c = c > 0 ? 1.0f / (float)c : 0.f;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
@@ -87,6 +90,7 @@ __device__ __forceinline__ void repr_one_block(const __nv_bfloat16* __restrict__
     }
 }
 
+template <int BM>
 __global__ void __launch_bounds__(kWarpsPerCta * 32)
 block_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict__ mask, int Hkv,
                   int L, int T, long long n_blocks, float lambda,
@@ -97,8 +101,9 @@ block_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict
     const int t = (int)(wid % T);
     const long long bg = wid / T;  // b * Hkv + g
     const int b = (int)(bg / Hkv);
-    repr_one_block(K + ((size_t)bg * L + (size_t)t * kM) * kD, mask + (size_t)b * L + (size_t)t * kM,
-                   lambda, Krepr + ((size_t)bg * T + t) * kD, lane);
+    repr_one_block<BM>(K + ((size_t)bg * L + (size_t)t * BM) * kD,
+                       mask + (size_t)b * L + (size_t)t * BM, lambda,
+                       Krepr + ((size_t)bg * T + t) * kD, lane);
 }
 
 // Decode: one CTA of four warps per (sequence, KV head). A sequence whose
@@ -172,12 +177,15 @@ decode_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restric
 
 cudaError_t launch_block_repr(const void* K, const uint8_t* mask, const phsa_shape& s,
                               float lambda, void* Krepr, cudaStream_t st) {
-    const int T = s.L / kM;
+    const int bm = s.block_size;
+    if (bm != 16 && bm != 32 && bm != 64) return cudaErrorInvalidValue;
+    const int T = s.L / bm;
     const long long n_blocks = (long long)s.B * s.Hkv * T;
     if (n_blocks == 0) return cudaSuccess;
     const long long grid = (n_blocks + kWarpsPerCta - 1) / kWarpsPerCta;
+    auto kern = bm == 16 ? block_repr_kernel<16> : bm == 32 ? block_repr_kernel<32> : block_repr_kernel<64>;
     ProfScope prof(K_REPR, st);
-    block_repr_kernel<<<(unsigned)grid, kWarpsPerCta * 32, 0, st>>>(
+    kern<<<(unsigned)grid, kWarpsPerCta * 32, 0, st>>>(
         static_cast<const __nv_bfloat16*>(K), mask, s.Hkv, s.L, T, n_blocks, lambda,
         static_cast<__nv_bfloat16*>(Krepr));
     return cudaGetLastError();

@@ -29,15 +29,18 @@ int* status_ptr() {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Common shape checks; returns PHSA_OK or an error code.
-int check_shape(const phsa_shape& s) {
+// Common shape checks; returns PHSA_OK or an error code. Block sizes 16 and
+// 32 are accepted only by the prefill forward calls (any_block).
+int check_shape(const phsa_shape& s, bool any_block = false) {
     if (s.B < 0 || s.L < 0 || s.Hq <= 0 || s.Hkv <= 0 || s.D <= 0 || s.block_size <= 0)
         return PHSA_ERR_INVALID_ARG;
     if (s.Hq % s.Hkv != 0) return PHSA_ERR_INVALID_ARG;
-    if (s.D != phsa::kD || s.block_size != phsa::kM) return PHSA_ERR_UNSUPPORTED;
+    if (s.D != phsa::kD) return PHSA_ERR_UNSUPPORTED;
+    const int bm = s.block_size;
+    if (any_block ? (bm != 16 && bm != 32 && bm != 64) : bm != phsa::kM) return PHSA_ERR_UNSUPPORTED;
     const int G = s.Hq / s.Hkv;
     if (G != 1 && G != 2) return PHSA_ERR_UNSUPPORTED;
-    const long long nqb = ((long long)s.L + phsa::kM - 1) / phsa::kM;
+    const long long nqb = ((long long)s.L + bm - 1) / bm;
     if ((long long)s.B * s.Hkv * nqb > 0x7fffffffLL) return PHSA_ERR_UNSUPPORTED;
     if ((long long)s.B * s.Hq > 0x7fffffffLL / (s.L > 0 ? s.L : 1)) return PHSA_ERR_UNSUPPORTED;
     if (s.B > 65535 * 8 || (long long)s.B * s.Hkv > 65535) return PHSA_ERR_UNSUPPORTED;
@@ -68,10 +71,10 @@ extern "C" {
 
 int phsa_build_block_repr(const void* K, const uint8_t* punct_mask, phsa_shape s, float lambda,
                           void* Krepr, void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
-    if (empty(s) || s.L < phsa::kM) return PHSA_OK;  // no full block: nothing to write
+    if (empty(s) || s.L < s.block_size) return PHSA_OK;  // no full block: nothing to write
     if (!K || !punct_mask || !Krepr || !aligned16(K) || !aligned16(Krepr))
         return PHSA_ERR_INVALID_ARG;
     return from_cuda(phsa::launch_block_repr(K, punct_mask, s, lambda, Krepr,
@@ -80,7 +83,7 @@ int phsa_build_block_repr(const void* K, const uint8_t* punct_mask, phsa_shape s
 
 int phsa_select_blocks(const void* Q, const void* Krepr, phsa_shape s, phsa_select_params p,
                        int32_t* block_idx, int32_t* block_cnt, void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
     if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
@@ -88,7 +91,7 @@ int phsa_select_blocks(const void* Q, const void* Krepr, phsa_shape s, phsa_sele
         return PHSA_ERR_INVALID_ARG;
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (empty(s)) return PHSA_OK;
-    const bool need_repr = s.L >= 2 * phsa::kM;  // some query block has a candidate
+    const bool need_repr = s.L >= 2 * s.block_size;  // some query block has a candidate
     if (!Q || !block_idx || !block_cnt || !aligned16(Q) || (need_repr && (!Krepr || !aligned16(Krepr))))
         return PHSA_ERR_INVALID_ARG;
     if (phsa::select_smem_bytes(s, p.topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
@@ -99,7 +102,7 @@ int phsa_select_blocks(const void* Q, const void* Krepr, phsa_shape s, phsa_sele
 int phsa_sparse_attn_fwd(const void* Q, const void* K, const void* V, const int32_t* block_idx,
                          const int32_t* block_cnt, phsa_shape s, int topk, float sm_scale,
                          void* O, float* lse, void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if ((rc = check_topk(s, topk)) != PHSA_OK) return rc;
     if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;

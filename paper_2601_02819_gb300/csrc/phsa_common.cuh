@@ -115,6 +115,23 @@ __device__ __forceinline__ void load_tile64(uint32_t dst, const __nv_bfloat16* s
     }
 }
 
+// Copies ROWS rows (a [ROWS][128] bf16 tile) starting at row `row0` of a
+// [nrows][128] matrix into swizzled shared memory; rows >= nrows are
+// zero-filled. ROWS * 16 must be a multiple of NTHREADS.
+template <int NTHREADS, int ROWS>
+__device__ __forceinline__ void load_rows(uint32_t dst, const __nv_bfloat16* src, int row0,
+                                          int nrows, int tid) {
+    static_assert((ROWS * kRowChunks) % NTHREADS == 0, "tile split");
+#pragma unroll
+    for (int it = 0; it < (ROWS * kRowChunks) / NTHREADS; ++it) {
+        int e = it * NTHREADS + tid;
+        int r = e / kRowChunks, c = e % kRowChunks;
+        bool ok = row0 + r < nrows;
+        const __nv_bfloat16* p = src + (size_t)(ok ? row0 + r : 0) * kD + c * 8;
+        cp_async16(dst + swz(r, c), p, ok);
+    }
+}
+
 // Copies the valid entries of a selected-block list into shared memory.
 // Valid: 0 <= t <= qb and strictly ascending; -1 entries are skipped silently;
 // anything else is skipped and recorded in the status word. Returns the count.

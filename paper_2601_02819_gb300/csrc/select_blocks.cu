@@ -1,9 +1,10 @@
 // Stage (b): query-to-block relevance and Top-K block selection (Eq. 8;
-// Algorithm 1 step 3), one CTA per (query block qb, KV head g).
+// Algorithm 1 step 3), one CTA per (query block qb, KV head g), for block
+// sizes m = 16, 32, 64.
 //
-// The G*64 query rows of the group are held as bf16 MMA fragments (one warp
+// The G*m query rows of the group are held as bf16 MMA fragments (one warp
 // per 16 rows). The candidate representative keys C = [n_init, qb - n_local]
-// are streamed through shared memory in 64-row tiles (double-buffered
+// are streamed through shared memory in tiles of 64 candidates (double-buffered
 // cp.async). Scores never leave the SM:
 //   pass 1  S = q . Krepr^T * scale, running row max and row sum (online
 //           softmax over the candidates only);
@@ -23,13 +24,15 @@ namespace phsa {
 
 namespace {
 
-template <int G>
+constexpr int kCT = 64;  // candidates per Krepr tile
+
+template <int G, int BM>
 struct SelCfg {
-    static constexpr int kWarps = 4 * G;
+    static constexpr int kWarps = G * BM / 16;
     static constexpr int kThreads = 32 * kWarps;
-    static constexpr int kRows = 64 * G;
+    static constexpr int kRows = BM * G;
     static constexpr int kQBytes = kRows * kD * 2;
-    static constexpr int kTileBytes = kM * kD * 2;
+    static constexpr int kTileBytes = kCT * kD * 2;  // one Krepr tile
     static constexpr int kPartOff = kQBytes + 2 * kTileBytes;          // float [kWarps][64]
     static constexpr int kBestOff = kPartOff + kWarps * 64 * 4;        // u64 [kWarps]
     static constexpr int kAOff = kBestOff + kWarps * 8;                // float [nC]
@@ -42,13 +45,13 @@ __device__ __forceinline__ unsigned long long u64_max(unsigned long long a, unsi
     return a > b ? a : b;
 }
 
-template <int G>
-__global__ void __launch_bounds__(SelCfg<G>::kThreads)
+template <int G, int BM>
+__global__ void __launch_bounds__(SelCfg<G, BM>::kThreads)
 select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ Krepr,
                      int Hq, int Hkv, int L, int T, int NQB, int topk, int n_init, int n_local,
                      int agg, float scale_log2, float scale, int32_t* __restrict__ idx_out,
                      int32_t* __restrict__ cnt_out) {
-    using C = SelCfg<G>;
+    using C = SelCfg<G, BM>;
     extern __shared__ __align__(128) uint8_t smem[];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int unit = blockIdx.x;
@@ -85,21 +88,22 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
     float* A = reinterpret_cast<float*>(smem + C::kAOff);
     int* sel = reinterpret_cast<int*>(smem + C::kAOff + (size_t)NQB * 4);
 
-    // Query rows of every head of the group: tile hl holds head g*G + hl.
+    // Query rows of every head of the group: rows [hl*BM, hl*BM + BM) hold head g*G + hl.
 #pragma unroll
     for (int hl = 0; hl < G; ++hl) {
         const __nv_bfloat16* Qh = Q + ((size_t)(b * Hq + g * G + hl) * L) * kD;
-        load_tile64<C::kThreads>(sQ + hl * C::kTileBytes, Qh, qb * kM, L, tid);
+        load_rows<C::kThreads, BM>(sQ + hl * BM * kD * 2, Qh, qb * BM, L, tid);
     }
     const __nv_bfloat16* Kr = Krepr + (size_t)bg * T * kD;
-    const int n_tiles = (nC + kM - 1) / kM;
-    load_tile64<C::kThreads>(sK, Kr, c_lo, c_hi + 1, tid);
+    const int n_tiles = (nC + kCT - 1) / kCT;
+    load_rows<C::kThreads, kCT>(sK, Kr, c_lo, c_hi + 1, tid);
     cp_async_commit();
 
-    // Row bookkeeping: this lane holds rows r0 and r0 + 8 of the warp's 16.
+    // Row bookkeeping: this lane holds rows r0 and r0 + 8 of the warp's 16
+    // (row r: token r % BM of head r / BM).
     const int r0 = warp * 16 + (lane >> 2);
-    const bool row_ok0 = qb * kM + (r0 & 63) < L;
-    const bool row_ok1 = qb * kM + ((r0 + 8) & 63) < L;
+    const bool row_ok0 = qb * BM + (r0 & (BM - 1)) < L;
+    const bool row_ok1 = qb * BM + ((r0 + 8) & (BM - 1)) < L;
 
     uint32_t qf[8][4];
     float mrow[2] = {-INFINITY, -INFINITY}, zrow[2] = {0.f, 0.f}, inv_z[2] = {0.f, 0.f};
@@ -110,8 +114,8 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
             const int it = pass * n_tiles + j;
             if (it + 1 < n_pass * n_tiles) {
                 const int jn = (j + 1 < n_tiles) ? j + 1 : 0;
-                load_tile64<C::kThreads>(sK + ((it + 1) & 1) * C::kTileBytes, Kr, c_lo + jn * kM,
-                                         c_hi + 1, tid);
+                load_rows<C::kThreads, kCT>(sK + ((it + 1) & 1) * C::kTileBytes, Kr,
+                                            c_lo + jn * kCT, c_hi + 1, tid);
                 cp_async_commit();
                 cp_async_wait<1>();
             } else {
@@ -140,7 +144,7 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
             }
             // scale (to the log2 domain for the softmax) and mask columns past the
             // candidate range; for max logits also the rows past L
-            const int col0 = c_lo + j * kM + (lane & 3) * 2;
+            const int col0 = c_lo + j * kCT + (lane & 3) * 2;
             const float sc = agg ? scale : scale_log2;
 #pragma unroll
             for (int n = 0; n < 8; ++n)
@@ -164,11 +168,11 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
                     }
                 }
                 __syncthreads();
-                if (tid < kM) {
+                for (int x = tid; x < kCT; x += C::kThreads) {
                     float a = -INFINITY;
 #pragma unroll
-                    for (int w = 0; w < C::kWarps; ++w) a = fmaxf(a, part[w * 64 + tid]);
-                    const int c = j * kM + tid;
+                    for (int w = 0; w < C::kWarps; ++w) a = fmaxf(a, part[w * 64 + x]);
+                    const int c = j * kCT + x;
                     if (c < nC) A[c] = a;
                 }
             } else if (pass == 0) {
@@ -201,11 +205,11 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
                     }
                 }
                 __syncthreads();
-                if (tid < kM) {
+                for (int x = tid; x < kCT; x += C::kThreads) {
                     float a = 0.f;
 #pragma unroll
-                    for (int w = 0; w < C::kWarps; ++w) a += part[w * 64 + tid];
-                    const int c = j * kM + tid;
+                    for (int w = 0; w < C::kWarps; ++w) a += part[w * 64 + x];
+                    const int c = j * kCT + x;
                     if (c < nC) A[c] = (a >= 0.f) ? a : 0.f;  // NaN inputs rank as zero
                 }
             }
@@ -267,8 +271,8 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
         else if (j >= n_init_q + ksel && j < nF + ksel) out[j] = loc_lo + (j - n_init_q - ksel);
         else if (j >= nF + ksel) out[j] = -1;
     }
-    if (tid < ksel) {
-        const int v = sel[tid];
+    for (int j = tid; j < ksel; j += C::kThreads) {
+        const int v = sel[j];
         int rank = 0;
         for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
         out[n_init_q + rank] = v;
@@ -276,18 +280,18 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
     if (tid == 0) cnt_out[out_unit] = nF + ksel;
 }
 
-template <int G>
+template <int G, int BM>
 cudaError_t launch_select_g(const phsa_shape& s, const phsa_select_params& p, const void* Q,
                             const void* Krepr, int32_t* idx, int32_t* cnt, cudaStream_t st) {
-    const int T = s.L / kM, NQB = (s.L + kM - 1) / kM;
-    const size_t smem = SelCfg<G>::smem_bytes(NQB, p.topk);
-    auto kern = select_blocks_kernel<G>;
+    const int T = s.L / BM, NQB = (s.L + BM - 1) / BM;
+    const size_t smem = SelCfg<G, BM>::smem_bytes(NQB, p.topk);
+    auto kern = select_blocks_kernel<G, BM>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
     const long long grid = (long long)s.B * s.Hkv * NQB;
     ProfScope prof(K_SELECT, st);
-    kern<<<(unsigned)grid, SelCfg<G>::kThreads, smem, st>>>(
+    kern<<<(unsigned)grid, SelCfg<G, BM>::kThreads, smem, st>>>(
         static_cast<const __nv_bfloat16*>(Q), static_cast<const __nv_bfloat16*>(Krepr), s.Hq,
         s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, p.aggregation, p.sm_scale * kLog2e,
         p.sm_scale, idx, cnt);
@@ -297,18 +301,29 @@ cudaError_t launch_select_g(const phsa_shape& s, const phsa_select_params& p, co
 }  // namespace
 
 size_t select_smem_bytes(const phsa_shape& s, int topk) {
-    const int NQB = (s.L + kM - 1) / kM;
-    return (s.Hq / s.Hkv == 2) ? select_tc_smem_bytes(s, topk) : SelCfg<1>::smem_bytes(NQB, topk);
+    const int bm = s.block_size, NQB = (s.L + bm - 1) / bm;
+    const int G = s.Hq / s.Hkv;
+    if (G == 2 && bm == kM) return select_tc_smem_bytes(s, topk);
+    // every instantiation has the same layout apart from the Q rows
+    return G == 2 ? SelCfg<2, 64>::smem_bytes(NQB, topk) : SelCfg<1, 64>::smem_bytes(NQB, topk);
 }
 
 cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_shape& s,
                                  const phsa_select_params& p, int32_t* idx, int32_t* cnt,
                                  int* status, cudaStream_t st) {
-    if ((long long)s.B * s.Hkv * ((s.L + kM - 1) / kM) == 0) return cudaSuccess;
-    // Two query heads per KV head fill a 128-row tcgen05 tile (select_tc.cu); a
-    // single head runs on the warp-level MMA kernel in this file.
-    if (s.Hq / s.Hkv == 2) return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
-    return launch_select_g<1>(s, p, Q, Krepr, idx, cnt, st);
+    const int bm = s.block_size;
+    if ((long long)s.B * s.Hkv * ((s.L + bm - 1) / bm) == 0) return cudaSuccess;
+    // Two query heads per KV head at m = 64 fill a 128-row tcgen05 tile
+    // (select_tc.cu); every other group size and block size runs on the
+    // warp-level MMA kernel in this file.
+    const int G = s.Hq / s.Hkv;
+    if (G == 2 && bm == 64) return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
+    if (G == 2)
+        return bm == 16 ? launch_select_g<2, 16>(s, p, Q, Krepr, idx, cnt, st)
+                        : launch_select_g<2, 32>(s, p, Q, Krepr, idx, cnt, st);
+    return bm == 16   ? launch_select_g<1, 16>(s, p, Q, Krepr, idx, cnt, st)
+           : bm == 32 ? launch_select_g<1, 32>(s, p, Q, Krepr, idx, cnt, st)
+                      : launch_select_g<1, 64>(s, p, Q, Krepr, idx, cnt, st);
 }
 
 }  // namespace phsa

@@ -163,33 +163,37 @@ def phsa_version() -> str:
     return load().phsa_version().decode()
 
 
-def phsa_build_block_repr(K, punct_mask, lam: float, Krepr=None, stream=None):
-    """Stage (a): representative keys [B, Hkv, L // 64, D] (bf16)."""
+def phsa_build_block_repr(K, punct_mask, lam: float, Krepr=None, stream=None,
+                          block_size: int = BLOCK_SIZE):
+    """Stage (a): representative keys [B, Hkv, L // m, D] (bf16), m = block_size
+    (64; 16 and 32 are accepted too)."""
     _check(K, "K", torch.bfloat16, 4)
     _check(punct_mask, "punct_mask", torch.uint8, 2)
     B, Hkv, L, D = K.shape
     if tuple(punct_mask.shape) != (B, L):
         raise ValueError("punct_mask must be [B, L]")
-    T = L // BLOCK_SIZE
+    T = L // int(block_size)
     if Krepr is None:
         Krepr = torch.empty((B, Hkv, T, D), dtype=torch.bfloat16, device=K.device)
     _check(Krepr, "Krepr", torch.bfloat16, 4)
-    rc = load().phsa_build_block_repr(_ptr(K), _ptr(punct_mask), make_shape(B, L, Hkv, Hkv, D),
-                                      float(lam), _ptr(Krepr), _stream(stream))
+    rc = load().phsa_build_block_repr(_ptr(K), _ptr(punct_mask),
+                                      make_shape(B, L, Hkv, Hkv, D, block_size), float(lam),
+                                      _ptr(Krepr), _stream(stream))
     _raise("phsa_build_block_repr", rc)
     return Krepr
 
 
 def phsa_select_blocks(Q, Krepr, Hkv: int, topk: int, n_init: int = 1, n_local: int = 1,
                        sm_scale: float | None = None, block_idx=None, block_cnt=None,
-                       stream=None, aggregation: str = "softmax_sum"):
+                       stream=None, aggregation: str = "softmax_sum",
+                       block_size: int = BLOCK_SIZE):
     """Stage (b): (block_idx [B, Hkv, NQB, topk] int32, block_cnt [B, Hkv, NQB] int32).
     ``aggregation``: "softmax_sum" (Eq. 8 probabilities summed over the unit's
     rows) or "max_logit" (the largest raw score over the rows)."""
     _check(Q, "Q", torch.bfloat16, 4)
     _check(Krepr, "Krepr", torch.bfloat16, 4)
     B, Hq, L, D = Q.shape
-    NQB = -(-L // BLOCK_SIZE)
+    NQB = -(-L // int(block_size))
     if sm_scale is None:
         sm_scale = D ** -0.5
     if block_idx is None:
@@ -199,14 +203,14 @@ def phsa_select_blocks(Q, Krepr, Hkv: int, topk: int, n_init: int = 1, n_local: 
     _check(block_idx, "block_idx", torch.int32, 4)
     _check(block_cnt, "block_cnt", torch.int32, 3)
     p = _params(topk, n_init, n_local, sm_scale, aggregation)
-    rc = load().phsa_select_blocks(_ptr(Q), _ptr(Krepr), make_shape(B, L, Hq, Hkv, D), p,
-                                   _ptr(block_idx), _ptr(block_cnt), _stream(stream))
+    rc = load().phsa_select_blocks(_ptr(Q), _ptr(Krepr), make_shape(B, L, Hq, Hkv, D, block_size),
+                                   p, _ptr(block_idx), _ptr(block_cnt), _stream(stream))
     _raise("phsa_select_blocks", rc)
     return block_idx, block_cnt
 
 
 def phsa_sparse_attn_fwd(Q, K, V, block_idx, block_cnt, sm_scale: float | None = None, O=None,
-                         lse=None, stream=None):
+                         lse=None, stream=None, block_size: int = BLOCK_SIZE):
     """Stage (c) forward: (O [B, Hq, L, D] bf16, lse [B, Hq, L] fp32)."""
     _check(Q, "Q", torch.bfloat16, 4)
     _check(K, "K", torch.bfloat16, 4)
@@ -225,8 +229,8 @@ def phsa_sparse_attn_fwd(Q, K, V, block_idx, block_cnt, sm_scale: float | None =
     _check(O, "O", torch.bfloat16, 4)
     _check(lse, "lse", torch.float32, 3)
     rc = load().phsa_sparse_attn_fwd(_ptr(Q), _ptr(K), _ptr(V), _ptr(block_idx), _ptr(block_cnt),
-                                     make_shape(B, L, Hq, Hkv, D), int(topk), float(sm_scale),
-                                     _ptr(O), _ptr(lse), _stream(stream))
+                                     make_shape(B, L, Hq, Hkv, D, block_size), int(topk),
+                                     float(sm_scale), _ptr(O), _ptr(lse), _stream(stream))
     _raise("phsa_sparse_attn_fwd", rc)
     return O, lse
 
@@ -535,10 +539,12 @@ def phsa_selftest_tcgen05(A, B, V, stream=None):
 
 
 def phsa_forward(Q, K, V, punct_mask, lam: float, topk: int, n_init: int = 1, n_local: int = 1,
-                 sm_scale: float | None = None, stream=None, aggregation: str = "softmax_sum"):
+                 sm_scale: float | None = None, stream=None, aggregation: str = "softmax_sum",
+                 block_size: int = BLOCK_SIZE):
     """The whole forward hot path: (a) -> (b) -> (c). Returns (O, lse, block_idx, block_cnt, Krepr)."""
-    Krepr = phsa_build_block_repr(K, punct_mask, lam, stream=stream)
+    Krepr = phsa_build_block_repr(K, punct_mask, lam, stream=stream, block_size=block_size)
     idx, cnt = phsa_select_blocks(Q, Krepr, K.shape[1], topk, n_init, n_local, sm_scale,
-                                  stream=stream, aggregation=aggregation)
-    O, lse = phsa_sparse_attn_fwd(Q, K, V, idx, cnt, sm_scale, stream=stream)
+                                  stream=stream, aggregation=aggregation, block_size=block_size)
+    O, lse = phsa_sparse_attn_fwd(Q, K, V, idx, cnt, sm_scale, stream=stream,
+                                  block_size=block_size)
     return O, lse, idx, cnt, Krepr

@@ -62,8 +62,17 @@ def test_host_validation_needs_no_gpu(lib):
     ok = phsa_shape(1, 4096, 16, 8, 128, 64)
     assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 16, 8, 64, 64), 0.5, None,
                                      None) == -2  # D = 64 unsupported
-    assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 16, 8, 128, 16), 0.5, None,
-                                     None) == -2  # block size 16 unsupported
+    for bs in (16, 32):  # the prefill forward calls take m = 16 and 32: past the block
+        # size check, a null pointer is what they reject
+        assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 16, 8, 128, bs), 0.5,
+                                         None, None) == -1
+        assert lib.phsa_select_blocks(None, None, phsa_shape(1, 4096, 16, 8, 128, bs),
+                                      phsa_select_params(8, 1, 1, 0.088), None, None, None) == -1
+        # the backward and its workspace stay at m = 64
+        assert lib.phsa_sparse_attn_bwd_workspace(phsa_shape(1, 4096, 16, 8, 128, bs), 14) == 0
+    for bs in (8, 48, 128):
+        assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 16, 8, 128, bs), 0.5,
+                                         None, None) == -2  # other block sizes unsupported
     assert lib.phsa_build_block_repr(None, None, phsa_shape(1, 4096, 12, 8, 128, 64), 0.5, None,
                                      None) == -1  # Hq not a multiple of Hkv
     assert lib.phsa_build_block_repr(None, None, ok, 1.5, None, None) == -1  # lambda > 1

@@ -1,0 +1,164 @@
+"""Block sizes 16 and 32 on the GPU vs the oracle: representative keys (Eq. 6-8),
+selection (Eq. 8, Algorithm 1 step 3) and sparse attention forward (Eq. 10-11).
+
+The paper's experiments use blocks of 16 tokens. Each stage gets the oracle's
+inputs for it (the oracle's representative keys for the selection, the
+oracle's block lists for the attention), so every check isolates one kernel;
+the end-to-end case runs the three calls in a row.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2601_02819_gb300 import inputs, phsa
+from parity import (LSE_ABS, assert_close, bf16_bits, bf16_to_f64, compare_selection,
+                    to_dev_bf16, ulp_distance)
+
+pytestmark = pytest.mark.gpu
+
+D = 128
+SCALE = D ** -0.5
+
+
+def rand(rng, *s):
+    return inputs.f32_to_bf16_bits(rng.standard_normal(s).astype(np.float32))
+
+
+@pytest.mark.parametrize("m,L,lam", [(16, 16 * 50 + 7, 0.5), (16, 16 * 64, 0.0), (32, 32 * 33 + 31, 1.0),
+                                     (32, 32 * 20, 0.3)])
+def test_block_repr_matches_oracle(m, L, lam):
+    rng = np.random.default_rng(m + L)
+    K = rand(rng, 2, 3, L, D)
+    mask = (rng.random((2, L)) < 0.08).astype(np.uint8)
+    mask[0, :m] = 1      # an all-punctuation block
+    mask[1, m:2 * m] = 0  # a block without punctuation
+    got = phsa.phsa_build_block_repr(to_dev_bf16(K), torch.from_numpy(mask).cuda(), lam,
+                                     block_size=m)
+    torch.cuda.synchronize()
+    ref = oracle.block_repr(K, mask, m, lam)
+    assert got.shape == ref.shape == (2, 3, L // m, D)
+    assert ulp_distance(bf16_bits(got), ref).max() <= 1
+
+
+def gpu_select(Q, Kr, Hkv, topk, n_init, n_local, m, aggregation="softmax_sum"):
+    idx, cnt = phsa.phsa_select_blocks(to_dev_bf16(Q), to_dev_bf16(Kr), Hkv, topk, n_init,
+                                       n_local, SCALE, aggregation=aggregation, block_size=m)
+    torch.cuda.synchronize()
+    return idx.cpu().numpy(), cnt.cpu().numpy()
+
+
+@pytest.mark.parametrize("m,B,Hq,Hkv,L,topk,n_init,n_local", [
+    (16, 1, 2, 1, 16 * 97 + 5, 8, 1, 1),      # G = 2, ragged tail
+    (16, 2, 2, 2, 16 * 80, 6, 1, 2),          # G = 1
+    (16, 1, 4, 2, 16 * 256, 56, 8, 32),       # the paper's 32k forced sets (8 + 32 blocks of 16)
+    (16, 1, 2, 1, 16 * 40, 41, 1, 1),         # budget covers everything: dense rows
+    (32, 1, 4, 2, 32 * 70 + 19, 10, 1, 1),    # m = 32, G = 2
+    (32, 1, 3, 3, 32 * 50, 7, 2, 2),          # m = 32, G = 1
+])
+@pytest.mark.parametrize("aggregation", ["softmax_sum", "max_logit"])
+def test_selection_matches_oracle(m, B, Hq, Hkv, L, topk, n_init, n_local, aggregation):
+    rng = np.random.default_rng(L + topk)
+    Q, K = rand(rng, B, Hq, L, D), rand(rng, B, Hkv, L, D)
+    mask = (rng.random((B, L)) < 0.06).astype(np.uint8)
+    Kr = oracle.block_repr(K, mask, m, 0.5)
+    gi, gc = gpu_select(Q, Kr, Hkv, topk, n_init, n_local, m, aggregation)
+    oi, oc, oa = oracle.select_blocks(Q, Kr, L, m, topk, n_init, n_local, SCALE, want_agg=True,
+                                      aggregation=aggregation)
+    assert gi.shape == oi.shape == (B, Hkv, -(-L // m), topk)
+    bad, excl, differ, msgs = compare_selection(gi, gc, oi, oc, oa)
+    assert bad == 0, msgs[:5]
+    assert differ <= max(2, 0.01 * oc.size), (differ, oc.size)
+
+
+def test_selection_exact_ties_go_to_the_lower_block_at_m16():
+    rng = np.random.default_rng(9)
+    L, T = 16 * 24, 24
+    Q = rand(rng, 1, 2, L, D)
+    row = rand(rng, D)
+    Kr = np.broadcast_to(row, (1, 1, T, D)).copy()
+    gi, gc = gpu_select(Q, Kr, 1, 6, 1, 1, 16)
+    for qb in range(6, 24):
+        assert list(gi[0, 0, qb]) == [0, 1, 2, 3, 4, qb], qb
+
+
+def gpu_fwd(Q, K, V, idx, cnt, m):
+    O, lse = phsa.phsa_sparse_attn_fwd(to_dev_bf16(Q), to_dev_bf16(K), to_dev_bf16(V),
+                                       torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda(),
+                                       block_size=m)
+    torch.cuda.synchronize()
+    return O, lse
+
+
+@pytest.mark.parametrize("m,B,Hq,Hkv,L,topk", [
+    (16, 1, 2, 1, 16 * 70 + 9, 7),    # G = 2, ragged tail; key tiles of four blocks, some short
+    (16, 2, 4, 2, 16 * 33, 5),        # B = 2
+    (16, 1, 3, 3, 16 * 41 + 1, 6),    # G = 1, a one-token tail block
+    (16, 1, 2, 1, 11, 2),             # shorter than one block
+    (32, 1, 4, 2, 32 * 25 + 17, 4),   # m = 32: key tiles of two blocks
+    (32, 1, 2, 2, 32 * 18, 3),        # m = 32, G = 1
+])
+def test_forward_matches_oracle(m, B, Hq, Hkv, L, topk):
+    rng = np.random.default_rng(L * 3 + m)
+    Q, K, V = rand(rng, B, Hq, L, D), rand(rng, B, Hkv, L, D), rand(rng, B, Hkv, L, D)
+    mask = (rng.random((B, L)) < 0.06).astype(np.uint8)
+    Kr = oracle.block_repr(K, mask, m, 0.5)
+    idx, cnt = oracle.select_blocks(Q, Kr, L, m, topk, 1, 1, SCALE)
+    O, lse = gpu_fwd(Q, K, V, idx, cnt, m)
+    Or, lser = oracle.sparse_attn_fwd(Q, K, V, idx, cnt, m, SCALE)
+    assert_close("O", bf16_to_f64(O), Or)
+    assert np.abs(lse.cpu().numpy() - lser).max() <= LSE_ABS
+    assert phsa.phsa_get_device_status() == 0
+
+
+@pytest.mark.parametrize("m", [16, 32])
+def test_forward_full_budget_is_dense_causal(m):
+    B, Hq, Hkv, L = 1, 4, 2, m * 21 + 5
+    NQB = -(-L // m)
+    rng = np.random.default_rng(m)
+    Q, K, V = rand(rng, B, Hq, L, D), rand(rng, B, Hkv, L, D), rand(rng, B, Hkv, L, D)
+    idx = np.full((B, Hkv, NQB, NQB), -1, np.int32)
+    cnt = np.zeros((B, Hkv, NQB), np.int32)
+    for qb in range(NQB):
+        idx[:, :, qb, :qb + 1] = np.arange(qb + 1)
+        cnt[:, :, qb] = qb + 1
+    O, lse = gpu_fwd(Q, K, V, idx, cnt, m)
+    Od, lsed = oracle.dense_causal(Q, K, V, SCALE)
+    assert_close("O", bf16_to_f64(O), Od)
+    assert np.abs(lse.cpu().numpy() - lsed).max() <= LSE_ABS
+
+
+def test_forward_constant_values_give_constant_output_at_m16():
+    rng = np.random.default_rng(4)
+    L, m = 16 * 30, 16
+    Q, K = rand(rng, 1, 2, L, D), rand(rng, 1, 1, L, D)
+    V = np.full((1, 1, L, D), inputs.f32_to_bf16_bits(np.array([0.75], np.float32))[0], np.uint16)
+    Kr = oracle.block_repr(K, np.zeros((1, L), np.uint8), m, 0.5)
+    idx, cnt = oracle.select_blocks(Q, Kr, L, m, 5, 1, 1, SCALE)
+    O, _ = gpu_fwd(Q, K, V, idx, cnt, m)
+    assert np.all(bf16_to_f64(O) == 0.75)
+
+
+def test_forward_path_end_to_end_at_m16():
+    # (a) -> (b) -> (c) through phsa_forward with the paper's block size; the
+    # selection is compared first, and the output whenever the sets agree.
+    B, Hq, Hkv, L, m, topk, n_init, n_local, lam = 1, 4, 2, 16 * 150 + 3, 16, 20, 2, 8, 0.5
+    rng = np.random.default_rng(77)
+    pset = inputs.punct_id_set(rng)
+    ids = inputs.draw_token_ids(rng, B, L, "uniform8", (9, 25), pset)
+    mask = oracle.punct_mask(ids, pset)
+    Q, K, V = rand(rng, B, Hq, L, D), rand(rng, B, Hkv, L, D), rand(rng, B, Hkv, L, D)
+    O, lse, gi, gc, Krd = phsa.phsa_forward(to_dev_bf16(Q), to_dev_bf16(K), to_dev_bf16(V),
+                                            torch.from_numpy(mask).cuda(), lam, topk, n_init,
+                                            n_local, block_size=m)
+    torch.cuda.synchronize()
+    Kr = oracle.block_repr(K, mask, m, lam)
+    assert ulp_distance(bf16_bits(Krd), Kr).max() <= 1
+    oi, oc, oa = oracle.select_blocks(Q, Kr, L, m, topk, n_init, n_local, SCALE, want_agg=True)
+    bad, _, differ, msgs = compare_selection(gi.cpu().numpy(), gc.cpu().numpy(), oi, oc, oa)
+    assert bad == 0, msgs[:5]
+    assert phsa.phsa_get_device_status() == 0
+    if differ == 0:  # the same sets: the outputs must agree too
+        Or, lser = oracle.sparse_attn_fwd(Q, K, V, oi, oc, m, SCALE)
+        assert_close("O", bf16_to_f64(O), Or)
+        assert np.abs(lse.cpu().numpy() - lser).max() <= LSE_ABS

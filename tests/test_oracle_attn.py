@@ -75,10 +75,9 @@ def torch_ref(Q, K, V, vis, scale, dO=None):
             v.grad.numpy())
 
 
-@pytest.mark.parametrize("L", [256, 300])
-def test_full_budget_equals_dense_causal(L):
+@pytest.mark.parametrize("L,m", [(256, 64), (300, 64), (300, 16), (160, 32)])
+def test_full_budget_equals_dense_causal(L, m):
     rng = np.random.default_rng(10)
-    m = 64
     Q, K, V = rand_qkv(rng, 1, 4, 2, L)
     NQB = -(-L // m)
     idx = np.tile(np.arange(NQB, dtype=np.int32), (1, 2, NQB, 1))
@@ -102,10 +101,10 @@ def test_dense_causal_matches_torch_fp64():
     np.testing.assert_allclose(lse, lset, rtol=0, atol=1e-12)
 
 
-@pytest.mark.parametrize("L,topk", [(64 * 9, 4), (64 * 6 + 23, 3)])
-def test_sparse_matches_torch_masked_fp64(L, topk):
+@pytest.mark.parametrize("L,topk,m", [(64 * 9, 4, 64), (64 * 6 + 23, 3, 64), (16 * 13 + 5, 5, 16),
+                                      (32 * 7 + 9, 3, 32)])
+def test_sparse_matches_torch_masked_fp64(L, topk, m):
     rng = np.random.default_rng(12)
-    m = 64
     Q, K, V = rand_qkv(rng, 2, 4, 2, L)
     idx, cnt = random_selection(rng, 2, 2, L, m, topk)
     O, lse = oracle.sparse_attn_fwd(Q, K, V, idx, cnt, m, D ** -0.5)

@@ -45,6 +45,21 @@ def test_no_punctuation_is_the_mean_of_each_block():
     assert list(r[0, 0, :, 0]) == [31.5, 95.5, 160.0, 224.0]
 
 
+def test_block_size_16_means_and_one_punctuation_token():
+    # Eq. 3 and 6 at m = 16 with K_i = i: block t averages 16t .. 16t+15 -> 16t + 7.5
+    # (all exact in bf16 below 256). Eq. 7-8 with one punctuation token j = 37 in
+    # block 2 and lambda = 0.5: 0.5 * 39.5 + 0.5 * 37 = 38.25 (exact).
+    K = ramp_keys(L=128)
+    r = repr_vals(K, np.zeros((1, 128), np.uint8), 0.5, m=16)
+    assert r.shape == (1, 1, 8, 128)
+    assert list(r[0, 0, :, 0]) == [16 * t + 7.5 for t in range(8)]
+    mask = np.zeros((1, 128), np.uint8)
+    mask[0, 37] = 1
+    r = repr_vals(K, mask, 0.5, m=16)
+    assert r[0, 0, 2, 0] == 38.25
+    assert [r[0, 0, t, 0] for t in (0, 1, 3)] == [7.5, 23.5, 55.5]
+
+
 @pytest.mark.parametrize("lam,j,expect", [
     (0.5, 10, 0.5 * 31.5 + 0.5 * 10),    # 20.75
     (0.25, 40, 38.0),  # 0.25*31.5 + 0.75*40 = 37.875 = 100101.111b: a bf16 tie -> even, 38

@@ -134,6 +134,23 @@ def test_relevance_is_the_summed_softmax_over_candidates_only():
     assert np.isnan(A[0, 0, 4, 0]) and np.isnan(A[0, 0, 4, 4])  # forced: never scored
 
 
+def test_relevance_at_block_size_16():
+    # The closed form above with m = 16: query block 4 has 16 rows; row 0 scores
+    # (100, 0, 0), rows 1..15 score (0, 0.5, 0). A_1 = 1 + 15/(2+e^0.5) = 5.11,
+    # A_2 = 15 e^0.5/(2+e^0.5) = 6.78 -> block 2 (64 rows would give the same pick
+    # with other values; a block size read as 64 would see 64 rows of zeros).
+    L, m, T = 16 * 5, 16, 5
+    Q = np.zeros((1, 1, L, D), np.float32)
+    for r in range(m):
+        Q[0, 0, 4 * m + r, [1, 2, 3]] = (100.0, 0.0, 0.0) if r == 0 else (0.0, 0.5, 0.0)
+        Q[0, 0, 4 * m + r, [0, 4]] = 10.0
+    idx, cnt, A = sel(bf(Q), onehot_repr(T), L, m, topk=3, agg=True)
+    assert list(idx[0, 0, 4]) == [0, 2, 4]
+    e = np.exp(0.5)
+    np.testing.assert_allclose(A[0, 0, 4, 1:4], [1 + 15 / (2 + e), 15 * e / (2 + e), 15 / (2 + e)],
+                               rtol=1e-12, atol=1e-12)
+
+
 @pytest.mark.parametrize("h1_score,expect", [(0.5, 1), (2.0, 2)])
 def test_both_heads_of_a_group_vote(h1_score, expect):
     # Head 0 rows score (1, 0, 0), head 1 rows score (0, s, 0).
