@@ -180,7 +180,8 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- oracle sample
-def oracle_sample_step(w, x, n_units: int, seed: int, aggregation: str = "softmax_sum"):
+def oracle_sample_step(w, x, n_units: int, seed: int, aggregation: str = "softmax_sum",
+                       fwd_only: bool = False):
     """Times the CPU oracle on a bounded sample of one step; returns estimated seconds
     for the whole step, the parts and a description.
 
@@ -231,6 +232,10 @@ def oracle_sample_step(w, x, n_units: int, seed: int, aggregation: str = "softma
     t0 = time.perf_counter()
     oracle.sparse_attn_rows(x["Q"], x["K"], x["V"], idx, cnt, w.block_size, scale, rows)
     t["fwd"] = (time.perf_counter() - t0) * frac
+    if fwd_only:
+        desc = (f"stage (a) in full; stages (b) and (c) fwd on {len(units)} of {U} (query block,"
+                f" KV head) units; each part scaled by total / sampled work")
+        return sum(t.values()), t, desc
     t0 = time.perf_counter()
     oracle.sparse_attn_bwd_dq_rows(x["Q"], x["K"], x["V"], x["dO"], idx, cnt, w.block_size, scale,
                                    rows)
@@ -299,32 +304,39 @@ def run_ours(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     w = workload_of(args, inputs.WORKLOADS)
+    # the backward runs at m = 64; other block sizes time the forward path alone
+    fwd_only = w.block_size != 64
     # weak scaling: every rank runs one batch of the workload on its own sequences
     mine = shard_sequences(world * w.B, world, rank)
-    x = inputs.make_inputs(w, with_grad=True, seed=rank_seed(w.seed, mine[0]))
+    x = inputs.make_inputs(w, with_grad=not fwd_only, seed=rank_seed(w.seed, mine[0]))
 
     def dev_bf16(a):
         return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
 
-    Q, K, V, dO = (dev_bf16(x[k]) for k in ("Q", "K", "V", "dO"))
+    Q, K, V = (dev_bf16(x[k]) for k in ("Q", "K", "V"))
+    dO = None if fwd_only else dev_bf16(x["dO"])
     mask = torch.from_numpy(x["mask"]).to(dev)
     Kr = torch.empty((w.B, w.Hkv, w.T, w.D), dtype=torch.bfloat16, device=dev)
     idx = torch.empty((w.B, w.Hkv, w.NQB, w.topk), dtype=torch.int32, device=dev)
     cnt = torch.empty((w.B, w.Hkv, w.NQB), dtype=torch.int32, device=dev)
     O = torch.empty_like(Q)
     lse = torch.empty((w.B, w.Hq, w.L), dtype=torch.float32, device=dev)
-    dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
-    ws = torch.empty(phsa.phsa_sparse_attn_bwd_workspace(w.B, w.L, w.Hq, w.Hkv, w.topk),
-                     dtype=torch.uint8, device=dev)
+    if not fwd_only:
+        dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
+        ws = torch.empty(phsa.phsa_sparse_attn_bwd_workspace(w.B, w.L, w.Hq, w.Hkv, w.topk),
+                         dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
+    bs = w.block_size
 
     def step():
-        phsa.phsa_build_block_repr(K, mask, w.lam, Krepr=Kr)
+        phsa.phsa_build_block_repr(K, mask, w.lam, Krepr=Kr, block_size=bs)
         phsa.phsa_select_blocks(Q, Kr, w.Hkv, w.topk, w.n_init, w.n_local, w.sm_scale,
-                                block_idx=idx, block_cnt=cnt, aggregation=args.aggregation)
-        phsa.phsa_sparse_attn_fwd(Q, K, V, idx, cnt, w.sm_scale, O=O, lse=lse)
-        phsa.phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, idx, cnt, w.sm_scale, workspace=ws,
-                                  dQ=dQ, dK=dK, dV=dV)
+                                block_idx=idx, block_cnt=cnt, aggregation=args.aggregation,
+                                block_size=bs)
+        phsa.phsa_sparse_attn_fwd(Q, K, V, idx, cnt, w.sm_scale, O=O, lse=lse, block_size=bs)
+        if not fwd_only:
+            phsa.phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, idx, cnt, w.sm_scale, workspace=ws,
+                                      dQ=dQ, dK=dK, dV=dV)
 
     def barrier():
         if world > 1:
@@ -364,8 +376,9 @@ def run_ours(args):
 
     # ---- end to end through the C ABI's host-buffer call: every step copies its
     # inputs from pinned host memory and its results back, inside the timed region
+    # (the host-buffer step includes the backward: m = 64 only)
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not fwd_only:
         pin = lambda a: torch.from_numpy(a).pin_memory()
         hQ, hK, hV, hdO = (pin(x[k].view(np.int16)) for k in ("Q", "K", "V", "dO"))
         hmask = pin(x["mask"])
@@ -462,7 +475,7 @@ def run_ours(args):
     if not args.no_cpu_baseline and world == 1:
         cores = oracle_threads()
         est_s, parts, desc = oracle_sample_step(w, x, args.cpu_units, seed=5,
-                                                aggregation=args.aggregation)
+                                                aggregation=args.aggregation, fwd_only=fwd_only)
         cpu = {"value": w.B * w.L / est_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                "sample": desc, "est_s_per_step": round(est_s, 2),
                "parts_s": {k: round(v, 3) for k, v in parts.items()}}
@@ -476,17 +489,20 @@ def run_ours(args):
                    "block_size": w.block_size, "topk": w.topk, "n_init": w.n_init,
                    "n_local": w.n_local, "lambda": w.lam, "aggregation": args.aggregation,
                    "sparsity": round(1 - w.topk * w.block_size / w.L, 5),
-                   "step": "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)",
+                   "step": ("fwd (repr + select + sparse attn); the backward runs at m = 64 only"
+                            if fwd_only else
+                            "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)"),
                    "l2": "inputs larger than L2 (Q 134 MB, K 67 MB, V 67 MB, dO 134 MB per step)",
                    "parallelism": f"dp{world} (independent sequences)"},
         "fwd": {"ms": round(fwd_ms, 4), "tokens_per_s": tokens / (fwd_ms / 1e3) if fwd_ms else None,
                 "eff_tflops": round(stages["fwd"]["flops"] / (fwd_ms / 1e3) / 1e12, 1) if fwd_ms else None,
                 "roofline_us": round(fwd_roof * 1e6, 1),
                 "roofline_frac": round(fwd_roof / (fwd_ms / 1e3), 4) if fwd_ms else None},
-        "bwd": {"ms": round(bwd_ms, 4),
-                "eff_tflops": round(stages["bwd"]["flops"] / (bwd_ms / 1e3) / 1e12, 1) if bwd_ms else None,
-                "roofline_us": round(bwd_roof * 1e6, 1),
-                "roofline_frac": round(bwd_roof / (bwd_ms / 1e3), 4) if bwd_ms else None},
+        "bwd": None if fwd_only else {
+            "ms": round(bwd_ms, 4),
+            "eff_tflops": round(stages["bwd"]["flops"] / (bwd_ms / 1e3) / 1e12, 1) if bwd_ms else None,
+            "roofline_us": round(bwd_roof * 1e6, 1),
+            "roofline_frac": round(bwd_roof / (bwd_ms / 1e3), 4) if bwd_ms else None},
         "roofline": roof,
         "kernels": kernels,
         "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
@@ -744,16 +760,18 @@ def run_reference(args):
     if rank != 0:
         return None
     w = workload_of(args, inputs.WORKLOADS)
-    x = inputs.make_inputs(w, with_grad=True)
+    fwd_only = w.block_size != 64  # the same step as our arm's
+    x = inputs.make_inputs(w, with_grad=not fwd_only)
     cores = oracle_threads()
     n_units = max(args.ref_units, cores)  # at least one unit per thread
     for s in range(args.warmup):
-        oracle_sample_step(w, x, n_units, seed=100 + s, aggregation=args.aggregation)
+        oracle_sample_step(w, x, n_units, seed=100 + s, aggregation=args.aggregation,
+                           fwd_only=fwd_only)
     ests, descs = [], None
     t0 = time.perf_counter()
     for s in range(args.steps):
         est, _, descs = oracle_sample_step(w, x, n_units, seed=1000 + s,
-                                           aggregation=args.aggregation)
+                                           aggregation=args.aggregation, fwd_only=fwd_only)
         ests.append(est)
     wall = time.perf_counter() - t0
     est = statistics.mean(ests)
@@ -766,7 +784,8 @@ def run_reference(args):
         "config": {"workload": w.name, "B": w.B, "L": w.L, "Hq": w.Hq, "Hkv": w.Hkv, "D": w.D,
                    "block_size": w.block_size, "topk": w.topk, "n_init": w.n_init,
                    "n_local": w.n_local, "lambda": w.lam, "aggregation": args.aggregation,
-                   "step": "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)"},
+                   "step": ("fwd (repr + select + sparse attn)" if fwd_only else
+                            "fwd (repr + select + sparse attn) + bwd (dQ, dK, dV)")},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                          "sample": descs},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,

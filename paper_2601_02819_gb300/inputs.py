@@ -73,6 +73,12 @@ WORKLOADS = {
     "prefill_32k": Workload("prefill_32k", B=1, L=32768, Hq=16, Hkv=8, topk=14,
                             punct="sentence", punct_gap=(9, 25),
                             per_head_scale=True, seed=1234 + 2),
+    # The paper's 32k setting as printed: blocks of 16 tokens, 128 initial and
+    # 512 local tokens (8 and 32 blocks) and 16 Top-K blocks; the same tensors
+    # as prefill_32k (same seed).
+    "prefill_32k_m16": Workload("prefill_32k_m16", B=1, L=32768, Hq=16, Hkv=8, block_size=16,
+                                topk=56, n_init=8, n_local=32, punct="sentence",
+                                punct_gap=(9, 25), per_head_scale=True, seed=1234 + 2),
     "train_8k_x4": Workload("train_8k_x4", B=4, L=8192, Hq=16, Hkv=8, topk=8,
                             punct="sentence", punct_gap=(9, 25), seed=1234 + 3),
     "long_131k_p0": Workload("long_131k_p0", B=1, L=131072, Hq=16, Hkv=8, topk=32,
@@ -205,6 +211,28 @@ def make_decode_inputs(w: Workload, device, seed: int | None = None) -> dict:
     return {"q": q, "K": K, "V": V, "mask": mask, "ids": ids, "punct_ids": pset,
             "mask_dev": torch.from_numpy(mask).to(device), "lens": lens,
             "lens_dev": torch.from_numpy(lens).to(device)}
+
+
+def random_block_lists(rng: np.random.Generator, B: int, Hkv: int, NQB: int,
+                       topk: int) -> tuple[np.ndarray, np.ndarray]:
+    """Random valid block lists for the attention stage alone: per (b, g, qb)
+    the first block, the query's own block and random earlier blocks,
+    min(topk, qb + 1) in all, ascending and -1 padded. Drawn, not selected:
+    feeding the same lists to both sides isolates the attention kernels.
+    Returns (block_idx [B, Hkv, NQB, topk] int32, block_cnt [B, Hkv, NQB] int32)."""
+    idx = np.full((B, Hkv, NQB, topk), -1, np.int32)
+    cnt = np.zeros((B, Hkv, NQB), np.int32)
+    for b in range(B):
+        for g in range(Hkv):
+            for qb in range(NQB):
+                n = min(topk, qb + 1)
+                s = {0, qb}
+                if n > len(s):
+                    s |= set((rng.choice(qb - 1, size=n - len(s), replace=False) + 1).tolist())
+                s = sorted(s)
+                idx[b, g, qb, :len(s)] = s
+                cnt[b, g, qb] = len(s)
+    return idx, cnt
 
 
 def custom(name: str = "custom", **kw) -> Workload:
