@@ -212,8 +212,8 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
                             v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
                             v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
                         } else {
-                            v = exp2f(acc[n][e] - mrow[0]) * inv_z[0] +
-                                exp2f(acc[n][e + 2] - mrow[1]) * inv_z[1];
+                            v = ex2_sfu(acc[n][e] - mrow[0]) * inv_z[0] +
+                                ex2_sfu(acc[n][e + 2] - mrow[1]) * inv_z[1];
                             v += __shfl_xor_sync(0xffffffffu, v, 4);
                             v += __shfl_xor_sync(0xffffffffu, v, 8);
                             v += __shfl_xor_sync(0xffffffffu, v, 16);
@@ -247,8 +247,8 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
                     float s = 0.f;
 #pragma unroll
                     for (int n = 0; n < C::kNt; ++n)
-                        s += exp2f(acc[n][2 * h] - mnew) + exp2f(acc[n][2 * h + 1] - mnew);
-                    zrow[h] = zrow[h] * exp2f(mrow[h] - mnew) + s;
+                        s += ex2_sfu(acc[n][2 * h] - mnew) + ex2_sfu(acc[n][2 * h + 1] - mnew);
+                    zrow[h] = zrow[h] * ex2_sfu(mrow[h] - mnew) + s;
                     mrow[h] = mnew;
                 }
             }
@@ -263,8 +263,8 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
                     const float mo = __shfl_xor_sync(0xffffffffu, mrow[h], off);
                     const float zo = __shfl_xor_sync(0xffffffffu, zrow[h], off);
                     const float mn = fmaxf(mrow[h], mo);
-                    const float za = mrow[h] == -INFINITY ? 0.f : zrow[h] * exp2f(mrow[h] - mn);
-                    const float zb = mo == -INFINITY ? 0.f : zo * exp2f(mo - mn);
+                    const float za = mrow[h] == -INFINITY ? 0.f : zrow[h] * ex2_sfu(mrow[h] - mn);
+                    const float zb = mo == -INFINITY ? 0.f : zo * ex2_sfu(mo - mn);
                     mrow[h] = mn;
                     zrow[h] = za + zb;
                 }
@@ -284,7 +284,7 @@ select_blocks_kernel(const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* _
 #pragma unroll
                 for (int c = 0; c < C::kColWarps; ++c) {
                     const float2 st = stat[c * C::kRows + r];
-                    if (st.x != -INFINITY) z += st.y * exp2f(st.x - mx);
+                    if (st.x != -INFINITY) z += st.y * ex2_sfu(st.x - mx);
                 }
                 mrow[h] = mx;
                 zrow[h] = z;
