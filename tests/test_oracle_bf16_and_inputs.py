@@ -70,3 +70,23 @@ def test_none_placement_has_no_punctuation():
     w = inputs.custom(B=1, L=512, Hq=2, Hkv=1, punct="none")
     x = inputs.make_inputs(w)
     assert x["mask"].sum() == 0
+
+
+def test_drawn_block_lists_are_valid_and_seeded():
+    # The attention-only parity tests feed these lists to both sides: every
+    # list must be ascending, unique, inside [0, qb], hold the first and the
+    # query's own block, have min(topk, qb + 1) entries and -1 padding.
+    from paper_2601_02819_gb300 import inputs
+    idx, cnt = inputs.random_block_lists(np.random.default_rng(3), 2, 3, 70, 9)
+    idx2, cnt2 = inputs.random_block_lists(np.random.default_rng(3), 2, 3, 70, 9)
+    assert np.array_equal(idx, idx2) and np.array_equal(cnt, cnt2)
+    assert idx.shape == (2, 3, 70, 9) and idx.dtype == np.int32 and cnt.dtype == np.int32
+    for b in range(2):
+        for g in range(3):
+            for qb in range(70):
+                n, row = cnt[b, g, qb], idx[b, g, qb]
+                assert n == min(9, qb + 1)
+                assert row[0] == 0 and row[n - 1] == qb
+                assert np.all(np.diff(row[:n]) > 0) and np.all(row[n:] == -1)
+    # not always the same earlier blocks
+    assert len({tuple(idx[0, 0, qb, 1:8]) for qb in range(40, 70)}) > 20
