@@ -382,8 +382,7 @@ cudaError_t launch_select_g(const phsa_shape& s, const phsa_select_params& p, co
 size_t select_smem_bytes(const phsa_shape& s, int topk) {
     const int bm = s.block_size, NQB = (s.L + bm - 1) / bm;
     const int G = s.Hq / s.Hkv;
-    if (G == 2 && bm == kM) return select_tc_smem_bytes(s, topk);
-    if (G == 2) return bm == 16 ? SelCfg<2, 16>::smem_bytes(NQB, topk) : SelCfg<2, 32>::smem_bytes(NQB, topk);
+    if (G == 2) return select_tc_smem_bytes(s, topk);
     return bm == 16   ? SelCfg<1, 16>::smem_bytes(NQB, topk)
            : bm == 32 ? SelCfg<1, 32>::smem_bytes(NQB, topk)
                       : SelCfg<1, 64>::smem_bytes(NQB, topk);
@@ -394,14 +393,11 @@ cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_sh
                                  int* status, cudaStream_t st) {
     const int bm = s.block_size;
     if ((long long)s.B * s.Hkv * ((s.L + bm - 1) / bm) == 0) return cudaSuccess;
-    // Two query heads per KV head at m = 64 fill a 128-row tcgen05 tile
-    // (select_tc.cu); every other group size and block size runs on the
-    // warp-level MMA kernel in this file.
+    // Two query heads per KV head fill a 128-row tcgen05 tile (select_tc.cu;
+    // at m = 16 and 32 the tile holds the query blocks of a 64-token span); a
+    // single head runs on the warp-level MMA kernel in this file.
     const int G = s.Hq / s.Hkv;
-    if (G == 2 && bm == 64) return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
-    if (G == 2)
-        return bm == 16 ? launch_select_g<2, 16>(s, p, Q, Krepr, idx, cnt, st)
-                        : launch_select_g<2, 32>(s, p, Q, Krepr, idx, cnt, st);
+    if (G == 2) return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
     return bm == 16   ? launch_select_g<1, 16>(s, p, Q, Krepr, idx, cnt, st)
            : bm == 32 ? launch_select_g<1, 32>(s, p, Q, Krepr, idx, cnt, st)
                       : launch_select_g<1, 64>(s, p, Q, Krepr, idx, cnt, st);

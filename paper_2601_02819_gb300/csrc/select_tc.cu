@@ -21,8 +21,13 @@
 // The max-logit rule (PHSA_AGG_MAX_LOGIT) needs no softmax statistics: it runs
 // pass 2 alone, each thread taking the largest score of its candidate over its
 // 64 rows (rows past L excluded), A[t] = max(half 0, half 1) * scale.
+// Block sizes 16 and 32 (kSub = 64/m query blocks per unit): the unit is a
+// 64-token span whose kSub query blocks fill the 128-row tile; the span's
+// union of candidate ranges is scored, pass 1 bounds every row by its own
+// query block, pass 2 keeps one sum (or maximum) per query block, and the
+// elementwise warps run each query block's top-k after pass 2.
 // Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs,
-// warp 10 the top-k. The ring, the TMEM buffers and every barrier run on
+// warp 10 the top-k (kSub = 1). The ring, the TMEM buffers and every barrier run on
 // counters that continue across units. Every wait is bounded in time.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
@@ -50,8 +55,12 @@ constexpr int kThreads = 352;
 constexpr uint32_t kTmemCols = 256;
 constexpr int kRegKeys = 16;  // candidate keys per lane kept in registers by the top-k warp
 
-size_t select_tc_smem(int nqb, int topk) {
-    return 1024 + (size_t)kOffA + (size_t)nqb * 16 + (size_t)topk * 4 + 16;
+// kSub query blocks of m = 64 / kSub tokens share a unit (the 64-token span):
+// A holds two buffers of two halves (kSub = 1) or one buffer of kSub x two
+// halves (kSub > 1, where the elementwise warps run the top-k themselves).
+size_t select_tc_smem(int nqb, int topk, int kSub) {
+    const size_t na = kSub == 1 ? 4 : (size_t)2 * kSub;
+    return 1024 + (size_t)kOffA + na * nqb * 4 + (size_t)topk * 4 + 16;
 }
 
 struct SelArgs {
@@ -60,6 +69,7 @@ struct SelArgs {
     int* status;
     int Hq, Hkv, L, T, NQB, topk, n_init, n_local, units, agg;
     float scale_log2, scale;
+    int nsb;  // units per (b, g): query blocks (kSub = 1) or 64-token spans
 };
 
 // Everything about a unit that every role derives the same way.
@@ -103,7 +113,64 @@ __device__ __forceinline__ bool step_resident(int s, int nch, bool pass2_only) {
     return !pass2_only && nch >= 2 && s >= nch && s < nch + 2;
 }
 
-template <bool kMaxLogit>
+// Query block qb's forced sets and candidate range (Algorithm 1), any block size.
+struct QbSel {
+    int n_init_q, loc_lo, c_hi, nC, nF, ksel;
+    bool scored;
+};
+__device__ __forceinline__ QbSel qb_sel(const SelArgs& a, int qb) {
+    QbSel q;
+    q.n_init_q = min(a.n_init, qb + 1);
+    q.loc_lo = max(q.n_init_q, qb - a.n_local + 1);
+    q.c_hi = qb - a.n_local;
+    q.nC = max(0, q.c_hi - a.n_init + 1);
+    q.nF = q.n_init_q + (qb - q.loc_lo + 1);
+    q.ksel = a.topk - q.nF;
+    q.scored = q.ksel < q.nC;
+    return q;
+}
+
+// A unit of kSub > 1 query blocks: the span's union of candidate ranges is
+// scored (that of its last query block); scored if any of them needs scoring.
+template <int kSub>
+__device__ __forceinline__ SelUnit sel_unit_k(const SelArgs& a, int u) {
+    if constexpr (kSub == 1) {
+        return sel_unit(a, u);
+    } else {
+        SelUnit d;
+        d.qb = a.nsb - 1 - (u % a.nsb);  // the span; heaviest first
+        d.bg = u / a.nsb;
+        d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
+        d.lu = (long long)d.bg * a.NQB + (long long)d.qb * kSub;
+        const int last = min(a.NQB - 1, d.qb * kSub + kSub - 1);
+        d.scored = false;
+        for (int qb = d.qb * kSub; qb <= last; ++qb) d.scored |= qb_sel(a, qb).scored;
+        d.c_lo = a.n_init;
+        d.c_hi = last - a.n_local;
+        d.nC = max(0, d.c_hi - d.c_lo + 1);
+        d.n_init_q = d.loc_lo = d.nF = d.ksel = 0;  // per query block: qb_sel
+        d.nch = d.scored ? (d.nC + kCand - 1) / kCand : 0;
+        return d;
+    }
+}
+
+// Writes query block qb's selection when its budget covers every candidate
+// (threads t0, t0 + step, ...).
+__device__ __forceinline__ void write_unscored(const SelArgs& a, int bg, int qb, const QbSel& q,
+                                               int t0, int step) {
+    int32_t* out = a.idx_out + ((long long)bg * a.NQB + qb) * a.topk;
+    const int n = q.nF + q.nC;
+    for (int j = t0; j < a.topk; j += step) {
+        int v = -1;
+        if (j < q.n_init_q) v = j;
+        else if (j < q.n_init_q + q.nC) v = a.n_init + (j - q.n_init_q);
+        else if (j < n) v = q.loc_lo + (j - q.n_init_q - q.nC);
+        out[j] = v;
+    }
+    if (t0 == 0) a.cnt_out[(long long)bg * a.NQB + qb] = n;
+}
+
+template <bool kMaxLogit, int kSub>
 __global__ void __launch_bounds__(kThreads, 2)
 select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKr,
                  const SelArgs a) {
@@ -118,7 +185,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
     float* pm = m2s + 128;  // [2][128] per-half running max (pass 1)
     float* pz = pm + 256;   // [2][128] per-half running sum
     float* Abuf = reinterpret_cast<float*>(smem + kOffA);  // [2][A0 | A1], NQB each
-    int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 16);
+    int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 4 * (kSub == 1 ? 4 : 2 * kSub));
 
     if (tid == 0) {
         mbar_init(bar(B_Q), 1);
@@ -152,7 +219,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             int gs = 0, su = 0, q_last = -1;  // chunk loads issued; scored units begun
             bool ok = true;
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                const SelUnit d = sel_unit(a, u);
+                const SelUnit d = sel_unit_k<kSub>(a, u);
                 if (!d.scored) continue;
                 const int steps = (kMaxLogit ? 1 : 2) * d.nch;
                 for (int s = 0; ok && s < steps; ++s, ++gs) {
@@ -200,7 +267,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             int gs = 0, su = 0;
             bool ok = true;
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                const SelUnit d = sel_unit(a, u);
+                const SelUnit d = sel_unit_k<kSub>(a, u);
                 if (!d.scored) continue;
                 ok = mbar_wait(bar(B_Q), su & 1, abort_flag, a.status);
                 tc_fence_after();
@@ -232,11 +299,11 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             mbar_wait_drain(bar(B_DRAIN), 0);
         }
     } else if (warp == 10) {
-        // ------------------------------------------------ top-k (one warp)
+        // ------------------------------------------------ top-k (one warp; kSub = 1)
         int su = 0;
-        bool ok = true;
+        bool ok = kSub == 1;
         for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-            const SelUnit d = sel_unit(a, u);
+            const SelUnit d = sel_unit_k<kSub>(a, u);
             int32_t* out = a.idx_out + d.lu * a.topk;
             if (!d.scored) {  // the budget covers every candidate
                 const int n = d.nF + d.nC;
@@ -317,15 +384,25 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
         int gs = 0, su = 0;
         // After a failed wait the loops keep running without work, so that all eight
         // warps reach the named barriers after pass 1 the same number of times.
+        const int et = threadIdx.x;  // 0..255 over the elementwise warps
         for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-            const SelUnit d = sel_unit(a, u);
+            const SelUnit d = sel_unit_k<kSub>(a, u);
+            if constexpr (kSub > 1) {
+                if (!d.scored) {  // every query block of the span is covered by its budget
+                    for (int j = 0; j < kSub && d.qb * kSub + j < a.NQB; ++j)
+                        write_unscored(a, d.bg, d.qb * kSub + j, qb_sel(a, d.qb * kSub + j), et, 256);
+                    continue;
+                }
+            }
             if (!d.scored) continue;
             const int nch = d.nch, steps = (kMaxLogit ? 1 : 2) * nch, c_lo = d.c_lo, c_hi = d.c_hi, nC = d.nC;
             const bool row_ok = d.qb * 64 + (r & 63) < a.L;
-            const int buf = su & 1;
+            // pass 1: this row's own candidate bound (its query block's, at kSub > 1)
+            const int c_hi_r = kSub == 1 ? c_hi : min(c_hi, d.qb * kSub + (r & 63) / (64 / kSub) - a.n_local);
+            const int buf = kSub == 1 ? (su & 1) : 0;
             float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
             float* A1 = A0 + a.NQB;
-            if (ok && su >= 2) {  // the top-k warp is done with this buffer's previous unit
+            if (kSub == 1 && ok && su >= 2) {  // the top-k warp is done with this buffer's previous unit
                 ok = mbar_wait(bar(B_AFREE + buf), ((su >> 1) - 1) & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
@@ -340,7 +417,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 if (ok && !kMaxLogit && s < nch) {
                     // pass 1: row r against 64 candidates of the chunk, two loads of 32
                     const int t0 = c_lo + c * kCand + 64 * hh;
-                    const bool full = t0 + 63 <= c_hi;
+                    const bool full = t0 + 63 <= c_hi_r;
 #pragma unroll 1
                     for (int q = 0; q < 2; ++q) {
                         if (t0 + 32 * q > c_hi) break;  // no candidate left in this group (warp-uniform)
@@ -351,7 +428,7 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                         if (!full) {
 #pragma unroll
                             for (int j = 0; j < 32; ++j)
-                                if (t0 + 32 * q + j > c_hi) v[j] = __float_as_uint(-INFINITY);
+                                if (t0 + 32 * q + j > c_hi_r) v[j] = __float_as_uint(-INFINITY);
                         }
 #pragma unroll
                         for (int j = 0; j < 32; ++j) m4[j & 3] = fmaxf(m4[j & 3], __uint_as_float(v[j]));
@@ -369,6 +446,62 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     }
                     tc_fence_before();
                     mbar_arrive(bar(B_SFREE + slot));
+                } else if (ok && kMaxLogit && kSub > 1) {
+                    // max logit, per query block of the span: candidate r against the
+                    // rows of half hh (head hh), kSub groups of 64 / kSub tokens
+                    float mxs[kSub];
+#pragma unroll
+                    for (int sb = 0; sb < kSub; ++sb) mxs[sb] = -INFINITY;
+                    if (c * kCand + (warp & 3) * 32 < nC) {
+#pragma unroll
+                        for (int q = 0; q < 2; ++q) {
+                            uint32_t v[32];
+                            tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+                            const int tok0 = d.qb * 64 + 32 * q;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) {
+                                constexpr int kTok = 64 / kSub;
+                                const float x = tok0 + j < a.L ? __uint_as_float(v[j]) : -INFINITY;
+                                mxs[(32 * q + j) / kTok] = fmaxf(mxs[(32 * q + j) / kTok], x);
+                            }
+                        }
+                    }
+                    tc_fence_before();
+                    mbar_arrive(bar(B_SFREE + slot));
+                    const int cj = c * kCand + r;
+                    if (cj < nC) {
+#pragma unroll
+                        for (int sb = 0; sb < kSub; ++sb)
+                            Abuf[(size_t)(2 * sb + hh) * a.NQB + cj] = mxs[sb] * a.scale;
+                    }
+                } else if (ok && !kMaxLogit && kSub > 1 && s >= nch) {
+                    // pass 2, per query block of the span: the sums over its rows of
+                    // head hh, in row order
+                    const float* mrow = m2s + 64 * hh;
+                    float accs[kSub][2];
+#pragma unroll
+                    for (int sb = 0; sb < kSub; ++sb) accs[sb][0] = accs[sb][1] = 0.f;
+                    if (c * kCand + (warp & 3) * 32 < nC) {
+#pragma unroll
+                        for (int q = 0; q < 2; ++q) {
+                            uint32_t v[32];
+                            tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) {
+                                constexpr int kTok = 64 / kSub;
+                                accs[(32 * q + j) / kTok][j & 1] +=
+                                    ex2_approx(fmaf(__uint_as_float(v[j]), a.scale_log2, -mrow[32 * q + j]));
+                            }
+                        }
+                    }
+                    tc_fence_before();
+                    mbar_arrive(bar(B_SFREE + slot));
+                    const int cj = c * kCand + r;
+                    if (cj < nC) {
+#pragma unroll
+                        for (int sb = 0; sb < kSub; ++sb)
+                            Abuf[(size_t)(2 * sb + hh) * a.NQB + cj] = accs[sb][0] + accs[sb][1];
+                    }
                 } else if (ok && kMaxLogit) {
                     // max logit: candidate r against the 64 rows of half hh (head hh)
                     float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
@@ -432,7 +565,56 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     named_barrier(1, 256);
                 }
             }
-            if (ok) mbar_arrive(bar(B_AFULL + buf));  // this thread's A entries are written
+            if constexpr (kSub == 1) {
+                if (ok) mbar_arrive(bar(B_AFULL + buf));  // this thread's A entries are written
+            } else {
+                // Top-k of each query block of the span, by the eight elementwise
+                // warps: the two-level selection (topk.cuh) when it applies, else
+                // one warp's rounds; every warp passes the same barriers.
+                named_barrier(1, 256);  // every A entry of the span is written
+                unsigned long long* fin = reinterpret_cast<unsigned long long*>(pm);  // 2 KB
+                for (int j = 0; j < kSub; ++j) {
+                    const int qb = d.qb * kSub + j;
+                    if (qb >= a.NQB) break;
+                    const QbSel q = qb_sel(a, qb);
+                    if (!q.scored) {
+                        write_unscored(a, d.bg, qb, q, et, 256);
+                        continue;
+                    }
+                    float* Aj0 = Abuf + (size_t)(2 * j) * a.NQB;
+                    float* Aj1 = Aj0 + a.NQB;
+                    auto key_of = [&](int cj) {
+                        return topk::make_key_agg(kMaxLogit ? fmaxf(Aj0[cj], Aj1[cj]) : Aj0[cj] + Aj1[cj],
+                                                  c_lo + cj, kMaxLogit);
+                    };
+                    if (topk::two_level(q.nC, q.ksel)) {
+                        topk::level1(q.nC, q.ksel, key_of, fin, warp, lane);
+                        named_barrier(1, 256);
+                        topk::level2(fin, q.ksel, sel, et);
+                    } else if (warp == 0) {
+                        // a pick is marked by a NaN bit pattern that arithmetic never produces
+                        topk::rounds_one_warp(
+                            q.nC, q.ksel, key_of,
+                            [&](int cj) { return __float_as_uint(Aj1[cj]) == 0xffffffffu; },
+                            [&](int t) { Aj1[t - c_lo] = __uint_as_float(0xffffffffu); }, sel, lane);
+                    }
+                    named_barrier(1, 256);
+                    int32_t* out = a.idx_out + ((long long)d.bg * a.NQB + qb) * a.topk;
+                    for (int x = et; x < a.topk; x += 256) {
+                        if (x < q.n_init_q) out[x] = x;
+                        else if (x >= q.n_init_q + q.ksel && x < q.nF + q.ksel) out[x] = q.loc_lo + (x - q.n_init_q - q.ksel);
+                        else if (x >= q.nF + q.ksel) out[x] = -1;
+                    }
+                    for (int x = et; x < q.ksel; x += 256) {
+                        const int v = sel[x];
+                        int rank = 0;
+                        for (int i = 0; i < q.ksel; ++i) rank += sel[i] < v;
+                        out[q.n_init_q + rank] = v;
+                    }
+                    if (et == 0) a.cnt_out[(long long)d.bg * a.NQB + qb] = q.nF + q.ksel;
+                    named_barrier(1, 256);  // sel and fin are reused
+                }
+            }
             ++su;
         }
     }
@@ -447,13 +629,15 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 }  // namespace
 
 size_t select_tc_smem_bytes(const phsa_shape& s, int topk) {
-    return select_tc_smem((s.L + 63) / 64, topk);
+    const int bm = s.block_size;
+    return select_tc_smem((s.L + bm - 1) / bm, topk, 64 / bm);
 }
 
 cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape& s,
                              const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,
                              cudaStream_t st) {
-    const int T = s.L / 64, NQB = (s.L + 63) / 64;
+    const int bm = s.block_size, kSub = 64 / bm;
+    const int T = s.L / bm, NQB = (s.L + bm - 1) / bm;
     CUtensorMap tq, tkr;
     if (!make_tmap_bf16_rows128(&tq, Q, s.L, (uint64_t)s.B * s.Hq, 64)) return cudaErrorInvalidValue;
     // Krepr may be absent when no query block has a candidate (T < 2): the map is
@@ -461,18 +645,22 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
     if (!make_tmap_bf16_rows128(&tkr, T > 0 ? Krepr : Q, T > 0 ? T : 1,
                                 (uint64_t)s.B * s.Hkv, 128))
         return cudaErrorInvalidValue;
-    const size_t smem = select_tc_smem(NQB, p.topk);
-    auto kern = p.aggregation == PHSA_AGG_MAX_LOGIT ? select_tc_kernel<true> : select_tc_kernel<false>;
+    const size_t smem = select_tc_smem(NQB, p.topk, kSub);
+    const bool mx = p.aggregation == PHSA_AGG_MAX_LOGIT;
+    auto kern = kSub == 1 ? (mx ? select_tc_kernel<true, 1> : select_tc_kernel<false, 1>)
+                : kSub == 2 ? (mx ? select_tc_kernel<true, 2> : select_tc_kernel<false, 2>)
+                            : (mx ? select_tc_kernel<true, 4> : select_tc_kernel<false, 4>);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
-    const int units = s.B * s.Hkv * NQB;
+    const int nsb = kSub == 1 ? NQB : (NQB + kSub - 1) / kSub;
+    const int units = s.B * s.Hkv * nsb;
     const int per_sm = smem * 2 + 2048 <= 228 * 1024 ? 2 : 1;  // two CTAs when shared memory allows
     SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, units,
-                 p.aggregation, p.sm_scale * kLog2e, p.sm_scale};
+                 p.aggregation, p.sm_scale * kLog2e, p.sm_scale, nsb};
     ProfScope prof(K_SELECT, st);
     kern<<<(unsigned)min(units, per_sm * nsm), kThreads, smem, st>>>(tq, tkr, args);
     return cudaGetLastError();
