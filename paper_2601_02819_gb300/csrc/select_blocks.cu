@@ -382,7 +382,13 @@ cudaError_t launch_select_g(const phsa_shape& s, const phsa_select_params& p, co
 size_t select_smem_bytes(const phsa_shape& s, int topk) {
     const int bm = s.block_size, NQB = (s.L + bm - 1) / bm;
     const int G = s.Hq / s.Hkv;
-    if (G == 2) return select_tc_smem_bytes(s, topk);
+    if (G == 2) {
+        // the tcgen05 kernel, unless its per-block sums outgrow shared memory at
+        // m < 64 (spans beyond about 64k tokens at m = 16): then the warp-MMA one
+        const size_t tc = select_tc_smem_bytes(s, topk);
+        if (bm == 64 || tc <= 227 * 1024) return tc;
+        return bm == 16 ? SelCfg<2, 16>::smem_bytes(NQB, topk) : SelCfg<2, 32>::smem_bytes(NQB, topk);
+    }
     return bm == 16   ? SelCfg<1, 16>::smem_bytes(NQB, topk)
            : bm == 32 ? SelCfg<1, 32>::smem_bytes(NQB, topk)
                       : SelCfg<1, 64>::smem_bytes(NQB, topk);
@@ -394,10 +400,16 @@ cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_sh
     const int bm = s.block_size;
     if ((long long)s.B * s.Hkv * ((s.L + bm - 1) / bm) == 0) return cudaSuccess;
     // Two query heads per KV head fill a 128-row tcgen05 tile (select_tc.cu;
-    // at m = 16 and 32 the tile holds the query blocks of a 64-token span); a
-    // single head runs on the warp-level MMA kernel in this file.
+    // at m = 16 and 32 the tile holds the query blocks of a 64-token span, as
+    // long as their per-block sums fit in shared memory); a single head, and
+    // longer sequences at m < 64, run on the warp-level MMA kernel in this file.
     const int G = s.Hq / s.Hkv;
-    if (G == 2) return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
+    if (G == 2) {
+        if (bm == 64 || select_tc_smem_bytes(s, p.topk) <= 227 * 1024)
+            return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
+        return bm == 16 ? launch_select_g<2, 16>(s, p, Q, Krepr, idx, cnt, st)
+                        : launch_select_g<2, 32>(s, p, Q, Krepr, idx, cnt, st);
+    }
     return bm == 16   ? launch_select_g<1, 16>(s, p, Q, Krepr, idx, cnt, st)
            : bm == 32 ? launch_select_g<1, 32>(s, p, Q, Krepr, idx, cnt, st)
                       : launch_select_g<1, 64>(s, p, Q, Krepr, idx, cnt, st);

@@ -162,3 +162,22 @@ def test_forward_path_end_to_end_at_m16():
         Or, lser = oracle.sparse_attn_fwd(Q, K, V, oi, oc, m, SCALE)
         assert_close("O", bf16_to_f64(O), Or)
         assert np.abs(lse.cpu().numpy() - lser).max() <= LSE_ABS
+
+
+def test_selection_long_sequence_at_m16_uses_the_warp_mma_kernel():
+    # 4200 query blocks of 16: the tcgen05 kernel's per-block sums no longer fit
+    # in shared memory, so the pair runs on the warp-MMA kernel; sampled units
+    # against the oracle's selection.
+    m, L, topk, n_init, n_local = 16, 16 * 4200 + 3, 20, 1, 2
+    rng = np.random.default_rng(4200)
+    Q, K = rand(rng, 1, 2, L, D), rand(rng, 1, 1, L, D)
+    mask = (rng.random((1, L)) < 0.06).astype(np.uint8)
+    Kr = oracle.block_repr(K, mask, m, 0.5)
+    gi, gc = gpu_select(Q, Kr, 1, topk, n_init, n_local, m)
+    NQB = -(-L // m)
+    units = np.unique(np.concatenate([[0, NQB - 1, NQB // 2], rng.integers(0, NQB, 24)]))
+    oi, oc, oa = oracle.select_units(Q, Kr, L, m, topk, n_init, n_local, SCALE, units)
+    bad, _, differ, msgs = compare_selection(gi.reshape(-1, topk)[units], gc.reshape(-1)[units],
+                                             oi, oc, oa)
+    assert bad == 0, msgs[:5]
+    assert differ <= 1
