@@ -360,6 +360,19 @@ int phsa_profile_read(int max_kinds, const char** names, double* total_ms, int* 
 int phsa_selftest_tcgen05(const void* A, const void* B, const void* V, float* S, float* O,
                           void* stream);
 
+/*
+ * Testing hook (no counterpart in the paper). With two query heads per KV
+ * head, phsa_select_blocks runs the tensor-core selection at every block size
+ * until, at block sizes 16 and 32, its per-query-block sums need more shared
+ * memory than a switch point (227 KB by default: beyond about 64k tokens at
+ * m = 16); longer sequences run on a warp-level MMA kernel. This call sets the
+ * switch point to `bytes` (0, or more than 227 KB, restores the default) so
+ * that a test can reach the warp-level pair kernels on short inputs; both
+ * kernels compute the same selection. Returns the previous value. Affects
+ * every later call in the process; not meant for production use.
+ */
+size_t phsa_test_set_select_tc_limit(size_t bytes);
+
 /* Library version as "major.minor.patch". */
 const char* phsa_version(void);
 

@@ -611,7 +611,7 @@ __device__ __forceinline__ uint32_t col_dp(int b) { return 64u + 128u * (uint32_
 __device__ __forceinline__ uint32_t col_dv(int c) { return 256u + 128u * (uint32_t)c; }
 __device__ __forceinline__ uint32_t col_dk(int c) { return 320u + 128u * (uint32_t)c; }
 constexpr size_t kSmem = 1024 + (size_t)kOffRing + kRing * 32;
-static_assert(kSmem <= 227 * 1024, "dK/dV shared memory");
+static_assert(kSmem <= kMaxDynSmem, "dK/dV shared memory");
 }  // namespace kv
 
 struct KvArgs {
@@ -1091,7 +1091,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 
 }  // namespace
 
-bool dq_tc_fits(int topk) { return dq::smem_bytes(topk) <= 227u * 1024u; }
+bool dq_tc_fits(int topk) { return dq::smem_bytes(topk) <= kMaxDynSmem; }
 
 cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* O,
                          const void* dO, const float* lse, float* delta, const int32_t* idx,

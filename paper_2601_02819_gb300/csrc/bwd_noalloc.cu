@@ -59,25 +59,24 @@ extern "C" int phsa_sparse_attn_bwd_noalloc(const void* Q, const void* K, const 
                                             const int32_t* block_idx, const int32_t* block_cnt,
                                             phsa_shape s, int topk, float sm_scale, void* dQ,
                                             void* dK, void* dV, void* stream) {
-    const size_t need = phsa_sparse_attn_bwd_workspace(s, topk);
-    if (s.B == 0 || s.L == 0) {
-        return (s.B < 0 || s.L < 0) ? PHSA_ERR_INVALID_ARG : PHSA_OK;
-    }
-    if (need == 0) return PHSA_ERR_UNSUPPORTED;  // shape or topk rejected by validation
-    if (need > kScratchBytes) return PHSA_ERR_WORKSPACE;
+    // The same checks, in the same order and with the same codes, as
+    // phsa_sparse_attn_bwd; only the workspace check differs (the fixed array).
+    int rc = phsa::validate_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = phsa::validate_topk(s, topk)) != PHSA_OK) return rc;
     if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;
-    if (s.Hq <= 0 || s.Hkv <= 0 || s.Hq % s.Hkv != 0) return PHSA_ERR_INVALID_ARG;
+    if (s.B == 0 || s.L == 0) return PHSA_OK;
     if (!Q || !K || !V || !O || !dO || !lse || !block_idx || !block_cnt || !dQ || !dK || !dV)
         return PHSA_ERR_INVALID_ARG;
     const void* ptrs[] = {Q, K, V, O, dO, dQ, dK, dV};
     for (const void* p : ptrs)
         if (!aligned16(p)) return PHSA_ERR_INVALID_ARG;
+    if (phsa::bwd_layout(s, topk).total > kScratchBytes) return PHSA_ERR_WORKSPACE;
     void* ws = nullptr;
     if (scratch_for_current_device(&ws) != cudaSuccess) return PHSA_ERR_CUDA;
     int* st = phsa::device_status_word();
     if (!st) return PHSA_ERR_CUDA;
-    return phsa::launch_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, s, topk, sm_scale, ws,
-                                 dQ, dK, dV, st, static_cast<cudaStream_t>(stream)) == cudaSuccess
-               ? PHSA_OK
-               : PHSA_ERR_CUDA;
+    return phsa::status_of(phsa::launch_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, s,
+                                                 topk, sm_scale, ws, dQ, dK, dV, st,
+                                                 static_cast<cudaStream_t>(stream)));
 }

@@ -105,7 +105,7 @@ size_t fixed_smem(int G, int Tc, int topk) {
            2 * (size_t)sbuf_floats(G, Tc) * 4 + 2 * (size_t)topk * 4 + 16;
 }
 int ring_slots(int G, int Tc, int topk) {
-    const size_t fixed = fixed_smem(G, Tc, topk) + 1024, cap = 227 * 1024;
+    const size_t fixed = fixed_smem(G, Tc, topk) + 1024, cap = kMaxDynSmem;
     size_t fit = fixed >= cap ? 0 : (cap - fixed) / kTile;
     if (fit > (size_t)kSlotsMax) fit = kSlotsMax;
     return fit >= 2 ? (int)fit : 0;

@@ -134,7 +134,7 @@ int phsa_step_host(const void* Q, const void* K, const void* V, const void* dO,
     if (p.aggregation != PHSA_AGG_SOFTMAX_SUM && p.aggregation != PHSA_AGG_MAX_LOGIT)
         return PHSA_ERR_INVALID_ARG;
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
-    if (phsa::select_smem_bytes(s, p.topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
+    if (phsa::select_smem_bytes(s, p.topk) > phsa::kMaxDynSmem) return PHSA_ERR_UNSUPPORTED;
     cudaStream_t cs = static_cast<cudaStream_t>(stream);
     cudaEvent_t done_ev = static_cast<cudaEvent_t>(done_event);
     if (s.B == 0 || s.L == 0) {

@@ -65,6 +65,7 @@ namespace phsa {
 int* device_status_word() { return status_ptr(); }
 int validate_shape(const phsa_shape& s) { return check_shape(s); }
 int validate_topk(const phsa_shape& s, int topk) { return check_topk(s, topk); }
+int status_of(cudaError_t e) { return from_cuda(e); }
 }  // namespace phsa
 
 extern "C" {
@@ -94,7 +95,7 @@ int phsa_select_blocks(const void* Q, const void* Krepr, phsa_shape s, phsa_sele
     const bool need_repr = s.L >= 2 * s.block_size;  // some query block has a candidate
     if (!Q || !block_idx || !block_cnt || !aligned16(Q) || (need_repr && (!Krepr || !aligned16(Krepr))))
         return PHSA_ERR_INVALID_ARG;
-    if (phsa::select_smem_bytes(s, p.topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
+    if (phsa::select_smem_bytes(s, p.topk) > phsa::kMaxDynSmem) return PHSA_ERR_UNSUPPORTED;
     return from_cuda(phsa::launch_select_blocks(Q, Krepr, s, p, block_idx, block_cnt, status_ptr(),
                                                 static_cast<cudaStream_t>(stream)));
 }
@@ -176,7 +177,7 @@ int phsa_decode_select(const void* q, const void* Krepr, const int32_t* seq_lens
     if (!q || !seq_lens || !block_idx || !block_cnt || !aligned16(q) ||
         (need_repr && (!Krepr || !aligned16(Krepr))))
         return PHSA_ERR_INVALID_ARG;
-    if (phsa::decode_select_smem_bytes(s, p.topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
+    if (phsa::decode_select_smem_bytes(s, p.topk) > phsa::kMaxDynSmem) return PHSA_ERR_UNSUPPORTED;
     int* st = status_ptr();
     if (!st) return PHSA_ERR_CUDA;
     return from_cuda(phsa::launch_decode_select(q, Krepr, seq_lens, s, p, block_idx, block_cnt, st,
@@ -195,7 +196,7 @@ int phsa_decode_attn(const void* q, const void* K, const void* V, const int32_t*
         return PHSA_ERR_INVALID_ARG;
     if (!aligned16(q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
         return PHSA_ERR_INVALID_ARG;
-    if (phsa::decode_attn_smem_bytes(s, topk) > 227 * 1024) return PHSA_ERR_UNSUPPORTED;
+    if (phsa::decode_attn_smem_bytes(s, topk) > phsa::kMaxDynSmem) return PHSA_ERR_UNSUPPORTED;
     int* st = status_ptr();
     if (!st) return PHSA_ERR_CUDA;
     return from_cuda(phsa::launch_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, s, topk,
@@ -222,8 +223,8 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
     if (!aligned16(q) || !aligned16(K) || !aligned16(V) || !aligned16(O) ||
         (Krepr && !aligned16(Krepr)))
         return PHSA_ERR_INVALID_ARG;
-    if (phsa::decode_select_smem_bytes(s, p.topk) > 227 * 1024 ||
-        phsa::decode_attn_smem_bytes(s, p.topk) > 227 * 1024)
+    if (phsa::decode_select_smem_bytes(s, p.topk) > phsa::kMaxDynSmem ||
+        phsa::decode_attn_smem_bytes(s, p.topk) > phsa::kMaxDynSmem)
         return PHSA_ERR_UNSUPPORTED;
     int* st = status_ptr();
     if (!st) return PHSA_ERR_CUDA;

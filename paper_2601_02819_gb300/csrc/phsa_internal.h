@@ -11,6 +11,10 @@
 
 namespace phsa {
 
+// Dynamic shared memory a CTA may use on sm_103a (227 KB); every kernel choice
+// and every UNSUPPORTED check against it uses this one constant.
+constexpr size_t kMaxDynSmem = 227u * 1024u;
+
 // Kernel identities for the optional per-kernel timing (profile.cu).
 enum KernelId {
     K_REPR = 0, K_SELECT, K_FWD, K_BWD_DELTA, K_BWD_MARK, K_BWD_BUILD, K_BWD_DKDV,
@@ -132,10 +136,16 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
 
 // The status word of the current device (phsa_api.cu); null if it cannot be found.
 int* device_status_word();
+// PHSA_OK for cudaSuccess, PHSA_ERR_CUDA otherwise (the mapping of every entry point).
+int status_of(cudaError_t e);
 // Shape and budget checks of the C ABI (phsa_api.cu): PHSA_OK or an error code.
 int validate_shape(const phsa_shape& s);
 int validate_topk(const phsa_shape& s, int topk);
 // Shared-memory bytes of the selection kernel for this shape and budget.
 size_t select_smem_bytes(const phsa_shape& s, int topk);
+// Whether a GQA-pair selection runs on the tcgen05 kernel (select_tc.cu): always
+// at m = 64; at m = 16 and 32 while its per-query-block sums fit under the
+// switch point (kMaxDynSmem, lowered only by phsa_test_set_select_tc_limit).
+bool select_uses_tc(const phsa_shape& s, int topk);
 
 }  // namespace phsa

@@ -20,6 +20,8 @@
 // The max-logit rule (agg = 1) makes one pass: A[t] is the column maximum of
 // S = q . Krepr^T * scale over the group's rows (rows past L excluded).
 // Forced blocks are never scored; the output is ascending and -1 padded.
+#include <atomic>
+
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "topk.cuh"
@@ -379,14 +381,24 @@ cudaError_t launch_select_g(const phsa_shape& s, const phsa_select_params& p, co
 
 }  // namespace
 
+// Switch point of the GQA-pair selection at m = 16 and 32: the tcgen05 kernel
+// while its shared memory stays at or below this many bytes, else the
+// warp-MMA kernel. Only phsa_test_set_select_tc_limit lowers it, so that tests
+// reach the warp-MMA pair kernels on short sequences.
+std::atomic<size_t> g_select_tc_limit{kMaxDynSmem};
+
+bool select_uses_tc(const phsa_shape& s, int topk) {
+    if (s.Hq != 2 * s.Hkv) return false;
+    return s.block_size == 64 || select_tc_smem_bytes(s, topk) <= g_select_tc_limit.load();
+}
+
 size_t select_smem_bytes(const phsa_shape& s, int topk) {
     const int bm = s.block_size, NQB = (s.L + bm - 1) / bm;
     const int G = s.Hq / s.Hkv;
     if (G == 2) {
         // the tcgen05 kernel, unless its per-block sums outgrow shared memory at
         // m < 64 (spans beyond about 64k tokens at m = 16): then the warp-MMA one
-        const size_t tc = select_tc_smem_bytes(s, topk);
-        if (bm == 64 || tc <= 227 * 1024) return tc;
+        if (select_uses_tc(s, topk)) return select_tc_smem_bytes(s, topk);
         return bm == 16 ? SelCfg<2, 16>::smem_bytes(NQB, topk) : SelCfg<2, 32>::smem_bytes(NQB, topk);
     }
     return bm == 16   ? SelCfg<1, 16>::smem_bytes(NQB, topk)
@@ -405,7 +417,7 @@ cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_sh
     // longer sequences at m < 64, run on the warp-level MMA kernel in this file.
     const int G = s.Hq / s.Hkv;
     if (G == 2) {
-        if (bm == 64 || select_tc_smem_bytes(s, p.topk) <= 227 * 1024)
+        if (select_uses_tc(s, p.topk))
             return launch_select_tc(Q, Krepr, s, p, idx, cnt, status, st);
         return bm == 16 ? launch_select_g<2, 16>(s, p, Q, Krepr, idx, cnt, st)
                         : launch_select_g<2, 32>(s, p, Q, Krepr, idx, cnt, st);
@@ -416,3 +428,8 @@ cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_sh
 }
 
 }  // namespace phsa
+
+extern "C" size_t phsa_test_set_select_tc_limit(size_t bytes) {
+    const size_t v = bytes == 0 || bytes > phsa::kMaxDynSmem ? phsa::kMaxDynSmem : bytes;
+    return phsa::g_select_tc_limit.exchange(v);
+}

@@ -476,8 +476,12 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                     }
                 } else if (ok && !kMaxLogit && kSub > 1 && s >= nch) {
                     // pass 2, per query block of the span: the sums over its rows of
-                    // head hh, in row order
+                    // head hh, in row order. Query block sb of the span has candidates
+                    // up to qb*kSub + sb - n_local; this thread's candidate t past that
+                    // bound takes no part in sb's sum (its 2^x is not evaluated).
                     const float* mrow = m2s + 64 * hh;
+                    const int t_c = c_lo + c * kCand + r;
+                    const int sb_bound = d.qb * kSub - a.n_local;  // + sb: query block sb's c_hi
                     float accs[kSub][2];
 #pragma unroll
                     for (int sb = 0; sb < kSub; ++sb) accs[sb][0] = accs[sb][1] = 0.f;
@@ -489,8 +493,10 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 #pragma unroll
                             for (int j = 0; j < 32; ++j) {
                                 constexpr int kTok = 64 / kSub;
-                                accs[(32 * q + j) / kTok][j & 1] +=
-                                    ex2_approx(fmaf(__uint_as_float(v[j]), a.scale_log2, -mrow[32 * q + j]));
+                                const int sb = (32 * q + j) / kTok;
+                                if (t_c <= sb_bound + sb)
+                                    accs[sb][j & 1] += ex2_approx(
+                                        fmaf(__uint_as_float(v[j]), a.scale_log2, -mrow[32 * q + j]));
                             }
                         }
                     }
@@ -658,7 +664,7 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
         return e;
     const int nsb = kSub == 1 ? NQB : (NQB + kSub - 1) / kSub;
     const int units = s.B * s.Hkv * nsb;
-    const int per_sm = smem * 2 + 2048 <= 228 * 1024 ? 2 : 1;  // two CTAs when shared memory allows
+    const int per_sm = smem * 2 + 2048 <= kMaxDynSmem + 1024 ? 2 : 1;  // two CTAs when shared memory allows
     SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, units,
                  p.aggregation, p.sm_scale * kLog2e, p.sm_scale, nsb};
     ProfScope prof(K_SELECT, st);

@@ -104,6 +104,8 @@ def _declare(L):
     L.phsa_punct_mask.argtypes = [P, ctypes.c_int64, P, I, P, P]
     L.phsa_decode_select.argtypes = [P, P, P, phsa_shape, phsa_select_params, P, P, P]
     L.phsa_decode_attn.argtypes = [P, P, P, P, P, P, phsa_shape, I, F, P, P, P]
+    L.phsa_test_set_select_tc_limit.argtypes = [SZ]
+    L.phsa_test_set_select_tc_limit.restype = SZ
     for fn in ("phsa_decode_update_repr", "phsa_decode_select", "phsa_decode_attn",
                "phsa_decode_append", "phsa_punct_mask",
                "phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
@@ -500,6 +502,13 @@ def phsa_decode_step(q, K, V, punct_mask, seq_lens, lam: float, Krepr, topk: int
                                  _stream(stream))
     _raise("phsa_decode_step", rc)
     return block_idx, block_cnt, O, lse
+
+
+def phsa_test_set_select_tc_limit(nbytes: int) -> int:
+    """Testing hook: the shared-memory switch point between the tensor-core and
+    the warp-level selection of GQA pairs at block sizes 16 and 32 (0 restores
+    the default of 227 KB). Returns the previous value."""
+    return int(load().phsa_test_set_select_tc_limit(int(nbytes)))
 
 
 def phsa_get_device_status(stream=None) -> int:

@@ -164,20 +164,85 @@ def test_forward_path_end_to_end_at_m16():
         assert np.abs(lse.cpu().numpy() - lser).max() <= LSE_ABS
 
 
-def test_selection_long_sequence_at_m16_uses_the_warp_mma_kernel():
-    # 4200 query blocks of 16: the tcgen05 kernel's per-block sums no longer fit
-    # in shared memory, so the pair runs on the warp-MMA kernel; sampled units
-    # against the oracle's selection.
-    m, L, topk, n_init, n_local = 16, 16 * 4200 + 3, 20, 1, 2
-    rng = np.random.default_rng(4200)
+def _sampled_selection(m, L, topk, n_init, n_local, aggregation, seed, extra_units=()):
+    """GPU selection of a GQA pair vs the oracle's on sampled units (the first,
+    middle and last query blocks, `extra_units` and 24 random ones)."""
+    rng = np.random.default_rng(seed)
     Q, K = rand(rng, 1, 2, L, D), rand(rng, 1, 1, L, D)
     mask = (rng.random((1, L)) < 0.06).astype(np.uint8)
     Kr = oracle.block_repr(K, mask, m, 0.5)
-    gi, gc = gpu_select(Q, Kr, 1, topk, n_init, n_local, m)
+    gi, gc = gpu_select(Q, Kr, 1, topk, n_init, n_local, m, aggregation)
     NQB = -(-L // m)
-    units = np.unique(np.concatenate([[0, NQB - 1, NQB // 2], rng.integers(0, NQB, 24)]))
-    oi, oc, oa = oracle.select_units(Q, Kr, L, m, topk, n_init, n_local, SCALE, units)
+    units = np.unique(np.concatenate([[0, NQB - 1, NQB // 2], list(extra_units),
+                                      rng.integers(0, NQB, 24)])).astype(np.int64)
+    oi, oc, oa = oracle.select_units(Q, Kr, L, m, topk, n_init, n_local, SCALE, units,
+                                     aggregation=aggregation)
     bad, _, differ, msgs = compare_selection(gi.reshape(-1, topk)[units], gc.reshape(-1)[units],
                                              oi, oc, oa)
     assert bad == 0, msgs[:5]
     assert differ <= 1
+    assert phsa.phsa_get_device_status() == 0
+
+
+@pytest.mark.parametrize("aggregation", ["softmax_sum", "max_logit"])
+def test_selection_long_sequence_at_m16_uses_the_warp_mma_kernel(aggregation):
+    # 4200 query blocks of 16: the tcgen05 kernel's per-block sums no longer fit
+    # in shared memory, so the pair runs on the warp-MMA kernel; sampled units
+    # against the oracle's selection.
+    _sampled_selection(16, 16 * 4200 + 3, 20, 1, 2, aggregation, 4200)
+
+
+@pytest.mark.parametrize("m,L,topk,n_init,n_local", [
+    (16, 16 * 300 + 9, 40, 1, 2),   # 37 picks per query block: beyond the two-level top-k
+    (32, 32 * 200 + 5, 36, 1, 1),   # 34 picks at m = 32
+])
+@pytest.mark.parametrize("aggregation", ["softmax_sum", "max_logit"])
+def test_selection_tcgen05_large_budget_uses_one_warp_rounds(m, L, topk, n_init, n_local,
+                                                             aggregation):
+    # At m < 64 the tcgen05 kernel runs each query block's top-k on its scoring
+    # warps; budgets above 32 picks take the one-warp rounds instead of the
+    # two-level selection. Full comparison with the oracle.
+    rng = np.random.default_rng(L + topk)
+    Q, K = rand(rng, 1, 2, L, D), rand(rng, 1, 1, L, D)
+    mask = (rng.random((1, L)) < 0.06).astype(np.uint8)
+    Kr = oracle.block_repr(K, mask, m, 0.5)
+    gi, gc = gpu_select(Q, Kr, 1, topk, n_init, n_local, m, aggregation)
+    oi, oc, oa = oracle.select_blocks(Q, Kr, L, m, topk, n_init, n_local, SCALE, want_agg=True,
+                                      aggregation=aggregation)
+    bad, _, differ, msgs = compare_selection(gi, gc, oi, oc, oa)
+    assert bad == 0, msgs[:5]
+    assert differ <= max(2, 0.01 * oc.size), (differ, oc.size)
+    assert phsa.phsa_get_device_status() == 0
+
+
+@pytest.mark.parametrize("aggregation", ["softmax_sum", "max_logit"])
+def test_selection_tcgen05_more_than_2048_candidates_at_m16(aggregation):
+    # 2300 query blocks of 16: the last ones have more than 2048 candidates,
+    # past the two-level top-k, so the tcgen05 kernel takes the one-warp rounds.
+    NQB = 2300
+    _sampled_selection(16, 16 * NQB, 14, 1, 2, aggregation, 2300,
+                       extra_units=[NQB - 2, NQB - 3, 2100, 2060])
+
+
+@pytest.mark.parametrize("m", [16, 32])
+@pytest.mark.parametrize("aggregation", ["softmax_sum", "max_logit"])
+def test_selection_warp_mma_pair_kernels_on_short_inputs(m, aggregation):
+    # The warp-MMA kernels for GQA pairs (select_blocks_kernel<2, m>) normally
+    # run only beyond ~64k tokens at m = 16 and ~250k at m = 32; a lowered
+    # switch point sends a short input to them.
+    prev = phsa.phsa_test_set_select_tc_limit(1)
+    try:
+        L, topk = m * 150 + 7, 12
+        rng = np.random.default_rng(m * 7 + len(aggregation))
+        Q, K = rand(rng, 1, 4, L, D), rand(rng, 1, 2, L, D)
+        mask = (rng.random((1, L)) < 0.06).astype(np.uint8)
+        Kr = oracle.block_repr(K, mask, m, 0.5)
+        gi, gc = gpu_select(Q, Kr, 2, topk, 1, 2, m, aggregation)
+        oi, oc, oa = oracle.select_blocks(Q, Kr, L, m, topk, 1, 2, SCALE, want_agg=True,
+                                          aggregation=aggregation)
+        bad, _, differ, msgs = compare_selection(gi, gc, oi, oc, oa)
+        assert bad == 0, msgs[:5]
+        assert differ <= max(2, 0.01 * oc.size), (differ, oc.size)
+        assert phsa.phsa_get_device_status() == 0
+    finally:
+        phsa.phsa_test_set_select_tc_limit(prev)
