@@ -67,6 +67,13 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
                              const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,
                              cudaStream_t st);
 size_t select_tc_smem_bytes(const phsa_shape& s, int topk);
+// The one-unit-per-step tcgen05 selection (select_tc_unit.cu), block size 64,
+// which launch_select_tc runs for sequences of up to kSelectUnitMaxNqb query blocks.
+constexpr int kSelectUnitMaxNqb = 1024;
+cudaError_t launch_select_tc_unit(const void* Q, const void* Krepr, const phsa_shape& s,
+                                  const phsa_select_params& p, int32_t* idx, int32_t* cnt,
+                                  int* status, cudaStream_t st);
+size_t select_tc_unit_smem_bytes(const phsa_shape& s, int topk);
 
 cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_shape& s,
                                  const phsa_select_params& p, int32_t* idx, int32_t* cnt,

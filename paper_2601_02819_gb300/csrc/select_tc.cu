@@ -1,34 +1,39 @@
 // Stage (b) on the tensor cores for GQA pairs (G*64 = 128 query rows):
 // query-to-block relevance and Top-K selection (Eq. 8; Algorithm 1 step 3).
-// Persistent: a CTA (352 threads, 2 per SM) walks the units (query block qb,
-// KV head g) u = blockIdx.x, blockIdx.x + gridDim.x, ...
 //
-// The candidate representative keys C = [n_init, qb - n_local] stream through
-// a two-slot shared-memory ring in chunks of 128 rows (TMA). Each chunk is
-// used twice, and the scores never leave the SM:
+// This kernel runs at block sizes 16 and 32, and at 64 beyond 1024 query
+// blocks (shorter sequences take the one-unit kernel of select_tc_unit.cu).
+//
+// Work unit: a batch of two 64-token spans of one (batch, KV head) -- each span
+// is kSub = 64/m query blocks and fills one 128-row tile (two heads x 64
+// tokens). Both spans score the same candidate representative keys (a span's
+// candidates are a prefix of Krepr), so one TMA load of a chunk of 128
+// candidates serves both. Persistent: one CTA per SM walks the batches,
+// heaviest first over all (batch, KV head) pairs.
+//
+// Each chunk is used twice, and the scores never leave the SM:
 //   pass 1  S = Q Kr^T   (M = 128 query rows, N = 128 candidates) in TMEM;
-//           two threads per row (TMEM lane r, one per half of the columns)
-//           keep a running max and sum of 2^(S*scale - max) (online
-//           softmax); the halves are merged once, after the last chunk;
-//   pass 2  S^T = Kr Q^T (M = 128 candidates, N = 128 rows) in TMEM;
-//           two threads per candidate j (lane j, one per half of the rows)
-//           sum p = 2^(S*scale - m_r - log2 Z_r) over their 64 rows in row order;
-//           A[t] = half 0 + half 1. Every candidate follows the same order,
-//           so equal candidates get bit-identical sums.
-//   top-k   a dedicated warp, on a double-buffered copy of A, while the
-//           elementwise warps already score the next unit: larger A first,
-//           lower t on exact ties (topk.cuh).
-// The max-logit rule (PHSA_AGG_MAX_LOGIT) needs no softmax statistics: it runs
-// pass 2 alone, each thread taking the largest score of its candidate over its
-// 64 rows (rows past L excluded), A[t] = max(half 0, half 1) * scale.
-// Block sizes 16 and 32 (kSub = 64/m query blocks per unit): the unit is a
-// 64-token span whose kSub query blocks fill the 128-row tile; the span's
-// union of candidate ranges is scored, pass 1 bounds every row by its own
-// query block, pass 2 keeps one sum (or maximum) per query block, and the
-// elementwise warps run each query block's top-k after pass 2.
-// Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs,
-// warp 10 the top-k (kSub = 1). The ring, the TMEM buffers and every barrier run on
-// counters that continue across units. Every wait is bounded in time.
+//           the thread owning a row keeps sum 2^(S*scale - m) over the
+//           candidates its query block may select, against a shift m that is
+//           the row's first maximum and moves only when a later score would
+//           overflow the sum; after the last chunk M_r = m + log2(sum).
+//   pass 2  S^T = Kr Q^T (M = 128 candidates, N = 128 rows) in TMEM, the
+//           chunks in reverse order (the last ones are still in the ring);
+//           the thread owning candidate t sums p = 2^(S*scale - M_r) over the
+//           rows of each query block of its span, in row order, so equal
+//           candidates get bit-identical sums: A[qb][t].
+//   top-k   per query block, by one warp of the span's warpgroup: larger A
+//           first, lower t on exact ties; output ascending with the forced
+//           initial and local blocks, -1 padded.
+// The max-logit rule (PHSA_AGG_MAX_LOGIT) needs no softmax statistics: pass 2
+// alone, A = max over the query block's rows (rows past L excluded) * scale.
+//
+// Roles: warps 0-3 own span 0 of a batch, warps 4-7 span 1 (one TMEM lane per
+// thread, two 128-column TMEM buffers per span), warp 8 issues TMA (the two Q
+// tiles and the chunk ring), warp 9 the MMAs. The chunk ring keeps the last
+// chunks of pass 1 for pass 2 (least recently used slot refilled first). The
+// ring, the TMEM buffers and every barrier run on counters that continue
+// across batches. Every wait is bounded in time.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "tc_common.cuh"
@@ -40,78 +45,66 @@ namespace {
 
 using namespace tc;
 
-constexpr int kCand = 128;                 // candidates per chunk
-constexpr int kHalf = 128 * 64 * 2;        // 128 rows x 64 columns bf16 (16 KB)
-constexpr int kTile = 2 * kHalf;           // 128 x 128 (32 KB)
-constexpr int kOffQ = 0;
-constexpr int kOffKr = kOffQ + kTile;      // 2 slots
-constexpr int kOffStats = kOffKr + 2 * kTile;  // m + log2 Z [128], half partials m[2][128], z[2][128]
-constexpr int kOffBar = kOffStats + 5 * 128 * 4;
-constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = 4, B_SFULL = 6, B_SFREE = 8,
-              B_AFULL = 10, B_AFREE = 12, B_DRAIN = 14, kNumBars = 15;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
-constexpr int kOffA = kOffMisc + 16;  // 2 buffers x (A0[NQB], A1[NQB]), then sel[topk]
-constexpr int kThreads = 352;
-constexpr uint32_t kTmemCols = 256;
-constexpr int kRegKeys = 16;  // candidate keys per lane kept in registers by the top-k warp
+constexpr int kCand = 128;              // candidates per chunk
+constexpr int kHalf = 128 * 64 * 2;     // [128 rows][64 columns] bf16 (16 KB)
+constexpr int kTile = 2 * kHalf;        // 128 x 128 bf16 (32 KB)
+constexpr int kBox = kHalf / 2;         // a 64-row TMA box of one column half (8 KB)
+constexpr int kMaxSlots = 3;            // chunk ring slots (2 when shared memory is short)
+constexpr int kThreads = 320;           // 8 elementwise warps, TMA, MMA
+constexpr uint32_t kTmemCols = 512;     // 4 buffers of 128 columns: span s uses 2s, 2s + 1
 
-// kSub query blocks of m = 64 / kSub tokens share a unit (the 64-token span):
-// A holds two buffers of two halves (kSub = 1) or one buffer of kSub x two
-// halves (kSub > 1, where the elementwise warps run the top-k themselves).
-size_t select_tc_smem(int nqb, int topk, int kSub) {
-    const size_t na = kSub == 1 ? 4 : (size_t)2 * kSub;
-    return 1024 + (size_t)kOffA + na * nqb * 4 + (size_t)topk * 4 + 16;
+// Q tile slots: span si of a batch uses slot si * nq + (its load count % nq), nq = 2
+// when shared memory allows (the next batch's tiles load during this one), else 1.
+constexpr int B_QFULL = 0, B_QFREE = 4, B_KFULL = 8, B_KEMPTY = B_KFULL + kMaxSlots,
+              B_SFULL = B_KEMPTY + kMaxSlots, B_SFREE = B_SFULL + 4, B_DRAIN = B_SFREE + 4,
+              kNumBars = B_DRAIN + 1;
+
+// Shared-memory layout (offsets from the 1024-aligned base).
+struct SelLayout {
+    int nq;              // Q tile slots per span (1 or 2)
+    int slots;           // chunk ring slots
+    int a_stride;        // floats per query block's aggregate array (>= NQB, multiple of 4)
+    size_t kr, stats, fin, A, bar, misc, total;
+};
+
+__host__ __device__ inline SelLayout sel_layout(int nqb, int kSub, int nq, int slots) {
+    SelLayout L;
+    L.nq = nq;
+    L.slots = slots;
+    L.a_stride = (nqb + 3) & ~3;
+    L.kr = 2 * (size_t)nq * kTile;                  // Q tiles of the two spans first
+    L.stats = L.kr + (size_t)slots * kTile;         // -M_r of the 128 rows, per span
+    L.fin = L.stats + 2 * 128 * 4;                  // top-k finalists [span][4 warps][32] u64
+    L.A = L.fin + 2 * 4 * 32 * 8;                   // A[span][query block of span][candidate]
+    L.bar = L.A + (size_t)2 * kSub * L.a_stride * 4;
+    L.misc = L.bar + kNumBars * 8;                  // tmem base, abort flag
+    L.total = 1024 + L.misc + 16;
+    return L;
+}
+
+// The largest layout that fits: two Q slots per span first, then ring depth.
+__host__ __device__ inline SelLayout sel_layout_fit(int nqb, int kSub) {
+    const int cfg[4][2] = {{2, 3}, {2, 2}, {1, 3}, {1, 2}};
+    for (int i = 0; i < 3; ++i) {
+        const SelLayout l = sel_layout(nqb, kSub, cfg[i][0], cfg[i][1]);
+        if (l.total <= kMaxDynSmem) return l;
+    }
+    return sel_layout(nqb, kSub, 1, 2);
 }
 
 struct SelArgs {
     int32_t* idx_out;
     int32_t* cnt_out;
     int* status;
-    int Hq, Hkv, L, T, NQB, topk, n_init, n_local, units, agg;
+    int Hq, Hkv, L, T, NQB, topk, n_init, n_local, agg;
+    int nsb;      // 64-token spans per (b, g)
+    int nbat;     // batches per (b, g): ceil(nsb / 2)
+    int BG;       // B * Hkv
+    int batches;  // BG * nbat
     float scale_log2, scale;
-    int nsb;  // units per (b, g): query blocks (kSub = 1) or 64-token spans
+    int nq, slots, a_stride;
+    uint32_t off_kr, off_stats, off_fin, off_A, off_bar, off_misc;
 };
-
-// Everything about a unit that every role derives the same way.
-struct SelUnit {
-    int qb, bg, hq0, n_init_q, loc_lo, c_lo, c_hi, nC, nF, ksel, nch;
-    long long lu;
-    bool scored;  // false: the budget covers every candidate, nothing to score
-};
-
-__device__ __forceinline__ SelUnit sel_unit(const SelArgs& a, int u) {
-    SelUnit d;
-    d.qb = a.NQB - 1 - (u % a.NQB);  // heaviest query blocks first
-    d.bg = u / a.NQB;
-    d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
-    d.lu = (long long)d.bg * a.NQB + d.qb;
-    d.n_init_q = min(a.n_init, d.qb + 1);                // forced initial [0, n_init_q)
-    d.loc_lo = max(d.n_init_q, d.qb - a.n_local + 1);    // forced local [loc_lo, qb]
-    d.c_lo = a.n_init;                                   // candidates [c_lo, c_hi]
-    d.c_hi = d.qb - a.n_local;
-    d.nC = max(0, d.c_hi - d.c_lo + 1);
-    d.nF = d.n_init_q + (d.qb - d.loc_lo + 1);
-    d.ksel = a.topk - d.nF;
-    d.scored = d.ksel < d.nC;
-    d.nch = d.scored ? (d.nC + kCand - 1) / kCand : 0;  // chunks per pass
-    return d;
-}
-
-// The chunk that step s of a unit with nch chunks per pass works on. Pass 2
-// takes the last two chunks of pass 1 first: they are still in the ring's two
-// slots (same slot parity, the ring alternates), so they are not loaded again;
-// then chunks 0 .. nch - 3. Each chunk holds its own candidates, so the order
-// of the chunks changes no sum.
-__device__ __forceinline__ int step_chunk(int s, int nch, bool pass2_only) {
-    if (pass2_only || s < nch) return s;
-    const int j = s - nch;
-    if (nch < 2) return 0;
-    return j < 2 ? nch - 2 + j : j - 2;
-}
-// Step s reuses the chunk already in its slot (pass 2's first two steps).
-__device__ __forceinline__ bool step_resident(int s, int nch, bool pass2_only) {
-    return !pass2_only && nch >= 2 && s >= nch && s < nch + 2;
-}
 
 // Query block qb's forced sets and candidate range (Algorithm 1), any block size.
 struct QbSel {
@@ -130,29 +123,84 @@ __device__ __forceinline__ QbSel qb_sel(const SelArgs& a, int qb) {
     return q;
 }
 
-// A unit of kSub > 1 query blocks: the span's union of candidate ranges is
-// scored (that of its last query block); scored if any of them needs scoring.
+// One span of a batch: its query blocks [s*kSub, s*kSub + nqb), the union of
+// their candidate ranges [n_init, c_hi] and the chunks of it that are scored.
+struct SpanInfo {
+    int s, nqb, c_hi, nC, nch;
+    bool present, scored;
+};
+struct BatchInfo {
+    int bg, hq0, n;  // n: chunks of the batch (max over its spans)
+    SpanInfo sp[2];
+};
+
 template <int kSub>
-__device__ __forceinline__ SelUnit sel_unit_k(const SelArgs& a, int u) {
-    if constexpr (kSub == 1) {
-        return sel_unit(a, u);
-    } else {
-        SelUnit d;
-        d.qb = a.nsb - 1 - (u % a.nsb);  // the span; heaviest first
-        d.bg = u / a.nsb;
-        d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
-        d.lu = (long long)d.bg * a.NQB + (long long)d.qb * kSub;
-        const int last = min(a.NQB - 1, d.qb * kSub + kSub - 1);
-        d.scored = false;
-        for (int qb = d.qb * kSub; qb <= last; ++qb) d.scored |= qb_sel(a, qb).scored;
-        d.c_lo = a.n_init;
-        d.c_hi = last - a.n_local;
-        d.nC = max(0, d.c_hi - d.c_lo + 1);
-        d.n_init_q = d.loc_lo = d.nF = d.ksel = 0;  // per query block: qb_sel
-        d.nch = d.scored ? (d.nC + kCand - 1) / kCand : 0;
-        return d;
+__device__ __forceinline__ BatchInfo batch_info(const SelArgs& a, int v) {
+    BatchInfo B;
+    const int k = v / a.BG;
+    B.bg = v - k * a.BG;
+    B.hq0 = (B.bg / a.Hkv) * a.Hq + (B.bg % a.Hkv) * 2;
+    B.n = 0;
+#pragma unroll
+    for (int si = 0; si < 2; ++si) {
+        SpanInfo& p = B.sp[si];
+        p.s = a.nsb - 1 - 2 * k - si;  // the heavier (later) span first
+        p.present = p.s >= 0;
+        p.scored = false;
+        p.nqb = 0;
+        p.c_hi = -1;
+        p.nC = 0;
+        p.nch = 0;
+        if (!p.present) continue;
+        p.nqb = min(kSub, a.NQB - p.s * kSub);
+        const int last = p.s * kSub + p.nqb - 1;
+        for (int qb = p.s * kSub; qb <= last; ++qb) p.scored |= qb_sel(a, qb).scored;
+        p.c_hi = last - a.n_local;
+        p.nC = max(0, p.c_hi - a.n_init + 1);
+        p.nch = p.scored ? (p.nC + kCand - 1) / kCand : 0;
+        B.n = max(B.n, p.nch);
     }
+    return B;
 }
+
+// The chunk ring as both the TMA and the MMA thread see it: the same sequence
+// of chunk uses gives both the same slots. A use finds its chunk still in a
+// slot (resident: no load) or refills the least recently used slot. Pass 2
+// runs the chunks in reverse order, so its first uses find the last chunks of
+// pass 1 (min(n, slots) of them) resident; every other use is a fill.
+struct ChunkRing {
+    int tag[kMaxSlots];
+    uint32_t stamp[kMaxSlots];
+    int fills[kMaxSlots];
+    uint32_t clock;
+    int n;
+    __device__ __forceinline__ void init(int slots) {
+        n = slots;
+        clock = 0;
+#pragma unroll
+        for (int i = 0; i < kMaxSlots; ++i) {
+            tag[i] = -1;
+            stamp[i] = 0;
+            fills[i] = 0;
+        }
+    }
+    __device__ __forceinline__ int take(int t, bool& load) {
+        int s = -1;
+#pragma unroll
+        for (int i = 0; i < kMaxSlots; ++i)
+            if (i < n && tag[i] == t) s = i;
+        load = s < 0;
+        if (load) {
+            s = 0;
+#pragma unroll
+            for (int i = 1; i < kMaxSlots; ++i)
+                if (i < n && stamp[i] < stamp[s]) s = i;
+            tag[s] = t;
+        }
+        stamp[s] = ++clock;
+        return s;
+    }
+};
 
 // Writes query block qb's selection when its budget covers every candidate
 // (threads t0, t0 + step, ...).
@@ -170,458 +218,428 @@ __device__ __forceinline__ void write_unscored(const SelArgs& a, int bg, int qb,
     if (t0 == 0) a.cnt_out[(long long)bg * a.NQB + qb] = n;
 }
 
+// Top-k of one scored query block by one warp over its aggregates Aq[cj]
+// (candidate t = n_init + cj), and its output row.
+template <bool kMaxLogit>
+__device__ __forceinline__ void topk_write(const SelArgs& a, int bg, int qb, const QbSel& q,
+                                           float* Aq, int lane) {
+    int32_t* out = a.idx_out + ((long long)bg * a.NQB + qb) * a.topk;
+    const int c_lo = a.n_init;
+    auto key_of = [&](int cj) { return topk::make_key_agg(Aq[cj], c_lo + cj, kMaxLogit); };
+    if (q.ksel <= 32) {
+        const unsigned long long mine = topk::warp_topk32(q.nC, q.ksel, key_of, lane);
+        const int blk = lane < q.ksel ? topk::key_block(mine) : 0x7fffffff;
+        int rank = 0;
+        for (int i = 0; i < q.ksel; ++i) rank += __shfl_sync(0xffffffffu, blk, i) < blk;
+        if (lane < q.ksel) out[q.n_init_q + rank] = blk;
+    } else {
+        // a pick is marked by a NaN bit pattern that arithmetic never produces;
+        // the marks are then read back in ascending order
+        auto taken = [&](int cj) { return __float_as_uint(Aq[cj]) == 0xffffffffu; };
+        topk::rounds_mark_one_warp(q.nC, q.ksel, key_of, taken,
+                                   [&](int t) { Aq[t - c_lo] = __uint_as_float(0xffffffffu); }, lane);
+        __syncwarp();
+        int pos = q.n_init_q;
+        for (int base = 0; base < q.nC; base += 32) {
+            const int cj = base + lane;
+            const bool pick = cj < q.nC && taken(cj);
+            const unsigned m = __ballot_sync(0xffffffffu, pick);
+            if (pick) out[pos + __popc(m & ((1u << lane) - 1u))] = c_lo + cj;
+            pos += __popc(m);
+        }
+    }
+    for (int x = lane; x < a.topk; x += 32) {
+        if (x < q.n_init_q) out[x] = x;
+        else if (x >= q.n_init_q + q.ksel && x < q.nF + q.ksel)
+            out[x] = q.loc_lo + (x - q.n_init_q - q.ksel);
+        else if (x >= q.nF + q.ksel) out[x] = -1;
+    }
+    if (lane == 0) a.cnt_out[(long long)bg * a.NQB + qb] = q.nF + q.ksel;
+}
+
+// Writes the output row of a scored query block whose picks are held one per
+// lane (lane < ksel, in any order): ascending, with the forced initial and local
+// blocks, -1 padded, and its count.
+__device__ __forceinline__ void write_picks(const SelArgs& a, int bg, int qb, const QbSel& q,
+                                            unsigned long long mine, int lane) {
+    int32_t* out = a.idx_out + ((long long)bg * a.NQB + qb) * a.topk;
+    const int blk = lane < q.ksel ? topk::key_block(mine) : 0x7fffffff;
+    int rank = 0;
+    for (int i = 0; i < q.ksel; ++i) rank += __shfl_sync(0xffffffffu, blk, i) < blk;
+    if (lane < q.ksel) out[q.n_init_q + rank] = blk;
+    for (int x = lane; x < a.topk; x += 32) {
+        if (x < q.n_init_q) out[x] = x;
+        else if (x >= q.n_init_q + q.ksel && x < q.nF + q.ksel)
+            out[x] = q.loc_lo + (x - q.n_init_q - q.ksel);
+        else if (x >= q.nF + q.ksel) out[x] = -1;
+    }
+    if (lane == 0) a.cnt_out[(long long)bg * a.NQB + qb] = q.nF + q.ksel;
+}
+
+// Top-k of one scored query block (ksel <= 32) by kW warps: warp wi takes a
+// kW-th of the candidates and keeps its best min(ksel, slice) in fin[wi]
+// (level 1); after the barrier, warp 0 takes the best ksel of the finalists
+// (level 2): every pick is within the best ksel of its own slice.
+template <bool kMaxLogit, int kW>
+__device__ __forceinline__ void topk_split(const SelArgs& a, int bg, int qb, const QbSel& q,
+                                           const float* Aq, unsigned long long* fin, int wi,
+                                           int lane, int bar_id, bool ok) {
+    const int per = (q.nC + kW - 1) / kW;
+    const int lo = min(q.nC, wi * per), hi = min(q.nC, lo + per);
+    const int k1 = min(q.ksel, hi - lo);
+    unsigned long long mine = 0ull;
+    if (k1 > 0)
+        mine = topk::warp_topk32(hi - lo, k1, [&](int cj) {
+            return topk::make_key_agg(Aq[lo + cj], a.n_init + lo + cj, kMaxLogit);
+        }, lane);
+    fin[wi * 32 + lane] = lane < k1 ? mine : 0ull;
+    named_barrier(bar_id, 32 * kW);
+    if (wi == 0) {
+        const unsigned long long best =
+            topk::warp_topk32(32 * kW, q.ksel, [&](int f) { return fin[f]; }, lane);
+        if (ok) write_picks(a, bg, qb, q, best, lane);
+    }
+}
+
+__device__ __forceinline__ float max32(const uint32_t* v) {
+    float m[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) m[i] = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 32; j += 4) {
+        const int i = (j >> 2) & 7;
+        m[i] = fmaxf(m[i], fmaxf(fmaxf(__uint_as_float(v[j]), __uint_as_float(v[j + 1])),
+                                 fmaxf(__uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]))));
+    }
+    return fmaxf(fmaxf(fmaxf(m[0], m[1]), fmaxf(m[2], m[3])), fmaxf(fmaxf(m[4], m[5]), fmaxf(m[6], m[7])));
+}
+
+// sum over 32 scores of 2^(x * c + o), packed two at a time, fixed order
+__device__ __forceinline__ float expsum32(const uint32_t* v, float c, float o) {
+    const float2 cc = make_float2(c, c), oo = make_float2(o, o);
+    float2 acc[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[i] = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < 32; j += 2) {
+        float2 e = __ffma2_rn(make_float2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), cc, oo);
+        e.x = ex2_approx(e.x);
+        e.y = ex2_approx(e.y);
+        acc[(j >> 1) & 3] = __fadd2_rn(acc[(j >> 1) & 3], e);
+    }
+    const float2 s01 = __fadd2_rn(acc[0], acc[1]), s23 = __fadd2_rn(acc[2], acc[3]);
+    const float2 s = __fadd2_rn(s01, s23);
+    return s.x + s.y;
+}
+
 template <bool kMaxLogit, int kSub>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
 select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKr,
                  const SelArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     const uint32_t sb = smem_u32(smem);
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
-    float* m2s = reinterpret_cast<float*>(smem + kOffStats);  // per row: max + log2 of the sum
-    float* pm = m2s + 128;  // [2][128] per-half running max (pass 1)
-    float* pz = pm + 256;   // [2][128] per-half running sum
-    float* Abuf = reinterpret_cast<float*>(smem + kOffA);  // [2][A0 | A1], NQB each
-    int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 4 * (kSub == 1 ? 4 : 2 * kSub));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    auto bar = [&](int i) { return sb + a.off_bar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + a.off_misc + 4);
+    constexpr int kTok = 64 / kSub;  // tokens per query block
 
-    if (tid == 0) {
-        mbar_init(bar(B_Q), 1);
-        mbar_init(bar(B_QFREE), 1);
-        for (int s = 0; s < 2; ++s) {
+    if (threadIdx.x == 0) {
+        for (int q = 0; q < 4; ++q) {
+            mbar_init(bar(B_QFULL + q), 1);
+            mbar_init(bar(B_QFREE + q), 1);
+        }
+        for (int s = 0; s < kMaxSlots; ++s) {
             mbar_init(bar(B_KFULL + s), 1);
             mbar_init(bar(B_KEMPTY + s), 1);
-            mbar_init(bar(B_SFULL + s), 1);
-            mbar_init(bar(B_SFREE + s), 256);
-            mbar_init(bar(B_AFULL + s), 256);
-            mbar_init(bar(B_AFREE + s), 1);
+        }
+        for (int b = 0; b < 4; ++b) {
+            mbar_init(bar(B_SFULL + b), 1);
+            mbar_init(bar(B_SFREE + b), 128);
         }
         mbar_init(bar(B_DRAIN), 1);
         fence_barrier_init();
         *abort_flag = 0;
     }
     if (warp == 9) {
-        tmem_alloc(sb + kOffMisc, kTmemCols);
+        tmem_alloc(sb + a.off_misc, kTmemCols);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + a.off_misc);
 
     if (warp == 8) {
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
             prefetch_tmap(&tmKr);
             prefetch_tmap(&tmQ);
-            int gs = 0, su = 0, q_last = -1;  // chunk loads issued; scored units begun
+            ChunkRing ring;
+            ring.init(a.slots);
+            int qloads[2] = {0, 0};
             bool ok = true;
-            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                const SelUnit d = sel_unit_k<kSub>(a, u);
-                if (!d.scored) continue;
-                const int steps = (kMaxLogit ? 1 : 2) * d.nch;
-                for (int s = 0; ok && s < steps; ++s, ++gs) {
-                    const int slot = gs & 1, c = step_chunk(s, d.nch, kMaxLogit);
-                    if (gs >= 2 && !mbar_wait(bar(B_KEMPTY + slot), ((gs >> 1) - 1) & 1, abort_flag, a.status)) {
+            int ib = 0;
+            for (int v = blockIdx.x; ok && v < a.batches; v += gridDim.x, ++ib) {
+                const BatchInfo B = batch_info<kSub>(a, v);
+                for (int si = 0; ok && si < 2; ++si) {
+                    if (!B.sp[si].scored) continue;
+                    const int qs = si * a.nq + qloads[si] % a.nq, use = qloads[si] / a.nq;
+                    if (use > 0 &&
+                        !mbar_wait(bar(B_QFREE + qs), (use - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
-                    if (step_resident(s, d.nch, kMaxLogit)) {
-                        // the slot holds this chunk: its last reader is done (KEMPTY
-                        // above), so the full phase completes without a copy
-                        mbar_arrive(bar(B_KFULL + slot));
-                        continue;
-                    }
-                    mbar_expect_tx(bar(B_KFULL + slot), kTile);
-                    for (int dh = 0; dh < 2; ++dh)
-                        tma_load_3d(sb + kOffKr + slot * kTile + dh * kHalf, &tmKr, bar(B_KFULL + slot),
-                                    dh * 64, d.c_lo + c * kCand, d.bg);
-                    if (s == 0) {  // Q once the previous unit's last MMA has read the old one
-                        if (su > 0 && !mbar_wait(bar(B_QFREE), (su - 1) & 1, abort_flag, a.status)) {
-                            ok = false;
-                            ++gs;
-                            break;
-                        }
-                        mbar_expect_tx(bar(B_Q), kTile);
-                        for (int hl = 0; hl < 2; ++hl)
-                            for (int dh = 0; dh < 2; ++dh)
-                                tma_load_3d(sb + kOffQ + dh * kHalf + hl * (kHalf / 2), &tmQ, bar(B_Q),
-                                            dh * 64, d.qb * 64, d.hq0 + hl);
-                        q_last = su;
-                    }
+                    mbar_expect_tx(bar(B_QFULL + qs), kTile);
+                    for (int hl = 0; hl < 2; ++hl)
+                        for (int dh = 0; dh < 2; ++dh)
+                            tma_load_3d(sb + qs * kTile + dh * kHalf + hl * kBox, &tmQ,
+                                        bar(B_QFULL + qs), dh * 64, B.sp[si].s * 64, B.hq0 + hl);
+                    ++qloads[si];
                 }
-                ++su;
+                auto use = [&](int c) {
+                    bool load;
+                    const int sl = ring.take(((ib & 0x7fff) << 16) | c, load);
+                    if (load) {
+                        // the slot's previous fill is done with (its last use has completed)
+                        if (ring.fills[sl] > 0 &&
+                            !mbar_wait(bar(B_KEMPTY + sl), (ring.fills[sl] - 1) & 1, abort_flag, a.status))
+                            return false;
+                        mbar_expect_tx(bar(B_KFULL + sl), kTile);
+                        const uint32_t dst = sb + a.off_kr + sl * kTile;
+                        for (int dh = 0; dh < 2; ++dh)
+                            for (int rh = 0; rh < 2; ++rh)
+                                tma_load_3d(dst + dh * kHalf + rh * kBox, &tmKr, bar(B_KFULL + sl),
+                                            dh * 64, a.n_init + c * kCand + rh * 64, B.bg);
+                        ++ring.fills[sl];
+                    }
+                    return true;
+                };
+                if (!kMaxLogit)
+                    for (int c = 0; ok && c < B.n; ++c) ok = use(c);
+                for (int c = B.n - 1; ok && c >= 0; --c) ok = use(c);
             }
-            if (q_last >= 0) mbar_wait_drain(bar(B_Q), q_last & 1);
-            for (int s = gs - 2; s < gs; ++s)
-                if (s >= 0) mbar_wait_drain(bar(B_KFULL + (s & 1)), (s >> 1) & 1);
+            for (int sl = 0; sl < a.slots; ++sl)
+                if (ring.fills[sl] > 0) mbar_wait_drain(bar(B_KFULL + sl), (ring.fills[sl] - 1) & 1);
+            for (int si = 0; si < 2; ++si)
+                for (int j = 0; j < a.nq && j < qloads[si]; ++j) {
+                    const int last = qloads[si] - 1 - j;  // the last load into each slot
+                    mbar_wait_drain(bar(B_QFULL + si * a.nq + last % a.nq), (last / a.nq) & 1);
+                }
         }
     } else if (warp == 9) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(128, 128, false);
-            const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
-            const uint64_t dKr0 = sdesc_sw128(sb + kOffKr, 16, 1024);
-            int gs = 0, su = 0;
+            const uint64_t dQ0 = sdesc_sw128(sb, 16, 1024);
+            const uint64_t dKr0 = sdesc_sw128(sb + a.off_kr, 16, 1024);
+            ChunkRing ring;
+            ring.init(a.slots);
+            int qfulls[2] = {0, 0}, k[2] = {0, 0};
             bool ok = true;
-            for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-                const SelUnit d = sel_unit_k<kSub>(a, u);
-                if (!d.scored) continue;
-                ok = mbar_wait(bar(B_Q), su & 1, abort_flag, a.status);
-                tc_fence_after();
-                const int steps = (kMaxLogit ? 1 : 2) * d.nch;
-                for (int s = 0; ok && s < steps; ++s, ++gs) {
-                    const int slot = gs & 1;
-                    ok = mbar_wait(bar(B_KFULL + slot), (gs >> 1) & 1, abort_flag, a.status) &&
-                         (gs < 2 || mbar_wait(bar(B_SFREE + slot), ((gs >> 1) - 1) & 1, abort_flag, a.status));
-                    if (!ok) break;
-                    tc_fence_after();
-                    const uint64_t kr = sdesc_at(dKr0, slot * kTile);
-                    const bool pass1 = !kMaxLogit && s < d.nch;
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
-                        const uint64_t dq = sdesc_at(dQ0, off);
-                        const uint64_t dk = sdesc_at(kr, off);
-                        // pass 1: rows x candidates; pass 2: candidates x rows
-                        mma_ss(tmem + 128u * slot, pass1 ? dq : dk, pass1 ? dk : dq, idesc,
-                               ks > 0 ? 1u : 0u);
+            int ib = 0;
+            for (int v = blockIdx.x; ok && v < a.batches; v += gridDim.x, ++ib) {
+                const BatchInfo B = batch_info<kSub>(a, v);
+                bool need_q[2] = {B.sp[0].scored, B.sp[1].scored};
+                auto step = [&](int c, bool pass1) {
+                    bool load;
+                    const int sl = ring.take(((ib & 0x7fff) << 16) | c, load);
+                    if (load) {
+                        if (!mbar_wait(bar(B_KFULL + sl), ring.fills[sl] & 1, abort_flag, a.status))
+                            return false;
+                        ++ring.fills[sl];
                     }
-                    mma_commit(bar(B_SFULL + slot));
-                    mma_commit(bar(B_KEMPTY + slot));
-                }
-                if (ok) mma_commit(bar(B_QFREE));  // this unit's MMAs are all issued
-                ++su;
+                    tc_fence_after();
+                    const uint64_t kr = sdesc_at(dKr0, sl * kTile);
+                    for (int si = 0; si < 2; ++si) {
+                        if (c >= B.sp[si].nch) continue;
+                        const int qs = si * a.nq + qfulls[si] % a.nq;
+                        if (need_q[si]) {
+                            if (!mbar_wait(bar(B_QFULL + qs), (qfulls[si] / a.nq) & 1, abort_flag,
+                                           a.status))
+                                return false;
+                            need_q[si] = false;
+                        }
+                        const int b = 2 * si + (k[si] & 1);
+                        if (k[si] >= 2 &&
+                            !mbar_wait(bar(B_SFREE + b), ((k[si] >> 1) - 1) & 1, abort_flag, a.status))
+                            return false;
+                        tc_fence_after();
+                        const uint64_t q = sdesc_at(dQ0, qs * kTile);
+#pragma unroll
+                        for (int ks = 0; ks < 8; ++ks) {
+                            const uint32_t off = (uint32_t)((ks >> 2) * kHalf + (ks & 3) * 32);
+                            // pass 1: rows x candidates; pass 2: candidates x rows
+                            mma_ss(tmem + 128u * b, sdesc_at(pass1 ? q : kr, off),
+                                   sdesc_at(pass1 ? kr : q, off), idesc, ks > 0 ? 1u : 0u);
+                        }
+                        mma_commit(bar(B_SFULL + b));
+                        ++k[si];
+                        if (!pass1 && c == 0) {  // the span's last MMA of the batch
+                            mma_commit(bar(B_QFREE + qs));
+                            ++qfulls[si];
+                        }
+                    }
+                    // One empty phase per fill, committed after the fill's last use: a
+                    // pass-2 use, or a pass-1 use of a chunk that does not stay in the
+                    // ring for pass 2 (the last `slots` chunks of pass 1 do). The
+                    // producer waits for exactly that phase before refilling the slot,
+                    // so the barrier never runs two phases ahead of it.
+                    if (!pass1 || c < B.n - a.slots) mma_commit(bar(B_KEMPTY + sl));
+                    return true;
+                };
+                if (!kMaxLogit)
+                    for (int c = 0; ok && c < B.n; ++c) ok = step(c, true);
+                for (int c = B.n - 1; ok && c >= 0; --c) ok = step(c, false);
             }
             mma_commit(bar(B_DRAIN));
             mbar_wait_drain(bar(B_DRAIN), 0);
         }
-    } else if (warp == 10) {
-        // ------------------------------------------------ top-k (one warp; kSub = 1)
-        int su = 0;
-        bool ok = kSub == 1;
-        for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-            const SelUnit d = sel_unit_k<kSub>(a, u);
-            int32_t* out = a.idx_out + d.lu * a.topk;
-            if (!d.scored) {  // the budget covers every candidate
-                const int n = d.nF + d.nC;
-                for (int j = lane; j < a.topk; j += 32) {
-                    int v = -1;
-                    if (j < d.n_init_q) v = j;
-                    else if (j < d.n_init_q + d.nC) v = d.c_lo + (j - d.n_init_q);
-                    else if (j < n) v = d.loc_lo + (j - d.n_init_q - d.nC);
-                    out[j] = v;
-                }
-                if (lane == 0) a.cnt_out[d.lu] = n;
-                continue;
-            }
-            const int buf = su & 1;
-            ok = mbar_wait(bar(B_AFULL + buf), (su >> 1) & 1, abort_flag, a.status);
-            ok = __all_sync(0xffffffffu, ok);
-            if (!ok) break;
-            float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
-            float* A1 = A0 + a.NQB;
-            // key = bits(A) << 32 | ~t, A = half 0 + half 1 (the same order for every
-            // candidate) or, for max logits, the larger half; each lane holds its
-            // candidates' keys in registers
-            const int nC = d.nC, ksel = d.ksel, c_lo = d.c_lo;
-            constexpr bool mx = kMaxLogit;
-            auto key_of = [&](int cj) {
-                return topk::make_key_agg(mx ? fmaxf(A0[cj], A1[cj]) : A0[cj] + A1[cj], c_lo + cj, mx);
-            };
-            if (nC <= 32 * kRegKeys) {
-                unsigned long long key[kRegKeys];
-#pragma unroll
-                for (int r = 0; r < kRegKeys; ++r) {
-                    const int cj = lane + 32 * r;
-                    key[r] = cj < nC ? key_of(cj) : 0ull;
-                }
-                for (int k = 0; k < ksel; ++k) {
-                    unsigned long long best = key[0];
-#pragma unroll
-                    for (int r = 1; r < kRegKeys; ++r) best = topk::umax64(best, key[r]);
-                    const unsigned mh = (unsigned)(best >> 32), ml = (unsigned)best;
-                    const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
-                    const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
-                    const unsigned long long win = ((unsigned long long)bh << 32) | bl;
-                    if (lane == 0) sel[k] = topk::key_block(win);
-#pragma unroll
-                    for (int r = 0; r < kRegKeys; ++r)
-                        if (key[r] == win) key[r] = 0ull;
-                }
-            } else {
-                // a pick is marked by a NaN bit pattern that arithmetic never produces
-                topk::rounds_one_warp(
-                    nC, ksel, key_of, [&](int cj) { return __float_as_uint(A1[cj]) == 0xffffffffu; },
-                    [&](int t) { A1[t - c_lo] = __uint_as_float(0xffffffffu); }, sel, lane);
-            }
-            __syncwarp();
-            // A is no longer needed: the elementwise warps may refill this buffer
-            if (lane == 0) mbar_arrive(bar(B_AFREE + buf));
-            for (int j = lane; j < a.topk; j += 32) {
-                if (j < d.n_init_q) out[j] = j;
-                else if (j >= d.n_init_q + ksel && j < d.nF + ksel) out[j] = d.loc_lo + (j - d.n_init_q - ksel);
-                else if (j >= d.nF + ksel) out[j] = -1;
-            }
-            for (int j = lane; j < ksel; j += 32) {
-                const int v = sel[j];
-                int rank = 0;
-                for (int i = 0; i < ksel; ++i) rank += sel[i] < v;
-                out[d.n_init_q + rank] = v;
-            }
-            if (lane == 0) a.cnt_out[d.lu] = d.nF + ksel;
-            __syncwarp();  // sel is reused by the next unit
-            ++su;
-        }
     } else {
-        // ------------------------------------------------ elementwise (8 warps)
-        const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-        const int r = (warp & 3) * 32 + lane;  // pass 1: query row; pass 2: candidate
-        const int hh = warp >> 2;              // half of the TMEM columns this thread reads
+        // ------------------------------------------------ elementwise: warps 4si .. 4si + 3
+        const int si = warp >> 2, wq = warp & 3;
+        const int r = wq * 32 + lane;  // TMEM lane: pass 1 query row, pass 2 candidate
+        const uint32_t lane_base = tmem + ((uint32_t)(wq * 32) << 16);
+        float* negM = reinterpret_cast<float*>(smem + a.off_stats) + si * 128;
+        float* Aspan = reinterpret_cast<float*>(smem + a.off_A) + (size_t)si * kSub * a.a_stride;
+        const float cs = a.scale_log2;
         bool ok = true;
-        int gs = 0, su = 0;
-        // After a failed wait the loops keep running without work, so that all eight
-        // warps reach the named barriers after pass 1 the same number of times.
-        const int et = threadIdx.x;  // 0..255 over the elementwise warps
-        for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-            const SelUnit d = sel_unit_k<kSub>(a, u);
-            if constexpr (kSub > 1) {
-                if (!d.scored) {  // every query block of the span is covered by its budget
-                    for (int j = 0; j < kSub && d.qb * kSub + j < a.NQB; ++j)
-                        write_unscored(a, d.bg, d.qb * kSub + j, qb_sel(a, d.qb * kSub + j), et, 256);
-                    continue;
-                }
-            }
-            if (!d.scored) continue;
-            const int nch = d.nch, steps = (kMaxLogit ? 1 : 2) * nch, c_lo = d.c_lo, c_hi = d.c_hi, nC = d.nC;
-            const bool row_ok = d.qb * 64 + (r & 63) < a.L;
-            // pass 1: this row's own candidate bound (its query block's, at kSub > 1)
-            const int c_hi_r = kSub == 1 ? c_hi : min(c_hi, d.qb * kSub + (r & 63) / (64 / kSub) - a.n_local);
-            const int buf = kSub == 1 ? (su & 1) : 0;
-            float* A0 = Abuf + (size_t)buf * 2 * a.NQB;
-            float* A1 = A0 + a.NQB;
-            if (kSub == 1 && ok && su >= 2) {  // the top-k warp is done with this buffer's previous unit
-                ok = mbar_wait(bar(B_AFREE + buf), ((su >> 1) - 1) & 1, abort_flag, a.status);
+        int kst = 0;  // this span slot's TMEM steps so far (the MMA thread's k[si])
+        // wait for the span's next TMEM buffer, load its 128 columns, release it
+        auto next_buffer = [&](uint32_t* v) {
+            const int b = 2 * si + (kst & 1);
+            if (ok) {
+                ok = mbar_wait(bar(B_SFULL + b), (kst >> 1) & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
-            float m = -INFINITY, z = 0.f;
-            for (int s = 0; s < steps; ++s, ++gs) {
-                const int slot = gs & 1, c = step_chunk(s, nch, kMaxLogit);
-                if (ok) {
-                    ok = mbar_wait(bar(B_SFULL + slot), (gs >> 1) & 1, abort_flag, a.status);
-                    ok = __all_sync(0xffffffffu, ok);
-                }
-                if (ok) tc_fence_after();
-                if (ok && !kMaxLogit && s < nch) {
-                    // pass 1: row r against 64 candidates of the chunk, two loads of 32
-                    const int t0 = c_lo + c * kCand + 64 * hh;
-                    const bool full = t0 + 63 <= c_hi_r;
-#pragma unroll 1
-                    for (int q = 0; q < 2; ++q) {
-                        if (t0 + 32 * q > c_hi) break;  // no candidate left in this group (warp-uniform)
-                        uint32_t v[32];
-                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
-                        // max of the raw scores, then the scale (positive) once
-                        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                        if (!full) {
+            if (ok) {
+                tc_fence_after();
+                tmem_ld128(lane_base + 128u * b, v);
+                tc_fence_before();
+                mbar_arrive(bar(B_SFREE + b));
+            }
+            ++kst;
+            return ok;
+        };
+        for (int v = blockIdx.x; v < a.batches; v += gridDim.x) {
+            const BatchInfo B = batch_info<kSub>(a, v);
+            const SpanInfo sp = si == 0 ? B.sp[0] : B.sp[1];
+            if (!sp.present) continue;
+            const int qb0 = sp.s * kSub;
+            if (!sp.scored) {  // every query block of the span is covered by its budget
+                for (int j = 0; j < sp.nqb; ++j)
+                    write_unscored(a, B.bg, qb0 + j, qb_sel(a, qb0 + j), r, 128);
+                continue;
+            }
+            uint32_t val[128];
+            if constexpr (!kMaxLogit) {
+                // ---- pass 1: row r = (head r / 64, token r % 64) of query block j_r
+                const int tok = r & 63, j_r = tok / kTok;
+                const bool row_ok = sp.s * 64 + tok < a.L && j_r < sp.nqb;
+                const int c_hi_r = qb0 + j_r - a.n_local;  // the row's last candidate
+                float m = -INFINITY, z = 0.f;
+                for (int c = 0; c < sp.nch; ++c) {
+                    if (!next_buffer(val)) continue;
+                    const int t0 = a.n_init + c * kCand;
+                    const int nv = row_ok ? min(kCand, c_hi_r - t0 + 1) : 0;  // valid columns
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        uint32_t* x = val + 32 * g;
+                        if (32 * g >= nv) continue;
+                        if (32 * g + 31 >= nv) {
 #pragma unroll
                             for (int j = 0; j < 32; ++j)
-                                if (t0 + 32 * q + j > c_hi_r) v[j] = __float_as_uint(-INFINITY);
+                                if (32 * g + j >= nv) x[j] = __float_as_uint(-INFINITY);
                         }
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) m4[j & 3] = fmaxf(m4[j & 3], __uint_as_float(v[j]));
-                        const float mn = fmaxf(m, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2);
-                        if (mn != -INFINITY) {
-                            float s4[4] = {0.f, 0.f, 0.f, 0.f};
-                            const float neg = -mn;
-#pragma unroll
-                            for (int j = 0; j < 32; ++j)
-                                s4[j & 3] += ex2_approx(fmaf(__uint_as_float(v[j]), a.scale_log2, neg));
-                            if (mn > m) z *= ex2_approx(m - mn);  // the running max moved
-                            z += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+                        if (m == -INFINITY) m = max32(x) * cs;  // the row's first shift
+                        float sg = expsum32(x, cs, -m);
+                        if (!(sg <= 3.0e38f)) {  // a score far above the shift: move it
+                            const float mn = max32(x) * cs;
+                            z *= ex2_approx(m - mn);
                             m = mn;
+                            sg = expsum32(x, cs, -m);
                         }
+                        z += sg;
                     }
-                    tc_fence_before();
-                    mbar_arrive(bar(B_SFREE + slot));
-                } else if (ok && kMaxLogit && kSub > 1) {
-                    // max logit, per query block of the span: candidate r against the
-                    // rows of half hh (head hh), kSub groups of 64 / kSub tokens
-                    float mxs[kSub];
-#pragma unroll
-                    for (int sb = 0; sb < kSub; ++sb) mxs[sb] = -INFINITY;
-                    if (c * kCand + (warp & 3) * 32 < nC) {
-#pragma unroll
-                        for (int q = 0; q < 2; ++q) {
-                            uint32_t v[32];
-                            tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
-                            const int tok0 = d.qb * 64 + 32 * q;
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) {
-                                constexpr int kTok = 64 / kSub;
-                                const float x = tok0 + j < a.L ? __uint_as_float(v[j]) : -INFINITY;
-                                mxs[(32 * q + j) / kTok] = fmaxf(mxs[(32 * q + j) / kTok], x);
-                            }
-                        }
-                    }
-                    tc_fence_before();
-                    mbar_arrive(bar(B_SFREE + slot));
-                    const int cj = c * kCand + r;
-                    if (cj < nC) {
-#pragma unroll
-                        for (int sb = 0; sb < kSub; ++sb)
-                            Abuf[(size_t)(2 * sb + hh) * a.NQB + cj] = mxs[sb] * a.scale;
-                    }
-                } else if (ok && !kMaxLogit && kSub > 1 && s >= nch) {
-                    // pass 2, per query block of the span: the sums over its rows of
-                    // head hh, in row order. Query block sb of the span has candidates
-                    // up to qb*kSub + sb - n_local; this thread's candidate t past that
-                    // bound takes no part in sb's sum (its 2^x is not evaluated).
-                    const float* mrow = m2s + 64 * hh;
-                    const int t_c = c_lo + c * kCand + r;
-                    const int sb_bound = d.qb * kSub - a.n_local;  // + sb: query block sb's c_hi
-                    float accs[kSub][2];
-#pragma unroll
-                    for (int sb = 0; sb < kSub; ++sb) accs[sb][0] = accs[sb][1] = 0.f;
-                    if (c * kCand + (warp & 3) * 32 < nC) {
-#pragma unroll
-                        for (int q = 0; q < 2; ++q) {
-                            uint32_t v[32];
-                            tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) {
-                                constexpr int kTok = 64 / kSub;
-                                const int sb = (32 * q + j) / kTok;
-                                if (t_c <= sb_bound + sb)
-                                    accs[sb][j & 1] += ex2_approx(
-                                        fmaf(__uint_as_float(v[j]), a.scale_log2, -mrow[32 * q + j]));
-                            }
-                        }
-                    }
-                    tc_fence_before();
-                    mbar_arrive(bar(B_SFREE + slot));
-                    const int cj = c * kCand + r;
-                    if (cj < nC) {
-#pragma unroll
-                        for (int sb = 0; sb < kSub; ++sb)
-                            Abuf[(size_t)(2 * sb + hh) * a.NQB + cj] = accs[sb][0] + accs[sb][1];
-                    }
-                } else if (ok && kMaxLogit) {
-                    // max logit: candidate r against the 64 rows of half hh (head hh)
-                    float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                    const bool live = c * kCand + (warp & 3) * 32 < nC;
-#pragma unroll 1
-                    for (int q = 0; q < (live ? 2 : 0); ++q) {
-                        uint32_t v[32];
-                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
-                        const int tok0 = d.qb * 64 + 32 * q;  // rows of head hh: tokens tok0 + j
-                        const bool all_rows = tok0 + 31 < a.L;
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            const float x = (all_rows || tok0 + j < a.L) ? __uint_as_float(v[j]) : -INFINITY;
-                            mx4[j & 3] = fmaxf(mx4[j & 3], x);
-                        }
-                    }
-                    tc_fence_before();
-                    mbar_arrive(bar(B_SFREE + slot));
-                    const int cj = c * kCand + r;
-                    if (cj < nC)
-                        (hh ? A1 : A0)[cj] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * a.scale;
-                } else if (ok) {
-                    // pass 2: candidate r against the 64 rows of half hh, in row order;
-                    // a warp whose 32 candidates all lie past the last one skips the work
-                    // p = 2^(S*scale - m_r - log2 Z_r): the row's max and sum in one offset
-                    const float* mrow = m2s + 64 * hh;
-                    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-                    const bool live = c * kCand + (warp & 3) * 32 < nC;
-#pragma unroll 1
-                    for (int q = 0; q < (live ? 2 : 0); ++q) {
-                        uint32_t v[32];
-                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
-#pragma unroll
-                        for (int j = 0; j < 32; j += 4) {
-                            const float4 mm = *reinterpret_cast<const float4*>(mrow + 32 * q + j);
-                            acc[0] += ex2_approx(fmaf(__uint_as_float(v[j + 0]), a.scale_log2, -mm.x));
-                            acc[1] += ex2_approx(fmaf(__uint_as_float(v[j + 1]), a.scale_log2, -mm.y));
-                            acc[2] += ex2_approx(fmaf(__uint_as_float(v[j + 2]), a.scale_log2, -mm.z));
-                            acc[3] += ex2_approx(fmaf(__uint_as_float(v[j + 3]), a.scale_log2, -mm.w));
-                        }
-                    }
-                    tc_fence_before();
-                    mbar_arrive(bar(B_SFREE + slot));
-                    const int cj = c * kCand + r;
-                    if (cj < nC) (hh ? A1 : A0)[cj] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
                 }
-                if (!kMaxLogit && s == nch - 1) {
-                    // merge the two column halves of every row: (m, z) -> max and 1/sum
-                    pm[hh * 128 + r] = m;
-                    pz[hh * 128 + r] = z;
-                    named_barrier(1, 256);
-                    if (hh == 0) {
-                        const float ma = pm[r], mb = pm[128 + r];
-                        const float mx = fmaxf(ma, mb);
-                        const float za = ma == -INFINITY ? 0.f : pz[r] * ex2_approx(ma - mx);
-                        const float zb = mb == -INFINITY ? 0.f : pz[128 + r] * ex2_approx(mb - mx);
-                        const float zz = za + zb;
-                        // a row past L (or without candidates) contributes 2^-inf = 0
-                        m2s[r] = (row_ok && zz > 0.f) ? mx + log2f(zz) : INFINITY;
-                    }
-                    named_barrier(1, 256);
-                }
+                // a row past L or without candidates contributes 2^-inf = 0 in pass 2
+                negM[r] = (row_ok && z > 0.f) ? -(m + log2f(z)) : -INFINITY;
+                named_barrier(1 + si, 128);
             }
-            if constexpr (kSub == 1) {
-                if (ok) mbar_arrive(bar(B_AFULL + buf));  // this thread's A entries are written
-            } else {
-                // Top-k of each query block of the span, by the eight elementwise
-                // warps: the two-level selection (topk.cuh) when it applies, else
-                // one warp's rounds; every warp passes the same barriers.
-                named_barrier(1, 256);  // every A entry of the span is written
-                unsigned long long* fin = reinterpret_cast<unsigned long long*>(pm);  // 2 KB
+            // ---- pass 2: candidate t of the chunk against the span's 128 rows
+            const bool tail = sp.s * 64 + 63 >= a.L;  // rows past L exist in this span
+            for (int c = sp.nch - 1; c >= 0; --c) {
+                if (!next_buffer(val)) continue;
+                const int cj = c * kCand + r, t = a.n_init + cj;
+                if (cj >= sp.nC) continue;
+#pragma unroll
                 for (int j = 0; j < kSub; ++j) {
-                    const int qb = d.qb * kSub + j;
-                    if (qb >= a.NQB) break;
-                    const QbSel q = qb_sel(a, qb);
-                    if (!q.scored) {
-                        write_unscored(a, d.bg, qb, q, et, 256);
-                        continue;
+                    if (j >= sp.nqb || t > qb0 + j - a.n_local) continue;  // not j's candidate
+                    float res;
+                    if constexpr (kMaxLogit) {
+                        float mx = -INFINITY;
+#pragma unroll
+                        for (int h = 0; h < 2; ++h)
+#pragma unroll
+                            for (int k2 = 0; k2 < kTok; ++k2) {
+                                const int col = h * 64 + j * kTok + k2;
+                                const float x = (!tail || sp.s * 64 + j * kTok + k2 < a.L)
+                                                    ? __uint_as_float(val[col]) : -INFINITY;
+                                mx = fmaxf(mx, x);
+                            }
+                        res = mx * a.scale;
+                    } else {
+                        const float2 cc = make_float2(cs, cs);
+                        float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+                        for (int h = 0; h < 2; ++h)
+#pragma unroll
+                            for (int k2 = 0; k2 < kTok; k2 += 4) {
+                                const int col = h * 64 + j * kTok + k2;
+                                const float4 mm = *reinterpret_cast<const float4*>(negM + col);
+                                float2 e0 = __ffma2_rn(make_float2(__uint_as_float(val[col]), __uint_as_float(val[col + 1])), cc,
+                                                       make_float2(mm.x, mm.y));
+                                float2 e1 = __ffma2_rn(make_float2(__uint_as_float(val[col + 2]), __uint_as_float(val[col + 3])), cc,
+                                                       make_float2(mm.z, mm.w));
+                                e0.x = ex2_approx(e0.x);
+                                e0.y = ex2_approx(e0.y);
+                                e1.x = ex2_approx(e1.x);
+                                e1.y = ex2_approx(e1.y);
+                                acc[0] = __fadd2_rn(acc[0], e0);
+                                acc[1] = __fadd2_rn(acc[1], e1);
+                            }
+                        const float2 s = __fadd2_rn(acc[0], acc[1]);
+                        res = s.x + s.y;
                     }
-                    float* Aj0 = Abuf + (size_t)(2 * j) * a.NQB;
-                    float* Aj1 = Aj0 + a.NQB;
-                    auto key_of = [&](int cj) {
-                        return topk::make_key_agg(kMaxLogit ? fmaxf(Aj0[cj], Aj1[cj]) : Aj0[cj] + Aj1[cj],
-                                                  c_lo + cj, kMaxLogit);
-                    };
-                    if (topk::two_level(q.nC, q.ksel)) {
-                        topk::level1(q.nC, q.ksel, key_of, fin, warp, lane);
-                        named_barrier(1, 256);
-                        topk::level2(fin, q.ksel, sel, et);
-                    } else if (warp == 0) {
-                        // a pick is marked by a NaN bit pattern that arithmetic never produces
-                        topk::rounds_one_warp(
-                            q.nC, q.ksel, key_of,
-                            [&](int cj) { return __float_as_uint(Aj1[cj]) == 0xffffffffu; },
-                            [&](int t) { Aj1[t - c_lo] = __uint_as_float(0xffffffffu); }, sel, lane);
-                    }
-                    named_barrier(1, 256);
-                    int32_t* out = a.idx_out + ((long long)d.bg * a.NQB + qb) * a.topk;
-                    for (int x = et; x < a.topk; x += 256) {
-                        if (x < q.n_init_q) out[x] = x;
-                        else if (x >= q.n_init_q + q.ksel && x < q.nF + q.ksel) out[x] = q.loc_lo + (x - q.n_init_q - q.ksel);
-                        else if (x >= q.nF + q.ksel) out[x] = -1;
-                    }
-                    for (int x = et; x < q.ksel; x += 256) {
-                        const int v = sel[x];
-                        int rank = 0;
-                        for (int i = 0; i < q.ksel; ++i) rank += sel[i] < v;
-                        out[q.n_init_q + rank] = v;
-                    }
-                    if (et == 0) a.cnt_out[(long long)d.bg * a.NQB + qb] = q.nF + q.ksel;
-                    named_barrier(1, 256);  // sel and fin are reused
+                    Aspan[(size_t)j * a.a_stride + cj] = res;
                 }
             }
-            ++su;
+            named_barrier(1 + si, 128);  // every aggregate of the span is written
+            // ---- top-k: kW = 4 / kSub warps per query block of the span
+            {
+                constexpr int kW = 4 / kSub;
+                const int j = wq / kW, wi = wq % kW;
+                if (j < sp.nqb) {
+                    const int qb = qb0 + j;
+                    const QbSel q = qb_sel(a, qb);
+                    float* Aq = Aspan + (size_t)j * a.a_stride;
+                    if (!q.scored) {
+                        if (wi == 0) write_unscored(a, B.bg, qb, q, lane, 32);
+                    } else if (kW == 1 || q.ksel > 32) {
+                        if (wi == 0 && ok) topk_write<kMaxLogit>(a, B.bg, qb, q, Aq, lane);
+                    } else {
+                        unsigned long long* fin =
+                            reinterpret_cast<unsigned long long*>(smem + a.off_fin) + si * 128 + j * 32 * kW;
+                        topk_split<kMaxLogit, kW>(a, B.bg, qb, q, Aq, fin, wi, lane,
+                                                  3 + 2 * si + j, ok);
+                    }
+                }
+            }
+            // pass 2 of the next batch rewrites A and negM only after the next
+            // pass-1 barrier (or, for max logits, the barrier below), which every
+            // warp reaches after its top-k
+            if constexpr (kMaxLogit) named_barrier(1 + si, 128);
         }
     }
     tc_fence_before();
@@ -634,14 +652,22 @@ select_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 
 }  // namespace
 
+namespace {
+bool use_unit_kernel(const phsa_shape& s) {
+    return s.block_size == 64 && (s.L + 63) / 64 <= kSelectUnitMaxNqb;
+}
+}  // namespace
+
 size_t select_tc_smem_bytes(const phsa_shape& s, int topk) {
+    if (use_unit_kernel(s)) return select_tc_unit_smem_bytes(s, topk);
     const int bm = s.block_size;
-    return select_tc_smem((s.L + bm - 1) / bm, topk, 64 / bm);
+    return sel_layout_fit((s.L + bm - 1) / bm, 64 / bm).total;
 }
 
 cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape& s,
                              const phsa_select_params& p, int32_t* idx, int32_t* cnt, int* status,
                              cudaStream_t st) {
+    if (use_unit_kernel(s)) return launch_select_tc_unit(Q, Krepr, s, p, idx, cnt, status, st);
     const int bm = s.block_size, kSub = 64 / bm;
     const int T = s.L / bm, NQB = (s.L + bm - 1) / bm;
     CUtensorMap tq, tkr;
@@ -649,26 +675,32 @@ cudaError_t launch_select_tc(const void* Q, const void* Krepr, const phsa_shape&
     // Krepr may be absent when no query block has a candidate (T < 2): the map is
     // then built over Q, which is never read through it.
     if (!make_tmap_bf16_rows128(&tkr, T > 0 ? Krepr : Q, T > 0 ? T : 1,
-                                (uint64_t)s.B * s.Hkv, 128))
+                                (uint64_t)s.B * s.Hkv, 64))
         return cudaErrorInvalidValue;
-    const size_t smem = select_tc_smem(NQB, p.topk, kSub);
+    const SelLayout lay = sel_layout_fit(NQB, kSub);
     const bool mx = p.aggregation == PHSA_AGG_MAX_LOGIT;
     auto kern = kSub == 1 ? (mx ? select_tc_kernel<true, 1> : select_tc_kernel<false, 1>)
                 : kSub == 2 ? (mx ? select_tc_kernel<true, 2> : select_tc_kernel<false, 2>)
                             : (mx ? select_tc_kernel<true, 4> : select_tc_kernel<false, 4>);
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lay.total);
     if (e != cudaSuccess) return e;
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
-    const int nsb = kSub == 1 ? NQB : (NQB + kSub - 1) / kSub;
-    const int units = s.B * s.Hkv * nsb;
-    const int per_sm = smem * 2 + 2048 <= kMaxDynSmem + 1024 ? 2 : 1;  // two CTAs when shared memory allows
-    SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local, units,
-                 p.aggregation, p.sm_scale * kLog2e, p.sm_scale, nsb};
+    const int nsb = (NQB + kSub - 1) / kSub;
+    const int nbat = (nsb + 1) / 2;
+    const int BG = s.B * s.Hkv;
+    const long long batches = (long long)BG * nbat;
+    if (batches == 0) return cudaSuccess;
+    SelArgs args{idx, cnt, status, s.Hq, s.Hkv, s.L, T, NQB, p.topk, p.n_init, p.n_local,
+                 p.aggregation, nsb, nbat, BG, (int)batches, p.sm_scale * kLog2e, p.sm_scale,
+                 lay.nq, lay.slots, lay.a_stride, (uint32_t)lay.kr, (uint32_t)lay.stats,
+                 (uint32_t)lay.fin, (uint32_t)lay.A, (uint32_t)lay.bar, (uint32_t)lay.misc};
     ProfScope prof(K_SELECT, st);
-    kern<<<(unsigned)min(units, per_sm * nsm), kThreads, smem, st>>>(tq, tkr, args);
+    const unsigned grid = (unsigned)(batches < nsm ? batches : nsm);
+    kern<<<grid, kThreads, lay.total, st>>>(tq, tkr, args);
     return cudaGetLastError();
 }
 

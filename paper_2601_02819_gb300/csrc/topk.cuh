@@ -136,5 +136,66 @@ __device__ __forceinline__ void rounds_one_warp(int nC, int ksel, KeyOf key_of, 
     }
 }
 
+// One warp, at most 32 picks, any number of candidates: the candidates are
+// taken 512 at a time (16 keys per lane in registers) together with the picks
+// so far (lane k holds the k-th best key, one register), and ksel rounds of a
+// warp-wide maximum keep the best ksel of them. Returns this lane's pick
+// (lane < ksel; 0 on the other lanes). Requires 1 <= ksel <= 32 and ksel <= nC.
+template <class KeyOf>
+__device__ __forceinline__ unsigned long long warp_topk32(int nC, int ksel, KeyOf key_of, int lane) {
+    unsigned long long best = 0ull;
+    for (int base = 0; base < nC; base += 512) {
+        unsigned long long key[16];
+#pragma unroll
+        for (int r = 0; r < 16; ++r) {
+            const int cj = base + lane + 32 * r;
+            key[r] = cj < nC ? key_of(cj) : 0ull;
+        }
+        unsigned long long carry = best;
+        best = 0ull;
+        for (int k = 0; k < ksel; ++k) {
+            unsigned long long m = carry;
+#pragma unroll
+            for (int r = 0; r < 16; ++r) m = umax64(m, key[r]);
+            const unsigned mh = (unsigned)(m >> 32), ml = (unsigned)m;
+            const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
+            const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
+            const unsigned long long win = ((unsigned long long)bh << 32) | bl;
+            if (lane == k) best = win;
+            if (carry == win) carry = 0ull;
+#pragma unroll
+            for (int r = 0; r < 16; ++r)
+                if (key[r] == win) key[r] = 0ull;
+        }
+    }
+    return best;
+}
+
+// One warp, any budget: rounds over all candidates that mark each pick with
+// take(t) in the caller's storage (taken(cj) tests the mark); no list of picks
+// is kept, so the caller reads the picks back in ascending order.
+template <class KeyOf, class Taken, class Take>
+__device__ __forceinline__ void rounds_mark_one_warp(int nC, int ksel, KeyOf key_of, Taken taken,
+                                                     Take take, int lane) {
+    auto lane_best = [&]() {
+        unsigned long long best = 0ull;
+        for (int cj = lane; cj < nC; cj += 32)
+            if (!taken(cj)) best = umax64(best, key_of(cj));
+        return best;
+    };
+    unsigned long long mine = lane_best();
+    for (int k = 0; k < ksel; ++k) {
+        const unsigned mh = (unsigned)(mine >> 32), ml = (unsigned)mine;
+        const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
+        const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
+        const unsigned long long win = ((unsigned long long)bh << 32) | bl;
+        if (bl != 0u && mine == win) {
+            take(key_block(win));
+            mine = lane_best();
+        }
+        __syncwarp();
+    }
+}
+
 }  // namespace topk
 }  // namespace phsa

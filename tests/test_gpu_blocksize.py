@@ -192,6 +192,17 @@ def test_selection_long_sequence_at_m16_uses_the_warp_mma_kernel(aggregation):
     _sampled_selection(16, 16 * 4200 + 3, 20, 1, 2, aggregation, 4200)
 
 
+@pytest.mark.parametrize("n_init,n_local", [(1, 1), (2, 8)])
+@pytest.mark.parametrize("aggregation", ["softmax_sum", "max_logit"])
+def test_selection_span_pair_kernel_at_m64_beyond_1024_query_blocks(n_init, n_local, aggregation):
+    # Past 1024 query blocks of 64 the pair selection runs on the span-pair
+    # kernel (two 64-token spans share every candidate chunk); its candidate
+    # ranges reach 9 chunks, more than the ring holds for pass 2.
+    NQB = 1100
+    _sampled_selection(64, 64 * NQB + 17, 14, n_init, n_local, aggregation, 1100 + n_local,
+                       extra_units=[NQB - 2, NQB - 3, 1025, 1024, 1023])
+
+
 @pytest.mark.parametrize("m,L,topk,n_init,n_local", [
     (16, 16 * 300 + 9, 40, 1, 2),   # 37 picks per query block: beyond the two-level top-k
     (32, 32 * 200 + 5, 36, 1, 1),   # 34 picks at m = 32
