@@ -500,21 +500,34 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 const bool live = e < n;          // false: the duplicate of an odd count
                 const bool diag = list[e] == qb;
                 uint32_t sv[64], dp[64];
-                tmem_ld64(lane_base + col_s(buf) + 64 * half, sv);
-                tmem_ld64(lane_base + kColDP + 64 * half, dp);
+                tmem_ld64x2(lane_base + col_s(buf) + 64 * half, lane_base + kColDP + 64 * half, sv, dp);
                 tc_fence_before();
                 mbar_arrive(bar(B_DPFREE));  // dP is in registers: the buffer may be refilled
+                // dS = P (dP - Delta), P = 2^(S scale_log2 - lse log2 e), two keys at a
+                // time (packed f32x2 arithmetic); the masks (the query's own block and the
+                // duplicate of an odd count) are warp-uniform branches off the main path
+                const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+                const float2 nl2v = make_float2(nl2, nl2), ndl = make_float2(-dlt, -dlt);
+                if (live && !diag) {
 #pragma unroll
-                for (int c = 0; c < 32; ++c) {
-                    float ds[2];
-#pragma unroll
-                    for (int x = 0; x < 2; ++x) {
-                        const int key = 2 * c + x;
-                        float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + x]), a.scale_log2, nl2));
-                        if (!live || (diag && key > tok)) pv = 0.f;
-                        ds[x] = pv * (__uint_as_float(dp[2 * c + x]) - dlt);
+                    for (int c = 0; c < 32; ++c) {
+                        float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
+                        pv.x = ex2_approx(pv.x);
+                        pv.y = ex2_approx(pv.y);
+                        const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
+                        const float2 ds = __fmul2_rn(pv, d);
+                        sv[c] = pack2_bf16(ds.x, ds.y);
                     }
-                    sv[c] = pack2_bf16(ds[0], ds[1]);
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) {
+                        float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
+                        pv.x = (live && 2 * c <= tok) ? ex2_approx(pv.x) : 0.f;
+                        pv.y = (live && 2 * c + 1 <= tok) ? ex2_approx(pv.y) : 0.f;
+                        const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
+                        const float2 ds = __fmul2_rn(pv, d);
+                        sv[c] = pack2_bf16(ds.x, ds.y);
+                    }
                 }
                 // dS columns [64 half, 64 half + 32): inside this thread's own S range
                 tmem_st32(lane_base + col_s(buf) + 64 * half, sv);
@@ -961,22 +974,27 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 if (!ok) break;
                 tc_fence_after();
                 uint32_t sv[32], dp[32];
-                tmem_ld32(lane_base + col_s(buf) + 32 * kh, sv);
-                tmem_ld32(lane_base + col_dp(buf) + 32 * kh, dp);
+                tmem_ld32x2(lane_base + col_s(buf) + 32 * kh, lane_base + col_dp(buf) + 32 * kh, sv, dp);
                 const bool diag = qb == t;
+                // P = 2^(S scale_log2 - lse log2 e), dS = P (dP - Delta), two keys at a
+                // time (packed f32x2); the causal mask only on the diagonal block
+                const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+                const float2 nl2v = make_float2(neg_lse2, neg_lse2), ndl = make_float2(-dlt, -dlt);
 #pragma unroll
                 for (int c = 0; c < 16; ++c) {
-                    float p[2], ds[2];
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int key = 32 * kh + 2 * c + e;
-                        float pv = ex2_approx(fmaf(__uint_as_float(sv[2 * c + e]), a.scale_log2, neg_lse2));
-                        if (diag && key > tok) pv = 0.f;
-                        p[e] = pv;
-                        ds[e] = pv * (__uint_as_float(dp[2 * c + e]) - dlt);
+                    float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
+                    if (!diag) {
+                        pv.x = ex2_approx(pv.x);
+                        pv.y = ex2_approx(pv.y);
+                    } else {
+                        const int key = 32 * kh + 2 * c;
+                        pv.x = key <= tok ? ex2_approx(pv.x) : 0.f;
+                        pv.y = key + 1 <= tok ? ex2_approx(pv.y) : 0.f;
                     }
-                    sv[c] = pack2_bf16(p[0], p[1]);
-                    dp[c] = pack2_bf16(ds[0], ds[1]);
+                    const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
+                    const float2 ds = __fmul2_rn(pv, d);
+                    sv[c] = pack2_bf16(pv.x, pv.y);
+                    dp[c] = pack2_bf16(ds.x, ds.y);
                 }
                 tc_fence_before();
                 if (gi >= 2) {  // the dV/dK MMAs two iterations back must have read this buffer

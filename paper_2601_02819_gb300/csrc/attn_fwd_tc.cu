@@ -383,10 +383,11 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     for (int c = 0; c < 64; ++c)
                         if (c > tok) sr[c] = __float_as_uint(-INFINITY);
                 }
-                // row max of the raw scores (the scale is positive)
+                // row max of the raw scores (the scale is positive), three-input maxima
                 float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                for (int c = 0; c < 64; ++c) m4[c & 3] = fmaxf(m4[c & 3], __uint_as_float(sr[c]));
+                for (int c = 0; c < 64; c += 2)
+                    m4[(c >> 1) & 3] = fmax3(m4[(c >> 1) & 3], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
                 const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;
                 if (j == 0) {
                     m_used = mx;
@@ -413,19 +414,22 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                         }
                     }
                 }
-                // p = 2^(s * scale_log2 - m): one FFMA and one SFU op per score
-                // P is packed in place: entry c (c < 32) takes the pair (2c, 2c+1), both
-                // read before entry c is overwritten.
-                float r4[4] = {0.f, 0.f, 0.f, 0.f};
-                const float neg_m = -m_used;
+                // p = 2^(s * scale_log2 - m): one packed FFMA per two scores and one SFU
+                // op per score. P is packed in place: entry c (c < 32) takes the pair
+                // (2c, 2c+1), both read before entry c is overwritten.
+                float2 r2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+                const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+                const float2 nm2 = make_float2(-m_used, -m_used);
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
-                    const float p0 = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), a.scale_log2, neg_m));
-                    const float p1 = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), a.scale_log2, neg_m));
-                    r4[c & 3] += p0 + p1;
-                    sr[c] = pack2_bf16(p0, p1);
+                    float2 p2 = __ffma2_rn(make_float2(__uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1])), sc2, nm2);
+                    p2.x = ex2_approx(p2.x);
+                    p2.y = ex2_approx(p2.y);
+                    r2[c & 1] = __fadd2_rn(r2[c & 1], p2);
+                    sr[c] = pack2_bf16(p2.x, p2.y);
                 }
-                const float rs = (r4[0] + r4[1]) + (r4[2] + r4[3]);
+                const float2 rr = __fadd2_rn(r2[0], r2[1]);
+                const float rs = rr.x + rr.y;
                 l += rs;
                 tmem_st32(lane_base + col_s(buf), sr);
                 tc_fence_before();
