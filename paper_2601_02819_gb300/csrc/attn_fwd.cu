@@ -258,10 +258,12 @@ cudaError_t launch_attn_fwd(const void* Q, const void* K, const void* V, const i
                             const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                             void* O, float* lse, int* status, cudaStream_t st) {
     if ((long long)s.B * s.Hkv * s.L == 0) return cudaSuccess;
-    // Two query heads per KV head at m = 64 fill a 128-row tcgen05 tile; every
-    // other group and block size runs on the warp-level MMA kernel in this file.
+    // Two query heads per KV head fill a 128-row tcgen05 tile at every block size
+    // (at m < 64 the tile is a 64-token span; its list union must fit in shared
+    // memory); a single head, and larger budgets at m < 64, run on the
+    // warp-level MMA kernel in this file.
     const int G = s.Hq / s.Hkv, bm = s.block_size;
-    if (G == 2 && bm == 64)
+    if (G == 2 && (bm == 64 || attn_fwd_tc_smem_bytes(s, topk) <= kMaxDynSmem))
         return launch_attn_fwd_tc(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st);
 #define PHSA_FWD(g_, bm_) launch_fwd_g<g_, bm_>(Q, K, V, idx, cnt, s, topk, sm_scale, O, lse, status, st)
     if (G == 2) return bm == 16 ? PHSA_FWD(2, 16) : PHSA_FWD(2, 32);

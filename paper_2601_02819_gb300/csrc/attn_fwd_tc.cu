@@ -1,15 +1,29 @@
 // Stage (c) forward on the 5th-generation tensor cores (tcgen05 + TMEM + TMA),
-// for GQA groups of two query heads (G*64 = 128 query rows per tile).
+// for GQA groups of two query heads (G*64 = 128 query rows per tile), at block
+// sizes m = 64, 32 and 16.
+//
+// A unit is a 64-token span of one KV head: its 128 query rows (two heads x 64
+// tokens) are the kSub = 64/m query blocks of the span. At m = 64 that is one
+// query block and its selected blocks are the unit's key sequence. At m < 64
+// the key sequence is the union of the span's kSub block lists (ascending), and
+// each union entry carries an owner mask: which of the span's query blocks
+// selected it. A 64-key tile holds kSub consecutive union entries (m rows of K
+// and V each, gathered by TMA), and row r of query block j = (r mod 64) / m
+// attends a tile slot only if bit j of its owner mask is set (and, in j's own
+// block, only keys at or before its token). Padding slots past the union
+// repeat its last block and are masked for every row.
 //
 // Persistent: two CTAs per SM, each walking the units (query block qb, KV
 // head g) u = blockIdx.x, blockIdx.x + gridDim.x, ... with 256 threads in
 // five roles; rings, TMEM buffers and barriers run on counters that continue
 // across units, so one unit's loads and first MMAs overlap the previous
 // unit's last blocks and epilogue:
-//   warp 4 (one lane)  stages each unit's block list into one of four list
-//                      slots, a unit ahead, and gathers the selected K tiles
-//                      (64 x 128, by block index) into a two-slot ring; a slot
-//                      is refilled as soon as the QK MMA that read it is done.
+//   warp 4             stages each unit's block list (at m < 64: the union and
+//                      its owner masks, built by the whole warp through one
+//                      bitmap per query block) into one of four list slots, a
+//                      unit ahead; its lane 0 gathers the K tiles (64 x 128, by
+//                      block index) into a two-slot ring; a slot is refilled as
+//                      soon as the QK MMA that read it is done.
 //   warp 6 (one lane)  loads each unit's Q tile (128 x 128) once the previous
 //                      unit's last QK MMA is done, and the selected V tiles
 //                      into their own two-slot ring, refilled when the PV MMA
@@ -79,9 +93,17 @@ constexpr uint32_t kColO = 0;
 constexpr float kRescaleLog2 = 8.0f;
 static_assert(kOffBar + kNumBars * 8 <= kOffMisc, "barrier region");
 
-__host__ __device__ constexpr int list_slot_ints(int topk) { return (topk + 4) & ~3; }
-__host__ __device__ constexpr size_t fwd_tc_smem(int topk) {
-    return 1024 + (size_t)kOffList + kListSlots * (size_t)list_slot_ints(topk) * 4;
+// A list slot: [0] the count n, then n block indices (capacity kSub * topk),
+// then (kSub > 1) one owner-mask byte per entry.
+__host__ __device__ constexpr int list_cap(int topk, int kSub) { return kSub * topk; }
+__host__ __device__ constexpr int list_slot_ints(int topk, int kSub) {
+    return (1 + list_cap(topk, kSub) + (kSub > 1 ? (list_cap(topk, kSub) + 3) / 4 : 0) + 3) & ~3;
+}
+// words of one query block's bitmap over the blocks [0, nqb)
+__host__ __device__ constexpr int bitmap_words(int nqb) { return (nqb + 31) / 32; }
+__host__ __device__ constexpr size_t fwd_tc_smem(int topk, int kSub, int nqb) {
+    return 1024 + (size_t)kOffList + kListSlots * (size_t)list_slot_ints(topk, kSub) * 4 +
+           (kSub > 1 ? (size_t)kSub * bitmap_words(nqb) * 4 : 0);
 }
 
 struct FwdTcArgs {
@@ -90,7 +112,8 @@ struct FwdTcArgs {
     __nv_bfloat16* O;
     float* lse;
     int* status;
-    int Hq, Hkv, L, NQB, topk, units;
+    int Hq, Hkv, L, NQB, topk, units;  // NQB: query blocks of m tokens
+    int nsb;                           // 64-token spans per (b, g)
     float scale_log2;
 };
 
@@ -99,13 +122,104 @@ struct FwdUnit {
     long long lu;
 };
 
+// d.qb is the 64-token span (the query block itself at m = 64); d.lu the flat
+// index of its first query block.
+template <int kSub>
 __device__ __forceinline__ FwdUnit fwd_unit(const FwdTcArgs& a, int u) {
     FwdUnit d;
-    d.qb = a.NQB - 1 - (u % a.NQB);  // heaviest query blocks first
-    d.bg = u / a.NQB;
+    d.qb = a.nsb - 1 - (u % a.nsb);  // heaviest spans first
+    d.bg = u / a.nsb;
     d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
-    d.lu = (long long)d.bg * a.NQB + d.qb;
+    d.lu = (long long)d.bg * a.NQB + (long long)d.qb * kSub;
     return d;
+}
+
+// Warp-collective (all 32 lanes): the union of the block lists of the span's
+// query blocks, ascending, with owner masks (bit j: query block j of the span
+// selected the block), into a list slot. Each list is validated as
+// compact_block_list does (-1 entries skipped silently; an entry outside
+// [0, qb] or not above the last accepted one skipped and recorded): an entry
+// is accepted when it is in range and above every earlier in-range entry. The
+// per-query-block bitmaps over [0, NQB) are left cleared.
+template <int kSub>
+__device__ __forceinline__ void stage_union(const FwdTcArgs& a, const FwdUnit& d, int* sl,
+                                            uint32_t* bm, int lane) {
+    const int W = bitmap_words(a.NQB);
+    int hi = -1;
+    for (int j = 0; j < kSub; ++j) {
+        const int qbj = d.qb * kSub + j;
+        if (qbj >= a.NQB) break;
+        const long long lu = d.lu + j;
+        int n = __ldg(a.cnt + lu);
+        if (n < 0 || n > a.topk) {
+            if (lane == 0) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
+            n = n < 0 ? 0 : a.topk;
+        }
+        int carry = -1;  // the largest in-range entry so far
+        for (int e0 = 0; e0 < n; e0 += 32) {
+            const int e = e0 + lane;
+            const int t = e < n ? __ldg(a.idx + lu * a.topk + e) : -1;
+            const bool inr = t >= 0 && t <= qbj;
+            // exclusive prefix maximum of the in-range entries over the lanes
+            int pm = inr ? t : -1;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, pm, off);
+                if (lane >= off) pm = max(pm, y);
+            }
+            int before = __shfl_up_sync(0xffffffffu, pm, 1);
+            before = lane == 0 ? carry : max(before, carry);
+            const bool accept = inr && t > before;
+            if (e < n && t != -1 && !accept) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
+            if (accept) {
+                atomicOr(bm + j * W + (t >> 5), 1u << (t & 31));
+                hi = max(hi, t);
+            }
+            carry = max(carry, __shfl_sync(0xffffffffu, pm, 31));
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, off));
+    __syncwarp();
+    const int cap = list_cap(a.topk, kSub);
+    int* ul = sl + 1;
+    uint8_t* own = reinterpret_cast<uint8_t*>(sl + 1 + cap);
+    const int wn = hi >= 0 ? (hi >> 5) + 1 : 0;
+    int pos = 0;
+    for (int w0 = 0; w0 < wn; w0 += 32) {
+        const int w = w0 + lane;
+        uint32_t bj[kSub], u = 0u;
+#pragma unroll
+        for (int j = 0; j < kSub; ++j) {
+            bj[j] = w < wn ? bm[j * W + w] : 0u;
+            u |= bj[j];
+        }
+        const int c = __popc(u);
+        int incl = c;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += y;
+        }
+        int p = pos + incl - c;
+        while (u) {
+            const int bit = __ffs(u) - 1;
+            u &= u - 1;
+            uint32_t m = 0;
+#pragma unroll
+            for (int j = 0; j < kSub; ++j) m |= ((bj[j] >> bit) & 1u) << j;
+            ul[p] = 32 * w + bit;
+            own[p] = (uint8_t)m;
+            ++p;
+        }
+        pos += __shfl_sync(0xffffffffu, incl, 31);
+        if (w < wn)
+#pragma unroll
+            for (int j = 0; j < kSub; ++j) bm[j * W + w] = 0u;
+    }
+    if (lane == 0) sl[0] = pos;
+    __threadfence_block();
+    __syncwarp();
 }
 
 __device__ __forceinline__ uint32_t col_s(int buf) { return 128u + 64u * (uint32_t)buf; }
@@ -131,9 +245,11 @@ __device__ __forceinline__ void xchg_pieces(uint4& a0, uint4& a1, uint4& b0, uin
     }
 }
 
+template <int kSub>
 __global__ void __launch_bounds__(kThreads, 2)
 attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const FwdTcArgs a) {
+    constexpr int kBm = 64 / kSub;  // block size m: rows of one gathered block
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -141,7 +257,13 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
-    const int lsi = list_slot_ints(a.topk);
+    const int lsi = list_slot_ints(a.topk, kSub);
+    const int cap = list_cap(a.topk, kSub);
+    // the K/V block of slot q of tile j of a list slot (padding repeats the last)
+    auto tile_block = [&](const int* sl, int j, int q) {
+        const int n = sl[0], ui = j * kSub + q;
+        return sl[1 + (ui < n ? ui : n - 1)];
+    };
     auto slot_ptr = [&](int k) {
         return reinterpret_cast<int*>(smem + kOffList) + (k % kListSlots) * lsi;
     };
@@ -171,6 +293,10 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         fence_barrier_init();
         *abort_flag = 0;
     }
+    if constexpr (kSub > 1) {  // the union bitmaps start cleared (stage_union leaves them so)
+        uint32_t* bm = reinterpret_cast<uint32_t*>(smem + kOffList + (size_t)kListSlots * lsi * 4);
+        for (int i = threadIdx.x; i < kSub * bitmap_words(a.NQB); i += kThreads) bm[i] = 0u;
+    }
     if (warp == 5) {
         tmem_alloc(sb + kOffMisc, kTmemCols);
         tmem_relinquish();
@@ -182,52 +308,69 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
 
     if (warp == 4) {
         // ------------------------------------------------ lists and K tiles
-        if (lane == 0) {
-            prefetch_tmap(&tmK);
-            // unit k's compacted list into its slot, once every role is done with
-            // the slot's previous unit (k - kListSlots)
+        // At m = 64 lane 0 alone compacts each list; at m < 64 the whole warp builds
+        // the union, so every lane runs this loop and lane 0 issues the copies.
+        if (kSub > 1 || lane == 0) {
+            if (lane == 0) prefetch_tmap(&tmK);
+            uint32_t* bm = reinterpret_cast<uint32_t*>(smem + kOffList + (size_t)kListSlots * lsi * 4);
+            // unit k's list into its slot, once every role is done with the slot's
+            // previous unit (k - kListSlots)
             auto stage = [&](int k) {
                 const int ls = k % kListSlots;
-                if (k >= kListSlots &&
-                    !mbar_wait(bar(B_UFREE + ls), ((k / kListSlots) - 1) & 1, abort_flag, a.status))
-                    return false;
-                const FwdUnit d = fwd_unit(a, unit_of(k));
+                bool ok1 = k < kListSlots ||
+                           mbar_wait(bar(B_UFREE + ls), ((k / kListSlots) - 1) & 1, abort_flag, a.status);
+                if constexpr (kSub > 1) ok1 = __all_sync(0xffffffffu, ok1);
+                if (!ok1) return false;
+                const FwdUnit d = fwd_unit<kSub>(a, unit_of(k));
                 int* sl = slot_ptr(k);
-                sl[0] = compact_block_list(a.idx + d.lu * a.topk, a.cnt[d.lu], a.topk, d.qb, sl + 1,
-                                           a.status);
-                mbar_arrive(bar(B_UFULL + ls));
+                if constexpr (kSub == 1) {
+                    sl[0] = compact_block_list(a.idx + d.lu * a.topk, a.cnt[d.lu], a.topk, d.qb,
+                                               sl + 1, a.status);
+                } else {
+                    stage_union<kSub>(a, d, sl, bm, lane);
+                }
+                if (lane == 0) mbar_arrive(bar(B_UFULL + ls));
                 return true;
             };
             bool ok = unit_of(0) >= a.units || stage(0);
             int gk = 0;  // K loads issued, over all units
             for (int k = 0; ok && unit_of(k) < a.units; ++k) {
-                const FwdUnit d = fwd_unit(a, unit_of(k));
+                const FwdUnit d = fwd_unit<kSub>(a, unit_of(k));
                 const int* sl = slot_ptr(k);
-                const int n = sl[0];
+                const int nt = (sl[0] + kSub - 1) / kSub;  // 64-key tiles
                 bool staged = false;  // the next unit's list, once this unit's ring is full
-                for (int j = 0; j < n; ++j, ++gk) {
+                for (int j = 0; j < nt; ++j, ++gk) {
                     if (j == kSlots && unit_of(k + 1) < a.units) {
                         if (!(ok = stage(k + 1))) break;
                         staged = true;
                     }
                     const int s = gk % kSlots;
-                    if (gk >= kSlots &&
-                        !mbar_wait(bar(B_KEMPTY + s), ((gk / kSlots) - 1) & 1, abort_flag, a.status)) {
+                    bool okw = gk < kSlots ||
+                               mbar_wait(bar(B_KEMPTY + s), ((gk / kSlots) - 1) & 1, abort_flag, a.status);
+                    if constexpr (kSub > 1) okw = __all_sync(0xffffffffu, okw);
+                    if (!okw) {
                         ok = false;
                         break;
                     }
-                    mbar_expect_tx(bar(B_KFULL + s), kKBytes);
-                    for (int dh = 0; dh < 2; ++dh)
-                        tma_load_3d(sb + kOffK + s * kKBytes + dh * kKVHalf, &tmK, bar(B_KFULL + s),
-                                    dh * 64, sl[1 + j] * 64, d.bg);
+                    if (lane == 0) {
+                        mbar_expect_tx(bar(B_KFULL + s), kKBytes);
+#pragma unroll
+                        for (int q = 0; q < kSub; ++q) {
+                            const int blk = tile_block(sl, j, q);
+                            for (int dh = 0; dh < 2; ++dh)
+                                tma_load_3d(sb + kOffK + s * kKBytes + dh * kKVHalf + q * kBm * 128, &tmK,
+                                            bar(B_KFULL + s), dh * 64, blk * kBm, d.bg);
+                        }
+                    }
                 }
                 if (!ok) break;
                 if (!staged && unit_of(k + 1) < a.units) ok = stage(k + 1);
-                mbar_arrive(bar(B_UFREE + k % kListSlots));
+                if (lane == 0) mbar_arrive(bar(B_UFREE + k % kListSlots));
             }
             // Own copies must have landed before the CTA may exit.
-            for (int g = gk - kSlots; g < gk; ++g)
-                if (g >= 0) mbar_wait_drain(bar(B_KFULL + g % kSlots), (g / kSlots) & 1);
+            if (lane == 0)
+                for (int g = gk - kSlots; g < gk; ++g)
+                    if (g >= 0) mbar_wait_drain(bar(B_KFULL + g % kSlots), (g / kSlots) & 1);
         }
     } else if (warp == 6) {
         // ------------------------------------------------ Q and V tiles
@@ -237,11 +380,11 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             int gv = 0, q_last = -1;  // V loads issued; last unit whose Q was loaded
             bool ok = true;
             for (int k = 0; ok && unit_of(k) < a.units; ++k) {
-                const FwdUnit d = fwd_unit(a, unit_of(k));
+                const FwdUnit d = fwd_unit<kSub>(a, unit_of(k));
                 ok = mbar_wait(bar(B_UFULL + k % kListSlots), (k / kListSlots) & 1, abort_flag, a.status);
                 if (!ok) break;
                 const int* sl = slot_ptr(k);
-                const int n = sl[0];
+                const int n = (sl[0] + kSub - 1) / kSub;  // 64-key tiles
                 // Q once the previous unit's last QK MMA has read the old tile
                 if (k >= 1 && !mbar_wait(bar(B_QFREE), (k - 1) & 1, abort_flag, a.status)) {
                     ok = false;
@@ -261,9 +404,13 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                         break;
                     }
                     mbar_expect_tx(bar(B_VFULL + s), kKBytes);
-                    for (int dh = 0; dh < 2; ++dh)
-                        tma_load_3d(sb + kOffV + s * kKBytes + dh * kKVHalf, &tmV, bar(B_VFULL + s),
-                                    dh * 64, sl[1 + j] * 64, d.bg);
+#pragma unroll
+                    for (int q = 0; q < kSub; ++q) {
+                        const int blk = tile_block(sl, j, q);
+                        for (int dh = 0; dh < 2; ++dh)
+                            tma_load_3d(sb + kOffV + s * kKBytes + dh * kKVHalf + q * kBm * 128, &tmV,
+                                        bar(B_VFULL + s), dh * 64, blk * kBm, d.bg);
+                    }
                 }
                 if (!ok) break;
                 mbar_arrive(bar(B_UFREE + k % kListSlots));
@@ -285,7 +432,7 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             for (int k = 0; ok && unit_of(k) < a.units; ++k) {
                 ok = mbar_wait(bar(B_UFULL + k % kListSlots), (k / kListSlots) & 1, abort_flag, a.status);
                 if (!ok) break;
-                const int n = slot_ptr(k)[0];
+                const int n = (slot_ptr(k)[0] + kSub - 1) / kSub;  // 64-key tiles
                 mbar_arrive(bar(B_UFREE + k % kListSlots));  // only the count is needed here
                 ok = mbar_wait(bar(B_Q), k & 1, abort_flag, a.status);
                 if (!ok) break;
@@ -361,14 +508,18 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
         int g0 = 0;
         bool ok = true;
+        const int jr = tok / kBm, tb = tok % kBm;  // the row's query block in the span, position in it
         for (int k = 0; unit_of(k) < a.units; ++k) {
-            const FwdUnit d = fwd_unit(a, unit_of(k));
+            const FwdUnit d = fwd_unit<kSub>(a, unit_of(k));
             ok = ok && mbar_wait(bar(B_UFULL + k % kListSlots), (k / kListSlots) & 1, abort_flag, a.status);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             const int* sl = slot_ptr(k);
-            const int n = sl[0];
+            const int nu = sl[0];
+            const int n = (nu + kSub - 1) / kSub;  // 64-key tiles
             const int* list = sl + 1;
+            const uint8_t* own = reinterpret_cast<const uint8_t*>(sl + 1 + cap);
+            const int qb_r = d.qb * kSub + jr;  // the row's query block
             float m_used = -INFINITY, l = 0.f;
             for (int j = 0; j < n; ++j) {
                 const int g = g0 + j, buf = g & 1;
@@ -378,10 +529,31 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 tc_fence_after();
                 uint32_t sr[64];
                 tmem_ld64(lane_base + col_s(buf), sr);
-                if (list[j] == d.qb) {  // the query's own block: token-level causal mask
+                if constexpr (kSub == 1) {
+                    if (list[j] == d.qb) {  // the query's own block: token-level causal mask
 #pragma unroll
-                    for (int c = 0; c < 64; ++c)
-                        if (c > tok) sr[c] = __float_as_uint(-INFINITY);
+                        for (int c = 0; c < 64; ++c)
+                            if (c > tok) sr[c] = __float_as_uint(-INFINITY);
+                    }
+                } else {
+                    // slot q: attended if the row's query block selected its block; in
+                    // the row's own block, only keys at or before its token
+                    uint32_t full = 0u, part = 0u;
+#pragma unroll
+                    for (int q = 0; q < kSub; ++q) {
+                        const int ui = j * kSub + q;
+                        const bool sel = ui < nu && ((own[ui] >> jr) & 1u);
+                        if (sel && list[ui] != qb_r) full |= 1u << q;
+                        if (sel && list[ui] == qb_r) part |= 1u << q;
+                    }
+                    if (full != (1u << kSub) - 1u) {
+#pragma unroll
+                        for (int c = 0; c < 64; ++c) {
+                            const int q = c / kBm;
+                            const bool keep = ((full >> q) & 1u) || (((part >> q) & 1u) && c % kBm <= tb);
+                            if (!keep) sr[c] = __float_as_uint(-INFINITY);
+                        }
+                    }
                 }
                 // row max of the raw scores (the scale is positive), three-input maxima
                 float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
@@ -419,7 +591,10 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 // (2c, 2c+1), both read before entry c is overwritten.
                 float2 r2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
                 const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
-                const float2 nm2 = make_float2(-m_used, -m_used);
+                // a row with no attended key so far (m_used = -inf) has only masked
+                // scores here: 2^(-inf) = 0 with a zero offset
+                const float nm = m_used == -INFINITY ? 0.f : -m_used;
+                const float2 nm2 = make_float2(nm, nm);
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
                     float2 p2 = __ffma2_rn(make_float2(__uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1])), sc2, nm2);
@@ -496,21 +671,27 @@ attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
 
 }  // namespace
 
+size_t attn_fwd_tc_smem_bytes(const phsa_shape& s, int topk) {
+    const int bm = s.block_size;
+    return fwd_tc_smem(topk, 64 / bm, (s.L + bm - 1) / bm);
+}
+
 cudaError_t launch_attn_fwd_tc(const void* Q, const void* K, const void* V, const int32_t* idx,
                                const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                                void* O, float* lse, int* status, cudaStream_t st) {
-    const int NQB = (s.L + 63) / 64;
+    const int bm = s.block_size, kSub = 64 / bm;
+    const int NQB = (s.L + bm - 1) / bm, nsb = (s.L + 63) / 64;
     CUtensorMap tq, tk, tv;
     if (!make_tmap_bf16_rows128(&tq, Q, s.L, (uint64_t)s.B * s.Hq, 64) ||
-        !make_tmap_bf16_rows128(&tk, K, s.L, (uint64_t)s.B * s.Hkv, 64) ||
-        !make_tmap_bf16_rows128(&tv, V, s.L, (uint64_t)s.B * s.Hkv, 64))
+        !make_tmap_bf16_rows128(&tk, K, s.L, (uint64_t)s.B * s.Hkv, (uint32_t)bm) ||
+        !make_tmap_bf16_rows128(&tv, V, s.L, (uint64_t)s.B * s.Hkv, (uint32_t)bm))
         return cudaErrorInvalidValue;
-    const size_t smem = fwd_tc_smem(topk);
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_tc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const size_t smem = fwd_tc_smem(topk, kSub, NQB);
+    auto kern = kSub == 1 ? attn_fwd_tc_kernel<1> : kSub == 2 ? attn_fwd_tc_kernel<2> : attn_fwd_tc_kernel<4>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    if ((e = cudaFuncSetAttribute(attn_fwd_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                  100)) != cudaSuccess)
+    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100)) !=
+        cudaSuccess)
         return e;
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -518,13 +699,13 @@ cudaError_t launch_attn_fwd_tc(const void* Q, const void* K, const void* V, cons
         return e;
     // Two CTAs per SM (shared memory and registers are sized for it); CTAs never
     // wait on one another, so the grid is correct whatever number is resident.
-    const long long units = (long long)s.B * s.Hkv * NQB;
+    const long long units = (long long)s.B * s.Hkv * nsb;
     const long long cap = 2LL * nsm;
     const unsigned grid = (unsigned)(units < cap ? units : cap);
     FwdTcArgs args{idx, cnt, static_cast<__nv_bfloat16*>(O), lse, status, s.Hq, s.Hkv, s.L, NQB,
-                   topk, (int)units, sm_scale * kLog2e};
+                   topk, (int)units, nsb, sm_scale * kLog2e};
     ProfScope prof(K_FWD, st);
-    attn_fwd_tc_kernel<<<grid, kThreads, smem, st>>>(tq, tk, tv, args);
+    kern<<<grid, kThreads, smem, st>>>(tq, tk, tv, args);
     return cudaGetLastError();
 }
 

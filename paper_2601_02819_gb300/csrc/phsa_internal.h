@@ -79,7 +79,9 @@ cudaError_t launch_select_blocks(const void* Q, const void* Krepr, const phsa_sh
                                  const phsa_select_params& p, int32_t* idx, int32_t* cnt,
                                  int* status, cudaStream_t st);
 
-// tcgen05 forward for G = 2 (attn_fwd_tc.cu); launch_attn_fwd dispatches to it.
+// tcgen05 forward for G = 2 at block sizes 64, 32, 16 (attn_fwd_tc.cu);
+// launch_attn_fwd dispatches to it while its shared memory fits.
+size_t attn_fwd_tc_smem_bytes(const phsa_shape& s, int topk);
 cudaError_t launch_attn_fwd_tc(const void* Q, const void* K, const void* V, const int32_t* idx,
                                const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
                                void* O, float* lse, int* status, cudaStream_t st);
