@@ -422,7 +422,7 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                         if (t0 + 32 * q > c_hi) break;  // no candidate left in this group (warp-uniform)
                         uint32_t v[32];
                         tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
-                        // max of the raw scores, then the scale (positive) once
+                        // max of the raw scores (three-input maxima), then the scale (positive) once
                         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
                         if (!full) {
 #pragma unroll
@@ -430,16 +430,23 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                                 if (t0 + 32 * q + j > c_hi_r) v[j] = __float_as_uint(-INFINITY);
                         }
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) m4[j & 3] = fmaxf(m4[j & 3], __uint_as_float(v[j]));
+                        for (int j = 0; j < 32; j += 2)
+                            m4[(j >> 1) & 3] = fmax3(m4[(j >> 1) & 3], __uint_as_float(v[j]), __uint_as_float(v[j + 1]));
                         const float mn = fmaxf(m, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2);
                         if (mn != -INFINITY) {
-                            float s4[4] = {0.f, 0.f, 0.f, 0.f};
-                            const float neg = -mn;
+                            // packed: two scores per FFMA2 and FADD2, one SFU op each
+                            const float2 cc = make_float2(a.scale_log2, a.scale_log2), nn = make_float2(-mn, -mn);
+                            float2 s2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
-                            for (int j = 0; j < 32; ++j)
-                                s4[j & 3] += ex2_approx(fmaf(__uint_as_float(v[j]), a.scale_log2, neg));
+                            for (int j = 0; j < 32; j += 2) {
+                                float2 e = __ffma2_rn(make_float2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), cc, nn);
+                                e.x = ex2_approx(e.x);
+                                e.y = ex2_approx(e.y);
+                                s2[(j >> 1) & 1] = __fadd2_rn(s2[(j >> 1) & 1], e);
+                            }
                             if (mn > m) z *= ex2_approx(m - mn);  // the running max moved
-                            z += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+                            const float2 st = __fadd2_rn(s2[0], s2[1]);
+                            z += st.x + st.y;
                             m = mn;
                         }
                     }
@@ -533,25 +540,34 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                     // a warp whose 32 candidates all lie past the last one skips the work
                     // p = 2^(S*scale - m_r - log2 Z_r): the row's max and sum in one offset
                     const float* mrow = m2s + 64 * hh;
-                    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                    float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
                     const bool live = c * kCand + (warp & 3) * 32 < nC;
+                    const float2 cc = make_float2(a.scale_log2, a.scale_log2);
 #pragma unroll 1
                     for (int q = 0; q < (live ? 2 : 0); ++q) {
-                        uint32_t v[32];
-                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, v);
+                        uint32_t vq[32];
+                        tmem_ld32(lane_base + 128u * slot + 64 * hh + 32 * q, vq);
 #pragma unroll
                         for (int j = 0; j < 32; j += 4) {
+                            // -(m_r + log2 Z_r) of four rows, two per packed FFMA2
                             const float4 mm = *reinterpret_cast<const float4*>(mrow + 32 * q + j);
-                            acc[0] += ex2_approx(fmaf(__uint_as_float(v[j + 0]), a.scale_log2, -mm.x));
-                            acc[1] += ex2_approx(fmaf(__uint_as_float(v[j + 1]), a.scale_log2, -mm.y));
-                            acc[2] += ex2_approx(fmaf(__uint_as_float(v[j + 2]), a.scale_log2, -mm.z));
-                            acc[3] += ex2_approx(fmaf(__uint_as_float(v[j + 3]), a.scale_log2, -mm.w));
+                            float2 e0 = __ffma2_rn(make_float2(__uint_as_float(vq[j]), __uint_as_float(vq[j + 1])), cc,
+                                                   make_float2(-mm.x, -mm.y));
+                            float2 e1 = __ffma2_rn(make_float2(__uint_as_float(vq[j + 2]), __uint_as_float(vq[j + 3])), cc,
+                                                   make_float2(-mm.z, -mm.w));
+                            e0.x = ex2_approx(e0.x);
+                            e0.y = ex2_approx(e0.y);
+                            e1.x = ex2_approx(e1.x);
+                            e1.y = ex2_approx(e1.y);
+                            acc[0] = __fadd2_rn(acc[0], e0);
+                            acc[1] = __fadd2_rn(acc[1], e1);
                         }
                     }
                     tc_fence_before();
                     mbar_arrive(bar(B_SFREE + slot));
                     const int cj = c * kCand + r;
-                    if (cj < nC) (hh ? A1 : A0)[cj] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+                    const float2 sacc = __fadd2_rn(acc[0], acc[1]);
+                    if (cj < nC) (hh ? A1 : A0)[cj] = sacc.x + sacc.y;
                 }
                 if (!kMaxLogit && s == nch - 1) {
                     // merge the two column halves of every row: (m, z) -> max and 1/sum
