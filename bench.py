@@ -773,6 +773,91 @@ def run_decode(args):
     }
 
 
+# ---------------------------------------------------------------- chunked prefill
+def run_chunked(args):
+    """Prefill of the workload's K, V and punctuation flags into caches in chunks
+    of args.chunked tokens through phsa_prefill_append (the representative keys
+    of completed blocks from the same loads), against the same chunks copied in
+    followed by one phsa_build_block_repr over the cache."""
+    from paper_2601_02819_gb300 import phsa
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    w = workload_of(args, inputs.WORKLOADS)
+    if w.block_size != 64:
+        raise SystemExit("--chunked runs at block size 64")
+    x = inputs.make_inputs(w, with_grad=False, seed=w.seed)
+    bf = lambda a: torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
+    Ksrc, Vsrc = bf(x["K"]), bf(x["V"])
+    msrc = torch.from_numpy(x["mask"]).to(dev)
+    C = args.chunked
+    starts = list(range(0, w.L, C))
+    chunks = [(Ksrc[:, :, p:p + C].contiguous(), Vsrc[:, :, p:p + C].contiguous(),
+               msrc[:, p:p + C].contiguous(), torch.full((w.B,), min(p + C, w.L), dtype=torch.int32, device=dev))
+              for p in starts]
+    K, V = torch.empty_like(Ksrc), torch.empty_like(Vsrc)
+    mask = torch.empty_like(msrc)
+    Kr = torch.empty((w.B, w.Hkv, w.T, w.D), dtype=torch.bfloat16, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def fused():
+        for kc, vc, fc, ln in chunks:
+            phsa.phsa_prefill_append(kc, vc, ln, K, V, mask, Kr, w.lam, flag_chunk=fc)
+
+    def unfused():
+        for (kc, vc, fc, ln), p in zip(chunks, starts):
+            n = kc.shape[2]
+            K[:, :, p:p + n].copy_(kc)
+            V[:, :, p:p + n].copy_(vc)
+            mask[:, p:p + n].copy_(fc)
+        phsa.phsa_build_block_repr(K, mask, w.lam, Krepr=Kr)
+
+    def timed(fn):
+        for _ in range(args.warmup):
+            flush.zero_()
+            fn()
+        ts = []
+        for _ in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return statistics.median(ts)
+
+    ms_f = timed(fused)
+    assert phsa.phsa_get_device_status() == 0
+    Kr_f = Kr.clone()
+    ms_u = timed(unfused)
+    same = bool(torch.equal(Kr_f.view(torch.int16), Kr.view(torch.int16)))
+    peaks, peak_src = load_peaks()
+    kv = w.B * w.Hkv * w.L * w.D * 2
+    # algorithmic bytes of the fused path: chunks read, caches written, flags,
+    # keys written, and the earlier rows of each block a chunk finishes (the
+    # part of the block before the chunk, when C is not a multiple of 64)
+    head = sum(p % 64 for p in starts[1:]) * w.B * w.Hkv * w.D * 2
+    nbytes = 4 * kv + 2 * w.B * w.L + w.B * w.Hkv * w.T * w.D * 2 + head
+    return {
+        "metric": "chunked prefill into the KV caches with fused representative keys, GB/s",
+        "value": nbytes / (ms_f / 1e3) / 1e9, "unit": "GB/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_f, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "L": w.L, "Hkv": w.Hkv, "D": w.D,
+                   "chunk": C, "chunks": len(starts),
+                   "step": "the whole sequence appended chunk by chunk (phsa_prefill_append)",
+                   "l2": "flushed before every timed pass (256 MB written)"},
+        "bytes_per_step": nbytes, "bytes_per_chunk": nbytes / len(starts),
+        "hbm_frac": round(nbytes / (ms_f / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
+        "unfused_ms": round(ms_u, 4),
+        "unfused_note": "the same chunks copied into the caches, then phsa_build_block_repr",
+        "keys_bit_identical": same,
+        "gpu_launches": len(starts),
+        "peaks": {"source": peak_src, "hbm_gbs": peaks["hbm_gbs"]},
+    }
+
+
 # ---------------------------------------------------------------- reference arm
 def run_reference(args):
     rank, world, _ = dist_env()
@@ -825,6 +910,8 @@ def main():
                     help="how a unit's query rows are combined per candidate block")
     ap.add_argument("--forced", choices=["workload", "paper"], default="workload",
                     help="forced blocks: the workload's, or the paper's 2 initial + 8 local")
+    ap.add_argument("--chunked", type=int, default=0,
+                    help="time a chunked prefill of the workload's keys (chunk length) instead")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-units", type=int, default=48,
@@ -834,7 +921,9 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
-    if args.workload in inputs.DECODE_WORKLOADS:
+    if args.chunked > 0:
+        out = run_chunked(args)
+    elif args.workload in inputs.DECODE_WORKLOADS:
         if args.impl == "reference":
             raise SystemExit("--impl reference times the prefill workloads only")
         out = run_decode(args)

@@ -325,6 +325,34 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
                      void* stream);
 
 /*
+ * Prefill in chunks (block-level caching of Section 3.2; Eq. 3, 6, 7, 8;
+ * Algorithm 1 step 2): appends a chunk of C = chunk_len tokens to every
+ * sequence's caches and, from the same loads, computes the representative key
+ * of every block of m = 64 tokens that the chunk completes, so a prefill does
+ * not read K a second time for stage (a). With len = seq_lens[b] (the length
+ * after the append, chunk included), the chunk takes positions
+ * p = len - C + i, i in [0, C):
+ *   K[b][g][p] = k_chunk[b][g][i], V[b][g][p] = v_chunk[b][g][i] for every
+ *   KV head g, punct_mask[b][p] = flag_chunk[b][i] (when flag_chunk is given;
+ *   otherwise the mask already holds the chunk's flags), and for every block t
+ *   with len - C < (t + 1) m <= len, Krepr[b][g][t] = lambda M0 + (1 - lambda)
+ *   Mp (Mp = M0 without punctuation), Eq. 6-8 over the block's m keys and
+ *   flags, earlier ones read from the caches. The keys equal, bit for bit,
+ *   those phsa_build_block_repr computes over the finished cache. Blocks the
+ *   chunk leaves partial get no key yet.
+ *   k_chunk, v_chunk bf16 [B, Hkv, C, D] in;  flag_chunk uint8 [B, C] in or NULL
+ *   seq_lens int32 [B] in (device); s.L is the cache capacity, s.block_size 64
+ *   K, V bf16 [B, Hkv, L, D], punct_mask uint8 [B, L], Krepr bf16
+ *   [B, Hkv, floor(L/64), D]: in/out (device, caller-owned)
+ * A length with len < C or len > L is a device-side error
+ * (PHSA_ERR_DEVICE_INDEX) and that sequence is left untouched. chunk_len = 0
+ * does nothing.
+ */
+int phsa_prefill_append(const void* k_chunk, const void* v_chunk, const uint8_t* flag_chunk,
+                        const int32_t* seq_lens, int chunk_len, phsa_shape s, float lambda,
+                        void* K, void* V, uint8_t* punct_mask, void* Krepr, void* stream);
+
+/*
  * Synchronises `stream`, returns the device status word of the current
  * device (PHSA_OK or the first device-side error code recorded since the
  * last call) and clears it. Returns PHSA_ERR_CUDA if the synchronisation

@@ -263,6 +263,27 @@ int phsa_decode_append(const void* k_new, const void* v_new, const uint8_t* flag
                                                 static_cast<cudaStream_t>(stream)));
 }
 
+int phsa_prefill_append(const void* k_chunk, const void* v_chunk, const uint8_t* flag_chunk,
+                        const int32_t* seq_lens, int chunk_len, phsa_shape s, float lambda,
+                        void* K, void* V, uint8_t* punct_mask, void* Krepr, void* stream) {
+    int rc = check_shape(s);
+    if (rc != PHSA_OK) return rc;
+    if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
+    if (chunk_len < 0 || chunk_len > s.L) return PHSA_ERR_INVALID_ARG;
+    if (s.B == 0 || chunk_len == 0) return PHSA_OK;
+    if (!k_chunk || !v_chunk || !seq_lens || !K || !V || !punct_mask ||
+        (s.L >= phsa::kM && !Krepr))
+        return PHSA_ERR_INVALID_ARG;
+    if (!aligned16(k_chunk) || !aligned16(v_chunk) || !aligned16(K) || !aligned16(V) ||
+        (Krepr && !aligned16(Krepr)))
+        return PHSA_ERR_INVALID_ARG;
+    int* st = status_ptr();
+    if (!st) return PHSA_ERR_CUDA;
+    return from_cuda(phsa::launch_prefill_append(k_chunk, v_chunk, flag_chunk, seq_lens, chunk_len,
+                                                 s, lambda, K, V, punct_mask, Krepr, st,
+                                                 static_cast<cudaStream_t>(stream)));
+}
+
 int phsa_get_device_status(void* stream) {
     if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
         return PHSA_ERR_CUDA;

@@ -18,7 +18,7 @@ constexpr size_t kMaxDynSmem = 227u * 1024u;
 // Kernel identities for the optional per-kernel timing (profile.cu).
 enum KernelId {
     K_REPR = 0, K_SELECT, K_FWD, K_BWD_DELTA, K_BWD_MARK, K_BWD_BUILD, K_BWD_DKDV,
-    K_BWD_DKDV_SUM, K_BWD_DQ, K_DEC_REPR, K_DEC_SELECT, K_DEC_ATTN, K_COUNT
+    K_BWD_DKDV_SUM, K_BWD_DQ, K_DEC_REPR, K_DEC_SELECT, K_DEC_ATTN, K_PREFILL_APPEND, K_COUNT
 };
 void prof_begin(int kid, cudaStream_t st);
 void prof_end(int kid, cudaStream_t st);
@@ -59,6 +59,13 @@ size_t decode_attn_smem_bytes(const phsa_shape& s, int topk);
 cudaError_t launch_decode_append(const void* k_new, const void* v_new, const uint8_t* flag,
                                  const int32_t* lens, const phsa_shape& s, void* K, void* V,
                                  uint8_t* mask, int* status, cudaStream_t st);
+// Writes a chunk of C tokens (k, v, punctuation flags) at positions
+// [len - C, len) of every sequence and the representative key of every block
+// the chunk completes (prefill_append.cu).
+cudaError_t launch_prefill_append(const void* k_chunk, const void* v_chunk, const uint8_t* flags,
+                                  const int32_t* lens, int C, const phsa_shape& s, float lambda,
+                                  void* K, void* V, uint8_t* mask, void* Krepr, int* status,
+                                  cudaStream_t st);
 // Punctuation indicator of token ids against a set of <= 4096 ids (punct.cu).
 cudaError_t launch_punct_mask(const int32_t* ids, long long n, const int32_t* punct_ids,
                               int n_punct, uint8_t* mask, cudaStream_t st);

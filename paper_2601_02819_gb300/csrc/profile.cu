@@ -15,7 +15,7 @@ namespace {
 const char* const kNames[K_COUNT] = {
     "block_repr", "select_blocks", "attn_fwd", "bwd_delta", "bwd_idx_mark",
     "bwd_idx_build", "bwd_dkdv", "bwd_dkdv_sum", "bwd_dq", "decode_repr", "decode_select",
-    "decode_attn",
+    "decode_attn", "prefill_append",
 };
 
 struct Record {

@@ -104,6 +104,8 @@ def _declare(L):
     L.phsa_punct_mask.argtypes = [P, ctypes.c_int64, P, I, P, P]
     L.phsa_decode_select.argtypes = [P, P, P, phsa_shape, phsa_select_params, P, P, P]
     L.phsa_decode_attn.argtypes = [P, P, P, P, P, P, phsa_shape, I, F, P, P, P]
+    L.phsa_prefill_append.argtypes = [P, P, P, P, I, phsa_shape, F, P, P, P, P, P]
+    L.phsa_prefill_append.restype = I
     L.phsa_test_set_select_tc_limit.argtypes = [SZ]
     L.phsa_test_set_select_tc_limit.restype = SZ
     for fn in ("phsa_decode_update_repr", "phsa_decode_select", "phsa_decode_attn",
@@ -396,6 +398,40 @@ def phsa_decode_append(k_new, v_new, seq_lens, K, V, flag_new=None, punct_mask=N
                                    _ptr(punct_mask), _stream(stream))
     _raise("phsa_decode_append", rc)
     return K, V
+
+
+def phsa_prefill_append(k_chunk, v_chunk, seq_lens, K, V, punct_mask, Krepr, lam: float,
+                        flag_chunk=None, stream=None):
+    """Append a chunk of C tokens to every sequence's caches (positions
+    seq_lens[b] - C .. seq_lens[b] - 1, seq_lens counting the chunk) and write
+    the representative key of every block of 64 the chunk completes, from the
+    same loads: k_chunk/v_chunk [B, Hkv, C, D] bf16 into K/V [B, Hkv, Lc, D],
+    flag_chunk [B, C] uint8 (optional) into punct_mask [B, Lc], keys into
+    Krepr [B, Hkv, Lc // 64, D]."""
+    _check(k_chunk, "k_chunk", torch.bfloat16, 4)
+    _check(v_chunk, "v_chunk", torch.bfloat16, 4)
+    _check(seq_lens, "seq_lens", torch.int32, 1)
+    _check(K, "K", torch.bfloat16, 4)
+    _check(V, "V", torch.bfloat16, 4)
+    _check(punct_mask, "punct_mask", torch.uint8, 2)
+    _check(Krepr, "Krepr", torch.bfloat16, 4)
+    B, Hkv, Lc, D = K.shape
+    C = k_chunk.shape[2]
+    if tuple(V.shape) != tuple(K.shape) or tuple(k_chunk.shape) != (B, Hkv, C, D) or \
+            tuple(v_chunk.shape) != (B, Hkv, C, D) or tuple(seq_lens.shape) != (B,) or \
+            tuple(punct_mask.shape) != (B, Lc) or tuple(Krepr.shape) != (B, Hkv, Lc // BLOCK_SIZE, D):
+        raise ValueError("k_chunk/v_chunk must be [B, Hkv, C, D], K/V [B, Hkv, Lc, D], "
+                         "seq_lens [B], punct_mask [B, Lc], Krepr [B, Hkv, Lc // 64, D]")
+    if flag_chunk is not None:
+        _check(flag_chunk, "flag_chunk", torch.uint8, 2)
+        if tuple(flag_chunk.shape) != (B, C):
+            raise ValueError("flag_chunk must be [B, C]")
+    rc = load().phsa_prefill_append(_ptr(k_chunk), _ptr(v_chunk), _ptr(flag_chunk),
+                                    _ptr(seq_lens), int(C), make_shape(B, Lc, Hkv, Hkv, D),
+                                    float(lam), _ptr(K), _ptr(V), _ptr(punct_mask), _ptr(Krepr),
+                                    _stream(stream))
+    _raise("phsa_prefill_append", rc)
+    return K, V, Krepr
 
 
 def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=None):

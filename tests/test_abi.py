@@ -136,3 +136,20 @@ def test_punct_mask_and_append_validation_needs_no_gpu(lib):
     assert lib.phsa_decode_append(odd, dummy, None, dummy, ok, dummy, dummy, None, None) == -1
     assert lib.phsa_decode_append(None, None, None, None, phsa_shape(0, 256, 8, 8, 128, 64),
                                   None, None, None, None) == 0  # empty batch
+
+
+def test_prefill_append_validation_needs_no_gpu(lib):
+    from paper_2601_02819_gb300.phsa import phsa_shape
+    P, I, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    lib.phsa_prefill_append.argtypes = [P, P, P, P, I, phsa_shape, F, P, P, P, P, P]
+    ok = phsa_shape(2, 512, 4, 2, 128, 64)
+    f = lib.phsa_prefill_append
+    assert f(None, None, None, None, 0, ok, 0.5, None, None, None, None, None) == 0   # empty chunk
+    assert f(None, None, None, None, 16, ok, 1.5, None, None, None, None, None) == -1  # lambda > 1
+    assert f(None, None, None, None, -1, ok, 0.5, None, None, None, None, None) == -1  # C < 0
+    assert f(None, None, None, None, 513, ok, 0.5, None, None, None, None, None) == -1  # C > L
+    assert f(None, None, None, None, 16, ok, 0.5, None, None, None, None, None) == -1  # null pointers
+    m16 = phsa_shape(2, 512, 4, 2, 128, 16)
+    assert f(None, None, None, None, 16, m16, 0.5, None, None, None, None, None) == -2  # m = 64 only
+    d64 = phsa_shape(2, 512, 4, 2, 64, 64)
+    assert f(None, None, None, None, 16, d64, 0.5, None, None, None, None, None) == -2  # D = 128 only
