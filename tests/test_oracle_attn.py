@@ -143,10 +143,10 @@ def test_block_order_does_not_matter():
     np.testing.assert_allclose(lse, lse2, rtol=0, atol=1e-12)
 
 
-@pytest.mark.parametrize("L,topk", [(64 * 5, 3), (64 * 4 + 9, 2)])
-def test_backward_matches_torch_autograd_fp64(L, topk):
-    rng = np.random.default_rng(15)
-    m = 64
+@pytest.mark.parametrize("L,topk,m", [(64 * 5, 3, 64), (64 * 4 + 9, 2, 64), (16 * 13 + 5, 5, 16),
+                                      (16 * 9, 9, 16), (32 * 7 + 3, 3, 32)])
+def test_backward_matches_torch_autograd_fp64(L, topk, m):
+    rng = np.random.default_rng(15 + m)
     Q, K, V = rand_qkv(rng, 1, 4, 2, L)
     dO = bf(rng.standard_normal(Q.shape))
     idx, cnt = random_selection(rng, 1, 2, L, m, topk)
@@ -157,11 +157,11 @@ def test_backward_matches_torch_autograd_fp64(L, topk):
     np.testing.assert_allclose(dV, tv, rtol=0, atol=1e-11)
 
 
-def test_backward_invariants():
+@pytest.mark.parametrize("L,m", [(64 * 6 + 5, 64), (16 * 20 + 7, 16)])
+def test_backward_invariants(L, m):
     # Softmax rows sum to one, so sum_j dV_j = sum_i dO_i (per KV head, over its query
     # heads), and the dS of each row sums to zero, so sum_j dK_j = 0.
-    rng = np.random.default_rng(16)
-    L, m = 64 * 6 + 5, 64
+    rng = np.random.default_rng(16 + m)
     Q, K, V = rand_qkv(rng, 2, 4, 2, L)
     dO = bf(rng.standard_normal(Q.shape))
     idx, cnt = random_selection(rng, 2, 2, L, m, 3)
