@@ -21,6 +21,7 @@
 // Every sum runs in a fixed order, so results are bit-reproducible.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
+#include "union.cuh"
 
 namespace phsa {
 
@@ -56,9 +57,15 @@ delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restric
 }
 
 // ---------------------------------------------------------------- index transpose
+// Rows of the transposed selection are KV spans of 64 keys (kSub = 64/m blocks
+// each; one block at m = 64), columns are query blocks of m tokens. At m < 64
+// each (span, query block) pair also records which of the span's kSub blocks
+// the query block selected: kSub bits at bit (qb * kSub) % 32 of word
+// (qb * kSub) / 32 of the span's mask row.
 __global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt,
-                                long long units, int NQB, int topk, int words,
-                                uint32_t* __restrict__ bits, int* status) {
+                                long long units, int NQB, int nrows, int kSub, int topk, int words,
+                                int mwords, uint32_t* __restrict__ bits, uint32_t* __restrict__ masks,
+                                int* status) {
     const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (u >= units) return;
     const int qb = (int)(u % NQB);
@@ -77,7 +84,11 @@ __global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* 
             continue;
         }
         prev = t;
-        atomicOr(&bits[(bg * NQB + t) * words + (qb >> 5)], 1u << (qb & 31));
+        const int T = t / kSub;
+        atomicOr(&bits[(bg * nrows + T) * words + (qb >> 5)], 1u << (qb & 31));
+        if (kSub > 1)
+            atomicOr(&masks[(bg * nrows + T) * mwords + ((qb * kSub) >> 5)],
+                     (1u << (t - T * kSub)) << ((qb * kSub) & 31));
     }
 }
 
@@ -110,18 +121,22 @@ __device__ int block_excl_scan(int v, int* tmp, int& total) {
     return before;
 }
 
+// One CTA per (b, g): the ascending query-block list of every row (KV span),
+// cut into work items of at most kChunk iterations of kSub query blocks each.
 __global__ void __launch_bounds__(1024)
-idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words, int work_max,
-                 int slot_max, TInfo* __restrict__ tinfo, int32_t* __restrict__ qlist,
-                 int2* __restrict__ work, int32_t* __restrict__ nwork, int* __restrict__ arrive,
-                 int2* __restrict__ queue, int* __restrict__ qcount, int* status) {
+idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub, int topk,
+                 int words, int work_max, int slot_max, TInfo* __restrict__ tinfo,
+                 int32_t* __restrict__ qlist, int2* __restrict__ work, int32_t* __restrict__ nwork,
+                 int* __restrict__ arrive, int2* __restrict__ queue, int* __restrict__ qcount,
+                 int* status) {
     __shared__ int tmp[32];
     __shared__ int bin[kChunk + 1];  // items per iteration count, then queue cursors
-    __shared__ int ncache[kBuildCache];  // selecting-query count of each KV block
+    __shared__ int ncache[kBuildCache];  // selecting-query count of each KV span
     const int bg = blockIdx.x;
-    const int per = (NQB + 1023) / 1024;  // KV blocks counted by each thread
+    const int kChunkQ = kChunk * kSub;  // query blocks per work item
+    const int per = (nrows + 1023) / 1024;  // KV spans counted by each thread
     const int t0 = threadIdx.x * per;
-    const uint32_t* bb = bits + (size_t)bg * NQB * words;
+    const uint32_t* bb = bits + (size_t)bg * nrows * words;
     // The count of a block: its bitmap row's popcount, read with independent
     // loads. The first kBuildCache blocks keep theirs in shared memory for the
     // later passes (each thread reads back only its own entries); any block
@@ -136,15 +151,15 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     auto count_of = [&](int t) { return t < kBuildCache ? ncache[t] : count_row(t); };
     for (int k = 0; k < per; ++k) {
         const int t = t0 + k;
-        if (t >= NQB) break;
+        if (t >= nrows) break;
         if (t < kBuildCache) ncache[t] = count_row(t);
     }
     int sn = 0, sch = 0, ssl = 0;
     for (int k = 0; k < per; ++k) {
         const int t = t0 + k;
-        if (t >= NQB) break;
+        if (t >= nrows) break;
         const int n = count_of(t);
-        const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
+        const int nch = n <= kChunkQ ? 1 : (n + kChunkQ - 1) / kChunkQ;
         sn += n;
         sch += nch;
         ssl += nch > 1 ? nch : 0;
@@ -163,11 +178,11 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     // each class's queue for this (b, g), sorted by iteration count, descending
     for (int k = 0, ch = och; k < per; ++k) {
         const int t = t0 + k;
-        if (t >= NQB) break;
+        if (t >= nrows) break;
         const int n = count_of(t);
-        const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
+        const int nch = n <= kChunkQ ? 1 : (n + kChunkQ - 1) / kChunkQ;
         for (int c = 0; c < nch && ch + c < work_max; ++c)
-            atomicAdd(&bin[min(n, kChunk * c + kChunk) - kChunk * c], 1);
+            atomicAdd(&bin[(min(n, kChunkQ * c + kChunkQ) - kChunkQ * c + kSub - 1) / kSub], 1);
         ch += nch;
     }
     __syncthreads();
@@ -184,24 +199,24 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     }
     __syncthreads();
     const size_t qcap = (size_t)gridDim.x * work_max;
-    TInfo* ti = tinfo + (size_t)bg * NQB;
+    TInfo* ti = tinfo + (size_t)bg * nrows;
     int2* wk = work + (size_t)bg * work_max;
     for (int k = 0; k < per; ++k) {
         const int t = t0 + k;
-        if (t >= NQB) break;
+        if (t >= nrows) break;
         const int n = count_of(t);
-        const int nch = n <= kChunk ? 1 : (n + kChunk - 1) / kChunk;
+        const int nch = n <= kChunkQ ? 1 : (n + kChunkQ - 1) / kChunkQ;
         TInfo info;
         info.off = on;
         info.n = n;
         info.nch = nch;
         info.slot = (nch > 1 && osl + nch <= slot_max) ? osl : -1;
         ti[t] = info;
-        arrive[(size_t)bg * NQB + t] = 0;
+        arrive[(size_t)bg * nrows + t] = 0;
         for (int c = 0; c < nch && och + c < work_max; ++c) {
             wk[och + c] = make_int2(t, c);
-            const int n_it = min(n, kChunk * c + kChunk) - kChunk * c;
-            queue[queue_class(n_it) * qcap + atomicAdd(&bin[n_it], 1)] = make_int2(bg * NQB + t, c);
+            const int n_it = (min(n, kChunkQ * c + kChunkQ) - kChunkQ * c + kSub - 1) / kSub;
+            queue[queue_class(n_it) * qcap + atomicAdd(&bin[n_it], 1)] = make_int2(bg * nrows + t, c);
         }
         on += n;
         och += nch;
@@ -215,12 +230,12 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
     int32_t* ql = qlist + (size_t)bg * NQB * topk;
     const int cap = NQB * topk;
     constexpr int kBatch = 8;
-    for (int tb = warp; tb < NQB; tb += 32 * kBatch) {
+    for (int tb = warp; tb < nrows; tb += 32 * kBatch) {
         int pos[kBatch];
 #pragma unroll
         for (int j = 0; j < kBatch; ++j) {
             const int t = tb + 32 * j;
-            pos[j] = t < NQB ? ti[t].off : 0;
+            pos[j] = t < nrows ? ti[t].off : 0;
         }
         for (int w0 = 0; w0 < words; w0 += 32) {
             const int w = w0 + lane;
@@ -228,7 +243,7 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int topk, int words
 #pragma unroll
             for (int j = 0; j < kBatch; ++j) {
                 const int t = tb + 32 * j;
-                m[j] = (t < NQB && w < words) ? bb[(size_t)t * words + w] : 0u;
+                m[j] = (t < nrows && w < words) ? bb[(size_t)t * words + w] : 0u;
             }
 #pragma unroll
             for (int j = 0; j < kBatch; ++j) {
@@ -655,26 +670,58 @@ cudaError_t launch_dq_g(const void* Q, const void* K, const void* V, const void*
 
 BwdLayout bwd_layout(const phsa_shape& s, int topk) {
     BwdLayout l{};
-    l.nqb = (s.L + kM - 1) / kM;
+    const int bm = s.block_size;
+    l.kSub = kM / bm;
+    l.nqb = (s.L + bm - 1) / bm;
+    l.nrows = (s.L + kM - 1) / kM;
     l.words = (l.nqb + 31) / 32;
-    l.chunk = kChunk;
+    l.mwords = l.kSub > 1 ? (l.nqb * l.kSub + 31) / 32 : 0;
+    l.chunk = kChunk * l.kSub;  // query blocks per dK/dV work item
+    l.ucap = l.kSub * topk;
     const long long bgs = (long long)s.B * s.Hkv;
     const long long nnz_max = (long long)l.nqb * topk;  // per (b, g)
-    l.work_max = (int)(l.nqb + (nnz_max + kChunk - 1) / kChunk);
-    l.slot_max = (int)((2 * nnz_max + kChunk - 1) / kChunk);
+    l.work_max = (int)(l.nrows + (nnz_max + l.chunk - 1) / l.chunk);
+    l.slot_max = (int)((2 * nnz_max + l.chunk - 1) / l.chunk);
+    const long long spans = bgs * l.nrows;
     size_t off = 0;
     l.qctl = off;    off = align256(off + 8 * 4);
-    l.bits = off;    off = align256(off + (size_t)bgs * l.nqb * l.words * 4);
-    l.tinfo = off;   off = align256(off + (size_t)bgs * l.nqb * sizeof(TInfo));
+    l.bits = off;    off = align256(off + (size_t)spans * l.words * 4);
+    l.masks = off;   off = align256(off + (size_t)spans * l.mwords * 4);
+    l.tinfo = off;   off = align256(off + (size_t)spans * sizeof(TInfo));
     l.qlist = off;   off = align256(off + (size_t)bgs * nnz_max * 4);
     l.work = off;    off = align256(off + (size_t)bgs * l.work_max * sizeof(int2));
     l.nwork = off;   off = align256(off + (size_t)bgs * 4);
     l.queue = off;   off = align256(off + (size_t)kQueueClasses * bgs * l.work_max * sizeof(int2));
     l.delta = off;   off = align256(off + (size_t)s.B * s.Hq * s.L * 4);
     l.partial = off; off = align256(off + (size_t)bgs * l.slot_max * 2 * kM * kD * 4);
-    l.arrive = off;  off = align256(off + (size_t)bgs * l.nqb * 4);
+    l.arrive = off;  off = align256(off + (size_t)spans * 4);
+    l.ucnt = off;    off = align256(off + (l.kSub > 1 ? (size_t)spans * 4 : 0));
+    l.ulist = off;   off = align256(off + (l.kSub > 1 ? (size_t)spans * l.ucap * 4 : 0));
+    l.umask = off;   off = align256(off + (l.kSub > 1 ? (size_t)spans * l.ucap : 0));
     l.total = off;
     return l;
+}
+
+// The union of the block lists of every span's query blocks (block size
+// m < 64), with owner masks, for the dQ pass: one warp per (b, g, span).
+template <int kSub>
+__global__ void __launch_bounds__(128)
+span_union_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt, int NQB,
+                  int nrows, long long spans, int topk, int ucap, int32_t* __restrict__ ucnt,
+                  int32_t* __restrict__ ulist, uint8_t* __restrict__ umask, int* status) {
+    extern __shared__ uint32_t ubm[];  // per warp: kSub bitmaps of W words
+    const int W = (NQB + 31) / 32;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t* bm = ubm + (size_t)warp * kSub * W;
+    for (int i = lane; i < kSub * W; i += 32) bm[i] = 0u;
+    __syncwarp();
+    const long long u = (long long)blockIdx.x * 4 + warp;
+    if (u >= spans) return;
+    const long long bg = u / nrows;
+    const int sp = (int)(u - bg * nrows);
+    const int qb0 = sp * kSub;
+    build_block_union<kSub>(idx, cnt, bg * NQB + qb0, qb0, min(kSub, NQB - qb0), topk, bm, W,
+                            ulist + u * ucap, umask + u * ucap, ucnt + u, status, lane);
 }
 
 cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const void* O,
@@ -687,6 +734,10 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     const BwdLayout l = bwd_layout(s, topk);
     uint8_t* w = static_cast<uint8_t*>(ws);
     uint32_t* bits = reinterpret_cast<uint32_t*>(w + l.bits);
+    uint32_t* masks = reinterpret_cast<uint32_t*>(w + l.masks);
+    int32_t* ucnt = reinterpret_cast<int32_t*>(w + l.ucnt);
+    int32_t* ulist = reinterpret_cast<int32_t*>(w + l.ulist);
+    uint8_t* umask = reinterpret_cast<uint8_t*>(w + l.umask);
     TInfo* tinfo = reinterpret_cast<TInfo*>(w + l.tinfo);
     int32_t* qlist = reinterpret_cast<int32_t*>(w + l.qlist);
     int2* work = reinterpret_cast<int2*>(w + l.work);
@@ -701,11 +752,26 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     cudaError_t e;
 
     // Two query heads per KV head: tcgen05 kernels (M = 128 rows per MMA), as
-    // long as the block list fits beside dq_tc_kernel's tiles.
-    const bool pair = s.Hq / s.Hkv == 2 && dq_tc_fits(topk);
+    // long as the block list fits beside dq_tc_kernel's tiles. Block sizes
+    // 16 and 32 run on them only (the API rejects them otherwise).
+    const bool pair = s.Hq / s.Hkv == 2 && dq_tc_fits(topk, s.block_size);
+    if (l.kSub > 1 && !pair) return cudaErrorInvalidValue;
+    if (l.kSub > 1) {  // the span unions the dQ pass reads
+        const long long spans = (long long)bgs * l.nrows;
+        const size_t ush = (size_t)4 * l.kSub * l.words * 4;
+        ProfScope prof(K_BWD_MARK, st);
+        if (l.kSub == 2)
+            span_union_kernel<2><<<(unsigned)((spans + 3) / 4), 128, ush, st>>>(
+                idx, cnt, l.nqb, l.nrows, spans, topk, l.ucap, ucnt, ulist, umask, status);
+        else
+            span_union_kernel<4><<<(unsigned)((spans + 3) / 4), 128, ush, st>>>(
+                idx, cnt, l.nqb, l.nrows, spans, topk, l.ucap, ucnt, ulist, umask, status);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     if (pair) {
         // dQ first: it also computes Delta from O and dO, which dK/dV then read.
-        e = launch_dq_tc(Q, K, V, O, dO, lse, delta, idx, cnt, s, topk, sm_scale, dQ, status, st);
+        e = launch_dq_tc(Q, K, V, O, dO, lse, delta, idx, cnt, ulist, ucnt, umask, s, topk,
+                         sm_scale, dQ, status, st);
         if (e != cudaSuccess) return e;
         if (after_dq && (e = cudaEventRecord(after_dq, st)) != cudaSuccess) return e;
     } else {
@@ -716,29 +782,29 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
-    // the queue counters and the bitmap, in one memset
-    if ((e = cudaMemsetAsync(w + l.qctl, 0, l.bits - l.qctl + (size_t)bgs * l.nqb * l.words * 4,
-                             st)) != cudaSuccess)
+    // the queue counters, the bitmap and the mask rows, in one memset
+    if ((e = cudaMemsetAsync(w + l.qctl, 0,
+                             l.masks - l.qctl + (size_t)bgs * l.nrows * l.mwords * 4, st)) !=
+        cudaSuccess)
         return e;
     const long long units = (long long)bgs * l.nqb;
     {
         ProfScope prof(K_BWD_MARK, st);
         idx_mark_kernel<<<(unsigned)((units + 255) / 256), 256, 0, st>>>(
-            idx, cnt, units, l.nqb, topk, l.words, bits, status);
+            idx, cnt, units, l.nqb, l.nrows, l.kSub, topk, l.words, l.mwords, bits, masks, status);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     {
         ProfScope prof(K_BWD_BUILD, st);
-        idx_build_kernel<<<bgs, 1024, 0, st>>>(bits, l.nqb, topk, l.words, l.work_max,
-                                               l.slot_max, tinfo, qlist, work, nwork, arrive,
-                                               queue, qctl, status);
+        idx_build_kernel<<<bgs, 1024, 0, st>>>(bits, l.nqb, l.nrows, l.kSub, topk, l.words,
+                                               l.work_max, l.slot_max, tinfo, qlist, work, nwork,
+                                               arrive, queue, qctl, status);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
     if (pair)  // sums multi-chunk partials itself
-        return launch_dkdv_tc(Q, K, V, dO, lse, delta, tinfo, qlist, queue, qctl, s, topk,
-                              l.work_max, l.slot_max, sm_scale, dK, dV, partial, arrive, status,
-                              st);
+        return launch_dkdv_tc(Q, K, V, dO, lse, delta, tinfo, qlist, masks, queue, qctl, s, topk,
+                              l, sm_scale, dK, dV, partial, arrive, status, st);
 
     e = cudaFuncSetAttribute(dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kKvSmem);
     if (e != cudaSuccess) return e;

@@ -64,41 +64,58 @@ __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
 // unit's Q/dO and first K/V pairs load while the current one finishes.
 // Blocks are processed in pairs, so the S and dP MMAs have N = 128 keys.
 namespace dq {
-constexpr int kKSlots = 3, kVSlots = 2;        // ring slots, one block pair each
-constexpr int kPair = 2 * kTile64;              // two 64 x 128 blocks (32 KB)
-constexpr int kOffQ = 0;
-constexpr int kOffDO = kOffQ + kTile128;
-constexpr int kOffK = kOffDO + kTile128;
-constexpr int kOffV = kOffK + kKSlots * kPair;
-constexpr int kOffBar = kOffV + kVSlots * kPair;
-constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = B_KFULL + kKSlots,
-              B_VFULL = B_KEMPTY + kKSlots, B_VEMPTY = B_VFULL + kVSlots,
-              B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2, B_DPFREE = B_DSFULL + 2,
-              B_FINAL = B_DPFREE + 1, B_DQFREE = B_FINAL + 1, B_DRAIN = B_DQFREE + 1,
-              kNumBars = B_DRAIN + 1;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;
-constexpr int kOffDPart = kOffMisc + 16;  // Delta of the 128 rows, fp32
-constexpr int kOffList = kOffDPart + 128 * 4;  // block lists: 7 slots of list_stride(topk) ints
+// Ring depths and shared-memory layout per block size: at m < 64 the K ring
+// has two slots instead of three, so that the longer lists (the unions of a
+// span's query-block lists, with owner masks) fit beside the tiles.
+template <int kSub>
+struct Cfg {
+    static constexpr int kKSlots = kSub == 1 ? 3 : 2, kVSlots = 2;  // ring slots, one tile pair each
+    static constexpr int kPair = 2 * kTile64;                        // two 64 x 128 tiles (32 KB)
+    static constexpr int kOffQ = 0;
+    static constexpr int kOffDO = kOffQ + kTile128;
+    static constexpr int kOffK = kOffDO + kTile128;
+    static constexpr int kOffV = kOffK + kKSlots * kPair;
+    static constexpr int kOffBar = kOffV + kVSlots * kPair;
+    static constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = B_KFULL + kKSlots,
+                         B_VFULL = B_KEMPTY + kKSlots, B_VEMPTY = B_VFULL + kVSlots,
+                         B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2,
+                         B_DPFREE = B_DSFULL + 2, B_FINAL = B_DPFREE + 1, B_DQFREE = B_FINAL + 1,
+                         B_DRAIN = B_DQFREE + 1, kNumBars = B_DRAIN + 1;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+    static constexpr int kOffDPart = kOffMisc + 16;  // Delta of the 128 rows, fp32
+    static constexpr int kOffList = kOffDPart + 128 * 4;  // block lists: 7 slots
+};
 constexpr int kListK = 0, kListV = 2, kListM = 4, kListE = 5, kListSlots = 7;
 constexpr int kThreads = 384;  // 8 elementwise warps, K producer, MMA, V producer, Q/dO producer
 // TMEM: dQ [0,128), S of pair buffer b at [128 + 128b, +128), dP [384, 512).
 // dS of key half h overwrites S columns [64h, 64h + 32) (read by the same thread).
 constexpr uint32_t kColDQ = 0, kColDP = 384;
 __device__ __forceinline__ uint32_t col_s(int b) { return 128u + 128u * (uint32_t)b; }
+// A list slot: the entries (capacity kSub * topk, one padding entry, the count
+// in the last int of the entry region), then at m < 64 the owner masks (bytes).
+__host__ __device__ constexpr int list_ints(int topk, int kSub) { return (kSub * topk + 2 + 15) & ~15; }
+__host__ __device__ constexpr int slot_ints(int topk, int kSub) {
+    return list_ints(topk, kSub) + (kSub > 1 ? (kSub * topk + 15) / 16 * 4 : 0);
+}
+template <int kSub>
 constexpr size_t smem_bytes(int topk) {
-    return 1024 + (size_t)kOffList + (size_t)kListSlots * ((topk + 2 + 15) & ~15) * 4;
+    return 1024 + (size_t)Cfg<kSub>::kOffList + (size_t)kListSlots * slot_ints(topk, kSub) * 4;
 }
 }  // namespace dq
 
 struct DqArgs {
     const int32_t* idx;
     const int32_t* cnt;
+    const int32_t* ulist;   // m < 64: per span, the union of its query blocks' lists
+    const int32_t* ucnt;
+    const uint8_t* umask;   //         and the owner masks of its entries
     const float* lse;
     const __nv_bfloat16* O;
     float* delta;  // written: Delta_i = dO_i . O_i for every valid row
     __nv_bfloat16* dQ;
     int* status;
-    int Hq, Hkv, L, NQB, topk, units;
+    int Hq, Hkv, L, NQB, topk, units;  // NQB: query blocks of m tokens
+    int nsb, ucap;                     // 64-token spans per (b, g); union capacity
     float scale_log2, sm_scale;
 };
 
@@ -131,98 +148,131 @@ __device__ __forceinline__ int stage_list(const int32_t* __restrict__ row,
     return k;
 }
 
-__host__ __device__ constexpr int list_stride(int topk) { return (topk + 2 + 15) & ~15; }
-
+// A unit is a 64-token span of one (b, g) (the query block itself at m = 64);
+// lu indexes its list row: idx/cnt at m = 64, the union rows at m < 64.
 struct DqUnit {
     int qb, bg, hq0;
     long long lu;
 };
 
+template <int kSub>
 __device__ __forceinline__ DqUnit dq_unit(const DqArgs& a, int u) {
     DqUnit d;
-    d.qb = a.NQB - 1 - (u % a.NQB);  // heaviest query blocks first
-    d.bg = u / a.NQB;
+    d.qb = a.nsb - 1 - (u % a.nsb);  // heaviest spans first
+    d.bg = u / a.nsb;
     d.hq0 = (d.bg / a.Hkv) * a.Hq + (d.bg % a.Hkv) * 2;
-    d.lu = (long long)d.bg * a.NQB + d.qb;
+    d.lu = kSub == 1 ? (long long)d.bg * a.NQB + d.qb : (long long)d.bg * a.nsb + d.qb;
     return d;
 }
 
+// Copies a span's union list (already validated, ascending) to shared memory
+// with independent loads, and its owner masks when mout is given. Returns the
+// count; out[n] repeats the last entry.
+__device__ __forceinline__ int stage_union_list(const DqArgs& a, long long row, int* out,
+                                                uint8_t* mout) {
+    const int n = min(__ldg(a.ucnt + row), a.ucap);
+    const int32_t* src = a.ulist + row * a.ucap;
+    for (int j0 = 0; j0 < n; j0 += 16) {
+        int v[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) v[k] = j0 + k < n ? __ldg(src + j0 + k) : 0;
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+            if (j0 + k < n) out[j0 + k] = v[k];
+    }
+    if (mout)
+        for (int j = 0; j < n; ++j) mout[j] = __ldg(a.umask + row * a.ucap + j);
+    out[n] = n > 0 ? out[n - 1] : 0;
+    return n;
+}
+
+// The unit's list into a slot (entries; masks too when mout is given).
+template <int kSub>
+__device__ __forceinline__ int stage_unit(const DqArgs& a, const DqUnit& d, int* out, uint8_t* mout) {
+    if constexpr (kSub == 1)
+        return stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, out);
+    else
+        return stage_union_list(a, d.lu, out, mout);
+}
+
+template <int kSub>
 __global__ void __launch_bounds__(dq::kThreads, 1)
 dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
              const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
              const DqArgs a) {
     using namespace dq;
+    using C = Cfg<kSub>;
+    constexpr int kMq = 64 / kSub;  // tokens of a query block (and keys of a KV block)
+    const int li = list_ints(a.topk, kSub);  // entry ints of a list slot
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     const uint32_t sb = smem_u32(smem);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    auto bar = [&](int i) { return sb + kOffBar + 8u * (uint32_t)i; };
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
+    auto bar = [&](int i) { return sb + C::kOffBar + 8u * (uint32_t)i; };
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
     if (threadIdx.x == 0) {
-        mbar_init(bar(B_Q), 1);
-        mbar_init(bar(B_QFREE), 257);  // the MMA commit after the unit's last dP + 256 Delta readers
-        for (int s = 0; s < kKSlots; ++s) {
-            mbar_init(bar(B_KFULL + s), 1);
-            mbar_init(bar(B_KEMPTY + s), 1);
+        mbar_init(bar(C::B_Q), 1);
+        mbar_init(bar(C::B_QFREE), 257);  // the MMA commit after the unit's last dP + 256 Delta readers
+        for (int s = 0; s < C::kKSlots; ++s) {
+            mbar_init(bar(C::B_KFULL + s), 1);
+            mbar_init(bar(C::B_KEMPTY + s), 1);
         }
-        for (int s = 0; s < kVSlots; ++s) {
-            mbar_init(bar(B_VFULL + s), 1);
-            mbar_init(bar(B_VEMPTY + s), 1);
+        for (int s = 0; s < C::kVSlots; ++s) {
+            mbar_init(bar(C::B_VFULL + s), 1);
+            mbar_init(bar(C::B_VEMPTY + s), 1);
         }
-        mbar_init(bar(B_SPFULL), 1);
-        mbar_init(bar(B_SPFULL + 1), 1);
+        mbar_init(bar(C::B_SPFULL), 1);
+        mbar_init(bar(C::B_SPFULL + 1), 1);
         // dS barriers alternate by pair: once dP is released early, a thread may
         // finish pair p+1 before another has finished pair p, so their arrivals
         // must go to different barriers. dP_{p+1} needs every thread's release of
         // dP_p, so no thread gets two pairs ahead and two barriers suffice.
-        mbar_init(bar(B_DSFULL), 256);
-        mbar_init(bar(B_DSFULL + 1), 256);
-        mbar_init(bar(B_DPFREE), 256);
-        mbar_init(bar(B_FINAL), 1);
-        mbar_init(bar(B_DQFREE), 256);
-        mbar_init(bar(B_DRAIN), 1);
+        mbar_init(bar(C::B_DSFULL), 256);
+        mbar_init(bar(C::B_DSFULL + 1), 256);
+        mbar_init(bar(C::B_DPFREE), 256);
+        mbar_init(bar(C::B_FINAL), 1);
+        mbar_init(bar(C::B_DQFREE), 256);
+        mbar_init(bar(C::B_DRAIN), 1);
         fence_barrier_init();
         *abort_flag = 0;
     }
     if (warp == 9) {
-        tmem_alloc(sb + kOffMisc, kTmemCols);
+        tmem_alloc(sb + C::kOffMisc, kTmemCols);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffMisc);
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + C::kOffMisc);
 
     if (warp == 8 || warp == 10) {
         // ------------------------------------------------ K and V producers (block pairs)
         if (lane == 0) {
             const bool is_k = warp == 8;
             const CUtensorMap* map = is_k ? &tmK : &tmV;
-            const int slots = is_k ? kKSlots : kVSlots;
-            const int full = is_k ? B_KFULL : B_VFULL, empty = is_k ? B_KEMPTY : B_VEMPTY;
-            const uint32_t ring = sb + (is_k ? kOffK : kOffV);
+            const int slots = is_k ? C::kKSlots : C::kVSlots;
+            const int full = is_k ? C::B_KFULL : C::B_VFULL, empty = is_k ? C::B_KEMPTY : C::B_VEMPTY;
+            const uint32_t ring = sb + (is_k ? C::kOffK : C::kOffV);
             prefetch_tmap(map);
-            const int ls = list_stride(a.topk);
-            int* lists = reinterpret_cast<int*>(smem + kOffList) + (is_k ? kListK : kListV) * ls;
+            const int ls = slot_ints(a.topk, kSub);
+            int* lists = reinterpret_cast<int*>(smem + C::kOffList) + (is_k ? kListK : kListV) * ls;
             // Two list slots by unit parity. The next unit's list is staged once the
             // current unit's pairs are all issued, while the ring is still full, so
             // its memory latency stays off the load path.
             auto stage = [&](int u, int slot) {
-                const DqUnit d = dq_unit(a, u);
-                return stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb,
-                                  lists + slot * ls);
+                return stage_unit<kSub>(a, dq_unit<kSub>(a, u), lists + slot * ls, nullptr);
             };
             int n_cur = blockIdx.x < a.units ? stage(blockIdx.x, 0) : 0;
             int gp = 0;  // pairs issued so far, over all units
             bool ok = true;
             int ul = 0;
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++ul) {
-                const DqUnit d = dq_unit(a, u);
+                const DqUnit d = dq_unit<kSub>(a, u);
                 const int* list = lists + (ul & 1) * ls;
                 const int n = n_cur;
-                const int np = (n + 1) >> 1;
+                const int np = ((n + kSub - 1) / kSub + 1) >> 1;  // pairs of 64-key tiles
                 for (int p = 0; p < np; ++p, ++gp) {
                     const int s = gp % slots;
                     if (gp >= slots &&
@@ -230,15 +280,19 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                         ok = false;
                         break;
                     }
-                    mbar_expect_tx(bar(full + s), kPair);
-                    // slot layout: [d half][block of the pair][64 rows][64 columns]; an
-                    // odd count pairs the last block with itself (masked by the consumer)
-                    for (int dh = 0; dh < 2; ++dh) {
-                        tma_load_3d(ring + s * kPair + dh * kHalf128, map, bar(full + s), dh * 64,
-                                    list[2 * p] * 64, d.bg);
-                        tma_load_3d(ring + s * kPair + dh * kHalf128 + kHalf64, map, bar(full + s),
-                                    dh * 64, list[2 * p + 1] * 64, d.bg);
-                    }
+                    mbar_expect_tx(bar(full + s), C::kPair);
+                    // slot layout: [d half][tile of the pair][64 rows][64 columns]; a tile
+                    // holds kSub blocks of kMq rows; entries past the list repeat its
+                    // last block (masked by the consumer)
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int q = 0; q < kSub; ++q) {
+                            const int e = (2 * p + h) * kSub + q;
+                            const int blk = list[e < n ? e : n - 1];
+                            for (int dh = 0; dh < 2; ++dh)
+                                tma_load_3d(ring + s * C::kPair + dh * kHalf128 + h * kHalf64 + q * kMq * 128,
+                                            map, bar(full + s), dh * 64, blk * kMq, d.bg);
+                        }
                 }
                 const int u2 = u + (int)gridDim.x;
                 n_cur = ok && u2 < a.units ? stage(u2, (ul + 1) & 1) : 0;
@@ -251,27 +305,27 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         if (lane == 0) {
             prefetch_tmap(&tmQ);
             prefetch_tmap(&tmdO);
-            const int ls = list_stride(a.topk);
-            int* elists = reinterpret_cast<int*>(smem + kOffList) + kListE * ls;
+            const int ls = slot_ints(a.topk, kSub);
+            int* elists = reinterpret_cast<int*>(smem + C::kOffList) + kListE * ls;
             int ul = 0, last = -1;
             for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
-                if (ul > 0 && !mbar_wait(bar(B_QFREE), (ul - 1) & 1, abort_flag, a.status)) break;
+                if (ul > 0 && !mbar_wait(bar(C::B_QFREE), (ul - 1) & 1, abort_flag, a.status)) break;
                 last = ul;
-                const DqUnit d = dq_unit(a, u);
+                const DqUnit d = dq_unit<kSub>(a, u);
                 // The tiles first; then the elementwise warps' copy of the block list
                 // (its slot's previous unit is done: they have passed that unit's
-                // Delta), published by this thread's arrival on B_Q.
-                mbar_expect_tx_only(bar(B_Q), 2 * kTile128);
+                // Delta), published by this thread's arrival on C::B_Q.
+                mbar_expect_tx_only(bar(C::B_Q), 2 * kTile128);
                 for (int hl = 0; hl < 2; ++hl)
                     for (int dh = 0; dh < 2; ++dh) {
-                        tma_load_3d(sb + kOffQ + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_Q),
+                        tma_load_3d(sb + C::kOffQ + dh * kHalf128 + hl * kHalf64, &tmQ, bar(C::B_Q),
                                     dh * 64, d.qb * 64, d.hq0 + hl);
-                        tma_load_3d(sb + kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(B_Q),
+                        tma_load_3d(sb + C::kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(C::B_Q),
                                     dh * 64, d.qb * 64, d.hq0 + hl);
                     }
                 int* el = elists + (ul & 1) * ls;
-                el[ls - 1] = stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, el);
-                mbar_arrive(bar(B_Q));
+                el[li - 1] = stage_unit<kSub>(a, d, el, reinterpret_cast<uint8_t*>(el + li));
+                mbar_arrive(bar(C::B_Q));
                 // The next unit's Q and dO come from HBM: start bringing them into L2
                 // now, a whole unit before they are loaded.
                 const int u2 = u + (int)gridDim.x;
@@ -285,20 +339,20 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                         }
                 }
             }
-            if (last >= 0) mbar_wait_drain(bar(B_Q), last & 1);
+            if (last >= 0) mbar_wait_drain(bar(C::B_Q), last & 1);
         }
     } else if (warp == 9) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t id_s = idesc_bf16(128, 128, false);
             constexpr uint32_t id_dq = idesc_bf16(128, 128, true);
-            const uint64_t dQ0 = sdesc_sw128(sb + kOffQ, 16, 1024);
-            const uint64_t dDO0 = sdesc_sw128(sb + kOffDO, 16, 1024);
-            const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
-            const uint64_t dKmn0 = sdesc_sw128(sb + kOffK, kHalf128, 1024);  // K read MN-major
-            const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
+            const uint64_t dQ0 = sdesc_sw128(sb + C::kOffQ, 16, 1024);
+            const uint64_t dDO0 = sdesc_sw128(sb + C::kOffDO, 16, 1024);
+            const uint64_t dK0 = sdesc_sw128(sb + C::kOffK, 16, 1024);
+            const uint64_t dKmn0 = sdesc_sw128(sb + C::kOffK, kHalf128, 1024);  // K read MN-major
+            const uint64_t dV0 = sdesc_sw128(sb + C::kOffV, 16, 1024);
             auto issue_s = [&](int gp) {  // S = Q Kpair^T into buffer gp & 1
-                const uint64_t kd = sdesc_at(dK0, (gp % kKSlots) * kPair);
+                const uint64_t kd = sdesc_at(dK0, (gp % C::kKSlots) * C::kPair);
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
                     const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
@@ -307,35 +361,37 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 }
             };
             auto issue_dp = [&](int gp) {  // dP = dO Vpair^T; releases the V slot
-                const uint64_t vd = sdesc_at(dV0, (gp % kVSlots) * kPair);
+                const uint64_t vd = sdesc_at(dV0, (gp % C::kVSlots) * C::kPair);
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
                     const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
                     mma_ss(tmem + kColDP, sdesc_at(dDO0, off), sdesc_at(vd, off), id_s,
                            ks > 0 ? 1u : 0u);
                 }
-                mma_commit(bar(B_SPFULL + (gp & 1)));  // S and dP of this pair are both complete
-                mma_commit(bar(B_VEMPTY + gp % kVSlots));
+                mma_commit(bar(C::B_SPFULL + (gp & 1)));  // S and dP of this pair are both complete
+                mma_commit(bar(C::B_VEMPTY + gp % C::kVSlots));
             };
             auto wait_k = [&](int gp) {
-                return mbar_wait(bar(B_KFULL + gp % kKSlots), (gp / kKSlots) & 1, abort_flag, a.status);
+                return mbar_wait(bar(C::B_KFULL + gp % C::kKSlots), (gp / C::kKSlots) & 1, abort_flag, a.status);
             };
             auto wait_v = [&](int gp) {
-                return mbar_wait(bar(B_VFULL + gp % kVSlots), (gp / kVSlots) & 1, abort_flag, a.status);
+                return mbar_wait(bar(C::B_VFULL + gp % C::kVSlots), (gp / C::kVSlots) & 1, abort_flag, a.status);
             };
             // dP has one TMEM buffer: dP(gp) waits until the elementwise warps hold
             // dP(gp - 1) in registers (they release it before computing dS).
             auto wait_dpfree = [&](int gp) {
-                return gp == 0 || mbar_wait(bar(B_DPFREE), (gp - 1) & 1, abort_flag, a.status);
+                return gp == 0 || mbar_wait(bar(C::B_DPFREE), (gp - 1) & 1, abort_flag, a.status);
             };
             bool ok = true;
             int gp0 = 0, ul = 0;
             // Order per unit: S_0 dP_0 S_1 | dP_1 | dS_0 -> dQ_0 S_2 | dP_2 | dS_1 -> dQ_1 S_3 ...
-            int* mlist = reinterpret_cast<int*>(smem + kOffList) + kListM * list_stride(a.topk);
+            int* mlist = reinterpret_cast<int*>(smem + C::kOffList) + kListM * slot_ints(a.topk, kSub);
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++ul) {
-                const DqUnit d = dq_unit(a, u);
-                const int np = (stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, mlist) + 1) >> 1;
-                ok = mbar_wait(bar(B_Q), ul & 1, abort_flag, a.status);
+                const DqUnit d = dq_unit<kSub>(a, u);
+                const int nu = kSub == 1 ? stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, mlist)
+                                         : min(__ldg(a.ucnt + d.lu), a.ucap);
+                const int np = ((nu + kSub - 1) / kSub + 1) >> 1;
+                ok = mbar_wait(bar(C::B_Q), ul & 1, abort_flag, a.status);
                 if (!ok) break;
                 tc_fence_after();
                 if (np >= 1) {
@@ -344,7 +400,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                     tc_fence_after();
                     issue_s(gp0);
                     issue_dp(gp0);
-                    if (np == 1) mma_commit(bar(B_QFREE));
+                    if (np == 1) mma_commit(bar(C::B_QFREE));
                 }
                 if (np >= 2) {
                     ok = wait_k(gp0 + 1);
@@ -353,11 +409,11 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                     issue_s(gp0 + 1);
                 }
                 if (np == 0) {
-                    mma_commit(bar(B_QFREE));
+                    mma_commit(bar(C::B_QFREE));
                     // the previous unit's dQ must be read out before FINAL completes again
-                    ok = ul == 0 || mbar_wait(bar(B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
+                    ok = ul == 0 || mbar_wait(bar(C::B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
                     if (!ok) break;
-                    mma_commit(bar(B_FINAL));
+                    mma_commit(bar(C::B_FINAL));
                 }
                 for (int p = 0; ok && p < np; ++p) {
                     const int gp = gp0 + p;
@@ -366,22 +422,22 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                         if (!ok) break;
                         tc_fence_after();
                         issue_dp(gp + 1);
-                        if (p + 2 == np) mma_commit(bar(B_QFREE));  // last MMA reading Q/dO
+                        if (p + 2 == np) mma_commit(bar(C::B_QFREE));  // last MMA reading Q/dO
                     }
-                    ok = mbar_wait(bar(B_DSFULL + (gp & 1)), (gp >> 1) & 1, abort_flag, a.status);
+                    ok = mbar_wait(bar(C::B_DSFULL + (gp & 1)), (gp >> 1) & 1, abort_flag, a.status);
                     if (ok && p == 0 && ul > 0)  // dQ's accumulator: the previous unit is read out
-                        ok = mbar_wait(bar(B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
+                        ok = mbar_wait(bar(C::B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
                     if (!ok) break;
                     tc_fence_after();
                     // dQ += dS Kpair: A = dS (TMEM), B = the K pair read MN-major
-                    const uint64_t kmn = sdesc_at(dKmn0, (gp % kKSlots) * kPair);
+                    const uint64_t kmn = sdesc_at(dKmn0, (gp % C::kKSlots) * C::kPair);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
                         mma_ts(tmem + kColDQ, tmem + col_s(gp & 1) + (ks >> 2) * 64 + (ks & 3) * 8,
                                sdesc_at(kmn, ks * 2048), id_dq, (p > 0 || ks > 0) ? 1u : 0u);
-                    mma_commit(bar(B_KEMPTY + gp % kKSlots));
+                    mma_commit(bar(C::B_KEMPTY + gp % C::kKSlots));
                     if (p == np - 1) {
-                        mma_commit(bar(B_FINAL));
+                        mma_commit(bar(C::B_FINAL));
                     } else if (p + 2 < np) {  // S_{p+2} reuses the S buffer dQ_p has just read
                         ok = wait_k(gp + 2);
                         if (!ok) break;
@@ -391,8 +447,8 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 }
                 gp0 += np;
             }
-            mma_commit(bar(B_DRAIN));
-            mbar_wait_drain(bar(B_DRAIN), 0);
+            mma_commit(bar(C::B_DRAIN));
+            mbar_wait_drain(bar(C::B_DRAIN), 0);
         }
     } else {
         // ------------------------------------------------ elementwise (8 warps)
@@ -402,18 +458,18 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         const int et = threadIdx.x;  // 0..255 over the elementwise warps
         const int pc = et & 15;      // 16-byte piece of a row in the Delta pass
-        float* dpart = reinterpret_cast<float*>(smem + kOffDPart);
+        float* dpart = reinterpret_cast<float*>(smem + C::kOffDPart);
         bool ok = true;
         int gp0 = 0, ul = 0;
-        const int ls = list_stride(a.topk);
-        int* lists = reinterpret_cast<int*>(smem + kOffList) + kListE * ls;
+        const int ls = slot_ints(a.topk, kSub);
+        int* lists = reinterpret_cast<int*>(smem + C::kOffList) + kListE * ls;
         // A unit's O rows and lse (for Delta and P) are fetched at the end of the
         // previous unit, so that they are in hand when its Q and dO arrive; its
-        // block list is staged by the Q/dO producer before it arrives on B_Q.
+        // block list is staged by the Q/dO producer before it arrives on C::B_Q.
         uint4 ov[8];
         float neg_lse2 = 0.f;
         auto fetch_unit = [&](int u) {
-            const DqUnit d = dq_unit(a, u);
+            const DqUnit d = dq_unit<kSub>(a, u);
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
                 const int rr = k * 16 + (et >> 4);
@@ -430,7 +486,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         // named barrier per unit is reached the same number of times by all.
         for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
             const int* list = lists + (ul & 1) * ls;
-            const DqUnit d = dq_unit(a, u);
+            const DqUnit d = dq_unit<kSub>(a, u);
             const int qb = d.qb;
             const int i = qb * 64 + tok;
             const bool valid = i < a.L;
@@ -440,20 +496,25 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                // read a unit's list; O and lse are fetched into registers a unit ahead)
                 const int u3 = u + 2 * (int)gridDim.x;
                 if (u3 < a.units) {
-                    const DqUnit d3 = dq_unit(a, u3);
+                    const DqUnit d3 = dq_unit<kSub>(a, u3);
                     const int r3 = et >> 1, i3 = d3.qb * 64 + (r3 & 63);
                     if (i3 < a.L) {
                         const size_t row3 = (size_t)(d3.hq0 + (r3 >> 6)) * a.L + i3;
                         prefetch_l2(a.O + row3 * 128 + 64 * (et & 1));
                         if ((r3 & 31) == 0 && (et & 1) == 0) prefetch_l2(a.lse + row3);
                     }
-                    if (et == 0) prefetch_l2(a.cnt + d3.lu);
-                    if (et < 4 && et * 32 < a.topk) prefetch_l2(a.idx + d3.lu * a.topk + et * 32);
-                    if (et == 4) prefetch_l2(a.idx + d3.lu * a.topk + a.topk - 1);
+                    if constexpr (kSub == 1) {
+                        if (et == 0) prefetch_l2(a.cnt + d3.lu);
+                        if (et < 4 && et * 32 < a.topk) prefetch_l2(a.idx + d3.lu * a.topk + et * 32);
+                        if (et == 4) prefetch_l2(a.idx + d3.lu * a.topk + a.topk - 1);
+                    } else {
+                        if (et == 0) prefetch_l2(a.ucnt + d3.lu);
+                        if (et < 8 && et * 32 < a.ucap) prefetch_l2(a.ulist + d3.lu * a.ucap + et * 32);
+                    }
                 }
             }
             if (ok) {
-                ok = mbar_wait(bar(B_Q), ul & 1, abort_flag, a.status);
+                ok = mbar_wait(bar(C::B_Q), ul & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
             // Delta_i = dO_i . O_i: O in coalesced 16-byte pieces (16 threads per
@@ -465,7 +526,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 float acc = 0.f;
                 if (ok) {
                     const uint4 dv = *reinterpret_cast<const uint4*>(
-                        smem + kOffDO + (pc >> 3) * kHalf128 + (rr >> 6) * kHalf64 + sw_off(rr & 63, pc & 7));
+                        smem + C::kOffDO + (pc >> 3) * kHalf128 + (rr >> 6) * kHalf64 + sw_off(rr & 63, pc & 7));
                     const uint32_t ow[4] = {ov[k].x, ov[k].y, ov[k].z, ov[k].w};
                     const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w};
 #pragma unroll
@@ -484,31 +545,44 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const float dlt = dpart[row];
             // This thread is done with dO and with Delta's exchange slots: the next
             // unit's dO may be loaded (and dpart rewritten) once all have arrived.
-            if (ok) mbar_arrive(bar(B_QFREE));
-            const int n = list[ls - 1];
-            const int np = (n + 1) >> 1;
+            if (ok) mbar_arrive(bar(C::B_QFREE));
+            const int n = list[li - 1];
+            const int nt = (n + kSub - 1) / kSub;  // 64-key tiles
+            const int np = (nt + 1) >> 1;
+            const uint8_t* own = reinterpret_cast<const uint8_t*>(list + li);
+            const int jr = tok / kMq, tt = tok % kMq;  // the row's query block in the span, token in it
+            const int qb_r = qb * kSub + jr;
             if (ok && half == 0 && valid) a.delta[ridx] = dlt;
             const int u2 = u + (int)gridDim.x;
             for (int p = 0; ok && p < np; ++p) {
                 const int gp = gp0 + p;
                 const int buf = gp & 1;
-                ok = mbar_wait(bar(B_SPFULL + buf), (gp >> 1) & 1, abort_flag, a.status);
+                ok = mbar_wait(bar(C::B_SPFULL + buf), (gp >> 1) & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
                 tc_fence_after();
-                const int e = 2 * p + half;       // this half's block in the list
-                const bool live = e < n;          // false: the duplicate of an odd count
-                const bool diag = list[e] == qb;
+                const int tile = 2 * p + half;    // this half's tile of the pair
+                // slot q of the tile: attended by the row if its query block selected
+                // the slot's block (full), or only up to its token (part: its own block)
+                uint32_t full = 0u, part = 0u;
+#pragma unroll
+                for (int q = 0; q < kSub; ++q) {
+                    const int e = tile * kSub + q;
+                    const bool sel = e < n && (kSub == 1 || ((own[e] >> jr) & 1u));
+                    const bool mine = sel && list[e] == qb_r;
+                    full |= (uint32_t)(sel && !mine) << q;
+                    part |= (uint32_t)mine << q;
+                }
                 uint32_t sv[64], dp[64];
                 tmem_ld64x2(lane_base + col_s(buf) + 64 * half, lane_base + kColDP + 64 * half, sv, dp);
                 tc_fence_before();
-                mbar_arrive(bar(B_DPFREE));  // dP is in registers: the buffer may be refilled
+                mbar_arrive(bar(C::B_DPFREE));  // dP is in registers: the buffer may be refilled
                 // dS = P (dP - Delta), P = 2^(S scale_log2 - lse log2 e), two keys at a
                 // time (packed f32x2 arithmetic); the masks (the query's own block and the
                 // duplicate of an odd count) are warp-uniform branches off the main path
                 const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
                 const float2 nl2v = make_float2(nl2, nl2), ndl = make_float2(-dlt, -dlt);
-                if (live && !diag) {
+                if (full == (1u << kSub) - 1u) {
 #pragma unroll
                     for (int c = 0; c < 32; ++c) {
                         float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
@@ -522,8 +596,11 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
 #pragma unroll
                     for (int c = 0; c < 32; ++c) {
                         float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
-                        pv.x = (live && 2 * c <= tok) ? ex2_approx(pv.x) : 0.f;
-                        pv.y = (live && 2 * c + 1 <= tok) ? ex2_approx(pv.y) : 0.f;
+                        const int q0 = (2 * c) / kMq, q1 = (2 * c + 1) / kMq;
+                        const bool k0 = ((full >> q0) & 1u) || (((part >> q0) & 1u) && (2 * c) % kMq <= tt);
+                        const bool k1 = ((full >> q1) & 1u) || (((part >> q1) & 1u) && (2 * c + 1) % kMq <= tt);
+                        pv.x = k0 ? ex2_approx(pv.x) : 0.f;
+                        pv.y = k1 ? ex2_approx(pv.y) : 0.f;
                         const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
                         const float2 ds = __fmul2_rn(pv, d);
                         sv[c] = pack2_bf16(ds.x, ds.y);
@@ -532,14 +609,14 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 // dS columns [64 half, 64 half + 32): inside this thread's own S range
                 tmem_st32(lane_base + col_s(buf) + 64 * half, sv);
                 tc_fence_before();
-                mbar_arrive(bar(B_DSFULL + buf));
+                mbar_arrive(bar(C::B_DSFULL + buf));
             }
             gp0 += np;
             // the next unit's inputs: their latency overlaps this unit's last dQ
             // MMAs and its epilogue
             if (u2 < a.units) fetch_unit(u2);
             if (ok) {
-                ok = mbar_wait(bar(B_FINAL), ul & 1, abort_flag, a.status);
+                ok = mbar_wait(bar(C::B_FINAL), ul & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
             if (ok) {
@@ -557,7 +634,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                     }
                     if (c2 == 1) {
                         tc_fence_before();
-                        mbar_arrive(bar(B_DQFREE));
+                        mbar_arrive(bar(C::B_DQFREE));
                     }
                     if (valid) {
                         uint4* dst = reinterpret_cast<uint4*>(a.dQ + ridx * 128 + 64 * half + 32 * c2);
@@ -614,7 +691,8 @@ constexpr int B_KV = 0, B_KVFREE = 1, B_QFULL = 2, B_QEMPTY = 4, B_SPFULL = 6, B
 constexpr int kIFreeCount = 9;  // the MMA thread and the 8 elementwise warps
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag, last-arriver flag
 constexpr int kOffQL = kOffMisc + 16;  // the producer's copy of an item's query blocks
-constexpr int kOffN = kOffQL + kBwdChunk * 4;  // iteration counts of recent items [4]
+constexpr int kMaxItemQ = kBwdChunk * 4;      // query blocks per item at m = 16
+constexpr int kOffN = kOffQL + kMaxItemQ * 4;  // iteration counts of recent items [4]
 constexpr int kOffRing = (kOffN + 16 + 15) / 16 * 16;  // item descriptors [kRing][8 ints]
 constexpr int kThreads = 320;  // 8 elementwise warps, producer, MMA
 // TMEM: S of iteration buffer b at 128b, dP at 64 + 128b; dV^T and dK^T of
@@ -627,12 +705,18 @@ constexpr size_t kSmem = 1024 + (size_t)kOffRing + kRing * 32;
 static_assert(kSmem <= kMaxDynSmem, "dK/dV shared memory");
 }  // namespace kv
 
+// Rows of the transposed selection are KV spans t of 64 keys (kSub = 64/m
+// blocks of m keys; the span is the block at m = 64); an item iterates over
+// kSub selecting query blocks (of m tokens) at a time: 2 heads x kSub x m =
+// 128 query rows, gathered by TMA. At m < 64, masks holds per (span, query
+// block) which of the span's blocks the query block selected (kSub bits).
 struct KvArgs {
     const float* lse;
     const float* delta;
     const BwdTInfo* tinfo;
     const int32_t* qlist;
-    const int2* queue;    // [kQueueClasses][qcap] {bg * NQB + t, chunk}
+    const uint32_t* masks;
+    const int2* queue;    // [kQueueClasses][qcap] {bg * nrows + t, chunk}
     const int* qcount;    // items per class
     int* ticket;          // next queue position to take
     float* partial;
@@ -641,7 +725,8 @@ struct KvArgs {
     __nv_bfloat16* dV;
     int* status;
     long long qcap;
-    int Hq, Hkv, L, NQB, topk, slot_max;
+    long long nnzq;  // query-list entries per (b, g)
+    int Hq, Hkv, L, nrows, topk, slot_max, mwords, chunkq;
     float scale_log2, sm_scale;
 };
 
@@ -651,7 +736,13 @@ struct KvItem {
     BwdTInfo info;
 };
 
-// Queue position j -> its entry {bg * NQB + t, chunk}; valid = false past the end.
+// Query blocks of an item (chunk c of span t's list): its iterations take kSub at a time.
+__device__ __forceinline__ int item_nq(const KvArgs& a, const KvItem& it) {
+    const int q_begin = it.chunk * a.chunkq;
+    return max(0, min(it.info.n, q_begin + a.chunkq) - q_begin);
+}
+
+// Queue position j -> its entry {bg * nrows + t, chunk}; valid = false past the end.
 __device__ __forceinline__ int2 queue_entry(const KvArgs& a, const int* qn, int j, bool& valid) {
     int c = 0;
 #pragma unroll
@@ -664,19 +755,30 @@ __device__ __forceinline__ int2 queue_entry(const KvArgs& a, const int* qn, int 
     return valid ? a.queue[(size_t)c * a.qcap + j] : make_int2(0, 0);
 }
 
+template <int kSub>
 __device__ __forceinline__ KvItem item_of(const KvArgs& a, int2 e, const BwdTInfo& info) {
     KvItem it;
-    it.bg = e.x / a.NQB;
-    it.t = e.x - it.bg * a.NQB;
+    it.bg = e.x / a.nrows;
+    it.t = e.x - it.bg * a.nrows;
     it.chunk = e.y;
     it.info = info;
-    const int q_begin = e.y * kBwdChunk;
-    it.n_it = max(0, min(info.n, q_begin + kBwdChunk) - q_begin);
+    it.n_it = (item_nq(a, it) + kSub - 1) / kSub;
     return it;
 }
 
 __device__ __forceinline__ const int32_t* item_qlist(const KvArgs& a, const KvItem& it) {
-    return a.qlist + (size_t)it.bg * a.NQB * a.topk + it.info.off + it.chunk * kBwdChunk;
+    return a.qlist + (size_t)it.bg * a.nnzq + it.info.off + it.chunk * a.chunkq;
+}
+
+// The kSub-bit mask of the blocks of span t that query block qb selected.
+template <int kSub>
+__device__ __forceinline__ uint32_t span_mask(const KvArgs& a, int bg, int t, int qb) {
+    if constexpr (kSub == 1) {
+        return 1u;
+    } else {
+        const uint32_t w = __ldg(a.masks + ((size_t)bg * a.nrows + t) * a.mwords + ((qb * kSub) >> 5));
+        return (w >> ((qb * kSub) & 31)) & ((1u << kSub) - 1u);
+    }
 }
 
 __device__ __forceinline__ void ring_put(int* e, const KvItem& it) {
@@ -699,11 +801,13 @@ __device__ __forceinline__ KvItem ring_get(const int* e) {
     return it;
 }
 
+template <int kSub>
 __global__ void __launch_bounds__(kv::kThreads, 1)
 dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
                const KvArgs a) {
     using namespace kv;
+    constexpr int kMq = 64 / kSub;  // tokens of a query block (and keys of a KV block)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -772,7 +876,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             int2 e = entry_of(atomicAdd(a.ticket, 1), valid);
             KvItem it;
             it.n_it = -1;
-            if (valid) it = item_of(a, e, a.tinfo[e.x]);
+            if (valid) it = item_of<kSub>(a, e, a.tinfo[e.x]);
             ok = publish(it);
             while (ok && it.n_it >= 0) {
                 // the next item's ticket now, its queue entry after this item's
@@ -782,12 +886,15 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 bool nx_valid = false;
                 if (it.n_it > 0) {
                     const int32_t* ql = item_qlist(a, it);
-                    // this item's query blocks, one batch of independent loads
-                    int v[kBwdChunk];
+                    const int nq = item_nq(a, it);
+                    // this item's query blocks, batches of independent loads
+                    for (int j0 = 0; j0 < kSub * kBwdChunk; j0 += kBwdChunk) {
+                        int v[kBwdChunk];
 #pragma unroll
-                    for (int j = 0; j < kBwdChunk; ++j) v[j] = j < it.n_it ? __ldg(ql + j) : 0;
+                        for (int j = 0; j < kBwdChunk; ++j) v[j] = j0 + j < nq ? __ldg(ql + j0 + j) : 0;
 #pragma unroll
-                    for (int j = 0; j < kBwdChunk; ++j) qls[j] = v[j];
+                        for (int j = 0; j < kBwdChunk; ++j) qls[j0 + j] = v[j];
+                    }
                     // K_t and V_t, once the previous item's S/dP MMAs have read theirs
                     if (kvc > 0 && !mbar_wait(bar(B_KVFREE), (kvc - 1) & 1, abort_flag, a.status)) {
                         ok = false;
@@ -808,23 +915,30 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                             ok = false;
                             break;
                         }
-                        const int qb = qls[i];
                         const uint32_t st = sb + kOffStage + s * kStage;
                         mbar_expect_tx(bar(B_QFULL + s), kStage);
-                        for (int hl = 0; hl < 2; ++hl)
-                            for (int dh = 0; dh < 2; ++dh) {
-                                tma_load_3d(st + dh * kHalf128 + hl * kHalf64, &tmQ, bar(B_QFULL + s),
-                                            dh * 64, qb * 64, hq0 + hl);
-                                tma_load_3d(st + kTile128 + dh * kHalf128 + hl * kHalf64, &tmdO,
-                                            bar(B_QFULL + s), dh * 64, qb * 64, hq0 + hl);
-                            }
+                        // kSub query blocks of kMq tokens, both heads (a short last
+                        // iteration repeats its last block; the rows are masked)
+#pragma unroll
+                        for (int j = 0; j < kSub; ++j) {
+                            const int e = i * kSub + j;
+                            const int qb = qls[e < nq ? e : nq - 1];
+                            const uint32_t r0 = (uint32_t)(j * kMq * 128);
+                            for (int hl = 0; hl < 2; ++hl)
+                                for (int dh = 0; dh < 2; ++dh) {
+                                    tma_load_3d(st + dh * kHalf128 + hl * kHalf64 + r0, &tmQ,
+                                                bar(B_QFULL + s), dh * 64, qb * kMq, hq0 + hl);
+                                    tma_load_3d(st + kTile128 + dh * kHalf128 + hl * kHalf64 + r0, &tmdO,
+                                                bar(B_QFULL + s), dh * 64, qb * kMq, hq0 + hl);
+                                }
+                        }
                     }
                     if (!ok) break;
                 } else {
                     e = entry_of(j_nx, nx_valid);
                 }
                 it.n_it = -1;
-                if (nx_valid) it = item_of(a, e, a.tinfo[e.x]);
+                if (nx_valid) it = item_of<kSub>(a, e, a.tinfo[e.x]);
                 ok = publish(it);
             }
             if (kvc > 0) mbar_wait_drain(bar(B_KV), (kvc - 1) & 1);
@@ -949,25 +1063,31 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             if (lane == 0) mbar_arrive(bar(B_IFREE + slot));
             if (it.n_it < 0) break;
             const int32_t* ql = item_qlist(a, it);
-            const int n_it = it.n_it, t = it.t, bg = it.bg;
+            const int n_it = it.n_it, t = it.t, bg = it.bg, nq = item_nq(a, it);
             const size_t hoff = (size_t)((bg / a.Hkv) * a.Hq + (bg % a.Hkv) * 2 + hl) * a.L;
-            // Row data (query block, lse, Delta) is fetched one iteration ahead so its
-            // global-memory latency overlaps the previous iteration.
-            auto fetch = [&](int it2, int& qb2, float& nl2, float& dl2) {
-                qb2 = __ldg(ql + it2);
-                const int i2 = qb2 * 64 + tok;
-                const bool v2 = i2 < a.L;
+            const int jr = tok / kMq, tt = tok % kMq;  // the row's query block in the iteration, token in it
+            // Row data (query block, its mask over the span's blocks, lse, Delta)
+            // is fetched one iteration ahead so its latency overlaps the previous one.
+            auto fetch = [&](int it2, int& qb2, uint32_t& mb2, float& nl2, float& dl2) {
+                const int e = it2 * kSub + jr;
+                const bool live = e < nq;
+                qb2 = live ? __ldg(ql + e) : -1;
+                mb2 = live ? span_mask<kSub>(a, bg, t, qb2) : 0u;
+                const int i2 = qb2 * kMq + tt;
+                const bool v2 = live && i2 < a.L;
                 nl2 = v2 ? -__ldg(a.lse + hoff + i2) * kLog2e : -INFINITY;
                 dl2 = v2 ? __ldg(a.delta + hoff + i2) : 0.f;
             };
             int qb_n = 0;
+            uint32_t mb_n = 0u;
             float nl_n = 0.f, dl_n = 0.f;
-            if (n_it > 0) fetch(0, qb_n, nl_n, dl_n);
+            if (n_it > 0) fetch(0, qb_n, mb_n, nl_n, dl_n);
             for (int i = 0; ok && i < n_it; ++i, ++gi) {
                 const int qb = qb_n;
+                const uint32_t mbits = mb_n;
                 const float neg_lse2 = nl_n;
                 const float dlt = dl_n;
-                if (i + 1 < n_it) fetch(i + 1, qb_n, nl_n, dl_n);
+                if (i + 1 < n_it) fetch(i + 1, qb_n, mb_n, nl_n, dl_n);
                 const int buf = gi & 1;
                 ok = mbar_wait(bar(B_SPFULL + buf), (gi >> 1) & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
@@ -975,21 +1095,28 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 tc_fence_after();
                 uint32_t sv[32], dp[32];
                 tmem_ld32x2(lane_base + col_s(buf) + 32 * kh, lane_base + col_dp(buf) + 32 * kh, sv, dp);
-                const bool diag = qb == t;
+                // the row's query block lies in this span: causal mask in its own block
+                const bool diag = qb >= 0 && qb / kSub == t;
+                const bool all = mbits == (1u << kSub) - 1u && !diag;  // every key of the tile
                 // P = 2^(S scale_log2 - lse log2 e), dS = P (dP - Delta), two keys at a
-                // time (packed f32x2); the causal mask only on the diagonal block
+                // time (packed f32x2); masks (blocks the row's query block did not
+                // select, its own block's later keys, padding rows) off the main path
                 const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
                 const float2 nl2v = make_float2(neg_lse2, neg_lse2), ndl = make_float2(-dlt, -dlt);
 #pragma unroll
                 for (int c = 0; c < 16; ++c) {
                     float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
-                    if (!diag) {
+                    if (all) {
                         pv.x = ex2_approx(pv.x);
                         pv.y = ex2_approx(pv.y);
                     } else {
                         const int key = 32 * kh + 2 * c;
-                        pv.x = key <= tok ? ex2_approx(pv.x) : 0.f;
-                        pv.y = key + 1 <= tok ? ex2_approx(pv.y) : 0.f;
+                        const int q0 = key / kMq, q1 = (key + 1) / kMq;
+                        const bool k0 = ((mbits >> q0) & 1u) && !(diag && t * kSub + q0 == qb && key % kMq > tt);
+                        const bool k1 = ((mbits >> q1) & 1u) &&
+                                        !(diag && t * kSub + q1 == qb && (key + 1) % kMq > tt);
+                        pv.x = k0 ? ex2_approx(pv.x) : 0.f;
+                        pv.y = k1 ? ex2_approx(pv.y) : 0.f;
                     }
                     const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
                     const float2 ds = __fmul2_rn(pv, d);
@@ -1057,7 +1184,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 volatile int* last_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 8);
                 if (threadIdx.x == 0)
                     *last_flag = (ok && info.slot >= 0 &&
-                                  atomicAdd(a.arrive + (size_t)bg * a.NQB + t, 1) == info.nch - 1);
+                                  atomicAdd(a.arrive + (size_t)bg * a.nrows + t, 1) == info.nch - 1);
                 named_barrier(1, 256);
                 store = ok && *last_flag;
                 named_barrier(1, 256);  // every thread has read the flag before it is reused
@@ -1109,61 +1236,74 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 
 }  // namespace
 
-bool dq_tc_fits(int topk) { return dq::smem_bytes(topk) <= kMaxDynSmem; }
+bool dq_tc_fits(int topk, int block_size) {
+    const size_t b = block_size == 16   ? dq::smem_bytes<4>(topk)
+                     : block_size == 32 ? dq::smem_bytes<2>(topk)
+                                        : dq::smem_bytes<1>(topk);
+    return b <= kMaxDynSmem;
+}
 
 cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* O,
                          const void* dO, const float* lse, float* delta, const int32_t* idx,
-                         const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                         const int32_t* cnt, const int32_t* ulist, const int32_t* ucnt,
+                         const uint8_t* umask, const phsa_shape& s, int topk, float sm_scale,
                          void* dQ, int* status, cudaStream_t st) {
-    const int NQB = (s.L + 63) / 64;
+    const int bm = s.block_size, kSub = 64 / bm;
+    const int NQB = (s.L + bm - 1) / bm, nsb = (s.L + 63) / 64;
     CUtensorMap tq, tk, tv, tdo;
     const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
-    if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) || !make_tmap_bf16_rows128(&tk, K, s.L, pk, 64) ||
-        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64))
+    // Q and dO in 64-row boxes (the span's tokens); K and V gathered in boxes of one block
+    if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) ||
+        !make_tmap_bf16_rows128(&tk, K, s.L, pk, (uint32_t)bm) ||
+        !make_tmap_bf16_rows128(&tv, V, s.L, pk, (uint32_t)bm) ||
+        !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64))
         return cudaErrorInvalidValue;
-    const size_t smem = dq::smem_bytes(topk);
-    cudaError_t e =
-        cudaFuncSetAttribute(dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const size_t smem = kSub == 1 ? dq::smem_bytes<1>(topk) : kSub == 2 ? dq::smem_bytes<2>(topk)
+                                                                         : dq::smem_bytes<4>(topk);
+    auto kern = kSub == 1 ? dq_tc_kernel<1> : kSub == 2 ? dq_tc_kernel<2> : dq_tc_kernel<4>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
-    const int units = s.B * s.Hkv * NQB;
-    DqArgs args{idx, cnt, lse, static_cast<const __nv_bfloat16*>(O), delta,
-                static_cast<__nv_bfloat16*>(dQ), status, s.Hq, s.Hkv, s.L, NQB, topk, units,
-                sm_scale * kLog2e, sm_scale};
+    const int units = s.B * s.Hkv * nsb;
+    DqArgs args{idx, cnt, ulist, ucnt, umask, lse, static_cast<const __nv_bfloat16*>(O), delta,
+                static_cast<__nv_bfloat16*>(dQ), status, s.Hq, s.Hkv, s.L, NQB, topk, units, nsb,
+                kSub * topk, sm_scale * kLog2e, sm_scale};
     ProfScope prof(K_BWD_DQ, st);
-    dq_tc_kernel<<<(unsigned)min(units, nsm), dq::kThreads, smem, st>>>(tq, tk, tv, tdo, args);
+    kern<<<(unsigned)min(units, nsm), dq::kThreads, smem, st>>>(tq, tk, tv, tdo, args);
     return cudaGetLastError();
 }
 
 cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
-                           const int32_t* qlist, const int2* queue, int* qctl,
-                           const phsa_shape& s, int topk, int work_max, int slot_max,
+                           const int32_t* qlist, const uint32_t* masks, const int2* queue,
+                           int* qctl, const phsa_shape& s, int topk, const BwdLayout& l,
                            float sm_scale, void* dK, void* dV, float* partial, int* arrive,
                            int* status, cudaStream_t st) {
-    const int NQB = (s.L + 63) / 64;
+    const int kSub = l.kSub, bm = s.block_size;
     CUtensorMap tq, tk, tv, tdo;
     const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
-    if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) || !make_tmap_bf16_rows128(&tk, K, s.L, pk, 64) ||
-        !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) || !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64))
+    // Q and dO in boxes of one query block (m rows); K and V in 64-key spans
+    if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, (uint32_t)bm) ||
+        !make_tmap_bf16_rows128(&tk, K, s.L, pk, 64) || !make_tmap_bf16_rows128(&tv, V, s.L, pk, 64) ||
+        !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, (uint32_t)bm))
         return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(dkdv_tc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kv::kSmem);
+    auto kern = kSub == 1 ? dkdv_tc_kernel<1> : kSub == 2 ? dkdv_tc_kernel<2> : dkdv_tc_kernel<4>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kv::kSmem);
     if (e != cudaSuccess) return e;
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
-    const long long qcap = (long long)s.B * s.Hkv * work_max;  // entries per queue class
-    KvArgs args{lse, delta, tinfo, qlist, queue, qctl, qctl + kQueueClasses, partial, arrive,
+    const long long qcap = (long long)s.B * s.Hkv * l.work_max;  // entries per queue class
+    KvArgs args{lse, delta, tinfo, qlist, masks, queue, qctl, qctl + kQueueClasses, partial, arrive,
                 static_cast<__nv_bfloat16*>(dK), static_cast<__nv_bfloat16*>(dV), status, qcap,
-                s.Hq, s.Hkv, s.L, NQB, topk, slot_max, sm_scale * kLog2e, sm_scale};
+                (long long)l.nqb * topk, s.Hq, s.Hkv, s.L, l.nrows, topk, l.slot_max, l.mwords,
+                l.chunk, sm_scale * kLog2e, sm_scale};
     ProfScope prof(K_BWD_DKDV, st);
-    dkdv_tc_kernel<<<(unsigned)(qcap < nsm ? qcap : nsm), kv::kThreads, kv::kSmem, st>>>(
-        tq, tk, tv, tdo, args);
+    kern<<<(unsigned)(qcap < nsm ? qcap : nsm), kv::kThreads, kv::kSmem, st>>>(tq, tk, tv, tdo, args);
     return cudaGetLastError();
 }
 

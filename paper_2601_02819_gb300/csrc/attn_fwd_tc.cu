@@ -51,6 +51,7 @@
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "tc_common.cuh"
+#include "union.cuh"
 
 namespace phsa {
 
@@ -135,89 +136,15 @@ __device__ __forceinline__ FwdUnit fwd_unit(const FwdTcArgs& a, int u) {
 }
 
 // Warp-collective (all 32 lanes): the union of the block lists of the span's
-// query blocks, ascending, with owner masks (bit j: query block j of the span
-// selected the block), into a list slot. Each list is validated as
-// compact_block_list does (-1 entries skipped silently; an entry outside
-// [0, qb] or not above the last accepted one skipped and recorded): an entry
-// is accepted when it is in range and above every earlier in-range entry. The
+// query blocks with owner masks (union.cuh) into a list slot; the
 // per-query-block bitmaps over [0, NQB) are left cleared.
 template <int kSub>
 __device__ __forceinline__ void stage_union(const FwdTcArgs& a, const FwdUnit& d, int* sl,
                                             uint32_t* bm, int lane) {
-    const int W = bitmap_words(a.NQB);
-    int hi = -1;
-    for (int j = 0; j < kSub; ++j) {
-        const int qbj = d.qb * kSub + j;
-        if (qbj >= a.NQB) break;
-        const long long lu = d.lu + j;
-        int n = __ldg(a.cnt + lu);
-        if (n < 0 || n > a.topk) {
-            if (lane == 0) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
-            n = n < 0 ? 0 : a.topk;
-        }
-        int carry = -1;  // the largest in-range entry so far
-        for (int e0 = 0; e0 < n; e0 += 32) {
-            const int e = e0 + lane;
-            const int t = e < n ? __ldg(a.idx + lu * a.topk + e) : -1;
-            const bool inr = t >= 0 && t <= qbj;
-            // exclusive prefix maximum of the in-range entries over the lanes
-            int pm = inr ? t : -1;
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const int y = __shfl_up_sync(0xffffffffu, pm, off);
-                if (lane >= off) pm = max(pm, y);
-            }
-            int before = __shfl_up_sync(0xffffffffu, pm, 1);
-            before = lane == 0 ? carry : max(before, carry);
-            const bool accept = inr && t > before;
-            if (e < n && t != -1 && !accept) set_status(a.status, PHSA_ERR_DEVICE_INDEX);
-            if (accept) {
-                atomicOr(bm + j * W + (t >> 5), 1u << (t & 31));
-                hi = max(hi, t);
-            }
-            carry = max(carry, __shfl_sync(0xffffffffu, pm, 31));
-        }
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, off));
-    __syncwarp();
     const int cap = list_cap(a.topk, kSub);
-    int* ul = sl + 1;
-    uint8_t* own = reinterpret_cast<uint8_t*>(sl + 1 + cap);
-    const int wn = hi >= 0 ? (hi >> 5) + 1 : 0;
-    int pos = 0;
-    for (int w0 = 0; w0 < wn; w0 += 32) {
-        const int w = w0 + lane;
-        uint32_t bj[kSub], u = 0u;
-#pragma unroll
-        for (int j = 0; j < kSub; ++j) {
-            bj[j] = w < wn ? bm[j * W + w] : 0u;
-            u |= bj[j];
-        }
-        const int c = __popc(u);
-        int incl = c;
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, off);
-            if (lane >= off) incl += y;
-        }
-        int p = pos + incl - c;
-        while (u) {
-            const int bit = __ffs(u) - 1;
-            u &= u - 1;
-            uint32_t m = 0;
-#pragma unroll
-            for (int j = 0; j < kSub; ++j) m |= ((bj[j] >> bit) & 1u) << j;
-            ul[p] = 32 * w + bit;
-            own[p] = (uint8_t)m;
-            ++p;
-        }
-        pos += __shfl_sync(0xffffffffu, incl, 31);
-        if (w < wn)
-#pragma unroll
-            for (int j = 0; j < kSub; ++j) bm[j * W + w] = 0u;
-    }
-    if (lane == 0) sl[0] = pos;
+    build_block_union<kSub>(a.idx, a.cnt, d.lu, d.qb * kSub, min(kSub, a.NQB - d.qb * kSub), a.topk,
+                            bm, bitmap_words(a.NQB), sl + 1, reinterpret_cast<uint8_t*>(sl + 1 + cap),
+                            sl, a.status, lane);
     __threadfence_block();
     __syncwarp();
 }

@@ -61,9 +61,8 @@ extern "C" int phsa_sparse_attn_bwd_noalloc(const void* Q, const void* K, const 
                                             void* dK, void* dV, void* stream) {
     // The same checks, in the same order and with the same codes, as
     // phsa_sparse_attn_bwd; only the workspace check differs (the fixed array).
-    int rc = phsa::validate_shape(s);
+    const int rc = phsa::validate_bwd(s, topk);
     if (rc != PHSA_OK) return rc;
-    if ((rc = phsa::validate_topk(s, topk)) != PHSA_OK) return rc;
     if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (s.B == 0 || s.L == 0) return PHSA_OK;
     if (!Q || !K || !V || !O || !dO || !lse || !block_idx || !block_cnt || !dQ || !dK || !dV)

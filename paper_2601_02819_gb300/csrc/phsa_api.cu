@@ -58,12 +58,24 @@ int check_topk(const phsa_shape& s, int topk) {
     return PHSA_OK;
 }
 
+// The backward takes block sizes 16 and 32 for GQA pairs (two query heads
+// per KV head, the tcgen05 kernels) when their lists fit in shared memory.
+int check_bwd(const phsa_shape& s, int topk) {
+    int rc = check_shape(s, true);
+    if (rc != PHSA_OK) return rc;
+    if ((rc = check_topk(s, topk)) != PHSA_OK) return rc;
+    if (s.block_size != phsa::kM && (s.Hq != 2 * s.Hkv || !phsa::dq_tc_fits(topk, s.block_size)))
+        return PHSA_ERR_UNSUPPORTED;
+    return PHSA_OK;
+}
+
 }  // namespace
 
 namespace phsa {
 // The status word of the current device, for entry points in other files.
 int* device_status_word() { return status_ptr(); }
 int validate_shape(const phsa_shape& s) { return check_shape(s); }
+int validate_bwd(const phsa_shape& s, int topk) { return check_bwd(s, topk); }
 int validate_topk(const phsa_shape& s, int topk) { return check_topk(s, topk); }
 int status_of(cudaError_t e) { return from_cuda(e); }
 }  // namespace phsa
@@ -118,7 +130,7 @@ int phsa_sparse_attn_fwd(const void* Q, const void* K, const void* V, const int3
 }
 
 size_t phsa_sparse_attn_bwd_workspace(phsa_shape s, int topk) {
-    if (check_shape(s) != PHSA_OK || check_topk(s, topk) != PHSA_OK) return 0;
+    if (check_bwd(s, topk) != PHSA_OK) return 0;
     if (empty(s)) return 0;
     return phsa::bwd_layout(s, topk).total;
 }
@@ -128,9 +140,8 @@ int phsa_sparse_attn_bwd(const void* Q, const void* K, const void* V, const void
                          const int32_t* block_cnt, phsa_shape s, int topk, float sm_scale,
                          void* workspace, size_t workspace_bytes, void* dQ, void* dK, void* dV,
                          void* stream) {
-    int rc = check_shape(s);
+    const int rc = check_bwd(s, topk);
     if (rc != PHSA_OK) return rc;
-    if ((rc = check_topk(s, topk)) != PHSA_OK) return rc;
     if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (empty(s)) return PHSA_OK;
     if (!Q || !K || !V || !O || !dO || !lse || !block_idx || !block_cnt || !dQ || !dK || !dV)

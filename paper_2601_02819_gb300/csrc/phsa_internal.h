@@ -120,25 +120,37 @@ __host__ __device__ __forceinline__ int queue_class(int n_it) {
 }
 
 // tcgen05 backward kernels for G = 2 (attn_bwd_tc.cu).
+struct BwdLayout;
 cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
-                           const int32_t* qlist, const int2* queue, int* qctl,
-                           const phsa_shape& s, int topk, int work_max, int slot_max,
+                           const int32_t* qlist, const uint32_t* masks, const int2* queue,
+                           int* qctl, const phsa_shape& s, int topk, const BwdLayout& l,
                            float sm_scale, void* dK, void* dV, float* partial, int* arrive,
                            int* status, cudaStream_t st);
-// Whether dq_tc_kernel's shared memory (tiles + the block list) fits for topk.
-bool dq_tc_fits(int topk);
+// Whether dq_tc_kernel's shared memory (tiles + the block list) fits for topk
+// at block size m.
+bool dq_tc_fits(int topk, int block_size = 64);
+// dQ (and Delta). At m < 64 the span lists are ulist/ucnt/umask (the unions
+// of the span's query-block lists); at m = 64, idx/cnt.
 cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void* O,
                          const void* dO, const float* lse, float* delta, const int32_t* idx,
-                         const int32_t* cnt, const phsa_shape& s, int topk, float sm_scale,
+                         const int32_t* cnt, const int32_t* ulist, const int32_t* ucnt,
+                         const uint8_t* umask, const phsa_shape& s, int topk, float sm_scale,
                          void* dQ, int* status, cudaStream_t st);
 
-// Backward workspace layout (all offsets 256-byte aligned).
+// Backward workspace layout (all offsets 256-byte aligned). The transposed
+// selection has one row per KV span of 64 keys and one column per query block
+// of m tokens (at m = 64 a span is a block); at m < 64 a mask row per span
+// records which of its kSub blocks each query block selected, and the dQ pass
+// reads the union of each span's query-block lists (ucnt, ulist, umask).
 struct BwdLayout {
     // qctl: item counts of the kQueueClasses queue classes, then the ticket
-    // counter of the persistent dK/dV kernel (zeroed with bits by one memset)
-    size_t qctl, bits, tinfo, qlist, work, nwork, queue, delta, partial, arrive, total;
-    int nqb, words, chunk, work_max, slot_max;
+    // counter of the persistent dK/dV kernel (zeroed with bits and masks by one memset)
+    size_t qctl, bits, masks, tinfo, qlist, work, nwork, queue, delta, partial, arrive, ucnt, ulist,
+        umask, total;
+    int nqb;    // query blocks of m tokens
+    int nrows;  // KV spans of 64 keys
+    int kSub, words, mwords, chunk, work_max, slot_max, ucap;
 };
 BwdLayout bwd_layout(const phsa_shape& s, int topk);
 
@@ -156,6 +168,8 @@ int* device_status_word();
 int status_of(cudaError_t e);
 // Shape and budget checks of the C ABI (phsa_api.cu): PHSA_OK or an error code.
 int validate_shape(const phsa_shape& s);
+// The backward's shape and budget checks (block sizes 16 and 32 for GQA pairs).
+int validate_bwd(const phsa_shape& s, int topk);
 int validate_topk(const phsa_shape& s, int topk);
 // Shared-memory bytes of the selection kernel for this shape and budget.
 size_t select_smem_bytes(const phsa_shape& s, int topk);

@@ -239,13 +239,16 @@ def phsa_sparse_attn_fwd(Q, K, V, block_idx, block_cnt, sm_scale: float | None =
     return O, lse
 
 
-def phsa_sparse_attn_bwd_workspace(B, L, Hq, Hkv, topk, D=HEAD_DIM) -> int:
-    return int(load().phsa_sparse_attn_bwd_workspace(make_shape(B, L, Hq, Hkv, D), int(topk)))
+def phsa_sparse_attn_bwd_workspace(B, L, Hq, Hkv, topk, D=HEAD_DIM, block_size=BLOCK_SIZE) -> int:
+    return int(load().phsa_sparse_attn_bwd_workspace(make_shape(B, L, Hq, Hkv, D, block_size),
+                                                     int(topk)))
 
 
 def phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_scale=None,
-                         workspace=None, dQ=None, dK=None, dV=None, stream=None):
-    """Stage (c) backward: (dQ, dK, dV) in bf16."""
+                         workspace=None, dQ=None, dK=None, dV=None, stream=None,
+                         block_size=BLOCK_SIZE):
+    """Stage (c) backward: (dQ, dK, dV) in bf16 (block sizes 16 and 32 for two
+    query heads per KV head)."""
     for name, t in (("Q", Q), ("K", K), ("V", V), ("O", O), ("dO", dO)):
         _check(t, name, torch.bfloat16, 4)
     _check(lse, "lse", torch.float32, 3)
@@ -256,7 +259,7 @@ def phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_scale=Non
     topk = block_idx.shape[-1]
     if sm_scale is None:
         sm_scale = D ** -0.5
-    ws_bytes = phsa_sparse_attn_bwd_workspace(B, L, Hq, Hkv, topk, D)
+    ws_bytes = phsa_sparse_attn_bwd_workspace(B, L, Hq, Hkv, topk, D, block_size)
     if workspace is None:
         workspace = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=Q.device)
     _check(workspace, "workspace", torch.uint8, 1)
@@ -265,7 +268,7 @@ def phsa_sparse_attn_bwd(Q, K, V, O, dO, lse, block_idx, block_cnt, sm_scale=Non
     dV = torch.empty_like(V) if dV is None else dV
     rc = load().phsa_sparse_attn_bwd(
         _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(dO), _ptr(lse), _ptr(block_idx), _ptr(block_cnt),
-        make_shape(B, L, Hq, Hkv, D), int(topk), float(sm_scale), _ptr(workspace),
+        make_shape(B, L, Hq, Hkv, D, block_size), int(topk), float(sm_scale), _ptr(workspace),
         ctypes.c_size_t(workspace.numel()), _ptr(dQ), _ptr(dK), _ptr(dV), _stream(stream))
     _raise("phsa_sparse_attn_bwd", rc)
     return dQ, dK, dV

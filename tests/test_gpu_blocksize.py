@@ -257,3 +257,37 @@ def test_selection_warp_mma_pair_kernels_on_short_inputs(m, aggregation):
         assert phsa.phsa_get_device_status() == 0
     finally:
         phsa.phsa_test_set_select_tc_limit(prev)
+
+
+@pytest.mark.parametrize("m,B,Hq,Hkv,L,topk,n_init,n_local", [
+    (16, 1, 2, 1, 16 * 70 + 9, 7, 1, 1),     # ragged tail; four blocks of 16 per 64-key span
+    (16, 2, 4, 2, 16 * 33, 5, 1, 1),         # B = 2, two KV heads
+    (16, 1, 2, 1, 16 * 300 + 5, 20, 2, 8),   # the first spans' lists exceed one work item (128)
+    (16, 1, 2, 1, 16 * 24, 30, 1, 1),        # budget covers everything: dense rows
+    (32, 1, 4, 2, 32 * 25 + 17, 4, 1, 1),    # m = 32: two blocks per span
+    (32, 1, 2, 1, 32 * 150 + 31, 9, 2, 2),   # m = 32, lists over one work item (64)
+])
+def test_backward_matches_oracle(m, B, Hq, Hkv, L, topk, n_init, n_local):
+    # The backward at the paper's block size on the tcgen05 kernels: dQ over the
+    # union of a span's lists, dK/dV over 64-key spans with gathered query blocks.
+    rng = np.random.default_rng(L * 5 + m)
+    Q, K, V = rand(rng, B, Hq, L, D), rand(rng, B, Hkv, L, D), rand(rng, B, Hkv, L, D)
+    dO = rand(rng, B, Hq, L, D)
+    mask = (rng.random((B, L)) < 0.06).astype(np.uint8)
+    Kr = oracle.block_repr(K, mask, m, 0.5)
+    idx, cnt = oracle.select_blocks(Q, Kr, L, m, topk, n_init, n_local, SCALE)
+    it, ct = torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda()
+    Qd, Kd, Vd, dOd = (to_dev_bf16(x) for x in (Q, K, V, dO))
+    O, lse = phsa.phsa_sparse_attn_fwd(Qd, Kd, Vd, it, ct, block_size=m)
+    dQ, dK, dV = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct, block_size=m)
+    torch.cuda.synchronize()
+    assert phsa.phsa_get_device_status() == 0
+    rq, rk, rv = oracle.sparse_attn_bwd(Q, K, V, dO, idx, cnt, m, SCALE)
+    assert_close("dQ", bf16_to_f64(dQ), rq)
+    assert_close("dK", bf16_to_f64(dK), rk)
+    assert_close("dV", bf16_to_f64(dV), rv)
+
+
+def test_backward_at_m16_rejects_a_single_query_head_per_kv_head():
+    B, Hq, Hkv, L = 1, 2, 2, 16 * 8
+    assert phsa.phsa_sparse_attn_bwd_workspace(B, L, Hq, Hkv, 4, block_size=16) == 0
