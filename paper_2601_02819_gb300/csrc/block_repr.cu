@@ -109,14 +109,14 @@ block_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict
 // Decode: one CTA of four warps per (sequence, KV head). A sequence whose
 // length is a positive multiple of m has just filled its last block: that
 // block's representative key is computed (Eq. 6-8, the arithmetic of
-// repr_one_block); nothing else is touched. Warp w sums rows [16w, 16w + 16)
-// with all of its 16-byte loads issued at once; the four partial sums are
-// added in warp order in shared memory.
+// repr_one_block); nothing else is touched. Warp w < m / 16 sums rows
+// [16w, 16w + 16) with all of its 16-byte loads issued at once; the m / 16
+// partial sums are added in warp order in shared memory.
 constexpr int kDecReprWarps = 4;
 
 __global__ void __launch_bounds__(kDecReprWarps * 32)
 decode_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restrict__ mask,
-                   const int32_t* __restrict__ lens, int Hkv, int L, int T, float lambda,
+                   const int32_t* __restrict__ lens, int Hkv, int L, int T, int bm, float lambda,
                    __nv_bfloat16* __restrict__ Krepr, int* status) {
     __shared__ float part[kDecReprWarps][2][kD];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -127,47 +127,50 @@ decode_repr_kernel(const __nv_bfloat16* __restrict__ K, const uint8_t* __restric
         if (threadIdx.x == 0) set_status(status, PHSA_ERR_DEVICE_INDEX);
         return;
     }
-    if (len == 0 || len % kM != 0) return;
-    const int t = len / kM - 1;
-    const uint8_t* mb = mask + (size_t)b * L + (size_t)t * kM;
-    const unsigned lo = __ballot_sync(0xffffffffu, mb[lane] != 0);
-    const unsigned hi = __ballot_sync(0xffffffffu, mb[32 + lane] != 0);
+    if (len == 0 || len % bm != 0) return;
+    const int t = len / bm - 1;
+    const uint8_t* mb = mask + (size_t)b * L + (size_t)t * bm;
+    const unsigned lo = __ballot_sync(0xffffffffu, lane < bm && mb[lane] != 0);
+    const unsigned hi = __ballot_sync(0xffffffffu, bm > 32 && mb[bm > 32 ? 32 + lane : 0] != 0);
     const int c = __popc(lo) + __popc(hi);
     const int half = lane >> 4, col = lane & 15;
-    const __nv_bfloat16* kb = K + ((size_t)bg * L + (size_t)t * kM + 16 * warp) * kD + col * 8;
-    uint4 v[8];
+    const int nw = bm / 16;  // warps with rows
+    if (warp < nw) {
+        const __nv_bfloat16* kb = K + ((size_t)bg * L + (size_t)t * bm + 16 * warp) * kD + col * 8;
+        uint4 v[8];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) v[u] = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)(2 * u + half) * kD));
-    float s0[8], sp[8];
+        for (int u = 0; u < 8; ++u)
+            v[u] = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)(2 * u + half) * kD));
+        float s0[8], sp[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) { s0[j] = 0.f; sp[j] = 0.f; }
+        for (int j = 0; j < 8; ++j) { s0[j] = 0.f; sp[j] = 0.f; }
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-        const int r = 16 * warp + 2 * u + half;
-        add8(s0, v[u]);
-        if (((r < 32 ? lo >> r : hi >> (r - 32)) & 1u) != 0) add8(sp, v[u]);
-    }
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        s0[j] += __shfl_xor_sync(0xffffffffu, s0[j], 16);
-        sp[j] += __shfl_xor_sync(0xffffffffu, sp[j], 16);
-    }
-    if (half == 0) {
+        for (int u = 0; u < 8; ++u) {
+            const int r = 16 * warp + 2 * u + half;
+            add8(s0, v[u]);
+            if (((r < 32 ? lo >> r : hi >> (r - 32)) & 1u) != 0) add8(sp, v[u]);
+        }
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-            part[warp][0][col * 8 + j] = s0[j];
-            part[warp][1][col * 8 + j] = sp[j];
+            s0[j] += __shfl_xor_sync(0xffffffffu, s0[j], 16);
+            sp[j] += __shfl_xor_sync(0xffffffffu, sp[j], 16);
+        }
+        if (half == 0) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                part[warp][0][col * 8 + j] = s0[j];
+                part[warp][1][col * 8 + j] = sp[j];
+            }
         }
     }
     __syncthreads();
     const int d = threadIdx.x;  // one column per thread
     float a0 = 0.f, ap = 0.f;
-#pragma unroll
-    for (int w = 0; w < kDecReprWarps; ++w) {
+    for (int w = 0; w < nw; ++w) {
         a0 += part[w][0][d];
         ap += part[w][1][d];
     }
-    const float m0 = a0 * (1.0f / kM);                               // Eq. 6
+    const float m0 = a0 * (1.0f / (float)bm);                        // Eq. 6
     const float o = c > 0 ? lambda * m0 + (1.0f - lambda) * (ap * (1.0f / (float)c))  // Eq. 7-8
                           : m0;                                      // no punctuation
     Krepr[((size_t)bg * T + t) * kD + d] = __float2bfloat16_rn(o);
@@ -198,12 +201,14 @@ namespace phsa {
 cudaError_t launch_decode_repr(const void* K, const uint8_t* mask, const int32_t* lens,
                                const phsa_shape& s, float lambda, void* Krepr, int* status,
                                cudaStream_t st) {
-    const int T = s.L / kM;
+    const int bm = s.block_size;
+    if (bm != 16 && bm != 32 && bm != 64) return cudaErrorInvalidValue;
+    const int T = s.L / bm;
     const long long n_units = (long long)s.B * s.Hkv;
     if (n_units == 0 || T == 0) return cudaSuccess;
     ProfScope prof(K_DEC_REPR, st);
     decode_repr_kernel<<<(unsigned)n_units, kDecReprWarps * 32, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(K), mask, lens, s.Hkv, s.L, T, lambda,
+        static_cast<const __nv_bfloat16*>(K), mask, lens, s.Hkv, s.L, T, bm, lambda,
         static_cast<__nv_bfloat16*>(Krepr), status);
     return cudaGetLastError();
 }

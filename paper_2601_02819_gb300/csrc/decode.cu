@@ -4,16 +4,18 @@
 // selection itself is in decode_select_tc.cu.
 //
 // The kernel reads little per unit (sequence, KV head) and is bound by HBM
-// bandwidth, so it runs on the CUDA cores. Every selected K or V block is 64
-// consecutive rows, so a producer warp streams them into a shared-memory ring
-// with 1-D bulk copies (cp.async.bulk, completion counted on an mbarrier per
-// slot) and the compute warps work from shared memory: a half-warp per
-// 256-byte key row (lane c holds columns 8c..8c+7). The kernel is persistent:
+// bandwidth, so it runs on the CUDA cores. Every selected K or V block is m
+// consecutive rows (m = 16, 32 or 64), so a producer warp streams them into a
+// shared-memory ring with 1-D bulk copies (cp.async.bulk, completion counted
+// on an mbarrier per slot) and the compute warps work from shared memory: a
+// half-warp per 256-byte key row (lane c holds columns 8c..8c+7). A ring slot
+// holds 64 rows: 64 / m consecutive entries of the block list, each at row
+// offset j m of the slot. The kernel is persistent:
 // a CTA walks the units u = blockIdx.x, blockIdx.x + gridDim.x, ..., and its
 // ring runs across unit boundaries, so the next unit's blocks are in flight
 // while a unit finishes.
 //
-// Each half-warp runs an online softmax over 4 keys of every selected block;
+// Each half-warp runs an online softmax over 4 keys of every slot;
 // the 16 partial states are merged (two per warp with shuffles, then the 8
 // warps in shared memory). Keys after p (the unfilled part of the local block)
 // are neither copied nor attended. Optionally the kernel also refreshes the
@@ -33,7 +35,7 @@ using namespace tc;
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kRowBytes = kD * 2;                  // one bf16 key row
-constexpr int kSlotRows = 64;                      // rows per ring slot (one block)
+constexpr int kSlotRows = 64;                      // rows per ring slot (64 / m blocks)
 constexpr int kSlotBytes = kSlotRows * kRowBytes;  // 16 KB
 constexpr int kAttnSlots = 3;                      // attention ring: 3 x (K, V) = 96 KB
 
@@ -119,9 +121,10 @@ size_t dec_attn_smem(int G, int topk) {
            (size_t)kWarps * G * 130 * 4 + 4 * 2 * kD * 4;
 }
 
-template <int G>
+template <int G, int kBm>
 __global__ void __launch_bounds__(kAttnThreads, 2)
 decode_attn_kernel(const DecAttnArgs a) {
+    constexpr int kSub = kSlotRows / kBm;  // blocks per ring slot
     extern __shared__ __align__(128) uint8_t smem[];
     const uint32_t sb = smem_u32(smem);
     auto bar = [&](int i) { return sb + kAttnOffBar + 8u * (uint32_t)i; };
@@ -166,13 +169,13 @@ decode_attn_kernel(const DecAttnArgs a) {
                     reinterpret_cast<const uint4*>(a.q + ((size_t)b * a.Hq + g * G) * kD) + lane);
             int n = 0;
             if (valid)
-                n = stage_list_warp(a.idx + (size_t)u * a.topk, a.cnt + u, a.topk, (len - 1) / kM,
-                                    list, a.status, lane);
+                n = stage_list_warp(a.idx + (size_t)u * a.topk, a.cnt + u, a.topk,
+                                    (len - 1) / kBm, list, a.status, lane);
             unsigned plo = 0, phi = 0;
-            if (refresh && valid && len % kM == 0) {
-                const uint8_t* mb = a.mask + (size_t)b * a.L + (size_t)(len / kM - 1) * kM;
-                plo = __ballot_sync(0xffffffffu, mb[lane] != 0);
-                phi = __ballot_sync(0xffffffffu, mb[32 + lane] != 0);
+            if (refresh && valid && len % kBm == 0) {  // the m flags of the just-filled block
+                const uint8_t* mb = a.mask + (size_t)b * a.L + (size_t)(len - kBm);
+                plo = __ballot_sync(0xffffffffu, lane < kBm && mb[lane] != 0);
+                phi = __ballot_sync(0xffffffffu, kBm > 32 && mb[kBm > 32 ? 32 + lane : 0] != 0);
             }
             if (lane == 0) {
                 hdr[0] = len;
@@ -186,7 +189,7 @@ decode_attn_kernel(const DecAttnArgs a) {
         // Event loop: a copy whenever a ring slot is free and the next block is
         // known; otherwise stage the next unit (up to two ahead of the copies),
         // so that the loads of staging never hold back a copy.
-        int staged = -1, ik = 0, ii = 0;  // last unit staged; copy cursor (unit, block)
+        int staged = -1, ik = 0, ii = 0;  // last unit staged; copy cursor (unit, ring slot)
         Deadline dl;
         while (ok) {
             bool progressed = false;
@@ -194,7 +197,7 @@ decode_attn_kernel(const DecAttnArgs a) {
             if (more && ik <= staged) {
                 const int* hdr = reinterpret_cast<const int*>(units0 + (ik % kUnitSlots) * ubytes);
                 const int n = hdr[1];
-                if (ii >= n) {
+                if (ii * kSub >= n) {
                     ++ik;
                     ii = 0;
                     continue;
@@ -206,15 +209,26 @@ decode_attn_kernel(const DecAttnArgs a) {
                 free_slot = __shfl_sync(0xffffffffu, free_slot, 0) != 0;
                 if (free_slot) {
                     if (lane == 0) {
-                        const int t = hdr[4 + G * kD / 2 + ii];
-                        const int len = hdr[0], p = len - 1;
-                        const int rows = t == p / kM ? p - t * kM + 1 : kM;  // keys up to p
-                        const size_t off = ((size_t)unit_of(ik) * a.L + (size_t)t * kM) * kD;
-                        const uint32_t bytes = (uint32_t)rows * kRowBytes;
-                        mbar_expect_tx(bar(kAB_FULL + sl), 2 * bytes);
-                        bulk_load(sb + sl * 2 * kSlotBytes, a.K + off, bytes, bar(kAB_FULL + sl));
-                        bulk_load(sb + sl * 2 * kSlotBytes + kSlotBytes, a.V + off, bytes,
-                                  bar(kAB_FULL + sl));
+                        // entries e0 .. e1 - 1 of the list, entry e0 + j at slot row j m
+                        const int* lst = hdr + 4 + G * kD / 2;
+                        const int len = hdr[0], p = len - 1, qb = p / kBm;
+                        const int e0 = ii * kSub, e1 = min(n, e0 + kSub);
+                        uint32_t total = 0;
+                        for (int e = e0; e < e1; ++e) {
+                            const int t = lst[e];
+                            total += (uint32_t)(t == qb ? p - t * kBm + 1 : kBm) * kRowBytes;
+                        }
+                        mbar_expect_tx(bar(kAB_FULL + sl), 2 * total);
+                        for (int e = e0; e < e1; ++e) {
+                            const int t = lst[e];
+                            const int rows = t == qb ? p - t * kBm + 1 : kBm;  // keys up to p
+                            const size_t off = ((size_t)unit_of(ik) * a.L + (size_t)t * kBm) * kD;
+                            const uint32_t bytes = (uint32_t)rows * kRowBytes;
+                            const uint32_t dst = sb + sl * 2 * kSlotBytes +
+                                                 (uint32_t)((e - e0) * kBm) * kRowBytes;
+                            bulk_load(dst, a.K + off, bytes, bar(kAB_FULL + sl));
+                            bulk_load(dst + kSlotBytes, a.V + off, bytes, bar(kAB_FULL + sl));
+                        }
                     }
                     ++issued;
                     ++ii;
@@ -281,8 +295,8 @@ decode_attn_kernel(const DecAttnArgs a) {
             if (lane == 0) mbar_arrive(bar(kAB_UFREE + us));
             continue;
         }
-        const int p = len - 1, qb = p / kM;
-        const bool fill = refresh && len % kM == 0;  // refresh block qb's representative key
+        const int p = len - 1, qb = p / kBm;
+        const bool fill = refresh && len % kBm == 0;  // refresh block qb's representative key
         float qv[G][8];
 #pragma unroll
         for (int h = 0; h < G; ++h) {
@@ -304,12 +318,16 @@ decode_attn_kernel(const DecAttnArgs a) {
             for (int e = 0; e < 8; ++e) o[h][e] = 0.f;
         }
         bool filled = false;
-        // Half-warp hw takes keys [4 hw, 4 hw + 4) of each block: four consecutive rows.
-        for (int i = 0; i < nb; ++i, ++gc) {
+        // Half-warp hw takes slot rows [4 hw, 4 hw + 4): four consecutive keys of
+        // one block (list entry i sub + jh), from its row rh on.
+        const int jh = (4 * hw) / kBm, rh = 4 * hw - jh * kBm;
+        const int ng = (nb + kSub - 1) / kSub;
+        for (int i = 0; i < ng; ++i, ++gc) {
             const int sl = gc % kAttnSlots;
             ok = ok && mbar_wait(bar(kAB_FULL + sl), (gc / kAttnSlots) & 1, abort_flag, a.status);
-            const int t = list[i];
-            const int rows = t == qb ? p - t * kM + 1 : kM;
+            const int e = i * kSub + jh;
+            const int t = e < nb ? list[e] : -1;
+            const int rows = t < 0 ? 0 : t == qb ? p - t * kBm + 1 : kBm;
             const uint8_t* ks = smem + sl * 2 * kSlotBytes;
             const uint8_t* vs = ks + kSlotBytes;
             // scores first, then the values: K and V fragments are not live together
@@ -318,7 +336,7 @@ decode_attn_kernel(const DecAttnArgs a) {
 #pragma unroll
             for (int r = 0; r < 4; ++r) {
                 const int key = 4 * hw + r;
-                vis[r] = ok && key < rows;
+                vis[r] = ok && rh + r < rows;
                 const uint4 kr = vis[r] ? *reinterpret_cast<const uint4*>(ks + key * kRowBytes + c16 * 16)
                                         : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
@@ -359,11 +377,14 @@ decode_attn_kernel(const DecAttnArgs a) {
                 }
                 m[h] = mn;
             }
-            if (fill && t == qb && ok && warp < 4) {
-                // Eq. 6-8 over the 64 rows in the slot, in the summation order of
-                // decode_repr_kernel: warp w rows [16w, 16w + 16), even and odd rows
-                // per lane half, halves added, then the warps in order
+            // the slot's entry for block qb (the list's last, when present)
+            const int eq = min(nb, i * kSub + kSub) - 1;
+            if (fill && ok && eq >= i * kSub && list[eq] == qb && warp < kBm / 16) {
+                // Eq. 6-8 over the block's m rows in the slot, in the summation order
+                // of decode_repr_kernel: warp w rows [16w, 16w + 16), even and odd
+                // rows per lane half, halves added, then the warps in order
                 const int half = lane >> 4, col = lane & 15;
+                const uint8_t* kq = ks + (size_t)((eq - i * kSub) * kBm) * kRowBytes;
                 float s0[8], sp[8];
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
@@ -373,7 +394,7 @@ decode_attn_kernel(const DecAttnArgs a) {
 #pragma unroll
                 for (int uu = 0; uu < 8; ++uu) {
                     const int r = 16 * warp + 2 * uu + half;
-                    const uint4 kv = *reinterpret_cast<const uint4*>(ks + r * kRowBytes + col * 16);
+                    const uint4 kv = *reinterpret_cast<const uint4*>(kq + r * kRowBytes + col * 16);
                     const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
                     const bool pu = ((r < 32 ? plo >> r : phi >> (r - 32)) & 1u) != 0;
 #pragma unroll
@@ -448,13 +469,12 @@ decode_attn_kernel(const DecAttnArgs a) {
         }
         if (ok && filled && tid < kD) {
             float a0 = 0.f, ap = 0.f;
-#pragma unroll
-            for (int w = 0; w < 4; ++w) {
+            for (int w = 0; w < kBm / 16; ++w) {
                 a0 += rpart[(w * 2 + 0) * kD + tid];
                 ap += rpart[(w * 2 + 1) * kD + tid];
             }
             const int c = __popc(plo) + __popc(phi);
-            const float m0 = a0 * (1.0f / kM);  // Eq. 6
+            const float m0 = a0 * (1.0f / (float)kBm);  // Eq. 6
             const float ov = c > 0 ? a.lambda * m0 + (1.0f - a.lambda) * (ap * (1.0f / (float)c))
                                    : m0;  // Eq. 7-8; no punctuation: the mean
             a.Krepr[((size_t)u * a.T + qb) * kD + tid] = __float2bfloat16_rn(ov);
@@ -498,9 +518,15 @@ cudaError_t launch_decode_attn_any(const void* q, const void* K, const void* V, 
     DecAttnArgs args{static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(K),
                      static_cast<const __nv_bfloat16*>(V), idx, cnt, lens,
                      static_cast<__nv_bfloat16*>(O), lse, status, mask,
-                     static_cast<__nv_bfloat16*>(Krepr), lambda, s.Hq, s.Hkv, s.L, s.L / kM, topk,
-                     (int)units, sm_scale * kLog2e};
-    auto kern = G == 2 ? decode_attn_kernel<2> : decode_attn_kernel<1>;
+                     static_cast<__nv_bfloat16*>(Krepr), lambda, s.Hq, s.Hkv, s.L,
+                     s.L / s.block_size, topk, (int)units, sm_scale * kLog2e};
+    const int bm = s.block_size;
+    auto kern = G == 2 ? (bm == 16   ? decode_attn_kernel<2, 16>
+                          : bm == 32 ? decode_attn_kernel<2, 32>
+                                     : decode_attn_kernel<2, 64>)
+                       : (bm == 16   ? decode_attn_kernel<1, 16>
+                          : bm == 32 ? decode_attn_kernel<1, 32>
+                                     : decode_attn_kernel<1, 64>);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     unsigned grid = 0;

@@ -66,7 +66,7 @@ struct Args {
     int32_t* idx;
     int32_t* cnt;
     int* status;
-    int Hq, Hkv, L, Tc, topk, n_init, n_local, units, slots, agg;
+    int Hq, Hkv, L, Tc, topk, n_init, n_local, units, slots, agg, bm;
     float scale_log2, scale;
 };
 
@@ -79,7 +79,7 @@ struct SelUnit {
 __device__ __forceinline__ SelUnit sel_unit(const Args& a, int len) {
     SelUnit s{};
     if (len <= 0 || len > a.L) return s;
-    s.qb = (len - 1) / kM;
+    s.qb = (len - 1) / a.bm;
     s.n_init_q = min(a.n_init, s.qb + 1);              // forced initial [0, n_init_q)
     s.loc_lo = max(s.n_init_q, s.qb - a.n_local + 1);  // forced local [loc_lo, qb]
     s.c_lo = a.n_init;                                 // candidates [c_lo, qb - n_local]
@@ -490,7 +490,13 @@ decode_select_tc_kernel(const __grid_constant__ CUtensorMap tmKr,
                         for (int rr = 1; rr < kRegKeys; ++rr) best = topk::umax64(best, key[rr]);
                     }
                 }
-            } else {  // long contexts: rounds over shared memory; a pick is marked by a NaN score
+            } else if (ksel <= 32) {
+                // long candidate lists: 512 keys at a time in registers, with the
+                // best ksel so far carried in one register per lane
+                const unsigned long long mine = topk::warp_topk32(nC, ksel, key_of, lane);
+                if (lane < ksel) sel[lane] = topk::key_block(mine);
+            } else {  // long lists, large budgets: rounds over shared memory; a pick is
+                      // marked by a NaN score
                 topk::rounds_one_warp(
                     nC, ksel, key_of, [&](int cj) { return Sb[cj] != Sb[cj]; },
                     [&](int t) { Sb[t - c_lo] = __int_as_float(0x7fc00000); }, sel, lane);
@@ -525,7 +531,7 @@ decode_select_tc_kernel(const __grid_constant__ CUtensorMap tmKr,
 }  // namespace
 
 size_t decode_select_smem_bytes(const phsa_shape& s, int topk) {
-    const int G = s.Hq / s.Hkv, Tc = s.L / kM;
+    const int G = s.Hq / s.Hkv, Tc = s.L / s.block_size;
     const int n = ring_slots(G, Tc, topk);
     return n > 0 ? smem_bytes(G, Tc, topk, n) : (size_t)-1;
 }
@@ -533,7 +539,7 @@ size_t decode_select_smem_bytes(const phsa_shape& s, int topk) {
 cudaError_t launch_decode_select(const void* q, const void* Krepr, const int32_t* lens,
                                  const phsa_shape& s, const phsa_select_params& p, int32_t* idx,
                                  int32_t* cnt, int* status, cudaStream_t st) {
-    const int G = s.Hq / s.Hkv, Tc = s.L / kM;
+    const int G = s.Hq / s.Hkv, Tc = s.L / s.block_size;
     const long long units = (long long)s.B * s.Hkv;
     const int slots = ring_slots(G, Tc, p.topk);
     if (slots == 0) return cudaErrorInvalidValue;
@@ -549,8 +555,8 @@ cudaError_t launch_decode_select(const void* q, const void* Krepr, const int32_t
         return cudaErrorInvalidValue;
     const size_t smem = smem_bytes(G, Tc, p.topk, slots);
     Args args{static_cast<const __nv_bfloat16*>(q), lens, idx, cnt, status, s.Hq, s.Hkv, s.L, Tc,
-              p.topk, p.n_init, p.n_local, (int)units, slots, p.aggregation, p.sm_scale * kLog2e,
-              p.sm_scale};
+              p.topk, p.n_init, p.n_local, (int)units, slots, p.aggregation, s.block_size,
+              p.sm_scale * kLog2e, p.sm_scale};
     auto kern = G == 2 ? decode_select_tc_kernel<2> : decode_select_tc_kernel<1>;
     cudaError_t e;
     if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=

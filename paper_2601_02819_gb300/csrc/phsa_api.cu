@@ -30,7 +30,8 @@ int* status_ptr() {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Common shape checks; returns PHSA_OK or an error code. Block sizes 16 and
-// 32 are accepted only by the prefill forward calls (any_block).
+// 32 are accepted only where any_block is set (every call but the host-buffer
+// step; the backward adds its own condition).
 int check_shape(const phsa_shape& s, bool any_block = false) {
     if (s.B < 0 || s.L < 0 || s.Hq <= 0 || s.Hkv <= 0 || s.D <= 0 || s.block_size <= 0)
         return PHSA_ERR_INVALID_ARG;
@@ -161,10 +162,10 @@ int phsa_sparse_attn_bwd(const void* Q, const void* K, const void* V, const void
 
 int phsa_decode_update_repr(const void* K, const uint8_t* punct_mask, const int32_t* seq_lens,
                             phsa_shape s, float lambda, void* Krepr, void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
-    if (empty(s) || s.L < phsa::kM) return PHSA_OK;  // no block can fill
+    if (empty(s) || s.L < s.block_size) return PHSA_OK;  // no block can fill
     if (!K || !punct_mask || !seq_lens || !Krepr || !aligned16(K) || !aligned16(Krepr))
         return PHSA_ERR_INVALID_ARG;
     int* st = status_ptr();
@@ -176,7 +177,7 @@ int phsa_decode_update_repr(const void* K, const uint8_t* punct_mask, const int3
 int phsa_decode_select(const void* q, const void* Krepr, const int32_t* seq_lens, phsa_shape s,
                        phsa_select_params p, int32_t* block_idx, int32_t* block_cnt,
                        void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
     if (p.n_init < 0 || p.n_local < 1 || p.topk < p.n_init + p.n_local) return PHSA_ERR_INVALID_ARG;
@@ -184,7 +185,7 @@ int phsa_decode_select(const void* q, const void* Krepr, const int32_t* seq_lens
         return PHSA_ERR_INVALID_ARG;
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (empty(s)) return PHSA_OK;
-    const bool need_repr = s.L >= 2 * phsa::kM;  // some length can have a candidate
+    const bool need_repr = s.L >= 2 * s.block_size;  // some length can have a candidate
     if (!q || !seq_lens || !block_idx || !block_cnt || !aligned16(q) ||
         (need_repr && (!Krepr || !aligned16(Krepr))))
         return PHSA_ERR_INVALID_ARG;
@@ -198,7 +199,7 @@ int phsa_decode_select(const void* q, const void* Krepr, const int32_t* seq_lens
 int phsa_decode_attn(const void* q, const void* K, const void* V, const int32_t* block_idx,
                      const int32_t* block_cnt, const int32_t* seq_lens, phsa_shape s, int topk,
                      float sm_scale, void* O, float* lse, void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if ((rc = check_topk(s, topk)) != PHSA_OK) return rc;
     if (!(sm_scale > 0.f) || !isfinite(sm_scale)) return PHSA_ERR_INVALID_ARG;
@@ -219,7 +220,7 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
                      const int32_t* seq_lens, phsa_shape s, float lambda, phsa_select_params p,
                      void* Krepr, int32_t* block_idx, int32_t* block_cnt, void* O, float* lse,
                      void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if ((rc = check_topk(s, p.topk)) != PHSA_OK) return rc;
     if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
@@ -229,7 +230,7 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
     if (!(p.sm_scale > 0.f) || !isfinite(p.sm_scale)) return PHSA_ERR_INVALID_ARG;
     if (s.B == 0) return PHSA_OK;
     if (!q || !K || !V || !punct_mask || !seq_lens || !block_idx || !block_cnt || !O || !lse ||
-        (s.L >= phsa::kM && !Krepr))
+        (s.L >= s.block_size && !Krepr))
         return PHSA_ERR_INVALID_ARG;
     if (!aligned16(q) || !aligned16(K) || !aligned16(V) || !aligned16(O) ||
         (Krepr && !aligned16(Krepr)))
@@ -244,7 +245,8 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
     if (e != cudaSuccess) return PHSA_ERR_CUDA;
     return from_cuda(phsa::launch_decode_attn_repr(q, K, V, block_idx, block_cnt, seq_lens, s,
                                                    p.topk, p.sm_scale, O, lse, punct_mask, lambda,
-                                                   s.L >= phsa::kM ? Krepr : nullptr, st, cs));
+                                                   s.L >= s.block_size ? Krepr : nullptr, st,
+                                                   cs));
 }
 
 int phsa_punct_mask(const int32_t* ids, int64_t n, const int32_t* punct_ids, int n_punct,
@@ -260,7 +262,7 @@ int phsa_punct_mask(const int32_t* ids, int64_t n, const int32_t* punct_ids, int
 int phsa_decode_append(const void* k_new, const void* v_new, const uint8_t* flag_new,
                        const int32_t* seq_lens, phsa_shape s, void* K, void* V,
                        uint8_t* punct_mask, void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if (s.B == 0) return PHSA_OK;
     if (!k_new || !v_new || !seq_lens || !K || !V || (flag_new && !punct_mask))
@@ -277,13 +279,13 @@ int phsa_decode_append(const void* k_new, const void* v_new, const uint8_t* flag
 int phsa_prefill_append(const void* k_chunk, const void* v_chunk, const uint8_t* flag_chunk,
                         const int32_t* seq_lens, int chunk_len, phsa_shape s, float lambda,
                         void* K, void* V, uint8_t* punct_mask, void* Krepr, void* stream) {
-    int rc = check_shape(s);
+    int rc = check_shape(s, true);
     if (rc != PHSA_OK) return rc;
     if (!(lambda >= 0.f && lambda <= 1.f)) return PHSA_ERR_INVALID_ARG;
     if (chunk_len < 0 || chunk_len > s.L) return PHSA_ERR_INVALID_ARG;
     if (s.B == 0 || chunk_len == 0) return PHSA_OK;
     if (!k_chunk || !v_chunk || !seq_lens || !K || !V || !punct_mask ||
-        (s.L >= phsa::kM && !Krepr))
+        (s.L >= s.block_size && !Krepr))
         return PHSA_ERR_INVALID_ARG;
     if (!aligned16(k_chunk) || !aligned16(v_chunk) || !aligned16(K) || !aligned16(V) ||
         (Krepr && !aligned16(Krepr)))

@@ -10,10 +10,11 @@
 // completes block t ((t + 1) m <= len), it also sums all m rows of the block
 // -- rows before the chunk read back from the cache, the chunk's rows from
 // the registers that carry them to the cache -- and writes the block's
-// representative key. The loads and sums follow block_repr_kernel<64>'s
-// order exactly (half-warps on alternate rows, eight row pairs per batch,
-// then the two halves), so a sequence built chunk by chunk has bit-identical
-// representative keys to phsa_build_block_repr over the finished cache.
+// representative key. The loads and sums follow block_repr_kernel<m>'s order
+// exactly (half-warps on alternate rows, eight row pairs per batch, then the
+// two halves), so a sequence built chunk by chunk has bit-identical
+// representative keys to phsa_build_block_repr over the finished cache, at
+// each block size m = 16, 32, 64.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 
@@ -36,7 +37,7 @@ __device__ __forceinline__ void add8(float* acc, const uint4& v) {
 __global__ void __launch_bounds__(kWarps * 32)
 prefill_append_kernel(const __nv_bfloat16* __restrict__ kc, const __nv_bfloat16* __restrict__ vc,
                       const uint8_t* __restrict__ fc, const int32_t* __restrict__ lens, int B,
-                      int Hkv, int L, int C, int T, int nj, float lambda,
+                      int Hkv, int L, int C, int T, int nj, int bm, float lambda,
                       __nv_bfloat16* __restrict__ K, __nv_bfloat16* __restrict__ V,
                       uint8_t* __restrict__ mask, __nv_bfloat16* __restrict__ Krepr, int* status) {
     const int lane = threadIdx.x & 31;
@@ -51,10 +52,10 @@ prefill_append_kernel(const __nv_bfloat16* __restrict__ kc, const __nv_bfloat16*
         return;
     }
     const int p0 = len - C;           // the chunk's first position
-    const int t = p0 / kM + j;        // the block this warp handles
-    if (t * kM >= len) return;        // past the chunk
-    const bool complete = (t + 1) * kM <= len;
-    const size_t blk0 = (size_t)t * kM;  // the block's first position
+    const int t = p0 / bm + j;        // the block this warp handles
+    if (t * bm >= len) return;        // past the chunk
+    const bool complete = (t + 1) * bm <= len;
+    const size_t blk0 = (size_t)t * bm;  // the block's first position
     const uint8_t* mrow = mask + (size_t)b * L;
     const uint8_t* frow = fc ? fc + (size_t)b * C : nullptr;
 
@@ -66,10 +67,10 @@ prefill_append_kernel(const __nv_bfloat16* __restrict__ kc, const __nv_bfloat16*
         if (p >= p0 && frow) return frow[p - p0] != 0;
         return mrow[p] != 0;
     };
-    const unsigned lo = __ballot_sync(0xffffffffu, flag_of(lane));
-    const unsigned hi = __ballot_sync(0xffffffffu, flag_of(32 + lane));
+    const unsigned lo = __ballot_sync(0xffffffffu, lane < bm && flag_of(lane));
+    const unsigned hi = __ballot_sync(0xffffffffu, bm > 32 && flag_of(32 + lane));
     if (frow && g == 0) {
-        for (int r = lane; r < kM; r += 32) {
+        for (int r = lane; r < bm; r += 32) {
             const int p = (int)blk0 + r;
             if (p >= p0 && p < len) mask[(size_t)b * L + p] = frow[p - p0] ? 1 : 0;
         }
@@ -86,8 +87,7 @@ prefill_append_kernel(const __nv_bfloat16* __restrict__ kc, const __nv_bfloat16*
     float s0[8], sp[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) { s0[q] = 0.f; sp[q] = 0.f; }
-#pragma unroll
-    for (int base = 0; base < kM; base += 16) {
+    for (int base = 0; base < bm; base += 16) {
         uint4 v[8], vv[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
@@ -124,7 +124,7 @@ prefill_append_kernel(const __nv_bfloat16* __restrict__ kc, const __nv_bfloat16*
     }
     if (half == 0) {
         float o[8];
-        const float inv_m = 1.0f / kM;
+        const float inv_m = 1.0f / (float)bm;
         const float inv_c = c > 0 ? 1.0f / (float)c : 0.f;
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
@@ -147,14 +147,16 @@ cudaError_t launch_prefill_append(const void* k_chunk, const void* v_chunk, cons
                                   const int32_t* lens, int C, const phsa_shape& s, float lambda,
                                   void* K, void* V, uint8_t* mask, void* Krepr, int* status,
                                   cudaStream_t st) {
-    const int nj = (C + kM - 1) / kM + 1;  // blocks a chunk of C tokens can touch
+    const int bm = s.block_size;
+    if (bm != 16 && bm != 32 && bm != 64) return cudaErrorInvalidValue;
+    const int nj = (C + bm - 1) / bm + 1;  // blocks a chunk of C tokens can touch
     const long long warps = (long long)s.B * s.Hkv * nj;
     if (warps == 0 || C == 0) return cudaSuccess;
     const unsigned grid = (unsigned)((warps + kWarps - 1) / kWarps);
     ProfScope prof(K_PREFILL_APPEND, st);
     prefill_append_kernel<<<grid, kWarps * 32, 0, st>>>(
         static_cast<const __nv_bfloat16*>(k_chunk), static_cast<const __nv_bfloat16*>(v_chunk),
-        flags, lens, s.B, s.Hkv, s.L, C, s.L / kM, nj, lambda, static_cast<__nv_bfloat16*>(K),
+        flags, lens, s.B, s.Hkv, s.L, C, s.L / bm, nj, bm, lambda, static_cast<__nv_bfloat16*>(K),
         static_cast<__nv_bfloat16*>(V), mask, static_cast<__nv_bfloat16*>(Krepr), status);
     return cudaGetLastError();
 }

@@ -95,6 +95,11 @@ WORKLOADS = {
 DECODE_WORKLOADS = {
     "decode_32k_b64": Workload("decode_32k_b64", B=64, L=32768, Hq=16, Hkv=8, topk=14,
                                punct="sentence", punct_gap=(9, 25), seed=1234 + 4),
+    # the paper's 32k block setting (blocks of 16; 8 initial, 32 local and 16
+    # Top-K blocks) on the same caches
+    "decode_32k_b64_m16": Workload("decode_32k_b64_m16", B=64, L=32768, Hq=16, Hkv=8,
+                                   block_size=16, topk=56, n_init=8, n_local=32,
+                                   punct="sentence", punct_gap=(9, 25), seed=1234 + 4),
 }
 
 

@@ -404,13 +404,13 @@ def phsa_decode_append(k_new, v_new, seq_lens, K, V, flag_new=None, punct_mask=N
 
 
 def phsa_prefill_append(k_chunk, v_chunk, seq_lens, K, V, punct_mask, Krepr, lam: float,
-                        flag_chunk=None, stream=None):
+                        flag_chunk=None, stream=None, block_size: int = BLOCK_SIZE):
     """Append a chunk of C tokens to every sequence's caches (positions
     seq_lens[b] - C .. seq_lens[b] - 1, seq_lens counting the chunk) and write
-    the representative key of every block of 64 the chunk completes, from the
-    same loads: k_chunk/v_chunk [B, Hkv, C, D] bf16 into K/V [B, Hkv, Lc, D],
-    flag_chunk [B, C] uint8 (optional) into punct_mask [B, Lc], keys into
-    Krepr [B, Hkv, Lc // 64, D]."""
+    the representative key of every block of m = block_size the chunk
+    completes, from the same loads: k_chunk/v_chunk [B, Hkv, C, D] bf16 into
+    K/V [B, Hkv, Lc, D], flag_chunk [B, C] uint8 (optional) into punct_mask
+    [B, Lc], keys into Krepr [B, Hkv, Lc // m, D]."""
     _check(k_chunk, "k_chunk", torch.bfloat16, 4)
     _check(v_chunk, "v_chunk", torch.bfloat16, 4)
     _check(seq_lens, "seq_lens", torch.int32, 1)
@@ -422,26 +422,29 @@ def phsa_prefill_append(k_chunk, v_chunk, seq_lens, K, V, punct_mask, Krepr, lam
     C = k_chunk.shape[2]
     if tuple(V.shape) != tuple(K.shape) or tuple(k_chunk.shape) != (B, Hkv, C, D) or \
             tuple(v_chunk.shape) != (B, Hkv, C, D) or tuple(seq_lens.shape) != (B,) or \
-            tuple(punct_mask.shape) != (B, Lc) or tuple(Krepr.shape) != (B, Hkv, Lc // BLOCK_SIZE, D):
+            tuple(punct_mask.shape) != (B, Lc) or \
+            tuple(Krepr.shape) != (B, Hkv, Lc // int(block_size), D):
         raise ValueError("k_chunk/v_chunk must be [B, Hkv, C, D], K/V [B, Hkv, Lc, D], "
-                         "seq_lens [B], punct_mask [B, Lc], Krepr [B, Hkv, Lc // 64, D]")
+                         "seq_lens [B], punct_mask [B, Lc], Krepr [B, Hkv, Lc // m, D]")
     if flag_chunk is not None:
         _check(flag_chunk, "flag_chunk", torch.uint8, 2)
         if tuple(flag_chunk.shape) != (B, C):
             raise ValueError("flag_chunk must be [B, C]")
     rc = load().phsa_prefill_append(_ptr(k_chunk), _ptr(v_chunk), _ptr(flag_chunk),
-                                    _ptr(seq_lens), int(C), make_shape(B, Lc, Hkv, Hkv, D),
-                                    float(lam), _ptr(K), _ptr(V), _ptr(punct_mask), _ptr(Krepr),
+                                    _ptr(seq_lens), int(C),
+                                    make_shape(B, Lc, Hkv, Hkv, D, block_size), float(lam),
+                                    _ptr(K), _ptr(V), _ptr(punct_mask), _ptr(Krepr),
                                     _stream(stream))
     _raise("phsa_prefill_append", rc)
     return K, V, Krepr
 
 
-def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=None):
+def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=None,
+                            block_size: int = BLOCK_SIZE):
     """Decode: refresh the representative key of every block the new token has
-    just filled (a sequence whose length is a positive multiple of 64).
+    just filled (a sequence whose length is a positive multiple of m = block_size).
     K [B, Hkv, Lc, D] bf16 cache, punct_mask [B, Lc] uint8, seq_lens [B] int32,
-    Krepr [B, Hkv, Lc // 64, D] bf16 (updated in place; returned)."""
+    Krepr [B, Hkv, Lc // m, D] bf16 (updated in place; returned)."""
     _check(K, "K", torch.bfloat16, 4)
     _check(punct_mask, "punct_mask", torch.uint8, 2)
     _check(seq_lens, "seq_lens", torch.int32, 1)
@@ -449,18 +452,22 @@ def phsa_decode_update_repr(K, punct_mask, seq_lens, lam: float, Krepr, stream=N
     B, Hkv, Lc, D = K.shape
     if tuple(punct_mask.shape) != (B, Lc) or tuple(seq_lens.shape) != (B,):
         raise ValueError("punct_mask must be [B, Lc] and seq_lens [B]")
+    if tuple(Krepr.shape) != (B, Hkv, Lc // int(block_size), D):
+        raise ValueError("Krepr must be [B, Hkv, Lc // m, D]")
     rc = load().phsa_decode_update_repr(_ptr(K), _ptr(punct_mask), _ptr(seq_lens),
-                                        make_shape(B, Lc, Hkv, Hkv, D), float(lam), _ptr(Krepr),
-                                        _stream(stream))
+                                        make_shape(B, Lc, Hkv, Hkv, D, block_size), float(lam),
+                                        _ptr(Krepr), _stream(stream))
     _raise("phsa_decode_update_repr", rc)
     return Krepr
 
 
 def phsa_decode_select(q, Krepr, seq_lens, Lc: int, topk: int, n_init: int = 1,
                        n_local: int = 1, sm_scale: float | None = None, block_idx=None,
-                       block_cnt=None, stream=None, aggregation: str = "softmax_sum"):
+                       block_cnt=None, stream=None, aggregation: str = "softmax_sum",
+                       block_size: int = BLOCK_SIZE):
     """Decode selection for the new token of every sequence: q [B, Hq, D] bf16,
-    Krepr [B, Hkv, Lc // 64, D]; returns (block_idx [B, Hkv, topk], block_cnt [B, Hkv])."""
+    Krepr [B, Hkv, Lc // m, D] (m = block_size); returns (block_idx [B, Hkv, topk],
+    block_cnt [B, Hkv])."""
     _check(q, "q", torch.bfloat16, 3)
     _check(Krepr, "Krepr", torch.bfloat16, 4)
     _check(seq_lens, "seq_lens", torch.int32, 1)
@@ -475,16 +482,19 @@ def phsa_decode_select(q, Krepr, seq_lens, Lc: int, topk: int, n_init: int = 1,
     _check(block_idx, "block_idx", torch.int32, 3)
     _check(block_cnt, "block_cnt", torch.int32, 2)
     p = _params(topk, n_init, n_local, sm_scale, aggregation)
+    if tuple(Krepr.shape) != (B, Hkv, Lc // int(block_size), D):
+        raise ValueError("Krepr must be [B, Hkv, Lc // m, D]")
     rc = load().phsa_decode_select(_ptr(q), _ptr(Krepr), _ptr(seq_lens),
-                                   make_shape(B, Lc, Hq, Hkv, D), p, _ptr(block_idx),
+                                   make_shape(B, Lc, Hq, Hkv, D, block_size), p, _ptr(block_idx),
                                    _ptr(block_cnt), _stream(stream))
     _raise("phsa_decode_select", rc)
     return block_idx, block_cnt
 
 
 def phsa_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, sm_scale: float | None = None,
-                     O=None, lse=None, stream=None):
-    """Decode attention of the new token: (O [B, Hq, D] bf16, lse [B, Hq] fp32)."""
+                     O=None, lse=None, stream=None, block_size: int = BLOCK_SIZE):
+    """Decode attention of the new token over the selected blocks of m =
+    block_size keys: (O [B, Hq, D] bf16, lse [B, Hq] fp32)."""
     _check(q, "q", torch.bfloat16, 3)
     _check(K, "K", torch.bfloat16, 4)
     _check(V, "V", torch.bfloat16, 4)
@@ -500,7 +510,7 @@ def phsa_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, sm_scale: float | 
     _check(O, "O", torch.bfloat16, 3)
     _check(lse, "lse", torch.float32, 2)
     rc = load().phsa_decode_attn(_ptr(q), _ptr(K), _ptr(V), _ptr(block_idx), _ptr(block_cnt),
-                                 _ptr(seq_lens), make_shape(B, Lc, Hq, Hkv, D),
+                                 _ptr(seq_lens), make_shape(B, Lc, Hq, Hkv, D, block_size),
                                  int(block_idx.shape[-1]), float(sm_scale), _ptr(O), _ptr(lse),
                                  _stream(stream))
     _raise("phsa_decode_attn", rc)
@@ -510,11 +520,11 @@ def phsa_decode_attn(q, K, V, block_idx, block_cnt, seq_lens, sm_scale: float | 
 def phsa_decode_step(q, K, V, punct_mask, seq_lens, lam: float, Krepr, topk: int,
                      n_init: int = 1, n_local: int = 1, sm_scale: float | None = None,
                      block_idx=None, block_cnt=None, O=None, lse=None, stream=None,
-                     aggregation: str = "softmax_sum"):
+                     aggregation: str = "softmax_sum", block_size: int = BLOCK_SIZE):
     """One decode step in two launches (selection; attention fused with the
     refresh of the blocks the new tokens have just filled). q [B, Hq, D], K/V
     [B, Hkv, Lc, D] bf16 caches, punct_mask [B, Lc] uint8, seq_lens [B] int32,
-    Krepr [B, Hkv, Lc // 64, D] (read, and updated in place).
+    Krepr [B, Hkv, Lc // m, D] (m = block_size; read, and updated in place).
     Returns (block_idx, block_cnt, O, lse)."""
     _check(q, "q", torch.bfloat16, 3)
     _check(K, "K", torch.bfloat16, 4)
@@ -534,10 +544,13 @@ def phsa_decode_step(q, K, V, punct_mask, seq_lens, lam: float, Krepr, topk: int
         O = torch.empty_like(q)
     if lse is None:
         lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device)
+    if tuple(Krepr.shape) != (B, Hkv, Lc // int(block_size), D):
+        raise ValueError("Krepr must be [B, Hkv, Lc // m, D]")
     p = _params(topk, n_init, n_local, sm_scale, aggregation)
     rc = load().phsa_decode_step(_ptr(q), _ptr(K), _ptr(V), _ptr(punct_mask), _ptr(seq_lens),
-                                 make_shape(B, Lc, Hq, Hkv, D), float(lam), p, _ptr(Krepr),
-                                 _ptr(block_idx), _ptr(block_cnt), _ptr(O), _ptr(lse),
+                                 make_shape(B, Lc, Hq, Hkv, D, block_size), float(lam), p,
+                                 _ptr(Krepr), _ptr(block_idx), _ptr(block_cnt), _ptr(O),
+                                 _ptr(lse),
                                  _stream(stream))
     _raise("phsa_decode_step", rc)
     return block_idx, block_cnt, O, lse

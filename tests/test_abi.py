@@ -150,7 +150,30 @@ def test_prefill_append_validation_needs_no_gpu(lib):
     assert f(None, None, None, None, -1, ok, 0.5, None, None, None, None, None) == -1  # C < 0
     assert f(None, None, None, None, 513, ok, 0.5, None, None, None, None, None) == -1  # C > L
     assert f(None, None, None, None, 16, ok, 0.5, None, None, None, None, None) == -1  # null pointers
-    m16 = phsa_shape(2, 512, 4, 2, 128, 16)
-    assert f(None, None, None, None, 16, m16, 0.5, None, None, None, None, None) == -2  # m = 64 only
+    for bs in (16, 32):  # accepted: the null pointers are what is rejected
+        mb = phsa_shape(2, 512, 4, 2, 128, bs)
+        assert f(None, None, None, None, 16, mb, 0.5, None, None, None, None, None) == -1
+    m8 = phsa_shape(2, 512, 4, 2, 128, 8)
+    assert f(None, None, None, None, 16, m8, 0.5, None, None, None, None, None) == -2  # m = 8
     d64 = phsa_shape(2, 512, 4, 2, 64, 64)
     assert f(None, None, None, None, 16, d64, 0.5, None, None, None, None, None) == -2  # D = 128 only
+
+
+def test_decode_calls_take_block_sizes_16_and_32(lib):
+    # past the block size check, a null pointer is what the decode calls reject
+    from paper_2601_02819_gb300.phsa import phsa_shape, phsa_select_params
+    P, F, I = ctypes.c_void_p, ctypes.c_float, ctypes.c_int
+    lib.phsa_decode_update_repr.argtypes = [P, P, P, phsa_shape, F, P, P]
+    lib.phsa_decode_select.argtypes = [P, P, P, phsa_shape, phsa_select_params, P, P, P]
+    lib.phsa_decode_attn.argtypes = [P, P, P, P, P, P, phsa_shape, I, F, P, P, P]
+    lib.phsa_decode_step.argtypes = [P, P, P, P, P, phsa_shape, F, phsa_select_params, P, P, P,
+                                     P, P, P]
+    p = phsa_select_params(12, 1, 2, 0.088)
+    for bs, want in ((16, -1), (32, -1), (8, -2), (128, -2)):
+        s = phsa_shape(2, 4096, 16, 8, 128, bs)
+        assert lib.phsa_decode_update_repr(None, None, None, s, 0.5, None, None) == want
+        assert lib.phsa_decode_select(None, None, None, s, p, None, None, None) == want
+        assert lib.phsa_decode_attn(None, None, None, None, None, None, s, 12, 0.088, None, None,
+                                    None) == want
+        assert lib.phsa_decode_step(None, None, None, None, None, s, 0.5, p, None, None, None,
+                                    None, None, None) == want

@@ -26,35 +26,39 @@ def _rand(rng, *s):
 
 
 class Caches:
-    def __init__(self, B, Hkv, Lc):
+    def __init__(self, B, Hkv, Lc, bm=M):
+        self.bm = bm
         self.K = torch.zeros((B, Hkv, Lc, D), dtype=torch.bfloat16, device="cuda")
         self.V = torch.zeros_like(self.K)
         self.mask = torch.zeros((B, Lc), dtype=torch.uint8, device="cuda")
-        self.Kr = torch.zeros((B, Hkv, Lc // M, D), dtype=torch.bfloat16, device="cuda")
+        self.Kr = torch.zeros((B, Hkv, Lc // bm, D), dtype=torch.bfloat16, device="cuda")
 
     def append(self, b0, b1, kc, vc, fc, lens, lam):
         """One call over sequences [b0, b1) (a contiguous slice of the caches)."""
         phsa.phsa_prefill_append(to_dev_bf16(kc), to_dev_bf16(vc),
                                  torch.tensor(lens, dtype=torch.int32, device="cuda"),
                                  self.K[b0:b1], self.V[b0:b1], self.mask[b0:b1], self.Kr[b0:b1],
-                                 lam, flag_chunk=None if fc is None else torch.from_numpy(fc).cuda())
+                                 lam, flag_chunk=None if fc is None else torch.from_numpy(fc).cuda(),
+                                 block_size=self.bm)
 
 
 def _check(c, Kfull, Vfull, flags, totals, lam):
+    bm = c.bm
     Kh, Vh, mh = bf16_bits(c.K), bf16_bits(c.V), c.mask.cpu().numpy()
     for b, n in enumerate(totals):
         assert np.array_equal(Kh[b, :, :n], Kfull[b, :, :n])
         assert np.array_equal(Vh[b, :, :n], Vfull[b, :, :n])
         assert np.array_equal(mh[b, :n], flags[b, :n])
         assert not Kh[b, :, n:].any() and not Vh[b, :, n:].any()
-        T = n // M
+        T = n // bm
         if T == 0:
             continue
         got = bf16_bits(c.Kr)[b:b + 1, :, :T]
-        ref = oracle.block_repr(Kfull[b:b + 1, :, :n], flags[b:b + 1, :n], M, lam)
+        ref = oracle.block_repr(Kfull[b:b + 1, :, :n], flags[b:b + 1, :n], bm, lam)
         assert ulp_distance(got, ref[:, :, :T]).max() <= 1
-        full = phsa.phsa_build_block_repr(c.K[b:b + 1, :, :T * M].contiguous(),
-                                          c.mask[b:b + 1, :T * M].contiguous(), lam)
+        full = phsa.phsa_build_block_repr(c.K[b:b + 1, :, :T * bm].contiguous(),
+                                          c.mask[b:b + 1, :T * bm].contiguous(), lam,
+                                          block_size=bm)
         torch.cuda.synchronize()
         assert np.array_equal(bf16_bits(full), got)
 
@@ -132,3 +136,29 @@ def test_lengths_that_do_not_fit_are_rejected_on_the_device():
     assert np.array_equal(Kh[0, :, :64], kc[0])
     assert not Kh[1].any() and not Kh[2].any()
     assert c.mask.cpu().numpy()[1:].sum() == 0
+
+
+@pytest.mark.parametrize("bm", [16, 32])
+def test_chunked_prefill_at_small_block_sizes(bm):
+    # chunks shorter than a block, chunks that complete several blocks, and
+    # chunk boundaries on and off the block grid
+    rng = np.random.default_rng(40 + bm)
+    B, Hkv, Lc, lam = 3, 2, 64 * 5, 0.5
+    plans = [[1, bm - 1, bm, 3 * bm + 5, 7, 100, 64 * 5 - 5 * bm - 112],
+             [bm + 3, 2 * bm - 3, 1, 150], [bm // 2, bm // 2, bm // 2]]
+    totals = [sum(p) for p in plans]
+    Kfull, Vfull = _rand(rng, B, Hkv, Lc, D), _rand(rng, B, Hkv, Lc, D)
+    flags = (rng.random((B, Lc)) < 0.08).astype(np.uint8)
+    flags[0, :bm] = 1                     # an all-punctuation block
+    flags[1, bm:2 * bm] = 0               # a block without punctuation
+    c = Caches(B, Hkv, Lc, bm)
+    for b, plan in enumerate(plans):
+        p0 = 0
+        for C in plan:
+            c.append(b, b + 1, np.ascontiguousarray(Kfull[b:b + 1, :, p0:p0 + C]),
+                     np.ascontiguousarray(Vfull[b:b + 1, :, p0:p0 + C]),
+                     np.ascontiguousarray(flags[b:b + 1, p0:p0 + C]), [p0 + C], lam)
+            p0 += C
+    torch.cuda.synchronize()
+    assert phsa.phsa_get_device_status() == 0
+    _check(c, Kfull, Vfull, flags, totals, lam)
