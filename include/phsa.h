@@ -31,10 +31,11 @@
  *     reports argument validation and launch errors only. Errors detected by
  *     a kernel (an out-of-range block index, a bounded wait that expired) are
  *     recorded in a device status word read by phsa_get_device_status.
- *   - Supported today: D = 128, G in {1, 2}, block_size = 64 in every call;
- *     phsa_build_block_repr, phsa_select_blocks and phsa_sparse_attn_fwd also
- *     take block_size 16 and 32 (16 is the block size of the paper's experiment
- *     settings).
+ *   - Supported today: D = 128, G in {1, 2}, block_size 16, 32 or 64 (16 is
+ *     the block size of the paper's experiment settings) in every call, with
+ *     two exceptions: the backward (phsa_sparse_attn_bwd, its workspace query
+ *     and the no-allocation entry point) takes 16 and 32 only for G = 2, and
+ *     the host-buffer step (phsa_step_host) takes 64 only.
  *     Other shapes return PHSA_ERR_UNSUPPORTED, never a wrong answer.
  *   - Calls are thread-safe with respect to each other; concurrent calls on
  *     different streams that write the same output race, as any CUDA work.
@@ -328,7 +329,7 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
  * Prefill in chunks (block-level caching of Section 3.2; Eq. 3, 6, 7, 8;
  * Algorithm 1 step 2): appends a chunk of C = chunk_len tokens to every
  * sequence's caches and, from the same loads, computes the representative key
- * of every block of m = 64 tokens that the chunk completes, so a prefill does
+ * of every block of m = s.block_size tokens that the chunk completes, so a prefill does
  * not read K a second time for stage (a). With len = seq_lens[b] (the length
  * after the append, chunk included), the chunk takes positions
  * p = len - C + i, i in [0, C):
@@ -341,9 +342,9 @@ int phsa_decode_step(const void* q, const void* K, const void* V, const uint8_t*
  *   those phsa_build_block_repr computes over the finished cache. Blocks the
  *   chunk leaves partial get no key yet.
  *   k_chunk, v_chunk bf16 [B, Hkv, C, D] in;  flag_chunk uint8 [B, C] in or NULL
- *   seq_lens int32 [B] in (device); s.L is the cache capacity, s.block_size 64
+ *   seq_lens int32 [B] in (device); s.L is the cache capacity
  *   K, V bf16 [B, Hkv, L, D], punct_mask uint8 [B, L], Krepr bf16
- *   [B, Hkv, floor(L/64), D]: in/out (device, caller-owned)
+ *   [B, Hkv, floor(L/m), D]: in/out (device, caller-owned)
  * A length with len < C or len > L is a device-side error
  * (PHSA_ERR_DEVICE_INDEX) and that sequence is left untouched. chunk_len = 0
  * does nothing.
