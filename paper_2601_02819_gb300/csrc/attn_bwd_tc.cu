@@ -20,15 +20,19 @@
 //   arrives on the barrier that the tiles complete.
 //
 // dkdv_tc_kernel: persistent, one CTA per SM over the work items (KV block t,
-//   chunk of <= 32 query blocks that selected t), 320 threads; K_t and V_t are
+//   chunk of <= 32 query blocks that selected t), 352 threads; K_t and V_t are
 //   reloaded per item as soon as its predecessor's S/dP MMAs are done, and the
 //   dV^T/dK^T accumulators are double-buffered in TMEM. K_t and V_t stay in shared memory;
 //   the Q and dO tiles (both heads stacked: 128 rows) of every listed query
 //   block stream through a two-stage ring:
-//     S  = Q K_t^T, dP = dO V_t^T            (M128 N64 K128)
-//     P, dS (8 warps) -> shared memory (bf16, 128 rows x 64 keys, two buffers)
+//     S  = Q K_t^T, dP = dO V_t^T            (M128 N64 K128; one MMA thread)
+//     P, then dS (8 warps) -> shared memory  (bf16, 128 rows x 64 keys, two buffers)
 //     dV^T += dO^T P, dK^T += Q^T dS          (M128 N64 K128; A = dO / Q read
-//                                             MN-major, B = P / dS MN-major)
+//                                             MN-major, B = P / dS MN-major; a
+//                                             second MMA thread)
+//   Each product has its own barrier: P is formed while dP is still being
+//   computed, and dV^T runs while dS is being formed. One issuing thread per
+//   stream keeps either stream from waiting behind the other's 16 MMAs.
 //   dK^T and dV^T live in TMEM with the head dimension on the lanes. A KV
 //   block with a single chunk writes bf16 dK, dV straight from registers; a longer
 //   list writes fp32 partials, and the chunk that finishes last (an atomic
@@ -685,16 +689,24 @@ constexpr int kOffPDS = kOffStage + 2 * kStage;
 constexpr int kPDS = 2 * kHalf128;
 constexpr int kOffBar = kOffPDS + 2 * kPDS;
 constexpr int kRing = 8;  // item descriptors in flight
-constexpr int B_KV = 0, B_KVFREE = 1, B_QFULL = 2, B_QEMPTY = 4, B_SPFULL = 6, B_PDSFULL = 8,
-              B_PDSFREE = 10, B_FINAL = 12, B_DKVFREE = 14, B_DRAIN = 16, B_IFULL = 17,
-              B_IFREE = B_IFULL + kRing, kNumBars = B_IFREE + kRing;
-constexpr int kIFreeCount = 9;  // the MMA thread and the 8 elementwise warps
+// Barriers (pairs are indexed by iteration parity or accumulator buffer):
+//   KV/KVFREE     K_t, V_t landed / the item's last dP has read them
+//   QFULL/QEMPTY  Q/dO stage landed / the iteration's dK^T (and dV^T) MMAs are done
+//   SFULL/DPFULL  S / dP of the iteration are in TMEM
+//   PFULL/DSFULL  the elementwise warps have read S / dP and stored P / dS
+//   PFREE/DSFREE  the dV^T / dK^T MMAs that read P / dS are done
+//   FINAL/DKVFREE an item's accumulators are complete / have been read
+constexpr int B_KV = 0, B_KVFREE = 1, B_QFULL = 2, B_QEMPTY = 4, B_SFULL = 6, B_DPFULL = 8,
+              B_PFULL = 10, B_DSFULL = 12, B_PFREE = 14, B_DSFREE = 16, B_FINAL = 18,
+              B_DKVFREE = 20, B_DRAIN = 22, B_IFULL = 24, B_IFREE = B_IFULL + kRing,
+              kNumBars = B_IFREE + kRing;
+constexpr int kIFreeCount = 10;  // the two MMA threads and the 8 elementwise warps
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag, last-arriver flag
 constexpr int kOffQL = kOffMisc + 16;  // the producer's copy of an item's query blocks
 constexpr int kMaxItemQ = kBwdChunk * 4;      // query blocks per item at m = 16
 constexpr int kOffN = kOffQL + kMaxItemQ * 4;  // iteration counts of recent items [4]
 constexpr int kOffRing = (kOffN + 16 + 15) / 16 * 16;  // item descriptors [kRing][8 ints]
-constexpr int kThreads = 320;  // 8 elementwise warps, producer, MMA
+constexpr int kThreads = 352;  // 8 elementwise warps, producer, S/dP MMA, dV/dK MMA
 // TMEM: S of iteration buffer b at 128b, dP at 64 + 128b; dV^T and dK^T of
 // accumulator buffer c at 256 + 128c and 320 + 128c.
 __device__ __forceinline__ uint32_t col_s(int b) { return 128u * (uint32_t)b; }
@@ -822,13 +834,16 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int s = 0; s < 2; ++s) {
             mbar_init(bar(B_QFULL + s), 1);
             mbar_init(bar(B_QEMPTY + s), 1);
-            mbar_init(bar(B_SPFULL + s), 1);
-            mbar_init(bar(B_PDSFULL + s), 256);
-            mbar_init(bar(B_PDSFREE + s), 1);
+            mbar_init(bar(B_SFULL + s), 1);
+            mbar_init(bar(B_DPFULL + s), 1);
+            mbar_init(bar(B_PFULL + s), 256);
+            mbar_init(bar(B_DSFULL + s), 256);
+            mbar_init(bar(B_PFREE + s), 1);
+            mbar_init(bar(B_DSFREE + s), 1);
             mbar_init(bar(B_FINAL + s), 1);
             mbar_init(bar(B_DKVFREE + s), 256);
+            mbar_init(bar(B_DRAIN + s), 1);
         }
-        mbar_init(bar(B_DRAIN), 1);
         for (int r = 0; r < kRing; ++r) {
             mbar_init(bar(B_IFULL + r), 1);
             mbar_init(bar(B_IFREE + r), kIFreeCount);
@@ -946,102 +961,105 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 if (i >= 0) mbar_wait_drain(bar(B_QFULL + (i & 1)), (i >> 1) & 1);
         }
     } else if (warp == 9) {
-        // ------------------------------------------------ MMA issuer
+        // ------------------------------------------------ S / dP MMA issuer
+        // S = Q K_t^T and dP = dO V_t^T (M128 N64 K128) of every iteration, each
+        // into its TMEM buffer as soon as the elementwise warps have read that
+        // buffer two iterations back; separate commits, so P can be formed while
+        // dP is still being computed.
         if (lane == 0) {
             constexpr uint32_t id_s = idesc_bf16(128, 64, false);
-            constexpr uint32_t id_t = idesc_bf16(128, 64, true, true);  // A and B MN-major
-            const uint64_t dSt0 = sdesc_sw128(sb + kOffStage, 16, 1024);          // Q/dO K-major
-            const uint64_t dStT0 = sdesc_sw128(sb + kOffStage, kHalf128, 1024);   // Q/dO MN-major
+            const uint64_t dSt0 = sdesc_sw128(sb + kOffStage, 16, 1024);  // Q/dO K-major
             const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
             const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
-            const uint64_t dP0 = sdesc_sw128(sb + kOffPDS, kHalf128, 1024);
-            const uint64_t dS0 = sdesc_sw128(sb + kOffPDS + kHalf128, kHalf128, 1024);
-            int* nring = reinterpret_cast<int*>(smem + kOffN);  // iteration counts, by item & 3
-            // Two streams over the items with at least one iteration:
-            //   S/dP stream  (ns: global iteration, s_item/s_pos/s_n: its item)
-            //   dV/dK stream (nv, v_item/v_pos), at most two iterations behind.
             const int* ring = reinterpret_cast<const int*>(smem + kOffRing);
-            int ns = 0, nv = 0, s_item = 0, s_pos = 0, v_item = 0, v_pos = 0;
-            int r = 0, s_n = 0;       // ring items read; iterations of the S/dP stream's item
-            bool s_more = true;       // the ring has not ended
+            int ns = 0, kvi = 0;  // global iteration; items with iterations
             bool ok = true;
-            Deadline dl;
-            while (ok && (s_more || nv < ns)) {
-                bool progressed = false;
-                if (s_more && s_n == 0 && mbar_test_wait(bar(B_IFULL + r % kRing), (r / kRing) & 1)) {
-                    // the next item; one without iterations has nothing to multiply
-                    const int n = ring_get(ring + (r % kRing) * 8).n_it;
-                    mbar_arrive(bar(B_IFREE + r % kRing));
-                    ++r;
-                    if (n < 0) s_more = false;
-                    s_n = max(n, 0);
-                    if (s_n > 0) nring[s_item & 3] = s_n;
-                    progressed = true;
-                }
-                if (s_n > 0 && ns <= nv + 1 &&
-                    (s_pos > 0 || mbar_test_wait(bar(B_KV), s_item & 1)) &&
-                    mbar_test_wait(bar(B_QFULL + (ns & 1)), (ns >> 1) & 1)) {
+            for (int r = 0; ok; ++r) {
+                if (!mbar_wait(bar(B_IFULL + r % kRing), (r / kRing) & 1, abort_flag, a.status)) break;
+                const int n = ring_get(ring + (r % kRing) * 8).n_it;
+                mbar_arrive(bar(B_IFREE + r % kRing));
+                if (n < 0) break;
+                if (n == 0) continue;
+                if (!mbar_wait(bar(B_KV), kvi & 1, abort_flag, a.status)) break;
+                for (int pos = 0; pos < n; ++pos, ++ns) {
+                    const int b = ns & 1;
+                    const uint32_t ph = (uint32_t)((ns >> 1) & 1), pp = ph ^ 1u;
+                    ok = mbar_wait(bar(B_QFULL + b), ph, abort_flag, a.status) &&
+                         (ns < 2 || mbar_wait(bar(B_PFULL + b), pp, abort_flag, a.status));
+                    if (!ok) break;
                     tc_fence_after();
-                    const uint64_t qd = sdesc_at(dSt0, (ns & 1) * kStage);
+                    const uint64_t qd = sdesc_at(dSt0, b * kStage);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + col_s(ns & 1),
-                               sdesc_at(qd, (ks >> 2) * kHalf128 + (ks & 3) * 32),
-                               sdesc_at(dK0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s,
-                               ks > 0 ? 1u : 0u);
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + col_dp(ns & 1),
-                               sdesc_at(qd, kTile128 + (ks >> 2) * kHalf128 + (ks & 3) * 32),
-                               sdesc_at(dV0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s,
-                               ks > 0 ? 1u : 0u);
-                    mma_commit(bar(B_SPFULL + (ns & 1)));
-                    ++ns;
-                    if (++s_pos == s_n) {  // the item's last S/dP: K_t/V_t may be replaced
-                        mma_commit(bar(B_KVFREE));
-                        ++s_item;
-                        s_pos = 0;
-                        s_n = 0;
-                    }
-                    progressed = true;
-                }
-                const int c = v_item & 1;  // accumulator buffer
-                if (nv < ns && mbar_test_wait(bar(B_PDSFULL + (nv & 1)), (nv >> 1) & 1) &&
-                    (v_pos > 0 || v_item < 2 || mbar_test_wait(bar(B_DKVFREE + c), ((v_item >> 1) - 1) & 1))) {
+                        mma_ss(tmem + col_s(b), sdesc_at(qd, (ks >> 2) * kHalf128 + (ks & 3) * 32),
+                               sdesc_at(dK0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s, ks > 0 ? 1u : 0u);
+                    mma_commit(bar(B_SFULL + b));
+                    ok = ns < 2 || mbar_wait(bar(B_DSFULL + b), pp, abort_flag, a.status);
+                    if (!ok) break;
                     tc_fence_after();
-                    const uint64_t qt = sdesc_at(dStT0, (nv & 1) * kStage);
-                    const uint32_t pb = (nv & 1) * kPDS;
-                    // K dimension = the 128 stacked query rows, 16 per MMA
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + col_dv(c), sdesc_at(qt, kTile128 + ks * 2048),
-                               sdesc_at(dP0, pb + ks * 2048), id_t, (v_pos > 0 || ks > 0) ? 1u : 0u);
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + col_dk(c), sdesc_at(qt, ks * 2048), sdesc_at(dS0, pb + ks * 2048),
-                               id_t, (v_pos > 0 || ks > 0) ? 1u : 0u);
-                    mma_commit(bar(B_PDSFREE + (nv & 1)));
-                    mma_commit(bar(B_QEMPTY + (nv & 1)));
-                    ++nv;
-                    if (++v_pos == nring[v_item & 3]) {
-                        mma_commit(bar(B_FINAL + c));
-                        ++v_item;
-                        v_pos = 0;
-                    }
-                    progressed = true;
+                        mma_ss(tmem + col_dp(b), sdesc_at(qd, kTile128 + (ks >> 2) * kHalf128 + (ks & 3) * 32),
+                               sdesc_at(dV0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s, ks > 0 ? 1u : 0u);
+                    mma_commit(bar(B_DPFULL + b));
                 }
-                if (progressed) {
-                    dl.reset();
-                } else if (*abort_flag) {
-                    ok = false;
-                } else if (dl.expired()) {
-                    *abort_flag = 1;
-                    atomicCAS(a.status, 0, PHSA_ERR_TIMEOUT);
-                    ok = false;
-                }
+                mma_commit(bar(B_KVFREE));  // the item's last S/dP: K_t/V_t may be replaced
+                ++kvi;
             }
             mma_commit(bar(B_DRAIN));
             mbar_wait_drain(bar(B_DRAIN), 0);
+        }
+    } else if (warp == 10) {
+        // ------------------------------------------------ dV^T / dK^T MMA issuer
+        // dV^T += dO^T P as soon as P is stored, dK^T += Q^T dS as soon as dS is
+        // (M128 N64 K128, both operands MN-major), into the item's accumulator pair.
+        if (lane == 0) {
+            constexpr uint32_t id_t = idesc_bf16(128, 64, true, true);  // A and B MN-major
+            const uint64_t dStT0 = sdesc_sw128(sb + kOffStage, kHalf128, 1024);  // Q/dO MN-major
+            const uint64_t dP0 = sdesc_sw128(sb + kOffPDS, kHalf128, 1024);
+            const uint64_t dS0 = sdesc_sw128(sb + kOffPDS + kHalf128, kHalf128, 1024);
+            const int* ring = reinterpret_cast<const int*>(smem + kOffRing);
+            int nv = 0, vi = 0;  // global iteration; items with iterations
+            bool ok = true;
+            for (int r = 0; ok; ++r) {
+                if (!mbar_wait(bar(B_IFULL + r % kRing), (r / kRing) & 1, abort_flag, a.status)) break;
+                const int n = ring_get(ring + (r % kRing) * 8).n_it;
+                mbar_arrive(bar(B_IFREE + r % kRing));
+                if (n < 0) break;
+                if (n == 0) continue;
+                const int c = vi & 1;  // accumulator buffer
+                if (vi >= 2 && !mbar_wait(bar(B_DKVFREE + c), ((vi >> 1) - 1) & 1, abort_flag, a.status))
+                    break;
+                for (int pos = 0; pos < n; ++pos, ++nv) {
+                    const int b = nv & 1;
+                    const uint32_t ph = (uint32_t)((nv >> 1) & 1);
+                    const uint64_t qt = sdesc_at(dStT0, b * kStage);
+                    const uint32_t pb = b * kPDS;
+                    // K dimension = the 128 stacked query rows, 16 per MMA
+                    ok = mbar_wait(bar(B_PFULL + b), ph, abort_flag, a.status);
+                    if (!ok) break;
+                    tc_fence_after();
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(tmem + col_dv(c), sdesc_at(qt, kTile128 + ks * 2048), sdesc_at(dP0, pb + ks * 2048),
+                               id_t, (pos > 0 || ks > 0) ? 1u : 0u);
+                    mma_commit(bar(B_PFREE + b));
+                    ok = mbar_wait(bar(B_DSFULL + b), ph, abort_flag, a.status);
+                    if (!ok) break;
+                    tc_fence_after();
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(tmem + col_dk(c), sdesc_at(qt, ks * 2048), sdesc_at(dS0, pb + ks * 2048), id_t,
+                               (pos > 0 || ks > 0) ? 1u : 0u);
+                    mma_commit(bar(B_DSFREE + b));
+                    mma_commit(bar(B_QEMPTY + b));
+                }
+                if (!ok) break;
+                mma_commit(bar(B_FINAL + c));
+                ++vi;
+            }
+            mma_commit(bar(B_DRAIN + 1));
+            mbar_wait_drain(bar(B_DRAIN + 1), 0);
         }
     } else {
         // ------------------------------------------------ elementwise (8 warps)
@@ -1089,57 +1107,86 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const float dlt = dl_n;
                 if (i + 1 < n_it) fetch(i + 1, qb_n, mb_n, nl_n, dl_n);
                 const int buf = gi & 1;
-                ok = mbar_wait(bar(B_SPFULL + buf), (gi >> 1) & 1, abort_flag, a.status);
+                const uint32_t ph = (uint32_t)((gi >> 1) & 1), pp = ph ^ 1u;
+                uint8_t* pds = smem + kOffPDS + buf * kPDS;
+                // ---- P = 2^(S scale_log2 - lse log2 e), published as soon as S is in
+                ok = mbar_wait(bar(B_SFULL + buf), ph, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
                 tc_fence_after();
-                uint32_t sv[32], dp[32];
-                tmem_ld32x2(lane_base + col_s(buf) + 32 * kh, lane_base + col_dp(buf) + 32 * kh, sv, dp);
+                uint32_t sv[32];
+                tmem_ld32(lane_base + col_s(buf) + 32 * kh, sv);
                 // the row's query block lies in this span: causal mask in its own block
                 const bool diag = qb >= 0 && qb / kSub == t;
                 const bool all = mbits == (1u << kSub) - 1u && !diag;  // every key of the tile
-                // P = 2^(S scale_log2 - lse log2 e), dS = P (dP - Delta), two keys at a
-                // time (packed f32x2); masks (blocks the row's query block did not
-                // select, its own block's later keys, padding rows) off the main path
-                const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
-                const float2 nl2v = make_float2(neg_lse2, neg_lse2), ndl = make_float2(-dlt, -dlt);
+                // two keys at a time (packed f32x2); masks (blocks the row's query
+                // block did not select, its own block's later keys, padding rows)
+                // off the main path
+                float pf[32];
+                {
+                    const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+                    const float2 nl2v = make_float2(neg_lse2, neg_lse2);
 #pragma unroll
-                for (int c = 0; c < 16; ++c) {
-                    float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
-                    if (all) {
-                        pv.x = ex2_approx(pv.x);
-                        pv.y = ex2_approx(pv.y);
-                    } else {
-                        const int key = 32 * kh + 2 * c;
-                        const int q0 = key / kMq, q1 = (key + 1) / kMq;
-                        const bool k0 = ((mbits >> q0) & 1u) && !(diag && t * kSub + q0 == qb && key % kMq > tt);
-                        const bool k1 = ((mbits >> q1) & 1u) &&
-                                        !(diag && t * kSub + q1 == qb && (key + 1) % kMq > tt);
-                        pv.x = k0 ? ex2_approx(pv.x) : 0.f;
-                        pv.y = k1 ? ex2_approx(pv.y) : 0.f;
+                    for (int c = 0; c < 16; ++c) {
+                        float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])),
+                                               sc2, nl2v);
+                        if (all) {
+                            pv.x = ex2_approx(pv.x);
+                            pv.y = ex2_approx(pv.y);
+                        } else {
+                            const int key = 32 * kh + 2 * c;
+                            const int q0 = key / kMq, q1 = (key + 1) / kMq;
+                            const bool k0 = ((mbits >> q0) & 1u) && !(diag && t * kSub + q0 == qb && key % kMq > tt);
+                            const bool k1 = ((mbits >> q1) & 1u) &&
+                                            !(diag && t * kSub + q1 == qb && (key + 1) % kMq > tt);
+                            pv.x = k0 ? ex2_approx(pv.x) : 0.f;
+                            pv.y = k1 ? ex2_approx(pv.y) : 0.f;
+                        }
+                        pf[2 * c] = pv.x;
+                        pf[2 * c + 1] = pv.y;
+                        sv[c] = pack2_bf16(pv.x, pv.y);
                     }
-                    const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
-                    const float2 ds = __fmul2_rn(pv, d);
-                    sv[c] = pack2_bf16(pv.x, pv.y);
-                    dp[c] = pack2_bf16(ds.x, ds.y);
                 }
                 tc_fence_before();
-                if (gi >= 2) {  // the dV/dK MMAs two iterations back must have read this buffer
-                    ok = mbar_wait(bar(B_PDSFREE + buf), ((gi >> 1) - 1) & 1, abort_flag, a.status);
+                if (gi >= 2) {  // the dV^T MMAs two iterations back must have read this buffer
+                    ok = mbar_wait(bar(B_PFREE + buf), pp, abort_flag, a.status);
                     ok = __all_sync(0xffffffffu, ok);
                     if (!ok) break;
                 }
-                uint8_t* pds = smem + kOffPDS + buf * kPDS;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint32_t off = sw_off(row, 4 * kh + q);
-                    *reinterpret_cast<uint4*>(pds + off) =
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<uint4*>(pds + sw_off(row, 4 * kh + q)) =
                         make_uint4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
-                    *reinterpret_cast<uint4*>(pds + kHalf128 + off) =
-                        make_uint4(dp[4 * q], dp[4 * q + 1], dp[4 * q + 2], dp[4 * q + 3]);
-                }
                 fence_proxy_async_smem();
-                mbar_arrive(bar(B_PDSFULL + buf));
+                mbar_arrive(bar(B_PFULL + buf));
+                // ---- dS = P (dP - Delta)
+                ok = mbar_wait(bar(B_DPFULL + buf), ph, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+                tc_fence_after();
+                uint32_t dp[32];
+                tmem_ld32(lane_base + col_dp(buf) + 32 * kh, dp);
+                {
+                    const float2 ndl = make_float2(-dlt, -dlt);
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) {
+                        const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
+                        const float2 ds = __fmul2_rn(make_float2(pf[2 * c], pf[2 * c + 1]), d);
+                        dp[c] = pack2_bf16(ds.x, ds.y);
+                    }
+                }
+                tc_fence_before();
+                if (gi >= 2) {  // the dK^T MMAs two iterations back must have read this buffer
+                    ok = mbar_wait(bar(B_DSFREE + buf), pp, abort_flag, a.status);
+                    ok = __all_sync(0xffffffffu, ok);
+                    if (!ok) break;
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<uint4*>(pds + kHalf128 + sw_off(row, 4 * kh + q)) =
+                        make_uint4(dp[4 * q], dp[4 * q + 1], dp[4 * q + 2], dp[4 * q + 3]);
+                fence_proxy_async_smem();
+                mbar_arrive(bar(B_DSFULL + buf));
             }
             // ---- epilogue: dV^T / dK^T, lane = head-dimension index d, keys [32 kh, +32)
             const int d = row;
