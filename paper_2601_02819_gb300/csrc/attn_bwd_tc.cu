@@ -1126,26 +1126,30 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 {
                     const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
                     const float2 nl2v = make_float2(neg_lse2, neg_lse2);
+                    if (all) {  // warp-uniform: one loop per case, no per-key branch
 #pragma unroll
-                    for (int c = 0; c < 16; ++c) {
-                        float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])),
-                                               sc2, nl2v);
-                        if (all) {
-                            pv.x = ex2_approx(pv.x);
-                            pv.y = ex2_approx(pv.y);
-                        } else {
+                        for (int c = 0; c < 16; ++c) {
+                            const float2 pv = __ffma2_rn(
+                                make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
+                            pf[2 * c] = ex2_approx(pv.x);
+                            pf[2 * c + 1] = ex2_approx(pv.y);
+                        }
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) {
+                            const float2 pv = __ffma2_rn(
+                                make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
                             const int key = 32 * kh + 2 * c;
                             const int q0 = key / kMq, q1 = (key + 1) / kMq;
                             const bool k0 = ((mbits >> q0) & 1u) && !(diag && t * kSub + q0 == qb && key % kMq > tt);
                             const bool k1 = ((mbits >> q1) & 1u) &&
                                             !(diag && t * kSub + q1 == qb && (key + 1) % kMq > tt);
-                            pv.x = k0 ? ex2_approx(pv.x) : 0.f;
-                            pv.y = k1 ? ex2_approx(pv.y) : 0.f;
+                            pf[2 * c] = k0 ? ex2_approx(pv.x) : 0.f;
+                            pf[2 * c + 1] = k1 ? ex2_approx(pv.y) : 0.f;
                         }
-                        pf[2 * c] = pv.x;
-                        pf[2 * c + 1] = pv.y;
-                        sv[c] = pack2_bf16(pv.x, pv.y);
                     }
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) sv[c] = pack2_bf16(pf[2 * c], pf[2 * c + 1]);
                 }
                 tc_fence_before();
                 if (gi >= 2) {  // the dV^T MMAs two iterations back must have read this buffer
