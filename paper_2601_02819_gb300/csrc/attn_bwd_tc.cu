@@ -681,25 +681,29 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
 namespace kv {
 constexpr int kOffK = 0;
 constexpr int kOffV = kOffK + kTile64;
-constexpr int kOffStage = kOffV + kTile64;      // 2 x (Q 32 KB, dO 32 KB)
-constexpr int kStage = 2 * kTile128;
-// P and dS [128 rows][64 keys] bf16, double-buffered: buffer b holds P at
-// kOffPDS + b * kPDS and dS kHalf128 after it
-constexpr int kOffPDS = kOffStage + 2 * kStage;
-constexpr int kPDS = 2 * kHalf128;
-constexpr int kOffBar = kOffPDS + 2 * kPDS;
+// Q and dO tiles (128 rows x 128 columns, 32 KB each) stream through a ring of
+// kSlots half-slots in the order Q_0, dO_0, Q_1, dO_1, ...: load l of the CTA
+// goes to slot l % kSlots. dO_i is released by the dV^T MMAs of iteration i,
+// Q_i by its dK^T MMAs, so the next iterations' tiles load while one finishes.
+constexpr int kSlots = 5;
+constexpr int kOffSlot = kOffV + kTile64;
+// P and dS [128 rows][64 keys] bf16, one buffer each
+constexpr int kOffP = kOffSlot + kSlots * kTile128;
+constexpr int kOffDS = kOffP + kHalf128;
+constexpr int kOffBar = kOffDS + kHalf128;
 constexpr int kRing = 8;  // item descriptors in flight
 // Barriers (pairs are indexed by iteration parity or accumulator buffer):
 //   KV/KVFREE     K_t, V_t landed / the item's last dP has read them
-//   QFULL/QEMPTY  Q/dO stage landed / the iteration's dK^T (and dV^T) MMAs are done
+//   HFULL/HEMPTY  a half-slot has landed / its last MMA is done (kSlots each)
 //   SFULL/DPFULL  S / dP of the iteration are in TMEM
 //   PFULL/DSFULL  the elementwise warps have read S / dP and stored P / dS
 //   PFREE/DSFREE  the dV^T / dK^T MMAs that read P / dS are done
 //   FINAL/DKVFREE an item's accumulators are complete / have been read
-constexpr int B_KV = 0, B_KVFREE = 1, B_QFULL = 2, B_QEMPTY = 4, B_SFULL = 6, B_DPFULL = 8,
-              B_PFULL = 10, B_DSFULL = 12, B_PFREE = 14, B_DSFREE = 16, B_FINAL = 18,
-              B_DKVFREE = 20, B_DRAIN = 22, B_IFULL = 24, B_IFREE = B_IFULL + kRing,
-              kNumBars = B_IFREE + kRing;
+constexpr int B_KV = 0, B_KVFREE = 1, B_HFULL = 2, B_HEMPTY = B_HFULL + kSlots,
+              B_SFULL = B_HEMPTY + kSlots, B_DPFULL = B_SFULL + 2, B_PFULL = B_DPFULL + 2,
+              B_DSFULL = B_PFULL + 2, B_PFREE = B_DSFULL + 2, B_DSFREE = B_PFREE + 2,
+              B_FINAL = B_DSFREE + 2, B_DKVFREE = B_FINAL + 2, B_DRAIN = B_DKVFREE + 2,
+              B_IFULL = B_DRAIN + 2, B_IFREE = B_IFULL + kRing, kNumBars = B_IFREE + kRing;
 constexpr int kIFreeCount = 10;  // the two MMA threads and the 8 elementwise warps
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag, last-arriver flag
 constexpr int kOffQL = kOffMisc + 16;  // the producer's copy of an item's query blocks
@@ -831,9 +835,11 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_KV), 1);
         mbar_init(bar(B_KVFREE), 1);
+        for (int h = 0; h < kSlots; ++h) {
+            mbar_init(bar(B_HFULL + h), 1);
+            mbar_init(bar(B_HEMPTY + h), 1);
+        }
         for (int s = 0; s < 2; ++s) {
-            mbar_init(bar(B_QFULL + s), 1);
-            mbar_init(bar(B_QEMPTY + s), 1);
             mbar_init(bar(B_SFULL + s), 1);
             mbar_init(bar(B_DPFULL + s), 1);
             mbar_init(bar(B_PFULL + s), 256);
@@ -873,7 +879,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
             for (int c = 0; c < kQueueClasses; ++c)
                 qn[c] = (int)min((long long)max(a.qcount[c], 0), a.qcap);
-            int gi = 0, kvc = 0, r = 0;  // Q/dO stages issued; items with K/V loaded; ring items
+            int gl = 0, kvc = 0, r = 0;  // Q/dO half-slot loads issued; items with K/V loaded; ring items
             bool ok = true;
             // hands item x to the other roles once its ring slot's last reader is done
             auto publish = [&](const KvItem& x) {
@@ -923,29 +929,30 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     ++kvc;
                     e = entry_of(j_nx, nx_valid);
                     const int hq0 = (it.bg / a.Hkv) * a.Hq + (it.bg % a.Hkv) * 2;
-                    for (int i = 0; i < it.n_it; ++i, ++gi) {
-                        const int s = gi & 1;
-                        if (gi >= 2 &&
-                            !mbar_wait(bar(B_QEMPTY + s), ((gi >> 1) - 1) & 1, abort_flag, a.status)) {
-                            ok = false;
-                            break;
-                        }
-                        const uint32_t st = sb + kOffStage + s * kStage;
-                        mbar_expect_tx(bar(B_QFULL + s), kStage);
-                        // kSub query blocks of kMq tokens, both heads (a short last
-                        // iteration repeats its last block; the rows are masked)
+                    for (int i = 0; ok && i < it.n_it; ++i) {
+                        // Q_i then dO_i, each into the next half-slot of the ring
+                        for (int h = 0; h < 2; ++h, ++gl) {
+                            const int slot = gl % kSlots;
+                            if (gl >= kSlots && !mbar_wait(bar(B_HEMPTY + slot), ((gl / kSlots) - 1) & 1,
+                                                           abort_flag, a.status)) {
+                                ok = false;
+                                break;
+                            }
+                            const uint32_t st = sb + kOffSlot + slot * kTile128;
+                            const CUtensorMap* tm = h == 0 ? &tmQ : &tmdO;
+                            mbar_expect_tx(bar(B_HFULL + slot), kTile128);
+                            // kSub query blocks of kMq tokens, both heads (a short last
+                            // iteration repeats its last block; the rows are masked)
 #pragma unroll
-                        for (int j = 0; j < kSub; ++j) {
-                            const int e = i * kSub + j;
-                            const int qb = qls[e < nq ? e : nq - 1];
-                            const uint32_t r0 = (uint32_t)(j * kMq * 128);
-                            for (int hl = 0; hl < 2; ++hl)
-                                for (int dh = 0; dh < 2; ++dh) {
-                                    tma_load_3d(st + dh * kHalf128 + hl * kHalf64 + r0, &tmQ,
-                                                bar(B_QFULL + s), dh * 64, qb * kMq, hq0 + hl);
-                                    tma_load_3d(st + kTile128 + dh * kHalf128 + hl * kHalf64 + r0, &tmdO,
-                                                bar(B_QFULL + s), dh * 64, qb * kMq, hq0 + hl);
-                                }
+                            for (int j = 0; j < kSub; ++j) {
+                                const int e = i * kSub + j;
+                                const int qb = qls[e < nq ? e : nq - 1];
+                                const uint32_t r0 = (uint32_t)(j * kMq * 128);
+                                for (int hl = 0; hl < 2; ++hl)
+                                    for (int dh = 0; dh < 2; ++dh)
+                                        tma_load_3d(st + dh * kHalf128 + hl * kHalf64 + r0, tm,
+                                                    bar(B_HFULL + slot), dh * 64, qb * kMq, hq0 + hl);
+                            }
                         }
                     }
                     if (!ok) break;
@@ -957,8 +964,8 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 ok = publish(it);
             }
             if (kvc > 0) mbar_wait_drain(bar(B_KV), (kvc - 1) & 1);
-            for (int i = gi - 2; i < gi; ++i)
-                if (i >= 0) mbar_wait_drain(bar(B_QFULL + (i & 1)), (i >> 1) & 1);
+            for (int l = gl - kSlots; l < gl; ++l)
+                if (l >= 0) mbar_wait_drain(bar(B_HFULL + l % kSlots), (l / kSlots) & 1);
         }
     } else if (warp == 9) {
         // ------------------------------------------------ S / dP MMA issuer
@@ -968,7 +975,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // dP is still being computed.
         if (lane == 0) {
             constexpr uint32_t id_s = idesc_bf16(128, 64, false);
-            const uint64_t dSt0 = sdesc_sw128(sb + kOffStage, 16, 1024);  // Q/dO K-major
+            const uint64_t dSl0 = sdesc_sw128(sb + kOffSlot, 16, 1024);  // Q/dO K-major
             const uint64_t dK0 = sdesc_sw128(sb + kOffK, 16, 1024);
             const uint64_t dV0 = sdesc_sw128(sb + kOffV, 16, 1024);
             const int* ring = reinterpret_cast<const int*>(smem + kOffRing);
@@ -984,22 +991,27 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 for (int pos = 0; pos < n; ++pos, ++ns) {
                     const int b = ns & 1;
                     const uint32_t ph = (uint32_t)((ns >> 1) & 1), pp = ph ^ 1u;
-                    ok = mbar_wait(bar(B_QFULL + b), ph, abort_flag, a.status) &&
+                    const int lq = 2 * ns, ld = lq + 1;  // the iteration's Q and dO loads
+                    // S: Q_i landed, and the elementwise warps have read S two iterations back
+                    ok = mbar_wait(bar(B_HFULL + lq % kSlots), (lq / kSlots) & 1, abort_flag, a.status) &&
                          (ns < 2 || mbar_wait(bar(B_PFULL + b), pp, abort_flag, a.status));
                     if (!ok) break;
                     tc_fence_after();
-                    const uint64_t qd = sdesc_at(dSt0, b * kStage);
+                    const uint64_t qd = sdesc_at(dSl0, (lq % kSlots) * kTile128);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
                         mma_ss(tmem + col_s(b), sdesc_at(qd, (ks >> 2) * kHalf128 + (ks & 3) * 32),
                                sdesc_at(dK0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s, ks > 0 ? 1u : 0u);
                     mma_commit(bar(B_SFULL + b));
-                    ok = ns < 2 || mbar_wait(bar(B_DSFULL + b), pp, abort_flag, a.status);
+                    // dP: dO_i landed, and dP two iterations back has been read
+                    ok = mbar_wait(bar(B_HFULL + ld % kSlots), (ld / kSlots) & 1, abort_flag, a.status) &&
+                         (ns < 2 || mbar_wait(bar(B_DSFULL + b), pp, abort_flag, a.status));
                     if (!ok) break;
                     tc_fence_after();
+                    const uint64_t dd = sdesc_at(dSl0, (ld % kSlots) * kTile128);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + col_dp(b), sdesc_at(qd, kTile128 + (ks >> 2) * kHalf128 + (ks & 3) * 32),
+                        mma_ss(tmem + col_dp(b), sdesc_at(dd, (ks >> 2) * kHalf128 + (ks & 3) * 32),
                                sdesc_at(dV0, (ks >> 2) * kHalf64 + (ks & 3) * 32), id_s, ks > 0 ? 1u : 0u);
                     mma_commit(bar(B_DPFULL + b));
                 }
@@ -1015,9 +1027,9 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // (M128 N64 K128, both operands MN-major), into the item's accumulator pair.
         if (lane == 0) {
             constexpr uint32_t id_t = idesc_bf16(128, 64, true, true);  // A and B MN-major
-            const uint64_t dStT0 = sdesc_sw128(sb + kOffStage, kHalf128, 1024);  // Q/dO MN-major
-            const uint64_t dP0 = sdesc_sw128(sb + kOffPDS, kHalf128, 1024);
-            const uint64_t dS0 = sdesc_sw128(sb + kOffPDS + kHalf128, kHalf128, 1024);
+            const uint64_t dSlT0 = sdesc_sw128(sb + kOffSlot, kHalf128, 1024);  // Q/dO MN-major
+            const uint64_t dP0 = sdesc_sw128(sb + kOffP, kHalf128, 1024);
+            const uint64_t dS0 = sdesc_sw128(sb + kOffDS, kHalf128, 1024);
             const int* ring = reinterpret_cast<const int*>(smem + kOffRing);
             int nv = 0, vi = 0;  // global iteration; items with iterations
             bool ok = true;
@@ -1033,26 +1045,31 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 for (int pos = 0; pos < n; ++pos, ++nv) {
                     const int b = nv & 1;
                     const uint32_t ph = (uint32_t)((nv >> 1) & 1);
-                    const uint64_t qt = sdesc_at(dStT0, b * kStage);
-                    const uint32_t pb = b * kPDS;
+                    const int sq = (2 * nv) % kSlots, sd = (2 * nv + 1) % kSlots;  // Q_i, dO_i
                     // K dimension = the 128 stacked query rows, 16 per MMA
                     ok = mbar_wait(bar(B_PFULL + b), ph, abort_flag, a.status);
                     if (!ok) break;
                     tc_fence_after();
+                    const uint64_t dt = sdesc_at(dSlT0, sd * kTile128);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + col_dv(c), sdesc_at(qt, kTile128 + ks * 2048), sdesc_at(dP0, pb + ks * 2048),
-                               id_t, (pos > 0 || ks > 0) ? 1u : 0u);
+                        mma_ss(tmem + col_dv(c), sdesc_at(dt, ks * 2048), sdesc_at(dP0, ks * 2048), id_t,
+                               (pos > 0 || ks > 0) ? 1u : 0u);
                     mma_commit(bar(B_PFREE + b));
+                    // dO_i is free once dV^T and the other thread's dP of the iteration are done
+                    ok = mbar_wait(bar(B_DPFULL + b), ph, abort_flag, a.status);
+                    if (!ok) break;
+                    mma_commit(bar(B_HEMPTY + sd));
                     ok = mbar_wait(bar(B_DSFULL + b), ph, abort_flag, a.status);
                     if (!ok) break;
                     tc_fence_after();
+                    const uint64_t qt = sdesc_at(dSlT0, sq * kTile128);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + col_dk(c), sdesc_at(qt, ks * 2048), sdesc_at(dS0, pb + ks * 2048), id_t,
+                        mma_ss(tmem + col_dk(c), sdesc_at(qt, ks * 2048), sdesc_at(dS0, ks * 2048), id_t,
                                (pos > 0 || ks > 0) ? 1u : 0u);
                     mma_commit(bar(B_DSFREE + b));
-                    mma_commit(bar(B_QEMPTY + b));
+                    mma_commit(bar(B_HEMPTY + sq));
                 }
                 if (!ok) break;
                 mma_commit(bar(B_FINAL + c));
@@ -1107,8 +1124,10 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const float dlt = dl_n;
                 if (i + 1 < n_it) fetch(i + 1, qb_n, mb_n, nl_n, dl_n);
                 const int buf = gi & 1;
-                const uint32_t ph = (uint32_t)((gi >> 1) & 1), pp = ph ^ 1u;
-                uint8_t* pds = smem + kOffPDS + buf * kPDS;
+                const uint32_t ph = (uint32_t)((gi >> 1) & 1);
+                // the single P and dS buffers were last read by iteration gi - 1
+                const int bq = (gi - 1) & 1;
+                const uint32_t pq = (uint32_t)(((gi - 1) >> 1) & 1);
                 // ---- P = 2^(S scale_log2 - lse log2 e), published as soon as S is in
                 ok = mbar_wait(bar(B_SFULL + buf), ph, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
@@ -1152,14 +1171,14 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     for (int c = 0; c < 16; ++c) sv[c] = pack2_bf16(pf[2 * c], pf[2 * c + 1]);
                 }
                 tc_fence_before();
-                if (gi >= 2) {  // the dV^T MMAs two iterations back must have read this buffer
-                    ok = mbar_wait(bar(B_PFREE + buf), pp, abort_flag, a.status);
+                if (gi >= 1) {  // the previous iteration's dV^T MMAs must have read P
+                    ok = mbar_wait(bar(B_PFREE + bq), pq, abort_flag, a.status);
                     ok = __all_sync(0xffffffffu, ok);
                     if (!ok) break;
                 }
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    *reinterpret_cast<uint4*>(pds + sw_off(row, 4 * kh + q)) =
+                    *reinterpret_cast<uint4*>(smem + kOffP + sw_off(row, 4 * kh + q)) =
                         make_uint4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
                 fence_proxy_async_smem();
                 mbar_arrive(bar(B_PFULL + buf));
@@ -1180,14 +1199,14 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     }
                 }
                 tc_fence_before();
-                if (gi >= 2) {  // the dK^T MMAs two iterations back must have read this buffer
-                    ok = mbar_wait(bar(B_DSFREE + buf), pp, abort_flag, a.status);
+                if (gi >= 1) {  // the previous iteration's dK^T MMAs must have read dS
+                    ok = mbar_wait(bar(B_DSFREE + bq), pq, abort_flag, a.status);
                     ok = __all_sync(0xffffffffu, ok);
                     if (!ok) break;
                 }
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    *reinterpret_cast<uint4*>(pds + kHalf128 + sw_off(row, 4 * kh + q)) =
+                    *reinterpret_cast<uint4*>(smem + kOffDS + sw_off(row, 4 * kh + q)) =
                         make_uint4(dp[4 * q], dp[4 * q + 1], dp[4 * q + 2], dp[4 * q + 3]);
                 fence_proxy_async_smem();
                 mbar_arrive(bar(B_DSFULL + buf));
