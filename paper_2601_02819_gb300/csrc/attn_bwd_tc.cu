@@ -5,19 +5,22 @@
 //   KV head g), 384 threads; rings and barriers continue across units. The
 //   selected blocks are taken in pairs (an odd count pairs the last block with
 //   a masked copy of itself); each pair's K and V tiles (128 keys) are gathered
-//   by TMA into 3- and 2-slot rings. Per pair p:
-//     S_p  = Q Kp^T       (M128 N128 K128)
-//     dP_p = dO Vp^T      (M128 N128 K128)
+//   by TMA into 3- and 2-slot rings. At the start of a unit its Q and dO tiles
+//   are copied from their staging buffers into TMEM (tcgen05.cp), where they
+//   are the A operands of S and dP; the staging buffers then load the next
+//   unit's tiles, a whole unit ahead. Per pair p:
+//     S_p  = Q Kp^T       (M128 N128 K128, A = Q in TMEM)
+//     dP_p = dO Vp^T      (M128 N128 K128, A = dO in TMEM)
 //     dS_p = P_p (dP_p - Delta), P_p = exp(S_p * scale - lse)   (8 warps, TMEM)
 //     dQ  += dS_p Kp      (M128 N128 K128, A = dS_p in TMEM, B = Kp MN-major)
-//   S is double-buffered in TMEM, so S_{p+1} runs while the elementwise warps
-//   work on pair p; dQ * scale is stored from registers. Before the first pair
-//   the elementwise warps compute Delta_i = dO_i . O_i (O read from global
-//   memory, dO from the loaded tile) and write it for the dK/dV kernel, which
-//   runs after this one. A fourth producer warp loads each unit's Q and dO as
-//   soon as the previous unit's last dP has been issued and its Delta read,
-//   and stages the elementwise warps' copy of the unit's block list before it
-//   arrives on the barrier that the tiles complete.
+//   S and dP have one TMEM buffer each: S_{p+1} is computed as soon as the
+//   elementwise warps hold S_p in registers, dP_{p+1} once dQ_p has read the
+//   dS_p written over dP_p. dQ * scale is stored from registers. Before the
+//   first pair the elementwise warps compute Delta_i = dO_i . O_i (O read from
+//   global memory, dO from its staging tile) and write it for the dK/dV
+//   kernel, which runs after this one. A fourth producer warp loads each
+//   unit's Q and dO and stages the elementwise warps' copy of the unit's block
+//   list before it arrives on the barrier that the Q tile completes.
 //
 // dkdv_tc_kernel: persistent, one CTA per SM over the work items (KV block t,
 //   chunk of <= 32 query blocks that selected t), 352 threads; K_t and V_t are
@@ -80,21 +83,26 @@ struct Cfg {
     static constexpr int kOffK = kOffDO + kTile128;
     static constexpr int kOffV = kOffK + kKSlots * kPair;
     static constexpr int kOffBar = kOffV + kVSlots * kPair;
-    static constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = B_KFULL + kKSlots,
-                         B_VFULL = B_KEMPTY + kKSlots, B_VEMPTY = B_VFULL + kVSlots,
-                         B_SPFULL = B_VEMPTY + kVSlots, B_DSFULL = B_SPFULL + 2,
-                         B_DPFREE = B_DSFULL + 2, B_FINAL = B_DPFREE + 1, B_DQFREE = B_FINAL + 1,
-                         B_DRAIN = B_DQFREE + 1, kNumBars = B_DRAIN + 1;
+    // B_Q/B_DO: a unit's Q / dO tile is in its staging buffer; B_QFREE/B_DOFREE:
+    // the staging buffer may be refilled (copied into TMEM, and seen by the
+    // elementwise warps / read for Delta); B_SFULL/B_SFREE, B_DPFULL: the single
+    // S and dP buffers in TMEM; B_DSFULL: dS is in TMEM (two barriers by pair parity)
+    static constexpr int B_Q = 0, B_QFREE = 1, B_DO = 2, B_DOFREE = 3, B_KFULL = 4,
+                         B_KEMPTY = B_KFULL + kKSlots, B_VFULL = B_KEMPTY + kKSlots,
+                         B_VEMPTY = B_VFULL + kVSlots, B_SFULL = B_VEMPTY + kVSlots,
+                         B_SFREE = B_SFULL + 1, B_DPFULL = B_SFREE + 1, B_DSFULL = B_DPFULL + 1,
+                         B_FINAL = B_DSFULL + 2, B_DQFREE = B_FINAL + 1, B_DRAIN = B_DQFREE + 1,
+                         kNumBars = B_DRAIN + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kOffDPart = kOffMisc + 16;  // Delta of the 128 rows, fp32
     static constexpr int kOffList = kOffDPart + 128 * 4;  // block lists: 7 slots
 };
 constexpr int kListK = 0, kListV = 2, kListM = 4, kListE = 5, kListSlots = 7;
 constexpr int kThreads = 384;  // 8 elementwise warps, K producer, MMA, V producer, Q/dO producer
-// TMEM: dQ [0,128), S of pair buffer b at [128 + 128b, +128), dP [384, 512).
-// dS of key half h overwrites S columns [64h, 64h + 32) (read by the same thread).
-constexpr uint32_t kColDQ = 0, kColDP = 384;
-__device__ __forceinline__ uint32_t col_s(int b) { return 128u + 128u * (uint32_t)b; }
+// TMEM: dQ [0,128), S [128,256), dP [256,384), the unit's Q [384,448) and dO
+// [448,512) as bf16 A operands (copied from their staging tiles). dS of key
+// half h overwrites dP columns [64h, 64h + 32) (read by the same thread).
+constexpr uint32_t kColDQ = 0, kColS = 128, kColDP = 256, kColQ = 384, kColDO = 448;
 // A list slot: the entries (capacity kSub * topk, one padding entry, the count
 // in the last int of the entry region), then at m < 64 the owner masks (bytes).
 __host__ __device__ constexpr int list_ints(int topk, int kSub) { return (kSub * topk + 2 + 15) & ~15; }
@@ -217,8 +225,14 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
     if (threadIdx.x == 0) {
+        // Q's staging buffer is free once its copy into TMEM is done and the
+        // elementwise warps have seen this unit's Q barrier (so that it cannot
+        // complete twice before they wait on it); dO's once its copy is done and
+        // the elementwise warps have read it for Delta
         mbar_init(bar(C::B_Q), 1);
-        mbar_init(bar(C::B_QFREE), 257);  // the MMA commit after the unit's last dP + 256 Delta readers
+        mbar_init(bar(C::B_QFREE), 257);
+        mbar_init(bar(C::B_DO), 1);
+        mbar_init(bar(C::B_DOFREE), 257);
         for (int s = 0; s < C::kKSlots; ++s) {
             mbar_init(bar(C::B_KFULL + s), 1);
             mbar_init(bar(C::B_KEMPTY + s), 1);
@@ -227,15 +241,11 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             mbar_init(bar(C::B_VFULL + s), 1);
             mbar_init(bar(C::B_VEMPTY + s), 1);
         }
-        mbar_init(bar(C::B_SPFULL), 1);
-        mbar_init(bar(C::B_SPFULL + 1), 1);
-        // dS barriers alternate by pair: once dP is released early, a thread may
-        // finish pair p+1 before another has finished pair p, so their arrivals
-        // must go to different barriers. dP_{p+1} needs every thread's release of
-        // dP_p, so no thread gets two pairs ahead and two barriers suffice.
+        mbar_init(bar(C::B_SFULL), 1);
+        mbar_init(bar(C::B_SFREE), 256);
+        mbar_init(bar(C::B_DPFULL), 1);
         mbar_init(bar(C::B_DSFULL), 256);
         mbar_init(bar(C::B_DSFULL + 1), 256);
-        mbar_init(bar(C::B_DPFREE), 256);
         mbar_init(bar(C::B_FINAL), 1);
         mbar_init(bar(C::B_DQFREE), 256);
         mbar_init(bar(C::B_DRAIN), 1);
@@ -313,25 +323,29 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             int* elists = reinterpret_cast<int*>(smem + C::kOffList) + kListE * ls;
             int ul = 0, last = -1;
             for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
+                // Q once the previous unit's has been copied into TMEM (at that unit's start)
                 if (ul > 0 && !mbar_wait(bar(C::B_QFREE), (ul - 1) & 1, abort_flag, a.status)) break;
                 last = ul;
                 const DqUnit d = dq_unit<kSub>(a, u);
-                // The tiles first; then the elementwise warps' copy of the block list
-                // (its slot's previous unit is done: they have passed that unit's
-                // Delta), published by this thread's arrival on C::B_Q.
-                mbar_expect_tx_only(bar(C::B_Q), 2 * kTile128);
+                // The tile first; then the elementwise warps' copy of the block list
+                // (its slot's unit two back is done: they have passed the previous
+                // unit's Q barrier), published by this thread's arrival on C::B_Q.
+                mbar_expect_tx_only(bar(C::B_Q), kTile128);
                 for (int hl = 0; hl < 2; ++hl)
-                    for (int dh = 0; dh < 2; ++dh) {
+                    for (int dh = 0; dh < 2; ++dh)
                         tma_load_3d(sb + C::kOffQ + dh * kHalf128 + hl * kHalf64, &tmQ, bar(C::B_Q),
                                     dh * 64, d.qb * 64, d.hq0 + hl);
-                        tma_load_3d(sb + C::kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(C::B_Q),
-                                    dh * 64, d.qb * 64, d.hq0 + hl);
-                    }
                 int* el = elists + (ul & 1) * ls;
                 el[li - 1] = stage_unit<kSub>(a, d, el, reinterpret_cast<uint8_t*>(el + li));
                 mbar_arrive(bar(C::B_Q));
-                // The next unit's Q and dO come from HBM: start bringing them into L2
-                // now, a whole unit before they are loaded.
+                // dO once the previous unit's has been copied and read for Delta
+                if (ul > 0 && !mbar_wait(bar(C::B_DOFREE), (ul - 1) & 1, abort_flag, a.status)) break;
+                mbar_expect_tx(bar(C::B_DO), kTile128);
+                for (int hl = 0; hl < 2; ++hl)
+                    for (int dh = 0; dh < 2; ++dh)
+                        tma_load_3d(sb + C::kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(C::B_DO),
+                                    dh * 64, d.qb * 64, d.hq0 + hl);
+                // Q and dO come from HBM: start bringing the next unit's into L2 now.
                 const int u2 = u + (int)gridDim.x;
                 if (u2 < a.units) {
                     const int qb2 = a.NQB - 1 - (u2 % a.NQB), bg2 = u2 / a.NQB;
@@ -343,7 +357,10 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                         }
                 }
             }
-            if (last >= 0) mbar_wait_drain(bar(C::B_Q), last & 1);
+            if (last >= 0) {
+                mbar_wait_drain(bar(C::B_Q), last & 1);
+                mbar_wait_drain(bar(C::B_DO), last & 1);
+            }
         }
     } else if (warp == 9) {
         // ------------------------------------------------ MMA issuer
@@ -355,24 +372,21 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const uint64_t dK0 = sdesc_sw128(sb + C::kOffK, 16, 1024);
             const uint64_t dKmn0 = sdesc_sw128(sb + C::kOffK, kHalf128, 1024);  // K read MN-major
             const uint64_t dV0 = sdesc_sw128(sb + C::kOffV, 16, 1024);
-            auto issue_s = [&](int gp) {  // S = Q Kpair^T into buffer gp & 1
+            // K step ks of a [d half][128 rows][64] tile: 16 columns of the head dimension
+            auto koff = [](int ks) { return (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32); };
+            auto issue_s = [&](int gp) {  // S = Q Kpair^T (A = Q in TMEM)
                 const uint64_t kd = sdesc_at(dK0, (gp % C::kKSlots) * C::kPair);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {
-                    const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
-                    mma_ss(tmem + col_s(gp & 1), sdesc_at(dQ0, off), sdesc_at(kd, off), id_s,
-                           ks > 0 ? 1u : 0u);
-                }
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ts(tmem + kColS, tmem + kColQ + ks * 8, sdesc_at(kd, koff(ks)), id_s, ks > 0 ? 1u : 0u);
+                mma_commit(bar(C::B_SFULL));
             };
-            auto issue_dp = [&](int gp) {  // dP = dO Vpair^T; releases the V slot
+            auto issue_dp = [&](int gp) {  // dP = dO Vpair^T (A = dO in TMEM); releases the V slot
                 const uint64_t vd = sdesc_at(dV0, (gp % C::kVSlots) * C::kPair);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {
-                    const uint32_t off = (uint32_t)((ks >> 2) * kHalf128 + (ks & 3) * 32);
-                    mma_ss(tmem + kColDP, sdesc_at(dDO0, off), sdesc_at(vd, off), id_s,
-                           ks > 0 ? 1u : 0u);
-                }
-                mma_commit(bar(C::B_SPFULL + (gp & 1)));  // S and dP of this pair are both complete
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ts(tmem + kColDP, tmem + kColDO + ks * 8, sdesc_at(vd, koff(ks)), id_s, ks > 0 ? 1u : 0u);
+                mma_commit(bar(C::B_DPFULL));
                 mma_commit(bar(C::B_VEMPTY + gp % C::kVSlots));
             };
             auto wait_k = [&](int gp) {
@@ -381,39 +395,53 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             auto wait_v = [&](int gp) {
                 return mbar_wait(bar(C::B_VFULL + gp % C::kVSlots), (gp / C::kVSlots) & 1, abort_flag, a.status);
             };
-            // dP has one TMEM buffer: dP(gp) waits until the elementwise warps hold
-            // dP(gp - 1) in registers (they release it before computing dS).
-            auto wait_dpfree = [&](int gp) {
-                return gp == 0 || mbar_wait(bar(C::B_DPFREE), (gp - 1) & 1, abort_flag, a.status);
+            // S_gp reuses the S buffer once the elementwise warps hold S_{gp-1}
+            auto wait_sfree = [&](int gp) {
+                return gp == 0 || mbar_wait(bar(C::B_SFREE), (gp - 1) & 1, abort_flag, a.status);
+            };
+            // dP_gp reuses the dP buffer once dQ_{gp-1} has read the dS written over it
+            // (its commit is the K slot's release)
+            auto wait_dq_done = [&](int gp) {
+                return gp == 0 || mbar_wait(bar(C::B_KEMPTY + (gp - 1) % C::kKSlots), ((gp - 1) / C::kKSlots) & 1,
+                                            abort_flag, a.status);
             };
             bool ok = true;
             int gp0 = 0, ul = 0;
-            // Order per unit: S_0 dP_0 S_1 | dP_1 | dS_0 -> dQ_0 S_2 | dP_2 | dS_1 -> dQ_1 S_3 ...
+            // Per unit: Q and dO copied into TMEM, then S_0 dP_0 | S_1 | dS_0 -> dQ_0 |
+            // dP_1 | S_2 | dS_1 -> dQ_1 | dP_2 ...
             int* mlist = reinterpret_cast<int*>(smem + C::kOffList) + kListM * slot_ints(a.topk, kSub);
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++ul) {
                 const DqUnit d = dq_unit<kSub>(a, u);
                 const int nu = kSub == 1 ? stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, mlist)
                                          : min(__ldg(a.ucnt + d.lu), a.ucap);
                 const int np = ((nu + kSub - 1) / kSub + 1) >> 1;
-                ok = mbar_wait(bar(C::B_Q), ul & 1, abort_flag, a.status);
+                // Q into TMEM once it has landed and the previous unit's last S has read
+                // the previous Q; its staging buffer is then free for the next unit's
+                ok = mbar_wait(bar(C::B_Q), ul & 1, abort_flag, a.status) &&
+                     (gp0 == 0 || mbar_wait(bar(C::B_SFULL), (gp0 - 1) & 1, abort_flag, a.status));
                 if (!ok) break;
                 tc_fence_after();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) tmem_cp_128x256b(tmem + kColQ + ks * 8, sdesc_at(dQ0, koff(ks)));
+                mma_commit(bar(C::B_QFREE));
+                // dO likewise, after the previous unit's last dP
+                ok = mbar_wait(bar(C::B_DO), ul & 1, abort_flag, a.status) &&
+                     (gp0 == 0 || mbar_wait(bar(C::B_DPFULL), (gp0 - 1) & 1, abort_flag, a.status));
+                if (!ok) break;
+                tc_fence_after();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) tmem_cp_128x256b(tmem + kColDO + ks * 8, sdesc_at(dDO0, koff(ks)));
+                mma_commit(bar(C::B_DOFREE));
                 if (np >= 1) {
-                    ok = wait_k(gp0) && wait_v(gp0) && wait_dpfree(gp0);
+                    ok = wait_k(gp0) && wait_sfree(gp0);
                     if (!ok) break;
                     tc_fence_after();
                     issue_s(gp0);
-                    issue_dp(gp0);
-                    if (np == 1) mma_commit(bar(C::B_QFREE));
-                }
-                if (np >= 2) {
-                    ok = wait_k(gp0 + 1);
+                    ok = wait_v(gp0) && wait_dq_done(gp0);
                     if (!ok) break;
                     tc_fence_after();
-                    issue_s(gp0 + 1);
-                }
-                if (np == 0) {
-                    mma_commit(bar(C::B_QFREE));
+                    issue_dp(gp0);
+                } else {
                     // the previous unit's dQ must be read out before FINAL completes again
                     ok = ul == 0 || mbar_wait(bar(C::B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
                     if (!ok) break;
@@ -422,31 +450,29 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 for (int p = 0; ok && p < np; ++p) {
                     const int gp = gp0 + p;
                     if (p + 1 < np) {
-                        ok = wait_dpfree(gp + 1) && wait_v(gp + 1);
+                        ok = wait_k(gp + 1) && wait_sfree(gp + 1);
                         if (!ok) break;
                         tc_fence_after();
-                        issue_dp(gp + 1);
-                        if (p + 2 == np) mma_commit(bar(C::B_QFREE));  // last MMA reading Q/dO
+                        issue_s(gp + 1);
                     }
                     ok = mbar_wait(bar(C::B_DSFULL + (gp & 1)), (gp >> 1) & 1, abort_flag, a.status);
                     if (ok && p == 0 && ul > 0)  // dQ's accumulator: the previous unit is read out
                         ok = mbar_wait(bar(C::B_DQFREE), (ul - 1) & 1, abort_flag, a.status);
                     if (!ok) break;
                     tc_fence_after();
-                    // dQ += dS Kpair: A = dS (TMEM), B = the K pair read MN-major
+                    // dQ += dS Kpair: A = dS (TMEM, over dP), B = the K pair read MN-major
                     const uint64_t kmn = sdesc_at(dKmn0, (gp % C::kKSlots) * C::kPair);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks)
-                        mma_ts(tmem + kColDQ, tmem + col_s(gp & 1) + (ks >> 2) * 64 + (ks & 3) * 8,
+                        mma_ts(tmem + kColDQ, tmem + kColDP + (ks >> 2) * 64 + (ks & 3) * 8,
                                sdesc_at(kmn, ks * 2048), id_dq, (p > 0 || ks > 0) ? 1u : 0u);
                     mma_commit(bar(C::B_KEMPTY + gp % C::kKSlots));
-                    if (p == np - 1) {
-                        mma_commit(bar(C::B_FINAL));
-                    } else if (p + 2 < np) {  // S_{p+2} reuses the S buffer dQ_p has just read
-                        ok = wait_k(gp + 2);
+                    if (p == np - 1) mma_commit(bar(C::B_FINAL));
+                    if (p + 1 < np) {
+                        ok = wait_v(gp + 1) && wait_dq_done(gp + 1);
                         if (!ok) break;
                         tc_fence_after();
-                        issue_s(gp + 2);
+                        issue_dp(gp + 1);
                     }
                 }
                 gp0 += np;
@@ -519,6 +545,8 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             }
             if (ok) {
                 ok = mbar_wait(bar(C::B_Q), ul & 1, abort_flag, a.status);
+                if (ok) mbar_arrive(bar(C::B_QFREE));
+                ok = ok && mbar_wait(bar(C::B_DO), ul & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
             // Delta_i = dO_i . O_i: O in coalesced 16-byte pieces (16 threads per
@@ -549,7 +577,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const float dlt = dpart[row];
             // This thread is done with dO and with Delta's exchange slots: the next
             // unit's dO may be loaded (and dpart rewritten) once all have arrived.
-            if (ok) mbar_arrive(bar(C::B_QFREE));
+            if (ok) mbar_arrive(bar(C::B_DOFREE));
             const int n = list[li - 1];
             const int nt = (n + kSub - 1) / kSub;  // 64-key tiles
             const int np = (nt + 1) >> 1;
@@ -560,8 +588,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const int u2 = u + (int)gridDim.x;
             for (int p = 0; ok && p < np; ++p) {
                 const int gp = gp0 + p;
-                const int buf = gp & 1;
-                ok = mbar_wait(bar(C::B_SPFULL + buf), (gp >> 1) & 1, abort_flag, a.status);
+                ok = mbar_wait(bar(C::B_SFULL), gp & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
                 tc_fence_after();
@@ -577,43 +604,59 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                     full |= (uint32_t)(sel && !mine) << q;
                     part |= (uint32_t)mine << q;
                 }
-                uint32_t sv[64], dp[64];
-                tmem_ld64x2(lane_base + col_s(buf) + 64 * half, lane_base + kColDP + 64 * half, sv, dp);
-                tc_fence_before();
-                mbar_arrive(bar(C::B_DPFREE));  // dP is in registers: the buffer may be refilled
-                // dS = P (dP - Delta), P = 2^(S scale_log2 - lse log2 e), two keys at a
-                // time (packed f32x2 arithmetic); the masks (the query's own block and the
-                // duplicate of an odd count) are warp-uniform branches off the main path
-                const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
-                const float2 nl2v = make_float2(nl2, nl2), ndl = make_float2(-dlt, -dlt);
-                if (full == (1u << kSub) - 1u) {
+                float pf[64];
+                {
+                    uint32_t sv[64];
+                    tmem_ld64(lane_base + kColS + 64 * half, sv);
+                    tc_fence_before();
+                    mbar_arrive(bar(C::B_SFREE));  // S is in registers: the next S may be computed
+                    // P = 2^(S scale_log2 - lse log2 e), two keys at a time (packed f32x2);
+                    // the masks (the query's own block and the duplicate of an odd count)
+                    // are warp-uniform branches off the main path
+                    const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+                    const float2 nl2v = make_float2(nl2, nl2);
+                    if (full == (1u << kSub) - 1u) {
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) {
-                        float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
-                        pv.x = ex2_approx(pv.x);
-                        pv.y = ex2_approx(pv.y);
-                        const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
-                        const float2 ds = __fmul2_rn(pv, d);
-                        sv[c] = pack2_bf16(ds.x, ds.y);
-                    }
-                } else {
+                        for (int c = 0; c < 32; ++c) {
+                            const float2 pv = __ffma2_rn(
+                                make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
+                            pf[2 * c] = ex2_approx(pv.x);
+                            pf[2 * c + 1] = ex2_approx(pv.y);
+                        }
+                    } else {
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) {
-                        float2 pv = __ffma2_rn(make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
-                        const int q0 = (2 * c) / kMq, q1 = (2 * c + 1) / kMq;
-                        const bool k0 = ((full >> q0) & 1u) || (((part >> q0) & 1u) && (2 * c) % kMq <= tt);
-                        const bool k1 = ((full >> q1) & 1u) || (((part >> q1) & 1u) && (2 * c + 1) % kMq <= tt);
-                        pv.x = k0 ? ex2_approx(pv.x) : 0.f;
-                        pv.y = k1 ? ex2_approx(pv.y) : 0.f;
-                        const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
-                        const float2 ds = __fmul2_rn(pv, d);
-                        sv[c] = pack2_bf16(ds.x, ds.y);
+                        for (int c = 0; c < 32; ++c) {
+                            const float2 pv = __ffma2_rn(
+                                make_float2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nl2v);
+                            const int q0 = (2 * c) / kMq, q1 = (2 * c + 1) / kMq;
+                            const bool k0 = ((full >> q0) & 1u) || (((part >> q0) & 1u) && (2 * c) % kMq <= tt);
+                            const bool k1 = ((full >> q1) & 1u) || (((part >> q1) & 1u) && (2 * c + 1) % kMq <= tt);
+                            pf[2 * c] = k0 ? ex2_approx(pv.x) : 0.f;
+                            pf[2 * c + 1] = k1 ? ex2_approx(pv.y) : 0.f;
+                        }
                     }
                 }
-                // dS columns [64 half, 64 half + 32): inside this thread's own S range
-                tmem_st32(lane_base + col_s(buf) + 64 * half, sv);
+                // dS = P (dP - Delta), written over this half's dP columns [64 half, +32)
+                ok = mbar_wait(bar(C::B_DPFULL), gp & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+                tc_fence_after();
+                const float2 ndl = make_float2(-dlt, -dlt);
+                uint32_t dsv[32];
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {  // 32 keys at a time, for fewer live registers
+                    uint32_t dp[32];
+                    tmem_ld32(lane_base + kColDP + 64 * half + 32 * hh, dp);
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) {
+                        const float2 d = __fadd2_rn(make_float2(__uint_as_float(dp[2 * c]), __uint_as_float(dp[2 * c + 1])), ndl);
+                        const float2 ds = __fmul2_rn(make_float2(pf[32 * hh + 2 * c], pf[32 * hh + 2 * c + 1]), d);
+                        dsv[16 * hh + c] = pack2_bf16(ds.x, ds.y);
+                    }
+                }
+                tmem_st32(lane_base + kColDP + 64 * half, dsv);
                 tc_fence_before();
-                mbar_arrive(bar(C::B_DSFULL + buf));
+                mbar_arrive(bar(C::B_DSFULL + (gp & 1)));
             }
             gp0 += np;
             // the next unit's inputs: their latency overlaps this unit's last dQ

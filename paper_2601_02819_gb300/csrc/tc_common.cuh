@@ -245,6 +245,13 @@ __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_
         "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+// Copies 128 rows x 256 bits (16 bf16 of every row of a K-major shared-memory
+// tile, described as for an MMA operand) into TMEM: row r to lane r, 8 columns
+// from taddr, in the layout from which an MMA reads its A operand. An MMA that
+// the same thread issues later reads the copied data.
+__device__ __forceinline__ void tmem_cp_128x256b(uint32_t taddr, uint64_t sdesc) {
+    asm volatile("tcgen05.cp.cta_group::1.128x256b [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
+}
 // Arrives once on `bar` when every tcgen05 operation issued so far by this
 // thread has completed.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
