@@ -85,9 +85,10 @@ struct Cfg {
     static constexpr int kOffBar = kOffV + kVSlots * kPair;
     // B_Q/B_DO: a unit's Q / dO tile is in its staging buffer; B_QFREE/B_DOFREE:
     // the staging buffer may be refilled (copied into TMEM, and seen by the
-    // elementwise warps / read for Delta); B_SFULL/B_SFREE, B_DPFULL: the single
+    // elementwise warps / read for Delta); B_O/B_OFREE: the unit's O tile is in
+    // the Q staging buffer / has been read for Delta; B_SFULL/B_SFREE, B_DPFULL: the single
     // S and dP buffers in TMEM; B_DSFULL: dS is in TMEM (two barriers by pair parity)
-    static constexpr int B_Q = 0, B_QFREE = 1, B_DO = 2, B_DOFREE = 3, B_KFULL = 4,
+    static constexpr int B_Q = 0, B_QFREE = 1, B_DO = 2, B_DOFREE = 3, B_O = 4, B_OFREE = 5, B_KFULL = 6,
                          B_KEMPTY = B_KFULL + kKSlots, B_VFULL = B_KEMPTY + kKSlots,
                          B_VEMPTY = B_VFULL + kVSlots, B_SFULL = B_VEMPTY + kVSlots,
                          B_SFREE = B_SFULL + 1, B_DPFULL = B_SFREE + 1, B_DSFULL = B_DPFULL + 1,
@@ -95,9 +96,9 @@ struct Cfg {
                          kNumBars = B_DRAIN + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kOffDPart = kOffMisc + 16;  // Delta of the 128 rows, fp32
-    static constexpr int kOffList = kOffDPart + 128 * 4;  // block lists: 7 slots
+    static constexpr int kOffList = kOffDPart + 128 * 4;  // block lists: 6 slots
 };
-constexpr int kListK = 0, kListV = 2, kListM = 4, kListE = 5, kListSlots = 7;
+constexpr int kListK = 0, kListV = 2, kListE = 4, kListSlots = 6;
 constexpr int kThreads = 384;  // 8 elementwise warps, K producer, MMA, V producer, Q/dO producer
 // TMEM: dQ [0,128), S [128,256), dP [256,384), the unit's Q [384,448) and dO
 // [448,512) as bf16 A operands (copied from their staging tiles). dS of key
@@ -211,7 +212,7 @@ template <int kSub>
 __global__ void __launch_bounds__(dq::kThreads, 1)
 dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
              const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
-             const DqArgs a) {
+             const __grid_constant__ CUtensorMap tmO, const DqArgs a) {
     using namespace dq;
     using C = Cfg<kSub>;
     constexpr int kMq = 64 / kSub;  // tokens of a query block (and keys of a KV block)
@@ -233,6 +234,8 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         mbar_init(bar(C::B_QFREE), 257);
         mbar_init(bar(C::B_DO), 1);
         mbar_init(bar(C::B_DOFREE), 257);
+        mbar_init(bar(C::B_O), 1);
+        mbar_init(bar(C::B_OFREE), 256);
         for (int s = 0; s < C::kKSlots; ++s) {
             mbar_init(bar(C::B_KFULL + s), 1);
             mbar_init(bar(C::B_KEMPTY + s), 1);
@@ -315,52 +318,59 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 if (q >= 0) mbar_wait_drain(bar(full + q % slots), (q / slots) & 1);
         }
     } else if (warp == 11) {
-        // ------------------------------------------------ Q / dO producer, one load per unit
+        // ------------------------------------------------ Q / dO / O producer
+        // Per unit j, in this order: O_j into the Q staging buffer (once Q_{j-1}
+        // has been copied into TMEM), dO_j into the dO staging buffer (once
+        // dO_{j-1} has been copied and read for Delta), then Q_j over O_j once the
+        // elementwise warps have taken Delta_j from both (during unit j - 1).
         if (lane == 0) {
             prefetch_tmap(&tmQ);
             prefetch_tmap(&tmdO);
+            prefetch_tmap(&tmO);
             const int ls = slot_ints(a.topk, kSub);
             int* elists = reinterpret_cast<int*>(smem + C::kOffList) + kListE * ls;
-            int ul = 0, last = -1;
+            int ul = 0, last_q = -1, last_o = -1, last_do = -1;
+            auto load_tile = [&](uint32_t dst, const CUtensorMap* map, uint32_t b, const DqUnit& d) {
+                for (int hl = 0; hl < 2; ++hl)
+                    for (int dh = 0; dh < 2; ++dh)
+                        tma_load_3d(dst + dh * kHalf128 + hl * kHalf64, map, b, dh * 64, d.qb * 64, d.hq0 + hl);
+            };
             for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
-                // Q once the previous unit's has been copied into TMEM (at that unit's start)
-                if (ul > 0 && !mbar_wait(bar(C::B_QFREE), (ul - 1) & 1, abort_flag, a.status)) break;
-                last = ul;
                 const DqUnit d = dq_unit<kSub>(a, u);
+                if (ul > 0 && !mbar_wait(bar(C::B_QFREE), (ul - 1) & 1, abort_flag, a.status)) break;
+                mbar_expect_tx(bar(C::B_O), kTile128);
+                load_tile(sb + C::kOffQ, &tmO, bar(C::B_O), d);
+                last_o = ul;
+                if (ul > 0 && !mbar_wait(bar(C::B_DOFREE), (ul - 1) & 1, abort_flag, a.status)) break;
+                mbar_expect_tx(bar(C::B_DO), kTile128);
+                load_tile(sb + C::kOffDO, &tmdO, bar(C::B_DO), d);
+                last_do = ul;
+                // this unit's and the next unit's tiles come from HBM: bring the next
+                // unit's into L2 now
+                const int u2 = u + (int)gridDim.x;
+                if (u2 < a.units) {
+                    const DqUnit d2 = dq_unit<kSub>(a, u2);
+                    for (int hl = 0; hl < 2; ++hl)
+                        for (int dh = 0; dh < 2; ++dh) {
+                            tma_prefetch_3d(&tmO, dh * 64, d2.qb * 64, d2.hq0 + hl);
+                            tma_prefetch_3d(&tmdO, dh * 64, d2.qb * 64, d2.hq0 + hl);
+                            tma_prefetch_3d(&tmQ, dh * 64, d2.qb * 64, d2.hq0 + hl);
+                        }
+                }
+                if (!mbar_wait(bar(C::B_OFREE), ul & 1, abort_flag, a.status)) break;
                 // The tile first; then the elementwise warps' copy of the block list
                 // (its slot's unit two back is done: they have passed the previous
                 // unit's Q barrier), published by this thread's arrival on C::B_Q.
                 mbar_expect_tx_only(bar(C::B_Q), kTile128);
-                for (int hl = 0; hl < 2; ++hl)
-                    for (int dh = 0; dh < 2; ++dh)
-                        tma_load_3d(sb + C::kOffQ + dh * kHalf128 + hl * kHalf64, &tmQ, bar(C::B_Q),
-                                    dh * 64, d.qb * 64, d.hq0 + hl);
+                load_tile(sb + C::kOffQ, &tmQ, bar(C::B_Q), d);
                 int* el = elists + (ul & 1) * ls;
                 el[li - 1] = stage_unit<kSub>(a, d, el, reinterpret_cast<uint8_t*>(el + li));
                 mbar_arrive(bar(C::B_Q));
-                // dO once the previous unit's has been copied and read for Delta
-                if (ul > 0 && !mbar_wait(bar(C::B_DOFREE), (ul - 1) & 1, abort_flag, a.status)) break;
-                mbar_expect_tx(bar(C::B_DO), kTile128);
-                for (int hl = 0; hl < 2; ++hl)
-                    for (int dh = 0; dh < 2; ++dh)
-                        tma_load_3d(sb + C::kOffDO + dh * kHalf128 + hl * kHalf64, &tmdO, bar(C::B_DO),
-                                    dh * 64, d.qb * 64, d.hq0 + hl);
-                // Q and dO come from HBM: start bringing the next unit's into L2 now.
-                const int u2 = u + (int)gridDim.x;
-                if (u2 < a.units) {
-                    const int qb2 = a.NQB - 1 - (u2 % a.NQB), bg2 = u2 / a.NQB;
-                    const int hq2 = (bg2 / a.Hkv) * a.Hq + (bg2 % a.Hkv) * 2;
-                    for (int hl = 0; hl < 2; ++hl)
-                        for (int dh = 0; dh < 2; ++dh) {
-                            tma_prefetch_3d(&tmQ, dh * 64, qb2 * 64, hq2 + hl);
-                            tma_prefetch_3d(&tmdO, dh * 64, qb2 * 64, hq2 + hl);
-                        }
-                }
+                last_q = ul;
             }
-            if (last >= 0) {
-                mbar_wait_drain(bar(C::B_Q), last & 1);
-                mbar_wait_drain(bar(C::B_DO), last & 1);
-            }
+            if (last_o >= 0) mbar_wait_drain(bar(C::B_O), last_o & 1);
+            if (last_do >= 0) mbar_wait_drain(bar(C::B_DO), last_do & 1);
+            if (last_q >= 0) mbar_wait_drain(bar(C::B_Q), last_q & 1);
         }
     } else if (warp == 9) {
         // ------------------------------------------------ MMA issuer
@@ -409,17 +419,18 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             int gp0 = 0, ul = 0;
             // Per unit: Q and dO copied into TMEM, then S_0 dP_0 | S_1 | dS_0 -> dQ_0 |
             // dP_1 | S_2 | dS_1 -> dQ_1 | dP_2 ...
-            int* mlist = reinterpret_cast<int*>(smem + C::kOffList) + kListM * slot_ints(a.topk, kSub);
+            // the unit's entry count, staged with its list by the Q/dO producer before
+            // it arrives on C::B_Q (no global load on this thread's path)
+            const int ls = slot_ints(a.topk, kSub);
+            const int* elists = reinterpret_cast<const int*>(smem + C::kOffList) + kListE * ls;
             for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++ul) {
-                const DqUnit d = dq_unit<kSub>(a, u);
-                const int nu = kSub == 1 ? stage_list(a.idx + d.lu * a.topk, a.cnt + d.lu, a.topk, d.qb, mlist)
-                                         : min(__ldg(a.ucnt + d.lu), a.ucap);
-                const int np = ((nu + kSub - 1) / kSub + 1) >> 1;
                 // Q into TMEM once it has landed and the previous unit's last S has read
                 // the previous Q; its staging buffer is then free for the next unit's
                 ok = mbar_wait(bar(C::B_Q), ul & 1, abort_flag, a.status) &&
                      (gp0 == 0 || mbar_wait(bar(C::B_SFULL), (gp0 - 1) & 1, abort_flag, a.status));
                 if (!ok) break;
+                const int nu = elists[(ul & 1) * ls + li - 1];
+                const int np = ((nu + kSub - 1) / kSub + 1) >> 1;
                 tc_fence_after();
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) tmem_cp_128x256b(tmem + kColQ + ks * 8, sdesc_at(dQ0, koff(ks)));
@@ -493,27 +504,58 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         int gp0 = 0, ul = 0;
         const int ls = slot_ints(a.topk, kSub);
         int* lists = reinterpret_cast<int*>(smem + C::kOffList) + kListE * ls;
-        // A unit's O rows and lse (for Delta and P) are fetched at the end of the
-        // previous unit, so that they are in hand when its Q and dO arrive; its
-        // block list is staged by the Q/dO producer before it arrives on C::B_Q.
-        uint4 ov[8];
+        // A unit's lse (for P) is fetched at the end of the previous unit; its block
+        // list is staged by the producer before it arrives on C::B_Q.
         float neg_lse2 = 0.f;
         auto fetch_unit = [&](int u) {
             const DqUnit d = dq_unit<kSub>(a, u);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const int rr = k * 16 + (et >> 4);
-                const int ii = d.qb * 64 + (rr & 63);
-                ov[k] = ii < a.L ? __ldg(reinterpret_cast<const uint4*>(
-                                       a.O + ((size_t)(d.hq0 + (rr >> 6)) * a.L + ii) * 128) + pc)
-                                 : make_uint4(0u, 0u, 0u, 0u);
-            }
             const int i = d.qb * 64 + tok;
             neg_lse2 = i < a.L ? -__ldg(a.lse + (size_t)(d.hq0 + hl) * a.L + i) * kLog2e : -INFINITY;
         };
         if (blockIdx.x < a.units) fetch_unit(blockIdx.x);
-        // Every warp runs every unit (doing no work after an abort), so the one
-        // named barrier per unit is reached the same number of times by all.
+        // Delta_i = dO_i . O_i of local unit ulx from its O tile (in the Q staging
+        // buffer) and dO tile (in its own), both waited for here: the warps of d
+        // half 0 take one row each over the whole head dimension. Returns this
+        // thread's row's value. Every warp calls it once per unit, also after an
+        // abort (doing no work then), so its named barrier is reached the same
+        // number of times by all.
+        auto delta_pass = [&](int ulx) -> float {
+            if (ok) {
+                ok = mbar_wait(bar(C::B_O), ulx & 1, abort_flag, a.status) &&
+                     mbar_wait(bar(C::B_DO), ulx & 1, abort_flag, a.status);
+                ok = __all_sync(0xffffffffu, ok);
+            }
+            if (ok && half == 0) {
+                float acc = 0.f;
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    const uint32_t off = (uint32_t)((c >> 3) * kHalf128) + sw_off(row, c & 7);
+                    const uint4 ov = *reinterpret_cast<const uint4*>(smem + C::kOffQ + off);
+                    const uint4 dv = *reinterpret_cast<const uint4*>(smem + C::kOffDO + off);
+                    const uint32_t ow[4] = {ov.x, ov.y, ov.z, ov.w};
+                    const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float2 fo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ow[j]));
+                        const float2 fd = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&dw[j]));
+                        acc = fmaf(fo.x, fd.x, acc);
+                        acc = fmaf(fo.y, fd.y, acc);
+                    }
+                }
+                dpart[row] = acc;
+            }
+            named_barrier(1, 256);  // Delta is visible
+            const float v = dpart[row];
+            // This thread is done with O, dO and Delta's exchange slots: Q may be
+            // loaded over O, the next unit's dO loaded once dO has been copied, and
+            // dpart rewritten once all have arrived.
+            if (ok) {
+                mbar_arrive(bar(C::B_OFREE));
+                mbar_arrive(bar(C::B_DOFREE));
+            }
+            return v;
+        };
+        float dlt_next = 0.f;
         for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
             const int* list = lists + (ul & 1) * ls;
             const DqUnit d = dq_unit<kSub>(a, u);
@@ -522,17 +564,17 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const bool valid = i < a.L;
             const size_t ridx = (size_t)(d.hq0 + hl) * a.L + (valid ? i : 0);
             const float nl2 = neg_lse2;
-            {  // two units ahead: block list, count, O rows and lse into L2 (all roles
-               // read a unit's list; O and lse are fetched into registers a unit ahead)
-                const int u3 = u + 2 * (int)gridDim.x;
+            {  // into L2: the next unit's lse (read at the end of this unit), and the
+               // block list and count two units ahead (staged a unit ahead)
+                const int u1 = u + (int)gridDim.x, u3 = u + 2 * (int)gridDim.x;
+                if (u1 < a.units) {
+                    const DqUnit d1 = dq_unit<kSub>(a, u1);
+                    const int r1 = et >> 1, i1 = d1.qb * 64 + (r1 & 63);
+                    if (i1 < a.L && (r1 & 31) == 0 && (et & 1) == 0)
+                        prefetch_l2(a.lse + (size_t)(d1.hq0 + (r1 >> 6)) * a.L + i1);
+                }
                 if (u3 < a.units) {
                     const DqUnit d3 = dq_unit<kSub>(a, u3);
-                    const int r3 = et >> 1, i3 = d3.qb * 64 + (r3 & 63);
-                    if (i3 < a.L) {
-                        const size_t row3 = (size_t)(d3.hq0 + (r3 >> 6)) * a.L + i3;
-                        prefetch_l2(a.O + row3 * 128 + 64 * (et & 1));
-                        if ((r3 & 31) == 0 && (et & 1) == 0) prefetch_l2(a.lse + row3);
-                    }
                     if constexpr (kSub == 1) {
                         if (et == 0) prefetch_l2(a.cnt + d3.lu);
                         if (et < 4 && et * 32 < a.topk) prefetch_l2(a.idx + d3.lu * a.topk + et * 32);
@@ -543,41 +585,15 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                     }
                 }
             }
+            // Delta of the CTA's first unit here (its Q is loaded over its O only after
+            // that); every later unit's was computed during the previous unit
+            if (ul == 0) dlt_next = delta_pass(0);
             if (ok) {
                 ok = mbar_wait(bar(C::B_Q), ul & 1, abort_flag, a.status);
                 if (ok) mbar_arrive(bar(C::B_QFREE));
-                ok = ok && mbar_wait(bar(C::B_DO), ul & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
-            // Delta_i = dO_i . O_i: O in coalesced 16-byte pieces (16 threads per
-            // 256-byte row, 16 rows per pass), dO from the tile loaded for the dP
-            // MMAs; a fixed shuffle tree adds the pieces.
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const int rr = k * 16 + (et >> 4);
-                float acc = 0.f;
-                if (ok) {
-                    const uint4 dv = *reinterpret_cast<const uint4*>(
-                        smem + C::kOffDO + (pc >> 3) * kHalf128 + (rr >> 6) * kHalf64 + sw_off(rr & 63, pc & 7));
-                    const uint32_t ow[4] = {ov[k].x, ov[k].y, ov[k].z, ov[k].w};
-                    const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w};
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const float2 fo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ow[j]));
-                        const float2 fd = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&dw[j]));
-                        acc = fmaf(fo.x, fd.x, acc);
-                        acc = fmaf(fo.y, fd.y, acc);
-                    }
-                }
-#pragma unroll
-                for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-                if (pc == 0) dpart[rr] = acc;
-            }
-            named_barrier(1, 256);  // Delta's pieces are visible
-            const float dlt = dpart[row];
-            // This thread is done with dO and with Delta's exchange slots: the next
-            // unit's dO may be loaded (and dpart rewritten) once all have arrived.
-            if (ok) mbar_arrive(bar(C::B_DOFREE));
+            const float dlt = dlt_next;
             const int n = list[li - 1];
             const int nt = (n + kSub - 1) / kSub;  // 64-key tiles
             const int np = (nt + 1) >> 1;
@@ -586,6 +602,10 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const int qb_r = qb * kSub + jr;
             if (ok && half == 0 && valid) a.delta[ridx] = dlt;
             const int u2 = u + (int)gridDim.x;
+            // the next unit's Delta, after pair pd of this one (its O and dO tiles
+            // were loaded at the start of this unit)
+            const int pd = min(2, np - 1);
+            bool next_delta = u2 < a.units;
             for (int p = 0; ok && p < np; ++p) {
                 const int gp = gp0 + p;
                 ok = mbar_wait(bar(C::B_SFULL), gp & 1, abort_flag, a.status);
@@ -657,44 +677,42 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 tmem_st32(lane_base + kColDP + 64 * half, dsv);
                 tc_fence_before();
                 mbar_arrive(bar(C::B_DSFULL + (gp & 1)));
+                if (p == pd && next_delta) {
+                    dlt_next = delta_pass(ul + 1);
+                    next_delta = false;
+                }
             }
             gp0 += np;
-            // the next unit's inputs: their latency overlaps this unit's last dQ
-            // MMAs and its epilogue
-            if (u2 < a.units) fetch_unit(u2);
+            if (next_delta) dlt_next = delta_pass(ul + 1);  // no pair reached pd (or an abort)
+            if (u2 < a.units) fetch_unit(u2);  // the next unit's lse
             if (ok) {
                 ok = mbar_wait(bar(C::B_FINAL), ul & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
             }
             if (ok) {
-                // dQ row `row`, columns [64 half, 64 half + 64), straight to global
-                // memory, 32 columns at a time
+                // dQ row `row`, columns [64 half, 64 half + 64): read out of TMEM in
+                // one go, so that the next unit's dQ MMAs may start, then stored
                 tc_fence_after();
-#pragma unroll 1
-                for (int c2 = 0; c2 < 2; ++c2) {
-                    uint32_t o[32];
-                    if (n > 0) {
-                        tmem_ld32(lane_base + kColDQ + 64 * half + 32 * c2, o);
-                    } else {
+                uint32_t o[64];
+                if (n > 0) {
+                    tmem_ld64(lane_base + kColDQ + 64 * half, o);
+                } else {
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) o[c] = 0u;
-                    }
-                    if (c2 == 1) {
-                        tc_fence_before();
-                        mbar_arrive(bar(C::B_DQFREE));
-                    }
-                    if (valid) {
-                        uint4* dst = reinterpret_cast<uint4*>(a.dQ + ridx * 128 + 64 * half + 32 * c2);
-                        const float s = a.sm_scale;
+                    for (int c = 0; c < 64; ++c) o[c] = 0u;
+                }
+                tc_fence_before();
+                mbar_arrive(bar(C::B_DQFREE));
+                if (valid) {
+                    uint4* dst = reinterpret_cast<uint4*>(a.dQ + ridx * 128 + 64 * half);
+                    const float s = a.sm_scale;
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            uint4 v;
-                            v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * s, __uint_as_float(o[8 * q + 1]) * s);
-                            v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * s, __uint_as_float(o[8 * q + 3]) * s);
-                            v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * s, __uint_as_float(o[8 * q + 5]) * s);
-                            v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * s, __uint_as_float(o[8 * q + 7]) * s);
-                            dst[q] = v;
-                        }
+                    for (int q = 0; q < 8; ++q) {
+                        uint4 v;
+                        v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * s, __uint_as_float(o[8 * q + 1]) * s);
+                        v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * s, __uint_as_float(o[8 * q + 3]) * s);
+                        v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * s, __uint_as_float(o[8 * q + 5]) * s);
+                        v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * s, __uint_as_float(o[8 * q + 7]) * s);
+                        dst[q] = v;
                     }
                 }
             }
@@ -1363,13 +1381,13 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
                          void* dQ, int* status, cudaStream_t st) {
     const int bm = s.block_size, kSub = 64 / bm;
     const int NQB = (s.L + bm - 1) / bm, nsb = (s.L + 63) / 64;
-    CUtensorMap tq, tk, tv, tdo;
+    CUtensorMap tq, tk, tv, tdo, to;
     const uint64_t pq = (uint64_t)s.B * s.Hq, pk = (uint64_t)s.B * s.Hkv;
-    // Q and dO in 64-row boxes (the span's tokens); K and V gathered in boxes of one block
+    // Q, dO and O in 64-row boxes (the span's tokens); K and V gathered in boxes of one block
     if (!make_tmap_bf16_rows128(&tq, Q, s.L, pq, 64) ||
         !make_tmap_bf16_rows128(&tk, K, s.L, pk, (uint32_t)bm) ||
         !make_tmap_bf16_rows128(&tv, V, s.L, pk, (uint32_t)bm) ||
-        !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64))
+        !make_tmap_bf16_rows128(&tdo, dO, s.L, pq, 64) || !make_tmap_bf16_rows128(&to, O, s.L, pq, 64))
         return cudaErrorInvalidValue;
     const size_t smem = kSub == 1 ? dq::smem_bytes<1>(topk) : kSub == 2 ? dq::smem_bytes<2>(topk)
                                                                          : dq::smem_bytes<4>(topk);
@@ -1385,7 +1403,7 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
                 static_cast<__nv_bfloat16*>(dQ), status, s.Hq, s.Hkv, s.L, NQB, topk, units, nsb,
                 kSub * topk, sm_scale * kLog2e, sm_scale};
     ProfScope prof(K_BWD_DQ, st);
-    kern<<<(unsigned)min(units, nsm), dq::kThreads, smem, st>>>(tq, tk, tv, tdo, args);
+    kern<<<(unsigned)min(units, nsm), dq::kThreads, smem, st>>>(tq, tk, tv, tdo, to, args);
     return cudaGetLastError();
 }
 
