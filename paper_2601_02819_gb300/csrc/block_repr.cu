@@ -4,7 +4,7 @@
 // One warp reduces one m x 128 bf16 block (m = 64: 16 KB; the kernel is
 // instantiated for m = 16, 32, 64). Each half-warp streams one
 // 256-byte row per step with 16-byte read-only loads (lane c of the half owns
-// columns 8c..8c+7), so a warp keeps eight 512-byte row pairs in flight. The
+// columns 8c..8c+7), so a warp keeps up to sixteen 512-byte row pairs in flight. The
 // punctuation count of the block comes from warp ballots over its m mask
 // bytes. The sum and the punctuation-masked sum are kept in fp32 and combined
 // once across the two half-warps; the result is rounded to bf16 once.
@@ -50,16 +50,18 @@ __device__ __forceinline__ void repr_one_block(const __nv_bfloat16* __restrict__
 #pragma unroll
     for (int j = 0; j < 8; ++j) { s0[j] = 0.f; sp[j] = 0.f; }
 
+    // up to 32 rows (16 loads of 16 bytes per lane, 8 KB per warp) in flight per batch
+    constexpr int kRB = BM < 32 ? BM : 32;
 #pragma unroll
-    for (int base = 0; base < BM; base += 16) {
-        uint4 v[8];
+    for (int base = 0; base < BM; base += kRB) {
+        uint4 v[kRB / 2];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < kRB / 2; ++u) {
             const int r = base + 2 * u + half;
             v[u] = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)r * kD));
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < kRB / 2; ++u) {
             const int r = base + 2 * u + half;
             add8(s0, v[u]);
             const bool p = ((r < 32 ? lo >> r : hi >> (r - 32)) & 1u) != 0;
