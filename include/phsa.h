@@ -402,6 +402,18 @@ int phsa_selftest_tcgen05(const void* A, const void* B, const void* V, float* S,
  */
 size_t phsa_test_set_select_tc_limit(size_t bytes);
 
+/* Testing hook. The backward transposes the block lists (KV block -> the
+ * query blocks that selected it) in one launch while one (batch, KV head)'s
+ * bitmap of (KV span, query block) pairs fits in 160 KB of shared memory
+ * (up to 1140 query blocks of 64 tokens, or 2048 of 16), else in two
+ * launches through a bitmap in global memory. This call sets that switch
+ * point to `bytes` (0, or more than 160 KB, restores the default) so that a
+ * test can reach the two-launch form on short inputs; both build the same
+ * lists. Returns the previous value. Affects every later call in the
+ * process; not meant for production use.
+ */
+size_t phsa_test_set_idx_smem_limit(size_t bytes);
+
 /* Library version as "major.minor.patch". */
 const char* phsa_version(void);
 

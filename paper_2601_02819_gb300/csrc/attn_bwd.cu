@@ -4,7 +4,8 @@
 //
 // Kernels, in launch order, all on the caller's stream:
 //   delta      Delta_i = dO_i . O_i (fp32), half a warp per row.
-//   idx_mark   sets bit qb of bitmap[(b,g,t)] for every selected (qb -> t).
+//   idx_mark   sets bit qb of bitmap[(b,g,t)] for every selected (qb -> t)
+//              (inside idx_build, in shared memory, when the bitmap fits).
 //   idx_build  one CTA per (b,g): counts each KV block's selecting query
 //              blocks, scans, writes the ascending query-block list of every
 //              KV block (a CSR transpose of block_idx), and cuts lists longer
@@ -19,6 +20,8 @@
 //   dq         one CTA per (query block, KV head): recomputes S, P, dP, dS
 //              over the selected blocks and accumulates dQ += dS K.
 // Every sum runs in a fixed order, so results are bit-reproducible.
+#include <atomic>
+
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "union.cuh"
@@ -29,6 +32,14 @@ namespace {
 
 constexpr int kChunk = kBwdChunk;  // query blocks per dK/dV work item
 constexpr int kBuildCache = 8192;   // KV blocks whose counts the index build keeps on chip
+// Largest bitmap of one (b, g) that the index build keeps in shared memory
+// (beside its 32 KB of counts): 160 KB covers 1140 query blocks of 64 and
+// 2048 query blocks of 16 (32k tokens at m = 16).
+constexpr size_t kIdxSmemBits = 160u * 1024u;
+// The switch point in use; only phsa_test_set_idx_smem_limit lowers it, so
+// that tests reach the two-launch transpose (bitmap in global memory) on
+// short sequences.
+std::atomic<size_t> g_idx_smem_limit{kIdxSmemBits};
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -62,6 +73,45 @@ delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restric
 // each (span, query block) pair also records which of the span's kSub blocks
 // the query block selected: kSub bits at bit (qb * kSub) % 32 of word
 // (qb * kSub) / 32 of the span's mask row.
+// Marks the selections of unit u (query block qb of one (b, g)) in the bitmap
+// rows `bits` of that (b, g) (global or shared memory) and, at m < 64, in its
+// mask rows. The entries are loaded eight at a time (independent loads), then
+// checked in list order: -1 is skipped, an index that is negative, in the
+// query's future or not ascending is recorded as a device index error.
+__device__ __forceinline__ void mark_unit(const int32_t* __restrict__ idx,
+                                          const int32_t* __restrict__ cnt, long long u, int qb,
+                                          int kSub, int topk, int words, int mwords,
+                                          uint32_t* bits, uint32_t* __restrict__ masks,
+                                          int* status) {
+    int n = cnt[u];
+    if (n < 0 || n > topk) {
+        set_status(status, PHSA_ERR_DEVICE_INDEX);
+        n = n < 0 ? 0 : topk;
+    }
+    const int32_t* row = idx + u * topk;
+    int prev = -1;
+    for (int j0 = 0; j0 < n; j0 += 8) {
+        int tv[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) tv[k] = j0 + k < n ? __ldg(row + j0 + k) : -1;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int t = tv[k];
+            if (t == -1) continue;
+            if (t < 0 || t > qb || t <= prev) {
+                set_status(status, PHSA_ERR_DEVICE_INDEX);
+                continue;
+            }
+            prev = t;
+            const int T = t / kSub;
+            atomicOr(&bits[T * words + (qb >> 5)], 1u << (qb & 31));
+            if (kSub > 1)
+                atomicOr(&masks[(size_t)T * mwords + ((qb * kSub) >> 5)],
+                         (1u << (t - T * kSub)) << ((qb * kSub) & 31));
+        }
+    }
+}
+
 __global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt,
                                 long long units, int NQB, int nrows, int kSub, int topk, int words,
                                 int mwords, uint32_t* __restrict__ bits, uint32_t* __restrict__ masks,
@@ -70,25 +120,54 @@ __global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* 
     if (u >= units) return;
     const int qb = (int)(u % NQB);
     const long long bg = u / NQB;
-    int n = cnt[u];
-    if (n < 0 || n > topk) {
-        set_status(status, PHSA_ERR_DEVICE_INDEX);
-        n = n < 0 ? 0 : topk;
-    }
-    int prev = -1;
-    for (int j = 0; j < n; ++j) {
-        const int t = idx[u * topk + j];
-        if (t == -1) continue;
-        if (t < 0 || t > qb || t <= prev) {
+    mark_unit(idx, cnt, u, qb, kSub, topk, words, mwords, bits + bg * nrows * words,
+              masks + bg * nrows * mwords, status);
+}
+
+// The bitmap of one (b, g) in shared memory, rows of rs words: thread q marks
+// query block q's selections. The 32 query blocks of a warp share one bitmap
+// column (word q / 32), so at each list position the lanes that selected the
+// same KV span set their bits with one OR (the lanes of __match_any_sync are
+// exactly those bits). The checks are mark_unit's, in list order per lane.
+__device__ __forceinline__ void mark_warp(const int32_t* __restrict__ idx,
+                                          const int32_t* __restrict__ cnt, long long u0, int NQB,
+                                          int kSub, int topk, int rs, int mwords, uint32_t* bits,
+                                          uint32_t* __restrict__ masks, int* status) {
+    const int lane = threadIdx.x & 31;
+    for (int qw = threadIdx.x & ~31; qw < NQB; qw += blockDim.x) {
+        const int qb = qw + lane;
+        const bool live = qb < NQB;
+        int n = live ? cnt[u0 + qb] : 0;
+        if (n < 0 || n > topk) {
             set_status(status, PHSA_ERR_DEVICE_INDEX);
-            continue;
+            n = n < 0 ? 0 : topk;
         }
-        prev = t;
-        const int T = t / kSub;
-        atomicOr(&bits[(bg * nrows + T) * words + (qb >> 5)], 1u << (qb & 31));
-        if (kSub > 1)
-            atomicOr(&masks[(bg * nrows + T) * mwords + ((qb * kSub) >> 5)],
-                     (1u << (t - T * kSub)) << ((qb * kSub) & 31));
+        const int nmax = __reduce_max_sync(0xffffffffu, n);
+        const int32_t* row = idx + (u0 + (live ? qb : 0)) * topk;
+        int prev = -1;
+        for (int j0 = 0; j0 < nmax; j0 += 8) {
+            int tv[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) tv[k] = j0 + k < n ? __ldg(row + j0 + k) : -1;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                int t = tv[k];
+                if (t != -1) {
+                    if (t < 0 || t > qb || t <= prev) {
+                        set_status(status, PHSA_ERR_DEVICE_INDEX);
+                        t = -1;
+                    } else {
+                        prev = t;
+                    }
+                }
+                const int T = t < 0 ? -1 : t / kSub;
+                const unsigned grp = __match_any_sync(0xffffffffu, T);
+                if (T >= 0 && lane == __ffs(grp) - 1) atomicOr(&bits[T * rs + (qw >> 5)], grp);
+                if (kSub > 1 && T >= 0)
+                    atomicOr(&masks[(size_t)T * mwords + ((qb * kSub) >> 5)],
+                             (1u << (t - T * kSub)) << ((qb * kSub) & 31));
+            }
+        }
     }
 }
 
@@ -123,12 +202,19 @@ __device__ int block_excl_scan(int v, int* tmp, int& total) {
 
 // One CTA per (b, g): the ascending query-block list of every row (KV span),
 // cut into work items of at most kChunk iterations of kSub query blocks each.
+// kMark: the CTA first builds its (b, g)'s bitmap in shared memory from the
+// block lists itself (mark_warp), so that the transpose is
+// one launch and the bitmap never goes through global memory; otherwise it
+// reads the bitmap idx_mark_kernel left in `bits`.
+template <bool kMark>
 __global__ void __launch_bounds__(1024)
-idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub, int topk,
-                 int words, int work_max, int slot_max, TInfo* __restrict__ tinfo,
-                 int32_t* __restrict__ qlist, int2* __restrict__ work, int32_t* __restrict__ nwork,
-                 int* __restrict__ arrive, int2* __restrict__ queue, int* __restrict__ qcount,
-                 int* status) {
+idx_build_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt,
+                 const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub, int topk,
+                 int words, int mwords, uint32_t* __restrict__ masks, int work_max, int slot_max,
+                 TInfo* __restrict__ tinfo, int32_t* __restrict__ qlist, int2* __restrict__ work,
+                 int32_t* __restrict__ nwork, int* __restrict__ arrive, int2* __restrict__ queue,
+                 int* __restrict__ qcount, int* status) {
+    extern __shared__ uint32_t sbits[];  // kMark: the bitmap of this (b, g)
     __shared__ int tmp[32];
     __shared__ int bin[kChunk + 1];  // items per iteration count, then queue cursors
     __shared__ int ncache[kBuildCache];  // selecting-query count of each KV span
@@ -136,16 +222,29 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub
     const int kChunkQ = kChunk * kSub;  // query blocks per work item
     const int per = (nrows + 1023) / 1024;  // KV spans counted by each thread
     const int t0 = threadIdx.x * per;
-    const uint32_t* bb = bits + (size_t)bg * nrows * words;
+    const uint32_t* bb;
+    int rs;  // words per bitmap row: odd in shared memory, so that rows fall in different banks
+    if constexpr (kMark) {
+        rs = words | 1;
+        for (int i = threadIdx.x; i < nrows * rs; i += blockDim.x) sbits[i] = 0u;
+        __syncthreads();
+        mark_warp(idx, cnt, (long long)bg * NQB, NQB, kSub, topk, rs, mwords, sbits,
+                  masks + (size_t)bg * nrows * mwords, status);
+        __syncthreads();
+        bb = sbits;
+    } else {
+        rs = words;
+        bb = bits + (size_t)bg * nrows * words;
+    }
     // The count of a block: its bitmap row's popcount, read with independent
     // loads. The first kBuildCache blocks keep theirs in shared memory for the
     // later passes (each thread reads back only its own entries); any block
     // beyond is counted again where it is needed.
     auto count_row = [&](int t) {
-        const uint32_t* row = bb + (size_t)t * words;
+        const uint32_t* row = bb + (size_t)t * rs;
         int n = 0;
 #pragma unroll 8
-        for (int w = 0; w < words; ++w) n += __popc(__ldg(row + w));
+        for (int w = 0; w < words; ++w) n += __popc(row[w]);
         return n;
     };
     auto count_of = [&](int t) { return t < kBuildCache ? ncache[t] : count_row(t); };
@@ -212,6 +311,7 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub
         info.nch = nch;
         info.slot = (nch > 1 && osl + nch <= slot_max) ? osl : -1;
         ti[t] = info;
+        if (t < kBuildCache) ncache[t] = on;  // from here on: the list's offset
         arrive[(size_t)bg * nrows + t] = 0;
         for (int c = 0; c < nch && och + c < work_max; ++c) {
             wk[och + c] = make_int2(t, c);
@@ -235,7 +335,7 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub
 #pragma unroll
         for (int j = 0; j < kBatch; ++j) {
             const int t = tb + 32 * j;
-            pos[j] = t < nrows ? ti[t].off : 0;
+            pos[j] = t >= nrows ? 0 : t < kBuildCache ? ncache[t] : ti[t].off;
         }
         for (int w0 = 0; w0 < words; w0 += 32) {
             const int w = w0 + lane;
@@ -243,7 +343,7 @@ idx_build_kernel(const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub
 #pragma unroll
             for (int j = 0; j < kBatch; ++j) {
                 const int t = tb + 32 * j;
-                m[j] = (t < nrows && w < words) ? bb[(size_t)t * words + w] : 0u;
+                m[j] = (t < nrows && w < words) ? bb[(size_t)t * rs + w] : 0u;
             }
 #pragma unroll
             for (int j = 0; j < kBatch; ++j) {
@@ -788,17 +888,29 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
         cudaSuccess)
         return e;
     const long long units = (long long)bgs * l.nqb;
-    {
-        ProfScope prof(K_BWD_MARK, st);
-        idx_mark_kernel<<<(unsigned)((units + 255) / 256), 256, 0, st>>>(
-            idx, cnt, units, l.nqb, l.nrows, l.kSub, topk, l.words, l.mwords, bits, masks, status);
-    }
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    {
+    const size_t sbits = (size_t)l.nrows * (l.words | 1) * 4;  // one (b, g)'s bitmap
+    if (sbits <= g_idx_smem_limit.load()) {
+        // mark and build in one launch, the bitmap in shared memory
+        auto kern = idx_build_kernel<true>;
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)sbits)) != cudaSuccess)
+            return e;
         ProfScope prof(K_BWD_BUILD, st);
-        idx_build_kernel<<<bgs, 1024, 0, st>>>(bits, l.nqb, l.nrows, l.kSub, topk, l.words,
-                                               l.work_max, l.slot_max, tinfo, qlist, work, nwork,
-                                               arrive, queue, qctl, status);
+        kern<<<bgs, 1024, sbits, st>>>(idx, cnt, bits, l.nqb, l.nrows, l.kSub, topk, l.words,
+                                       l.mwords, masks, l.work_max, l.slot_max, tinfo, qlist, work,
+                                       nwork, arrive, queue, qctl, status);
+    } else {
+        {
+            ProfScope prof(K_BWD_MARK, st);
+            idx_mark_kernel<<<(unsigned)((units + 255) / 256), 256, 0, st>>>(
+                idx, cnt, units, l.nqb, l.nrows, l.kSub, topk, l.words, l.mwords, bits, masks,
+                status);
+        }
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        ProfScope prof(K_BWD_BUILD, st);
+        idx_build_kernel<false><<<bgs, 1024, 0, st>>>(
+            idx, cnt, bits, l.nqb, l.nrows, l.kSub, topk, l.words, l.mwords, masks, l.work_max,
+            l.slot_max, tinfo, qlist, work, nwork, arrive, queue, qctl, status);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
@@ -833,3 +945,8 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
 }
 
 }  // namespace phsa
+
+extern "C" size_t phsa_test_set_idx_smem_limit(size_t bytes) {
+    const size_t v = bytes == 0 || bytes > phsa::kIdxSmemBits ? phsa::kIdxSmemBits : bytes;
+    return phsa::g_idx_smem_limit.exchange(v);
+}

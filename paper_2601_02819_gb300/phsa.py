@@ -108,6 +108,8 @@ def _declare(L):
     L.phsa_prefill_append.restype = I
     L.phsa_test_set_select_tc_limit.argtypes = [SZ]
     L.phsa_test_set_select_tc_limit.restype = SZ
+    L.phsa_test_set_idx_smem_limit.argtypes = [SZ]
+    L.phsa_test_set_idx_smem_limit.restype = SZ
     for fn in ("phsa_decode_update_repr", "phsa_decode_select", "phsa_decode_attn",
                "phsa_decode_append", "phsa_punct_mask",
                "phsa_build_block_repr", "phsa_select_blocks", "phsa_sparse_attn_fwd",
@@ -561,6 +563,13 @@ def phsa_test_set_select_tc_limit(nbytes: int) -> int:
     the warp-level selection of GQA pairs at block sizes 16 and 32 (0 restores
     the default of 227 KB). Returns the previous value."""
     return int(load().phsa_test_set_select_tc_limit(int(nbytes)))
+
+
+def phsa_test_set_idx_smem_limit(nbytes: int) -> int:
+    """Testing hook: the shared-memory switch point between the one-launch and
+    the two-launch transpose of the block lists in the backward (0 restores
+    the default of 160 KB). Returns the previous value."""
+    return int(load().phsa_test_set_idx_smem_limit(int(nbytes)))
 
 
 def phsa_get_device_status(stream=None) -> int:

@@ -157,3 +157,38 @@ def test_argument_errors_raise():
         phsa.phsa_sparse_attn_fwd(Q, K, K, idx, cnt, sm_scale=-1.0)
     with pytest.raises(phsa.PhsaError):
         phsa.phsa_select_blocks(Q, K[:, :, :2], 1, topk=1, n_init=1, n_local=1)
+
+
+@pytest.mark.parametrize("m,B,Hq,Hkv,L,topk,n_init", [
+    (64, 1, 2, 1, 64 * 100 + 13, 8, 4),   # GQA pair; multi-chunk lists
+    (64, 2, 3, 3, 64 * 21 + 5, 6, 1),     # one query head per KV head
+    (16, 1, 2, 1, 16 * 300 + 5, 20, 2),   # m = 16: mask rows per span
+    (32, 1, 4, 2, 32 * 25 + 17, 4, 1),    # m = 32
+])
+def test_backward_index_transpose_forms_agree(m, B, Hq, Hkv, L, topk, n_init):
+    # The one-launch transpose (bitmap in shared memory) and the two-launch
+    # form (bitmap in global memory, used when a (b, g)'s bitmap exceeds
+    # 160 KB) build the same KV-block lists, so the gradients are identical.
+    rng = np.random.default_rng(L + 17 * m)
+    f = lambda *s: inputs.f32_to_bf16_bits(rng.standard_normal(s).astype(np.float32))
+    Q, K, V, dO = f(B, Hq, L, D), f(B, Hkv, L, D), f(B, Hkv, L, D), f(B, Hq, L, D)
+    mask = (rng.random((B, L)) < 0.06).astype(np.uint8)
+    Kr = oracle.block_repr(K, mask, m, 0.5)
+    idx, cnt = oracle.select_blocks(Q, Kr, L, m, topk, n_init, 1, SCALE)
+    Qd, Kd, Vd, dOd = (to_dev_bf16(a) for a in (Q, K, V, dO))
+    it, ct = torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda()
+    O, lse = phsa.phsa_sparse_attn_fwd(Qd, Kd, Vd, it, ct, block_size=m)
+    g_smem = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct, block_size=m)
+    prev = phsa.phsa_test_set_idx_smem_limit(1)
+    try:
+        g_glob = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct, block_size=m)
+        torch.cuda.synchronize()
+    finally:
+        phsa.phsa_test_set_idx_smem_limit(prev)
+    assert phsa.phsa_get_device_status() == 0
+    for a, b in zip(g_smem, g_glob):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    rQ, rK, rV = oracle.sparse_attn_bwd(Q, K, V, dO, idx, cnt, m, SCALE)
+    assert_close("dQ", bf16_to_f64(g_smem[0]), rQ)
+    assert_close("dK", bf16_to_f64(g_smem[1]), rK)
+    assert_close("dV", bf16_to_f64(g_smem[2]), rV)
