@@ -233,10 +233,13 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                         mbar_arrive(bar(B_KFULL + slot));
                         continue;
                     }
+                    // four 8 KB boxes (64 rows x 64 columns): TMA moves them faster into one
+                    // SM than two 16 KB boxes
                     mbar_expect_tx(bar(B_KFULL + slot), kTile);
                     for (int dh = 0; dh < 2; ++dh)
-                        tma_load_3d(sb + kOffKr + slot * kTile + dh * kHalf, &tmKr, bar(B_KFULL + slot),
-                                    dh * 64, d.c_lo + c * kCand, d.bg);
+                        for (int rh = 0; rh < 2; ++rh)
+                            tma_load_3d(sb + kOffKr + slot * kTile + dh * kHalf + rh * (kHalf / 2), &tmKr,
+                                        bar(B_KFULL + slot), dh * 64, d.c_lo + c * kCand + 64 * rh, d.bg);
                     if (s == 0) {  // Q once the previous unit's last MMA has read the old one
                         if (su > 0 && !mbar_wait(bar(B_QFREE), (su - 1) & 1, abort_flag, a.status)) {
                             ok = false;
@@ -338,9 +341,15 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                     key[r] = cj < nC ? key_of(cj) : 0ull;
                 }
                 for (int k = 0; k < ksel; ++k) {
-                    unsigned long long best = key[0];
+                    // the lane's largest key: a tree of depth 4 instead of a chain of 15
+                    unsigned long long tr[kRegKeys / 2];
 #pragma unroll
-                    for (int r = 1; r < kRegKeys; ++r) best = topk::umax64(best, key[r]);
+                    for (int r = 0; r < kRegKeys / 2; ++r) tr[r] = topk::umax64(key[r], key[r + kRegKeys / 2]);
+#pragma unroll
+                    for (int w = kRegKeys / 4; w >= 1; w >>= 1)
+#pragma unroll
+                        for (int r = 0; r < w; ++r) tr[r] = topk::umax64(tr[r], tr[r + w]);
+                    const unsigned long long best = tr[0];
                     const unsigned mh = (unsigned)(best >> 32), ml = (unsigned)best;
                     const unsigned bh = __reduce_max_sync(0xffffffffu, mh);
                     const unsigned bl = __reduce_max_sync(0xffffffffu, mh == bh ? ml : 0u);
@@ -663,7 +672,7 @@ cudaError_t launch_select_tc_unit(const void* Q, const void* Krepr, const phsa_s
     // Krepr may be absent when no query block has a candidate (T < 2): the map is
     // then built over Q, which is never read through it.
     if (!make_tmap_bf16_rows128(&tkr, T > 0 ? Krepr : Q, T > 0 ? T : 1,
-                                (uint64_t)s.B * s.Hkv, 128))
+                                (uint64_t)s.B * s.Hkv, 64))
         return cudaErrorInvalidValue;
     const size_t smem = select_tc_smem(NQB, p.topk, kSub);
     const bool mx = p.aggregation == PHSA_AGG_MAX_LOGIT;
