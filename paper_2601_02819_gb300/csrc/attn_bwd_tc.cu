@@ -1107,8 +1107,12 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     const int b = nv & 1;
                     const uint32_t ph = (uint32_t)((nv >> 1) & 1);
                     const int sq = (2 * nv) % kSlots, sd = (2 * nv + 1) % kSlots;  // Q_i, dO_i
-                    // K dimension = the 128 stacked query rows, 16 per MMA
-                    ok = mbar_wait(bar(B_PFULL + b), ph, abort_flag, a.status);
+                    // K dimension = the 128 stacked query rows, 16 per MMA. P being stored
+                    // implies that S, hence Q_i, has landed, but not dO_i: its half-slot
+                    // has its own barrier, which this thread waits on too.
+                    ok = mbar_wait(bar(B_PFULL + b), ph, abort_flag, a.status) &&
+                         mbar_wait(bar(B_HFULL + sd), (uint32_t)(((2 * nv + 1) / kSlots) & 1), abort_flag,
+                                   a.status);
                     if (!ok) break;
                     tc_fence_after();
                     const uint64_t dt = sdesc_at(dSlT0, sd * kTile128);
@@ -1121,7 +1125,8 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     ok = mbar_wait(bar(B_DPFULL + b), ph, abort_flag, a.status);
                     if (!ok) break;
                     mma_commit(bar(B_HEMPTY + sd));
-                    ok = mbar_wait(bar(B_DSFULL + b), ph, abort_flag, a.status);
+                    ok = mbar_wait(bar(B_DSFULL + b), ph, abort_flag, a.status) &&
+                         mbar_wait(bar(B_HFULL + sq), (uint32_t)(((2 * nv) / kSlots) & 1), abort_flag, a.status);
                     if (!ok) break;
                     tc_fence_after();
                     const uint64_t qt = sdesc_at(dSlT0, sq * kTile128);

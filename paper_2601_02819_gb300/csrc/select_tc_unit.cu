@@ -26,8 +26,10 @@
 // pass 2 alone, each thread taking the largest score of its candidate over its
 // 64 rows (rows past L excluded), A[t] = max(half 0, half 1) * scale.
 // Warps 0-7 do the elementwise work, warp 8 issues TMA, warp 9 the MMAs,
-// warp 10 the top-k. The ring, the TMEM buffers and every barrier run on
-// counters that continue across units. Every wait is bounded in time.
+// warps 10 and 11 the top-k of alternate units (one warp's top-k of a long
+// unit took longer than the elementwise warps' scoring of the next one). The
+// ring, the TMEM buffers and every barrier run on counters that continue
+// across units. Every wait is bounded in time.
 #include "phsa_common.cuh"
 #include "phsa_internal.h"
 #include "tc_common.cuh"
@@ -49,17 +51,17 @@ constexpr int kOffBar = kOffStats + 5 * 128 * 4;
 constexpr int B_Q = 0, B_QFREE = 1, B_KFULL = 2, B_KEMPTY = 4, B_SFULL = 6, B_SFREE = 8,
               B_AFULL = 10, B_AFREE = 12, B_DRAIN = 14, kNumBars = 15;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
-constexpr int kOffA = kOffMisc + 16;  // 2 buffers x (A0[NQB], A1[NQB]), then sel[topk]
-constexpr int kThreads = 352;
+constexpr int kOffA = kOffMisc + 16;  // 2 buffers x (A0[NQB], A1[NQB]), then sel[2][topk]
+constexpr int kThreads = 384;
 constexpr uint32_t kTmemCols = 256;
-constexpr int kRegKeys = 16;  // candidate keys per lane kept in registers by the top-k warp
+constexpr int kRegKeys = 16;  // candidate keys per lane kept in registers by the top-k warps
 
 // kSub query blocks of m = 64 / kSub tokens share a unit (the 64-token span):
 // A holds two buffers of two halves (kSub = 1) or one buffer of kSub x two
 // halves (kSub > 1, where the elementwise warps run the top-k themselves).
 size_t select_tc_smem(int nqb, int topk, int kSub) {
     const size_t na = kSub == 1 ? 4 : (size_t)2 * kSub;
-    return 1024 + (size_t)kOffA + na * nqb * 4 + (size_t)topk * 4 + 16;
+    return 1024 + (size_t)kOffA + na * nqb * 4 + (size_t)2 * topk * 4 + 16;
 }
 
 struct SelArgs {
@@ -184,7 +186,7 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
     float* pm = m2s + 128;  // [2][128] per-half running max (pass 1)
     float* pz = pm + 256;   // [2][128] per-half running sum
     float* Abuf = reinterpret_cast<float*>(smem + kOffA);  // [2][A0 | A1], NQB each
-    int* sel = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 4 * (kSub == 1 ? 4 : 2 * kSub));
+    int* sel0 = reinterpret_cast<int*>(smem + kOffA + (size_t)a.NQB * 4 * (kSub == 1 ? 4 : 2 * kSub));
 
     if (tid == 0) {
         mbar_init(bar(B_Q), 1);
@@ -300,14 +302,18 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
             mma_commit(bar(B_DRAIN));
             mbar_wait_drain(bar(B_DRAIN), 0);
         }
-    } else if (warp == 10) {
-        // ------------------------------------------------ top-k (one warp; kSub = 1)
+    } else if (warp >= 10) {
+        // ------------------------------------------------ top-k (kSub = 1): warp 10 takes
+        // the even scored units (A buffer 0), warp 11 the odd ones (buffer 1)
+        const int tw = warp - 10;
+        int* sel = sel0 + tw * a.topk;
         int su = 0;
         bool ok = kSub == 1;
         for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
             const SelUnit d = sel_unit_k<kSub>(a, u);
             int32_t* out = a.idx_out + d.lu * a.topk;
             if (!d.scored) {  // the budget covers every candidate
+                if (tw != 0) continue;
                 const int n = d.nF + d.nC;
                 for (int j = lane; j < a.topk; j += 32) {
                     int v = -1;
@@ -320,6 +326,10 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                 continue;
             }
             const int buf = su & 1;
+            if (buf != tw) {
+                ++su;
+                continue;
+            }
             ok = mbar_wait(bar(B_AFULL + buf), (su >> 1) & 1, abort_flag, a.status);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
@@ -620,13 +630,13 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                     if (topk::two_level(q.nC, q.ksel)) {
                         topk::level1(q.nC, q.ksel, key_of, fin, warp, lane);
                         named_barrier(1, 256);
-                        topk::level2(fin, q.ksel, sel, et);
+                        topk::level2(fin, q.ksel, sel0, et);
                     } else if (warp == 0) {
                         // a pick is marked by a NaN bit pattern that arithmetic never produces
                         topk::rounds_one_warp(
                             q.nC, q.ksel, key_of,
                             [&](int cj) { return __float_as_uint(Aj1[cj]) == 0xffffffffu; },
-                            [&](int t) { Aj1[t - c_lo] = __uint_as_float(0xffffffffu); }, sel, lane);
+                            [&](int t) { Aj1[t - c_lo] = __uint_as_float(0xffffffffu); }, sel0, lane);
                     }
                     named_barrier(1, 256);
                     int32_t* out = a.idx_out + ((long long)d.bg * a.NQB + qb) * a.topk;
@@ -636,9 +646,9 @@ select_tc_unit_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                         else if (x >= q.nF + q.ksel) out[x] = -1;
                     }
                     for (int x = et; x < q.ksel; x += 256) {
-                        const int v = sel[x];
+                        const int v = sel0[x];
                         int rank = 0;
-                        for (int i = 0; i < q.ksel; ++i) rank += sel[i] < v;
+                        for (int i = 0; i < q.ksel; ++i) rank += sel0[i] < v;
                         out[q.n_init_q + rank] = v;
                     }
                     if (et == 0) a.cnt_out[(long long)d.bg * a.NQB + qb] = q.nF + q.ksel;
