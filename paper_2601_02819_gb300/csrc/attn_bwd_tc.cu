@@ -64,6 +64,27 @@ __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
     return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
+__device__ __forceinline__ uint4 shfl_xor4(const uint4& v, int m) {
+    return make_uint4(__shfl_xor_sync(0xffffffffu, v.x, m), __shfl_xor_sync(0xffffffffu, v.y, m),
+                      __shfl_xor_sync(0xffffffffu, v.z, m), __shfl_xor_sync(0xffffffffu, v.w, m));
+}
+
+// One round of a 4 x 4 transpose among lanes r and r ^ m: a lane with sel = 0
+// keeps (a0, a1) and replaces (b0, b1) with its partner's (a0, a1); a lane
+// with sel = 1 keeps (b0, b1) and replaces (a0, a1) with its partner's (b0, b1).
+__device__ __forceinline__ void xchg_pieces(uint4& a0, uint4& a1, uint4& b0, uint4& b1, int sel,
+                                            int m) {
+    const uint4 r0 = shfl_xor4(sel ? a0 : b0, m);
+    const uint4 r1 = shfl_xor4(sel ? a1 : b1, m);
+    if (sel) {
+        a0 = r0;
+        a1 = r1;
+    } else {
+        b0 = r0;
+        b1 = r1;
+    }
+}
+
 // ============================================================== dQ
 // Persistent: one CTA per SM walks the units (query block, KV head) u =
 // blockIdx.x, blockIdx.x + gridDim.x, ...; the K/V rings, the S/dP buffers and
@@ -702,17 +723,33 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
                 }
                 tc_fence_before();
                 mbar_arrive(bar(C::B_DQFREE));
-                if (valid) {
-                    uint4* dst = reinterpret_cast<uint4*>(a.dQ + ridx * 128 + 64 * half);
-                    const float s = a.sm_scale;
+                // Rows go out through a 4 x 4 transpose of 16-byte pieces among each
+                // four lanes (two rounds of xor shuffles): afterwards lane 4j + c holds
+                // piece c of rows 4j .. 4j + 3 of a group of four pieces, so a store
+                // instruction writes eight 64-byte row segments instead of thirty-two
+                // 16-byte pieces of 32 different rows.
+                const float s = a.sm_scale;
+                const int sel1 = (lane >> 1) & 1, sel0 = lane & 1;
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        uint4 v;
-                        v.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * s, __uint_as_float(o[8 * q + 1]) * s);
-                        v.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * s, __uint_as_float(o[8 * q + 3]) * s);
-                        v.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * s, __uint_as_float(o[8 * q + 5]) * s);
-                        v.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * s, __uint_as_float(o[8 * q + 7]) * s);
-                        dst[q] = v;
+                for (int c4 = 0; c4 < 2; ++c4) {
+                    uint4 x[4];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int b = 32 * c4 + 8 * q;
+                        x[q].x = pack2_bf16(__uint_as_float(o[b + 0]) * s, __uint_as_float(o[b + 1]) * s);
+                        x[q].y = pack2_bf16(__uint_as_float(o[b + 2]) * s, __uint_as_float(o[b + 3]) * s);
+                        x[q].z = pack2_bf16(__uint_as_float(o[b + 4]) * s, __uint_as_float(o[b + 5]) * s);
+                        x[q].w = pack2_bf16(__uint_as_float(o[b + 6]) * s, __uint_as_float(o[b + 7]) * s);
+                    }
+                    xchg_pieces(x[0], x[1], x[2], x[3], sel1, 2);  // rows r, r^2: halves of the pieces
+                    xchg_pieces(x[0], x[2], x[1], x[3], sel0, 1);  // rows r, r^1: single pieces
+#pragma unroll
+                    for (int s4 = 0; s4 < 4; ++s4) {
+                        const int r = (warp & 3) * 32 + (lane & ~3) + s4;  // the row of piece x[s4]
+                        const int ri = qb * 64 + (r & 63);
+                        if (ri < a.L)
+                            reinterpret_cast<uint4*>(a.dQ + ((size_t)(d.hq0 + (r >> 6)) * a.L + ri) * 128)
+                                [8 * half + 4 * c4 + (lane & 3)] = x[s4];
                     }
                 }
             }
