@@ -576,6 +576,28 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             }
             return v;
         };
+        // Into L2: unit u's successor's lse (read at the end of unit u), and the
+        // block list and count two units after it (staged a unit ahead).
+        auto prefetch_ahead = [&](int u) {
+            const int u1 = u + (int)gridDim.x, u3 = u + 2 * (int)gridDim.x;
+            if (u1 < a.units) {
+                const DqUnit d1 = dq_unit<kSub>(a, u1);
+                const int r1 = et >> 1, i1 = d1.qb * 64 + (r1 & 63);
+                if (i1 < a.L && (r1 & 31) == 0 && (et & 1) == 0)
+                    prefetch_l2(a.lse + (size_t)(d1.hq0 + (r1 >> 6)) * a.L + i1);
+            }
+            if (u3 < a.units) {
+                const DqUnit d3 = dq_unit<kSub>(a, u3);
+                if constexpr (kSub == 1) {
+                    if (et == 0) prefetch_l2(a.cnt + d3.lu);
+                    if (et < 4 && et * 32 < a.topk) prefetch_l2(a.idx + d3.lu * a.topk + et * 32);
+                    if (et == 4) prefetch_l2(a.idx + d3.lu * a.topk + a.topk - 1);
+                } else {
+                    if (et == 0) prefetch_l2(a.ucnt + d3.lu);
+                    if (et < 8 && et * 32 < a.ucap) prefetch_l2(a.ulist + d3.lu * a.ucap + et * 32);
+                }
+            }
+        };
         float dlt_next = 0.f;
         for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
             const int* list = lists + (ul & 1) * ls;
@@ -585,27 +607,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             const bool valid = i < a.L;
             const size_t ridx = (size_t)(d.hq0 + hl) * a.L + (valid ? i : 0);
             const float nl2 = neg_lse2;
-            {  // into L2: the next unit's lse (read at the end of this unit), and the
-               // block list and count two units ahead (staged a unit ahead)
-                const int u1 = u + (int)gridDim.x, u3 = u + 2 * (int)gridDim.x;
-                if (u1 < a.units) {
-                    const DqUnit d1 = dq_unit<kSub>(a, u1);
-                    const int r1 = et >> 1, i1 = d1.qb * 64 + (r1 & 63);
-                    if (i1 < a.L && (r1 & 31) == 0 && (et & 1) == 0)
-                        prefetch_l2(a.lse + (size_t)(d1.hq0 + (r1 >> 6)) * a.L + i1);
-                }
-                if (u3 < a.units) {
-                    const DqUnit d3 = dq_unit<kSub>(a, u3);
-                    if constexpr (kSub == 1) {
-                        if (et == 0) prefetch_l2(a.cnt + d3.lu);
-                        if (et < 4 && et * 32 < a.topk) prefetch_l2(a.idx + d3.lu * a.topk + et * 32);
-                        if (et == 4) prefetch_l2(a.idx + d3.lu * a.topk + a.topk - 1);
-                    } else {
-                        if (et == 0) prefetch_l2(a.ucnt + d3.lu);
-                        if (et < 8 && et * 32 < a.ucap) prefetch_l2(a.ulist + d3.lu * a.ucap + et * 32);
-                    }
-                }
-            }
+            if (ul == 0) prefetch_ahead(u);  // later units': during the previous unit's last dQ
             // Delta of the CTA's first unit here (its Q is loaded over its O only after
             // that); every later unit's was computed during the previous unit
             if (ul == 0) dlt_next = delta_pass(0);
@@ -706,6 +708,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             gp0 += np;
             if (next_delta) dlt_next = delta_pass(ul + 1);  // no pair reached pd (or an abort)
             if (u2 < a.units) fetch_unit(u2);  // the next unit's lse
+            if (u2 < a.units) prefetch_ahead(u2);  // while this unit's last dQ MMAs run
             if (ok) {
                 ok = mbar_wait(bar(C::B_FINAL), ul & 1, abort_flag, a.status);
                 ok = __all_sync(0xffffffffu, ok);
