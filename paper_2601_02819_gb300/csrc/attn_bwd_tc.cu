@@ -528,12 +528,18 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         // A unit's lse (for P) is fetched at the end of the previous unit; its block
         // list is staged by the producer before it arrives on C::B_Q.
         float neg_lse2 = 0.f;
-        auto fetch_unit = [&](int u) {
-            const DqUnit d = dq_unit<kSub>(a, u);
+        auto fetch_unit = [&](const DqUnit& d) {
             const int i = d.qb * 64 + tok;
             neg_lse2 = i < a.L ? -__ldg(a.lse + (size_t)(d.hq0 + hl) * a.L + i) * kLog2e : -INFINITY;
         };
-        if (blockIdx.x < a.units) fetch_unit(blockIdx.x);
+        // Each unit's coordinates are worked out during the previous unit's wait for
+        // its last dQ MMAs: their integer divisions (and the special-function unit
+        // they use) stay off the unit boundary.
+        DqUnit d_cur{};
+        if (blockIdx.x < a.units) {
+            d_cur = dq_unit<kSub>(a, blockIdx.x);
+            fetch_unit(d_cur);
+        }
         // Delta_i = dO_i . O_i of local unit ulx from its O tile (in the Q staging
         // buffer) and dO tile (in its own), both waited for here: the warps of d
         // half 0 take one row each over the whole head dimension. Returns this
@@ -601,7 +607,7 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
         float dlt_next = 0.f;
         for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++ul) {
             const int* list = lists + (ul & 1) * ls;
-            const DqUnit d = dq_unit<kSub>(a, u);
+            const DqUnit d = d_cur;
             const int qb = d.qb;
             const int i = qb * 64 + tok;
             const bool valid = i < a.L;
@@ -707,7 +713,10 @@ dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CU
             }
             gp0 += np;
             if (next_delta) dlt_next = delta_pass(ul + 1);  // no pair reached pd (or an abort)
-            if (u2 < a.units) fetch_unit(u2);  // the next unit's lse
+            if (u2 < a.units) {
+                d_cur = dq_unit<kSub>(a, u2);
+                fetch_unit(d_cur);  // the next unit's lse
+            }
             if (u2 < a.units) prefetch_ahead(u2);  // while this unit's last dQ MMAs run
             if (ok) {
                 ok = mbar_wait(bar(C::B_FINAL), ul & 1, abort_flag, a.status);
