@@ -71,8 +71,10 @@ delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restric
 // Rows of the transposed selection are KV spans of 64 keys (kSub = 64/m blocks
 // each; one block at m = 64), columns are query blocks of m tokens. At m < 64
 // each (span, query block) pair also records which of the span's kSub blocks
-// the query block selected: kSub bits at bit (qb * kSub) % 32 of word
-// (qb * kSub) / 32 of the span's mask row.
+// the query block selected: kSub bits in byte qb of the span's mask row. A
+// query block's entries in one span are consecutive in its ascending list, so
+// the byte is written once, by a plain store; bytes of pairs that are not
+// selected are never read and need no clearing.
 // Marks the selections of unit u (query block qb of one (b, g)) in the bitmap
 // rows `bits` of that (b, g) (global or shared memory) and, at m < 64, in its
 // mask rows. The entries are loaded eight at a time (independent loads), then
@@ -80,8 +82,8 @@ delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restric
 // query's future or not ascending is recorded as a device index error.
 __device__ __forceinline__ void mark_unit(const int32_t* __restrict__ idx,
                                           const int32_t* __restrict__ cnt, long long u, int qb,
-                                          int kSub, int topk, int words, int mwords,
-                                          uint32_t* bits, uint32_t* __restrict__ masks,
+                                          int kSub, int topk, int words, int mrow,
+                                          uint32_t* bits, uint8_t* __restrict__ masks,
                                           int* status) {
     int n = cnt[u];
     if (n < 0 || n > topk) {
@@ -89,7 +91,8 @@ __device__ __forceinline__ void mark_unit(const int32_t* __restrict__ idx,
         n = n < 0 ? 0 : topk;
     }
     const int32_t* row = idx + u * topk;
-    int prev = -1;
+    int prev = -1, curT = -1;
+    uint32_t curm = 0u;  // the blocks of span curT this query block selected
     for (int j0 = 0; j0 < n; j0 += 8) {
         int tv[8];
 #pragma unroll
@@ -104,24 +107,28 @@ __device__ __forceinline__ void mark_unit(const int32_t* __restrict__ idx,
             }
             prev = t;
             const int T = t / kSub;
-            atomicOr(&bits[T * words + (qb >> 5)], 1u << (qb & 31));
-            if (kSub > 1)
-                atomicOr(&masks[(size_t)T * mwords + ((qb * kSub) >> 5)],
-                         (1u << (t - T * kSub)) << ((qb * kSub) & 31));
+            if (T != curT) {
+                atomicOr(&bits[T * words + (qb >> 5)], 1u << (qb & 31));
+                if (kSub > 1 && curT >= 0) masks[(size_t)curT * mrow + qb] = (uint8_t)curm;
+                curT = T;
+                curm = 0u;
+            }
+            curm |= 1u << (t - T * kSub);
         }
     }
+    if (kSub > 1 && curT >= 0) masks[(size_t)curT * mrow + qb] = (uint8_t)curm;
 }
 
 __global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt,
                                 long long units, int NQB, int nrows, int kSub, int topk, int words,
-                                int mwords, uint32_t* __restrict__ bits, uint32_t* __restrict__ masks,
+                                int mrow, uint32_t* __restrict__ bits, uint8_t* __restrict__ masks,
                                 int* status) {
     const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (u >= units) return;
     const int qb = (int)(u % NQB);
     const long long bg = u / NQB;
-    mark_unit(idx, cnt, u, qb, kSub, topk, words, mwords, bits + bg * nrows * words,
-              masks + bg * nrows * mwords, status);
+    mark_unit(idx, cnt, u, qb, kSub, topk, words, mrow, bits + bg * nrows * words,
+              masks + bg * nrows * mrow, status);
 }
 
 // The bitmap of one (b, g) in shared memory, rows of rs words: thread q marks
@@ -131,8 +138,8 @@ __global__ void idx_mark_kernel(const int32_t* __restrict__ idx, const int32_t* 
 // exactly those bits). The checks are mark_unit's, in list order per lane.
 __device__ __forceinline__ void mark_warp(const int32_t* __restrict__ idx,
                                           const int32_t* __restrict__ cnt, long long u0, int NQB,
-                                          int kSub, int topk, int rs, int mwords, uint32_t* bits,
-                                          uint32_t* __restrict__ masks, int* status) {
+                                          int kSub, int topk, int rs, int mrow, uint32_t* bits,
+                                          uint8_t* __restrict__ masks, int* status) {
     const int lane = threadIdx.x & 31;
     for (int qw = threadIdx.x & ~31; qw < NQB; qw += blockDim.x) {
         const int qb = qw + lane;
@@ -144,7 +151,8 @@ __device__ __forceinline__ void mark_warp(const int32_t* __restrict__ idx,
         }
         const int nmax = __reduce_max_sync(0xffffffffu, n);
         const int32_t* row = idx + (u0 + (live ? qb : 0)) * topk;
-        int prev = -1;
+        int prev = -1, curT = -1;
+        uint32_t curm = 0u;  // the blocks of span curT this query block selected
         for (int j0 = 0; j0 < nmax; j0 += 8) {
             int tv[8];
 #pragma unroll
@@ -160,14 +168,22 @@ __device__ __forceinline__ void mark_warp(const int32_t* __restrict__ idx,
                         prev = t;
                     }
                 }
+                // a span is marked once per query block: at its first entry in the list
                 const int T = t < 0 ? -1 : t / kSub;
-                const unsigned grp = __match_any_sync(0xffffffffu, T);
-                if (T >= 0 && lane == __ffs(grp) - 1) atomicOr(&bits[T * rs + (qw >> 5)], grp);
-                if (kSub > 1 && T >= 0)
-                    atomicOr(&masks[(size_t)T * mwords + ((qb * kSub) >> 5)],
-                             (1u << (t - T * kSub)) << ((qb * kSub) & 31));
+                const int Tn = T == curT ? -1 : T;
+                const unsigned grp = __match_any_sync(0xffffffffu, Tn);
+                if (Tn >= 0 && lane == __ffs(grp) - 1) atomicOr(&bits[Tn * rs + (qw >> 5)], grp);
+                if (T >= 0) {
+                    if (T != curT) {
+                        if (kSub > 1 && curT >= 0) masks[(size_t)curT * mrow + qb] = (uint8_t)curm;
+                        curT = T;
+                        curm = 0u;
+                    }
+                    curm |= 1u << (t - T * kSub);
+                }
             }
         }
+        if (kSub > 1 && curT >= 0) masks[(size_t)curT * mrow + qb] = (uint8_t)curm;
     }
 }
 
@@ -210,7 +226,7 @@ template <bool kMark>
 __global__ void __launch_bounds__(1024)
 idx_build_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cnt,
                  const uint32_t* __restrict__ bits, int NQB, int nrows, int kSub, int topk,
-                 int words, int mwords, uint32_t* __restrict__ masks, int work_max, int slot_max,
+                 int words, int mrow, uint8_t* __restrict__ masks, int work_max, int slot_max,
                  TInfo* __restrict__ tinfo, int32_t* __restrict__ qlist, int2* __restrict__ work,
                  int32_t* __restrict__ nwork, int* __restrict__ arrive, int2* __restrict__ queue,
                  int* __restrict__ qcount, int* status) {
@@ -228,8 +244,8 @@ idx_build_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ cn
         rs = words | 1;
         for (int i = threadIdx.x; i < nrows * rs; i += blockDim.x) sbits[i] = 0u;
         __syncthreads();
-        mark_warp(idx, cnt, (long long)bg * NQB, NQB, kSub, topk, rs, mwords, sbits,
-                  masks + (size_t)bg * nrows * mwords, status);
+        mark_warp(idx, cnt, (long long)bg * NQB, NQB, kSub, topk, rs, mrow, sbits,
+                  masks + (size_t)bg * nrows * mrow, status);
         __syncthreads();
         bb = sbits;
     } else {
@@ -775,7 +791,7 @@ BwdLayout bwd_layout(const phsa_shape& s, int topk) {
     l.nqb = (s.L + bm - 1) / bm;
     l.nrows = (s.L + kM - 1) / kM;
     l.words = (l.nqb + 31) / 32;
-    l.mwords = l.kSub > 1 ? (l.nqb * l.kSub + 31) / 32 : 0;
+    l.mrow = l.kSub > 1 ? l.nqb : 0;  // mask bytes per span row
     l.chunk = kChunk * l.kSub;  // query blocks per dK/dV work item
     l.ucap = l.kSub * topk;
     const long long bgs = (long long)s.B * s.Hkv;
@@ -786,7 +802,7 @@ BwdLayout bwd_layout(const phsa_shape& s, int topk) {
     size_t off = 0;
     l.qctl = off;    off = align256(off + 8 * 4);
     l.bits = off;    off = align256(off + (size_t)spans * l.words * 4);
-    l.masks = off;   off = align256(off + (size_t)spans * l.mwords * 4);
+    l.masks = off;   off = align256(off + (size_t)spans * l.mrow);
     l.tinfo = off;   off = align256(off + (size_t)spans * sizeof(TInfo));
     l.qlist = off;   off = align256(off + (size_t)bgs * nnz_max * 4);
     l.work = off;    off = align256(off + (size_t)bgs * l.work_max * sizeof(int2));
@@ -834,7 +850,7 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     const BwdLayout l = bwd_layout(s, topk);
     uint8_t* w = static_cast<uint8_t*>(ws);
     uint32_t* bits = reinterpret_cast<uint32_t*>(w + l.bits);
-    uint32_t* masks = reinterpret_cast<uint32_t*>(w + l.masks);
+    uint8_t* masks = w + l.masks;
     int32_t* ucnt = reinterpret_cast<int32_t*>(w + l.ucnt);
     int32_t* ulist = reinterpret_cast<int32_t*>(w + l.ulist);
     uint8_t* umask = reinterpret_cast<uint8_t*>(w + l.umask);
@@ -882,11 +898,8 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
-    // the queue counters, the bitmap and the mask rows, in one memset
-    if ((e = cudaMemsetAsync(w + l.qctl, 0,
-                             l.masks - l.qctl + (size_t)bgs * l.nrows * l.mwords * 4, st)) !=
-        cudaSuccess)
-        return e;
+    // the queue counters and the bitmap, in one memset (the mask rows need none)
+    if ((e = cudaMemsetAsync(w + l.qctl, 0, l.masks - l.qctl, st)) != cudaSuccess) return e;
     const long long units = (long long)bgs * l.nqb;
     const size_t sbits = (size_t)l.nrows * (l.words | 1) * 4;  // one (b, g)'s bitmap
     if (sbits <= g_idx_smem_limit.load()) {
@@ -897,19 +910,19 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
             return e;
         ProfScope prof(K_BWD_BUILD, st);
         kern<<<bgs, 1024, sbits, st>>>(idx, cnt, bits, l.nqb, l.nrows, l.kSub, topk, l.words,
-                                       l.mwords, masks, l.work_max, l.slot_max, tinfo, qlist, work,
+                                       l.mrow, masks, l.work_max, l.slot_max, tinfo, qlist, work,
                                        nwork, arrive, queue, qctl, status);
     } else {
         {
             ProfScope prof(K_BWD_MARK, st);
             idx_mark_kernel<<<(unsigned)((units + 255) / 256), 256, 0, st>>>(
-                idx, cnt, units, l.nqb, l.nrows, l.kSub, topk, l.words, l.mwords, bits, masks,
+                idx, cnt, units, l.nqb, l.nrows, l.kSub, topk, l.words, l.mrow, bits, masks,
                 status);
         }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         ProfScope prof(K_BWD_BUILD, st);
         idx_build_kernel<false><<<bgs, 1024, 0, st>>>(
-            idx, cnt, bits, l.nqb, l.nrows, l.kSub, topk, l.words, l.mwords, masks, l.work_max,
+            idx, cnt, bits, l.nqb, l.nrows, l.kSub, topk, l.words, l.mrow, masks, l.work_max,
             l.slot_max, tinfo, qlist, work, nwork, arrive, queue, qctl, status);
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;

@@ -841,7 +841,7 @@ struct KvArgs {
     const float* delta;
     const BwdTInfo* tinfo;
     const int32_t* qlist;
-    const uint32_t* masks;
+    const uint8_t* masks;  // m < 64: per span row, a byte per query block
     const int2* queue;    // [kQueueClasses][qcap] {bg * nrows + t, chunk}
     const int* qcount;    // items per class
     int* ticket;          // next queue position to take
@@ -852,7 +852,7 @@ struct KvArgs {
     int* status;
     long long qcap;
     long long nnzq;  // query-list entries per (b, g)
-    int Hq, Hkv, L, nrows, topk, slot_max, mwords, chunkq;
+    int Hq, Hkv, L, nrows, topk, slot_max, mrow, chunkq;
     float scale_log2, sm_scale;
 };
 
@@ -902,8 +902,7 @@ __device__ __forceinline__ uint32_t span_mask(const KvArgs& a, int bg, int t, in
     if constexpr (kSub == 1) {
         return 1u;
     } else {
-        const uint32_t w = __ldg(a.masks + ((size_t)bg * a.nrows + t) * a.mwords + ((qb * kSub) >> 5));
-        return (w >> ((qb * kSub) & 31)) & ((1u << kSub) - 1u);
+        return __ldg(a.masks + ((size_t)bg * a.nrows + t) * a.mrow + qb);
     }
 }
 
@@ -1463,7 +1462,7 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
 
 cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
-                           const int32_t* qlist, const uint32_t* masks, const int2* queue,
+                           const int32_t* qlist, const uint8_t* masks, const int2* queue,
                            int* qctl, const phsa_shape& s, int topk, const BwdLayout& l,
                            float sm_scale, void* dK, void* dV, float* partial, int* arrive,
                            int* status, cudaStream_t st) {
@@ -1485,7 +1484,7 @@ cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const vo
     const long long qcap = (long long)s.B * s.Hkv * l.work_max;  // entries per queue class
     KvArgs args{lse, delta, tinfo, qlist, masks, queue, qctl, qctl + kQueueClasses, partial, arrive,
                 static_cast<__nv_bfloat16*>(dK), static_cast<__nv_bfloat16*>(dV), status, qcap,
-                (long long)l.nqb * topk, s.Hq, s.Hkv, s.L, l.nrows, topk, l.slot_max, l.mwords,
+                (long long)l.nqb * topk, s.Hq, s.Hkv, s.L, l.nrows, topk, l.slot_max, l.mrow,
                 l.chunk, sm_scale * kLog2e, sm_scale};
     ProfScope prof(K_BWD_DKDV, st);
     kern<<<(unsigned)(qcap < nsm ? qcap : nsm), kv::kThreads, kv::kSmem, st>>>(tq, tk, tv, tdo, args);

@@ -123,7 +123,7 @@ __host__ __device__ __forceinline__ int queue_class(int n_it) {
 struct BwdLayout;
 cudaError_t launch_dkdv_tc(const void* Q, const void* K, const void* V, const void* dO,
                            const float* lse, const float* delta, const BwdTInfo* tinfo,
-                           const int32_t* qlist, const uint32_t* masks, const int2* queue,
+                           const int32_t* qlist, const uint8_t* masks, const int2* queue,
                            int* qctl, const phsa_shape& s, int topk, const BwdLayout& l,
                            float sm_scale, void* dK, void* dV, float* partial, int* arrive,
                            int* status, cudaStream_t st);
@@ -145,12 +145,12 @@ cudaError_t launch_dq_tc(const void* Q, const void* K, const void* V, const void
 // reads the union of each span's query-block lists (ucnt, ulist, umask).
 struct BwdLayout {
     // qctl: item counts of the kQueueClasses queue classes, then the ticket
-    // counter of the persistent dK/dV kernel (zeroed with bits and masks by one memset)
+    // counter of the persistent dK/dV kernel (zeroed with the bitmap by one memset)
     size_t qctl, bits, masks, tinfo, qlist, work, nwork, queue, delta, partial, arrive, ucnt, ulist,
         umask, total;
     int nqb;    // query blocks of m tokens
     int nrows;  // KV spans of 64 keys
-    int kSub, words, mwords, chunk, work_max, slot_max, ucap;
+    int kSub, words, mrow, chunk, work_max, slot_max, ucap;
 };
 BwdLayout bwd_layout(const phsa_shape& s, int topk);
 
