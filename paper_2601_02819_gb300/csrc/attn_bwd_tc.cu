@@ -1156,8 +1156,9 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     const uint32_t ph = (uint32_t)((nv >> 1) & 1);
                     const int sq = (2 * nv) % kSlots, sd = (2 * nv + 1) % kSlots;  // Q_i, dO_i
                     // K dimension = the 128 stacked query rows, 16 per MMA. P being stored
-                    // implies that S, hence Q_i, has landed, but not dO_i: its half-slot
-                    // has its own barrier, which this thread waits on too.
+                    // implies that S, hence Q_i, has landed (so dK^T below needs no wait
+                    // of its own on Q_i), but not dO_i: its half-slot has its own
+                    // barrier, which this thread waits on.
                     ok = mbar_wait(bar(B_PFULL + b), ph, abort_flag, a.status) &&
                          mbar_wait(bar(B_HFULL + sd), (uint32_t)(((2 * nv + 1) / kSlots) & 1), abort_flag,
                                    a.status);
@@ -1173,8 +1174,7 @@ dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     ok = mbar_wait(bar(B_DPFULL + b), ph, abort_flag, a.status);
                     if (!ok) break;
                     mma_commit(bar(B_HEMPTY + sd));
-                    ok = mbar_wait(bar(B_DSFULL + b), ph, abort_flag, a.status) &&
-                         mbar_wait(bar(B_HFULL + sq), (uint32_t)(((2 * nv) / kSlots) & 1), abort_flag, a.status);
+                    ok = mbar_wait(bar(B_DSFULL + b), ph, abort_flag, a.status);
                     if (!ok) break;
                     tc_fence_after();
                     const uint64_t qt = sdesc_at(dSlT0, sq * kTile128);
