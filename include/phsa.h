@@ -403,14 +403,16 @@ int phsa_selftest_tcgen05(const void* A, const void* B, const void* V, float* S,
 size_t phsa_test_set_select_tc_limit(size_t bytes);
 
 /* Testing hook. The backward transposes the block lists (KV block -> the
- * query blocks that selected it) in one launch while one (batch, KV head)'s
- * bitmap of (KV span, query block) pairs fits in 160 KB of shared memory
- * (up to 1140 query blocks of 64 tokens, or 2048 of 16), else in two
- * launches through a bitmap in global memory. This call sets that switch
- * point to `bytes` (0, or more than 160 KB, restores the default) so that a
- * test can reach the two-launch form on short inputs; both build the same
- * lists. Returns the previous value. Affects every later call in the
- * process; not meant for production use.
+ * query blocks that selected it) either in one launch, with one (batch, KV
+ * head)'s bitmap of (KV span, query block) pairs in at most 160 KB of shared
+ * memory, or in two launches through a bitmap in global memory. By default
+ * the one-launch form runs at block size 64 while the bitmap fits (up to 1140
+ * query blocks) and the two-launch form otherwise and at block sizes 16 and
+ * 32. A nonzero `bytes` makes every block size take the one-launch form
+ * while the bitmap fits in min(bytes, 160 KB), so that a test can reach
+ * either form on short inputs; 0 restores the default. Both forms build the
+ * same lists. Returns the previous setting (0: the default). Affects every
+ * later call in the process; not meant for production use.
  */
 size_t phsa_test_set_idx_smem_limit(size_t bytes);
 

@@ -36,10 +36,15 @@ constexpr int kBuildCache = 8192;   // KV blocks whose counts the index build ke
 // (beside its 32 KB of counts): 160 KB covers 1140 query blocks of 64 and
 // 2048 query blocks of 16 (32k tokens at m = 16).
 constexpr size_t kIdxSmemBits = 160u * 1024u;
-// The switch point in use; only phsa_test_set_idx_smem_limit lowers it, so
-// that tests reach the two-launch transpose (bitmap in global memory) on
-// short sequences.
-std::atomic<size_t> g_idx_smem_limit{kIdxSmemBits};
+// Which form of the transpose runs. 0, the default: one launch at m = 64 while
+// the bitmap fits in kIdxSmemBits, two launches otherwise and at every m < 64,
+// where marking the (64/m)-times longer lists is most of the work and the
+// separate marking kernel spreads it over the whole GPU instead of one CTA per
+// (b, g) (32k at m = 16: 23 + 146 us in one launch, 45 + 78 us in two; at
+// m = 64: 31 us against 9 + 24). Nonzero: set by phsa_test_set_idx_smem_limit
+// so that tests reach either form at any block size, one launch at every m
+// while the bitmap fits in that many bytes.
+std::atomic<size_t> g_idx_smem_override{0};
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -902,7 +907,8 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
     if ((e = cudaMemsetAsync(w + l.qctl, 0, l.masks - l.qctl, st)) != cudaSuccess) return e;
     const long long units = (long long)bgs * l.nqb;
     const size_t sbits = (size_t)l.nrows * (l.words | 1) * 4;  // one (b, g)'s bitmap
-    if (sbits <= g_idx_smem_limit.load()) {
+    const size_t ov = g_idx_smem_override.load();
+    if (ov ? sbits <= ov : l.kSub == 1 && sbits <= kIdxSmemBits) {
         // mark and build in one launch, the bitmap in shared memory
         auto kern = idx_build_kernel<true>;
         if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -960,6 +966,6 @@ cudaError_t launch_attn_bwd(const void* Q, const void* K, const void* V, const v
 }  // namespace phsa
 
 extern "C" size_t phsa_test_set_idx_smem_limit(size_t bytes) {
-    const size_t v = bytes == 0 || bytes > phsa::kIdxSmemBits ? phsa::kIdxSmemBits : bytes;
-    return phsa::g_idx_smem_limit.exchange(v);
+    const size_t v = bytes > phsa::kIdxSmemBits ? phsa::kIdxSmemBits : bytes;
+    return phsa::g_idx_smem_override.exchange(v);
 }

@@ -566,9 +566,11 @@ def phsa_test_set_select_tc_limit(nbytes: int) -> int:
 
 
 def phsa_test_set_idx_smem_limit(nbytes: int) -> int:
-    """Testing hook: the shared-memory switch point between the one-launch and
-    the two-launch transpose of the block lists in the backward (0 restores
-    the default of 160 KB). Returns the previous value."""
+    """Testing hook: a nonzero value makes the backward transpose the block
+    lists in one launch at every block size while a (b, g)'s bitmap fits in
+    min(nbytes, 160 KB) of shared memory, else in two launches; 0 restores the
+    default (one launch at block size 64 while it fits in 160 KB, two launches
+    otherwise). Returns the previous setting."""
     return int(load().phsa_test_set_idx_smem_limit(int(nbytes)))
 
 

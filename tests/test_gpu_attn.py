@@ -167,8 +167,9 @@ def test_argument_errors_raise():
 ])
 def test_backward_index_transpose_forms_agree(m, B, Hq, Hkv, L, topk, n_init):
     # The one-launch transpose (bitmap in shared memory) and the two-launch
-    # form (bitmap in global memory, used when a (b, g)'s bitmap exceeds
-    # 160 KB) build the same KV-block lists, so the gradients are identical.
+    # form (bitmap in global memory: at m < 64, and when a (b, g)'s bitmap
+    # exceeds 160 KB) build the same KV-block lists, so the gradients are
+    # identical. The hook forces each form at every block size.
     rng = np.random.default_rng(L + 17 * m)
     f = lambda *s: inputs.f32_to_bf16_bits(rng.standard_normal(s).astype(np.float32))
     Q, K, V, dO = f(B, Hq, L, D), f(B, Hkv, L, D), f(B, Hkv, L, D), f(B, Hq, L, D)
@@ -178,16 +179,19 @@ def test_backward_index_transpose_forms_agree(m, B, Hq, Hkv, L, topk, n_init):
     Qd, Kd, Vd, dOd = (to_dev_bf16(a) for a in (Q, K, V, dO))
     it, ct = torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda()
     O, lse = phsa.phsa_sparse_attn_fwd(Qd, Kd, Vd, it, ct, block_size=m)
-    g_smem = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct, block_size=m)
-    prev = phsa.phsa_test_set_idx_smem_limit(1)
+    g_default = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct, block_size=m)
+    prev = phsa.phsa_test_set_idx_smem_limit(160 * 1024)
     try:
+        g_smem = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct, block_size=m)
+        phsa.phsa_test_set_idx_smem_limit(1)
         g_glob = phsa.phsa_sparse_attn_bwd(Qd, Kd, Vd, O, dOd, lse, it, ct, block_size=m)
         torch.cuda.synchronize()
     finally:
         phsa.phsa_test_set_idx_smem_limit(prev)
     assert phsa.phsa_get_device_status() == 0
-    for a, b in zip(g_smem, g_glob):
+    for a, b, c in zip(g_smem, g_glob, g_default):
         assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+        assert torch.equal(a.view(torch.int16), c.view(torch.int16))
     rQ, rK, rV = oracle.sparse_attn_bwd(Q, K, V, dO, idx, cnt, m, SCALE)
     assert_close("dQ", bf16_to_f64(g_smem[0]), rQ)
     assert_close("dK", bf16_to_f64(g_smem[1]), rK)
