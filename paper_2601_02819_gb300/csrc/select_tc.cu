@@ -277,9 +277,10 @@ __device__ __forceinline__ void write_picks(const SelArgs& a, int bg, int qb, co
 }
 
 // Top-k of one scored query block (ksel <= 32) by kW warps: warp wi takes a
-// kW-th of the candidates and keeps its best min(ksel, slice) in fin[wi]
-// (level 1); after the barrier, warp 0 takes the best ksel of the finalists
-// (level 2): every pick is within the best ksel of its own slice.
+// kW-th of the candidates and keeps its best min(ksel, slice) in fin[wi],
+// sorted (level 1); after the barrier, warp 0 merges the kW sorted lists two
+// at a time, keeping the best 32 (level 2): every pick is within the best ksel
+// of its own slice.
 template <bool kMaxLogit, int kW>
 __device__ __forceinline__ void topk_split(const SelArgs& a, int bg, int qb, const QbSel& q,
                                            const float* Aq, unsigned long long* fin, int wi,
@@ -295,8 +296,9 @@ __device__ __forceinline__ void topk_split(const SelArgs& a, int bg, int qb, con
     fin[wi * 32 + lane] = lane < k1 ? mine : 0ull;
     named_barrier(bar_id, 32 * kW);
     if (wi == 0) {
-        const unsigned long long best =
-            topk::warp_topk32(32 * kW, q.ksel, [&](int f) { return fin[f]; }, lane);
+        unsigned long long best = fin[lane];
+#pragma unroll
+        for (int w = 1; w < kW; ++w) best = topk::merge_top32(best, fin[w * 32 + lane], lane);
         if (ok) write_picks(a, bg, qb, q, best, lane);
     }
 }

@@ -155,6 +155,31 @@ __device__ __forceinline__ unsigned long long shfl_up64(unsigned long long v, in
     return ((unsigned long long)h << 32) | l;
 }
 
+__device__ __forceinline__ unsigned long long umin64(unsigned long long a, unsigned long long b) {
+    return a < b ? a : b;
+}
+
+__device__ __forceinline__ unsigned long long shfl_xor64(unsigned long long v, int m) {
+    const unsigned h = __shfl_xor_sync(0xffffffffu, (unsigned)(v >> 32), m);
+    const unsigned l = __shfl_xor_sync(0xffffffffu, (unsigned)v, m);
+    return ((unsigned long long)h << 32) | l;
+}
+
+// The 32 largest keys of two lists sorted descending across the lanes (lane k
+// holds the k-th largest of each), sorted descending again: the lane-wise
+// maximum of one list and the other reversed holds the 32 largest keys of
+// both as a bitonic sequence, and five half-cleaner stages sort it.
+__device__ __forceinline__ unsigned long long merge_top32(unsigned long long a, unsigned long long b,
+                                                          int lane) {
+    unsigned long long v = umax64(a, shfl64(b, 31 - lane));
+#pragma unroll
+    for (int j = 16; j >= 1; j >>= 1) {
+        const unsigned long long o = shfl_xor64(v, j);
+        v = (lane & j) ? umin64(v, o) : umax64(v, o);
+    }
+    return v;
+}
+
 // One warp, at most 32 picks, any number of candidates. A first pass takes the
 // largest key of each lane's candidates; the ksel-th largest of those 32
 // maxima, tau, is at most the ksel-th largest key of all (ksel lanes hold a key
